@@ -1,0 +1,167 @@
+"""CPU ORACLE — test infrastructure only.
+
+A plain, slow, obviously correct CPU implementation of the prefix-cache curve
+computation (``oracle.cpp``), wrapped for numpy.  Only ``tests/``, the smoke
+check in ``__graft_entry__`` and ``bench.py``'s CPU-baseline leg may import
+this package; the product path (``paper_2609_28870_gb300``) never does.
+
+Functions and the passages they restate:
+
+* ``block_offsets``, ``block_ids`` — Sec. 2.2: 16-token KV blocks, reusable iff
+  the whole preceding sequence matches; exact trie identity, ids numbered by
+  first occurrence.
+* ``reuse`` — previous / next access of each block (Belady's next use, Sec. 3.2).
+* ``sd_mattson``, ``sd_fenwick`` — LRU stack distance (App. B), by Mattson's
+  move-to-front stack and by Bennett-Kruskal counting.
+* ``lru_curves`` — direct LRU simulation per capacity (Sec. 3.1-3.2) with
+  prefix-contiguous hits (Sec. 2.2) and compute saved (Sec. 5.2, App. C).
+* ``prefix_hash`` — the polynomial prefix key the GPU path writes, evaluated
+  token by token.
+* ``run`` — all of the above on one trace.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "oracle.cpp")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB = os.path.join(_BUILD, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+NONE = 0xFFFFFFFF
+
+# Cost-model kinds (Sec. 5.2 and App. C)
+COST_UNIFORM, COST_MEASURED, COST_LINEAR = 0, 1, 2
+# Per-token constants of the measured-shape model: F_lin = 2 * 3.3e9 FLOPs per
+# token for the active parameters; F_attn = 4 * 48 layers * 32 heads * 128 dims
+# per attended position.
+F_LIN = 6_600_000_000
+F_ATTN = 4 * 48 * 32 * 128
+
+
+def build(force: bool = False) -> str:
+    """Compile ``oracle.cpp`` into ``oracle/_build/liboracle.so``."""
+    with _lock:
+        if not force and os.path.exists(_LIB) and os.path.getmtime(_LIB) >= os.path.getmtime(_SRC):
+            return _LIB
+        os.makedirs(_BUILD, exist_ok=True)
+        tmp = _LIB + f".tmp{os.getpid()}"
+        subprocess.run(["g++", "-O2", "-std=c++17", "-fPIC", "-shared", "-pthread", _SRC, "-o", tmp], check=True)
+        os.replace(tmp, _LIB)
+        return _LIB
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        lib = ctypes.CDLL(build())
+        vp, u32, u64, i32 = ctypes.c_void_p, ctypes.c_uint32, ctypes.c_uint64, ctypes.c_int
+        lib.orc_block_offsets.restype = u64
+        lib.orc_block_offsets.argtypes = [vp, u32, u32, vp]
+        lib.orc_block_ids.restype = u64
+        lib.orc_block_ids.argtypes = [vp, vp, u32, u32, vp]
+        lib.orc_reuse.argtypes = [vp, u64, u64, vp, vp]
+        lib.orc_sd_mattson.argtypes = [vp, u64, vp]
+        lib.orc_sd_fenwick.argtypes = [vp, u64, vp]
+        lib.orc_lru_curves.restype = i32
+        lib.orc_lru_curves.argtypes = [vp, vp, u32, u32, i32, u64, u64, vp, u32, i32, vp, vp, vp, vp, vp]
+        lib.orc_prefix_hash.argtypes = [vp, vp, u32, u32, u64, vp]
+        _lib = lib
+    return _lib
+
+
+def _p(a):
+    return a.ctypes.data
+
+
+def _c(a, dt):
+    return np.ascontiguousarray(a, dtype=dt)
+
+
+def block_offsets(req_tok_off, B: int) -> np.ndarray:
+    off = _c(req_tok_off, np.uint64)
+    out = np.empty(off.shape[0], dtype=np.uint64)
+    _load().orc_block_offsets(_p(off), off.shape[0] - 1, int(B), _p(out))
+    return out
+
+
+def block_ids(tokens, req_tok_off, B: int):
+    """(ids uint32[N], D) with exact prefix identity."""
+    tok, off = _c(tokens, np.uint32), _c(req_tok_off, np.uint64)
+    n = int(block_offsets(off, B)[-1])
+    ids = np.empty(n, dtype=np.uint32)
+    d = _load().orc_block_ids(_p(tok), _p(off), off.shape[0] - 1, int(B), _p(ids))
+    return ids, int(d)
+
+
+def reuse(ids, n_distinct: int):
+    ids = _c(ids, np.uint32)
+    prev = np.empty_like(ids)
+    nxt = np.empty_like(ids)
+    _load().orc_reuse(_p(ids), ids.shape[0], int(n_distinct), _p(prev), _p(nxt))
+    return prev, nxt
+
+
+def sd_mattson(ids) -> np.ndarray:
+    ids = _c(ids, np.uint32)
+    sd = np.empty_like(ids)
+    _load().orc_sd_mattson(_p(ids), ids.shape[0], _p(sd))
+    return sd
+
+
+def sd_fenwick(prev) -> np.ndarray:
+    prev = _c(prev, np.uint32)
+    sd = np.empty_like(prev)
+    _load().orc_sd_fenwick(_p(prev), prev.shape[0], _p(sd))
+    return sd
+
+
+def lru_curves(ids, req_blk_off, B: int, caps, kind: int = COST_MEASURED, f_lin: int = F_LIN,
+               f_attn: int = F_ATTN, threads: int | None = None):
+    """Direct LRU simulation at each capacity.  Returns (hits list[int],
+    saved list[int] (exact, from 128-bit sums), total_cost int)."""
+    ids, bo, caps = _c(ids, np.uint32), _c(req_blk_off, np.uint64), _c(caps, np.uint64)
+    G = caps.shape[0]
+    hits = np.zeros(G, dtype=np.uint64)
+    slo = np.zeros(G, dtype=np.uint64)
+    shi = np.zeros(G, dtype=np.uint64)
+    tlo = np.zeros(1, dtype=np.uint64)
+    thi = np.zeros(1, dtype=np.uint64)
+    nthreads = threads or max(1, min(G, os.cpu_count() or 1))
+    rc = _load().orc_lru_curves(_p(ids), _p(bo), bo.shape[0] - 1, int(B), int(kind), int(f_lin), int(f_attn),
+                                _p(caps), G, nthreads, _p(hits), _p(slo), _p(shi), _p(tlo), _p(thi))
+    if rc != 0:
+        raise ValueError("bad capacity grid (capacities must be >= 1)")
+    saved = [int(h) << 64 | int(l) for l, h in zip(slo, shi)]
+    return [int(h) for h in hits], saved, int(thi[0]) << 64 | int(tlo[0])
+
+
+def prefix_hash(tokens, req_tok_off, B: int, seed: int) -> np.ndarray:
+    """Keys uint64[N, 2]: the polynomial prefix hash with the two seeded bases."""
+    tok, off = _c(tokens, np.uint32), _c(req_tok_off, np.uint64)
+    n = int(block_offsets(off, B)[-1])
+    keys = np.empty((n, 2), dtype=np.uint64)
+    _load().orc_prefix_hash(_p(tok), _p(off), off.shape[0] - 1, int(B), int(seed) & (2**64 - 1), _p(keys))
+    return keys
+
+
+def run(tokens, req_tok_off, B: int, caps, kind: int = COST_MEASURED, f_lin: int = F_LIN, f_attn: int = F_ATTN,
+        threads: int | None = None, mattson: bool = False) -> dict:
+    """Every oracle stage on one trace."""
+    off = block_offsets(req_tok_off, B)
+    ids, D = block_ids(tokens, req_tok_off, B)
+    prev, nxt = reuse(ids, D)
+    sd = sd_fenwick(prev)
+    out = dict(req_blk_off=off, ids=ids, n_access=int(ids.shape[0]), n_distinct=D, prev=prev, next=nxt, sd=sd)
+    if mattson:
+        out["sd_mattson"] = sd_mattson(ids)
+    hits, saved, total = lru_curves(ids, off, B, caps, kind, f_lin, f_attn, threads)
+    out.update(hits=hits, saved=saved, total_cost=total)
+    return out

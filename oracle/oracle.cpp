@@ -1,0 +1,318 @@
+// CPU ORACLE — test infrastructure only.
+//
+// A plain, slow, obviously correct restatement of what the GPU path computes:
+// block-level LRU prefix-cache hit curves and compute-saved curves over a
+// request trace.  Only the tests, the package's smoke check and the bench's
+// CPU-baseline leg may load this library.  It shares no code, header, table or
+// constant generator with the CUDA path.
+//
+// Definitions followed (paper: "When Fancy Eviction Fails: Rethinking Cache
+// Replacement For LLM Prefix Reuse"):
+//   * Sec. 2.2: KV state is cached in fixed-size token blocks (16 tokens), and
+//     a cached block is reusable iff its whole preceding sequence matches.
+//     -> orc_block_ids: a trie keyed by (parent block id, the block's tokens),
+//        compared token by token (no hashing decides identity).
+//   * Sec. 3.1-3.2: block hit ratio of an LRU cache of C blocks replaying the
+//     trace.  -> orc_lru_curves: one direct hashmap + recency-list LRU per
+//        capacity; a block counts as a prefix hit only if it and every earlier
+//        block of its request are resident (prefix reuse, Sec. 2.2).
+//   * Sec. 5.2: compute-savings ratio = cost of hits / cost of all accesses,
+//     with a per-block recompute cost that grows with depth.  -> cost_of().
+//   * Appendix B: the stack distance between reuses ("reuses reachable within
+//     C").  -> orc_sd_mattson (move-to-front list, Mattson et al. 1970) and
+//        orc_sd_fenwick (Bennett & Kruskal 1975 counting), two independent ways.
+//   * Belady's next use (Sec. 3.2, 5.2).  -> orc_reuse: previous and next
+//     access of the same block.
+// The GPU path's block keys are polynomial hashes of each block's whole
+// prefix; orc_prefix_hash evaluates that polynomial token by token (Horner)
+// so the keys themselves can be compared.
+//
+// Readings where the paper is silent (listed with the design notes): requests
+// are replayed in trace order and blocks root-first; a trailing partial block is
+// not cached; ids are numbered by first occurrence; stack distances are 1-based
+// with "never seen" = 0xFFFFFFFF; costs are summed in unsigned 128-bit integers.
+#include <algorithm>
+#include <atomic>
+#include <cstdint>
+#include <cstring>
+#include <list>
+#include <thread>
+#include <unordered_map>
+#include <vector>
+
+typedef unsigned __int128 u128;
+static const uint32_t NONE = 0xFFFFFFFFu;
+
+// ---------------------------------------------------------------------------
+// Exact block identity (Sec. 2.2).
+// ---------------------------------------------------------------------------
+namespace {
+struct BlockKey {
+  uint32_t parent;   // id of the previous block of the request, or NONE for the first block
+  uint64_t tok_off;  // offset of the block's first token in the token array
+};
+struct BlockHash {
+  const uint32_t* tok;
+  uint32_t B;
+  size_t operator()(const BlockKey& k) const {
+    // FNV-1a over the parent id and the B token values (used only to bucket;
+    // equality below compares the tokens themselves).
+    uint64_t h = 1469598103934665603ULL;
+    auto mix = [&](uint32_t v) {
+      for (int b = 0; b < 4; ++b) { h ^= (v >> (8 * b)) & 0xFF; h *= 1099511628211ULL; }
+    };
+    mix(k.parent);
+    for (uint32_t t = 0; t < B; ++t) mix(tok[k.tok_off + t]);
+    return (size_t)h;
+  }
+};
+struct BlockEq {
+  const uint32_t* tok;
+  uint32_t B;
+  bool operator()(const BlockKey& a, const BlockKey& b) const {
+    if (a.parent != b.parent) return false;
+    for (uint32_t t = 0; t < B; ++t)
+      if (tok[a.tok_off + t] != tok[b.tok_off + t]) return false;
+    return true;
+  }
+};
+}  // namespace
+
+extern "C" {
+
+// Number of full blocks of each request and their offsets in the access
+// stream: req_blk_off[r] = sum over earlier requests of floor(len / B).
+// Returns the total N.
+uint64_t orc_block_offsets(const uint64_t* req_tok_off, uint32_t n_req, uint32_t B, uint64_t* req_blk_off) {
+  req_blk_off[0] = 0;
+  for (uint32_t r = 0; r < n_req; ++r) {
+    uint64_t len = req_tok_off[r + 1] - req_tok_off[r];
+    req_blk_off[r + 1] = req_blk_off[r] + len / B;  // a trailing partial block is not a cache object
+  }
+  return req_blk_off[n_req];
+}
+
+// Dense block ids in first-occurrence order of the access stream (requests in
+// trace order, blocks root-first).  Two blocks get the same id iff their whole
+// prefixes [0, B(k+1)) are equal token by token: by induction over k, since a
+// block's trie key is (id of its parent, its own B tokens).
+// ids must hold N entries (N from orc_block_offsets).  Returns D.
+uint64_t orc_block_ids(const uint32_t* tokens, const uint64_t* req_tok_off, uint32_t n_req, uint32_t B,
+                       uint32_t* ids) {
+  BlockHash hasher{tokens, B};
+  BlockEq eq{tokens, B};
+  std::unordered_map<BlockKey, uint32_t, BlockHash, BlockEq> trie(16, hasher, eq);
+  uint32_t next_id = 0;
+  uint64_t i = 0;
+  for (uint32_t r = 0; r < n_req; ++r) {
+    uint64_t len = req_tok_off[r + 1] - req_tok_off[r];
+    uint64_t nblk = len / B;
+    uint32_t parent = NONE;
+    for (uint64_t k = 0; k < nblk; ++k) {
+      BlockKey key{parent, req_tok_off[r] + k * B};
+      auto it = trie.find(key);
+      uint32_t id;
+      if (it == trie.end()) {
+        id = next_id++;
+        trie.emplace(key, id);
+      } else {
+        id = it->second;
+      }
+      ids[i++] = id;
+      parent = id;
+    }
+  }
+  return next_id;
+}
+
+// prev[i] = largest j < i with ids[j] == ids[i], else NONE;
+// next[i] = smallest j > i with ids[j] == ids[i], else NONE (Belady's next use).
+void orc_reuse(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev, uint32_t* next) {
+  std::vector<uint32_t> last(n_distinct, NONE);
+  for (uint64_t i = 0; i < n; ++i) {
+    prev[i] = last[ids[i]];
+    last[ids[i]] = (uint32_t)i;
+  }
+  std::fill(last.begin(), last.end(), NONE);
+  for (uint64_t i = n; i-- > 0;) {
+    next[i] = last[ids[i]];
+    last[ids[i]] = (uint32_t)i;
+  }
+}
+
+// LRU stack distance by Mattson's stack: keep blocks in recency order (most
+// recent first); an access at depth d (1-based) has distance d, a block never
+// seen has distance NONE, and the block moves to the top.  O(N * D): tiny
+// inputs only.
+void orc_sd_mattson(const uint32_t* ids, uint64_t n, uint32_t* sd) {
+  std::vector<uint32_t> stack;  // stack[0] is the most recent
+  for (uint64_t i = 0; i < n; ++i) {
+    uint32_t x = ids[i];
+    size_t pos = 0;
+    while (pos < stack.size() && stack[pos] != x) ++pos;
+    if (pos == stack.size()) {
+      sd[i] = NONE;
+      stack.insert(stack.begin(), x);
+    } else {
+      sd[i] = (uint32_t)(pos + 1);
+      stack.erase(stack.begin() + pos);
+      stack.insert(stack.begin(), x);
+    }
+  }
+}
+
+// LRU stack distance by counting (Bennett & Kruskal): mark, for every block,
+// the position of its latest access so far; the distance of access i with
+// previous access p is 1 + (number of marked positions strictly between p and
+// i), i.e. 1 + the number of distinct blocks touched since p.  A Fenwick tree
+// over positions holds the marks.
+void orc_sd_fenwick(const uint32_t* prev, uint64_t n, uint32_t* sd) {
+  std::vector<uint32_t> tree(n + 1, 0);
+  auto add = [&](uint64_t pos, int32_t v) {
+    for (uint64_t x = pos + 1; x <= n; x += x & (~x + 1)) tree[x] += (uint32_t)v;
+  };
+  auto prefix = [&](uint64_t cnt) {  // marks in positions [0, cnt)
+    uint64_t s = 0;
+    for (uint64_t x = cnt; x > 0; x -= x & (~x + 1)) s += tree[x];
+    return s;
+  };
+  for (uint64_t i = 0; i < n; ++i) {
+    uint32_t p = prev[i];
+    if (p == NONE) {
+      sd[i] = NONE;
+    } else {
+      uint64_t between = prefix(i) - prefix((uint64_t)p + 1);
+      sd[i] = (uint32_t)(1 + between);
+      add(p, -1);
+    }
+    add(i, +1);
+  }
+}
+
+}  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Recompute cost of block k (0-based depth) of a request (Sec. 5.2, App. C).
+//   kind 0 (uniform): every block costs 1, so compute saved = hits.
+//   kind 1 (measured-shape): B*f_lin for the position-independent work plus
+//           f_attn * (t+1) for each token t of the block (token t attends to
+//           t+1 positions), t = Bk .. Bk+B-1.
+//   kind 2 (linear): the attention term alone, proportional to depth.
+// ---------------------------------------------------------------------------
+static u128 cost_of(uint64_t k, uint32_t B, int kind, uint64_t f_lin, uint64_t f_attn) {
+  if (kind == 0) return 1;
+  u128 c = 0;
+  if (kind == 1) c += (u128)B * f_lin;
+  for (uint64_t t = (uint64_t)B * k; t < (uint64_t)B * k + B; ++t) c += (u128)f_attn * (t + 1);
+  return c;
+}
+
+extern "C" {
+
+// Direct LRU simulation, one capacity at a time (Sec. 3.1-3.2 with prefix
+// reuse from Sec. 2.2).  For capacity C: replay requests in trace order and
+// their blocks root-first; a resident block moves to the most-recent end, a
+// missing block is inserted there and, if the cache then holds more than C
+// blocks, the least recent one is evicted.  Block k of a request is a hit iff
+// blocks 0..k of that request were all resident when touched.
+//
+// caps[G] are capacities in blocks (>= 1).  Outputs per capacity: hits[g] and
+// the 128-bit compute saved as saved_lo[g] / saved_hi[g].  total_cost gets the
+// 128-bit cost of every access.  Capacities are spread over `threads` host
+// threads.  Returns 0, or -1 on a bad argument.
+int orc_lru_curves(const uint32_t* ids, const uint64_t* req_blk_off, uint32_t n_req, uint32_t B, int kind,
+                   uint64_t f_lin, uint64_t f_attn, const uint64_t* caps, uint32_t G, int threads, uint64_t* hits,
+                   uint64_t* saved_lo, uint64_t* saved_hi, uint64_t* total_lo, uint64_t* total_hi) {
+  for (uint32_t g = 0; g < G; ++g)
+    if (caps[g] == 0) return -1;
+  u128 total = 0;
+  for (uint32_t r = 0; r < n_req; ++r)
+    for (uint64_t k = 0; k < req_blk_off[r + 1] - req_blk_off[r]; ++k) total += cost_of(k, B, kind, f_lin, f_attn);
+  *total_lo = (uint64_t)total;
+  *total_hi = (uint64_t)(total >> 64);
+
+  std::atomic<uint32_t> next_cap{0};
+  auto simulate = [&]() {
+    for (;;) {
+      uint32_t g = next_cap.fetch_add(1);
+      if (g >= G) return;
+      uint64_t C = caps[g];
+      std::list<uint32_t> recency;  // front = most recent
+      std::unordered_map<uint32_t, std::list<uint32_t>::iterator> where;
+      uint64_t h = 0;
+      u128 saved = 0;
+      for (uint32_t r = 0; r < n_req; ++r) {
+        bool prefix_ok = true;
+        for (uint64_t k = 0; k < req_blk_off[r + 1] - req_blk_off[r]; ++k) {
+          uint32_t id = ids[req_blk_off[r] + k];
+          auto it = where.find(id);
+          bool resident = it != where.end();
+          if (resident) {
+            recency.splice(recency.begin(), recency, it->second);
+          } else {
+            recency.push_front(id);
+            where[id] = recency.begin();
+            if (recency.size() > C) {
+              where.erase(recency.back());
+              recency.pop_back();
+            }
+          }
+          prefix_ok = prefix_ok && resident;
+          if (prefix_ok) {
+            ++h;
+            saved += cost_of(k, B, kind, f_lin, f_attn);
+          }
+        }
+      }
+      hits[g] = h;
+      saved_lo[g] = (uint64_t)saved;
+      saved_hi[g] = (uint64_t)(saved >> 64);
+    }
+  };
+  if (threads < 1) threads = 1;
+  std::vector<std::thread> pool;
+  for (int t = 1; t < threads; ++t) pool.emplace_back(simulate);
+  simulate();
+  for (auto& th : pool) th.join();
+  return 0;
+}
+
+// Polynomial prefix hash over GF(p), p = 2^61 - 1, evaluated token by token:
+// the prefix tok_0 .. tok_{m-1} of a request maps to
+//     H(m) = rho^m + sum_{t<m} tok_t * rho^(m-1-t)   (mod p),
+// i.e. the polynomial of the sequence (1, tok_0, ..., tok_{m-1}); the leading 1
+// keeps prefixes of different lengths apart.  For each block k of each request
+// the key is (H(B(k+1)) with rho_0, H(B(k+1)) with rho_1), written as
+// keys[2i], keys[2i+1].  The two bases come from `seed` by SplitMix64
+// (Steele, Lea, Flood 2014): rho_b = 2 + (output b of the stream seeded `seed`)
+// mod (p - 3).
+void orc_prefix_hash(const uint32_t* tokens, const uint64_t* req_tok_off, uint32_t n_req, uint32_t B, uint64_t seed,
+                     uint64_t* keys) {
+  const uint64_t P = (1ULL << 61) - 1;
+  uint64_t rho[2];
+  for (int b = 0; b < 2; ++b) {
+    uint64_t z = seed + (uint64_t)(b + 1) * 0x9E3779B97F4A7C15ULL;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+    z = z ^ (z >> 31);
+    rho[b] = 2 + z % (P - 3);
+  }
+  uint64_t i = 0;
+  for (uint32_t r = 0; r < n_req; ++r) {
+    uint64_t len = req_tok_off[r + 1] - req_tok_off[r];
+    uint64_t nblk = len / B;
+    u128 h0 = 1, h1 = 1;  // the leading coefficient 1
+    for (uint64_t t = 0; t < nblk * B; ++t) {
+      uint64_t x = tokens[req_tok_off[r] + t];
+      h0 = (h0 * rho[0] + x) % P;
+      h1 = (h1 * rho[1] + x) % P;
+      if ((t + 1) % B == 0) {
+        keys[2 * i] = (uint64_t)h0;
+        keys[2 * i + 1] = (uint64_t)h1;
+        ++i;
+      }
+    }
+  }
+}
+
+}  // extern "C"
