@@ -1,0 +1,210 @@
+/*
+ * ptc.h — prefix-cache curves on one GPU (GB300, sm_103a).
+ *
+ * Turns a request trace into block-level LRU prefix-cache hit curves and
+ * compute-saved curves for every capacity at once, after "When Fancy Eviction
+ * Fails: Rethinking Cache Replacement For LLM Prefix Reuse":
+ *
+ *   trace (session, timestamp, tokens)       Sec. 3.1 (traces), Sec. 2.3 (sessions)
+ *     -> ptc_hash_blocks     chained per-block prefix keys     Sec. 2.2 (block identity)
+ *     -> ptc_assign_ids      dense block ids                   Sec. 4 ("each KV block is a distinct cache object")
+ *     -> ptc_reuse_indices   previous / next use of each block Sec. 3.2, 5.2 (Belady's next access)
+ *     -> ptc_stack_distance  LRU stack distance of each access App. B ("reuses reachable within C")
+ *     -> ptc_curves          hits and compute saved per C      Sec. 3.2 (hit ratio), Sec. 5.2 (compute savings)
+ *
+ * Conventions shared by every call
+ *   - Pointers are caller-owned DEVICE memory unless the name ends in _host.
+ *     The library allocates nothing: each call takes a device workspace `ws`
+ *     of at least ptc_<call>_workspace_bytes(...) bytes, 256-byte aligned.
+ *     The workspace holds no state between calls.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Work is
+ *     enqueued on it.  Every call returns after reading its device status
+ *     word, so it synchronizes `stream` once before returning; outputs are
+ *     ready when it returns PTC_OK.
+ *   - Errors are returned, never thrown or aborted.  Device-side checks
+ *     (ordering, ranges, bounded waits) set a status word that the call reads
+ *     before returning.  A CUDA runtime error maps to PTC_ERR_CUDA.  On any
+ *     error the contents of the outputs are unspecified.
+ *   - Sizes: the number of block accesses N and of distinct blocks D must be
+ *     below 2^32 - 1 (0xFFFFFFFF is the "none / infinite" marker, PTC_NONE);
+ *     token counts and offsets are 64-bit.
+ *   - Indices are 0-based.  The access stream is requests in trace order and,
+ *     within a request, blocks root-first (depth k = 0, 1, ...).
+ */
+#ifndef PTC_H
+#define PTC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define PTC_NONE 0xFFFFFFFFu
+#define PTC_MAX_BLOCK_SIZE 512u
+#define PTC_MAX_CAPACITIES 1024u
+
+typedef enum {
+  PTC_OK = 0,
+  PTC_ERR_INVALID_ARG = 1,    /* a host-checked argument is out of range, or device data is malformed */
+  PTC_ERR_UNSORTED = 2,       /* request timestamps decrease */
+  PTC_ERR_OVERFLOW = 3,       /* N or D would reach 2^32 - 1, or a cost constant overflows 64 bits */
+  PTC_ERR_WORKSPACE = 4,      /* ws is NULL, misaligned or smaller than the size query returned */
+  PTC_ERR_CUDA = 5,           /* a CUDA runtime call failed */
+  PTC_ERR_TIMEOUT = 6,        /* a device-side wait gave up (bounded spin); no result */
+  PTC_ERR_HASH_COLLISION = 7, /* ptc_verify_ids found two different prefixes under one id */
+  PTC_ERR_NOT_IMPLEMENTED = 8
+} ptc_status;
+
+/* Unsigned 128-bit integer, little-endian halves. */
+typedef struct {
+  uint64_t lo, hi;
+} ptc_u128;
+
+/*
+ * Per-block recompute cost (Sec. 5.2 "compute-savings ratio"; App. C linear
+ * model).  Block k (0-based depth) of a request with block size B costs
+ *   PTC_COST_UNIFORM   1                                   (compute saved = hits)
+ *   PTC_COST_MEASURED  B*f_lin + f_attn * sum_{t=Bk}^{Bk+B-1} (t+1)
+ *   PTC_COST_LINEAR    f_attn * sum_{t=Bk}^{Bk+B-1} (t+1)  (attention term only)
+ * The sum counts, for each token of the block, the positions it attends to.
+ * The measured-shape constants for a 48-layer, 32-head, head-dim-128 MoE with
+ * ~3.3B active parameters are f_lin = 2*3.3e9 and f_attn = 4*48*32*128.
+ */
+enum { PTC_COST_UNIFORM = 0, PTC_COST_MEASURED = 1, PTC_COST_LINEAR = 2 };
+typedef struct {
+  uint64_t f_lin;
+  uint64_t f_attn;
+  int32_t kind;
+} ptc_cost_model;
+
+/* Human-readable name of a status code (static storage). */
+const char* ptc_strerror(ptc_status s);
+/* Library version string (static storage). */
+const char* ptc_version(void);
+
+/*
+ * ptc_hash_blocks — chained block keys (Sec. 2.2: KV state is kept in blocks of
+ * B tokens, 16 in the paper's setup, and a cached block is reusable iff its
+ * entire preceding sequence matches).
+ *
+ * Request r owns tokens[req_tok_off[r] : req_tok_off[r+1]] and has
+ * n_r = floor(len_r / B) full blocks; a trailing partial block is not a cache
+ * object.  Block k of request r gets the key of its whole prefix
+ * [0, B(k+1)): the polynomial of the sequence (1, tok_0, ..., tok_{B(k+1)-1})
+ * over GF(2^61 - 1) at two bases rho_0, rho_1 drawn from `seed` with
+ * SplitMix64 (rho_b = 2 + (output b) mod (2^61 - 4)).  keys_out[i].lo / .hi
+ * are the values at rho_0 / rho_1.  Two different prefixes of at most m
+ * tokens share a key with probability at most (m / (2^61 - 1))^2 (the
+ * Schwartz-Zippel bound for each base); ptc_verify_ids checks exactly.
+ *
+ *   tokens          u32[n_tok]; any alignment (16-byte aligned is fastest)
+ *   req_tok_off     u64[n_req + 1], non-decreasing, req_tok_off[n_req] <= n_tok
+ *   req_ts_us       i64[n_req] arrival times, must be non-decreasing
+ *                   (PTC_ERR_UNSORTED otherwise); may be NULL to skip the check
+ *   block_size      B in [1, PTC_MAX_BLOCK_SIZE]
+ *   keys_out        ptc_u128[keys_cap]; keys_cap >= N is required, and
+ *                   floor(n_tok / B) always suffices
+ *   req_blk_off_out u64[n_req + 1]: first access index of each request; [n_req] = N
+ *   n_access_host_out  receives N on the host
+ */
+size_t ptc_hash_blocks_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size);
+ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off,
+                           const int64_t* req_ts_us, uint32_t n_req, uint32_t block_size, uint64_t seed,
+                           ptc_u128* keys_out, uint64_t keys_cap, uint64_t* req_blk_off_out,
+                           uint64_t* n_access_host_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * ptc_assign_ids — dense block ids (Sec. 4: each KV block is a distinct cache
+ * object).  ids_out[i] in [0, D), numbered by first occurrence in the access
+ * stream: the first access with a given key gets the next unused id.  Equal
+ * keys get equal ids.  D is returned in n_distinct_host_out.
+ *
+ *   keys      ptc_u128[n] from ptc_hash_blocks (values below 2^61 - 1 in both halves)
+ *   ids_out   u32[n]
+ */
+size_t ptc_assign_ids_workspace_bytes(uint64_t n);
+ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t* ids_out, uint64_t* n_distinct_host_out,
+                          void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * ptc_verify_ids — exact check of the ids (Sec. 2.2 identity, without hashing):
+ * every access must carry the same B tokens as the first access of its id,
+ * and its parent (the previous block of its request, or "none" at depth 0)
+ * must have the same id as that first access's parent.  By induction over
+ * depth this makes equal ids equivalent to equal prefixes.  Returns
+ * PTC_ERR_HASH_COLLISION if any access fails the check.
+ *
+ *   tokens, n_tok, req_tok_off, n_req, block_size  as given to ptc_hash_blocks
+ *   req_blk_off  u64[n_req + 1] from ptc_hash_blocks
+ *   ids          u32[n] from ptc_assign_ids, n = req_blk_off[n_req]
+ */
+size_t ptc_verify_ids_workspace_bytes(uint64_t n, uint64_t n_distinct);
+ptc_status ptc_verify_ids(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off, const uint64_t* req_blk_off,
+                          uint32_t n_req, uint32_t block_size, const uint32_t* ids, uint64_t n,
+                          uint64_t n_distinct, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * ptc_reuse_indices — previous and next use of each block (Sec. 3.2 and 5.2:
+ * Belady's policy needs the time until each block's next access).
+ *   prev_out[i] = max{ j < i : ids[j] == ids[i] }, or PTC_NONE
+ *   next_out[i] = min{ j > i : ids[j] == ids[i] }, or PTC_NONE
+ * Computed from a stable radix sort of (id, i) pairs.
+ *
+ *   ids        u32[n], every value < n_distinct (PTC_ERR_INVALID_ARG otherwise)
+ *   prev_out, next_out  u32[n]
+ */
+size_t ptc_reuse_indices_workspace_bytes(uint64_t n, uint64_t n_distinct);
+ptc_status ptc_reuse_indices(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev_out,
+                             uint32_t* next_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * ptc_stack_distance — LRU stack distance of every access (App. B: the stack
+ * distance between reuses decides whether a reuse is reachable within a
+ * cache of C blocks).  With p = prev[i]:
+ *   dist_out[i] = 1 + #{distinct blocks accessed in positions p+1 .. i-1}
+ *               = 1 + #{ j : p < j < i, prev[j] < p or prev[j] == PTC_NONE }
+ * and PTC_NONE (never seen) when p == PTC_NONE.  An access hits in an LRU
+ * cache of C >= 1 blocks iff dist <= C (Mattson et al. 1970).  The count is a
+ * 2-D dominance count answered by N range-rank queries on a wavelet matrix
+ * (Claude, Navarro, Ordonez 2015) built over v_j = prev[j] + 1.
+ *
+ *   prev      u32[n] from ptc_reuse_indices (prev[i] < i or PTC_NONE)
+ *   dist_out  u32[n], 1-based; PTC_NONE for a first access
+ */
+size_t ptc_stack_distance_workspace_bytes(uint64_t n);
+ptc_status ptc_stack_distance(const uint32_t* prev, uint64_t n, uint32_t* dist_out, void* ws, size_t ws_bytes,
+                              void* stream);
+
+/*
+ * ptc_curves — hit and compute-saved curves for every capacity at once
+ * (Sec. 3.2 block hit ratio; Sec. 5.2 compute-savings ratio; prefix reuse
+ * from Sec. 2.2).  Block k of a request is counted as a hit at capacity C iff
+ * every block 0..k of that request is resident, i.e. iff
+ *   e_i = max(dist[j] : j in the request, depth(j) <= k) <= C.
+ *   hits_host_out[g]      = #{ i : e_i <= cap_host[g] }
+ *   saved_host_out[g]     = sum of cost(k_i) over those i   (128-bit)
+ *   total_cost_host_out   = sum of cost(k_i) over all i     (128-bit)
+ * Block hit ratio = hits / N; compute-savings ratio = saved / total.
+ *
+ *   dist          u32[n] from ptc_stack_distance
+ *   req_blk_off   u64[n_req + 1] from ptc_hash_blocks, req_blk_off[n_req] == n
+ *   cm            cost model (host pointer); PTC_ERR_OVERFLOW if a per-block
+ *                 cost could exceed 64 bits
+ *   cap_host      u64[n_cap] capacities in blocks, strictly ascending, >= 1,
+ *                 1 <= n_cap <= PTC_MAX_CAPACITIES (host memory)
+ *   hits_host_out u64[n_cap], saved_host_out ptc_u128[n_cap], total_cost_host_out
+ *                 ptc_u128[1] (host memory)
+ */
+size_t ptc_curves_workspace_bytes(uint64_t n, uint32_t n_req, uint32_t n_cap);
+ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,
+                      uint32_t block_size, const ptc_cost_model* cm, const uint64_t* cap_host, uint32_t n_cap,
+                      uint64_t* hits_host_out, ptc_u128* saved_host_out, ptc_u128* total_cost_host_out, void* ws,
+                      size_t ws_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PTC_H */

@@ -1,0 +1,278 @@
+"""ptc — prefix-cache curves on one GPU (GB300, sm_103a).
+
+A thin binding over the C-ABI library ``libptc.so`` (declared in
+``include/ptc.h``).  Each function marshals arguments and calls the C entry
+point of the same name; every step of the computation runs in the library's
+CUDA kernels.  PyTorch provides device memory and the current CUDA stream.
+
+    keys, req_blk_off, n = ptc_hash_blocks(tokens, req_tok_off, req_ts_us, 16, seed)
+    ids, d               = ptc_assign_ids(keys)
+    prev, nxt            = ptc_reuse_indices(ids, d)
+    dist                 = ptc_stack_distance(prev)
+    curves               = ptc_curves(dist, req_blk_off, 16, caps, PTC_COST_MEASURED)
+
+Arrays are torch CUDA tensors.  Unsigned 32/64-bit arrays travel as int32 /
+int64 tensors holding the same bits (``u32()`` / ``u64()`` give numpy views).
+There is no CPU fallback: without the built library every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import numpy as np
+import torch
+
+from . import build as _build
+
+PTC_NONE = 0xFFFFFFFF
+PTC_COST_UNIFORM, PTC_COST_MEASURED, PTC_COST_LINEAR = 0, 1, 2
+F_LIN = 6_600_000_000          # 2 x 3.3e9 active parameters, FLOPs per token
+F_ATTN = 4 * 48 * 32 * 128     # per attended position: 4 x layers x heads x head_dim
+MAX_CAPACITIES = 1024
+MAX_BLOCK_SIZE = 512
+
+_lock = threading.Lock()
+_lib = None
+
+STATUS = {
+    0: "PTC_OK", 1: "PTC_ERR_INVALID_ARG", 2: "PTC_ERR_UNSORTED", 3: "PTC_ERR_OVERFLOW",
+    4: "PTC_ERR_WORKSPACE", 5: "PTC_ERR_CUDA", 6: "PTC_ERR_TIMEOUT", 7: "PTC_ERR_HASH_COLLISION",
+    8: "PTC_ERR_NOT_IMPLEMENTED",
+}
+
+
+class PtcError(RuntimeError):
+    def __init__(self, call: str, status: int):
+        self.status = status
+        self.name = STATUS.get(status, str(status))
+        super().__init__(f"{call}: {self.name} ({lib().ptc_strerror(status).decode()})")
+
+
+class CostModel(ctypes.Structure):
+    _fields_ = [("f_lin", ctypes.c_uint64), ("f_attn", ctypes.c_uint64), ("kind", ctypes.c_int32)]
+
+
+class U128(ctypes.Structure):
+    _fields_ = [("lo", ctypes.c_uint64), ("hi", ctypes.c_uint64)]
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def lib():
+    """The loaded ``libptc.so``.  Raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        with _lock:
+            if _lib is None:
+                path = _build.LIB
+                if not os.path.exists(path):
+                    raise RuntimeError(f"libptc.so is not built ({path}); run "
+                                       "`python -c 'import __graft_entry__ as g; g.build()'`")
+                L = ctypes.CDLL(path)
+                vp, u32, u64, i64, sz = ctypes.c_void_p, ctypes.c_uint32, ctypes.c_uint64, ctypes.c_int64, ctypes.c_size_t
+                st = ctypes.c_int
+                L.ptc_strerror.restype = ctypes.c_char_p
+                L.ptc_strerror.argtypes = [st]
+                L.ptc_version.restype = ctypes.c_char_p
+                L.ptc_version.argtypes = []
+                L.ptc_hash_blocks_workspace_bytes.restype = sz
+                L.ptc_hash_blocks_workspace_bytes.argtypes = [u32, u64, u32]
+                L.ptc_hash_blocks.restype = st
+                L.ptc_hash_blocks.argtypes = [vp, u64, vp, vp, u32, u32, u64, vp, u64, vp,
+                                              ctypes.POINTER(u64), vp, sz, vp]
+                L.ptc_assign_ids_workspace_bytes.restype = sz
+                L.ptc_assign_ids_workspace_bytes.argtypes = [u64]
+                L.ptc_assign_ids.restype = st
+                L.ptc_assign_ids.argtypes = [vp, u64, vp, ctypes.POINTER(u64), vp, sz, vp]
+                L.ptc_verify_ids_workspace_bytes.restype = sz
+                L.ptc_verify_ids_workspace_bytes.argtypes = [u64, u64]
+                L.ptc_verify_ids.restype = st
+                L.ptc_verify_ids.argtypes = [vp, u64, vp, vp, u32, u32, vp, u64, u64, vp, sz, vp]
+                L.ptc_reuse_indices_workspace_bytes.restype = sz
+                L.ptc_reuse_indices_workspace_bytes.argtypes = [u64, u64]
+                L.ptc_reuse_indices.restype = st
+                L.ptc_reuse_indices.argtypes = [vp, u64, u64, vp, vp, vp, sz, vp]
+                L.ptc_stack_distance_workspace_bytes.restype = sz
+                L.ptc_stack_distance_workspace_bytes.argtypes = [u64]
+                L.ptc_stack_distance.restype = st
+                L.ptc_stack_distance.argtypes = [vp, u64, vp, vp, sz, vp]
+                L.ptc_curves_workspace_bytes.restype = sz
+                L.ptc_curves_workspace_bytes.argtypes = [u64, u32, u32]
+                L.ptc_curves.restype = st
+                L.ptc_curves.argtypes = [vp, u64, vp, u32, u32, ctypes.POINTER(CostModel), vp, u32, vp, vp,
+                                         ctypes.POINTER(U128), vp, sz, vp]
+                del i64
+                _lib = L
+    return _lib
+
+
+def version() -> str:
+    return lib().ptc_version().decode()
+
+
+def _check(call: str, rc: int):
+    if rc != 0:
+        raise PtcError(call, rc)
+
+
+def _dev(t: torch.Tensor) -> torch.device:
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    return t.device
+
+
+def _stream(device) -> int:
+    return torch.cuda.current_stream(device).cuda_stream
+
+
+def _ptr(t) -> int | None:
+    return None if t is None else t.data_ptr()
+
+
+def _workspace(nbytes: int, device, ws: torch.Tensor | None = None) -> torch.Tensor:
+    nbytes = max(int(nbytes), 256)
+    if ws is not None and ws.numel() >= nbytes and ws.device == device:
+        return ws
+    return torch.empty(nbytes, dtype=torch.uint8, device=device)
+
+
+def u32(t: torch.Tensor) -> np.ndarray:
+    """A host numpy uint32 view of an int32 tensor's bits."""
+    return t.detach().cpu().numpy().view(np.uint32)
+
+
+def u64(t: torch.Tensor) -> np.ndarray:
+    return t.detach().cpu().numpy().view(np.uint64)
+
+
+def to_device_u32(a, device="cuda") -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.uint32).view(np.int32)).to(device)
+
+
+def to_device_u64(a, device="cuda") -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.uint64).view(np.int64)).to(device)
+
+
+# ---------------------------------------------------------------- the five calls
+def ptc_hash_blocks(tokens: torch.Tensor, req_tok_off: torch.Tensor, req_ts_us: torch.Tensor | None,
+                    block_size: int, seed: int, keys_cap: int | None = None, ws: torch.Tensor | None = None):
+    """Chained block keys.  Returns (keys int64[N, 2], req_blk_off int64[R+1], N)."""
+    dev = _dev(req_tok_off)
+    n_req = req_tok_off.numel() - 1
+    n_tok = tokens.numel()
+    cap = n_tok // block_size if keys_cap is None else int(keys_cap)
+    keys = torch.empty((max(cap, 1), 2), dtype=torch.int64, device=dev)
+    blk_off = torch.empty(n_req + 1, dtype=torch.int64, device=dev)
+    need = lib().ptc_hash_blocks_workspace_bytes(n_req, n_tok, block_size)
+    w = _workspace(need, dev, ws)
+    n = ctypes.c_uint64(0)
+    rc = lib().ptc_hash_blocks(_ptr(tokens), n_tok, _ptr(req_tok_off), _ptr(req_ts_us), n_req, block_size,
+                               int(seed) & (2**64 - 1), _ptr(keys), cap, _ptr(blk_off), ctypes.byref(n),
+                               _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_hash_blocks", rc)
+    return keys[: n.value], blk_off, int(n.value)
+
+
+def ptc_assign_ids(keys: torch.Tensor, ws: torch.Tensor | None = None):
+    """Dense ids in first-occurrence order.  Returns (ids int32[N], D)."""
+    dev = _dev(keys)
+    n = keys.shape[0]
+    ids = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
+    w = _workspace(lib().ptc_assign_ids_workspace_bytes(n), dev, ws)
+    d = ctypes.c_uint64(0)
+    rc = lib().ptc_assign_ids(_ptr(keys), n, _ptr(ids), ctypes.byref(d), _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_assign_ids", rc)
+    return ids[:n], int(d.value)
+
+
+def ptc_verify_ids(tokens, req_tok_off, req_blk_off, block_size: int, ids: torch.Tensor, n_distinct: int,
+                   ws: torch.Tensor | None = None) -> None:
+    """Exact check of ids against tokens; raises PtcError(PTC_ERR_HASH_COLLISION)."""
+    dev = _dev(ids)
+    n = ids.numel()
+    w = _workspace(lib().ptc_verify_ids_workspace_bytes(n, n_distinct), dev, ws)
+    rc = lib().ptc_verify_ids(_ptr(tokens), tokens.numel(), _ptr(req_tok_off), _ptr(req_blk_off), req_tok_off.numel() - 1,
+                              block_size, _ptr(ids), n, n_distinct, _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_verify_ids", rc)
+
+
+def ptc_reuse_indices(ids: torch.Tensor, n_distinct: int, ws: torch.Tensor | None = None):
+    """Previous / next use of every access.  Returns (prev int32[N], next int32[N])."""
+    dev = _dev(ids)
+    n = ids.numel()
+    prev = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
+    nxt = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
+    w = _workspace(lib().ptc_reuse_indices_workspace_bytes(n, n_distinct), dev, ws)
+    rc = lib().ptc_reuse_indices(_ptr(ids), n, n_distinct, _ptr(prev), _ptr(nxt), _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_reuse_indices", rc)
+    return prev[:n], nxt[:n]
+
+
+def ptc_stack_distance(prev: torch.Tensor, ws: torch.Tensor | None = None) -> torch.Tensor:
+    """LRU stack distance of every access (1-based; PTC_NONE for a first access)."""
+    dev = _dev(prev)
+    n = prev.numel()
+    dist = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
+    w = _workspace(lib().ptc_stack_distance_workspace_bytes(n), dev, ws)
+    rc = lib().ptc_stack_distance(_ptr(prev), n, _ptr(dist), _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_stack_distance", rc)
+    return dist[:n]
+
+
+def ptc_curves(dist: torch.Tensor, req_blk_off: torch.Tensor, block_size: int, caps, kind: int = PTC_COST_MEASURED,
+               f_lin: int = F_LIN, f_attn: int = F_ATTN, ws: torch.Tensor | None = None) -> dict:
+    """Hit and compute-saved curves over the capacity grid ``caps`` (blocks).
+
+    Returns {"hits": [int], "saved": [int], "total_cost": int} with exact
+    integers (the 128-bit sums joined)."""
+    dev = _dev(req_blk_off)
+    n = dist.numel()
+    caps = np.ascontiguousarray(caps, dtype=np.uint64)
+    G = caps.shape[0]
+    hits = np.zeros(G, dtype=np.uint64)
+    saved = np.zeros(2 * G, dtype=np.uint64)
+    total = U128()
+    cm = CostModel(int(f_lin), int(f_attn), int(kind))
+    w = _workspace(lib().ptc_curves_workspace_bytes(n, req_blk_off.numel() - 1, G), dev, ws)
+    rc = lib().ptc_curves(_ptr(dist), n, _ptr(req_blk_off), req_blk_off.numel() - 1, block_size, ctypes.byref(cm),
+                          caps.ctypes.data, G, hits.ctypes.data, saved.ctypes.data, ctypes.byref(total),
+                          _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_curves", rc)
+    return {"hits": [int(h) for h in hits],
+            "saved": [int(saved[2 * g + 1]) << 64 | int(saved[2 * g]) for g in range(G)],
+            "total_cost": int(total.hi) << 64 | int(total.lo)}
+
+
+def workspace_bytes(n_req: int, n_tok: int, block_size: int, n: int | None = None, n_cap: int = MAX_CAPACITIES) -> int:
+    """Largest workspace any of the five calls needs for a trace of this size
+    (N defaults to its upper bound n_tok // block_size)."""
+    L = lib()
+    n = n_tok // block_size if n is None else n
+    return max(L.ptc_hash_blocks_workspace_bytes(n_req, n_tok, block_size), L.ptc_assign_ids_workspace_bytes(n),
+               L.ptc_reuse_indices_workspace_bytes(n, n), L.ptc_stack_distance_workspace_bytes(n),
+               L.ptc_curves_workspace_bytes(n, n_req, n_cap), L.ptc_verify_ids_workspace_bytes(n, n))
+
+
+def pipeline(tokens, req_tok_off, req_ts_us, block_size: int, caps_for, kind: int = PTC_COST_MEASURED,
+             seed: int = 0, f_lin: int = F_LIN, f_attn: int = F_ATTN, ws: torch.Tensor | None = None,
+             keep: bool = True) -> dict:
+    """All five calls on one trace resident on the GPU.  ``caps_for`` is the
+    capacity grid, or a function of D (distinct blocks) returning it.  One
+    workspace (``ws``, grown if too small) serves every call."""
+    dev = _dev(req_tok_off)
+    if ws is None:
+        ws = _workspace(workspace_bytes(req_tok_off.numel() - 1, tokens.numel(), block_size), dev)
+    keys, blk_off, n = ptc_hash_blocks(tokens, req_tok_off, req_ts_us, block_size, seed, ws=ws)
+    ids, d = ptc_assign_ids(keys, ws=ws)
+    prev, nxt = ptc_reuse_indices(ids, d, ws=ws)
+    dist = ptc_stack_distance(prev, ws=ws)
+    caps = caps_for(d) if callable(caps_for) else caps_for
+    cur = ptc_curves(dist, blk_off, block_size, caps, kind, f_lin, f_attn, ws=ws)
+    out = dict(n_access=n, n_distinct=d, caps=np.asarray(caps, dtype=np.uint64), **cur)
+    if keep:
+        out.update(keys=keys, req_blk_off=blk_off, ids=ids, prev=prev, next=nxt, dist=dist)
+    return out

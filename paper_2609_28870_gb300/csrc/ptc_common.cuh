@@ -1,0 +1,283 @@
+// Shared device/host helpers of the ptc kernels (sm_103a).
+//
+//  * Device status block: every call's workspace starts with one.  Kernels
+//    report malformed input and give-ups of bounded waits by OR-ing flags into
+//    it; the C-ABI entry reads it back before returning.  No kernel traps.
+//  * Decoupled look-back (Merrill & Garland 2016) for single-pass scans: tiles
+//    take dynamic ids from a counter so that every predecessor of a running
+//    tile has started, publish their aggregate, then their inclusive prefix.
+//    Status words carry a 6-bit epoch (one per launch inside a call), so one
+//    zeroing per call serves every launch.  Every wait is bounded.
+//  * Arithmetic in GF(p), p = 2^61 - 1.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace ptc {
+
+constexpr uint32_t kNone = 0xFFFFFFFFu;
+constexpr uint64_t kP61 = (1ULL << 61) - 1;
+constexpr uint32_t kFull = 0xFFFFFFFFu;
+
+// error flags in DevStatus::err
+enum : uint32_t {
+  kErrTimeout = 1u,
+  kErrUnsorted = 2u,
+  kErrInvalid = 4u,
+  kErrOverflow = 8u,
+  kErrCollision = 16u,
+  kErrTableFull = 32u,
+};
+
+constexpr int kMaxEpochs = 64;
+
+struct DevStatus {
+  uint32_t err;
+  uint32_t pad0;
+  uint64_t value[8];              // per-call results (N, D, max depth ...)
+  uint32_t tile_ctr[kMaxEpochs];  // dynamic tile counter of each launch
+};
+static_assert(sizeof(DevStatus) <= 512, "status block");
+constexpr size_t kStatusBytes = 512;
+
+// Bounded spin: about 2^20 polls with capped exponential back-off (~1 s).
+constexpr uint32_t kSpinCap = 1u << 20;
+
+__device__ __forceinline__ void raise_err(DevStatus* st, uint32_t f) { atomicOr(&st->err, f); }
+
+__device__ __forceinline__ uint32_t next_tile(DevStatus* st, int epoch) {
+  __shared__ uint32_t s_tile;
+  if (threadIdx.x == 0) s_tile = atomicAdd(&st->tile_ctr[epoch], 1u);
+  __syncthreads();
+  return s_tile;
+}
+
+__device__ __forceinline__ uint64_t ld_relaxed_u64(const uint64_t* p) {
+  uint64_t v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_relaxed_u64(uint64_t* p, uint64_t v) {
+  asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+__device__ __forceinline__ uint32_t ld_relaxed_u32(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_relaxed_u32(uint32_t* p, uint32_t v) {
+  asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint64_t ld_cg_u64(const uint64_t* p) {
+  uint64_t v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ uint64_t warp_sum_u64(uint64_t v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+  return v;
+}
+
+// ---------------------------------------------------------------------------
+// Packed look-back for sums below 2^56: word = epoch(6) | flag(2) | value(56).
+// flag 1 = aggregate, 2 = inclusive prefix.  Called by all 32 lanes of ONE
+// warp; returns the exclusive prefix of `tile` (0 if the wait gave up, with
+// kErrTimeout raised).
+// ---------------------------------------------------------------------------
+constexpr uint64_t kLbValMask = (1ULL << 56) - 1;
+__device__ __forceinline__ uint64_t lb_pack(uint32_t epoch, uint32_t flag, uint64_t v) {
+  return ((uint64_t)epoch << 58) | ((uint64_t)flag << 56) | (v & kLbValMask);
+}
+
+__device__ inline uint64_t lookback_sum(uint64_t* words, uint32_t tile, uint64_t agg, uint32_t epoch,
+                                        DevStatus* st) {
+  const uint32_t lane = threadIdx.x & 31;
+  if (tile == 0) {
+    if (lane == 0) st_relaxed_u64(&words[0], lb_pack(epoch, 2, agg));
+    return 0;
+  }
+  if (lane == 0) st_relaxed_u64(&words[tile], lb_pack(epoch, 1, agg));
+  uint64_t excl = 0;
+  int64_t base = (int64_t)tile - 1;
+  uint32_t spins = 0, ns = 20;
+  for (;;) {
+    int64_t idx = base - (int64_t)lane;
+    uint32_t f = 2;
+    uint64_t v = 0;
+    if (idx >= 0) {
+      uint64_t w = ld_relaxed_u64(&words[idx]);
+      f = ((uint32_t)(w >> 58) == epoch) ? (uint32_t)((w >> 56) & 3) : 0u;
+      v = w & kLbValMask;
+    }
+    if (__any_sync(kFull, f == 0)) {
+      if (++spins > kSpinCap) {
+        if (lane == 0) raise_err(st, kErrTimeout);
+        return 0;
+      }
+      __nanosleep(ns);
+      if (ns < 1000) ns += ns;
+      continue;
+    }
+    uint32_t incl = __ballot_sync(kFull, f == 2);
+    if (incl) {
+      uint32_t first = __ffs(incl) - 1;
+      if (lane > first) v = 0;
+      excl += warp_sum_u64(v);
+      break;
+    }
+    excl += warp_sum_u64(v);
+    base -= 32;
+  }
+  if (lane == 0) st_relaxed_u64(&words[tile], lb_pack(epoch, 2, excl + agg));
+  return excl;
+}
+
+// ---------------------------------------------------------------------------
+// Generic look-back for a payload T with an associative operator `op` and a
+// two-sided identity.  Status word per tile: epoch << 2 | flag.  Payloads go
+// to separate aggregate / inclusive arrays, published before the flag with a
+// fence.  Called by ONE thread.
+// ---------------------------------------------------------------------------
+template <class T>
+struct LbArrays {
+  uint32_t* status;
+  T* agg;
+  T* incl;
+};
+
+template <class T>
+__device__ __forceinline__ void lb_store(T* dst, const T& v) {
+  volatile uint64_t* d = reinterpret_cast<volatile uint64_t*>(dst);
+  const uint64_t* s = reinterpret_cast<const uint64_t*>(&v);
+#pragma unroll
+  for (int i = 0; i < (int)(sizeof(T) / 8); ++i) d[i] = s[i];
+}
+template <class T>
+__device__ __forceinline__ T lb_load(const T* src) {
+  T v;
+  const volatile uint64_t* s = reinterpret_cast<const volatile uint64_t*>(src);
+  uint64_t* d = reinterpret_cast<uint64_t*>(&v);
+#pragma unroll
+  for (int i = 0; i < (int)(sizeof(T) / 8); ++i) d[i] = s[i];
+  return v;
+}
+
+template <class T, class Op>
+__device__ inline T lookback_generic(LbArrays<T> a, uint32_t tile, const T& agg, const T& identity, Op op,
+                                     uint32_t epoch, DevStatus* st) {
+  static_assert(sizeof(T) % 8 == 0, "payload must be a multiple of 8 bytes");
+  if (tile == 0) {
+    lb_store(&a.incl[0], agg);
+    __threadfence();
+    st_relaxed_u32(&a.status[0], (epoch << 2) | 2u);
+    return identity;
+  }
+  lb_store(&a.agg[tile], agg);
+  __threadfence();
+  st_relaxed_u32(&a.status[tile], (epoch << 2) | 1u);
+  T acc = identity;
+  int64_t j = (int64_t)tile - 1;
+  uint32_t spins = 0, ns = 20;
+  while (j >= 0) {
+    uint32_t s = ld_relaxed_u32(&a.status[j]);
+    uint32_t f = ((s >> 2) == epoch) ? (s & 3u) : 0u;
+    if (f == 0) {
+      if (++spins > kSpinCap) {
+        raise_err(st, kErrTimeout);
+        return identity;
+      }
+      __nanosleep(ns);
+      if (ns < 1000) ns += ns;
+      continue;
+    }
+    __threadfence();
+    if (f == 2) {
+      acc = op(lb_load(&a.incl[j]), acc);
+      break;
+    }
+    acc = op(lb_load(&a.agg[j]), acc);
+    --j;
+  }
+  T inc = op(acc, agg);
+  lb_store(&a.incl[tile], inc);
+  __threadfence();
+  st_relaxed_u32(&a.status[tile], (epoch << 2) | 2u);
+  return acc;
+}
+
+// ---------------------------------------------------------------------------
+// GF(2^61 - 1)
+// ---------------------------------------------------------------------------
+__host__ __device__ __forceinline__ uint64_t p61_fold(uint64_t x) {  // x < 2^64 -> [0, p)
+  x = (x & kP61) + (x >> 61);
+  x = (x & kP61) + (x >> 61);
+  return x >= kP61 ? x - kP61 : x;
+}
+__host__ __device__ __forceinline__ uint64_t p61_add(uint64_t a, uint64_t b) {  // a, b < p
+  uint64_t r = a + b;
+  return r >= kP61 ? r - kP61 : r;
+}
+__host__ __device__ __forceinline__ uint64_t p61_mul(uint64_t a, uint64_t b) {  // a, b < p
+#ifdef __CUDA_ARCH__
+  uint64_t lo = a * b, hi = __umul64hi(a, b);
+#else
+  unsigned __int128 t = (unsigned __int128)a * b;
+  uint64_t lo = (uint64_t)t, hi = (uint64_t)(t >> 64);
+#endif
+  // a*b < 2^122, so hi < 2^58 and hi << 3 does not overflow
+  uint64_t r = (lo & kP61) + (lo >> 61) + (hi << 3);
+  r = (r & kP61) + (r >> 61);
+  return r >= kP61 ? r - kP61 : r;
+}
+__host__ __device__ inline uint64_t p61_pow(uint64_t b, uint64_t e) {
+  uint64_t r = 1;
+  while (e) {
+    if (e & 1) r = p61_mul(r, b);
+    b = p61_mul(b, b);
+    e >>= 1;
+  }
+  return r;
+}
+
+__host__ __device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t n) {
+  uint64_t z = seed + (n + 1) * 0x9E3779B97F4A7C15ULL;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+  return z ^ (z >> 31);
+}
+
+__device__ __forceinline__ uint32_t lanemask_lt() {
+  uint32_t m;
+  asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+  return m;
+}
+
+}  // namespace ptc
+
+// ---------------------------------------------------------------------------
+// Host side: workspace carving and status read-back
+// ---------------------------------------------------------------------------
+#include <cstddef>
+
+namespace ptc {
+
+struct Carver {
+  char* base;
+  size_t off = 0;
+  explicit Carver(void* b) : base((char*)b) {}
+  template <class T>
+  T* take(size_t count, size_t align = 256) {
+    off = (off + align - 1) / align * align;
+    T* p = base ? (T*)(base + off) : nullptr;
+    off += count * sizeof(T);
+    return p;
+  }
+  size_t bytes() const { return (off + 255) / 256 * 256; }
+};
+
+inline uint32_t ceil_div_u32(uint64_t a, uint64_t b) { return (uint32_t)((a + b - 1) / b); }
+
+}  // namespace ptc

@@ -1,0 +1,342 @@
+// Stage d: hit and compute-saved curves for every capacity at once
+// (paper Sec. 3.2 block hit ratio, Sec. 5.2 compute-savings ratio, prefix
+// reuse from Sec. 2.2).
+//
+// Block k of a request is a prefix hit at capacity C iff blocks 0..k of the
+// request are all resident, i.e. iff e_i = max(dist over the request's blocks
+// up to k) <= C (an access hits alone iff dist <= C: Mattson inclusion).  So
+// one pass computes e_i (a per-request running max: segmented scan with
+// decoupled look-back), finds the first capacity >= e_i, and histograms
+// count and depth per capacity bin.  Every cost model is affine in depth,
+// cost(k) = alpha + beta k, so compute saved = alpha * hits + beta * (sum of k),
+// formed exactly in 128 bits by the finalize kernel.
+//   k_heads     marks the first access of every non-empty request (bitmap)
+//   k_curves    running max, bin search in shared memory, run-merged
+//               shared histograms, one global atomic per non-empty bin
+//   k_finalize  cumulative sums over bins; 128-bit saved and total cost
+#include "ptc_internal.h"
+
+namespace ptc {
+namespace {
+
+constexpr int kCvThreads = 512;
+constexpr int kCvPer = 8;
+constexpr int kCvTile = kCvThreads * kCvPer;
+constexpr int kEpochCurves = 1;
+
+__global__ void k_heads(const uint64_t* __restrict__ blk_off, uint32_t R, uint64_t n, uint32_t* __restrict__ bitmap,
+                        DevStatus* st) {
+  const uint64_t r = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= R) return;
+  const uint64_t a = blk_off[r], b = blk_off[r + 1];
+  if (b < a || b > n || (r == 0 && a != 0) || (r + 1 == R && b != n)) {
+    raise_err(st, kErrInvalid);
+    return;
+  }
+  if (b > a) atomicOr(&bitmap[a >> 5], 1u << (a & 31));
+}
+
+struct RunMax {  // (segment-start flag, running max, start index of the segment)
+  uint64_t m;
+  uint64_t start;
+  uint64_t f;
+};
+struct RunMaxOp {
+  __device__ RunMax operator()(const RunMax& a, const RunMax& b) const {
+    RunMax r;
+    r.f = a.f | b.f;
+    r.m = b.f ? b.m : (a.m > b.m ? a.m : b.m);
+    r.start = b.f ? b.start : a.start;
+    return r;
+  }
+};
+
+struct CurveArgs {
+  const uint32_t* dist;
+  uint64_t n;
+  const uint32_t* bitmap;
+  const uint64_t* caps;  // device copy of the grid
+  uint32_t G;
+  unsigned long long* cnt;   // G + 1 bins (last: miss at every capacity)
+  unsigned long long* ksum;  // G + 1 bins
+  LbArrays<RunMax> lb;
+  DevStatus* st;
+};
+
+__global__ void __launch_bounds__(kCvThreads) k_curves(CurveArgs a) {
+  __shared__ uint32_t s_cap[PTC_MAX_CAPACITIES];
+  __shared__ uint32_t s_cnt[PTC_MAX_CAPACITIES + 1];
+  __shared__ unsigned long long s_ks[PTC_MAX_CAPACITIES + 1];
+  __shared__ RunMax s_w[kCvThreads / 32];
+  __shared__ RunMax s_carry;
+  const uint32_t G = a.G;
+  for (uint32_t g = threadIdx.x; g < G; g += kCvThreads)
+    s_cap[g] = a.caps[g] >= (uint64_t)kNone ? kNone - 1 : (uint32_t)a.caps[g];
+  for (uint32_t g = threadIdx.x; g <= G; g += kCvThreads) {
+    s_cnt[g] = 0;
+    s_ks[g] = 0;
+  }
+  const uint32_t tile = next_tile(a.st, kEpochCurves);
+  const uint64_t i0 = (uint64_t)tile * kCvTile + (uint64_t)threadIdx.x * kCvPer;
+
+  uint32_t d[kCvPer];
+  if (i0 + kCvPer <= a.n && ((reinterpret_cast<uintptr_t>(a.dist) & 15) == 0)) {
+    const uint4 x = __ldcs(reinterpret_cast<const uint4*>(a.dist + i0));
+    const uint4 y = __ldcs(reinterpret_cast<const uint4*>(a.dist + i0 + 4));
+    d[0] = x.x; d[1] = x.y; d[2] = x.z; d[3] = x.w;
+    d[4] = y.x; d[5] = y.y; d[6] = y.z; d[7] = y.w;
+  } else {
+#pragma unroll
+    for (int j = 0; j < kCvPer; ++j) d[j] = i0 + j < a.n ? a.dist[i0 + j] : 0u;
+  }
+  const uint32_t heads = i0 < a.n ? (a.bitmap[i0 >> 5] >> (i0 & 31)) & 0xFFu : 0u;
+
+  // thread-local inclusive running max
+  RunMax loc{0, 0, 0};
+  uint64_t e[kCvPer], st_idx[kCvPer];
+  uint32_t has_head = 0;  // bit j: a head at or before j inside this thread
+#pragma unroll
+  for (int j = 0; j < kCvPer; ++j) {
+    const uint64_t dv = (i0 + j < a.n) ? d[j] : 0u;
+    if ((heads >> j) & 1u) {
+      loc.f = 1;
+      loc.m = dv;
+      loc.start = i0 + j;
+    } else {
+      loc.m = dv > loc.m ? dv : loc.m;
+    }
+    e[j] = loc.m;
+    st_idx[j] = loc.start;
+    if (loc.f) has_head |= 1u << j;
+  }
+  // CTA-wide exclusive segmented scan of thread aggregates
+  RunMaxOp op;
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  RunMax x = loc;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    RunMax y;
+    y.m = __shfl_up_sync(kFull, x.m, o);
+    y.start = __shfl_up_sync(kFull, x.start, o);
+    y.f = __shfl_up_sync(kFull, x.f, o);
+    if (lane >= (uint32_t)o) x = op(y, x);
+  }
+  if (lane == 31) s_w[w] = x;
+  __syncthreads();
+  if (w == 0) {
+    RunMax z = lane < kCvThreads / 32 ? s_w[lane] : RunMax{0, 0, 0};
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      RunMax y;
+      y.m = __shfl_up_sync(kFull, z.m, o);
+      y.start = __shfl_up_sync(kFull, z.start, o);
+      y.f = __shfl_up_sync(kFull, z.f, o);
+      if (lane >= (uint32_t)o) z = op(y, z);
+    }
+    if (lane < kCvThreads / 32) s_w[lane] = z;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) s_carry = lookback_generic(a.lb, tile, s_w[kCvThreads / 32 - 1], RunMax{0, 0, 0}, op,
+                                                   kEpochCurves, a.st);
+  __syncthreads();
+  // exclusive prefix of this thread = carry (+) warps before (+) lanes before
+  RunMax pre = s_carry;
+  if (w > 0) pre = op(pre, s_w[w - 1]);
+  {
+    RunMax y;
+    y.m = __shfl_up_sync(kFull, x.m, 1);
+    y.start = __shfl_up_sync(kFull, x.start, 1);
+    y.f = __shfl_up_sync(kFull, x.f, 1);
+    if (lane > 0) pre = op(pre, y);
+  }
+
+  // bin and accumulate with run merging
+  uint32_t cur_g = 0xFFFFFFFFu, run_c = 0;
+  unsigned long long run_k = 0;
+#pragma unroll
+  for (int j = 0; j < kCvPer; ++j) {
+    if (i0 + j >= a.n) break;
+    uint64_t ej = e[j], sj = st_idx[j];
+    if (!((has_head >> j) & 1u)) {
+      ej = pre.m > ej ? pre.m : ej;
+      sj = pre.start;
+    }
+    uint32_t g;
+    if (ej >= (uint64_t)kNone) {
+      g = G;
+    } else {  // first capacity >= ej
+      uint32_t lo = 0, hi = G;
+      while (lo < hi) {
+        const uint32_t mid = (lo + hi) >> 1;
+        if (s_cap[mid] >= (uint32_t)ej)
+          hi = mid;
+        else
+          lo = mid + 1;
+      }
+      g = lo;
+    }
+    const unsigned long long k = (i0 + j) - sj;
+    if (g != cur_g) {
+      if (run_c) {
+        atomicAdd(&s_cnt[cur_g], run_c);
+        atomicAdd(&s_ks[cur_g], run_k);
+      }
+      cur_g = g;
+      run_c = 0;
+      run_k = 0;
+    }
+    ++run_c;
+    run_k += k;
+  }
+  if (run_c) {
+    atomicAdd(&s_cnt[cur_g], run_c);
+    atomicAdd(&s_ks[cur_g], run_k);
+  }
+  __syncthreads();
+  for (uint32_t g = threadIdx.x; g <= G; g += kCvThreads) {
+    if (s_cnt[g]) {
+      atomicAdd(&a.cnt[g], (unsigned long long)s_cnt[g]);
+      atomicAdd(&a.ksum[g], s_ks[g]);
+    }
+  }
+}
+
+struct U128 {
+  uint64_t lo, hi;
+};
+__device__ __forceinline__ U128 mul_u64(uint64_t a, uint64_t b) { return U128{a * b, __umul64hi(a, b)}; }
+__device__ __forceinline__ U128 add_u128(U128 a, U128 b) {
+  U128 r;
+  r.lo = a.lo + b.lo;
+  r.hi = a.hi + b.hi + (r.lo < a.lo ? 1 : 0);
+  return r;
+}
+
+// out layout: hits[G] | saved[G] (lo, hi) | total (lo, hi)
+__global__ void k_finalize(const unsigned long long* __restrict__ cnt, const unsigned long long* __restrict__ ksum,
+                           uint32_t G, uint64_t alpha, uint64_t beta, uint64_t* __restrict__ out) {
+  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+  uint64_t h = 0, k = 0;
+  for (uint32_t g = 0; g < G; ++g) {
+    h += cnt[g];
+    k += ksum[g];
+    const U128 s = add_u128(mul_u64(alpha, h), mul_u64(beta, k));
+    out[g] = h;
+    out[G + 2 * g] = s.lo;
+    out[G + 2 * g + 1] = s.hi;
+  }
+  const uint64_t hn = h + cnt[G], kn = k + ksum[G];
+  const U128 t = add_u128(mul_u64(alpha, hn), mul_u64(beta, kn));
+  out[3 * G] = t.lo;
+  out[3 * G + 1] = t.hi;
+}
+
+struct CurvesLayout {
+  DevStatus* st;
+  unsigned long long* cnt;
+  unsigned long long* ksum;
+  uint32_t* bitmap;
+  uint32_t* lb_status;
+  RunMax* lb_agg;
+  RunMax* lb_incl;
+  uint64_t* caps;
+  uint64_t* out;
+  size_t zero_bytes;
+  size_t total;
+};
+
+CurvesLayout curves_layout(void* ws, uint64_t n, uint32_t G) {
+  CurvesLayout L;
+  Carver cv(ws);
+  const uint32_t tiles = ceil_div_u32(n, kCvTile) + 1;
+  L.st = cv.take<DevStatus>(1);
+  L.cnt = cv.take<unsigned long long>(PTC_MAX_CAPACITIES + 1);
+  L.ksum = cv.take<unsigned long long>(PTC_MAX_CAPACITIES + 1);
+  L.bitmap = cv.take<uint32_t>(n / 32 + 2);
+  L.lb_status = cv.take<uint32_t>(tiles);
+  L.zero_bytes = cv.off;
+  L.lb_agg = cv.take<RunMax>(tiles);
+  L.lb_incl = cv.take<RunMax>(tiles);
+  L.caps = cv.take<uint64_t>(PTC_MAX_CAPACITIES);
+  L.out = cv.take<uint64_t>(3 * PTC_MAX_CAPACITIES + 2);
+  L.total = cv.bytes();
+  (void)G;
+  return L;
+}
+
+bool mul_ok(uint64_t a, uint64_t b, uint64_t* r) {
+  unsigned __int128 t = (unsigned __int128)a * b;
+  *r = (uint64_t)t;
+  return (t >> 64) == 0;
+}
+
+}  // namespace
+}  // namespace ptc
+
+using namespace ptc;
+
+extern "C" size_t ptc_curves_workspace_bytes(uint64_t n, uint32_t n_req, uint32_t n_cap) {
+  (void)n_req;
+  return curves_layout(nullptr, n, n_cap).total;
+}
+
+extern "C" ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,
+                                 uint32_t block_size, const ptc_cost_model* cm, const uint64_t* cap_host, uint32_t n_cap,
+                                 uint64_t* hits_host_out, ptc_u128* saved_host_out, ptc_u128* total_cost_host_out,
+                                 void* ws, size_t ws_bytes, void* stream) {
+  if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
+  if (!cm || !cap_host || !hits_host_out || !saved_host_out || !total_cost_host_out) return PTC_ERR_INVALID_ARG;
+  if (n_cap < 1 || n_cap > PTC_MAX_CAPACITIES) return PTC_ERR_INVALID_ARG;
+  if (block_size < 1 || block_size > PTC_MAX_BLOCK_SIZE) return PTC_ERR_INVALID_ARG;
+  if (n > 0 && (!dist || !req_blk_off || n_req == 0)) return PTC_ERR_INVALID_ARG;
+  for (uint32_t g = 0; g < n_cap; ++g)
+    if (cap_host[g] < 1 || (g && cap_host[g] <= cap_host[g - 1])) return PTC_ERR_INVALID_ARG;
+  // cost(k) = alpha + beta k
+  const uint64_t B = block_size;
+  uint64_t alpha = 0, beta = 0, lin = 0, attn0 = 0;
+  if (cm->kind == PTC_COST_UNIFORM) {
+    alpha = 1;
+  } else if (cm->kind == PTC_COST_MEASURED || cm->kind == PTC_COST_LINEAR) {
+    if (!mul_ok(cm->f_attn, B * (B + 1) / 2, &attn0) || !mul_ok(cm->f_attn, B * B, &beta)) return PTC_ERR_OVERFLOW;
+    if (cm->kind == PTC_COST_MEASURED && !mul_ok(cm->f_lin, B, &lin)) return PTC_ERR_OVERFLOW;
+    alpha = lin + attn0;
+    if (alpha < lin) return PTC_ERR_OVERFLOW;
+  } else {
+    return PTC_ERR_INVALID_ARG;
+  }
+  if (!ws_ok(ws, ws_bytes, curves_layout(nullptr, n, n_cap).total)) return PTC_ERR_WORKSPACE;
+  cudaStream_t s = (cudaStream_t)stream;
+  const CurvesLayout L = curves_layout(ws, n, n_cap);
+  if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
+  if (cudaMemcpyAsync(L.caps, cap_host, sizeof(uint64_t) * n_cap, cudaMemcpyHostToDevice, s) != cudaSuccess)
+    return PTC_ERR_CUDA;
+  if (n > 0) {
+    k_heads<<<ceil_div_u32(n_req, 256), 256, 0, s>>>(req_blk_off, n_req, n, L.bitmap, L.st);
+    CurveArgs a;
+    a.dist = dist;
+    a.n = n;
+    a.bitmap = L.bitmap;
+    a.caps = L.caps;
+    a.G = n_cap;
+    a.cnt = L.cnt;
+    a.ksum = L.ksum;
+    a.lb = LbArrays<RunMax>{L.lb_status, L.lb_agg, L.lb_incl};
+    a.st = L.st;
+    k_curves<<<ceil_div_u32(n, kCvTile), kCvThreads, 0, s>>>(a);
+  }
+  k_finalize<<<1, 32, 0, s>>>(L.cnt, L.ksum, n_cap, alpha, beta, L.out);
+  static thread_local uint64_t host_out[3 * PTC_MAX_CAPACITIES + 2];
+  if (cudaMemcpyAsync(host_out, L.out, sizeof(uint64_t) * (3 * n_cap + 2), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+    return PTC_ERR_CUDA;
+  DevStatus h;
+  const ptc_status rc = end_call(L.st, s, &h);
+  if (rc != PTC_OK) return rc;
+  for (uint32_t g = 0; g < n_cap; ++g) {
+    hits_host_out[g] = host_out[g];
+    saved_host_out[g].lo = host_out[n_cap + 2 * g];
+    saved_host_out[g].hi = host_out[n_cap + 2 * g + 1];
+  }
+  total_cost_host_out->lo = host_out[3 * n_cap];
+  total_cost_host_out->hi = host_out[3 * n_cap + 1];
+  return PTC_OK;
+}

@@ -1,0 +1,514 @@
+// Stage a1: chained block keys (paper Sec. 2.2 block identity).
+//
+// Block k of a request covers tokens [Bk, Bk+B).  Its key is the polynomial
+// of the whole prefix sequence (1, tok_0, ..., tok_{B(k+1)-1}) over
+// GF(2^61 - 1) at two seeded bases.  Written per block:
+//     h_k = sum_{i<B} tok_{Bk+i} * rho^(B-1-i)                 (block-local)
+//     H_k = rho^(B(k+1)) * (1 + sum_{j<=k} h_j * rho^(-B(j+1)))
+// so the chain across a request is a plain segmented sum of the normalised
+// g_j = h_j * rho^(-B(j+1)) — one single-pass scan, no sequential chain.
+//
+// Kernels
+//   k_block_offsets  per-request block counts -> exclusive scan (look-back),
+//                    validates offsets and timestamp order, max blocks/request
+//   k_pow_tables     rho^(+-B e) for e < 2^32 as two 65,536-entry levels
+//   k_hash           tokens staged through padded shared memory with 16-byte
+//                    loads; each thread hashes 16 tokens (one "sub-chunk")
+//                    with 3 x 21-bit limbs of the powers held as constant
+//                    kernel parameters; sub-chunks of one block combine by
+//                    shuffles; the segmented sum runs across the CTA and
+//                    across CTAs by decoupled look-back.
+#include "ptc_internal.h"
+
+namespace ptc {
+namespace {
+
+constexpr int kOffThreads = 512;
+constexpr int kOffPer = 8;
+constexpr int kOffTile = kOffThreads * kOffPer;
+
+constexpr int kHashThreads = 512;
+constexpr int kWinTokens = 8192 + 256;
+constexpr int kWinWords = kWinTokens + kWinTokens / 16;
+
+constexpr int kEpochOffsets = 1;
+constexpr int kEpochHash = 2;
+
+// ---------------------------------------------------------------- block scans
+// Exclusive sum over a CTA of 512 threads; returns the CTA total in *total.
+__device__ __forceinline__ uint64_t cta_exclusive_sum(uint64_t v, uint64_t* total) {
+  __shared__ uint64_t s_w[kOffThreads / 32];
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  uint64_t x = v;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    uint64_t y = __shfl_up_sync(kFull, x, d);
+    if (lane >= (uint32_t)d) x += y;
+  }
+  if (lane == 31) s_w[w] = x;
+  __syncthreads();
+  if (w == 0) {
+    uint64_t t = lane < kOffThreads / 32 ? s_w[lane] : 0;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      uint64_t y = __shfl_up_sync(kFull, t, d);
+      if (lane >= (uint32_t)d) t += y;
+    }
+    if (lane < kOffThreads / 32) s_w[lane] = t;  // inclusive over warps
+  }
+  __syncthreads();
+  uint64_t warp_excl = w ? s_w[w - 1] : 0;
+  *total = s_w[kOffThreads / 32 - 1];
+  return warp_excl + x - v;
+}
+
+__global__ void __launch_bounds__(kOffThreads) k_block_offsets(const uint64_t* __restrict__ tok_off,
+                                                               const int64_t* __restrict__ ts, uint32_t R,
+                                                               uint64_t n_tok, uint32_t B,
+                                                               uint64_t* __restrict__ blk_off, uint64_t* lb,
+                                                               DevStatus* st) {
+  __shared__ uint64_t s_base;
+  const uint32_t tile = next_tile(st, kEpochOffsets);
+  const uint64_t r0 = (uint64_t)tile * kOffTile + (uint64_t)threadIdx.x * kOffPer;
+  uint64_t cnt[kOffPer];
+  uint64_t local = 0, kmax = 0;
+  uint32_t err = 0;
+#pragma unroll
+  for (int j = 0; j < kOffPer; ++j) {
+    uint64_t r = r0 + j;
+    cnt[j] = 0;
+    if (r < R) {
+      uint64_t a = tok_off[r], b = tok_off[r + 1];
+      if (b < a || b > n_tok) {
+        err |= kErrInvalid;
+      } else {
+        cnt[j] = (b - a) / B;
+      }
+      if (ts != nullptr && r + 1 < R && ts[r + 1] < ts[r]) err |= kErrUnsorted;
+      local += cnt[j];
+      kmax = cnt[j] > kmax ? cnt[j] : kmax;
+    }
+  }
+  if (err) raise_err(st, err);
+  if (kmax) atomicMax((unsigned long long*)&st->value[1], (unsigned long long)kmax);
+  uint64_t total;
+  uint64_t excl = cta_exclusive_sum(local, &total);
+  if (threadIdx.x < 32) {
+    uint64_t base = lookback_sum(lb, tile, total, kEpochOffsets, st);
+    if (threadIdx.x == 0) s_base = base;
+  }
+  __syncthreads();
+  uint64_t run = s_base + excl;
+#pragma unroll
+  for (int j = 0; j < kOffPer; ++j) {
+    uint64_t r = r0 + j;
+    if (r < R) blk_off[r] = run;
+    run += cnt[j];
+    if (r + 1 == R) {
+      blk_off[R] = run;
+      st->value[0] = run;
+      if (run >= (uint64_t)kNone) raise_err(st, kErrOverflow);
+    }
+  }
+}
+
+// ---------------------------------------------------------------- powers
+// tables[(b*4 + w) * 65536 + e] for base b in {0,1} and
+//   w = 0: rho_b^(B e)          w = 1: rho_b^(-B e)
+//   w = 2: rho_b^(B 65536 e)    w = 3: rho_b^(-B 65536 e)
+struct PowBases {
+  uint64_t base[8];
+};
+
+__global__ void k_pow_tables(PowBases pb, uint64_t* __restrict__ tables) {
+  const uint32_t gid = blockIdx.x * blockDim.x + threadIdx.x;  // 8 tables x 1024 chunks of 64
+  const uint32_t t = gid >> 10, chunk = gid & 1023;
+  if (t >= 8) return;
+  const uint64_t base = pb.base[t];
+  const uint64_t e0 = (uint64_t)chunk * 64;
+  uint64_t v = p61_pow(base, e0);
+  uint64_t* out = tables + (uint64_t)t * 65536 + e0;
+  for (int i = 0; i < 64; ++i) {
+    out[i] = v;
+    v = p61_mul(v, base);
+  }
+}
+
+__device__ __forceinline__ uint64_t pow_at(const uint64_t* __restrict__ lo, const uint64_t* __restrict__ hi,
+                                           uint64_t e) {
+  uint64_t v = __ldg(&lo[e & 0xFFFF]);
+  const uint64_t h = e >> 16;
+  if (h) v = p61_mul(v, __ldg(&hi[h & 0xFFFF]));
+  return v;
+}
+
+// ---------------------------------------------------------------- hash
+struct HashConsts {
+  uint32_t limb[2][3][16];   // 21-bit limbs of rho_b^(15 - j)
+  uint64_t sub_mul[2][32];   // rho_b^(16 q)
+};
+
+struct HashCarry {
+  uint64_t v0, v1, f;
+};
+
+struct SegSumOp {
+  __device__ HashCarry operator()(const HashCarry& a, const HashCarry& b) const {
+    HashCarry r;
+    r.f = a.f | b.f;
+    r.v0 = b.f ? b.v0 : p61_add(a.v0, b.v0);
+    r.v1 = b.f ? b.v1 : p61_add(a.v1, b.v1);
+    return r;
+  }
+};
+
+struct HashArgs {
+  const uint32_t* tokens;
+  uint64_t n_tok;
+  const uint64_t* tok_off;
+  const uint64_t* blk_off;
+  uint32_t R;
+  uint32_t B;
+  ulonglong2* keys;
+  uint64_t keys_cap;
+  const uint64_t* tables;
+  LbArrays<HashCarry> lb;
+  DevStatus* st;
+  int aligned;
+};
+
+__device__ __forceinline__ uint32_t pad16(uint32_t i) { return i + (i >> 4); }
+
+// (a0 + a1 2^21 + a2 2^42) mod p for a0, a1, a2 < 2^62 - 2^57 (sums of <= 32 products < 2^53)
+__device__ __forceinline__ uint64_t limbs_to_p61(uint64_t a0, uint64_t a1, uint64_t a2) {
+  uint64_t x = a0 + ((a1 & ((1ULL << 40) - 1)) << 21) + (a1 >> 40) + ((a2 & ((1ULL << 19) - 1)) << 42) + (a2 >> 19);
+  return p61_fold(x);
+}
+
+__device__ __forceinline__ uint32_t find_request(const uint64_t* __restrict__ blk_off, uint32_t lo, uint32_t hi,
+                                                 uint64_t b) {
+  // largest r in [lo, hi] with blk_off[r] <= b (blk_off[lo] <= b holds)
+  while (lo < hi) {
+    uint32_t mid = (lo + hi + 1) >> 1;
+    if (__ldg(&blk_off[mid]) <= b)
+      lo = mid;
+    else
+      hi = mid - 1;
+  }
+  return lo;
+}
+
+template <int G, bool FULL>
+__global__ void __launch_bounds__(kHashThreads) k_hash(HashArgs a, const __grid_constant__ HashConsts c) {
+  __shared__ uint32_t s_tok[kWinWords];
+  __shared__ uint64_t s_h0[kHashThreads / G], s_h1[kHashThreads / G];
+  __shared__ uint32_t s_k[kHashThreads / G];
+  __shared__ uint64_t s_bnd[4];
+  __shared__ HashCarry s_w[kHashThreads / 32];
+  __shared__ HashCarry s_carry;
+  constexpr uint32_t TB = kHashThreads / G;
+
+  const uint32_t tile = next_tile(a.st, kEpochHash);
+  uint64_t N = a.st->value[0];
+  if (N > a.keys_cap) N = a.keys_cap;
+  const uint64_t b0 = (uint64_t)tile * TB;
+  if (b0 >= N) return;
+  const uint64_t b_end = b0 + TB < N ? b0 + TB : N;
+  const uint32_t B = a.B;
+
+  if (threadIdx.x < 2) {
+    const uint64_t b = threadIdx.x == 0 ? b0 : b_end - 1;
+    s_bnd[threadIdx.x] = find_request(a.blk_off, 0, a.R - 1, b);
+  }
+  __syncthreads();
+  const uint32_t r_first = (uint32_t)s_bnd[0], r_last = (uint32_t)s_bnd[1];
+  const uint64_t t_begin = a.tok_off[r_first] + (uint64_t)B * (b0 - a.blk_off[r_first]);
+  const uint64_t t_end = a.tok_off[r_last] + (uint64_t)B * (b_end - a.blk_off[r_last]);
+  const uint64_t w0 = a.aligned ? (t_begin & ~3ULL) : t_begin;
+  uint64_t w_end = t_end < w0 + kWinTokens ? t_end : w0 + kWinTokens;
+  if (w_end > a.n_tok) w_end = a.n_tok;
+  __syncthreads();
+
+  // ---- stage the token window
+  if (a.aligned) {
+    const uint32_t nq = (uint32_t)((w_end - w0 + 3) >> 2);
+    for (uint32_t i = threadIdx.x; i < nq; i += kHashThreads) {
+      const uint64_t x = w0 + 4ULL * i;
+      uint4 v;
+      if (x + 3 < a.n_tok) {
+        v = __ldcs(reinterpret_cast<const uint4*>(a.tokens + x));
+      } else {
+        v.x = x < a.n_tok ? a.tokens[x] : 0u;
+        v.y = x + 1 < a.n_tok ? a.tokens[x + 1] : 0u;
+        v.z = x + 2 < a.n_tok ? a.tokens[x + 2] : 0u;
+        v.w = 0u;
+      }
+      const uint32_t o = pad16(4 * i);
+      s_tok[o] = v.x;
+      s_tok[o + 1] = v.y;
+      s_tok[o + 2] = v.z;
+      s_tok[o + 3] = v.w;
+    }
+  } else {
+    const uint32_t n = (uint32_t)(w_end - w0);
+    for (uint32_t i = threadIdx.x; i < n; i += kHashThreads) s_tok[pad16(i)] = a.tokens[w0 + i];
+  }
+  __syncthreads();
+
+  // ---- phase 1: 16-token sub-chunks
+  const uint32_t lb = threadIdx.x / G, s = threadIdx.x % G;
+  const uint64_t b = b0 + lb;
+  uint64_t h0 = 0, h1 = 0;
+  uint32_t k = 0;
+  if (b < b_end) {
+    const uint32_t r = find_request(a.blk_off, r_first, r_last, b);
+    k = (uint32_t)(b - a.blk_off[r]);
+    const int64_t first = (int64_t)B - 16 * G + 16 * (int64_t)s;  // block offset of this chunk's token 0
+    const uint64_t bstart = a.tok_off[r] + (uint64_t)B * k;
+    uint64_t a00 = 0, a01 = 0, a02 = 0, a10 = 0, a11 = 0, a12 = 0;
+    const uint64_t x0 = bstart + first;  // may wrap for the leading partial chunk; guarded below
+    const bool in_win = FULL && x0 >= w0 && x0 + 16 <= w_end;
+    if (in_win) {
+      const uint32_t rel = (uint32_t)(x0 - w0);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const uint64_t t = s_tok[pad16(rel + j)];
+        a00 += t * c.limb[0][0][j];
+        a01 += t * c.limb[0][1][j];
+        a02 += t * c.limb[0][2][j];
+        a10 += t * c.limb[1][0][j];
+        a11 += t * c.limb[1][1][j];
+        a12 += t * c.limb[1][2][j];
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        if (FULL || first + j >= 0) {
+          const uint64_t x = bstart + (uint64_t)(first + j);
+          uint64_t t;
+          if (x >= w0 && x < w_end)
+            t = s_tok[pad16((uint32_t)(x - w0))];
+          else
+            t = x < a.n_tok ? a.tokens[x] : 0u;
+          a00 += t * c.limb[0][0][j];
+          a01 += t * c.limb[0][1][j];
+          a02 += t * c.limb[0][2][j];
+          a10 += t * c.limb[1][0][j];
+          a11 += t * c.limb[1][1][j];
+          a12 += t * c.limb[1][2][j];
+        }
+      }
+    }
+    h0 = limbs_to_p61(a00, a01, a02);
+    h1 = limbs_to_p61(a10, a11, a12);
+    if (G > 1) {
+      const uint32_t q = G - 1 - s;
+      h0 = p61_mul(h0, c.sub_mul[0][q]);
+      h1 = p61_mul(h1, c.sub_mul[1][q]);
+    }
+  }
+  if (G > 1) {
+#pragma unroll
+    for (int o = G / 2; o > 0; o >>= 1) {
+      h0 = p61_add(h0, __shfl_xor_sync(kFull, h0, o));
+      h1 = p61_add(h1, __shfl_xor_sync(kFull, h1, o));
+    }
+  }
+  if (s == 0) {
+    s_h0[lb] = h0;
+    s_h1[lb] = h1;
+    s_k[lb] = k;
+  }
+  __syncthreads();
+
+  // ---- phase 2: normalise, segmented sum over requests, denormalise
+  const uint32_t t = threadIdx.x;
+  const bool valid = t < TB && b0 + t < b_end;
+  const uint64_t* T = a.tables;
+  HashCarry x{0, 0, 0};
+  uint32_t kk = 0;
+  if (valid) {
+    kk = s_k[t];
+    const uint64_t e = (uint64_t)kk + 1;
+    x.v0 = p61_mul(s_h0[t], pow_at(T + 1 * 65536, T + 3 * 65536, e));
+    x.v1 = p61_mul(s_h1[t], pow_at(T + 5 * 65536, T + 7 * 65536, e));
+    if (kk == 0) {
+      x.f = 1;
+      x.v0 = p61_add(x.v0, 1);
+      x.v1 = p61_add(x.v1, 1);
+    }
+  }
+  SegSumOp op;
+  const uint32_t lane = t & 31, w = t >> 5;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    HashCarry y;
+    y.v0 = __shfl_up_sync(kFull, x.v0, d);
+    y.v1 = __shfl_up_sync(kFull, x.v1, d);
+    y.f = __shfl_up_sync(kFull, x.f, d);
+    if (lane >= (uint32_t)d) x = op(y, x);
+  }
+  if (lane == 31) s_w[w] = x;
+  __syncthreads();
+  if (w == 0) {
+    HashCarry z = lane < kHashThreads / 32 ? s_w[lane] : HashCarry{0, 0, 0};
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      HashCarry y;
+      y.v0 = __shfl_up_sync(kFull, z.v0, d);
+      y.v1 = __shfl_up_sync(kFull, z.v1, d);
+      y.f = __shfl_up_sync(kFull, z.f, d);
+      if (lane >= (uint32_t)d) z = op(y, z);
+    }
+    if (lane < kHashThreads / 32) s_w[lane] = z;  // inclusive over warps
+  }
+  __syncthreads();
+  if (w > 0) x = op(s_w[w - 1], x);
+  if (t == 0) {
+    const HashCarry agg = s_w[kHashThreads / 32 - 1];
+    s_carry = lookback_generic(a.lb, tile, agg, HashCarry{0, 0, 0}, op, kEpochHash, a.st);
+  }
+  __syncthreads();
+  if (valid) {
+    if (!x.f) {
+      x.v0 = p61_add(x.v0, s_carry.v0);
+      x.v1 = p61_add(x.v1, s_carry.v1);
+    }
+    const uint64_t e = (uint64_t)kk + 1;
+    const uint64_t H0 = p61_mul(x.v0, pow_at(T + 0 * 65536, T + 2 * 65536, e));
+    const uint64_t H1 = p61_mul(x.v1, pow_at(T + 4 * 65536, T + 6 * 65536, e));
+    a.keys[b0 + t] = make_ulonglong2(H0, H1);
+  }
+}
+
+template <int G>
+void launch_hash(uint32_t grid, cudaStream_t s, const HashArgs& a, const HashConsts& c, bool full) {
+  if (full)
+    k_hash<G, true><<<grid, kHashThreads, 0, s>>>(a, c);
+  else
+    k_hash<G, false><<<grid, kHashThreads, 0, s>>>(a, c);
+}
+
+uint32_t chunks_per_block(uint32_t B) {  // G: power of two >= ceil(B / 16)
+  uint32_t need = (B + 15) / 16, g = 1;
+  while (g < need) g <<= 1;
+  return g;
+}
+
+struct HashLayout {
+  DevStatus* st;
+  uint64_t* lb_off;
+  uint32_t* lb_hash_status;
+  HashCarry* lb_hash_agg;
+  HashCarry* lb_hash_incl;
+  uint64_t* tables;
+  size_t zero_bytes;
+  size_t total;
+};
+
+HashLayout hash_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uint64_t keys_cap) {
+  HashLayout L;
+  Carver cv(ws);
+  const uint32_t off_tiles = ceil_div_u32(n_req, kOffTile) + 1;
+  const uint64_t nb = n_tok / B < keys_cap ? n_tok / B : keys_cap;
+  const uint32_t tb = kHashThreads / chunks_per_block(B);
+  const uint32_t hash_tiles = ceil_div_u32(nb, tb) + 1;
+  L.st = cv.take<DevStatus>(1);
+  L.lb_off = cv.take<uint64_t>(off_tiles);
+  L.lb_hash_status = cv.take<uint32_t>(hash_tiles);
+  L.zero_bytes = cv.off;
+  L.lb_hash_agg = cv.take<HashCarry>(hash_tiles);
+  L.lb_hash_incl = cv.take<HashCarry>(hash_tiles);
+  L.tables = cv.take<uint64_t>(8 * 65536);
+  L.total = cv.bytes();
+  return L;
+}
+
+}  // namespace
+}  // namespace ptc
+
+using namespace ptc;
+
+extern "C" size_t ptc_hash_blocks_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size) {
+  if (block_size == 0) block_size = 1;
+  return hash_layout(nullptr, n_req, n_tok, block_size, ~0ULL).total;
+}
+
+extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off,
+                                      const int64_t* req_ts_us, uint32_t n_req, uint32_t block_size, uint64_t seed,
+                                      ptc_u128* keys_out, uint64_t keys_cap, uint64_t* req_blk_off_out,
+                                      uint64_t* n_access_host_out, void* ws, size_t ws_bytes, void* stream) {
+  if (block_size < 1 || block_size > PTC_MAX_BLOCK_SIZE) return PTC_ERR_INVALID_ARG;
+  if (req_tok_off == nullptr || req_blk_off_out == nullptr || n_access_host_out == nullptr)
+    return PTC_ERR_INVALID_ARG;
+  if (n_tok > 0 && tokens == nullptr) return PTC_ERR_INVALID_ARG;
+  if (keys_cap > 0 && keys_out == nullptr) return PTC_ERR_INVALID_ARG;
+  cudaStream_t s = (cudaStream_t)stream;
+  const HashLayout need = hash_layout(nullptr, n_req, n_tok, block_size, ~0ULL);
+  if (!ws_ok(ws, ws_bytes, need.total)) return PTC_ERR_WORKSPACE;
+  const HashLayout L = hash_layout(ws, n_req, n_tok, block_size, ~0ULL);
+  *n_access_host_out = 0;
+  if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
+  if (n_req == 0) {
+    if (cudaMemsetAsync(req_blk_off_out, 0, sizeof(uint64_t), s) != cudaSuccess) return PTC_ERR_CUDA;
+    DevStatus h;
+    return end_call(L.st, s, &h);
+  }
+  k_block_offsets<<<ceil_div_u32(n_req, kOffTile), kOffThreads, 0, s>>>(req_tok_off, req_ts_us, n_req, n_tok,
+                                                                        block_size, req_blk_off_out, L.lb_off, L.st);
+
+  // seeded bases and their derived constants
+  PowBases pb;
+  HashConsts hc;
+  for (int b = 0; b < 2; ++b) {
+    const uint64_t rho = 2 + splitmix64_at(seed, (uint64_t)b) % (kP61 - 3);
+    const uint64_t rinv = p61_pow(rho, kP61 - 2);
+    const uint64_t rB = p61_pow(rho, block_size), riB = p61_pow(rinv, block_size);
+    pb.base[b * 4 + 0] = rB;
+    pb.base[b * 4 + 1] = riB;
+    pb.base[b * 4 + 2] = p61_pow(rB, 65536);
+    pb.base[b * 4 + 3] = p61_pow(riB, 65536);
+    for (int j = 0; j < 16; ++j) {
+      const uint64_t v = p61_pow(rho, 15 - j);
+      hc.limb[b][0][j] = (uint32_t)(v & 0x1FFFFF);
+      hc.limb[b][1][j] = (uint32_t)((v >> 21) & 0x1FFFFF);
+      hc.limb[b][2][j] = (uint32_t)(v >> 42);
+    }
+    for (int q = 0; q < 32; ++q) hc.sub_mul[b][q] = p61_pow(rho, 16ULL * q);
+  }
+  k_pow_tables<<<(8 * 1024) / 256, 256, 0, s>>>(pb, L.tables);
+
+  HashArgs a;
+  a.tokens = tokens;
+  a.n_tok = n_tok;
+  a.tok_off = req_tok_off;
+  a.blk_off = req_blk_off_out;
+  a.R = n_req;
+  a.B = block_size;
+  a.keys = reinterpret_cast<ulonglong2*>(keys_out);
+  a.keys_cap = keys_cap;
+  a.tables = L.tables;
+  a.lb = LbArrays<HashCarry>{L.lb_hash_status, L.lb_hash_agg, L.lb_hash_incl};
+  a.st = L.st;
+  a.aligned = (((uintptr_t)tokens) & 15) == 0;
+  const uint32_t G = chunks_per_block(block_size);
+  const bool full = block_size == 16 * G;
+  const uint64_t nb = n_tok / block_size < keys_cap ? n_tok / block_size : keys_cap;
+  const uint32_t grid = ceil_div_u32(nb, kHashThreads / G);
+  if (grid > 0) {
+    switch (G) {
+      case 1: launch_hash<1>(grid, s, a, hc, full); break;
+      case 2: launch_hash<2>(grid, s, a, hc, full); break;
+      case 4: launch_hash<4>(grid, s, a, hc, full); break;
+      case 8: launch_hash<8>(grid, s, a, hc, full); break;
+      case 16: launch_hash<16>(grid, s, a, hc, full); break;
+      default: launch_hash<32>(grid, s, a, hc, full); break;
+    }
+  }
+  DevStatus h;
+  ptc_status rc = end_call(L.st, s, &h);
+  *n_access_host_out = h.value[0];
+  if (rc != PTC_OK) return rc;
+  if (h.value[0] > keys_cap) return PTC_ERR_INVALID_ARG;
+  return PTC_OK;
+}

@@ -1,0 +1,36 @@
+// Host-side helpers shared by the C-ABI entry points.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include "../../include/ptc.h"
+#include "ptc_common.cuh"
+
+namespace ptc {
+
+// Zero the status block (and any extra prefix of the workspace) on `stream`.
+inline ptc_status begin_call(void* ws, size_t zero_bytes, cudaStream_t stream) {
+  if (cudaMemsetAsync(ws, 0, zero_bytes, stream) != cudaSuccess) return PTC_ERR_CUDA;
+  return PTC_OK;
+}
+
+// Wait for the call's work and translate the device status block.
+inline ptc_status end_call(const DevStatus* dev, cudaStream_t stream, DevStatus* host_copy) {
+  if (cudaGetLastError() != cudaSuccess) return PTC_ERR_CUDA;
+  if (cudaMemcpyAsync(host_copy, dev, sizeof(DevStatus), cudaMemcpyDeviceToHost, stream) != cudaSuccess)
+    return PTC_ERR_CUDA;
+  if (cudaStreamSynchronize(stream) != cudaSuccess) return PTC_ERR_CUDA;
+  uint32_t e = host_copy->err;
+  if (e & kErrTimeout) return PTC_ERR_TIMEOUT;
+  if (e & kErrUnsorted) return PTC_ERR_UNSORTED;
+  if (e & kErrOverflow) return PTC_ERR_OVERFLOW;
+  if (e & kErrCollision) return PTC_ERR_HASH_COLLISION;
+  if (e & (kErrInvalid | kErrTableFull)) return PTC_ERR_INVALID_ARG;
+  return PTC_OK;
+}
+
+inline bool ws_ok(const void* ws, size_t ws_bytes, size_t need) {
+  return ws != nullptr && ((uintptr_t)ws & 255) == 0 && ws_bytes >= need;
+}
+
+}  // namespace ptc

@@ -1,0 +1,76 @@
+"""The C-ABI library: it builds for sm_103a, loads, and exports every
+function that include/ptc.h declares.  No GPU work is launched here."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def libptc():
+    from paper_2609_28870_gb300 import build
+    path = build.build()
+    return ctypes.CDLL(path)
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "ptc.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(ptc_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_header_declares_the_five_calls():
+    names = declared_functions()
+    for n in ("ptc_hash_blocks", "ptc_assign_ids", "ptc_reuse_indices", "ptc_stack_distance", "ptc_curves"):
+        assert n in names and n + "_workspace_bytes" in names
+
+
+def test_every_declared_symbol_is_exported(libptc):
+    for name in declared_functions():
+        assert hasattr(libptc, name), name
+
+
+def test_strerror_and_version(libptc):
+    libptc.ptc_strerror.restype = ctypes.c_char_p
+    libptc.ptc_version.restype = ctypes.c_char_p
+    assert libptc.ptc_strerror(0) == b"ok"
+    assert b"timestamps" in libptc.ptc_strerror(2)
+    assert b"sm_103a" in libptc.ptc_version()
+
+
+def test_workspace_sizes_are_host_only_and_grow(libptc):
+    f = libptc.ptc_stack_distance_workspace_bytes
+    f.restype = ctypes.c_size_t
+    f.argtypes = [ctypes.c_uint64]
+    assert 0 < f(1000) < f(10**6) < f(10**8)
+    g = libptc.ptc_hash_blocks_workspace_bytes
+    g.restype = ctypes.c_size_t
+    g.argtypes = [ctypes.c_uint32, ctypes.c_uint64, ctypes.c_uint32]
+    assert g(10, 10**6, 16) % 256 == 0
+
+
+def test_host_argument_checks_need_no_gpu(libptc):
+    """Bad arguments are rejected before any CUDA call."""
+    import paper_2609_28870_gb300 as ptc
+    L = ptc.lib()
+    n = ctypes.c_uint64(0)
+    # block size 0 and above the maximum
+    for B in (0, ptc.MAX_BLOCK_SIZE + 1):
+        rc = L.ptc_hash_blocks(None, 0, 8, None, 1, B, 0, None, 0, 8, ctypes.byref(n), None, 0, None)
+        assert rc == 1
+    # workspace missing
+    rc = L.ptc_stack_distance(8, 10, 8, None, 0, None)
+    assert rc == 4
+    # too many accesses for 32-bit indices
+    assert L.ptc_stack_distance(8, 2**32 - 1, 8, None, 0, None) == 3
+
+
+def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
+    import paper_2609_28870_gb300 as ptc
+    monkeypatch.setattr(ptc, "_lib", None)
+    monkeypatch.setattr(ptc._build, "LIB", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="not built"):
+        ptc.lib()
