@@ -1,0 +1,418 @@
+#!/usr/bin/env python3
+"""Benchmark: request trace -> all-capacity LRU hit and compute-saved curves.
+
+One step is the whole path — ptc_hash_blocks, ptc_assign_ids,
+ptc_reuse_indices, ptc_stack_distance, ptc_curves — over one synthetic trace
+resident in HBM: the conversational chat workload (~154M tokens, ~9.6M block
+accesses, 16-token blocks, 64 log-spaced capacities from 64 blocks to all
+distinct blocks, measured-shape cost model).  The metric is trace tokens per
+second; the JSON line also carries block accesses per second and the fraction
+of the HBM roofline for the path's stage-byte model.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Timing: W untimed warm-up steps, then K steps, each bracketed by CUDA events
+on the launching stream, with a 256 MiB write between steps to flush L2
+(outside the events); barrier + synchronize on both sides; max over ranks.
+With N > 1 (torchrun) every rank runs an independent replica (the path has
+no cross-GPU exchange): value = tokens of all replicas / slowest rank's time.
+
+--impl reference times the CPU oracle (the plain restatement used as the
+parity reference) on the host cores, on a bounded sample of the same
+workload; rank 0 alone runs it.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "trace tokens/s to all-capacity LRU hit+compute-saved curves; % of HBM roofline"
+WORKLOAD = 1
+BLOCK = 16
+NOMINAL_HBM_GBS = 7900.0
+
+# Per-launch DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) from
+# the last ncu capture of each kernel, with the sha256 of the source file it
+# was taken on; a changed source reads as "no counters" (null).
+NCU_TRAFFIC: dict[str, tuple[float, str, str]] = {}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample", type=float, default=1.0,
+                    help="fraction of the workload's requests (a prefix in time) the CPU oracle runs on")
+    ap.add_argument("--ref-sample", type=float, default=1.0,
+                    help="fraction of requests per --impl reference step")
+    ap.add_argument("--json-out", default=None)
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------- helpers
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def value_bits(n):  # values of the wavelet matrix lie in [0, n]
+    L = 1
+    while L < 33 and (1 << L) <= n:
+        L += 1
+    return L
+
+
+def stage_model_bytes(T, N):
+    """Algorithmic bytes of each stage (the stage-byte model)."""
+    L = value_bits(N)
+    return {
+        "hash": 4 * T + 16 * N,
+        "ids": 20 * N,
+        "reuse": 12 * N,
+        "wavelet_build": 8.125 * L * N,
+        "queries": (8 + L / 8) * N,
+        "curves": 4 * N,
+    }, L
+
+
+def kernel_model_bytes(name, T, N, L):
+    """Algorithmic bytes one launch of `name` must move (0: not in the model)."""
+    per_level = ((L - 1) * 8.125 + 4.125) / L * N  # the last level writes no partition
+    return {
+        "k_hash": 4 * T + 16 * N,
+        "k_ids_insert": 16 * N,
+        "k_ids_gather": 4 * N,
+        "k_adjacent": 8 * N,
+        "k_sort_hist": 4 * N,
+        "k_wm_level": per_level,
+        "k_wm_query": (8 + L / 8) * N,
+        "k_curves": 4 * N,
+    }.get(name, 0.0)
+
+
+def source_sha(kernel):
+    files = {"k_hash": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu", "k_ids_rank": "ptc_ids.cu",
+             "k_ids_gather": "ptc_ids.cu", "k_sort_pass": "ptc_sort.cu", "k_adjacent": "ptc_sort.cu",
+             "k_sort_hist": "ptc_sort.cu", "k_wm_level": "ptc_wavelet.cu", "k_wm_query": "ptc_wavelet.cu",
+             "k_wm_zeros": "ptc_wavelet.cu", "k_curves": "ptc_curves.cu"}
+    f = files.get(kernel)
+    if f is None:
+        return None
+    with open(os.path.join(ROOT, "paper_2609_28870_gb300", "csrc", f), "rb") as fh:
+        return hashlib.sha256(fh.read()).hexdigest()[:16]
+
+
+class Clocks:
+    """nvidia-smi sampled every 200 ms while the timed region runs."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "", 1).isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "", 1).isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[k] for r in rows for k in range(4) if r[5 + k].lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------- our arm
+def run_ours(args, ws_world, rank, local):
+    import numpy as np
+    import torch
+
+    import paper_2609_28870_gb300 as ptc
+    import tracegen
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if ws_world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if ws_world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    def max_over_ranks(x):
+        if ws_world == 1:
+            return x
+        import torch.distributed as dist
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    L = ptc.lib()
+    # the trace, generated into pinned host memory (the end-to-end leg copies from it)
+    R, T, _ = tracegen.sizes(WORKLOAD)
+    tok_host = torch.empty(T, dtype=torch.int32, pin_memory=True)
+    tr = tracegen.make(WORKLOAD, token_buffer=tok_host.numpy().view(np.uint32))
+    off_host = torch.from_numpy(tr.req_tok_off.view(np.int64)).pin_memory()
+    ts_host = torch.from_numpy(tr.req_ts_us).pin_memory()
+    tok = tok_host.to(dev, non_blocking=True)
+    off = off_host.to(dev, non_blocking=True)
+    ts = ts_host.to(dev, non_blocking=True)
+    torch.cuda.synchronize(dev)
+    ws = torch.empty(ptc.workspace_bytes(tr.n_req, T, BLOCK, n_cap=64), dtype=torch.uint8, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    caps_for = lambda d: tracegen.workload_grid(WORKLOAD, d)
+
+    def step():
+        return ptc.pipeline(tok, off, ts, BLOCK, caps_for, kind=ptc.PTC_COST_MEASURED, seed=0, ws=ws, keep=False)
+
+    for _ in range(max(args.warmup, 0)):
+        out = step()
+    N, D = out["n_access"], out["n_distinct"]
+    stream = torch.cuda.current_stream(dev)
+
+    # ---- timed region (inputs resident in HBM)
+    L.ptc_timer_reset()
+    L.ptc_timer_enable(1)
+    clocks = Clocks(local)
+    barrier()
+    torch.cuda.synchronize(dev)
+    clocks.start()
+    launches0 = L.ptc_launch_count()
+    step_ms = []
+    for k in range(args.steps):
+        flush.fill_(k & 0xFF)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        out = step()
+        e1.record(stream)
+        e1.synchronize()
+        step_ms.append(e0.elapsed_time(e1))
+    torch.cuda.synchronize(dev)
+    launches = L.ptc_launch_count() - launches0
+    barrier()
+    clk = clocks.stop()
+    L.ptc_timer_enable(0)
+    ktimes = read_timer(ptc)
+    total_ms = max_over_ranks(sum(step_ms))
+    ms_per_step = total_ms / args.steps
+
+    # ---- end to end through the public API from pinned host memory
+    e2e_ms = []
+    for k in range(args.steps):
+        flush.fill_(k & 0xFF)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        tok2 = tok_host.to(dev, non_blocking=True)
+        off2 = off_host.to(dev, non_blocking=True)
+        ts2 = ts_host.to(dev, non_blocking=True)
+        o2 = ptc.pipeline(tok2, off2, ts2, BLOCK, caps_for, kind=ptc.PTC_COST_MEASURED, seed=0, ws=ws, keep=False)
+        e1.record(stream)
+        e1.synchronize()
+        e2e_ms.append(e0.elapsed_time(e1))
+        del tok2, off2, ts2
+    e2e_total = max_over_ranks(sum(e2e_ms))
+    assert o2["hits"] == out["hits"] and o2["saved"] == out["saved"]
+    h2d = 4 * T + 8 * (tr.n_req + 1) + 8 * tr.n_req
+    G = len(out["hits"])
+    d2h = 8 * G + 16 * G + 16 + 8 + 8  # hits, saved (u128), total cost, N, D
+
+    # ---- roofline
+    peak, peak_kind = measured_peaks()
+    stages, Lbits = stage_model_bytes(T, N)
+    model_total = sum(stages.values())
+    kernels = []
+    for name, launches_k, tot_ms in ktimes:
+        per = tot_ms / max(launches_k, 1)
+        mb = kernel_model_bytes(name, T, N, Lbits)
+        kernels.append({"name": name, "launches_per_step": launches_k / args.steps, "ms_per_step": tot_ms / args.steps,
+                        "avg_launch_ms": per, "model_bytes_per_launch": mb,
+                        "achieved_gbs": (mb / (per * 1e-3) / 1e9) if per > 0 else 0.0})
+    kernels.sort(key=lambda x: -x["ms_per_step"])
+    dom = kernels[0] if kernels else None
+    roof = None
+    if dom:
+        tr_entry = NCU_TRAFFIC.get(dom["name"])
+        traffic = tr_entry[0] if tr_entry and tr_entry[1] == source_sha(dom["name"]) else None
+        roof = {"kernel": dom["name"], "bound": "hbm", "achieved": round(dom["achieved_gbs"], 1), "peak": peak,
+                "unit": "GB/s", "frac": round(dom["achieved_gbs"] / peak, 4), "traffic": traffic,
+                "peak_source": f"{peak_kind} hbm_gbs"}
+
+    value = ws_world * T * args.steps / (total_ms * 1e-3)
+    acc_s = ws_world * N * args.steps / (total_ms * 1e-3)
+    e2e_value = ws_world * T * args.steps / (e2e_total * 1e-3)
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": ws_world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "u32/u64 integer", "data": "synthetic",
+        "config": {"workload": "conversational chat trace (workload 1, seed 1): 5,600 sessions, 60% single-turn, "
+                               "LN(300)/LN(600) turns, 50 Zipf system prompts, B=16, 64-point capacity grid, "
+                               "measured-shape cost",
+                   "tokens": T, "requests": tr.n_req, "accesses": N, "distinct_blocks": D, "block_size": BLOCK,
+                   "capacities": G, "l2": "flushed between timed steps (256 MiB write, outside the events)",
+                   "parallelism": "replicas" if ws_world > 1 else "single GPU"},
+        "accesses_per_s": round(acc_s, 1),
+        "hbm_roofline": {"stage_model_bytes": model_total, "L": Lbits,
+                         "frac_of_measured": round(model_total / (ms_per_step * 1e-3) / 1e9 / peak, 4),
+                         "frac_of_nominal_7900": round(model_total / (ms_per_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS, 4),
+                         "stages_bytes": stages},
+        "roofline": roof,
+        "kernels": [{k: (round(v, 5) if isinstance(v, float) else v) for k, v in x.items()} for x in kernels],
+        "e2e": {"value": round(e2e_value, 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_total / args.steps, 4)},
+        "gpu_launches": launches,
+        "clocks": clk,
+    }
+    if rank == 0 and ws_world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(tr, args.cpu_sample)
+    if rank == 0:
+        s = json.dumps(line)
+        print(s, flush=True)
+        if args.json_out:
+            with open(args.json_out, "w") as f:
+                f.write(s + "\n")
+    if ws_world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def read_timer(ptc):
+    import ctypes
+
+    class KT(ctypes.Structure):
+        _fields_ = [("name", ctypes.c_char * 48), ("launches", ctypes.c_uint64), ("total_ms", ctypes.c_double)]
+
+    L = ptc.lib()
+    L.ptc_timer_read.restype = ctypes.c_uint32
+    L.ptc_timer_read.argtypes = [ctypes.c_void_p, ctypes.c_uint32]
+    n = L.ptc_timer_read(None, 0)
+    buf = (KT * max(n, 1))()
+    n = L.ptc_timer_read(ctypes.cast(buf, ctypes.c_void_p), n)
+    return [(buf[i].name.decode(), int(buf[i].launches), float(buf[i].total_ms)) for i in range(n)]
+
+
+# ---------------------------------------------------------------- CPU oracle
+def oracle_on_sample(tr, fraction, threads):
+    import oracle
+    import tracegen
+    n_req = max(1, int(tr.n_req * fraction))
+    sub = tr.head(n_req)
+    t0 = time.perf_counter()
+    ids, D = oracle.block_ids(sub.tokens, sub.req_tok_off, BLOCK)
+    off = oracle.block_offsets(sub.req_tok_off, BLOCK)
+    prev, nxt = oracle.reuse(ids, D)
+    oracle.sd_fenwick(prev)
+    caps = tracegen.workload_grid(WORKLOAD, D)
+    oracle.lru_curves(ids, off, BLOCK, caps, oracle.COST_MEASURED, threads=threads)
+    dt = time.perf_counter() - t0
+    return sub, dt
+
+
+def cpu_baseline(tr, fraction):
+    threads = os.cpu_count() or 1
+    sub, dt = oracle_on_sample(tr, fraction, threads)
+    return {"value": round(sub.n_tok / dt, 1), "unit": "tokens/s", "cores": threads, "kind": "oracle",
+            "sample": f"first {sub.n_req} of {tr.n_req} requests ({sub.n_tok} tokens) of the same workload; "
+                      f"exact trie ids, prev/next, Fenwick stack distances, direct LRU simulation at all 64 "
+                      f"capacities on {threads} threads; {dt:.2f} s"}
+
+
+def run_reference(args, ws_world, rank):
+    if rank != 0:
+        return
+    import tracegen
+    tr = tracegen.make(WORKLOAD)
+    threads = os.cpu_count() or 1
+    for _ in range(max(args.warmup, 0)):
+        oracle_on_sample(tr, args.ref_sample, threads)
+    times = []
+    sub = None
+    for _ in range(args.steps):
+        sub, dt = oracle_on_sample(tr, args.ref_sample, threads)
+        times.append(dt)
+    total = sum(times)
+    value = sub.n_tok * args.steps / total
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": ws_world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(1e3 * total / args.steps, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u32/u64/u128 integer", "data": "synthetic",
+        "impl": "reference",
+        "config": {"workload": "conversational chat trace (workload 1, seed 1), B=16, 64-point capacity grid",
+                   "sample_requests": sub.n_req, "sample_tokens": sub.n_tok},
+        "cpu_baseline": {"value": round(value, 1), "unit": "tokens/s", "cores": threads, "kind": "oracle",
+                         "sample": f"first {sub.n_req} of {tr.n_req} requests per step"},
+        "e2e": {"value": round(value, 1), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    s = json.dumps(line)
+    print(s, flush=True)
+    if args.json_out:
+        with open(args.json_out, "w") as f:
+            f.write(s + "\n")
+
+
+def main():
+    args = parse_args()
+    ws_world, rank, local = dist_env()
+    if args.impl == "reference":
+        run_reference(args, ws_world, rank)
+    else:
+        run_ours(args, ws_world, rank, local)
+
+
+if __name__ == "__main__":
+    main()

@@ -203,6 +203,26 @@ ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_
                       uint64_t* hits_host_out, ptc_u128* saved_host_out, ptc_u128* total_cost_host_out, void* ws,
                       size_t ws_bytes, void* stream);
 
+/*
+ * Measurement hooks (no counterpart in the paper: instrumentation for the
+ * roofline figures).  ptc_launch_count() counts every kernel this library has
+ * launched in the process.  While ptc_timer_enable(1) is in force, every
+ * launch is bracketed by two CUDA events on its stream; each call resolves
+ * them when it synchronizes and adds the duration to a per-kernel total.
+ * ptc_timer_read() copies up to `cap` totals into `out` (host memory) and
+ * returns how many kernels have totals.  Not thread-safe across concurrent
+ * calls on different streams while enabled.
+ */
+typedef struct {
+  char name[48];
+  uint64_t launches;
+  double total_ms;
+} ptc_kernel_time;
+void ptc_timer_enable(int on);
+void ptc_timer_reset(void);
+uint32_t ptc_timer_read(ptc_kernel_time* out, uint32_t cap);
+uint64_t ptc_launch_count(void);
+
 #ifdef __cplusplus
 }
 #endif

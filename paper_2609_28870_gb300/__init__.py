@@ -105,6 +105,14 @@ def lib():
                 L.ptc_curves.restype = st
                 L.ptc_curves.argtypes = [vp, u64, vp, u32, u32, ctypes.POINTER(CostModel), vp, u32, vp, vp,
                                          ctypes.POINTER(U128), vp, sz, vp]
+                L.ptc_timer_enable.restype = None
+                L.ptc_timer_enable.argtypes = [ctypes.c_int]
+                L.ptc_timer_reset.restype = None
+                L.ptc_timer_reset.argtypes = []
+                L.ptc_timer_read.restype = u32
+                L.ptc_timer_read.argtypes = [vp, u32]
+                L.ptc_launch_count.restype = u64
+                L.ptc_launch_count.argtypes = []
                 del i64
                 _lib = L
     return _lib

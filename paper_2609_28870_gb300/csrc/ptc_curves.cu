@@ -311,7 +311,7 @@ extern "C" ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_
   if (cudaMemcpyAsync(L.caps, cap_host, sizeof(uint64_t) * n_cap, cudaMemcpyHostToDevice, s) != cudaSuccess)
     return PTC_ERR_CUDA;
   if (n > 0) {
-    k_heads<<<ceil_div_u32(n_req, 256), 256, 0, s>>>(req_blk_off, n_req, n, L.bitmap, L.st);
+    PTC_LAUNCH("k_heads", s, k_heads<<<ceil_div_u32(n_req, 256), 256, 0, s>>>(req_blk_off, n_req, n, L.bitmap, L.st));
     CurveArgs a;
     a.dist = dist;
     a.n = n;
@@ -322,9 +322,9 @@ extern "C" ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_
     a.ksum = L.ksum;
     a.lb = LbArrays<RunMax>{L.lb_status, L.lb_agg, L.lb_incl};
     a.st = L.st;
-    k_curves<<<ceil_div_u32(n, kCvTile), kCvThreads, 0, s>>>(a);
+    PTC_LAUNCH("k_curves", s, k_curves<<<ceil_div_u32(n, kCvTile), kCvThreads, 0, s>>>(a));
   }
-  k_finalize<<<1, 32, 0, s>>>(L.cnt, L.ksum, n_cap, alpha, beta, L.out);
+  PTC_LAUNCH("k_finalize", s, k_finalize<<<1, 32, 0, s>>>(L.cnt, L.ksum, n_cap, alpha, beta, L.out));
   static thread_local uint64_t host_out[3 * PTC_MAX_CAPACITIES + 2];
   if (cudaMemcpyAsync(host_out, L.out, sizeof(uint64_t) * (3 * n_cap + 2), cudaMemcpyDeviceToHost, s) != cudaSuccess)
     return PTC_ERR_CUDA;

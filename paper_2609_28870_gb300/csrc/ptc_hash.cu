@@ -384,9 +384,9 @@ __global__ void __launch_bounds__(kHashThreads) k_hash(HashArgs a, const __grid_
 template <int G>
 void launch_hash(uint32_t grid, cudaStream_t s, const HashArgs& a, const HashConsts& c, bool full) {
   if (full)
-    k_hash<G, true><<<grid, kHashThreads, 0, s>>>(a, c);
+    PTC_LAUNCH("k_hash", s, k_hash<G, true><<<grid, kHashThreads, 0, s>>>(a, c));
   else
-    k_hash<G, false><<<grid, kHashThreads, 0, s>>>(a, c);
+    PTC_LAUNCH("k_hash", s, k_hash<G, false><<<grid, kHashThreads, 0, s>>>(a, c));
 }
 
 uint32_t chunks_per_block(uint32_t B) {  // G: power of two >= ceil(B / 16)
@@ -454,8 +454,8 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
     DevStatus h;
     return end_call(L.st, s, &h);
   }
-  k_block_offsets<<<ceil_div_u32(n_req, kOffTile), kOffThreads, 0, s>>>(req_tok_off, req_ts_us, n_req, n_tok,
-                                                                        block_size, req_blk_off_out, L.lb_off, L.st);
+  PTC_LAUNCH("k_block_offsets", s, k_block_offsets<<<ceil_div_u32(n_req, kOffTile), kOffThreads, 0, s>>>(req_tok_off, req_ts_us, n_req, n_tok,
+                                                                        block_size, req_blk_off_out, L.lb_off, L.st));
 
   // seeded bases and their derived constants
   PowBases pb;
@@ -476,7 +476,7 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
     }
     for (int q = 0; q < 32; ++q) hc.sub_mul[b][q] = p61_pow(rho, 16ULL * q);
   }
-  k_pow_tables<<<(8 * 1024) / 256, 256, 0, s>>>(pb, L.tables);
+  PTC_LAUNCH("k_pow_tables", s, k_pow_tables<<<(8 * 1024) / 256, 256, 0, s>>>(pb, L.tables));
 
   HashArgs a;
   a.tokens = tokens;

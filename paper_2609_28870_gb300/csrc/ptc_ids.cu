@@ -262,9 +262,9 @@ extern "C" ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t*
   if (n > 0) {
     if (cudaMemsetAsync(L.table, 0xFF, sizeof(ulonglong2) << L.log2m, s) != cudaSuccess) return PTC_ERR_CUDA;
     const ulonglong2* k = reinterpret_cast<const ulonglong2*>(keys);
-    k_ids_insert<<<ceil_div_u32(n, kInsThreads), kInsThreads, 0, s>>>(k, n, L.table, L.log2m, L.slot_of, L.st);
-    k_ids_rank<<<ceil_div_u32(n, kRankTile), kRankThreads, 0, s>>>(L.table, L.slot_of, n, L.slot_id, L.lb, L.st);
-    k_ids_gather<<<ceil_div_u32(n, 256), 256, 0, s>>>(L.slot_of, L.slot_id, n, ids_out);
+    PTC_LAUNCH("k_ids_insert", s, k_ids_insert<<<ceil_div_u32(n, kInsThreads), kInsThreads, 0, s>>>(k, n, L.table, L.log2m, L.slot_of, L.st));
+    PTC_LAUNCH("k_ids_rank", s, k_ids_rank<<<ceil_div_u32(n, kRankTile), kRankThreads, 0, s>>>(L.table, L.slot_of, n, L.slot_id, L.lb, L.st));
+    PTC_LAUNCH("k_ids_gather", s, k_ids_gather<<<ceil_div_u32(n, 256), 256, 0, s>>>(L.slot_of, L.slot_id, n, ids_out));
   }
   DevStatus h;
   const ptc_status rc = end_call(L.st, s, &h);
@@ -296,9 +296,9 @@ extern "C" ptc_status ptc_verify_ids(const uint32_t* tokens, uint64_t n_tok, con
   if (begin_call(ws, kStatusBytes, s) != PTC_OK) return PTC_ERR_CUDA;
   if (cudaMemsetAsync(first, 0xFF, sizeof(uint32_t) * (n_distinct ? n_distinct : 1), s) != cudaSuccess)
     return PTC_ERR_CUDA;
-  k_verify_first<<<ceil_div_u32(n, 256), 256, 0, s>>>(ids, n, n_distinct, first, st);
-  k_verify<<<ceil_div_u32(n, 256), 256, 0, s>>>(tokens, n_tok, req_tok_off, req_blk_off, n_req, block_size, ids, n,
-                                               n_distinct, first, st);
+  PTC_LAUNCH("k_verify_first", s, k_verify_first<<<ceil_div_u32(n, 256), 256, 0, s>>>(ids, n, n_distinct, first, st));
+  PTC_LAUNCH("k_verify", s, k_verify<<<ceil_div_u32(n, 256), 256, 0, s>>>(tokens, n_tok, req_tok_off, req_blk_off, n_req, block_size, ids, n,
+                                               n_distinct, first, st));
   DevStatus h;
   return end_call(st, s, &h);
 }

@@ -8,6 +8,21 @@
 
 namespace ptc {
 
+// Launch accounting and optional per-kernel CUDA-event timing (ptc_timer_*).
+// Every kernel launch goes through PTC_LAUNCH, which counts it and, while
+// timing is enabled, brackets it with two events on the launch stream.  The
+// events are resolved when the call synchronizes (end_call).
+void timer_launch_begin(const char* name, cudaStream_t s);
+void timer_launch_end(cudaStream_t s);
+void timer_resolve();
+
+#define PTC_LAUNCH(name, stream, ...)           \
+  do {                                          \
+    ::ptc::timer_launch_begin(name, stream);    \
+    __VA_ARGS__;                                \
+    ::ptc::timer_launch_end(stream);            \
+  } while (0)
+
 // Zero the status block (and any extra prefix of the workspace) on `stream`.
 inline ptc_status begin_call(void* ws, size_t zero_bytes, cudaStream_t stream) {
   if (cudaMemsetAsync(ws, 0, zero_bytes, stream) != cudaSuccess) return PTC_ERR_CUDA;
@@ -20,6 +35,7 @@ inline ptc_status end_call(const DevStatus* dev, cudaStream_t stream, DevStatus*
   if (cudaMemcpyAsync(host_copy, dev, sizeof(DevStatus), cudaMemcpyDeviceToHost, stream) != cudaSuccess)
     return PTC_ERR_CUDA;
   if (cudaStreamSynchronize(stream) != cudaSuccess) return PTC_ERR_CUDA;
+  timer_resolve();
   uint32_t e = host_copy->err;
   if (e & kErrTimeout) return PTC_ERR_TIMEOUT;
   if (e & kErrUnsorted) return PTC_ERR_UNSORTED;

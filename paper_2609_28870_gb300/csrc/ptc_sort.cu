@@ -260,8 +260,8 @@ extern "C" ptc_status ptc_reuse_indices(const uint32_t* ids, uint64_t n, uint64_
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
   const uint32_t bits = key_bits(n_distinct);
   const uint32_t passes = (bits + 7) / 8;
-  k_sort_hist<<<1216, 256, 0, s>>>(ids, n, n_distinct, passes, bits, L.hist, L.st);
-  k_sort_offsets<<<1, kRadix, 0, s>>>(L.hist, passes, L.offs);
+  PTC_LAUNCH("k_sort_hist", s, k_sort_hist<<<1216, 256, 0, s>>>(ids, n, n_distinct, passes, bits, L.hist, L.st));
+  PTC_LAUNCH("k_sort_offsets", s, k_sort_offsets<<<1, kRadix, 0, s>>>(L.hist, passes, L.offs));
   const uint32_t tiles = ceil_div_u32(n, kSortTile);
   const uint32_t* kin = ids;
   const uint32_t* vin = nullptr;
@@ -279,13 +279,13 @@ extern "C" ptc_status ptc_reuse_indices(const uint32_t* ids, uint64_t n, uint64_
     a.lb = L.lb;
     a.st = L.st;
     a.epoch = 1 + (int)p;
-    k_sort_pass<<<tiles, kSortThreads, 0, s>>>(a);
+    PTC_LAUNCH("k_sort_pass", s, k_sort_pass<<<tiles, kSortThreads, 0, s>>>(a));
     kin = kout;
     vin = vout;
     kout = (kout == L.k0) ? L.k1 : L.k0;
     vout = (vout == L.v0) ? L.v1 : L.v0;
   }
-  k_adjacent<<<ceil_div_u32(n, 256), 256, 0, s>>>(kin, vin, n, prev_out, next_out);
+  PTC_LAUNCH("k_adjacent", s, k_adjacent<<<ceil_div_u32(n, 256), 256, 0, s>>>(kin, vin, n, prev_out, next_out));
   DevStatus h;
   return end_call(L.st, s, &h);
 }

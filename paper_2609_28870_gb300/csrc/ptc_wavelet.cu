@@ -249,7 +249,7 @@ extern "C" ptc_status ptc_stack_distance(const uint32_t* prev, uint64_t n, uint3
   cudaStream_t s = (cudaStream_t)stream;
   const WmLayout W = wm_layout(ws, n);
   if (begin_call(ws, W.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
-  k_wm_zeros<<<1216, 256, 0, s>>>(prev, n, W.L, W.ones, W.st);
+  PTC_LAUNCH("k_wm_zeros", s, k_wm_zeros<<<1216, 256, 0, s>>>(prev, n, W.L, W.ones, W.st));
   const uint32_t tiles = ceil_div_u32(n + 1, kLvTile);
   const uint32_t* vin = nullptr;
   uint32_t* vout = W.va;
@@ -265,12 +265,12 @@ extern "C" ptc_status ptc_stack_distance(const uint32_t* prev, uint64_t n, uint3
     a.level = l;
     a.lb = W.lb;
     a.st = W.st;
-    k_wm_level<<<tiles, kLvThreads, 0, s>>>(a);
+    PTC_LAUNCH("k_wm_level", s, k_wm_level<<<tiles, kLvThreads, 0, s>>>(a));
     vin = vout;
     vout = (vout == W.va) ? W.vb : W.va;
   }
-  k_wm_query<<<ceil_div_u32(n, kQThreads), kQThreads, 0, s>>>(prev, n, W.L, W.mat, W.level_words, W.ones, dist_out,
-                                                               W.st);
+  PTC_LAUNCH("k_wm_query", s, k_wm_query<<<ceil_div_u32(n, kQThreads), kQThreads, 0, s>>>(prev, n, W.L, W.mat, W.level_words, W.ones, dist_out,
+                                                               W.st));
   DevStatus h;
   return end_call(W.st, s, &h);
 }
