@@ -208,6 +208,274 @@ __device__ inline T lookback_generic(LbArrays<T> a, uint32_t tile, const T& agg,
   return acc;
 }
 
+// Warp-parallel variant of lookback_generic: called by all 32 lanes of ONE
+// warp; each round inspects 32 predecessors at once and folds them in order
+// (a higher lane holds an earlier tile, so it is the left operand).  Returns
+// the exclusive prefix in every lane.
+template <class T>
+__device__ __forceinline__ T shfl_down_payload(const T& v, int o) {
+  T r;
+  const uint64_t* s = reinterpret_cast<const uint64_t*>(&v);
+  uint64_t* d = reinterpret_cast<uint64_t*>(&r);
+#pragma unroll
+  for (int i = 0; i < (int)(sizeof(T) / 8); ++i) d[i] = __shfl_down_sync(kFull, s[i], o);
+  return r;
+}
+template <class T>
+__device__ __forceinline__ T shfl_payload(const T& v, int src) {
+  T r;
+  const uint64_t* s = reinterpret_cast<const uint64_t*>(&v);
+  uint64_t* d = reinterpret_cast<uint64_t*>(&r);
+#pragma unroll
+  for (int i = 0; i < (int)(sizeof(T) / 8); ++i) d[i] = __shfl_sync(kFull, s[i], src);
+  return r;
+}
+
+template <class T, class Op>
+__device__ inline T lookback_warp(LbArrays<T> a, uint32_t tile, const T& agg, const T& identity, Op op,
+                                  uint32_t epoch, DevStatus* st) {
+  static_assert(sizeof(T) % 8 == 0, "payload must be a multiple of 8 bytes");
+  const uint32_t lane = threadIdx.x & 31;
+  if (tile == 0) {
+    if (lane == 0) {
+      lb_store(&a.incl[0], agg);
+      __threadfence();
+      st_relaxed_u32(&a.status[0], (epoch << 2) | 2u);
+    }
+    return identity;
+  }
+  if (lane == 0) {
+    lb_store(&a.agg[tile], agg);
+    __threadfence();
+    st_relaxed_u32(&a.status[tile], (epoch << 2) | 1u);
+  }
+  T acc = identity;
+  int64_t base = (int64_t)tile - 1;
+  uint32_t spins = 0, ns = 20;
+  for (;;) {
+    const int64_t idx = base - (int64_t)lane;
+    uint32_t f = 2;
+    if (idx >= 0) {
+      const uint32_t s = ld_relaxed_u32(&a.status[idx]);
+      f = ((s >> 2) == epoch) ? (s & 3u) : 0u;
+    }
+    if (__any_sync(kFull, f == 0)) {
+      if (++spins > kSpinCap) {
+        if (lane == 0) raise_err(st, kErrTimeout);
+        return identity;
+      }
+      __nanosleep(ns);
+      if (ns < 1000) ns += ns;
+      continue;
+    }
+    __threadfence();
+    const uint32_t incl = __ballot_sync(kFull, f == 2);
+    const uint32_t first = incl ? (uint32_t)(__ffs(incl) - 1) : 31u;
+    T x = identity;
+    if (idx >= 0 && lane <= first) x = (f == 2) ? lb_load(&a.incl[idx]) : lb_load(&a.agg[idx]);
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const T y = shfl_down_payload(x, o);
+      if (lane + o < 32) x = op(y, x);
+    }
+    acc = op(shfl_payload(x, 0), acc);
+    if (incl) break;
+    base -= 32;
+  }
+  if (lane == 0) {
+    const T inc = op(acc, agg);
+    lb_store(&a.incl[tile], inc);
+    __threadfence();
+    st_relaxed_u32(&a.status[tile], (epoch << 2) | 2u);
+  }
+  return acc;
+}
+
+// ---------------------------------------------------------------------------
+// CTA-wide look-back: every thread of the CTA calls it, and each round
+// inspects blockDim.x predecessors at once, so the inclusive-prefix frontier
+// advances a whole CTA width per round trip.  blockDim.x must be a multiple of
+// 32 (at most 1024).  Returns the exclusive prefix in every thread.
+// ---------------------------------------------------------------------------
+__device__ inline uint64_t lookback_sum_cta(uint64_t* words, uint32_t tile, uint64_t agg, uint32_t epoch,
+                                            DevStatus* st) {
+  __shared__ uint64_t s_part[32];
+  __shared__ uint32_t s_first;
+  __shared__ uint64_t s_excl;
+  const uint32_t t = threadIdx.x, lane = t & 31, wid = t >> 5, nw = blockDim.x >> 5;
+  if (tile == 0) {
+    if (t == 0) st_relaxed_u64(&words[0], lb_pack(epoch, 2, agg));
+    return 0;
+  }
+  if (t == 0) {
+    st_relaxed_u64(&words[tile], lb_pack(epoch, 1, agg));
+    s_excl = 0;
+  }
+  int64_t base = (int64_t)tile - 1;
+  uint32_t spins = 0, ns = 20;
+  for (;;) {
+    const int64_t idx = base - (int64_t)t;
+    uint32_t f = 2;
+    uint64_t v = 0;
+    if (idx >= 0) {
+      const uint64_t wv = ld_relaxed_u64(&words[idx]);
+      f = ((uint32_t)(wv >> 58) == epoch) ? (uint32_t)((wv >> 56) & 3) : 0u;
+      v = wv & kLbValMask;
+    }
+    if (__syncthreads_or(f == 0)) {
+      if (++spins > kSpinCap) {
+        if (t == 0) {
+          raise_err(st, kErrTimeout);
+          s_excl = 0;
+        }
+        break;
+      }
+      __nanosleep(ns);
+      if (ns < 500) ns += ns;
+      continue;
+    }
+    if (t == 0) s_first = 0xFFFFFFFFu;
+    __syncthreads();
+    if (f == 2) atomicMin(&s_first, t);
+    __syncthreads();
+    const uint32_t first = s_first;
+    if (t > first) v = 0;
+    v = warp_sum_u64(v);
+    if (lane == 0) s_part[wid] = v;
+    __syncthreads();
+    if (t == 0) {
+      uint64_t sum = 0;
+      for (uint32_t k = 0; k < nw; ++k) sum += s_part[k];
+      s_excl += sum;
+    }
+    __syncthreads();
+    if (first != 0xFFFFFFFFu) break;
+    base -= (int64_t)blockDim.x;
+  }
+  if (t == 0) st_relaxed_u64(&words[tile], lb_pack(epoch, 2, s_excl + agg));
+  __syncthreads();
+  return s_excl;
+}
+
+template <class T, class Op>
+__device__ inline T lookback_cta(LbArrays<T> a, uint32_t tile, const T& agg, const T& identity, Op op,
+                                 uint32_t epoch, DevStatus* st) {
+  static_assert(sizeof(T) % 8 == 0, "payload must be a multiple of 8 bytes");
+  __shared__ T s_wres[32];
+  __shared__ T s_acc;
+  __shared__ uint32_t s_first;
+  const uint32_t t = threadIdx.x, lane = t & 31, wid = t >> 5, nw = blockDim.x >> 5;
+  if (tile == 0) {
+    if (t == 0) {
+      lb_store(&a.incl[0], agg);
+      __threadfence();
+      st_relaxed_u32(&a.status[0], (epoch << 2) | 2u);
+    }
+    return identity;
+  }
+  if (t == 0) {
+    lb_store(&a.agg[tile], agg);
+    __threadfence();
+    st_relaxed_u32(&a.status[tile], (epoch << 2) | 1u);
+    s_acc = identity;
+  }
+  int64_t base = (int64_t)tile - 1;
+  uint32_t spins = 0, ns = 20;
+  for (;;) {
+    const int64_t idx = base - (int64_t)t;
+    uint32_t f = 2;
+    if (idx >= 0) {
+      const uint32_t sv = ld_relaxed_u32(&a.status[idx]);
+      f = ((sv >> 2) == epoch) ? (sv & 3u) : 0u;
+    }
+    if (__syncthreads_or(f == 0)) {
+      if (++spins > kSpinCap) {
+        if (t == 0) {
+          raise_err(st, kErrTimeout);
+          s_acc = identity;
+        }
+        break;
+      }
+      __nanosleep(ns);
+      if (ns < 500) ns += ns;
+      continue;
+    }
+    __threadfence();
+    if (t == 0) s_first = 0xFFFFFFFFu;
+    __syncthreads();
+    if (f == 2 && idx >= 0) atomicMin(&s_first, t);
+    __syncthreads();
+    const uint32_t first = s_first;
+    T x = identity;
+    if (idx >= 0 && t <= first) x = (f == 2) ? lb_load(&a.incl[idx]) : lb_load(&a.agg[idx]);
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const T y = shfl_down_payload(x, o);
+      if (lane + o < 32) x = op(y, x);
+    }
+    if (lane == 0) s_wres[wid] = x;
+    __syncthreads();
+    if (t == 0) {
+      T r = identity;
+      for (int k = (int)nw - 1; k >= 0; --k) r = op(r, s_wres[k]);
+      s_acc = op(r, s_acc);
+    }
+    __syncthreads();
+    // a window reaching past tile 0 counts as complete (idx < 0 reads as inclusive)
+    if (first != 0xFFFFFFFFu || base < (int64_t)blockDim.x) break;
+    base -= (int64_t)blockDim.x;
+  }
+  if (t == 0) {
+    const T inc = op(s_acc, agg);
+    lb_store(&a.incl[tile], inc);
+    __threadfence();
+    st_relaxed_u32(&a.status[tile], (epoch << 2) | 2u);
+  }
+  __syncthreads();
+  return s_acc;
+}
+
+// ---------------------------------------------------------------------------
+// Bulk (TMA) copies global -> shared with mbarrier completion (sm_90+).
+// The source and destination must be 16-byte aligned and the size a multiple
+// of 16 bytes.  Waits are bounded: on give-up the caller raises kErrTimeout.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_init_fence() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_addr(dst)),
+               "l"(src), "r"(bytes), "r"(smem_addr(bar))
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t phase) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(phase)
+      : "memory");
+  return ok != 0;
+}
+// Wait for phase `phase` of `bar`; false if the bounded wait gave up.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t phase) {
+  for (uint32_t i = 0; i < (1u << 22); ++i)
+    if (mbar_try_wait(bar, phase)) return true;
+  return false;
+}
+
 // ---------------------------------------------------------------------------
 // GF(2^61 - 1)
 // ---------------------------------------------------------------------------

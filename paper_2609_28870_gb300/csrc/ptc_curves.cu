@@ -136,8 +136,10 @@ __global__ void __launch_bounds__(kCvThreads) k_curves(CurveArgs a) {
     if (lane < kCvThreads / 32) s_w[lane] = z;
   }
   __syncthreads();
-  if (threadIdx.x == 0) s_carry = lookback_generic(a.lb, tile, s_w[kCvThreads / 32 - 1], RunMax{0, 0, 0}, op,
-                                                   kEpochCurves, a.st);
+  {
+    const RunMax cin = lookback_cta(a.lb, tile, s_w[kCvThreads / 32 - 1], RunMax{0, 0, 0}, op, kEpochCurves, a.st);
+    if (threadIdx.x == 0) s_carry = cin;
+  }
   __syncthreads();
   // exclusive prefix of this thread = carry (+) warps before (+) lanes before
   RunMax pre = s_carry;

@@ -64,10 +64,10 @@ __device__ __forceinline__ uint64_t cta_exclusive_sum(uint64_t v, uint64_t* tota
 
 __global__ void __launch_bounds__(kOffThreads) k_block_offsets(const uint64_t* __restrict__ tok_off,
                                                                const int64_t* __restrict__ ts, uint32_t R,
-                                                               uint64_t n_tok, uint32_t B,
-                                                               uint64_t* __restrict__ blk_off, uint64_t* lb,
-                                                               DevStatus* st) {
-  __shared__ uint64_t s_base;
+                                                               uint64_t n_tok, uint32_t B, uint32_t tb,
+                                                               uint64_t* __restrict__ blk_off,
+                                                               uint32_t* __restrict__ tile_req, uint64_t tile_cap,
+                                                               uint64_t* lb, DevStatus* st) {
   const uint32_t tile = next_tile(st, kEpochOffsets);
   const uint64_t r0 = (uint64_t)tile * kOffTile + (uint64_t)threadIdx.x * kOffPer;
   uint64_t cnt[kOffPer];
@@ -93,16 +93,19 @@ __global__ void __launch_bounds__(kOffThreads) k_block_offsets(const uint64_t* _
   if (kmax) atomicMax((unsigned long long*)&st->value[1], (unsigned long long)kmax);
   uint64_t total;
   uint64_t excl = cta_exclusive_sum(local, &total);
-  if (threadIdx.x < 32) {
-    uint64_t base = lookback_sum(lb, tile, total, kEpochOffsets, st);
-    if (threadIdx.x == 0) s_base = base;
-  }
-  __syncthreads();
-  uint64_t run = s_base + excl;
+  const uint64_t base = lookback_sum_cta(lb, tile, total, kEpochOffsets, st);
+  uint64_t run = base + excl;
 #pragma unroll
   for (int j = 0; j < kOffPer; ++j) {
     uint64_t r = r0 + j;
-    if (r < R) blk_off[r] = run;
+    if (r < R) {
+      blk_off[r] = run;
+      // hash tiles whose first block lies in this request
+      if (cnt[j]) {
+        const uint64_t last = (run + cnt[j] - 1) / tb;
+        for (uint64_t t = (run + tb - 1) / tb; t <= last && t < tile_cap; ++t) tile_req[t] = (uint32_t)r;
+      }
+    }
     run += cnt[j];
     if (r + 1 == R) {
       blk_off[R] = run;
@@ -172,6 +175,7 @@ struct HashArgs {
   ulonglong2* keys;
   uint64_t keys_cap;
   const uint64_t* tables;
+  const uint32_t* tile_req;
   LbArrays<HashCarry> lb;
   DevStatus* st;
   int aligned;
@@ -216,9 +220,12 @@ __global__ void __launch_bounds__(kHashThreads) k_hash(HashArgs a, const __grid_
   const uint64_t b_end = b0 + TB < N ? b0 + TB : N;
   const uint32_t B = a.B;
 
-  if (threadIdx.x < 2) {
-    const uint64_t b = threadIdx.x == 0 ? b0 : b_end - 1;
-    s_bnd[threadIdx.x] = find_request(a.blk_off, 0, a.R - 1, b);
+  if (threadIdx.x == 0) {
+    const uint64_t ntiles = (N + TB - 1) / TB;
+    const uint32_t r0 = a.tile_req[tile];
+    const uint32_t rh = tile + 1 < ntiles ? a.tile_req[tile + 1] : a.R - 1;
+    s_bnd[0] = r0;
+    s_bnd[1] = find_request(a.blk_off, r0, rh, b_end - 1);
   }
   __syncthreads();
   const uint32_t r_first = (uint32_t)s_bnd[0], r_last = (uint32_t)s_bnd[1];
@@ -364,9 +371,10 @@ __global__ void __launch_bounds__(kHashThreads) k_hash(HashArgs a, const __grid_
   }
   __syncthreads();
   if (w > 0) x = op(s_w[w - 1], x);
-  if (t == 0) {
-    const HashCarry agg = s_w[kHashThreads / 32 - 1];
-    s_carry = lookback_generic(a.lb, tile, agg, HashCarry{0, 0, 0}, op, kEpochHash, a.st);
+  {
+    const HashCarry cin = lookback_cta(a.lb, tile, s_w[kHashThreads / 32 - 1], HashCarry{0, 0, 0}, op, kEpochHash,
+                                       a.st);
+    if (threadIdx.x == 0) s_carry = cin;
   }
   __syncthreads();
   if (valid) {
@@ -402,6 +410,8 @@ struct HashLayout {
   HashCarry* lb_hash_agg;
   HashCarry* lb_hash_incl;
   uint64_t* tables;
+  uint32_t* tile_req;
+  uint64_t hash_tiles;
   size_t zero_bytes;
   size_t total;
 };
@@ -420,6 +430,8 @@ HashLayout hash_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   L.lb_hash_agg = cv.take<HashCarry>(hash_tiles);
   L.lb_hash_incl = cv.take<HashCarry>(hash_tiles);
   L.tables = cv.take<uint64_t>(8 * 65536);
+  L.tile_req = cv.take<uint32_t>(hash_tiles + 1);
+  L.hash_tiles = hash_tiles;
   L.total = cv.bytes();
   return L;
 }
@@ -454,8 +466,11 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
     DevStatus h;
     return end_call(L.st, s, &h);
   }
-  PTC_LAUNCH("k_block_offsets", s, k_block_offsets<<<ceil_div_u32(n_req, kOffTile), kOffThreads, 0, s>>>(req_tok_off, req_ts_us, n_req, n_tok,
-                                                                        block_size, req_blk_off_out, L.lb_off, L.st));
+  const uint32_t G = chunks_per_block(block_size);
+  PTC_LAUNCH("k_block_offsets", s,
+             k_block_offsets<<<ceil_div_u32(n_req, kOffTile), kOffThreads, 0, s>>>(
+                 req_tok_off, req_ts_us, n_req, n_tok, block_size, kHashThreads / G, req_blk_off_out, L.tile_req,
+                 L.hash_tiles, L.lb_off, L.st));
 
   // seeded bases and their derived constants
   PowBases pb;
@@ -488,10 +503,10 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
   a.keys = reinterpret_cast<ulonglong2*>(keys_out);
   a.keys_cap = keys_cap;
   a.tables = L.tables;
+  a.tile_req = L.tile_req;
   a.lb = LbArrays<HashCarry>{L.lb_hash_status, L.lb_hash_agg, L.lb_hash_incl};
   a.st = L.st;
   a.aligned = (((uintptr_t)tokens) & 15) == 0;
-  const uint32_t G = chunks_per_block(block_size);
   const bool full = block_size == 16 * G;
   const uint64_t nb = n_tok / block_size < keys_cap ? n_tok / block_size : keys_cap;
   const uint32_t grid = ceil_div_u32(nb, kHashThreads / G);

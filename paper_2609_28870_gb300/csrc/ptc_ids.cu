@@ -47,7 +47,7 @@ __device__ __forceinline__ uint64_t home_slot(uint64_t h0, uint64_t h1, uint32_t
 }
 
 __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __restrict__ keys, uint64_t n,
-                                                            ulonglong2* table, uint32_t log2m,
+                                                            ulonglong2* table, uint32_t log2m, uint64_t probe_cap,
                                                             uint32_t* __restrict__ slot_of, DevStatus* st) {
   const uint64_t i = (uint64_t)blockIdx.x * kInsThreads + threadIdx.x;
   if (i >= n) return;
@@ -65,7 +65,7 @@ __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __
   const ulonglong2 empty = make_ulonglong2(~0ULL, ~0ULL);
   const uint64_t mask = (1ULL << log2m) - 1;
   uint64_t pos = home_slot(k.x, k.y, log2m);
-  for (uint64_t probe = 0; probe <= mask; ++probe) {
+  for (uint64_t probe = 0; probe <= mask && probe < probe_cap; ++probe) {
     const ulonglong2 old = cas128(&table[pos], empty, mine);
     if (old.x == ~0ULL && old.y == ~0ULL) {
       slot_of[i] = (uint32_t)pos;
@@ -111,7 +111,6 @@ __global__ void __launch_bounds__(kRankThreads) k_ids_rank(const ulonglong2* __r
                                                            const uint32_t* __restrict__ slot_of, uint64_t n,
                                                            uint32_t* __restrict__ slot_id, uint64_t* lb,
                                                            DevStatus* st) {
-  __shared__ uint64_t s_base;
   const uint32_t tile = next_tile(st, kEpochRank);
   const uint64_t i0 = (uint64_t)tile * kRankTile + (uint64_t)threadIdx.x * kRankPer;
   uint32_t slots[kRankPer];
@@ -131,12 +130,7 @@ __global__ void __launch_bounds__(kRankThreads) k_ids_rank(const ulonglong2* __r
   }
   uint64_t total;
   const uint64_t excl = cta_exclusive_sum512(cnt, &total);
-  if (threadIdx.x < 32) {
-    const uint64_t base = lookback_sum(lb, tile, total, kEpochRank, st);
-    if (threadIdx.x == 0) s_base = base;
-  }
-  __syncthreads();
-  uint64_t rank = s_base + excl;
+  uint64_t rank = lookback_sum_cta(lb, tile, total, kEpochRank, st) + excl;
 #pragma unroll
   for (int j = 0; j < kRankPer; ++j) {
     if (flags & (1u << j)) slot_id[slots[j]] = (uint32_t)rank++;
@@ -153,12 +147,19 @@ __global__ void k_ids_gather(const uint32_t* __restrict__ slot_of, const uint32_
   if (i < n) ids[i] = slot_id[slot_of[i]];
 }
 
-uint32_t table_log2(uint64_t n) {
-  const uint64_t want = n + n / 2 + 64;
-  uint32_t l = 6;
+// Slots for n keys at most: the full table holds 1.5 n; the first attempt
+// holds n / 3 (real traces repeat most blocks, so it is rarely more than 40%
+// full and, at this size, stays in L2).  If a probe sequence of the first
+// attempt runs past kSmallProbeCap slots, the call redoes the stage with the
+// full table.
+constexpr uint64_t kSmallProbeCap = 4096;
+uint32_t table_log2(uint64_t want) {
+  uint32_t l = 10;
   while ((1ULL << l) < want) ++l;
   return l;
 }
+uint32_t full_table_log2(uint64_t n) { return table_log2(n + n / 2 + 64); }
+uint32_t small_table_log2(uint64_t n) { return table_log2(n / 3 + 64); }
 
 struct IdsLayout {
   DevStatus* st;
@@ -174,7 +175,7 @@ struct IdsLayout {
 IdsLayout ids_layout(void* ws, uint64_t n) {
   IdsLayout L;
   Carver cv(ws);
-  L.log2m = table_log2(n);
+  L.log2m = full_table_log2(n);
   const uint64_t m = 1ULL << L.log2m;
   L.st = cv.take<DevStatus>(1);
   L.lb = cv.take<uint64_t>(ceil_div_u32(n, kRankTile) + 1);
@@ -259,12 +260,31 @@ extern "C" ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t*
   cudaStream_t s = (cudaStream_t)stream;
   const IdsLayout L = ids_layout(ws, n);
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
-  if (n > 0) {
-    if (cudaMemsetAsync(L.table, 0xFF, sizeof(ulonglong2) << L.log2m, s) != cudaSuccess) return PTC_ERR_CUDA;
+  auto run = [&](uint32_t log2m, uint64_t probe_cap) -> bool {
+    if (cudaMemsetAsync(L.table, 0xFF, sizeof(ulonglong2) << log2m, s) != cudaSuccess) return false;
     const ulonglong2* k = reinterpret_cast<const ulonglong2*>(keys);
-    PTC_LAUNCH("k_ids_insert", s, k_ids_insert<<<ceil_div_u32(n, kInsThreads), kInsThreads, 0, s>>>(k, n, L.table, L.log2m, L.slot_of, L.st));
-    PTC_LAUNCH("k_ids_rank", s, k_ids_rank<<<ceil_div_u32(n, kRankTile), kRankThreads, 0, s>>>(L.table, L.slot_of, n, L.slot_id, L.lb, L.st));
+    PTC_LAUNCH("k_ids_insert", s, k_ids_insert<<<ceil_div_u32(n, kInsThreads), kInsThreads, 0, s>>>(
+                                      k, n, L.table, log2m, probe_cap, L.slot_of, L.st));
+    PTC_LAUNCH("k_ids_rank", s, k_ids_rank<<<ceil_div_u32(n, kRankTile), kRankThreads, 0, s>>>(
+                                    L.table, L.slot_of, n, L.slot_id, L.lb, L.st));
     PTC_LAUNCH("k_ids_gather", s, k_ids_gather<<<ceil_div_u32(n, 256), 256, 0, s>>>(L.slot_of, L.slot_id, n, ids_out));
+    return true;
+  };
+  if (n > 0) {
+    const uint32_t small = small_table_log2(n);
+    if (!run(small, small < L.log2m ? kSmallProbeCap : ~0ULL)) return PTC_ERR_CUDA;
+    if (small < L.log2m) {
+      DevStatus h1;
+      const ptc_status rc1 = end_call(L.st, s, &h1);
+      if (rc1 == PTC_OK) {
+        *n_distinct_host_out = h1.value[0];
+        return PTC_OK;
+      }
+      if (!(h1.err & kErrTableFull)) return rc1;
+      // the small table overflowed: redo with the full one
+      if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
+      if (!run(L.log2m, ~0ULL)) return PTC_ERR_CUDA;
+    }
   }
   DevStatus h;
   const ptc_status rc = end_call(L.st, s, &h);

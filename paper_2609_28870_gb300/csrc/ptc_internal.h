@@ -45,6 +45,14 @@ inline ptc_status end_call(const DevStatus* dev, cudaStream_t stream, DevStatus*
   return PTC_OK;
 }
 
+// Streaming multiprocessors of the current device (persistent grids).
+inline int num_sms() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return 148;
+  return n;
+}
+
 inline bool ws_ok(const void* ws, size_t ws_bytes, size_t need) {
   return ws != nullptr && ((uintptr_t)ws & 255) == 0 && ws_bytes >= need;
 }

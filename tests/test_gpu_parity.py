@@ -236,3 +236,36 @@ def test_deterministic_repeat():
     for k in ("keys", "ids", "prev", "next", "dist"):
         assert np.array_equal(a[k], b[k])
     assert a["hits"] == b["hits"] and a["saved"] == b["saved"]
+
+
+def test_all_distinct_blocks_take_the_full_table():
+    """One long request: every block is distinct (different prefix lengths),
+    so the first, smaller hash table overflows and the call redoes the stage
+    with the full one."""
+    rng = np.random.default_rng(9)
+    tr = tracegen.from_lists([rng.integers(0, 2**32, 60000, dtype=np.uint64).tolist()])
+    gu = _g()
+    caps = [1, 2, 100]
+    g = gu.gpu_run(tr, 1, caps)
+    o = gu.oracle_run(tr, 1, caps)
+    gu.assert_same(g, o)
+    assert g["n_distinct"] == 60000
+
+
+def test_long_runs_and_run_breaks():
+    """Stack distances over long copied runs (a run's accesses share one
+    distance) with runs broken by truncation, interleaving and cold blocks."""
+    reqs, ctx = [], []
+    rng = np.random.default_rng(4)
+    for t in range(30):
+        ctx = ctx + rng.integers(0, 1000, int(rng.integers(40, 400))).tolist()
+        if t % 7 == 6:
+            ctx = ctx[:30] + ctx[200:]  # truncation breaks the run
+        reqs.append(list(ctx))
+        reqs.append(rng.integers(0, 1000, 50).tolist())  # an unrelated request in between
+    tr = tracegen.from_lists(reqs)
+    gu = _g()
+    for B in (1, 4, 16):
+        ids, D = oracle.block_ids(tr.tokens, tr.req_tok_off, B)
+        caps = tracegen.capacity_grid(1, D + 1, 40)
+        gu.assert_same(gu.gpu_run(tr, B, caps), gu.oracle_run(tr, B, caps))
