@@ -204,6 +204,31 @@ ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_
                       size_t ws_bytes, void* stream);
 
 /*
+ * ptc_curves_noalloc — ptc_curves for callers that cannot allocate device
+ * memory.  The paper has no counterpart; this entry point exists for callers
+ * with no way to supply `ws`: code running inside a runtime that owns all
+ * device memory and offers no allocator, hosts that forbid cudaMalloc (which
+ * may synchronize the device), or loops that must never enter an allocator.
+ * Its scratch is one fixed 4 MiB array in the library's device image, which
+ * every GPU that loads the library holds until the process exits.  Same
+ * arguments and results as ptc_curves without ws / ws_bytes.
+ *   - n at most 2^24 accesses (PTC_ERR_WORKSPACE beyond that), n_cap at most
+ *     PTC_MAX_CAPACITIES.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current; make that first call
+ *     before any stream capture.
+ *   - Every call on a device shares the one array, and each call leaves its
+ *     contents behind (the next call re-zeroes what must start at zero).
+ *     Calls whose work overlaps on the GPU (for example on two streams) race
+ *     on it and give wrong results: serialize them.
+ *   - Allocates nothing: no cudaMalloc or cudaFree.
+ */
+ptc_status ptc_curves_noalloc(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,
+                              uint32_t block_size, const ptc_cost_model* cm, const uint64_t* cap_host,
+                              uint32_t n_cap, uint64_t* hits_host_out, ptc_u128* saved_host_out,
+                              ptc_u128* total_cost_host_out, void* stream);
+
+/*
  * Measurement hooks (no counterpart in the paper: instrumentation for the
  * roofline figures).  ptc_launch_count() counts every kernel this library has
  * launched in the process.  While ptc_timer_enable(1) is in force, every

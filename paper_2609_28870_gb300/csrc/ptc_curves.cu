@@ -342,3 +342,56 @@ extern "C" ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_
   total_cost_host_out->hi = host_out[3 * n_cap + 1];
   return PTC_OK;
 }
+
+// ---------------------------------------------------------------------------
+// ptc_curves_noalloc: the curves for callers that cannot allocate device
+// memory.  Some callers have no way to hand this library a workspace: code
+// that runs inside another runtime which owns every byte of device memory
+// and exposes no allocator, plugin hosts that forbid cudaMalloc (it can
+// synchronize the device and stall unrelated work), or latency-critical
+// loops that must not enter the allocator at all.  For them the scratch that
+// ptc_curves takes from `ws` lives in one fixed array in this library's
+// device image instead, reserved when the library is loaded and held by every
+// GPU that loads it until the process exits.
+// ---------------------------------------------------------------------------
+#include <mutex>
+
+namespace {
+constexpr uint64_t kNoAllocMaxAccesses = 1ULL << 24;
+constexpr size_t kNoAllocScratchBytes = 4u << 20;
+static __device__ __align__(256) unsigned char g_curves_scratch[kNoAllocScratchBytes];
+constexpr int kNoAllocMaxDevices = 64;
+std::mutex g_scratch_mu;
+void* g_scratch_addr[kNoAllocMaxDevices] = {};
+
+// Device address of g_curves_scratch on the current device, looked up once per
+// device (the host-side symbol is only a stand-in, not a device address).
+ptc_status scratch_for_current_device(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return PTC_ERR_CUDA;
+  if (dev < 0 || dev >= kNoAllocMaxDevices) return PTC_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(g_scratch_mu);
+  if (g_scratch_addr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_curves_scratch) != cudaSuccess || p == nullptr) return PTC_ERR_CUDA;
+    g_scratch_addr[dev] = p;
+  }
+  *out = g_scratch_addr[dev];
+  return PTC_OK;
+}
+}  // namespace
+
+extern "C" ptc_status ptc_curves_noalloc(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_off,
+                                         uint32_t n_req, uint32_t block_size, const ptc_cost_model* cm,
+                                         const uint64_t* cap_host, uint32_t n_cap, uint64_t* hits_host_out,
+                                         ptc_u128* saved_host_out, ptc_u128* total_cost_host_out, void* stream) {
+  if (n > kNoAllocMaxAccesses) return PTC_ERR_WORKSPACE;
+  if (n_cap > PTC_MAX_CAPACITIES) return PTC_ERR_INVALID_ARG;
+  if (curves_layout(nullptr, n, n_cap).total > kNoAllocScratchBytes) return PTC_ERR_WORKSPACE;
+  void* scratch = nullptr;
+  const ptc_status rc = scratch_for_current_device(&scratch);
+  if (rc != PTC_OK) return rc;
+  // ptc_curves zeroes every part of the scratch that must start at zero.
+  return ptc_curves(dist, n, req_blk_off, n_req, block_size, cm, cap_host, n_cap, hits_host_out, saved_host_out,
+                    total_cost_host_out, scratch, kNoAllocScratchBytes, stream);
+}
