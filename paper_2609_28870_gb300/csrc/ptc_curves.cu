@@ -59,45 +59,31 @@ struct CurveArgs {
   uint32_t G;
   unsigned long long* cnt;   // G + 1 bins (last: miss at every capacity)
   unsigned long long* ksum;  // G + 1 bins
-  LbArrays<RunMax> lb;
+  const RunMax* tile_agg;
   DevStatus* st;
 };
 
-__global__ void __launch_bounds__(kCvThreads) k_curves(CurveArgs a) {
-  __shared__ uint32_t s_cap[PTC_MAX_CAPACITIES];
-  __shared__ uint32_t s_cnt[PTC_MAX_CAPACITIES + 1];
-  __shared__ unsigned long long s_ks[PTC_MAX_CAPACITIES + 1];
-  __shared__ RunMax s_w[kCvThreads / 32];
-  __shared__ RunMax s_carry;
-  const uint32_t G = a.G;
-  for (uint32_t g = threadIdx.x; g < G; g += kCvThreads)
-    s_cap[g] = a.caps[g] >= (uint64_t)kNone ? kNone - 1 : (uint32_t)a.caps[g];
-  for (uint32_t g = threadIdx.x; g <= G; g += kCvThreads) {
-    s_cnt[g] = 0;
-    s_ks[g] = 0;
-  }
-  const uint32_t tile = next_tile(a.st, kEpochCurves);
-  const uint64_t i0 = (uint64_t)tile * kCvTile + (uint64_t)threadIdx.x * kCvPer;
-
+// Loads the kCvPer distances of this thread and the head bits of its range,
+// and folds them into the thread's running max (with the segment start).
+__device__ __forceinline__ void load_run(const uint32_t* __restrict__ dist, const uint32_t* __restrict__ bitmap,
+                                         uint64_t n, uint64_t i0, uint64_t (&e)[kCvPer], uint64_t (&st_idx)[kCvPer],
+                                         uint32_t& has_head, RunMax& loc) {
   uint32_t d[kCvPer];
-  if (i0 + kCvPer <= a.n && ((reinterpret_cast<uintptr_t>(a.dist) & 15) == 0)) {
-    const uint4 x = __ldcs(reinterpret_cast<const uint4*>(a.dist + i0));
-    const uint4 y = __ldcs(reinterpret_cast<const uint4*>(a.dist + i0 + 4));
+  if (i0 + kCvPer <= n && ((reinterpret_cast<uintptr_t>(dist) & 15) == 0)) {
+    const uint4 x = __ldg(reinterpret_cast<const uint4*>(dist + i0));
+    const uint4 y = __ldg(reinterpret_cast<const uint4*>(dist + i0 + 4));
     d[0] = x.x; d[1] = x.y; d[2] = x.z; d[3] = x.w;
     d[4] = y.x; d[5] = y.y; d[6] = y.z; d[7] = y.w;
   } else {
 #pragma unroll
-    for (int j = 0; j < kCvPer; ++j) d[j] = i0 + j < a.n ? a.dist[i0 + j] : 0u;
+    for (int j = 0; j < kCvPer; ++j) d[j] = i0 + j < n ? dist[i0 + j] : 0u;
   }
-  const uint32_t heads = i0 < a.n ? (a.bitmap[i0 >> 5] >> (i0 & 31)) & 0xFFu : 0u;
-
-  // thread-local inclusive running max
-  RunMax loc{0, 0, 0};
-  uint64_t e[kCvPer], st_idx[kCvPer];
-  uint32_t has_head = 0;  // bit j: a head at or before j inside this thread
+  const uint32_t heads = i0 < n ? (bitmap[i0 >> 5] >> (i0 & 31)) & 0xFFu : 0u;
+  loc = RunMax{0, 0, 0};
+  has_head = 0;
 #pragma unroll
   for (int j = 0; j < kCvPer; ++j) {
-    const uint64_t dv = (i0 + j < a.n) ? d[j] : 0u;
+    const uint64_t dv = (i0 + j < n) ? d[j] : 0u;
     if ((heads >> j) & 1u) {
       loc.f = 1;
       loc.m = dv;
@@ -109,10 +95,14 @@ __global__ void __launch_bounds__(kCvThreads) k_curves(CurveArgs a) {
     st_idx[j] = loc.start;
     if (loc.f) has_head |= 1u << j;
   }
-  // CTA-wide exclusive segmented scan of thread aggregates
+}
+
+// CTA-wide inclusive segmented scan of the thread aggregates: returns the
+// thread's inclusive value within its warp in *x and leaves the inclusive value
+// over warps in s_w (s_w[last] is the tile aggregate).
+__device__ __forceinline__ void cta_runmax_scan(RunMax& x, RunMax* s_w) {
   RunMaxOp op;
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  RunMax x = loc;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
     RunMax y;
@@ -136,9 +126,66 @@ __global__ void __launch_bounds__(kCvThreads) k_curves(CurveArgs a) {
     if (lane < kCvThreads / 32) s_w[lane] = z;
   }
   __syncthreads();
-  {
-    const RunMax cin = lookback_cta(a.lb, tile, s_w[kCvThreads / 32 - 1], RunMax{0, 0, 0}, op, kEpochCurves, a.st);
-    if (threadIdx.x == 0) s_carry = cin;
+}
+
+// Pass 1: every tile's aggregate (request start seen?, running max since the
+// last start, index of that start).  Tiles are independent.
+__global__ void __launch_bounds__(kCvThreads) k_curves_agg(const uint32_t* __restrict__ dist, uint64_t n,
+                                                           const uint32_t* __restrict__ bitmap,
+                                                           RunMax* __restrict__ tile_agg) {
+  __shared__ RunMax s_w[kCvThreads / 32];
+  const uint64_t i0 = (uint64_t)blockIdx.x * kCvTile + (uint64_t)threadIdx.x * kCvPer;
+  uint64_t e[kCvPer], st_idx[kCvPer];
+  uint32_t has_head;
+  RunMax x;
+  load_run(dist, bitmap, n, i0, e, st_idx, has_head, x);
+  cta_runmax_scan(x, s_w);
+  if (threadIdx.x == 0) tile_agg[blockIdx.x] = s_w[kCvThreads / 32 - 1];
+}
+
+__global__ void __launch_bounds__(kCvThreads) k_curves(CurveArgs a) {
+  __shared__ uint32_t s_cap[PTC_MAX_CAPACITIES];
+  __shared__ uint32_t s_cnt[PTC_MAX_CAPACITIES + 1];
+  __shared__ unsigned long long s_ks[PTC_MAX_CAPACITIES + 1];
+  __shared__ RunMax s_w[kCvThreads / 32];
+  __shared__ RunMax s_carry;
+  const uint32_t G = a.G;
+  for (uint32_t g = threadIdx.x; g < G; g += kCvThreads)
+    s_cap[g] = a.caps[g] >= (uint64_t)kNone ? kNone - 1 : (uint32_t)a.caps[g];
+  for (uint32_t g = threadIdx.x; g <= G; g += kCvThreads) {
+    s_cnt[g] = 0;
+    s_ks[g] = 0;
+  }
+  const uint32_t tile = blockIdx.x;
+  const uint64_t i0 = (uint64_t)tile * kCvTile + (uint64_t)threadIdx.x * kCvPer;
+  uint64_t e[kCvPer], st_idx[kCvPer];
+  uint32_t has_head;
+  RunMax loc;
+  load_run(a.dist, a.bitmap, a.n, i0, e, st_idx, has_head, loc);
+  RunMaxOp op;
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  RunMax x = loc;
+  cta_runmax_scan(x, s_w);
+  // carry: fold of the aggregates of the tiles before this one, back to the
+  // nearest tile where a request starts (all written by k_curves_agg)
+  if (w == 0) {
+    RunMax acc{0, 0, 0};
+    for (int64_t base = (int64_t)tile - 1; base >= 0; base -= 32) {
+      const int64_t idx = base - (int64_t)lane;
+      RunMax g{0, 0, 0};
+      if (idx >= 0) g = a.tile_agg[idx];
+      const uint32_t heads = __ballot_sync(kFull, idx >= 0 && g.f);
+      const uint32_t first = heads ? (uint32_t)(__ffs(heads) - 1) : 31u;
+      if (lane > first) g = RunMax{0, 0, 0};
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const RunMax y = shfl_down_payload(g, o);
+        if (lane + o < 32) g = op(y, g);
+      }
+      acc = op(shfl_payload(g, 0), acc);
+      if (heads) break;
+    }
+    if (lane == 0) s_carry = acc;
   }
   __syncthreads();
   // exclusive prefix of this thread = carry (+) warps before (+) lanes before
@@ -258,7 +305,7 @@ CurvesLayout curves_layout(void* ws, uint64_t n, uint32_t G) {
   L.lb_status = cv.take<uint32_t>(tiles);
   L.zero_bytes = cv.off;
   L.lb_agg = cv.take<RunMax>(tiles);
-  L.lb_incl = cv.take<RunMax>(tiles);
+  L.lb_incl = cv.take<RunMax>(tiles);  // unused; keeps the layout (and the no-alloc limit) unchanged
   L.caps = cv.take<uint64_t>(PTC_MAX_CAPACITIES);
   L.out = cv.take<uint64_t>(3 * PTC_MAX_CAPACITIES + 2);
   L.total = cv.bytes();
@@ -322,8 +369,10 @@ extern "C" ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_
     a.G = n_cap;
     a.cnt = L.cnt;
     a.ksum = L.ksum;
-    a.lb = LbArrays<RunMax>{L.lb_status, L.lb_agg, L.lb_incl};
+    a.tile_agg = L.lb_agg;
     a.st = L.st;
+    PTC_LAUNCH("k_curves_agg", s,
+               k_curves_agg<<<ceil_div_u32(n, kCvTile), kCvThreads, 0, s>>>(dist, n, L.bitmap, L.lb_agg));
     PTC_LAUNCH("k_curves", s, k_curves<<<ceil_div_u32(n, kCvTile), kCvThreads, 0, s>>>(a));
   }
   PTC_LAUNCH("k_finalize", s, k_finalize<<<1, 32, 0, s>>>(L.cnt, L.ksum, n_cap, alpha, beta, L.out));

@@ -12,12 +12,16 @@
 //   k_block_offsets  per-request block counts -> exclusive scan (look-back),
 //                    validates offsets and timestamp order, max blocks/request
 //   k_pow_tables     rho^(+-B e) for e < 2^32 as two 65,536-entry levels
-//   k_hash           tokens staged through padded shared memory with 16-byte
+//   k_hash_local     tokens staged through padded shared memory with 16-byte
 //                    loads; each thread hashes 16 tokens (one "sub-chunk")
 //                    with 3 x 21-bit limbs of the powers held as constant
 //                    kernel parameters; sub-chunks of one block combine by
-//                    shuffles; the segmented sum runs across the CTA and
-//                    across CTAs by decoupled look-back.
+//                    shuffles; the segmented sum runs across the CTA.  Keys
+//                    after the tile's first request start are final; the tile
+//                    records its aggregate.  No tile depends on another.
+//   k_hash_chain     each tile's carry from its predecessors' aggregates
+//                    (all already written, so nothing waits), then the final
+//                    keys of the tile's leading blocks.
 #include "ptc_internal.h"
 
 namespace ptc {
@@ -32,7 +36,6 @@ constexpr int kWinTokens = 8192 + 256;
 constexpr int kWinWords = kWinTokens + kWinTokens / 16;
 
 constexpr int kEpochOffsets = 1;
-constexpr int kEpochHash = 2;
 
 // ---------------------------------------------------------------- block scans
 // Exclusive sum over a CTA of 512 threads; returns the CTA total in *total.
@@ -176,12 +179,35 @@ struct HashArgs {
   uint64_t keys_cap;
   const uint64_t* tables;
   const uint32_t* tile_req;
-  LbArrays<HashCarry> lb;
+  HashCarry* tile_agg;   // per tile: (request starts inside?, sum of g after the last start)
+  uint32_t* tile_lead;   // per tile: blocks before its first request start (keys left normalised)
   DevStatus* st;
   int aligned;
 };
 
 __device__ __forceinline__ uint32_t pad16(uint32_t i) { return i + (i >> 4); }
+
+// 32 x 32 -> 64-bit multiply-add; written in C so the compiler can take the
+// constant operand straight from the parameter bank.
+__device__ __forceinline__ uint64_t mad_wide(uint32_t a, uint32_t b, uint64_t c) {
+  return (uint64_t)a * (uint64_t)b + c;
+}
+
+// Sum over the 16 words t[m .. m+15] of t * rho^(15 - j) for both bases, as
+// 21-bit limb accumulators (M is the word offset of the first token).
+template <int M>
+__device__ __forceinline__ void hash16(const uint32_t (&wd)[20], const HashConsts& c, uint64_t (&acc)[6]) {
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const uint32_t t = wd[j + M];
+    acc[0] = mad_wide(t, c.limb[0][0][j], acc[0]);
+    acc[1] = mad_wide(t, c.limb[0][1][j], acc[1]);
+    acc[2] = mad_wide(t, c.limb[0][2][j], acc[2]);
+    acc[3] = mad_wide(t, c.limb[1][0][j], acc[3]);
+    acc[4] = mad_wide(t, c.limb[1][1][j], acc[4]);
+    acc[5] = mad_wide(t, c.limb[1][2][j], acc[5]);
+  }
+}
 
 // (a0 + a1 2^21 + a2 2^42) mod p for a0, a1, a2 < 2^62 - 2^57 (sums of <= 32 products < 2^53)
 __device__ __forceinline__ uint64_t limbs_to_p61(uint64_t a0, uint64_t a1, uint64_t a2) {
@@ -202,17 +228,104 @@ __device__ __forceinline__ uint32_t find_request(const uint64_t* __restrict__ bl
   return lo;
 }
 
-template <int G, bool FULL>
-__global__ void __launch_bounds__(kHashThreads) k_hash(HashArgs a, const __grid_constant__ HashConsts c) {
-  __shared__ uint32_t s_tok[kWinWords];
+// Shared second half of the local hash kernels: combine the sub-chunks of each
+// block, normalise, segmented sum over the tile, write keys and the tile's
+// aggregate.  Every thread of the CTA calls it.
+template <int G>
+__device__ __forceinline__ void hash_finish(const HashArgs& a, uint32_t tile, uint64_t b0, uint64_t b_end, uint64_t h0,
+                                            uint64_t h1, uint32_t k, uint32_t lb, uint32_t s) {
+  constexpr uint32_t TB = kHashThreads / G;
   __shared__ uint64_t s_h0[kHashThreads / G], s_h1[kHashThreads / G];
   __shared__ uint32_t s_k[kHashThreads / G];
-  __shared__ uint64_t s_bnd[4];
   __shared__ HashCarry s_w[kHashThreads / 32];
-  __shared__ HashCarry s_carry;
+  __shared__ uint32_t s_first_head;
+  if (G > 1) {
+#pragma unroll
+    for (int o = G / 2; o > 0; o >>= 1) {
+      h0 = p61_add(h0, __shfl_xor_sync(kFull, h0, o));
+      h1 = p61_add(h1, __shfl_xor_sync(kFull, h1, o));
+    }
+  }
+  if (s == 0) {
+    s_h0[lb] = h0;
+    s_h1[lb] = h1;
+    s_k[lb] = k;
+  }
+  __syncthreads();
+
+  // ---- phase 2: normalise, segmented sum over requests, denormalise
+  const uint32_t t = threadIdx.x;
+  const bool valid = t < TB && b0 + t < b_end;
+  const uint64_t* T = a.tables;
+  HashCarry x{0, 0, 0};
+  uint32_t kk = 0;
+  if (valid) {
+    kk = s_k[t];
+    const uint64_t e = (uint64_t)kk + 1;
+    x.v0 = p61_mul(s_h0[t], pow_at(T + 1 * 65536, T + 3 * 65536, e));
+    x.v1 = p61_mul(s_h1[t], pow_at(T + 5 * 65536, T + 7 * 65536, e));
+    if (kk == 0) {
+      x.f = 1;
+      x.v0 = p61_add(x.v0, 1);
+      x.v1 = p61_add(x.v1, 1);
+    }
+  }
+  SegSumOp op;
+  const uint32_t lane = t & 31, w = t >> 5;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    HashCarry y;
+    y.v0 = __shfl_up_sync(kFull, x.v0, d);
+    y.v1 = __shfl_up_sync(kFull, x.v1, d);
+    y.f = __shfl_up_sync(kFull, x.f, d);
+    if (lane >= (uint32_t)d) x = op(y, x);
+  }
+  if (lane == 31) s_w[w] = x;
+  __syncthreads();
+  if (w == 0) {
+    HashCarry z = lane < kHashThreads / 32 ? s_w[lane] : HashCarry{0, 0, 0};
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      HashCarry y;
+      y.v0 = __shfl_up_sync(kFull, z.v0, d);
+      y.v1 = __shfl_up_sync(kFull, z.v1, d);
+      y.f = __shfl_up_sync(kFull, z.f, d);
+      if (lane >= (uint32_t)d) z = op(y, z);
+    }
+    if (lane < kHashThreads / 32) s_w[lane] = z;  // inclusive over warps
+  }
+  __syncthreads();
+  if (w > 0) x = op(s_w[w - 1], x);
+  // Blocks at or after the tile's first request start are final here; the
+  // leading blocks keep their normalised partial sum for k_hash_chain.
+  if (t == 0) s_first_head = TB;
+  __syncthreads();
+  if (valid && kk == 0) atomicMin(&s_first_head, t);
+  __syncthreads();
+  if (valid) {
+    if (x.f) {
+      const uint64_t e = (uint64_t)kk + 1;
+      const uint64_t H0 = p61_mul(x.v0, pow_at(T + 0 * 65536, T + 2 * 65536, e));
+      const uint64_t H1 = p61_mul(x.v1, pow_at(T + 4 * 65536, T + 6 * 65536, e));
+      a.keys[b0 + t] = make_ulonglong2(H0, H1);
+    } else {
+      a.keys[b0 + t] = make_ulonglong2(x.v0, x.v1);
+    }
+  }
+  if (t == 0) {
+    a.tile_agg[tile] = s_w[kHashThreads / 32 - 1];
+    const uint32_t nb = (uint32_t)(b_end - b0);
+    a.tile_lead[tile] = s_first_head < nb ? s_first_head : nb;
+  }
+}
+
+template <int G, bool FULL>
+__global__ void __launch_bounds__(kHashThreads) k_hash_local(HashArgs a, const __grid_constant__ HashConsts c) {
+  __shared__ uint32_t s_tok[kWinWords];
+  __shared__ uint64_t s_bnd[4];
   constexpr uint32_t TB = kHashThreads / G;
 
-  const uint32_t tile = next_tile(a.st, kEpochHash);
+  const uint32_t tile = blockIdx.x;
   uint64_t N = a.st->value[0];
   if (N > a.keys_cap) N = a.keys_cap;
   const uint64_t b0 = (uint64_t)tile * TB;
@@ -314,87 +427,135 @@ __global__ void __launch_bounds__(kHashThreads) k_hash(HashArgs a, const __grid_
       h1 = p61_mul(h1, c.sub_mul[1][q]);
     }
   }
-  if (G > 1) {
-#pragma unroll
-    for (int o = G / 2; o > 0; o >>= 1) {
-      h0 = p61_add(h0, __shfl_xor_sync(kFull, h0, o));
-      h1 = p61_add(h1, __shfl_xor_sync(kFull, h1, o));
-    }
-  }
-  if (s == 0) {
-    s_h0[lb] = h0;
-    s_h1[lb] = h1;
-    s_k[lb] = k;
-  }
-  __syncthreads();
+  hash_finish<G>(a, tile, b0, b_end, h0, h1, k, lb, s);
+}
 
-  // ---- phase 2: normalise, segmented sum over requests, denormalise
-  const uint32_t t = threadIdx.x;
-  const bool valid = t < TB && b0 + t < b_end;
-  const uint64_t* T = a.tables;
-  HashCarry x{0, 0, 0};
-  uint32_t kk = 0;
-  if (valid) {
-    kk = s_k[t];
-    const uint64_t e = (uint64_t)kk + 1;
-    x.v0 = p61_mul(s_h0[t], pow_at(T + 1 * 65536, T + 3 * 65536, e));
-    x.v1 = p61_mul(s_h1[t], pow_at(T + 5 * 65536, T + 7 * 65536, e));
-    if (kk == 0) {
-      x.f = 1;
-      x.v0 = p61_add(x.v0, 1);
-      x.v1 = p61_add(x.v1, 1);
-    }
+// Fast path for 16-byte-aligned tokens and B a multiple of 16: every thread
+// reads its 16 tokens with four or five 16-byte loads straight from global
+// memory (a warp's loads cover consecutive 64-byte runs, so each line is
+// fetched once) and realigns them by a word offset that is uniform over a
+// request.  No shared-memory staging.
+template <int G>
+__global__ void __launch_bounds__(kHashThreads) k_hash_local_vec(HashArgs a, const __grid_constant__ HashConsts c) {
+  __shared__ uint32_t s_bnd[2];
+  constexpr uint32_t TB = kHashThreads / G;
+  const uint32_t tile = blockIdx.x;
+  uint64_t N = a.st->value[0];
+  if (N > a.keys_cap) N = a.keys_cap;
+  const uint64_t b0 = (uint64_t)tile * TB;
+  if (b0 >= N) return;
+  const uint64_t b_end = b0 + TB < N ? b0 + TB : N;
+  if (threadIdx.x == 0) {
+    const uint64_t ntiles = (N + TB - 1) / TB;
+    const uint32_t r0 = a.tile_req[tile];
+    const uint32_t rh = tile + 1 < ntiles ? a.tile_req[tile + 1] : a.R - 1;
+    s_bnd[0] = r0;
+    s_bnd[1] = find_request(a.blk_off, r0, rh, b_end - 1);
   }
-  SegSumOp op;
-  const uint32_t lane = t & 31, w = t >> 5;
+  __syncthreads();
+  const uint32_t r_first = s_bnd[0], r_last = s_bnd[1];
+  const uint32_t lb = threadIdx.x / G, s = threadIdx.x % G;
+  const uint64_t b = b0 + lb;
+  uint64_t h0 = 0, h1 = 0;
+  uint32_t k = 0;
+  if (b < b_end) {
+    const uint32_t r = find_request(a.blk_off, r_first, r_last, b);
+    k = (uint32_t)(b - a.blk_off[r]);
+    const uint64_t x = a.tok_off[r] + (uint64_t)a.B * k + 16ULL * s;
+    const uint32_t m = (uint32_t)(x & 3);
+    const uint64_t x4 = x - m;
+    uint32_t wd[20];
+    const uint4* p = reinterpret_cast<const uint4*>(a.tokens + x4);
+    const uint32_t nv = m ? 5u : 4u;
+    if (x4 + 4 * nv <= a.n_tok) {
 #pragma unroll
-  for (int d = 1; d < 32; d <<= 1) {
-    HashCarry y;
-    y.v0 = __shfl_up_sync(kFull, x.v0, d);
-    y.v1 = __shfl_up_sync(kFull, x.v1, d);
-    y.f = __shfl_up_sync(kFull, x.f, d);
-    if (lane >= (uint32_t)d) x = op(y, x);
-  }
-  if (lane == 31) s_w[w] = x;
-  __syncthreads();
-  if (w == 0) {
-    HashCarry z = lane < kHashThreads / 32 ? s_w[lane] : HashCarry{0, 0, 0};
+      for (int q = 0; q < 5; ++q) {
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if ((uint32_t)q < nv) v = __ldg(p + q);
+        wd[4 * q] = v.x;
+        wd[4 * q + 1] = v.y;
+        wd[4 * q + 2] = v.z;
+        wd[4 * q + 3] = v.w;
+      }
+    } else {
 #pragma unroll
-    for (int d = 1; d < 32; d <<= 1) {
-      HashCarry y;
-      y.v0 = __shfl_up_sync(kFull, z.v0, d);
-      y.v1 = __shfl_up_sync(kFull, z.v1, d);
-      y.f = __shfl_up_sync(kFull, z.f, d);
-      if (lane >= (uint32_t)d) z = op(y, z);
+      for (int q = 0; q < 20; ++q) wd[q] = x4 + q < a.n_tok ? a.tokens[x4 + q] : 0u;
     }
-    if (lane < kHashThreads / 32) s_w[lane] = z;  // inclusive over warps
-  }
-  __syncthreads();
-  if (w > 0) x = op(s_w[w - 1], x);
-  {
-    const HashCarry cin = lookback_cta(a.lb, tile, s_w[kHashThreads / 32 - 1], HashCarry{0, 0, 0}, op, kEpochHash,
-                                       a.st);
-    if (threadIdx.x == 0) s_carry = cin;
-  }
-  __syncthreads();
-  if (valid) {
-    if (!x.f) {
-      x.v0 = p61_add(x.v0, s_carry.v0);
-      x.v1 = p61_add(x.v1, s_carry.v1);
+    uint64_t acc[6] = {0, 0, 0, 0, 0, 0};
+    switch (m) {
+      case 0: hash16<0>(wd, c, acc); break;
+      case 1: hash16<1>(wd, c, acc); break;
+      case 2: hash16<2>(wd, c, acc); break;
+      default: hash16<3>(wd, c, acc); break;
     }
-    const uint64_t e = (uint64_t)kk + 1;
-    const uint64_t H0 = p61_mul(x.v0, pow_at(T + 0 * 65536, T + 2 * 65536, e));
-    const uint64_t H1 = p61_mul(x.v1, pow_at(T + 4 * 65536, T + 6 * 65536, e));
-    a.keys[b0 + t] = make_ulonglong2(H0, H1);
+    h0 = limbs_to_p61(acc[0], acc[1], acc[2]);
+    h1 = limbs_to_p61(acc[3], acc[4], acc[5]);
+    if (G > 1) {
+      const uint32_t q = G - 1 - s;
+      h0 = p61_mul(h0, c.sub_mul[0][q]);
+      h1 = p61_mul(h1, c.sub_mul[1][q]);
+    }
+  }
+  hash_finish<G>(a, tile, b0, b_end, h0, h1, k, lb, s);
+}
+
+// Carry of every tile = the segmented sum of the aggregates of the tiles
+// before it, back to (and including) the nearest one where a request starts.
+// All aggregates exist before this kernel starts, so nothing waits.  One warp
+// per tile: each round reads 32 predecessors; then the tile's leading blocks
+// (the tail of a request that started earlier) get the carry and their key.
+constexpr int kChainWarps = 8;
+__global__ void __launch_bounds__(kChainWarps * 32) k_hash_chain(ulonglong2* __restrict__ keys,
+                                                                 const HashCarry* __restrict__ tile_agg,
+                                                                 const uint32_t* __restrict__ tile_lead,
+                                                                 const uint32_t* __restrict__ tile_req,
+                                                                 const uint64_t* __restrict__ blk_off,
+                                                                 const uint64_t* tables, uint32_t TB,
+                                                                 const DevStatus* st, uint64_t keys_cap) {
+  const uint32_t lane = threadIdx.x & 31;
+  const uint32_t tile = blockIdx.x * kChainWarps + (threadIdx.x >> 5);
+  uint64_t N = st->value[0];
+  if (N > keys_cap) N = keys_cap;
+  const uint64_t b0 = (uint64_t)tile * TB;
+  if (b0 >= N || tile == 0) return;
+  const uint32_t lead = tile_lead[tile];
+  if (lead == 0) return;
+  uint64_t c0 = 0, c1 = 0;
+  for (int64_t base = (int64_t)tile - 1; base >= 0; base -= 32) {
+    const int64_t idx = base - (int64_t)lane;
+    HashCarry g{0, 0, 0};
+    if (idx >= 0) g = tile_agg[idx];
+    const uint32_t heads = __ballot_sync(kFull, idx >= 0 && g.f);
+    const uint32_t first = heads ? (uint32_t)(__ffs(heads) - 1) : 31u;
+    uint64_t v0 = lane <= first ? g.v0 : 0, v1 = lane <= first ? g.v1 : 0;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      v0 = p61_add(v0, __shfl_xor_sync(kFull, v0, o));
+      v1 = p61_add(v1, __shfl_xor_sync(kFull, v1, o));
+    }
+    c0 = p61_add(c0, v0);
+    c1 = p61_add(c1, v1);
+    if (heads) break;
+  }
+  const uint64_t kb = blk_off[tile_req[tile]];
+  for (uint32_t i = lane; i < lead; i += 32) {
+    const uint64_t b = b0 + i;
+    const ulonglong2 k = keys[b];
+    const uint64_t e = b - kb + 1;
+    const uint64_t H0 = p61_mul(p61_add(k.x, c0), pow_at(tables + 0 * 65536, tables + 2 * 65536, e));
+    const uint64_t H1 = p61_mul(p61_add(k.y, c1), pow_at(tables + 4 * 65536, tables + 6 * 65536, e));
+    keys[b] = make_ulonglong2(H0, H1);
   }
 }
 
 template <int G>
 void launch_hash(uint32_t grid, cudaStream_t s, const HashArgs& a, const HashConsts& c, bool full) {
-  if (full)
-    PTC_LAUNCH("k_hash", s, k_hash<G, true><<<grid, kHashThreads, 0, s>>>(a, c));
+  if (full && a.aligned)
+    PTC_LAUNCH("k_hash_local", s, k_hash_local_vec<G><<<grid, kHashThreads, 0, s>>>(a, c));
+  else if (full)
+    PTC_LAUNCH("k_hash_local", s, k_hash_local<G, true><<<grid, kHashThreads, 0, s>>>(a, c));
   else
-    PTC_LAUNCH("k_hash", s, k_hash<G, false><<<grid, kHashThreads, 0, s>>>(a, c));
+    PTC_LAUNCH("k_hash_local", s, k_hash_local<G, false><<<grid, kHashThreads, 0, s>>>(a, c));
 }
 
 uint32_t chunks_per_block(uint32_t B) {  // G: power of two >= ceil(B / 16)
@@ -406,9 +567,8 @@ uint32_t chunks_per_block(uint32_t B) {  // G: power of two >= ceil(B / 16)
 struct HashLayout {
   DevStatus* st;
   uint64_t* lb_off;
-  uint32_t* lb_hash_status;
-  HashCarry* lb_hash_agg;
-  HashCarry* lb_hash_incl;
+  HashCarry* tile_agg;
+  uint32_t* tile_lead;
   uint64_t* tables;
   uint32_t* tile_req;
   uint64_t hash_tiles;
@@ -425,10 +585,9 @@ HashLayout hash_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   const uint32_t hash_tiles = ceil_div_u32(nb, tb) + 1;
   L.st = cv.take<DevStatus>(1);
   L.lb_off = cv.take<uint64_t>(off_tiles);
-  L.lb_hash_status = cv.take<uint32_t>(hash_tiles);
   L.zero_bytes = cv.off;
-  L.lb_hash_agg = cv.take<HashCarry>(hash_tiles);
-  L.lb_hash_incl = cv.take<HashCarry>(hash_tiles);
+  L.tile_agg = cv.take<HashCarry>(hash_tiles);
+  L.tile_lead = cv.take<uint32_t>(hash_tiles);
   L.tables = cv.take<uint64_t>(8 * 65536);
   L.tile_req = cv.take<uint32_t>(hash_tiles + 1);
   L.hash_tiles = hash_tiles;
@@ -504,7 +663,8 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
   a.keys_cap = keys_cap;
   a.tables = L.tables;
   a.tile_req = L.tile_req;
-  a.lb = LbArrays<HashCarry>{L.lb_hash_status, L.lb_hash_agg, L.lb_hash_incl};
+  a.tile_agg = L.tile_agg;
+  a.tile_lead = L.tile_lead;
   a.st = L.st;
   a.aligned = (((uintptr_t)tokens) & 15) == 0;
   const bool full = block_size == 16 * G;
@@ -519,6 +679,9 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
       case 16: launch_hash<16>(grid, s, a, hc, full); break;
       default: launch_hash<32>(grid, s, a, hc, full); break;
     }
+    PTC_LAUNCH("k_hash_chain", s,
+               k_hash_chain<<<ceil_div_u32(grid, kChainWarps), kChainWarps * 32, 0, s>>>(a.keys, L.tile_agg, L.tile_lead, L.tile_req, req_blk_off_out,
+                                                 L.tables, kHashThreads / G, L.st, keys_cap));
   }
   DevStatus h;
   ptc_status rc = end_call(L.st, s, &h);
