@@ -19,16 +19,13 @@
 // values < 2^L.  Level l keeps one bit per position — bit (L-1-l) of the value
 // at that position in level l's order — and level l+1's order is the stable
 // partition of level l's order by that bit: its Z_l zeros, then its ones.
-// Level l's order is therefore the stable sort of v by its top l bits read
-// in reverse (the top bit least significant), so four levels are built per
-// pass from one LSD radix-16 step on the reversed 4-bit digit.
 //
 // Layout of one level: a plain bitvector (LSB first) plus a rank directory of
 // ones per 256-bit superblock (relative to its chunk of 256 superblocks) and
 // per chunk; a rank reads the superblock's 32-byte sector and two counts.
-//   k_wm_hist    per pass: tile histograms of the 4-bit key
-//   k_wm_scan    per pass: tile prefixes and totals of every key
-//   k_wm_pass    per pass: bits of 4 levels and the order after them
+//   k_wm_count0  level-0 zero counts of every tile and their prefixes
+//   k_wm_level   one level: ballot bits, stable partition by the bit (see
+//                the kernel's comment for how tile prefixes avoid waiting)
 //   k_wm_dir     rank directories of all levels
 //   k_wm_heads   run heads walk the L levels (early exit on an empty range)
 //                and write their distances; tiles record their last head.
@@ -40,95 +37,59 @@
 namespace ptc {
 namespace {
 
-constexpr int kWT = 256;                    // threads per tile
-constexpr int kWR = 8;                      // elements per thread
-constexpr int kWTile = kWT * kWR;           // 2048 positions per tile
-constexpr int kWW = kWT / 32;               // warps per tile
-constexpr int kWB = 4;                      // levels per pass
-constexpr int kOwners = 30;                 // (k, key) for k = 1..4: 2 + 4 + 8 + 16
-constexpr int kRegions = 14;                // (k, key) for k = 1..3
-constexpr int kRegionWords = kWTile / 32 + 1;
+constexpr int kLT = 256;                    // threads per tile
+constexpr int kLR = 8;                      // rounds (32 positions each) per warp
+constexpr int kLW = kLT / 32;               // warps per tile
+constexpr int kLTile = kLT * kLR;           // 2048 positions per tile; warp w owns [256 w, 256 w + 256)
 constexpr int kSbBits = 256;                // rank-directory superblock
 constexpr int kSbPerChunk = 256;
 constexpr int kQThreads = 256;
 constexpr int kQPer = 8;
 constexpr int kQTile = kQThreads * kQPer;
 
-// (k, key) pairs with k >= 1 numbered 2^k - 2 + key
-__device__ __forceinline__ uint32_t owner_of(uint32_t k, uint32_t key) { return (1u << k) - 2u + key; }
-
-struct PassArgs {
-  const uint32_t* src;        // this pass's input order (prev itself on pass 0)
-  int from_prev;              // values are prev + 1 (none -> 0)
-  uint32_t* dst;              // the order after this pass (null on the last pass)
-  uint32_t* bits;             // bitvectors, level l at bits + l * lw
-  uint64_t lw;
+struct LevelArgs {
+  const uint32_t* src;             // this level's order (prev itself at level 0)
+  int from_prev;                   // values are prev + 1 (none -> 0)
+  uint32_t* dst;                   // the next level's order (null at the last level)
+  uint32_t* bits;                  // this level's bitvector
   uint64_t n;
   uint32_t ntiles;
-  uint32_t lvl0, r, sh;       // first level, levels in the pass, shift of the digit
-  uint32_t* H;                // histogram of the pass key per tile, column-major [key][tile]
-  uint32_t* T;                // exclusive prefix of H over tiles, same layout
-  uint32_t* G;                // totals of the pass digit (16)
-  uint32_t* done;             // CTAs finished (histogram kernel)
-  unsigned long long* zcount; // Z_l for every level
+  uint32_t shift;                  // bit tested at this level
+  const uint32_t* tp;              // zeros before every tile of this level
+  const unsigned long long* zl;    // Z of this level
+  uint32_t* tz_next;               // zeros of every tile of the next level (accumulated here)
+  uint32_t* tp_next;               // ... their exclusive prefix (written by the last CTA)
+  unsigned long long* z_next;      // ... and their total, Z of the next level
+  uint32_t* done;                  // CTAs finished
   DevStatus* st;
 };
 
-__device__ __forceinline__ uint32_t load_v(const PassArgs& a, uint64_t j) {
+__device__ __forceinline__ uint32_t level_value(const LevelArgs& a, uint32_t j) {
   uint32_t x = a.src[j];
   if (a.from_prev) x = x == kNone ? 0u : x + 1u;
   return x;
 }
-// the r bits of levels lvl0 .. lvl0 + r - 1, reversed: bit k of the key is the
-// bit of level lvl0 + k
-__device__ __forceinline__ uint32_t key_of(uint32_t v, uint32_t sh, uint32_t r) {
-  return __brev((v >> sh) & ((1u << r) - 1u)) >> (32 - r);
-}
 
-// Histogram of the pass keys per tile, stored column-major: H[key * ntiles + tile].
-__global__ void __launch_bounds__(kWT) k_wm_hist(PassArgs a) {
-  __shared__ uint32_t s_h[16];
-  const uint32_t t = threadIdx.x, lane = t & 31;
-  const uint64_t base = (uint64_t)blockIdx.x * kWTile;
-  if (t < 16) s_h[t] = 0;
+// Run by every thread of the CTA that finished last (threadfence-reduction
+// pattern): tp[i] = tz[0] + ... + tz[i-1] for i < ntiles and *total = sum.
+// Each thread takes a contiguous run; loads bypass L1 (other CTAs' atomics).
+__device__ inline void finish_counts(uint32_t* done, const uint32_t* tz, uint32_t* tp, uint32_t ntiles,
+                                     unsigned long long* total) {
+  __shared__ bool s_last;
+  __shared__ uint32_t s_w[kLT / 32];
   __syncthreads();
-  bool bad = false;
-#pragma unroll
-  for (int rd = 0; rd < kWR; ++rd) {
-    const uint64_t j = base + (uint64_t)rd * kWT + t;
-    const bool valid = j < a.n;
-    uint32_t key = 0xFFFFu;
-    if (valid) {
-      if (a.from_prev) {
-        const uint32_t p = a.src[j];
-        if (p != kNone && (uint64_t)p >= j) bad = true;
-      }
-      key = key_of(load_v(a, j), a.sh, a.r);
-    }
-    const uint32_t peers = __match_any_sync(kFull, key);
-    if (valid && lane == (uint32_t)(__ffs(peers) - 1)) atomicAdd(&s_h[key], (uint32_t)__popc(peers));
+  if (threadIdx.x == 0) {
+    __threadfence();
+    s_last = atomicAdd(done, 1u) == gridDim.x - 1;
   }
-  if (bad) raise_err(a.st, kErrInvalid);
   __syncthreads();
-  if (t < 16) a.H[(uint64_t)t * a.ntiles + blockIdx.x] = s_h[t];
-}
-
-// One CTA per key: exclusive prefix of its histogram column over tiles, and
-// the key's total.  Each thread takes a contiguous run of tiles.
-constexpr int kScanThreads = 1024;
-__global__ void __launch_bounds__(kScanThreads) k_wm_scan(PassArgs a) {
-  __shared__ uint32_t s_w[kScanThreads / 32];
-  const uint32_t key = blockIdx.x, t = threadIdx.x, lane = t & 31, w = t >> 5;
-  if (key >= (1u << a.r)) {
-    if (t == 0) a.G[key] = 0;
-    return;
-  }
-  const uint32_t* col = a.H + (uint64_t)key * a.ntiles;
-  uint32_t* out = a.T + (uint64_t)key * a.ntiles;
-  const uint32_t per = (a.ntiles + kScanThreads - 1) / kScanThreads;
-  const uint32_t lo = t * per < a.ntiles ? t * per : a.ntiles, hi = lo + per < a.ntiles ? lo + per : a.ntiles;
+  if (!s_last) return;
+  __threadfence();
+  const uint32_t t = threadIdx.x, lane = t & 31, w = t >> 5;
+  const uint32_t per = (ntiles + kLT - 1) / kLT;
+  const uint32_t lo = t * per < ntiles ? t * per : ntiles, hi = lo + per < ntiles ? lo + per : ntiles;
   uint32_t sum = 0;
-  for (uint32_t i = lo; i < hi; ++i) sum += col[i];
+  for (uint32_t i = lo; i < hi; ++i) sum += __ldcg(&tz[i]);
   uint32_t x = sum;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
@@ -138,191 +99,142 @@ __global__ void __launch_bounds__(kScanThreads) k_wm_scan(PassArgs a) {
   if (lane == 31) s_w[w] = x;
   __syncthreads();
   uint32_t wpre = 0, tot = 0;
-#pragma unroll 4
-  for (int k = 0; k < kScanThreads / 32; ++k) {
+#pragma unroll
+  for (int k = 0; k < kLT / 32; ++k) {
     wpre += k < (int)w ? s_w[k] : 0u;
     tot += s_w[k];
   }
   uint32_t run = wpre + x - sum;
   for (uint32_t i = lo; i < hi; ++i) {
-    out[i] = run;
-    run += col[i];
+    tp[i] = run;
+    run += __ldcg(&tz[i]);
   }
-  if (t == 0) a.G[key] = tot;
+  if (t == 0) *total = tot;
 }
 
-// One pass = r levels.  Positions at level lvl0 + k are the stable order by
-// the low k bits of the key (the level lvl0 bit least significant), so a tile
-// of this pass's order lands, at level lvl0 + k, in 2^k runs (one per key),
-// each contiguous.  Level lvl0's bits are ballots in place; the bits of levels
-// lvl0 + 1 .. lvl0 + r - 1 are assembled per run in shared memory and written
-// at the runs' global bit offsets (whole words stored, words shared with a
-// neighbouring run OR-ed); the order after the pass is an LSD radix-2^r
-// scatter by the full key.
-__global__ void __launch_bounds__(kWT) k_wm_pass(PassArgs a) {
-  __shared__ uint32_t s_reg[kRegions][kRegionWords];
-  __shared__ uint32_t s_vals[kWTile];
-  __shared__ uint32_t s_cnt[kWW][32];
-  __shared__ uint32_t s_tot[32];
-  __shared__ uint32_t s_run[32];
-  __shared__ uint32_t s_lst[16];
-  __shared__ uint32_t s_G[16], s_T[16];
+// Level-0 zero count of every tile (bit L-1 of v = prev + 1), Z_0 and the
+// tile prefixes; also checks prev[j] < j.
+__global__ void __launch_bounds__(kLT) k_wm_count0(LevelArgs a) {
+  __shared__ uint32_t s_wz[kLW];
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const uint32_t n32 = (uint32_t)a.n;
+  const uint32_t wbase = blockIdx.x * kLTile + w * 256;
+  uint32_t zc = 0;
+  bool bad = false;
+#pragma unroll
+  for (int rd = 0; rd < kLR; ++rd) {
+    const uint32_t j = wbase + rd * 32 + lane;
+    bool zero = false;
+    if (j < n32) {
+      const uint32_t p = a.src[j];
+      if (p != kNone && p >= j) bad = true;
+      const uint32_t v = p == kNone ? 0u : p + 1u;
+      zero = !((v >> a.shift) & 1u);
+    }
+    zc += __popc(__ballot_sync(kFull, zero));
+  }
+  if (bad) raise_err(a.st, kErrInvalid);
+  if (lane == 0) s_wz[w] = zc;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t z = 0;
+    for (int k = 0; k < kLW; ++k) z += s_wz[k];
+    a.tz_next[blockIdx.x] = z;
+  }
+  finish_counts(a.done, a.tz_next, a.tp_next, a.ntiles, a.z_next);
+}
+
+// One level.  Each warp owns 256 consecutive positions (8 rounds of 32):
+// ballot of the level bit -> bitvector word; stable partition -> the zeros go
+// to [zeros before, ...), the ones to Z + [ones before, ...).  The tile's
+// prefix comes from the previous level (no waiting).  Every element counts
+// itself, in a packed per-lane counter, into the next level's tile it lands
+// in (the zeros and the ones of a tile each meet at most two such tiles); the
+// CTA that finishes last turns those counts into the next level's prefixes.
+__global__ void __launch_bounds__(kLT) k_wm_level(LevelArgs a) {
+  __shared__ uint32_t s_wz[kLW];
+  __shared__ uint32_t s_cnt[kLW][4];
   const uint32_t t = threadIdx.x, lane = t & 31, w = t >> 5;
-  const uint32_t r = a.r;
-  const uint32_t nown = (2u << r) - 2u;       // owners with k = 1..r
-  const uint32_t nreg = r > 1 ? (2u << (r - 1)) - 2u : 0u;  // regions with k = 1..r-1
+  const uint32_t n32 = (uint32_t)a.n;
   const uint32_t tile = blockIdx.x;
-  const uint64_t base = (uint64_t)tile * kWTile;
-  for (uint32_t i = t; i < kRegions * kRegionWords; i += kWT) (&s_reg[0][0])[i] = 0;
-  if (t < 16) {
-    s_G[t] = a.G[t];
-    s_T[t] = t < (1u << r) ? a.T[(uint64_t)t * a.ntiles + tile] : 0u;
-  }
-  uint32_t v[kWR];
+  const uint32_t wbase = tile * kLTile + w * 256;
+  uint32_t v[kLR];
 #pragma unroll
-  for (int rd = 0; rd < kWR; ++rd) {
-    const uint64_t j = base + (uint64_t)w * (32 * kWR) + (uint64_t)rd * 32 + lane;
-    v[rd] = j < a.n ? load_v(a, j) : 0u;
+  for (int rd = 0; rd < kLR; ++rd) {
+    const uint32_t j = wbase + rd * 32 + lane;
+    v[rd] = j < n32 ? level_value(a, j) : 0u;
   }
-  // this lane's (k, key) when it is an owner
-  const bool own = lane < nown;
-  uint32_t ok = 1, oc = 0;
-  if (own) {
-    while ((2u << ok) - 2u <= lane) ++ok;
-    oc = lane - ((1u << ok) - 2u);
+  const bool tail = wbase + 256 > n32;
+  uint32_t m[kLR];
+  uint32_t zc = 0;
+#pragma unroll
+  for (int rd = 0; rd < kLR; ++rd) {
+    const uint32_t vm = tail ? __ballot_sync(kFull, wbase + rd * 32 + lane < n32) : kFull;
+    m[rd] = __ballot_sync(kFull, (v[rd] >> a.shift) & 1u) & vm;
+    zc += __popc(vm & ~m[rd]);
+    if (lane == 0 && (vm & 1u)) a.bits[(wbase + rd * 32) >> 5] = m[rd];
   }
-  // ---- phase A: per-warp counts of every (k, key)
-  uint32_t cnt = 0;
-  uint32_t* bits0 = a.bits + (uint64_t)a.lvl0 * a.lw;
-#pragma unroll
-  for (int rd = 0; rd < kWR; ++rd) {
-    const uint64_t j = base + (uint64_t)w * (32 * kWR) + (uint64_t)rd * 32 + lane;
-    const uint32_t vm = __ballot_sync(kFull, j < a.n);
-    const uint32_t key = key_of(v[rd], a.sh, r);
-    uint32_t B[kWB];
-#pragma unroll
-    for (int i = 0; i < kWB; ++i) B[i] = (uint32_t)i < r ? __ballot_sync(kFull, (key >> i) & 1u) : 0u;
-    if (lane == 0 && (vm & 1u)) bits0[(base + (uint64_t)w * (32 * kWR) + (uint64_t)rd * 32) >> 5] = B[0] & vm;
-    if (own) {
-      uint32_t m = vm;
-#pragma unroll
-      for (int i = 0; i < kWB; ++i)
-        if ((uint32_t)i < ok) m &= ((oc >> i) & 1u) ? B[i] : ~B[i];
-      cnt += __popc(m);
-    }
-  }
-  if (own) s_cnt[w][lane] = cnt;
+  if (lane == 0) s_wz[w] = zc;
   __syncthreads();
-  if (tile == 0 && t < r) {  // zeros of level lvl0 + t: keys whose bit t is 0
-    uint64_t z = 0;
-    for (uint32_t key = 0; key < (1u << r); ++key)
-      if (!((key >> t) & 1u)) z += s_G[key];
-    a.zcount[a.lvl0 + t] = z;
+  uint32_t wp = 0, tzt = 0;
+#pragma unroll
+  for (int k = 0; k < kLW; ++k) {
+    const uint32_t z = s_wz[k];
+    wp += k < (int)w ? z : 0u;
+    tzt += z;
   }
-  if (t < nown) {  // warp prefixes and tile totals
-    uint32_t acc = 0;
-    for (int ww = 0; ww < kWW; ++ww) {
-      const uint32_t x = s_cnt[ww][t];
-      s_cnt[ww][t] = acc;
-      acc += x;
-    }
-    s_tot[t] = acc;
+  const uint32_t tile_base = a.tp[tile];
+  const uint32_t Z = (uint32_t)*a.zl;
+  if (t == 0) {  // the published count must match the data
+    const uint32_t next = tile + 1 < a.ntiles ? a.tp[tile + 1] : Z;
+    if (next - tile_base != tzt) raise_err(a.st, kErrInvalid);
   }
-  __syncthreads();
-  if (t < nown) {  // global start of every run at level lvl0 + k
-    uint32_t k = 1;
-    while ((2u << k) - 2u <= t) ++k;
-    const uint32_t c = t - ((1u << k) - 2u), msk = (1u << k) - 1u;
-    uint32_t off = 0, pre = 0;
-    for (uint32_t key = 0; key < (1u << r); ++key) {
-      if ((key & msk) < c) off += s_G[key];
-      if ((key & msk) == c) pre += s_T[key];
-    }
-    s_run[t] = off + pre;
-    if (k == r) {  // local start of the final key group
-      uint32_t ls = 0;
-      for (uint32_t c2 = 0; c2 < c; ++c2) ls += s_tot[owner_of(r, c2)];
-      s_lst[c] = ls;
-    }
-  }
-  __syncthreads();
-  // ---- phase B: ranks; bits of the middle levels into shared runs; reorder
-  cnt = 0;
+  if (a.dst == nullptr) return;
+  uint32_t zb = tile_base + wp;     // zeros before this warp's first position
+  uint32_t ob = wbase - zb;         // ones before it
+  const uint32_t SZ = (tile_base / kLTile + 1) * kLTile;
+  const uint32_t SO = ((Z + tile * kLTile - tile_base) / kLTile + 1) * kLTile;
+  const uint32_t nshift = a.shift - 1;
   const uint32_t lt = lanemask_lt();
+  uint32_t cz = 0, co = 0;  // (early count) | (late count) << 16, for landing zeros / ones
 #pragma unroll
-  for (int rd = 0; rd < kWR; ++rd) {
-    const uint64_t j = base + (uint64_t)w * (32 * kWR) + (uint64_t)rd * 32 + lane;
-    const bool valid = j < a.n;
-    const uint32_t vm = __ballot_sync(kFull, valid);
-    const uint32_t key = key_of(v[rd], a.sh, r);
-    uint32_t B[kWB];
+  for (int rd = 0; rd < kLR; ++rd) {
+    const uint32_t vm = tail ? __ballot_sync(kFull, wbase + rd * 32 + lane < n32) : kFull;
+    const uint32_t mz = vm & ~m[rd];
+    const uint32_t r0 = __popc(mz & lt);
+    const bool one = (m[rd] >> lane) & 1u;
+    const uint32_t dst = one ? Z + ob + (lane - r0) : zb + r0;
+    const bool valid = (vm >> lane) & 1u;
+    if (valid && dst < n32) a.dst[dst] = v[rd];
+    const uint32_t inc = (valid && !((v[rd] >> nshift) & 1u)) ? (dst < (one ? SO : SZ) ? 1u : 0x10000u) : 0u;
+    if (one)
+      co += inc;
+    else
+      cz += inc;
+    zb += __popc(mz);
+    ob += __popc(m[rd]);
+  }
 #pragma unroll
-    for (int i = 0; i < kWB; ++i) B[i] = (uint32_t)i < r ? __ballot_sync(kFull, (key >> i) & 1u) : 0u;
-    uint32_t eq = vm;
-#pragma unroll
-    for (int k = 1; k <= kWB; ++k) {
-      if ((uint32_t)k > r) break;
-      eq &= ((key >> (k - 1)) & 1u) ? B[k - 1] : ~B[k - 1];
-      const uint32_t kk = key & ((1u << k) - 1u);
-      const uint32_t o = owner_of(k, kk);
-      const uint32_t before = __shfl_sync(kFull, cnt, o);
-      const uint32_t rank = s_cnt[w][o] + before + __popc(eq & lt);
-      if (valid) {
-        if ((uint32_t)k < r) {
-          if ((key >> k) & 1u) atomicOr(&s_reg[o][rank >> 5], 1u << (rank & 31));
-        } else {
-          s_vals[s_lst[kk] + rank] = v[rd];
-        }
-      }
-    }
-    if (own) {
-      uint32_t m = vm;
-#pragma unroll
-      for (int i = 0; i < kWB; ++i)
-        if ((uint32_t)i < ok) m &= ((oc >> i) & 1u) ? B[i] : ~B[i];
-      cnt += __popc(m);
-    }
+  for (int o = 16; o > 0; o >>= 1) {
+    cz += __shfl_xor_sync(kFull, cz, o);
+    co += __shfl_xor_sync(kFull, co, o);
+  }
+  if (lane == 0) {
+    s_cnt[w][0] = cz & 0xFFFFu;
+    s_cnt[w][1] = cz >> 16;
+    s_cnt[w][2] = co & 0xFFFFu;
+    s_cnt[w][3] = co >> 16;
   }
   __syncthreads();
-  // ---- the order after this pass
-  const uint32_t tile_n = (uint32_t)(a.n - base < (uint64_t)kWTile ? a.n - base : kWTile);
-  if (a.dst != nullptr) {
-    for (uint32_t p = t; p < tile_n; p += kWT) {
-      const uint32_t x = s_vals[p];
-      const uint32_t key = key_of(x, a.sh, r);
-      const uint32_t d = s_run[owner_of(r, key)] + (p - s_lst[key]);
-      if ((uint64_t)d < a.n) a.dst[d] = x;  // in range on a well-formed input
+  if (t < 4) {
+    uint32_t c = 0;
+    for (int k = 0; k < kLW; ++k) c += s_cnt[k][t];
+    if (c) {
+      const uint32_t dt = t < 2 ? SZ / kLTile - (t == 0 ? 1u : 0u) : SO / kLTile - (t == 2 ? 1u : 0u);
+      if (dt < a.ntiles) atomicAdd(&a.tz_next[dt], c);
     }
   }
-  // ---- bit runs of levels lvl0 + 1 .. lvl0 + r - 1
-  for (uint32_t rg = 0; rg < nreg; ++rg) {
-    const uint32_t C = s_tot[rg];
-    if (C == 0) continue;
-    uint32_t k = 1;
-    while ((2u << k) - 2u <= rg) ++k;
-    const uint64_t S = s_run[rg];
-    const uint64_t g0 = S >> 5, g1 = (S + C - 1) >> 5;
-    uint32_t* lvl = a.bits + (uint64_t)(a.lvl0 + k) * a.lw;
-    for (uint64_t g = g0 + t; g <= g1; g += kWT) {
-      const int64_t q = (int64_t)(g * 32) - (int64_t)S;  // run offset of this word's bit 0
-      uint32_t x;
-      if (q < 0) {
-        x = s_reg[rg][0] << (uint32_t)(-q);
-      } else {
-        const uint32_t w0 = (uint32_t)(q >> 5), sft = (uint32_t)(q & 31);
-        x = s_reg[rg][w0] >> sft;
-        if (sft) x |= s_reg[rg][w0 + 1] << (32 - sft);
-      }
-      const int64_t blo = q < 0 ? -q : 0, bhi = (int64_t)C - q < 32 ? (int64_t)C - q : 32;
-      const uint32_t mask = (bhi >= 32 ? 0xFFFFFFFFu : ((1u << bhi) - 1u)) & ~((1u << blo) - 1u);
-      x &= mask;
-      if (mask == 0xFFFFFFFFu) {
-        if (x) lvl[g] = x;
-      } else if (x) {
-        atomicOr(&lvl[g], x);
-      }
-    }
-  }
+  finish_counts(a.done, a.tz_next, a.tp_next, a.ntiles, a.z_next);
 }
 
 // Rank directory of every level: dir[l][sb] = ones in the superblocks of its
@@ -598,9 +510,8 @@ struct WmLayout {
   DevStatus* st;
   unsigned long long* zcount;
   uint32_t* done;
-  uint32_t* G;
-  uint32_t* H;
-  uint32_t* T;
+  uint32_t* tz;   // L x ntiles
+  uint32_t* tp;   // L x ntiles
   uint32_t* csum;
   uint32_t* cpre;
   uint32_t* dir;
@@ -609,7 +520,7 @@ struct WmLayout {
   uint32_t *va, *vb;
   uint32_t* bits;
   uint64_t lw;
-  uint32_t L, ntiles, nsb, nchunk, passes;
+  uint32_t L, ntiles, nsb, nchunk;
   size_t zero_bytes;
   size_t total;
 };
@@ -618,8 +529,7 @@ WmLayout wm_layout(void* ws, uint64_t n) {
   WmLayout W;
   Carver cv(ws);
   W.L = value_bits(n);
-  W.passes = (W.L + kWB - 1) / kWB;
-  W.ntiles = ceil_div_u32(n, kWTile) + 1;
+  W.ntiles = ceil_div_u32(n, kLTile);
   W.nsb = (uint32_t)(n / kSbBits) + 1;
   W.nchunk = ceil_div_u32(W.nsb, kSbPerChunk);
   W.lw = (uint64_t)W.nsb * 8 + 8;
@@ -628,10 +538,9 @@ WmLayout wm_layout(void* ws, uint64_t n) {
   W.st = cv.take<DevStatus>(1);
   W.zcount = cv.take<unsigned long long>(40);
   W.done = cv.take<uint32_t>(64);
+  W.tz = cv.take<uint32_t>((uint64_t)W.L * (W.ntiles + 1));
   W.zero_bytes = cv.off;
-  W.G = cv.take<uint32_t>((uint64_t)W.passes * 16);
-  W.H = cv.take<uint32_t>((uint64_t)W.ntiles * 16);
-  W.T = cv.take<uint32_t>((uint64_t)W.ntiles * 16);
+  W.tp = cv.take<uint32_t>((uint64_t)W.L * (W.ntiles + 1));
   W.csum = cv.take<uint32_t>((uint64_t)W.L * W.nchunk);
   W.cpre = cv.take<uint32_t>((uint64_t)W.L * W.nchunk);
   W.dir = cv.take<uint32_t>((uint64_t)W.L * W.nsb);
@@ -661,31 +570,38 @@ extern "C" ptc_status ptc_stack_distance(const uint32_t* prev, uint64_t n, uint3
   const WmLayout W = wm_layout(ws, n);
   if (begin_call(ws, W.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
   if (cudaMemsetAsync(W.bits, 0, sizeof(uint32_t) * (uint64_t)W.L * W.lw, s) != cudaSuccess) return PTC_ERR_CUDA;
-  const uint32_t tiles = ceil_div_u32(n, kWTile);
-  const uint32_t* src = prev;
+  const uint32_t tiles = W.ntiles;
+  LevelArgs a;
+  a.src = prev;
+  a.from_prev = 1;
+  a.dst = nullptr;
+  a.bits = nullptr;
+  a.n = n;
+  a.ntiles = tiles;
+  a.shift = W.L - 1;
+  a.tp = nullptr;
+  a.zl = nullptr;
+  a.tz_next = W.tz;
+  a.tp_next = W.tp;
+  a.z_next = &W.zcount[0];
+  a.done = &W.done[62];
+  a.st = W.st;
+  PTC_LAUNCH("k_wm_count0", s, k_wm_count0<<<tiles, kLT, 0, s>>>(a));
   uint32_t* bufs[2] = {W.va, W.vb};
-  for (uint32_t pi = 0; pi < W.passes; ++pi) {
-    PassArgs a;
-    a.r = W.L - kWB * pi < (uint32_t)kWB ? W.L - kWB * pi : (uint32_t)kWB;
-    a.lvl0 = kWB * pi;
-    a.sh = W.L - a.lvl0 - a.r;
-    a.src = src;
-    a.from_prev = pi == 0;
-    a.dst = pi + 1 < W.passes ? bufs[pi & 1] : nullptr;
-    a.bits = W.bits;
-    a.lw = W.lw;
-    a.n = n;
-    a.ntiles = tiles;
-    a.H = W.H;
-    a.T = W.T;
-    a.G = W.G + 16 * pi;
-    a.done = &W.done[pi];
-    a.zcount = W.zcount;
-    a.st = W.st;
-    PTC_LAUNCH("k_wm_hist", s, k_wm_hist<<<tiles, kWT, 0, s>>>(a));
-    PTC_LAUNCH("k_wm_scan", s, k_wm_scan<<<16, kScanThreads, 0, s>>>(a));
-    PTC_LAUNCH("k_wm_pass", s, k_wm_pass<<<tiles, kWT, 0, s>>>(a));
-    src = a.dst;
+  for (uint32_t l = 0; l < W.L; ++l) {
+    const bool last = l + 1 == W.L;
+    a.src = l == 0 ? prev : bufs[(l + 1) & 1];
+    a.from_prev = l == 0;
+    a.dst = last ? nullptr : bufs[l & 1];
+    a.bits = W.bits + (uint64_t)l * W.lw;
+    a.shift = W.L - 1 - l;
+    a.tp = W.tp + (uint64_t)l * (tiles + 1);
+    a.zl = &W.zcount[l];
+    a.tz_next = last ? nullptr : W.tz + (uint64_t)(l + 1) * (tiles + 1);
+    a.tp_next = last ? nullptr : W.tp + (uint64_t)(l + 1) * (tiles + 1);
+    a.z_next = last ? nullptr : &W.zcount[l + 1];
+    a.done = &W.done[l];
+    PTC_LAUNCH("k_wm_level", s, k_wm_level<<<tiles, kLT, 0, s>>>(a));
   }
   PTC_LAUNCH("k_wm_dir", s,
              k_wm_dir<<<W.L * W.nchunk, kSbPerChunk, 0, s>>>(W.bits, W.lw, W.L, W.nsb, W.nchunk, W.dir, W.csum, W.cpre,
