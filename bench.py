@@ -1,8 +1,8 @@
 #!/usr/bin/env python3
 """Benchmark: request trace -> all-capacity LRU hit and compute-saved curves.
 
-One step is the whole path — ptc_hash_blocks, ptc_assign_ids,
-ptc_reuse_indices, ptc_stack_distance, ptc_curves — over one synthetic trace
+One step is the whole path — block hashing, dense ids, reuse indices, stack
+distances, curves — in one ptc_pipeline call over one synthetic trace
 resident in HBM: the conversational chat workload (~154M tokens, ~9.6M block
 accesses, 16-token blocks, 64 log-spaced capacities from 64 blocks to all
 distinct blocks, measured-shape cost model).  The metric is trace tokens per
@@ -14,6 +14,8 @@ of the HBM roofline for the path's stage-byte model.
 Timing: W untimed warm-up steps, then K steps, each bracketed by CUDA events
 on the launching stream, with a 256 MiB write between steps to flush L2
 (outside the events); barrier + synchronize on both sides; max over ranks.
+Per-kernel durations (for the roofline of the dominant kernel) come from a
+second pass of K steps with events around every launch.
 With N > 1 (torchrun) every rank runs an independent replica (the path has
 no cross-GPU exchange): value = tokens of all replicas / slowest rank's time.
 
@@ -102,26 +104,34 @@ def stage_model_bytes(T, N):
 
 
 def kernel_model_bytes(name, T, N, L):
-    """Algorithmic bytes one launch of `name` must move (0: not in the model)."""
+    """Algorithmic bytes one launch of `name` moves under the stage-byte model
+    (0: the kernel only touches scratch the model does not count)."""
     per_level = ((L - 1) * 8.125 + 4.125) / L * N  # the last level writes no partition
     return {
-        "k_hash": 4 * T + 16 * N,
-        "k_ids_insert": 16 * N,
-        "k_ids_gather": 4 * N,
-        "k_adjacent": 8 * N,
-        "k_sort_hist": 4 * N,
-        "k_wm_level": per_level,
-        "k_wm_query": (8 + L / 8) * N,
-        "k_curves": 4 * N,
+        "k_hash_local": 4 * T + 16 * N,   # token stream in, block keys out
+        "k_ids_insert": 16 * N,           # keys in
+        "k_ids_gather": 4 * N,            # ids out
+        "k_sort_hist": 4 * N,             # ids in
+        "k_adjacent": 8 * N,              # prev / next out
+        "k_wm_level": per_level,          # values in, partition + bit plane out
+        "k_wm_heads": (8 + L / 8) * N,    # prev in, one read of the bit planes, distances out
+        "k_curves": 4 * N,                # distances in
     }.get(name, 0.0)
 
 
+KERNEL_SOURCE = {
+    "k_block_offsets": "ptc_hash.cu", "k_pow_tables": "ptc_hash.cu", "k_hash_local": "ptc_hash.cu",
+    "k_hash_chain": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu", "k_ids_rank": "ptc_ids.cu",
+    "k_ids_gather": "ptc_ids.cu", "k_sort_hist": "ptc_sort.cu", "k_sort_offsets": "ptc_sort.cu",
+    "k_sort_pass": "ptc_sort.cu", "k_adjacent": "ptc_sort.cu", "k_wm_count0": "ptc_wavelet.cu",
+    "k_wm_level": "ptc_wavelet.cu", "k_wm_dir": "ptc_wavelet.cu", "k_wm_heads": "ptc_wavelet.cu",
+    "k_wm_propagate": "ptc_wavelet.cu", "k_heads": "ptc_curves.cu", "k_curves_agg": "ptc_curves.cu",
+    "k_curves": "ptc_curves.cu", "k_finalize": "ptc_curves.cu",
+}
+
+
 def source_sha(kernel):
-    files = {"k_hash": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu", "k_ids_rank": "ptc_ids.cu",
-             "k_ids_gather": "ptc_ids.cu", "k_sort_pass": "ptc_sort.cu", "k_adjacent": "ptc_sort.cu",
-             "k_sort_hist": "ptc_sort.cu", "k_wm_level": "ptc_wavelet.cu", "k_wm_query": "ptc_wavelet.cu",
-             "k_wm_zeros": "ptc_wavelet.cu", "k_curves": "ptc_curves.cu"}
-    f = files.get(kernel)
+    f = KERNEL_SOURCE.get(kernel)
     if f is None:
         return None
     with open(os.path.join(ROOT, "paper_2609_28870_gb300", "csrc", f), "rb") as fh:
@@ -212,64 +222,69 @@ def run_ours(args, ws_world, rank, local):
     off = off_host.to(dev, non_blocking=True)
     ts = ts_host.to(dev, non_blocking=True)
     torch.cuda.synchronize(dev)
-    ws = torch.empty(ptc.workspace_bytes(tr.n_req, T, BLOCK, n_cap=64), dtype=torch.uint8, device=dev)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
-    caps_for = lambda d: tracegen.workload_grid(WORKLOAD, d)
+    # the capacity grid spans 64 blocks .. D; D is a property of the trace, taken once before timing
+    ws_probe = torch.empty(ptc.workspace_bytes(tr.n_req, T, BLOCK, n_cap=64), dtype=torch.uint8, device=dev)
+    D = ptc.pipeline(tok, off, ts, BLOCK, lambda d: [1], ws=ws_probe, keep=False)["n_distinct"]
+    del ws_probe
+    caps = tracegen.workload_grid(WORKLOAD, D)
+    G = len(caps)
+    ws = torch.empty(L.ptc_pipeline_workspace_bytes(tr.n_req, T, BLOCK, G), dtype=torch.uint8, device=dev)
 
-    def step():
-        return ptc.pipeline(tok, off, ts, BLOCK, caps_for, kind=ptc.PTC_COST_MEASURED, seed=0, ws=ws, keep=False)
+    def step(t, o, s):
+        return ptc.ptc_pipeline(t, o, s, BLOCK, caps, kind=ptc.PTC_COST_MEASURED, seed=0, ws=ws)
 
     for _ in range(max(args.warmup, 0)):
-        out = step()
-    N, D = out["n_access"], out["n_distinct"]
+        out = step(tok, off, ts)
+    N = out["n_access"]
     stream = torch.cuda.current_stream(dev)
 
+    def timed(k_steps, body):
+        ms = []
+        for k in range(k_steps):
+            flush.fill_(k & 0xFF)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            r = body()
+            e1.record(stream)
+            e1.synchronize()
+            ms.append(e0.elapsed_time(e1))
+            assert r["hits"] == out["hits"] and r["saved"] == out["saved"]
+        return ms
+
     # ---- timed region (inputs resident in HBM)
-    L.ptc_timer_reset()
-    L.ptc_timer_enable(1)
     clocks = Clocks(local)
     barrier()
     torch.cuda.synchronize(dev)
     clocks.start()
     launches0 = L.ptc_launch_count()
-    step_ms = []
-    for k in range(args.steps):
-        flush.fill_(k & 0xFF)
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        out = step()
-        e1.record(stream)
-        e1.synchronize()
-        step_ms.append(e0.elapsed_time(e1))
+    step_ms = timed(args.steps, lambda: step(tok, off, ts))
     torch.cuda.synchronize(dev)
     launches = L.ptc_launch_count() - launches0
     barrier()
     clk = clocks.stop()
-    L.ptc_timer_enable(0)
-    ktimes = read_timer(ptc)
     total_ms = max_over_ranks(sum(step_ms))
     ms_per_step = total_ms / args.steps
 
+    # ---- per-kernel durations: the same K steps again with CUDA events
+    # around every launch on the launch stream (the events slow a step, so
+    # this pass is separate from the timed one)
+    L.ptc_timer_reset()
+    L.ptc_timer_enable(1)
+    inst_ms = timed(args.steps, lambda: step(tok, off, ts))
+    L.ptc_timer_enable(0)
+    ktimes = read_timer(ptc)
+
     # ---- end to end through the public API from pinned host memory
-    e2e_ms = []
-    for k in range(args.steps):
-        flush.fill_(k & 0xFF)
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
+    def e2e_body():
         tok2 = tok_host.to(dev, non_blocking=True)
         off2 = off_host.to(dev, non_blocking=True)
         ts2 = ts_host.to(dev, non_blocking=True)
-        o2 = ptc.pipeline(tok2, off2, ts2, BLOCK, caps_for, kind=ptc.PTC_COST_MEASURED, seed=0, ws=ws, keep=False)
-        e1.record(stream)
-        e1.synchronize()
-        e2e_ms.append(e0.elapsed_time(e1))
-        del tok2, off2, ts2
-    e2e_total = max_over_ranks(sum(e2e_ms))
-    assert o2["hits"] == out["hits"] and o2["saved"] == out["saved"]
+        return step(tok2, off2, ts2)
+
+    e2e_total = max_over_ranks(sum(timed(args.steps, e2e_body)))
     h2d = 4 * T + 8 * (tr.n_req + 1) + 8 * tr.n_req
-    G = len(out["hits"])
     d2h = 8 * G + 16 * G + 16 + 8 + 8  # hits, saved (u128), total cost, N, D
 
     # ---- roofline
@@ -313,6 +328,8 @@ def run_ours(args, ws_world, rank, local):
                          "stages_bytes": stages},
         "roofline": roof,
         "kernels": [{k: (round(v, 5) if isinstance(v, float) else v) for k, v in x.items()} for x in kernels],
+        "kernel_timing": {"how": "separate pass of the same K steps with CUDA events around every launch",
+                          "ms_per_step": round(sum(inst_ms) / len(inst_ms), 4)},
         "e2e": {"value": round(e2e_value, 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_total / args.steps, 4)},
         "gpu_launches": launches,

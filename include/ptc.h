@@ -204,6 +204,29 @@ ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_
                       size_t ws_bytes, void* stream);
 
 /*
+ * ptc_pipeline — the five calls in order (hash, ids, reuse, stack distance,
+ * curves) in one call, for a trace already on the device.  Semantics, limits
+ * and errors are those of the individual calls; the first error stops the
+ * pipeline and is returned.
+ *   keys_out, req_blk_off_out, ids_out, prev_out, next_out, dist_out
+ *       optional device outputs (NULL: kept in the workspace and discarded);
+ *       sizes as for the individual calls, keys_out at least
+ *       floor(n_tok / block_size) entries
+ *   cap_host, n_cap, cm, hits/saved/total outputs  as for ptc_curves
+ *   n_access_host_out, n_distinct_host_out        N and D on the host
+ * The workspace holds the intermediate arrays not supplied plus the largest
+ * scratch of any stage (ptc_pipeline_workspace_bytes).
+ */
+size_t ptc_pipeline_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size, uint32_t n_cap);
+ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off, const int64_t* req_ts_us,
+                        uint32_t n_req, uint32_t block_size, uint64_t seed, const ptc_cost_model* cm,
+                        const uint64_t* cap_host, uint32_t n_cap, ptc_u128* keys_out, uint64_t* req_blk_off_out,
+                        uint32_t* ids_out, uint32_t* prev_out, uint32_t* next_out, uint32_t* dist_out,
+                        uint64_t* n_access_host_out, uint64_t* n_distinct_host_out, uint64_t* hits_host_out,
+                        ptc_u128* saved_host_out, ptc_u128* total_cost_host_out, void* ws, size_t ws_bytes,
+                        void* stream);
+
+/*
  * ptc_curves_noalloc — ptc_curves for callers that cannot allocate device
  * memory.  The paper has no counterpart; this entry point exists for callers
  * with no way to supply `ws`: code running inside a runtime that owns all

@@ -105,6 +105,12 @@ def lib():
                 L.ptc_curves.restype = st
                 L.ptc_curves.argtypes = [vp, u64, vp, u32, u32, ctypes.POINTER(CostModel), vp, u32, vp, vp,
                                          ctypes.POINTER(U128), vp, sz, vp]
+                L.ptc_pipeline_workspace_bytes.restype = sz
+                L.ptc_pipeline_workspace_bytes.argtypes = [u32, u64, u32, u32]
+                L.ptc_pipeline.restype = st
+                L.ptc_pipeline.argtypes = [vp, u64, vp, vp, u32, u32, u64, ctypes.POINTER(CostModel), vp, u32,
+                                           vp, vp, vp, vp, vp, vp, ctypes.POINTER(u64), ctypes.POINTER(u64), vp, vp,
+                                           ctypes.POINTER(U128), vp, sz, vp]
                 L.ptc_timer_enable.restype = None
                 L.ptc_timer_enable.argtypes = [ctypes.c_int]
                 L.ptc_timer_reset.restype = None
@@ -284,3 +290,32 @@ def pipeline(tokens, req_tok_off, req_ts_us, block_size: int, caps_for, kind: in
     if keep:
         out.update(keys=keys, req_blk_off=blk_off, ids=ids, prev=prev, next=nxt, dist=dist)
     return out
+
+
+def ptc_pipeline(tokens, req_tok_off, req_ts_us, block_size: int, caps, kind: int = PTC_COST_MEASURED, seed: int = 0,
+                 f_lin: int = F_LIN, f_attn: int = F_ATTN, ws: torch.Tensor | None = None, outputs: dict | None = None):
+    """All five stages in one C call (trace already on the GPU).  ``outputs``
+    may map any of keys / req_blk_off / ids / prev / next / dist to
+    preallocated CUDA tensors that receive those arrays.  Returns the curves
+    with N and D."""
+    dev = _dev(req_tok_off)
+    n_req = req_tok_off.numel() - 1
+    n_tok = tokens.numel()
+    caps = np.ascontiguousarray(caps, dtype=np.uint64)
+    G = caps.shape[0]
+    w = _workspace(lib().ptc_pipeline_workspace_bytes(n_req, n_tok, block_size, G), dev, ws)
+    o = outputs or {}
+    hits = np.zeros(G, dtype=np.uint64)
+    saved = np.zeros(2 * G, dtype=np.uint64)
+    total = U128()
+    n, d = ctypes.c_uint64(0), ctypes.c_uint64(0)
+    cm = CostModel(int(f_lin), int(f_attn), int(kind))
+    rc = lib().ptc_pipeline(_ptr(tokens), n_tok, _ptr(req_tok_off), _ptr(req_ts_us), n_req, block_size,
+                            int(seed) & (2**64 - 1), ctypes.byref(cm), caps.ctypes.data, G, _ptr(o.get("keys")),
+                            _ptr(o.get("req_blk_off")), _ptr(o.get("ids")), _ptr(o.get("prev")), _ptr(o.get("next")),
+                            _ptr(o.get("dist")), ctypes.byref(n), ctypes.byref(d), hits.ctypes.data,
+                            saved.ctypes.data, ctypes.byref(total), _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_pipeline", rc)
+    return {"n_access": int(n.value), "n_distinct": int(d.value), "hits": [int(h) for h in hits],
+            "saved": [int(saved[2 * g + 1]) << 64 | int(saved[2 * g]) for g in range(G)],
+            "total_cost": int(total.hi) << 64 | int(total.lo)}

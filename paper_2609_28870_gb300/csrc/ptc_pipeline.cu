@@ -1,0 +1,91 @@
+// ptc_pipeline: the five calls in order inside the library, so a whole trace
+// needs one crossing of the C boundary.  Intermediate arrays live in caller
+// buffers when given, otherwise in the workspace; the stages' own scratch
+// reuses one region of the workspace because they run one after another on
+// the same stream.
+#include "ptc_internal.h"
+
+namespace {
+
+struct PipeLayout {
+  ptc_u128* keys;
+  uint64_t* blk_off;
+  uint32_t *ids, *prev, *next, *dist;
+  void* scratch;
+  size_t scratch_bytes;
+  size_t total;
+};
+
+size_t stage_scratch_bytes(uint32_t n_req, uint64_t n_tok, uint32_t B, uint32_t n_cap) {
+  const uint64_t n = n_tok / B;
+  size_t m = ptc_hash_blocks_workspace_bytes(n_req, n_tok, B);
+  const size_t c[] = {ptc_assign_ids_workspace_bytes(n), ptc_reuse_indices_workspace_bytes(n, n),
+                      ptc_stack_distance_workspace_bytes(n), ptc_curves_workspace_bytes(n, n_req, n_cap)};
+  for (size_t x : c) m = x > m ? x : m;
+  return m;
+}
+
+PipeLayout pipe_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uint32_t n_cap, bool keys, bool blk,
+                       bool ids, bool prev, bool next, bool dist) {
+  PipeLayout L;
+  ptc::Carver cv(ws);
+  const uint64_t n = n_tok / B ? n_tok / B : 1;
+  L.keys = keys ? nullptr : cv.take<ptc_u128>(n);
+  L.blk_off = blk ? nullptr : cv.take<uint64_t>((uint64_t)n_req + 1);
+  L.ids = ids ? nullptr : cv.take<uint32_t>(n);
+  L.prev = prev ? nullptr : cv.take<uint32_t>(n);
+  L.next = next ? nullptr : cv.take<uint32_t>(n);
+  L.dist = dist ? nullptr : cv.take<uint32_t>(n);
+  L.scratch_bytes = stage_scratch_bytes(n_req, n_tok, B, n_cap);
+  L.scratch = cv.take<unsigned char>(L.scratch_bytes);
+  L.total = cv.bytes();
+  return L;
+}
+
+}  // namespace
+
+extern "C" size_t ptc_pipeline_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size, uint32_t n_cap) {
+  if (block_size == 0) block_size = 1;
+  return pipe_layout(nullptr, n_req, n_tok, block_size, n_cap, false, false, false, false, false, false).total;
+}
+
+extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off,
+                                   const int64_t* req_ts_us, uint32_t n_req, uint32_t block_size, uint64_t seed,
+                                   const ptc_cost_model* cm, const uint64_t* cap_host, uint32_t n_cap,
+                                   ptc_u128* keys_out, uint64_t* req_blk_off_out, uint32_t* ids_out,
+                                   uint32_t* prev_out, uint32_t* next_out, uint32_t* dist_out,
+                                   uint64_t* n_access_host_out, uint64_t* n_distinct_host_out,
+                                   uint64_t* hits_host_out, ptc_u128* saved_host_out,
+                                   ptc_u128* total_cost_host_out, void* ws, size_t ws_bytes, void* stream) {
+  if (block_size < 1 || block_size > PTC_MAX_BLOCK_SIZE) return PTC_ERR_INVALID_ARG;
+  if (!n_access_host_out || !n_distinct_host_out) return PTC_ERR_INVALID_ARG;
+  const PipeLayout need = pipe_layout(nullptr, n_req, n_tok, block_size, n_cap, keys_out, req_blk_off_out, ids_out,
+                                      prev_out, next_out, dist_out);
+  if (!ptc::ws_ok(ws, ws_bytes, need.total)) return PTC_ERR_WORKSPACE;
+  const PipeLayout L = pipe_layout(ws, n_req, n_tok, block_size, n_cap, keys_out, req_blk_off_out, ids_out, prev_out,
+                                   next_out, dist_out);
+  ptc_u128* keys = keys_out ? keys_out : L.keys;
+  uint64_t* blk = req_blk_off_out ? req_blk_off_out : L.blk_off;
+  uint32_t* ids = ids_out ? ids_out : L.ids;
+  uint32_t* prev = prev_out ? prev_out : L.prev;
+  uint32_t* next = next_out ? next_out : L.next;
+  uint32_t* dist = dist_out ? dist_out : L.dist;
+  const uint64_t cap = n_tok / block_size ? n_tok / block_size : 1;
+  uint64_t n = 0, d = 0;
+  ptc_status rc = ptc_hash_blocks(tokens, n_tok, req_tok_off, req_ts_us, n_req, block_size, seed, keys, cap, blk, &n,
+                                  L.scratch, L.scratch_bytes, stream);
+  *n_access_host_out = n;
+  *n_distinct_host_out = 0;
+  if (rc != PTC_OK) return rc;
+  rc = ptc_assign_ids(keys, n, ids, &d, L.scratch, L.scratch_bytes, stream);
+  *n_distinct_host_out = d;
+  if (rc != PTC_OK) return rc;
+  if (n > 0) {
+    rc = ptc_reuse_indices(ids, n, d, prev, next, L.scratch, L.scratch_bytes, stream);
+    if (rc != PTC_OK) return rc;
+    rc = ptc_stack_distance(prev, n, dist, L.scratch, L.scratch_bytes, stream);
+    if (rc != PTC_OK) return rc;
+  }
+  return ptc_curves(dist, n, blk, n_req, block_size, cm, cap_host, n_cap, hits_host_out, saved_host_out,
+                    total_cost_host_out, L.scratch, L.scratch_bytes, stream);
+}
