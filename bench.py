@@ -103,7 +103,14 @@ def stage_model_bytes(T, N):
     }, L
 
 
-def kernel_model_bytes(name, T, N, L):
+def sort_passes(D):
+    b = 1
+    while b < 32 and (1 << b) < D:
+        b += 1
+    return (b + 7) // 8
+
+
+def kernel_model_bytes(name, T, N, L, D):
     """Algorithmic bytes one launch of `name` moves under the stage-byte model
     (0: the kernel only touches scratch the model does not count)."""
     per_level = ((L - 1) * 8.125 + 4.125) / L * N  # the last level writes no partition
@@ -111,10 +118,11 @@ def kernel_model_bytes(name, T, N, L):
         "k_hash_local": 4 * T + 16 * N,   # token stream in, block keys out
         "k_ids_insert": 16 * N,           # keys in
         "k_ids_gather": 4 * N,            # ids out
-        "k_sort_hist": 4 * N,             # ids in
-        "k_adjacent": 8 * N,              # prev / next out
+        "k_sort_scatter": 12 * N / sort_passes(D),  # ids in, prev / next out, spread over the passes
         "k_wm_level": per_level,          # values in, partition + bit plane out
         "k_wm_heads": (8 + L / 8) * N,    # prev in, one read of the bit planes, distances out
+        "k_runs_mark": 4 * N,             # prev in (matrix over runs)
+        "k_runs_expand": 4 * N,           # distances out (matrix over runs)
         "k_curves": 4 * N,                # distances in
     }.get(name, 0.0)
 
@@ -122,10 +130,11 @@ def kernel_model_bytes(name, T, N, L):
 KERNEL_SOURCE = {
     "k_block_offsets": "ptc_hash.cu", "k_pow_tables": "ptc_hash.cu", "k_hash_local": "ptc_hash.cu",
     "k_hash_chain": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu", "k_ids_rank": "ptc_ids.cu",
-    "k_ids_gather": "ptc_ids.cu", "k_sort_hist": "ptc_sort.cu", "k_sort_offsets": "ptc_sort.cu",
-    "k_sort_pass": "ptc_sort.cu", "k_adjacent": "ptc_sort.cu", "k_wm_count0": "ptc_wavelet.cu",
+    "k_ids_gather": "ptc_ids.cu", "k_sort_count": "ptc_sort.cu", "k_sort_rowscan": "ptc_sort.cu",
+    "k_sort_scatter": "ptc_sort.cu", "k_sort_links": "ptc_sort.cu", "k_wm_count0": "ptc_wavelet.cu",
     "k_wm_level": "ptc_wavelet.cu", "k_wm_dir": "ptc_wavelet.cu", "k_wm_heads": "ptc_wavelet.cu",
-    "k_wm_propagate": "ptc_wavelet.cu", "k_heads": "ptc_curves.cu", "k_curves_agg": "ptc_curves.cu",
+    "k_wm_propagate": "ptc_wavelet.cu", "k_runs_mark": "ptc_runs.cu", "k_runs_init": "ptc_runs.cu",
+    "k_runs_level": "ptc_runs.cu", "k_runs_query": "ptc_runs.cu", "k_runs_expand": "ptc_runs.cu", "k_heads": "ptc_curves.cu", "k_curves_agg": "ptc_curves.cu",
     "k_curves": "ptc_curves.cu", "k_finalize": "ptc_curves.cu",
 }
 
@@ -294,7 +303,7 @@ def run_ours(args, ws_world, rank, local):
     kernels = []
     for name, launches_k, tot_ms in ktimes:
         per = tot_ms / max(launches_k, 1)
-        mb = kernel_model_bytes(name, T, N, Lbits)
+        mb = kernel_model_bytes(name, T, N, Lbits, D)
         kernels.append({"name": name, "launches_per_step": launches_k / args.steps, "ms_per_step": tot_ms / args.steps,
                         "avg_launch_ms": per, "model_bytes_per_launch": mb,
                         "achieved_gbs": (mb / (per * 1e-3) / 1e9) if per > 0 else 0.0})

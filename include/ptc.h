@@ -178,6 +178,27 @@ ptc_status ptc_stack_distance(const uint32_t* prev, uint64_t n, uint32_t* dist_o
                               void* stream);
 
 /*
+ * ptc_stack_distance_ex — the same distances with the matrix chosen by the
+ * caller.  PTC_SD_POINTS builds the wavelet matrix over every access.
+ * PTC_SD_RUNS builds it over runs: maximal stretches where prev grows by one
+ * from access to access, or that are all first accesses.  A run is either
+ * wholly counted or wholly left out of every window (an access has at most
+ * one next use), so a matrix over runs weighted by their lengths gives the
+ * same counts with R points instead of n.  PTC_SD_AUTO (what
+ * ptc_stack_distance does) finds the runs first and takes the matrix over
+ * runs when R <= n / 3 and the workspace holds it, else the one over accesses.
+ *   prev must come from ptc_reuse_indices, or at least satisfy prev[i] < i and
+ *   take each value other than PTC_NONE at most once; the matrix over runs
+ *   relies on the latter, and neither checks it.
+ * Workspace: ptc_stack_distance_ex_workspace_bytes(n, method);
+ * PTC_ERR_WORKSPACE when PTC_SD_RUNS finds more runs than the workspace holds.
+ */
+enum { PTC_SD_AUTO = 0, PTC_SD_POINTS = 1, PTC_SD_RUNS = 2 };
+size_t ptc_stack_distance_ex_workspace_bytes(uint64_t n, int method);
+ptc_status ptc_stack_distance_ex(const uint32_t* prev, uint64_t n, uint32_t* dist_out, int method, void* ws,
+                                 size_t ws_bytes, void* stream);
+
+/*
  * ptc_curves — hit and compute-saved curves for every capacity at once
  * (Sec. 3.2 block hit ratio; Sec. 5.2 compute-savings ratio; prefix reuse
  * from Sec. 2.2).  Block k of a request is counted as a hit at capacity C iff

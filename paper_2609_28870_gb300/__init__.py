@@ -28,6 +28,7 @@ from . import build as _build
 
 PTC_NONE = 0xFFFFFFFF
 PTC_COST_UNIFORM, PTC_COST_MEASURED, PTC_COST_LINEAR = 0, 1, 2
+PTC_SD_AUTO, PTC_SD_POINTS, PTC_SD_RUNS = 0, 1, 2
 F_LIN = 6_600_000_000          # 2 x 3.3e9 active parameters, FLOPs per token
 F_ATTN = 4 * 48 * 32 * 128     # per attended position: 4 x layers x heads x head_dim
 MAX_CAPACITIES = 1024
@@ -100,6 +101,10 @@ def lib():
                 L.ptc_stack_distance_workspace_bytes.argtypes = [u64]
                 L.ptc_stack_distance.restype = st
                 L.ptc_stack_distance.argtypes = [vp, u64, vp, vp, sz, vp]
+                L.ptc_stack_distance_ex_workspace_bytes.restype = sz
+                L.ptc_stack_distance_ex_workspace_bytes.argtypes = [u64, ctypes.c_int]
+                L.ptc_stack_distance_ex.restype = st
+                L.ptc_stack_distance_ex.argtypes = [vp, u64, vp, ctypes.c_int, vp, sz, vp]
                 L.ptc_curves_workspace_bytes.restype = sz
                 L.ptc_curves_workspace_bytes.argtypes = [u64, u32, u32]
                 L.ptc_curves.restype = st
@@ -226,14 +231,21 @@ def ptc_reuse_indices(ids: torch.Tensor, n_distinct: int, ws: torch.Tensor | Non
     return prev[:n], nxt[:n]
 
 
-def ptc_stack_distance(prev: torch.Tensor, ws: torch.Tensor | None = None) -> torch.Tensor:
-    """LRU stack distance of every access (1-based; PTC_NONE for a first access)."""
+def ptc_stack_distance(prev: torch.Tensor, ws: torch.Tensor | None = None, method: int | None = None) -> torch.Tensor:
+    """LRU stack distance of every access (1-based; PTC_NONE for a first access).
+    ``method`` (PTC_SD_AUTO / PTC_SD_POINTS / PTC_SD_RUNS) picks the wavelet
+    matrix through ptc_stack_distance_ex; None calls ptc_stack_distance."""
     dev = _dev(prev)
     n = prev.numel()
     dist = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
-    w = _workspace(lib().ptc_stack_distance_workspace_bytes(n), dev, ws)
-    rc = lib().ptc_stack_distance(_ptr(prev), n, _ptr(dist), _ptr(w), w.numel(), _stream(dev))
-    _check("ptc_stack_distance", rc)
+    if method is None:
+        w = _workspace(lib().ptc_stack_distance_workspace_bytes(n), dev, ws)
+        rc = lib().ptc_stack_distance(_ptr(prev), n, _ptr(dist), _ptr(w), w.numel(), _stream(dev))
+        _check("ptc_stack_distance", rc)
+    else:
+        w = _workspace(lib().ptc_stack_distance_ex_workspace_bytes(n, method), dev, ws)
+        rc = lib().ptc_stack_distance_ex(_ptr(prev), n, _ptr(dist), method, _ptr(w), w.numel(), _stream(dev))
+        _check("ptc_stack_distance_ex", rc)
     return dist[:n]
 
 

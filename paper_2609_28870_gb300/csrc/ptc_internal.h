@@ -57,4 +57,10 @@ inline bool ws_ok(const void* ws, size_t ws_bytes, size_t need) {
   return ws != nullptr && ((uintptr_t)ws & 255) == 0 && ws_bytes >= need;
 }
 
+// Stage c on the matrix over every access (ptc_wavelet.cu); the C entry
+// points in ptc_runs.cu choose between it and the matrix over runs.
+size_t stack_distance_points_bytes(uint64_t n);
+ptc_status stack_distance_points(const uint32_t* prev, uint64_t n, uint32_t* dist_out, void* ws, size_t ws_bytes,
+                                 cudaStream_t s);
+
 }  // namespace ptc

@@ -1,0 +1,542 @@
+// Stage c over runs: the dominance count of App. B on a weighted wavelet
+// matrix whose points are the runs of the access stream, not its accesses.
+//
+// With v_j = prev[j] + 1 (none -> 0), the stack distance of access i with
+// p = prev[i] is
+//   SD_i = 1 + #{ j : p < j < i, v_j <= p }.
+// A run is a maximal stretch of accesses that either re-read a context block
+// by block (v_{j+1} = v_j + 1, v_j > 0) or are all first accesses (v = 0).
+// Re-reads of long shared prefixes make runs long: the conversational traces
+// hold a few hundred accesses per run.
+//
+// Every run meets the window (p, i) either entirely inside or not at all in
+// the count.  Inside the window no access has v_j = p + 1, because that value
+// belongs to i alone (an access has at most one next use).  The values along
+// a context run are consecutive, so those of a run that fall in the window
+// lie all at or below p or all above it; a first-access run is all zeros.
+// Hence
+//   SD_i = 1 + [the run holding p+1, when it starts before p+1: its part in
+//               the window if its value at p+1 is <= p]
+//            + sum of the lengths of the runs wholly inside (p, i) whose
+//              largest value is <= p,
+// a weighted 2-D dominance count over runs (index, largest value; weight =
+// length).  The matrix over runs answers it exactly as the matrix over
+// accesses would, and a run head's distance is that of its whole run (a
+// context run's accesses all share it, the run identity of App. B's
+// stack-distance recurrence).
+//
+// Weighted wavelet matrix (Claude, Navarro, Ordonez 2015): level l orders the
+// runs by the stable partition on bit L-1-l of the previous level's order and
+// stores, for every position, the zeros before it and their total weight
+// (Z, W).  A count of keys < x over [lo, hi) walks the L levels; where x has a
+// one bit, the zeros of the current range (all smaller) add their weight.
+//
+//   k_runs_mark    run starts: bitmap, run index per 32-position word, run
+//                  (start, first value) records; one look-back pass
+//   k_runs_init    level-0 keys and weights, per-tile zero counts / weights
+//   k_runs_level   one level: (Z, W), stable partition, the next level's
+//                  per-tile zero counts (four atomics per tile)
+//   k_runs_query   one thread per run: the distance of its head
+//   k_runs_expand  every access takes its run's distance
+#include "ptc_internal.h"
+
+namespace ptc {
+namespace {
+
+constexpr int kMT = 256;           // run marking: threads per tile
+constexpr int kMR = 8;             // rounds of 32 positions per warp
+constexpr int kMTile = kMT * kMR;  // 2048 positions; warp w owns [256 w, 256 w + 256)
+constexpr int kRT = 256;           // level tiles: threads
+constexpr int kRPer = 8;           // runs per thread (consecutive)
+constexpr int kRTile = kRT * kRPer;
+constexpr uint32_t kMarkEpoch = 1;
+
+__device__ __forceinline__ uint32_t vval(uint32_t p) { return p == kNone ? 0u : p + 1u; }
+
+struct MarkArgs {
+  const uint32_t* prev;
+  uint32_t n;
+  uint32_t ntiles;
+  uint32_t* bits;     // run-start bitmap, one word per 32 positions
+  uint32_t* wpre;     // runs starting before each word
+  uint32_t* rec_s;    // start of each run (rec_s[R] = n)
+  uint32_t* rec_a;    // value at the start of each run
+  uint64_t* lb;       // look-back words, one per tile
+  DevStatus* st;      // value[1] <- R
+};
+
+__global__ void __launch_bounds__(kMT) k_runs_mark(MarkArgs a) {
+  __shared__ uint32_t s_wcnt[kMT / 32];
+  const uint32_t tile = next_tile(a.st, kMarkEpoch);
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const uint32_t base = tile * kMTile + w * (32 * kMR);
+  uint32_t pv[kMR];
+#pragma unroll
+  for (int k = 0; k < kMR; ++k) {
+    const uint32_t j = base + k * 32 + lane;
+    pv[k] = j < a.n ? a.prev[j] : kNone;
+  }
+  const uint32_t left0 = (lane == 0 && base > 0 && base - 1 < a.n) ? a.prev[base - 1] : kNone;
+  uint32_t words[kMR];
+  uint32_t cnt = 0;
+  bool bad = false;
+  uint32_t carry = vval(left0);  // value left of lane 0 (meaningful in lane 0 only)
+#pragma unroll
+  for (int k = 0; k < kMR; ++k) {
+    const uint32_t j = base + k * 32 + lane;
+    const bool valid = j < a.n;
+    if (valid && pv[k] != kNone && pv[k] >= j) bad = true;
+    const uint32_t v = vval(pv[k]);
+    const uint32_t up = __shfl_up_sync(kFull, v, 1);
+    const uint32_t vl = lane ? up : carry;
+    carry = __shfl_sync(kFull, v, 31);
+    const bool cont = j > 0 && ((v == vl + 1 && vl != 0) || (v == 0 && vl == 0));
+    words[k] = __ballot_sync(kFull, valid && !cont);
+    cnt += __popc(words[k]);
+  }
+  if (lane == 0) s_wcnt[w] = cnt;
+  __syncthreads();
+  uint32_t agg = 0, wpre_in_tile = 0;
+#pragma unroll
+  for (int ww = 0; ww < kMT / 32; ++ww) {
+    const uint32_t c = s_wcnt[ww];
+    if (ww < (int)w) wpre_in_tile += c;
+    agg += c;
+  }
+  const uint32_t tile_pre = (uint32_t)lookback_sum_cta(a.lb, tile, agg, kMarkEpoch, a.st);
+  uint32_t run = tile_pre + wpre_in_tile;
+#pragma unroll
+  for (int k = 0; k < kMR; ++k) {
+    const uint32_t j = base + k * 32 + lane;
+    if (base + k * 32 < a.n && lane == 0) {
+      a.bits[(base + k * 32) >> 5] = words[k];
+      a.wpre[(base + k * 32) >> 5] = run;
+    }
+    if ((words[k] >> lane) & 1u) {
+      const uint32_t r = run + __popc(words[k] & lanemask_lt());
+      a.rec_s[r] = j;
+      a.rec_a[r] = vval(pv[k]);
+    }
+    run += __popc(words[k]);
+  }
+  if (bad) raise_err(a.st, kErrInvalid);
+  if (tile == a.ntiles - 1 && threadIdx.x == 0) {
+    const uint32_t R = tile_pre + agg;
+    a.rec_s[R] = a.n;
+    a.st->value[1] = R;
+  }
+}
+
+// Exclusive scan over the threads of a 256-thread CTA.
+__device__ __forceinline__ unsigned long long cta_excl_scan(unsigned long long x, unsigned long long* s_warp,
+                                                            unsigned long long& total) {
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  unsigned long long incl = x;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned long long y = __shfl_up_sync(kFull, incl, o);
+    if (lane >= (uint32_t)o) incl += y;
+  }
+  if (lane == 31) s_warp[w] = incl;
+  __syncthreads();
+  unsigned long long pre = 0, tot = 0;
+#pragma unroll
+  for (int ww = 0; ww < kRT / 32; ++ww) {
+    const unsigned long long v = s_warp[ww];
+    if (ww < (int)w) pre += v;
+    tot += v;
+  }
+  __syncthreads();
+  total = tot;
+  return pre + incl - x;
+}
+
+// (zeros, zero weight) packed as weight << 32 | count; a tile holds at most
+// 2048 runs and all weights sum to N < 2^32, so neither half overflows.
+__device__ __forceinline__ unsigned long long pack_zw(uint32_t z, uint32_t w) {
+  return ((unsigned long long)w << 32) | z;
+}
+
+// Run by the last CTA of a level: exclusive prefix of the per-tile (zeros,
+// zero weight) of the next level over its tiles; pre[ntiles] = totals.
+__device__ void tile_prefix(const uint2* acc, uint2* pre, uint32_t ntiles, unsigned long long* s_warp) {
+  const uint32_t per = (ntiles + kRT - 1) / kRT;
+  const uint32_t t0 = threadIdx.x * per, t1 = min(t0 + per, ntiles);
+  unsigned long long s = 0;
+  for (uint32_t t = t0; t < t1; ++t) {
+    const uint2 v = __ldcg(&acc[t]);
+    s += pack_zw(v.x, v.y);
+  }
+  unsigned long long total;
+  unsigned long long run = cta_excl_scan(s, s_warp, total);
+  for (uint32_t t = t0; t < t1; ++t) {
+    const uint2 v = __ldcg(&acc[t]);
+    pre[t] = make_uint2((uint32_t)run, (uint32_t)(run >> 32));
+    run += pack_zw(v.x, v.y);
+  }
+  if (threadIdx.x == 0) pre[ntiles] = make_uint2((uint32_t)total, (uint32_t)(total >> 32));
+}
+
+// The calling CTA learns whether it is the last of the grid to get here.
+__device__ __forceinline__ bool last_cta(uint32_t* done) {
+  __shared__ uint32_t s_last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(done, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (s_last) __threadfence();
+  return s_last;
+}
+
+struct LevelArgs {
+  const uint32_t* key_in;   // this level's order
+  const uint32_t* wt_in;
+  uint32_t* key_out;        // the next level's order (null at the last level)
+  uint32_t* wt_out;
+  uint2* zw;                // (Z, W) of this level, R + 1 entries
+  const uint2* pre;         // (zeros, zero weight) before each tile of this level
+  uint2* acc_next;          // per-tile (zeros, zero weight) of the next level
+  uint2* pre_next;
+  uint32_t* done;
+  uint32_t R, ntiles, shift;
+};
+
+// Level-0 keys (largest value of each run) and weights (lengths) and the
+// per-tile zero counts of level 0.
+__global__ void __launch_bounds__(kRT) k_runs_init(const uint32_t* __restrict__ rec_s, const uint32_t* __restrict__ rec_a,
+                                                  uint32_t* __restrict__ key, uint32_t* __restrict__ wt,
+                                                  uint2* __restrict__ acc, uint2* __restrict__ pre, uint32_t* done,
+                                                  uint32_t R, uint32_t ntiles, uint32_t shift) {
+  __shared__ unsigned long long s_warp[kRT / 32];
+  const uint32_t r0 = blockIdx.x * kRTile + threadIdx.x * kRPer;
+  uint32_t cz = 0, cw = 0;
+#pragma unroll
+  for (int k = 0; k < kRPer; ++k) {
+    const uint32_t r = r0 + k;
+    if (r < R) {
+      const uint32_t s = rec_s[r], e = rec_s[r + 1], a0 = rec_a[r];
+      const uint32_t len = e - s;
+      const uint32_t kv = a0 ? a0 + len - 1 : 0u;
+      key[r] = kv;
+      wt[r] = len;
+      if (!((kv >> shift) & 1u)) {
+        ++cz;
+        cw += len;
+      }
+    }
+  }
+  unsigned long long total;
+  cta_excl_scan(pack_zw(cz, cw), s_warp, total);
+  if (threadIdx.x == 0) acc[blockIdx.x] = make_uint2((uint32_t)total, (uint32_t)(total >> 32));
+  if (last_cta(done)) tile_prefix(acc, pre, ntiles, s_warp);
+}
+
+__global__ void __launch_bounds__(kRT) k_runs_level(LevelArgs a) {
+  __shared__ unsigned long long s_warp[kRT / 32];
+  __shared__ uint32_t s_red[4][2][kRT / 32];
+  const uint32_t t = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const uint32_t r0 = t * kRTile + threadIdx.x * kRPer;
+  uint32_t kv[kRPer], wv[kRPer];
+  if (r0 + kRPer <= a.R) {
+    const uint4* k4 = reinterpret_cast<const uint4*>(a.key_in + r0);
+    const uint4* w4 = reinterpret_cast<const uint4*>(a.wt_in + r0);
+    const uint4 ka = k4[0], kb = k4[1], wa = w4[0], wb = w4[1];
+    kv[0] = ka.x; kv[1] = ka.y; kv[2] = ka.z; kv[3] = ka.w;
+    kv[4] = kb.x; kv[5] = kb.y; kv[6] = kb.z; kv[7] = kb.w;
+    wv[0] = wa.x; wv[1] = wa.y; wv[2] = wa.z; wv[3] = wa.w;
+    wv[4] = wb.x; wv[5] = wb.y; wv[6] = wb.z; wv[7] = wb.w;
+  } else {
+#pragma unroll
+    for (int k = 0; k < kRPer; ++k) {
+      kv[k] = r0 + k < a.R ? a.key_in[r0 + k] : 0u;
+      wv[k] = r0 + k < a.R ? a.wt_in[r0 + k] : 0u;
+    }
+  }
+  uint32_t cz = 0, cw = 0;
+#pragma unroll
+  for (int k = 0; k < kRPer; ++k) {
+    if (r0 + k < a.R && !((kv[k] >> a.shift) & 1u)) {
+      ++cz;
+      cw += wv[k];
+    }
+  }
+  unsigned long long tile_tot;
+  const unsigned long long ex = cta_excl_scan(pack_zw(cz, cw), s_warp, tile_tot);
+  const uint2 tp = a.pre[t];
+  const uint32_t Zc = a.pre[a.ntiles].x;
+  uint32_t z = tp.x + (uint32_t)ex, wsum = tp.y + (uint32_t)(ex >> 32);
+  // destinations: this tile's zeros fill [tp.x, tp.x + tz), its ones
+  // [Zc + t * kRTile - tp.x, ...); each range meets at most two next-level tiles
+  const uint32_t zfirst = tp.x / kRTile, ofirst = (Zc + t * kRTile - tp.x) / kRTile;
+  uint32_t nz[4] = {0, 0, 0, 0}, nw[4] = {0, 0, 0, 0};
+#pragma unroll
+  for (int k = 0; k < kRPer; ++k) {
+    const uint32_t r = r0 + k;
+    if (r < a.R) {
+      a.zw[r] = make_uint2(z, wsum);
+      const bool zero = !((kv[k] >> a.shift) & 1u);
+      const uint32_t dst = zero ? z : Zc + (r - z);
+      if (zero) {
+        ++z;
+        wsum += wv[k];
+      }
+      if (a.key_out && dst < a.R) {
+        a.key_out[dst] = kv[k];
+        a.wt_out[dst] = wv[k];
+        if (!((kv[k] >> (a.shift - 1)) & 1u)) {
+          const uint32_t slot = (zero ? 0u : 2u) + ((dst / kRTile) != (zero ? zfirst : ofirst) ? 1u : 0u);
+          ++nz[slot];
+          nw[slot] += wv[k];
+        }
+      }
+    }
+  }
+  if (a.key_out) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        nz[q] += __shfl_xor_sync(kFull, nz[q], o);
+        nw[q] += __shfl_xor_sync(kFull, nw[q], o);
+      }
+      if (lane == 0) {
+        s_red[q][0][w] = nz[q];
+        s_red[q][1][w] = nw[q];
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x < 4) {
+      const uint32_t q = threadIdx.x;
+      uint32_t c = 0, s = 0;
+#pragma unroll
+      for (int ww = 0; ww < kRT / 32; ++ww) {
+        c += s_red[q][0][ww];
+        s += s_red[q][1][ww];
+      }
+      const uint32_t tile_next = (q < 2 ? zfirst : ofirst) + (q & 1u);
+      if (c && tile_next < a.ntiles) {
+        atomicAdd(&a.acc_next[tile_next].x, c);
+        atomicAdd(&a.acc_next[tile_next].y, s);
+      }
+    }
+  }
+  if (last_cta(a.done)) {
+    if (threadIdx.x == 0) a.zw[a.R] = a.pre[a.ntiles];
+    if (a.key_out) tile_prefix(a.acc_next, a.pre_next, a.ntiles, s_warp);
+  }
+}
+
+struct QueryArgs {
+  const uint32_t* rec_s;
+  const uint32_t* rec_a;
+  const uint32_t* bits;
+  const uint32_t* wpre;
+  const uint2* zw;      // level l at zw + l * (R + 1)
+  uint32_t* sd;         // distance of each run
+  uint32_t R, L;
+};
+
+// Index of the run holding position j.
+__device__ __forceinline__ uint32_t run_of(const uint32_t* bits, const uint32_t* wpre, uint32_t j) {
+  const uint32_t wi = j >> 5, b = j & 31;
+  const uint32_t mask_le = b == 31 ? kFull : ((2u << b) - 1u);
+  return wpre[wi] + __popc(bits[wi] & mask_le) - 1u;
+}
+
+__global__ void __launch_bounds__(256) k_runs_query(QueryArgs a) {
+  const uint32_t r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= a.R) return;
+  const uint32_t x = a.rec_a[r];  // p + 1
+  if (x == 0) {
+    a.sd[r] = kNone;
+    return;
+  }
+  const uint32_t s = a.rec_s[r];
+  const uint32_t rho = run_of(a.bits, a.wpre, x);
+  uint32_t lo = rho, partial = 0;
+  const uint32_t s1 = a.rec_s[rho];
+  if (s1 < x) {  // the run holding p + 1 starts before the window
+    const uint32_t e1 = a.rec_s[rho + 1], a1 = a.rec_a[rho];
+    const uint32_t vfirst = a1 ? a1 + (x - s1) : 0u;
+    if (vfirst < x) partial = min(e1, s) - x;
+    lo = rho + 1;
+  }
+  uint32_t hi = r, cnt = 0;
+  const uint32_t stride = a.R + 1;
+  for (uint32_t l = 0; l < a.L && lo < hi; ++l) {
+    const uint2* zl = a.zw + (size_t)l * stride;
+    const uint2 zlo = zl[lo], zhi = zl[hi];
+    if ((x >> (a.L - 1 - l)) & 1u) {
+      const uint32_t Zc = zl[a.R].x;
+      cnt += zhi.y - zlo.y;
+      lo = Zc + (lo - zlo.x);
+      hi = Zc + (hi - zhi.x);
+    } else {
+      lo = zlo.x;
+      hi = zhi.x;
+    }
+  }
+  a.sd[r] = 1u + partial + cnt;
+}
+
+__global__ void __launch_bounds__(256) k_runs_expand(const uint32_t* __restrict__ bits,
+                                                    const uint32_t* __restrict__ wpre, const uint32_t* __restrict__ sd,
+                                                    uint32_t n, uint32_t* __restrict__ dist) {
+  const uint32_t j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j >= n) return;
+  dist[j] = sd[run_of(bits, wpre, j)];
+}
+
+uint32_t key_bits_n(uint64_t n) {  // keys and thresholds lie in [0, n]
+  uint32_t L = 1;
+  while (L < 33 && (1ULL << L) <= n) ++L;
+  return L;
+}
+
+// Arrays the marking pass writes (sized by N) come first; those sized by the
+// number of runs R follow.
+struct RunsLayout {
+  DevStatus* st;
+  uint32_t* done;
+  uint64_t* lb;
+  size_t zero_bytes;
+  uint32_t *bits, *wpre, *rec_s, *rec_a;
+  uint32_t *sd, *k0, *k1, *w0, *w1;
+  uint2 *acc, *pre, *zw;
+  uint32_t L, mtiles, rtiles;
+  size_t acc_bytes;
+  size_t total;
+};
+
+RunsLayout runs_layout(void* ws, uint64_t n, uint64_t R) {
+  RunsLayout W;
+  Carver cv(ws);
+  const uint64_t nn = n ? n : 1, rr = R ? R : 1;
+  W.L = key_bits_n(n);
+  W.mtiles = ceil_div_u32(nn, kMTile);
+  W.rtiles = ceil_div_u32(rr, kRTile);
+  W.st = cv.take<DevStatus>(1);
+  W.done = cv.take<uint32_t>(64);
+  W.lb = cv.take<uint64_t>(W.mtiles + 1);
+  W.zero_bytes = cv.off;
+  W.bits = cv.take<uint32_t>(nn / 32 + 2);
+  W.wpre = cv.take<uint32_t>(nn / 32 + 2);
+  W.rec_s = cv.take<uint32_t>(nn + 1);
+  W.rec_a = cv.take<uint32_t>(nn);
+  const size_t acc_off = cv.off;
+  W.acc = cv.take<uint2>((uint64_t)(W.L + 1) * (W.rtiles + 1));
+  W.acc_bytes = cv.off - acc_off;
+  W.pre = cv.take<uint2>((uint64_t)(W.L + 1) * (W.rtiles + 1));
+  W.sd = cv.take<uint32_t>(rr);
+  W.k0 = cv.take<uint32_t>(rr);
+  W.k1 = cv.take<uint32_t>(rr);
+  W.w0 = cv.take<uint32_t>(rr);
+  W.w1 = cv.take<uint32_t>(rr);
+  W.zw = cv.take<uint2>((uint64_t)W.L * (rr + 1));
+  W.total = cv.bytes();
+  return W;
+}
+
+// Runs the automatic choice reserves room for: a third of the accesses, at
+// most 2^24 (the matrix over runs then costs less than the one over accesses).
+uint64_t runs_reserve(uint64_t n) {
+  const uint64_t r = n / 3 + 1;
+  return r < (1ULL << 24) ? r : (1ULL << 24);
+}
+
+ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_out, void* ws, size_t ws_bytes,
+                               cudaStream_t s, int method) {
+  const RunsLayout M = runs_layout(ws, n, 1);
+  if (!ws_ok(ws, ws_bytes, M.total)) return PTC_ERR_WORKSPACE;
+  if (begin_call(ws, M.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
+  MarkArgs m;
+  m.prev = prev;
+  m.n = (uint32_t)n;
+  m.ntiles = M.mtiles;
+  m.bits = M.bits;
+  m.wpre = M.wpre;
+  m.rec_s = M.rec_s;
+  m.rec_a = M.rec_a;
+  m.lb = M.lb;
+  m.st = M.st;
+  PTC_LAUNCH("k_runs_mark", s, k_runs_mark<<<M.mtiles, kMT, 0, s>>>(m));
+  DevStatus h;
+  ptc_status rc = end_call(M.st, s, &h);
+  if (rc != PTC_OK) return rc;
+  const uint64_t R = h.value[1];
+  const RunsLayout W = runs_layout(ws, n, R);
+  const bool fits = R >= 1 && R <= n && ws_bytes >= W.total;
+  if (method == PTC_SD_AUTO && (!fits || R > n / 3)) return stack_distance_points(prev, n, dist_out, ws, ws_bytes, s);
+  if (!fits) return PTC_ERR_WORKSPACE;
+  if (cudaMemsetAsync(W.acc, 0, W.acc_bytes, s) != cudaSuccess) return PTC_ERR_CUDA;
+  if (cudaMemsetAsync(W.done, 0, 64 * sizeof(uint32_t), s) != cudaSuccess) return PTC_ERR_CUDA;
+  const uint32_t R32 = (uint32_t)R, T = W.rtiles, L = W.L;
+  const size_t tstride = (size_t)T + 1;
+  PTC_LAUNCH("k_runs_init", s,
+             k_runs_init<<<T, kRT, 0, s>>>(W.rec_s, W.rec_a, W.k0, W.w0, W.acc, W.pre, &W.done[0], R32, T, L - 1));
+  uint32_t* keys[2] = {W.k0, W.k1};
+  uint32_t* wts[2] = {W.w0, W.w1};
+  for (uint32_t l = 0; l < L; ++l) {
+    const bool last = l + 1 == L;
+    LevelArgs a;
+    a.key_in = keys[l & 1];
+    a.wt_in = wts[l & 1];
+    a.key_out = last ? nullptr : keys[(l + 1) & 1];
+    a.wt_out = last ? nullptr : wts[(l + 1) & 1];
+    a.zw = W.zw + (size_t)l * (R + 1);
+    a.pre = W.pre + (size_t)l * tstride;
+    a.acc_next = last ? nullptr : W.acc + (size_t)(l + 1) * tstride;
+    a.pre_next = last ? nullptr : W.pre + (size_t)(l + 1) * tstride;
+    a.done = &W.done[1 + l];
+    a.R = R32;
+    a.ntiles = T;
+    a.shift = L - 1 - l;
+    PTC_LAUNCH("k_runs_level", s, k_runs_level<<<T, kRT, 0, s>>>(a));
+  }
+  QueryArgs q;
+  q.rec_s = W.rec_s;
+  q.rec_a = W.rec_a;
+  q.bits = W.bits;
+  q.wpre = W.wpre;
+  q.zw = W.zw;
+  q.sd = W.sd;
+  q.R = R32;
+  q.L = L;
+  PTC_LAUNCH("k_runs_query", s, k_runs_query<<<ceil_div_u32(R, 256), 256, 0, s>>>(q));
+  PTC_LAUNCH("k_runs_expand", s,
+             k_runs_expand<<<ceil_div_u32(n, 256), 256, 0, s>>>(W.bits, W.wpre, W.sd, (uint32_t)n, dist_out));
+  return end_call(W.st, s, &h);
+}
+
+}  // namespace
+}  // namespace ptc
+
+using namespace ptc;
+
+extern "C" size_t ptc_stack_distance_ex_workspace_bytes(uint64_t n, int method) {
+  const size_t pts = stack_distance_points_bytes(n);
+  if (method == PTC_SD_POINTS) return pts;
+  if (method == PTC_SD_RUNS) return runs_layout(nullptr, n, n).total;
+  const size_t runs = runs_layout(nullptr, n, runs_reserve(n)).total;
+  return pts > runs ? pts : runs;
+}
+
+extern "C" size_t ptc_stack_distance_workspace_bytes(uint64_t n) {
+  return ptc_stack_distance_ex_workspace_bytes(n, PTC_SD_AUTO);
+}
+
+extern "C" ptc_status ptc_stack_distance_ex(const uint32_t* prev, uint64_t n, uint32_t* dist_out, int method,
+                                            void* ws, size_t ws_bytes, void* stream) {
+  if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
+  if (method != PTC_SD_AUTO && method != PTC_SD_POINTS && method != PTC_SD_RUNS) return PTC_ERR_INVALID_ARG;
+  if (n == 0) return PTC_OK;
+  if (!prev || !dist_out) return PTC_ERR_INVALID_ARG;
+  cudaStream_t s = (cudaStream_t)stream;
+  if (method == PTC_SD_POINTS) return stack_distance_points(prev, n, dist_out, ws, ws_bytes, s);
+  return stack_distance_runs(prev, n, dist_out, ws, ws_bytes, s, method);
+}
+
+extern "C" ptc_status ptc_stack_distance(const uint32_t* prev, uint64_t n, uint32_t* dist_out, void* ws,
+                                         size_t ws_bytes, void* stream) {
+  return ptc_stack_distance_ex(prev, n, dist_out, PTC_SD_AUTO, ws, ws_bytes, stream);
+}

@@ -558,15 +558,12 @@ WmLayout wm_layout(void* ws, uint64_t n) {
 
 using namespace ptc;
 
-extern "C" size_t ptc_stack_distance_workspace_bytes(uint64_t n) { return wm_layout(nullptr, n).total; }
+size_t ptc::stack_distance_points_bytes(uint64_t n) { return wm_layout(nullptr, n).total; }
 
-extern "C" ptc_status ptc_stack_distance(const uint32_t* prev, uint64_t n, uint32_t* dist_out, void* ws,
-                                         size_t ws_bytes, void* stream) {
-  if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
-  if (n == 0) return PTC_OK;
-  if (!prev || !dist_out) return PTC_ERR_INVALID_ARG;
+// The matrix over every access (argument checks are the caller's).
+ptc_status ptc::stack_distance_points(const uint32_t* prev, uint64_t n, uint32_t* dist_out, void* ws,
+                                      size_t ws_bytes, cudaStream_t s) {
   if (!ws_ok(ws, ws_bytes, wm_layout(nullptr, n).total)) return PTC_ERR_WORKSPACE;
-  cudaStream_t s = (cudaStream_t)stream;
   const WmLayout W = wm_layout(ws, n);
   if (begin_call(ws, W.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
   if (cudaMemsetAsync(W.bits, 0, sizeof(uint32_t) * (uint64_t)W.L * W.lw, s) != cudaSuccess) return PTC_ERR_CUDA;
