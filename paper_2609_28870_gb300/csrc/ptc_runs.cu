@@ -38,7 +38,13 @@
 //                  per-tile zero counts (four atomics per tile)
 //   k_runs_query   one thread per run: the distance of its head
 //   k_runs_expand  every access takes its run's distance
+#include <cooperative_groups.h>
+
+#include <utility>
+
 #include "ptc_internal.h"
+
+namespace cg = cooperative_groups;
 
 namespace ptc {
 namespace {
@@ -326,6 +332,156 @@ __global__ void __launch_bounds__(kRT) k_runs_level(LevelArgs a) {
   }
 }
 
+// All L levels in one launch of one thread-block cluster when the runs fit in
+// its shared memory.  CTA c owns positions [c S, c S + S) of every level's
+// order.  A level: read the slice, stable-partition it locally (zeros, then
+// ones) into the same buffer, publish the CTA's (zeros, zero weight), and
+// after a cluster barrier copy the two partitioned segments, which are
+// contiguous in the next level's order, into their owners' other buffer with
+// coalesced distributed-shared-memory stores; a second barrier ends the level.
+// Same (Z, W) arrays as k_runs_level.
+constexpr int kCT = 1024;           // threads per CTA of the cluster
+constexpr int kCPer = 8;            // most elements a thread holds (one per round)
+constexpr int kCSlice = kCT * kCPer;
+constexpr int kCMax = 16;           // largest cluster (above 8 needs the non-portable attribute)
+
+struct BuildArgs {
+  const uint32_t* rec_s;
+  const uint32_t* rec_a;
+  uint2* zw;
+  uint32_t R, L, slice;
+};
+
+__global__ void __launch_bounds__(kCT) k_runs_build_cluster(BuildArgs a) {
+  extern __shared__ uint2 s_dyn[];  // two buffers of `slice` (key, weight)
+  __shared__ unsigned long long s_rw[kCPer * 32];  // per (round, warp) (zeros, zero weight)
+  __shared__ unsigned long long s_warp[kCT / 32];
+  __shared__ unsigned long long s_tot, s_pre, s_all;
+  cg::cluster_group cl = cg::this_cluster();
+  const uint32_t rank = cl.block_rank(), C = cl.num_blocks();
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const uint32_t S = a.slice, base = rank * S;
+  const uint32_t cnt = base < a.R ? min(S, a.R - base) : 0u;
+  const uint32_t q = (S + kCT - 1) / kCT;  // rounds (the same in every CTA)
+  const float invS = 1.0f / (float)S;
+  for (uint32_t i = threadIdx.x; i < cnt; i += kCT) {
+    const uint32_t r = base + i;
+    const uint32_t st = a.rec_s[r], e = a.rec_s[r + 1], a0 = a.rec_a[r];
+    const uint32_t len = e - st;
+    s_dyn[i] = make_uint2(a0 ? a0 + len - 1 : 0u, len);
+  }
+  cl.sync();
+  for (uint32_t l = 0; l < a.L; ++l) {
+    uint2* cur = s_dyn + (l & 1) * S;
+    uint2* nxt = s_dyn + ((l + 1) & 1) * S;
+    const uint32_t shift = a.L - 1 - l;
+    // round k holds positions [k * kCT, k * kCT + kCT): lane order is index order
+    uint2 el[kCPer];
+    uint32_t lz[kCPer], lw[kCPer];
+#pragma unroll
+    for (int k = 0; k < kCPer; ++k) {
+      if (k >= (int)q) break;  // q is the same for the whole CTA
+      const uint32_t i = k * kCT + threadIdx.x;
+      const bool valid = i < cnt;
+      el[k] = valid ? cur[i] : make_uint2(0u, 0u);
+      const bool zero = valid && !((el[k].x >> shift) & 1u);
+      const uint32_t m = __ballot_sync(kFull, zero);
+      uint32_t wi = zero ? el[k].y : 0u;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(kFull, wi, o);
+        if (lane >= (uint32_t)o) wi += y;
+      }
+      lz[k] = __popc(m & lanemask_lt());
+      lw[k] = wi - (zero ? el[k].y : 0u);
+      if (lane == 31 && k < (int)q) s_rw[k * 32 + w] = pack_zw(__popc(m), wi);
+    }
+    __syncthreads();
+    // exclusive scan of the (round, warp) totals in index order
+    {
+      const uint32_t t = threadIdx.x;
+      const unsigned long long x = t < q * 32 ? s_rw[t] : 0ull;
+      unsigned long long incl = x;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long y = __shfl_up_sync(kFull, incl, o);
+        if (lane >= (uint32_t)o) incl += y;
+      }
+      if (lane == 31) s_warp[w] = incl;
+      __syncthreads();
+      unsigned long long pre = 0, tot = 0;
+#pragma unroll
+      for (int ww = 0; ww < kCT / 32; ++ww) {
+        const unsigned long long v = s_warp[ww];
+        if (ww < (int)w) pre += v;
+        tot += v;
+      }
+      if (t < q * 32) s_rw[t] = pre + incl - x;
+      if (t == 0) s_tot = tot;
+      __syncthreads();
+    }
+    const uint32_t nz = (uint32_t)s_tot;
+    // local stable partition into `cur` (every element is in registers)
+#pragma unroll
+    for (int k = 0; k < kCPer; ++k) {
+      if (k >= (int)q) break;
+      const uint32_t i = k * kCT + threadIdx.x;
+      if (i < cnt) {
+        const unsigned long long rw = s_rw[k * 32 + w];
+        lz[k] += (uint32_t)rw;
+        lw[k] += (uint32_t)(rw >> 32);
+        const bool zero = !((el[k].x >> shift) & 1u);
+        cur[zero ? lz[k] : nz + (i - lz[k])] = el[k];
+      }
+    }
+    cl.sync();  // every CTA's total is published and every slice partitioned
+    if (w == 0) {
+      const unsigned long long v = lane < C ? *cl.map_shared_rank(&s_tot, lane) : 0ull;
+      unsigned long long in = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long y = __shfl_up_sync(kFull, in, o);
+        if (lane >= (uint32_t)o) in += y;
+      }
+      if (lane == rank) s_pre = in - v;
+      if (lane == 31) s_all = in;
+    }
+    __syncthreads();
+    const uint32_t Zpre = (uint32_t)s_pre, Wpre = (uint32_t)(s_pre >> 32), Zc = (uint32_t)s_all;
+    if (l + 1 < a.L) {
+      // zeros go to [Zpre, Zpre + nz), ones to [Zc + base - Zpre, ...)
+      const uint32_t one0 = Zc + (base - Zpre);
+      for (uint32_t j = threadIdx.x; j < cnt; j += kCT) {
+        const uint32_t dst = j < nz ? Zpre + j : one0 + (j - nz);
+        // dst / S through a float reciprocal (dst < 2^24, so dst is exact in
+        // a float and the estimate is off by at most one)
+        int32_t owner = (int32_t)((float)dst * invS);
+        int32_t off = (int32_t)dst - owner * (int32_t)S;
+        if (off < 0) {
+          --owner;
+          off += (int32_t)S;
+        } else if (off >= (int32_t)S) {
+          ++owner;
+          off -= (int32_t)S;
+        }
+        if (dst < a.R) *cl.map_shared_rank(&nxt[off], owner) = cur[j];
+      }
+    }
+    // the barrier orders the copies above; the (Z, W) stores, read only by
+    // the next kernel, go out while the other CTAs arrive
+    auto token = cl.barrier_arrive();
+    uint2* zl = a.zw + (size_t)l * (a.R + 1);
+#pragma unroll
+    for (int k = 0; k < kCPer; ++k) {
+      if (k >= (int)q) break;
+      const uint32_t i = k * kCT + threadIdx.x;
+      if (i < cnt) zl[base + i] = make_uint2(Zpre + lz[k], Wpre + lw[k]);
+    }
+    if (rank == 0 && threadIdx.x == 0) zl[a.R] = make_uint2(Zc, (uint32_t)(s_all >> 32));
+    cl.barrier_wait(std::move(token));  // the next level's order is in place
+  }
+}
+
 struct QueryArgs {
   const uint32_t* rec_s;
   const uint32_t* rec_a;
@@ -472,26 +628,71 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   if (cudaMemsetAsync(W.done, 0, 64 * sizeof(uint32_t), s) != cudaSuccess) return PTC_ERR_CUDA;
   const uint32_t R32 = (uint32_t)R, T = W.rtiles, L = W.L;
   const size_t tstride = (size_t)T + 1;
-  PTC_LAUNCH("k_runs_init", s,
-             k_runs_init<<<T, kRT, 0, s>>>(W.rec_s, W.rec_a, W.k0, W.w0, W.acc, W.pre, &W.done[0], R32, T, L - 1));
-  uint32_t* keys[2] = {W.k0, W.k1};
-  uint32_t* wts[2] = {W.w0, W.w1};
-  for (uint32_t l = 0; l < L; ++l) {
-    const bool last = l + 1 == L;
-    LevelArgs a;
-    a.key_in = keys[l & 1];
-    a.wt_in = wts[l & 1];
-    a.key_out = last ? nullptr : keys[(l + 1) & 1];
-    a.wt_out = last ? nullptr : wts[(l + 1) & 1];
-    a.zw = W.zw + (size_t)l * (R + 1);
-    a.pre = W.pre + (size_t)l * tstride;
-    a.acc_next = last ? nullptr : W.acc + (size_t)(l + 1) * tstride;
-    a.pre_next = last ? nullptr : W.pre + (size_t)(l + 1) * tstride;
-    a.done = &W.done[1 + l];
-    a.R = R32;
-    a.ntiles = T;
-    a.shift = L - 1 - l;
-    PTC_LAUNCH("k_runs_level", s, k_runs_level<<<T, kRT, 0, s>>>(a));
+  // one cluster when the runs fit in its shared memory, else one launch per level
+  bool built = false;
+  static int attrs_set = -1;  // per process: the attributes belong to the device function
+  if (attrs_set < 0)
+    attrs_set = cudaFuncSetAttribute(k_runs_build_cluster, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)(2 * kCSlice * sizeof(uint2))) == cudaSuccess &&
+                cudaFuncSetAttribute(k_runs_build_cluster, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) ==
+                    cudaSuccess;
+  for (uint32_t cmax = kCMax; attrs_set == 1 && !built && cmax >= 8; cmax /= 2) {
+    uint32_t C = ceil_div_u32(R, 2048);  // about two runs per thread
+    if (C > cmax) C = cmax;
+    if ((uint64_t)C * kCSlice < R) continue;
+    BuildArgs b;
+    b.rec_s = W.rec_s;
+    b.rec_a = W.rec_a;
+    b.zw = W.zw;
+    b.R = R32;
+    b.L = L;
+    b.slice = ceil_div_u32(R, C);
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = C;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(C);
+    cfg.blockDim = dim3(kCT);
+    cfg.dynamicSmemBytes = 2 * (size_t)b.slice * sizeof(uint2);
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, k_runs_build_cluster, &cfg) != cudaSuccess || clusters < 1) {
+      (void)cudaGetLastError();
+      continue;
+    }
+    cudaError_t e = cudaSuccess;
+    PTC_LAUNCH("k_runs_build_cluster", s, e = cudaLaunchKernelEx(&cfg, k_runs_build_cluster, b));
+    if (e == cudaSuccess)
+      built = true;
+    else
+      (void)cudaGetLastError();
+  }
+  if (!built) {
+    PTC_LAUNCH("k_runs_init", s,
+               k_runs_init<<<T, kRT, 0, s>>>(W.rec_s, W.rec_a, W.k0, W.w0, W.acc, W.pre, &W.done[0], R32, T, L - 1));
+    uint32_t* keys[2] = {W.k0, W.k1};
+    uint32_t* wts[2] = {W.w0, W.w1};
+    for (uint32_t l = 0; l < L; ++l) {
+      const bool last = l + 1 == L;
+      LevelArgs a;
+      a.key_in = keys[l & 1];
+      a.wt_in = wts[l & 1];
+      a.key_out = last ? nullptr : keys[(l + 1) & 1];
+      a.wt_out = last ? nullptr : wts[(l + 1) & 1];
+      a.zw = W.zw + (size_t)l * (R + 1);
+      a.pre = W.pre + (size_t)l * tstride;
+      a.acc_next = last ? nullptr : W.acc + (size_t)(l + 1) * tstride;
+      a.pre_next = last ? nullptr : W.pre + (size_t)(l + 1) * tstride;
+      a.done = &W.done[1 + l];
+      a.R = R32;
+      a.ntiles = T;
+      a.shift = L - 1 - l;
+      PTC_LAUNCH("k_runs_level", s, k_runs_level<<<T, kRT, 0, s>>>(a));
+    }
   }
   QueryArgs q;
   q.rec_s = W.rec_s;

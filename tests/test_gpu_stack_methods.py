@@ -103,3 +103,24 @@ def test_forced_runs_with_a_small_workspace_is_refused():
     assert rc == 0 and np.array_equal(ptc.u32(dist), want)
     rc = L.ptc_stack_distance_ex(p.data_ptr(), prev.size, dist.data_ptr(), 7, big.data_ptr(), big.numel(), stream)
     assert ptc.STATUS[rc] == "PTC_ERR_INVALID_ARG"
+
+
+def test_many_runs_take_the_per_level_build():
+    """More runs than one cluster's shared memory holds (131,072): the matrix
+    over runs is built one level per launch; a random reuse array with short
+    runs, forced onto the matrix over runs."""
+    import torch
+    import paper_2609_28870_gb300 as ptc
+    rng = np.random.default_rng(11)
+    ids = rng.integers(0, 60000, size=300000).astype(np.uint32)
+    _, first = np.unique(ids, return_index=True)
+    order = np.argsort(np.argsort(first))
+    dense = np.empty_like(ids)
+    remap = np.empty(ids.max() + 1, dtype=np.uint32)
+    remap[np.unique(ids)] = order.astype(np.uint32)
+    dense = remap[ids]
+    prev, _ = oracle.reuse(dense, int(dense.max()) + 1)
+    want = oracle.sd_fenwick(prev)
+    p = ptc.to_device_u32(prev)
+    got = ptc.u32(ptc.ptc_stack_distance(p, method=ptc.PTC_SD_RUNS))
+    assert np.array_equal(got, want)
