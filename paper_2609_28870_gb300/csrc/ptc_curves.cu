@@ -36,10 +36,11 @@ __global__ void k_heads(const uint64_t* __restrict__ blk_off, uint32_t R, uint64
   if (b > a) atomicOr(&bitmap[a >> 5], 1u << (a & 31));
 }
 
-struct RunMax {  // (segment-start flag, running max, start index of the segment)
-  uint64_t m;
-  uint64_t start;
-  uint64_t f;
+struct RunMax {  // (segment-start flag, running max, start index of the segment); n < 2^32 - 1
+  uint32_t m;
+  uint32_t start;
+  uint32_t f;
+  uint32_t pad;
 };
 struct RunMaxOp {
   __device__ RunMax operator()(const RunMax& a, const RunMax& b) const {
@@ -47,13 +48,14 @@ struct RunMaxOp {
     r.f = a.f | b.f;
     r.m = b.f ? b.m : (a.m > b.m ? a.m : b.m);
     r.start = b.f ? b.start : a.start;
+    r.pad = 0;
     return r;
   }
 };
 
 struct CurveArgs {
   const uint32_t* dist;
-  uint64_t n;
+  uint32_t n;
   const uint32_t* bitmap;
   const uint64_t* caps;  // device copy of the grid
   uint32_t G;
@@ -66,7 +68,7 @@ struct CurveArgs {
 // Loads the kCvPer distances of this thread and the head bits of its range,
 // and folds them into the thread's running max (with the segment start).
 __device__ __forceinline__ void load_run(const uint32_t* __restrict__ dist, const uint32_t* __restrict__ bitmap,
-                                         uint64_t n, uint64_t i0, uint64_t (&e)[kCvPer], uint64_t (&st_idx)[kCvPer],
+                                         uint32_t n, uint32_t i0, uint32_t (&e)[kCvPer], uint32_t (&st_idx)[kCvPer],
                                          uint32_t& has_head, RunMax& loc) {
   uint32_t d[kCvPer];
   if (i0 + kCvPer <= n && ((reinterpret_cast<uintptr_t>(dist) & 15) == 0)) {
@@ -79,11 +81,11 @@ __device__ __forceinline__ void load_run(const uint32_t* __restrict__ dist, cons
     for (int j = 0; j < kCvPer; ++j) d[j] = i0 + j < n ? dist[i0 + j] : 0u;
   }
   const uint32_t heads = i0 < n ? (bitmap[i0 >> 5] >> (i0 & 31)) & 0xFFu : 0u;
-  loc = RunMax{0, 0, 0};
+  loc = RunMax{0, 0, 0, 0};
   has_head = 0;
 #pragma unroll
   for (int j = 0; j < kCvPer; ++j) {
-    const uint64_t dv = (i0 + j < n) ? d[j] : 0u;
+    const uint32_t dv = (i0 + j < n) ? d[j] : 0u;
     if ((heads >> j) & 1u) {
       loc.f = 1;
       loc.m = dv;
@@ -97,6 +99,15 @@ __device__ __forceinline__ void load_run(const uint32_t* __restrict__ dist, cons
   }
 }
 
+__device__ __forceinline__ RunMax shfl_up_rm(const RunMax& x, int o) {
+  RunMax y;
+  y.m = __shfl_up_sync(kFull, x.m, o);
+  y.start = __shfl_up_sync(kFull, x.start, o);
+  y.f = __shfl_up_sync(kFull, x.f, o);
+  y.pad = 0;
+  return y;
+}
+
 // CTA-wide inclusive segmented scan of the thread aggregates: returns the
 // thread's inclusive value within its warp in *x and leaves the inclusive value
 // over warps in s_w (s_w[last] is the tile aggregate).
@@ -105,22 +116,16 @@ __device__ __forceinline__ void cta_runmax_scan(RunMax& x, RunMax* s_w) {
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    RunMax y;
-    y.m = __shfl_up_sync(kFull, x.m, o);
-    y.start = __shfl_up_sync(kFull, x.start, o);
-    y.f = __shfl_up_sync(kFull, x.f, o);
+    const RunMax y = shfl_up_rm(x, o);
     if (lane >= (uint32_t)o) x = op(y, x);
   }
   if (lane == 31) s_w[w] = x;
   __syncthreads();
   if (w == 0) {
-    RunMax z = lane < kCvThreads / 32 ? s_w[lane] : RunMax{0, 0, 0};
+    RunMax z = lane < kCvThreads / 32 ? s_w[lane] : RunMax{0, 0, 0, 0};
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      RunMax y;
-      y.m = __shfl_up_sync(kFull, z.m, o);
-      y.start = __shfl_up_sync(kFull, z.start, o);
-      y.f = __shfl_up_sync(kFull, z.f, o);
+      const RunMax y = shfl_up_rm(z, o);
       if (lane >= (uint32_t)o) z = op(y, z);
     }
     if (lane < kCvThreads / 32) s_w[lane] = z;
@@ -130,12 +135,12 @@ __device__ __forceinline__ void cta_runmax_scan(RunMax& x, RunMax* s_w) {
 
 // Pass 1: every tile's aggregate (request start seen?, running max since the
 // last start, index of that start).  Tiles are independent.
-__global__ void __launch_bounds__(kCvThreads) k_curves_agg(const uint32_t* __restrict__ dist, uint64_t n,
+__global__ void __launch_bounds__(kCvThreads) k_curves_agg(const uint32_t* __restrict__ dist, uint32_t n,
                                                            const uint32_t* __restrict__ bitmap,
                                                            RunMax* __restrict__ tile_agg) {
   __shared__ RunMax s_w[kCvThreads / 32];
-  const uint64_t i0 = (uint64_t)blockIdx.x * kCvTile + (uint64_t)threadIdx.x * kCvPer;
-  uint64_t e[kCvPer], st_idx[kCvPer];
+  const uint32_t i0 = blockIdx.x * kCvTile + threadIdx.x * kCvPer;
+  uint32_t e[kCvPer], st_idx[kCvPer];
   uint32_t has_head;
   RunMax x;
   load_run(dist, bitmap, n, i0, e, st_idx, has_head, x);
@@ -143,6 +148,9 @@ __global__ void __launch_bounds__(kCvThreads) k_curves_agg(const uint32_t* __res
   if (threadIdx.x == 0) tile_agg[blockIdx.x] = s_w[kCvThreads / 32 - 1];
 }
 
+// Persistent: each CTA walks tiles blockIdx.x, blockIdx.x + gridDim.x, ...
+// and keeps its bin histograms in shared memory across them, so the global
+// bins see one atomic per CTA and bin rather than per tile.
 __global__ void __launch_bounds__(kCvThreads) k_curves(CurveArgs a) {
   __shared__ uint32_t s_cap[PTC_MAX_CAPACITIES];
   __shared__ uint32_t s_cnt[PTC_MAX_CAPACITIES + 1];
@@ -156,92 +164,111 @@ __global__ void __launch_bounds__(kCvThreads) k_curves(CurveArgs a) {
     s_cnt[g] = 0;
     s_ks[g] = 0;
   }
-  const uint32_t tile = blockIdx.x;
-  const uint64_t i0 = (uint64_t)tile * kCvTile + (uint64_t)threadIdx.x * kCvPer;
-  uint64_t e[kCvPer], st_idx[kCvPer];
-  uint32_t has_head;
-  RunMax loc;
-  load_run(a.dist, a.bitmap, a.n, i0, e, st_idx, has_head, loc);
+  const uint32_t ntiles = (a.n + kCvTile - 1) / kCvTile;
   RunMaxOp op;
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  RunMax x = loc;
-  cta_runmax_scan(x, s_w);
-  // carry: fold of the aggregates of the tiles before this one, back to the
-  // nearest tile where a request starts (all written by k_curves_agg)
-  if (w == 0) {
-    RunMax acc{0, 0, 0};
-    for (int64_t base = (int64_t)tile - 1; base >= 0; base -= 32) {
-      const int64_t idx = base - (int64_t)lane;
-      RunMax g{0, 0, 0};
-      if (idx >= 0) g = a.tile_agg[idx];
-      const uint32_t heads = __ballot_sync(kFull, idx >= 0 && g.f);
-      const uint32_t first = heads ? (uint32_t)(__ffs(heads) - 1) : 31u;
-      if (lane > first) g = RunMax{0, 0, 0};
+  for (uint32_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+    const uint32_t i0 = tile * kCvTile + threadIdx.x * kCvPer;
+    uint32_t e[kCvPer], st_idx[kCvPer];
+    uint32_t has_head;
+    RunMax loc;
+    load_run(a.dist, a.bitmap, a.n, i0, e, st_idx, has_head, loc);
+    RunMax x = loc;
+    cta_runmax_scan(x, s_w);
+    // carry: fold of the aggregates of the tiles before this one, back to the
+    // nearest tile where a request starts (all written by k_curves_agg)
+    if (w == 0) {
+      RunMax acc{0, 0, 0, 0};
+      for (int64_t base = (int64_t)tile - 1; base >= 0; base -= 32) {
+        const int64_t idx = base - (int64_t)lane;
+        RunMax g{0, 0, 0, 0};
+        if (idx >= 0) g = a.tile_agg[idx];
+        const uint32_t heads = __ballot_sync(kFull, idx >= 0 && g.f);
+        const uint32_t first = heads ? (uint32_t)(__ffs(heads) - 1) : 31u;
+        if (lane > first) g = RunMax{0, 0, 0, 0};
 #pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const RunMax y = shfl_down_payload(g, o);
-        if (lane + o < 32) g = op(y, g);
+        for (int o = 1; o < 32; o <<= 1) {
+          const RunMax y = shfl_down_payload(g, o);
+          if (lane + o < 32) g = op(y, g);
+        }
+        acc = op(shfl_payload(g, 0), acc);
+        if (heads) break;
       }
-      acc = op(shfl_payload(g, 0), acc);
-      if (heads) break;
+      if (lane == 0) s_carry = acc;
     }
-    if (lane == 0) s_carry = acc;
-  }
-  __syncthreads();
-  // exclusive prefix of this thread = carry (+) warps before (+) lanes before
-  RunMax pre = s_carry;
-  if (w > 0) pre = op(pre, s_w[w - 1]);
-  {
-    RunMax y;
-    y.m = __shfl_up_sync(kFull, x.m, 1);
-    y.start = __shfl_up_sync(kFull, x.start, 1);
-    y.f = __shfl_up_sync(kFull, x.f, 1);
-    if (lane > 0) pre = op(pre, y);
-  }
+    __syncthreads();
+    // exclusive prefix of this thread = carry (+) warps before (+) lanes before
+    RunMax pre = s_carry;
+    if (w > 0) pre = op(pre, s_w[w - 1]);
+    {
+      const RunMax y = shfl_up_rm(x, 1);
+      if (lane > 0) pre = op(pre, y);
+    }
 
-  // bin and accumulate with run merging
-  uint32_t cur_g = 0xFFFFFFFFu, run_c = 0;
-  unsigned long long run_k = 0;
+    // bin and accumulate; consecutive accesses mostly share e (runs), so the
+    // bin is looked up only when e changes and counts merge until the bin does
+    uint32_t cur_g = 0xFFFFFFFFu, run_c = 0, last_e = 0xFFFFFFFFu, last_g = G;
+    unsigned long long run_k = 0;
 #pragma unroll
-  for (int j = 0; j < kCvPer; ++j) {
-    if (i0 + j >= a.n) break;
-    uint64_t ej = e[j], sj = st_idx[j];
-    if (!((has_head >> j) & 1u)) {
-      ej = pre.m > ej ? pre.m : ej;
-      sj = pre.start;
-    }
-    uint32_t g;
-    if (ej >= (uint64_t)kNone) {
-      g = G;
-    } else {  // first capacity >= ej
-      uint32_t lo = 0, hi = G;
-      while (lo < hi) {
-        const uint32_t mid = (lo + hi) >> 1;
-        if (s_cap[mid] >= (uint32_t)ej)
-          hi = mid;
-        else
-          lo = mid + 1;
+    for (int j = 0; j < kCvPer; ++j) {
+      if (i0 + j >= a.n) break;
+      uint32_t ej = e[j], sj = st_idx[j];
+      if (!((has_head >> j) & 1u)) {
+        ej = pre.m > ej ? pre.m : ej;
+        sj = pre.start;
       }
-      g = lo;
-    }
-    const unsigned long long k = (i0 + j) - sj;
-    if (g != cur_g) {
-      if (run_c) {
-        atomicAdd(&s_cnt[cur_g], run_c);
-        atomicAdd(&s_ks[cur_g], run_k);
+      uint32_t g = last_g;
+      if (ej != last_e) {
+        if (ej == kNone) {
+          g = G;
+        } else {  // first capacity >= ej
+          uint32_t lo = 0, hi = G;
+          while (lo < hi) {
+            const uint32_t mid = (lo + hi) >> 1;
+            if (s_cap[mid] >= ej)
+              hi = mid;
+            else
+              lo = mid + 1;
+          }
+          g = lo;
+        }
+        last_e = ej;
+        last_g = g;
       }
-      cur_g = g;
-      run_c = 0;
-      run_k = 0;
+      const uint32_t k = (i0 + j) - sj;
+      if (g != cur_g) {
+        if (run_c) {
+          atomicAdd(&s_cnt[cur_g], run_c);
+          atomicAdd(&s_ks[cur_g], run_k);
+        }
+        cur_g = g;
+        run_c = 0;
+        run_k = 0;
+      }
+      ++run_c;
+      run_k += k;
     }
-    ++run_c;
-    run_k += k;
+    // the open run of every lane; inside long runs the whole warp shares one
+    // bin, so it sums across lanes and adds once
+    const uint32_t g0 = __shfl_sync(kFull, cur_g, 0);
+    if (__all_sync(kFull, cur_g == g0 || run_c == 0)) {
+      uint32_t c = run_c;
+      unsigned long long kk = run_k;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        c += __shfl_xor_sync(kFull, c, o);
+        kk += __shfl_xor_sync(kFull, kk, o);
+      }
+      if (lane == 0 && c) {
+        atomicAdd(&s_cnt[g0], c);
+        atomicAdd(&s_ks[g0], kk);
+      }
+    } else if (run_c) {
+      atomicAdd(&s_cnt[cur_g], run_c);
+      atomicAdd(&s_ks[cur_g], run_k);
+    }
+    __syncthreads();  // s_w and s_carry are reused by the next tile
   }
-  if (run_c) {
-    atomicAdd(&s_cnt[cur_g], run_c);
-    atomicAdd(&s_ks[cur_g], run_k);
-  }
-  __syncthreads();
   for (uint32_t g = threadIdx.x; g <= G; g += kCvThreads) {
     if (s_cnt[g]) {
       atomicAdd(&a.cnt[g], (unsigned long long)s_cnt[g]);
@@ -285,9 +312,7 @@ struct CurvesLayout {
   unsigned long long* cnt;
   unsigned long long* ksum;
   uint32_t* bitmap;
-  uint32_t* lb_status;
   RunMax* lb_agg;
-  RunMax* lb_incl;
   uint64_t* caps;
   uint64_t* out;
   size_t zero_bytes;
@@ -302,10 +327,8 @@ CurvesLayout curves_layout(void* ws, uint64_t n, uint32_t G) {
   L.cnt = cv.take<unsigned long long>(PTC_MAX_CAPACITIES + 1);
   L.ksum = cv.take<unsigned long long>(PTC_MAX_CAPACITIES + 1);
   L.bitmap = cv.take<uint32_t>(n / 32 + 2);
-  L.lb_status = cv.take<uint32_t>(tiles);
   L.zero_bytes = cv.off;
   L.lb_agg = cv.take<RunMax>(tiles);
-  L.lb_incl = cv.take<RunMax>(tiles);  // unused; keeps the layout (and the no-alloc limit) unchanged
   L.caps = cv.take<uint64_t>(PTC_MAX_CAPACITIES);
   L.out = cv.take<uint64_t>(3 * PTC_MAX_CAPACITIES + 2);
   L.total = cv.bytes();
@@ -363,7 +386,7 @@ extern "C" ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_
     PTC_LAUNCH("k_heads", s, k_heads<<<ceil_div_u32(n_req, 256), 256, 0, s>>>(req_blk_off, n_req, n, L.bitmap, L.st));
     CurveArgs a;
     a.dist = dist;
-    a.n = n;
+    a.n = (uint32_t)n;
     a.bitmap = L.bitmap;
     a.caps = L.caps;
     a.G = n_cap;
@@ -372,8 +395,10 @@ extern "C" ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_
     a.tile_agg = L.lb_agg;
     a.st = L.st;
     PTC_LAUNCH("k_curves_agg", s,
-               k_curves_agg<<<ceil_div_u32(n, kCvTile), kCvThreads, 0, s>>>(dist, n, L.bitmap, L.lb_agg));
-    PTC_LAUNCH("k_curves", s, k_curves<<<ceil_div_u32(n, kCvTile), kCvThreads, 0, s>>>(a));
+               k_curves_agg<<<ceil_div_u32(n, kCvTile), kCvThreads, 0, s>>>(dist, (uint32_t)n, L.bitmap, L.lb_agg));
+    const uint32_t tiles = ceil_div_u32(n, kCvTile);
+    const uint32_t grid = tiles < (uint32_t)(2 * num_sms()) ? tiles : (uint32_t)(2 * num_sms());
+    PTC_LAUNCH("k_curves", s, k_curves<<<grid, kCvThreads, 0, s>>>(a));
   }
   PTC_LAUNCH("k_finalize", s, k_finalize<<<1, 32, 0, s>>>(L.cnt, L.ksum, n_cap, alpha, beta, L.out));
   static thread_local uint64_t host_out[3 * PTC_MAX_CAPACITIES + 2];

@@ -31,8 +31,9 @@
 // (Z, W).  A count of keys < x over [lo, hi) walks the L levels; where x has a
 // one bit, the zeros of the current range (all smaller) add their weight.
 //
-//   k_runs_mark    run starts: bitmap, run index per 32-position word, run
-//                  (start, first value) records; one look-back pass
+//   k_runs_count   run starts per tile; the last CTA scans the tile counts
+//   k_runs_mark    run starts again: bitmap, run index per 32-position word,
+//                  run (start, first value) records
 //   k_runs_init    level-0 keys and weights, per-tile zero counts / weights
 //   k_runs_level   one level: (Z, W), stable partition, the next level's
 //                  per-tile zero counts (four atomics per tile)
@@ -55,7 +56,6 @@ constexpr int kMTile = kMT * kMR;  // 2048 positions; warp w owns [256 w, 256 w 
 constexpr int kRT = 256;           // level tiles: threads
 constexpr int kRPer = 8;           // runs per thread (consecutive)
 constexpr int kRTile = kRT * kRPer;
-constexpr uint32_t kMarkEpoch = 1;
 
 __device__ __forceinline__ uint32_t vval(uint32_t p) { return p == kNone ? 0u : p + 1u; }
 
@@ -67,25 +67,22 @@ struct MarkArgs {
   uint32_t* wpre;     // runs starting before each word
   uint32_t* rec_s;    // start of each run (rec_s[R] = n)
   uint32_t* rec_a;    // value at the start of each run
-  uint64_t* lb;       // look-back words, one per tile
+  uint32_t* tcnt;     // run starts in each tile
+  uint32_t* tpre;     // runs starting before each tile; tpre[ntiles] = R
+  uint32_t* done;
   DevStatus* st;      // value[1] <- R
 };
 
-__global__ void __launch_bounds__(kMT) k_runs_mark(MarkArgs a) {
-  __shared__ uint32_t s_wcnt[kMT / 32];
-  const uint32_t tile = next_tile(a.st, kMarkEpoch);
-  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  const uint32_t base = tile * kMTile + w * (32 * kMR);
-  uint32_t pv[kMR];
+// Run-start bits of the warp's 8 x 32 positions from `base` (the previous
+// access decides whether one continues a run).
+__device__ __forceinline__ void start_words(const MarkArgs& a, uint32_t base, uint32_t lane, uint32_t (&pv)[kMR],
+                                            uint32_t (&words)[kMR], bool& bad) {
 #pragma unroll
   for (int k = 0; k < kMR; ++k) {
     const uint32_t j = base + k * 32 + lane;
     pv[k] = j < a.n ? a.prev[j] : kNone;
   }
   const uint32_t left0 = (lane == 0 && base > 0 && base - 1 < a.n) ? a.prev[base - 1] : kNone;
-  uint32_t words[kMR];
-  uint32_t cnt = 0;
-  bool bad = false;
   uint32_t carry = vval(left0);  // value left of lane 0 (meaningful in lane 0 only)
 #pragma unroll
   for (int k = 0; k < kMR; ++k) {
@@ -98,19 +95,85 @@ __global__ void __launch_bounds__(kMT) k_runs_mark(MarkArgs a) {
     carry = __shfl_sync(kFull, v, 31);
     const bool cont = j > 0 && ((v == vl + 1 && vl != 0) || (v == 0 && vl == 0));
     words[k] = __ballot_sync(kFull, valid && !cont);
-    cnt += __popc(words[k]);
   }
+}
+
+// The calling CTA learns whether it is the last of the grid to get here.
+__device__ __forceinline__ bool last_cta(uint32_t* done) {
+  __shared__ uint32_t s_last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(done, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (s_last) __threadfence();
+  return s_last;
+}
+
+// Pass 1: run starts per tile; the last CTA turns them into tile prefixes.
+__global__ void __launch_bounds__(kMT) k_runs_count(MarkArgs a) {
+  __shared__ uint32_t s_wcnt[kMT / 32];
+  __shared__ uint32_t s_scan[kMT / 32];
+  const uint32_t tile = blockIdx.x;
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  uint32_t pv[kMR], words[kMR];
+  bool bad = false;
+  start_words(a, tile * kMTile + w * (32 * kMR), lane, pv, words, bad);
+  uint32_t cnt = 0;
+#pragma unroll
+  for (int k = 0; k < kMR; ++k) cnt += __popc(words[k]);
+  if (lane == 0) s_wcnt[w] = cnt;
+  if (bad) raise_err(a.st, kErrInvalid);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t t = 0;
+    for (int ww = 0; ww < kMT / 32; ++ww) t += s_wcnt[ww];
+    a.tcnt[tile] = t;
+  }
+  if (!last_cta(a.done)) return;
+  // exclusive prefix of the tile counts
+  const uint32_t T = a.ntiles, per = (T + kMT - 1) / kMT;
+  const uint32_t t0 = threadIdx.x * per, t1 = min(t0 + per, T);
+  uint32_t sum = 0;
+  for (uint32_t t = t0; t < t1; ++t) sum += __ldcg(&a.tcnt[t]);
+  uint32_t incl = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(kFull, incl, o);
+    if (lane >= (uint32_t)o) incl += y;
+  }
+  if (lane == 31) s_scan[w] = incl;
+  __syncthreads();
+  uint32_t run = incl - sum, total = 0;
+  for (int ww = 0; ww < kMT / 32; ++ww) {
+    if (ww < (int)w) run += s_scan[ww];
+    total += s_scan[ww];
+  }
+  for (uint32_t t = t0; t < t1; ++t) {
+    a.tpre[t] = run;
+    run += __ldcg(&a.tcnt[t]);
+  }
+  if (threadIdx.x == 0) {
+    a.tpre[T] = total;
+    a.st->value[1] = total;
+  }
+}
+
+// Pass 2: bitmap, run index per word, and the (start, first value) records.
+__global__ void __launch_bounds__(kMT) k_runs_mark(MarkArgs a) {
+  __shared__ uint32_t s_wcnt[kMT / 32];
+  const uint32_t tile = blockIdx.x;
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const uint32_t base = tile * kMTile + w * (32 * kMR);
+  uint32_t pv[kMR], words[kMR];
+  bool bad = false;
+  start_words(a, base, lane, pv, words, bad);
+  uint32_t cnt = 0;
+#pragma unroll
+  for (int k = 0; k < kMR; ++k) cnt += __popc(words[k]);
   if (lane == 0) s_wcnt[w] = cnt;
   __syncthreads();
-  uint32_t agg = 0, wpre_in_tile = 0;
-#pragma unroll
-  for (int ww = 0; ww < kMT / 32; ++ww) {
-    const uint32_t c = s_wcnt[ww];
-    if (ww < (int)w) wpre_in_tile += c;
-    agg += c;
-  }
-  const uint32_t tile_pre = (uint32_t)lookback_sum_cta(a.lb, tile, agg, kMarkEpoch, a.st);
-  uint32_t run = tile_pre + wpre_in_tile;
+  uint32_t run = a.tpre[tile];
+  for (int ww = 0; ww < (int)w; ++ww) run += s_wcnt[ww];
 #pragma unroll
   for (int k = 0; k < kMR; ++k) {
     const uint32_t j = base + k * 32 + lane;
@@ -125,12 +188,7 @@ __global__ void __launch_bounds__(kMT) k_runs_mark(MarkArgs a) {
     }
     run += __popc(words[k]);
   }
-  if (bad) raise_err(a.st, kErrInvalid);
-  if (tile == a.ntiles - 1 && threadIdx.x == 0) {
-    const uint32_t R = tile_pre + agg;
-    a.rec_s[R] = a.n;
-    a.st->value[1] = R;
-  }
+  if (tile == a.ntiles - 1 && threadIdx.x == 0) a.rec_s[a.tpre[a.ntiles]] = a.n;
 }
 
 // Exclusive scan over the threads of a 256-thread CTA.
@@ -181,17 +239,6 @@ __device__ void tile_prefix(const uint2* acc, uint2* pre, uint32_t ntiles, unsig
     run += pack_zw(v.x, v.y);
   }
   if (threadIdx.x == 0) pre[ntiles] = make_uint2((uint32_t)total, (uint32_t)(total >> 32));
-}
-
-// The calling CTA learns whether it is the last of the grid to get here.
-__device__ __forceinline__ bool last_cta(uint32_t* done) {
-  __shared__ uint32_t s_last;
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) s_last = atomicAdd(done, 1u) == gridDim.x - 1;
-  __syncthreads();
-  if (s_last) __threadfence();
-  return s_last;
 }
 
 struct LevelArgs {
@@ -554,7 +601,7 @@ uint32_t key_bits_n(uint64_t n) {  // keys and thresholds lie in [0, n]
 struct RunsLayout {
   DevStatus* st;
   uint32_t* done;
-  uint64_t* lb;
+  uint32_t *tcnt, *tpre;
   size_t zero_bytes;
   uint32_t *bits, *wpre, *rec_s, *rec_a;
   uint32_t *sd, *k0, *k1, *w0, *w1;
@@ -573,8 +620,9 @@ RunsLayout runs_layout(void* ws, uint64_t n, uint64_t R) {
   W.rtiles = ceil_div_u32(rr, kRTile);
   W.st = cv.take<DevStatus>(1);
   W.done = cv.take<uint32_t>(64);
-  W.lb = cv.take<uint64_t>(W.mtiles + 1);
   W.zero_bytes = cv.off;
+  W.tcnt = cv.take<uint32_t>(W.mtiles + 1);
+  W.tpre = cv.take<uint32_t>(W.mtiles + 1);
   W.bits = cv.take<uint32_t>(nn / 32 + 2);
   W.wpre = cv.take<uint32_t>(nn / 32 + 2);
   W.rec_s = cv.take<uint32_t>(nn + 1);
@@ -613,8 +661,11 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   m.wpre = M.wpre;
   m.rec_s = M.rec_s;
   m.rec_a = M.rec_a;
-  m.lb = M.lb;
+  m.tcnt = M.tcnt;
+  m.tpre = M.tpre;
+  m.done = &M.done[63];
   m.st = M.st;
+  PTC_LAUNCH("k_runs_count", s, k_runs_count<<<M.mtiles, kMT, 0, s>>>(m));
   PTC_LAUNCH("k_runs_mark", s, k_runs_mark<<<M.mtiles, kMT, 0, s>>>(m));
   DevStatus h;
   ptc_status rc = end_call(M.st, s, &h);
