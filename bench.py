@@ -129,7 +129,8 @@ def kernel_model_bytes(name, T, N, L, D):
 
 KERNEL_SOURCE = {
     "k_block_offsets": "ptc_hash.cu", "k_pow_tables": "ptc_hash.cu", "k_hash_local": "ptc_hash.cu",
-    "k_hash_chain": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu", "k_ids_rank": "ptc_ids.cu",
+    "k_hash_chain": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu", "k_ids_flags": "ptc_ids.cu",
+    "k_ids_wordpre": "ptc_ids.cu",
     "k_ids_gather": "ptc_ids.cu", "k_sort_count": "ptc_sort.cu", "k_sort_rowscan": "ptc_sort.cu",
     "k_sort_scatter": "ptc_sort.cu", "k_sort_links": "ptc_sort.cu", "k_wm_count0": "ptc_wavelet.cu",
     "k_wm_level": "ptc_wavelet.cu", "k_wm_dir": "ptc_wavelet.cu", "k_wm_heads": "ptc_wavelet.cu",

@@ -2,14 +2,16 @@
 // key is one cache object), and the exact check of those ids against tokens.
 //
 // ptc_assign_ids
-//   k_ids_insert   open-addressing table, 16-byte slots claimed with one
-//                  128-bit CAS: 96 key bits + the smallest access index seen
-//                  (lowered with a 32-bit atomicMin); linear probing.
-//   k_ids_rank     access i is a first occurrence iff its slot's index == i;
-//                  an exclusive scan of those flags (decoupled look-back)
-//                  numbers the keys in access order; first occurrences
-//                  publish their rank into the slot's id word.
-//   k_ids_gather   ids[i] = id word of i's slot.
+//   k_ids_insert   open-addressing table, 16-byte slots: 96 key bits + the
+//                  smallest access index seen.  A slot is read first; only an
+//                  empty (or half-written) slot is claimed with one 128-bit
+//                  CAS, and a stored index above i is lowered with atomicMin.
+//                  Linear probing.
+//   k_ids_flags    first[i] = index stored in i's slot; access i is a first
+//                  occurrence iff first[i] == i: a bitmap of those, counts
+//                  per tile, and (last CTA) the tile prefixes
+//   k_ids_wordpre  first occurrences before every 32-position word
+//   k_ids_gather   ids[i] = rank of first[i] among the first occurrences.
 // ptc_verify_ids
 //   k_verify_first first access of every id (atomicMin)
 //   k_verify       compares every access's B tokens and parent id with those
@@ -20,10 +22,6 @@ namespace ptc {
 namespace {
 
 constexpr int kInsThreads = 256;
-constexpr int kRankThreads = 512;
-constexpr int kRankPer = 8;
-constexpr int kRankTile = kRankThreads * kRankPer;
-constexpr int kEpochRank = 1;
 
 __device__ __forceinline__ ulonglong2 cas128(ulonglong2* addr, ulonglong2 cmp, ulonglong2 val) {
   ulonglong2 old;
@@ -46,10 +44,16 @@ __device__ __forceinline__ uint64_t home_slot(uint64_t h0, uint64_t h1, uint32_t
   return log2m ? z >> (64 - log2m) : 0;
 }
 
-__global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __restrict__ keys, uint64_t n,
+__device__ __forceinline__ ulonglong2 ld_slot(const ulonglong2* p) {
+  ulonglong2 v;
+  asm volatile("ld.relaxed.gpu.global.v2.u64 {%0, %1}, [%2];" : "=l"(v.x), "=l"(v.y) : "l"(p) : "memory");
+  return v;
+}
+
+__global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __restrict__ keys, uint32_t n,
                                                             ulonglong2* table, uint32_t log2m, uint64_t probe_cap,
                                                             uint32_t* __restrict__ slot_of, DevStatus* st) {
-  const uint64_t i = (uint64_t)blockIdx.x * kInsThreads + threadIdx.x;
+  const uint32_t i = blockIdx.x * kInsThreads + threadIdx.x;
   if (i >= n) return;
   const ulonglong2 k = keys[i];
   if (k.x >= kP61 || k.y >= kP61) {
@@ -58,21 +62,25 @@ __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __
     return;
   }
   // 96 key bits: all of h0 (61) + 35 bits of h1.  Word 0 is never all-ones
-  // because h0 < 2^61 - 1, so all-ones marks an empty slot.
+  // because h0 < 2^61 - 1, and word 1 of a filled slot holds an index below
+  // 2^32 - 1, so an all-ones word marks an empty or half-written slot.
   const uint64_t w0 = k.x | ((k.y & 7ULL) << 61);
   const uint32_t w1lo = (uint32_t)(k.y >> 3);
-  const ulonglong2 mine = make_ulonglong2(w0, (uint64_t)w1lo | ((uint64_t)(uint32_t)i << 32));
+  const ulonglong2 mine = make_ulonglong2(w0, (uint64_t)w1lo | ((uint64_t)i << 32));
   const ulonglong2 empty = make_ulonglong2(~0ULL, ~0ULL);
   const uint64_t mask = (1ULL << log2m) - 1;
   uint64_t pos = home_slot(k.x, k.y, log2m);
   for (uint64_t probe = 0; probe <= mask && probe < probe_cap; ++probe) {
-    const ulonglong2 old = cas128(&table[pos], empty, mine);
-    if (old.x == ~0ULL && old.y == ~0ULL) {
-      slot_of[i] = (uint32_t)pos;
-      return;
+    ulonglong2 cur = ld_slot(&table[pos]);
+    if (cur.x == ~0ULL || cur.y == ~0ULL) {  // empty, or being filled: settle it with the CAS
+      cur = cas128(&table[pos], empty, mine);
+      if (cur.x == ~0ULL && cur.y == ~0ULL) {
+        slot_of[i] = (uint32_t)pos;
+        return;
+      }
     }
-    if (old.x == w0 && (uint32_t)old.y == w1lo) {
-      if ((uint32_t)(old.y >> 32) > (uint32_t)i) atomicMin(reinterpret_cast<uint32_t*>(&table[pos]) + 3, (uint32_t)i);
+    if (cur.x == w0 && (uint32_t)cur.y == w1lo) {
+      if ((uint32_t)(cur.y >> 32) > i) atomicMin(reinterpret_cast<uint32_t*>(&table[pos]) + 3, i);
       slot_of[i] = (uint32_t)pos;
       return;
     }
@@ -82,69 +90,102 @@ __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __
   slot_of[i] = 0;
 }
 
-__device__ __forceinline__ uint64_t cta_exclusive_sum512(uint64_t v, uint64_t* total) {
-  __shared__ uint64_t s_w[kRankThreads / 32];
-  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  uint64_t x = v;
-#pragma unroll
-  for (int d = 1; d < 32; d <<= 1) {
-    uint64_t y = __shfl_up_sync(kFull, x, d);
-    if (lane >= (uint32_t)d) x += y;
-  }
-  if (lane == 31) s_w[w] = x;
-  __syncthreads();
-  if (w == 0) {
-    uint64_t t = lane < kRankThreads / 32 ? s_w[lane] : 0;
-#pragma unroll
-    for (int d = 1; d < 32; d <<= 1) {
-      uint64_t y = __shfl_up_sync(kFull, t, d);
-      if (lane >= (uint32_t)d) t += y;
-    }
-    if (lane < kRankThreads / 32) s_w[lane] = t;
-  }
-  __syncthreads();
-  *total = s_w[kRankThreads / 32 - 1];
-  return (w ? s_w[w - 1] : 0) + x - v;
-}
+constexpr int kFlT = 256;             // flags: threads per tile
+constexpr int kFlR = 8;               // rounds of 32 positions per warp
+constexpr int kFlTile = kFlT * kFlR;  // 2048 positions; warp w owns [256 w, 256 w + 256)
 
-__global__ void __launch_bounds__(kRankThreads) k_ids_rank(const ulonglong2* __restrict__ table,
-                                                           const uint32_t* __restrict__ slot_of, uint64_t n,
-                                                           uint32_t* __restrict__ slot_id, uint64_t* lb,
-                                                           DevStatus* st) {
-  const uint32_t tile = next_tile(st, kEpochRank);
-  const uint64_t i0 = (uint64_t)tile * kRankTile + (uint64_t)threadIdx.x * kRankPer;
-  uint32_t slots[kRankPer];
-  uint32_t flags = 0, cnt = 0;
+// first[i] (in place of slot_of[i]) and the first-occurrence bitmap; tile
+// counts, and the last CTA's tile prefixes (tpre[ntiles] = D).
+__global__ void __launch_bounds__(kFlT) k_ids_flags(const ulonglong2* __restrict__ table, uint32_t* slot_first,
+                                                   uint32_t n, uint32_t ntiles, uint32_t* __restrict__ bits,
+                                                   uint32_t* tcnt, uint32_t* tpre, uint32_t* done, DevStatus* st) {
+  __shared__ uint32_t s_w[kFlT / 32];
+  __shared__ uint32_t s_last;
+  const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const uint32_t base = tile * kFlTile + w * (32 * kFlR);
+  uint32_t cnt = 0;
 #pragma unroll
-  for (int j = 0; j < kRankPer; ++j) {
-    const uint64_t i = i0 + j;
-    slots[j] = 0;
+  for (int k = 0; k < kFlR; ++k) {
+    const uint32_t i = base + k * 32 + lane;
+    bool first = false;
     if (i < n) {
-      slots[j] = slot_of[i];
-      const uint32_t first = reinterpret_cast<const uint32_t*>(&table[slots[j]])[3];
-      if (first == (uint32_t)i) {
-        flags |= 1u << j;
-        ++cnt;
-      }
+      const uint32_t f = reinterpret_cast<const uint32_t*>(&table[slot_first[i]])[3];
+      slot_first[i] = f;
+      first = f == i;
     }
+    const uint32_t m = __ballot_sync(kFull, first);
+    if (lane == 0 && base + k * 32 < n) bits[(base + k * 32) >> 5] = m;
+    cnt += __popc(m);
   }
-  uint64_t total;
-  const uint64_t excl = cta_exclusive_sum512(cnt, &total);
-  uint64_t rank = lookback_sum_cta(lb, tile, total, kEpochRank, st) + excl;
+  if (lane == 0) s_w[w] = cnt;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t t = 0;
+    for (int ww = 0; ww < kFlT / 32; ++ww) t += s_w[ww];
+    tcnt[tile] = t;
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(done, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const uint32_t per = (ntiles + kFlT - 1) / kFlT;
+  const uint32_t t0 = threadIdx.x * per, t1 = min(t0 + per, ntiles);
+  uint32_t sum = 0;
+  for (uint32_t t = t0; t < t1; ++t) sum += __ldcg(&tcnt[t]);
+  uint32_t incl = sum;
 #pragma unroll
-  for (int j = 0; j < kRankPer; ++j) {
-    if (flags & (1u << j)) slot_id[slots[j]] = (uint32_t)rank++;
-    if (i0 + j + 1 == n) {
-      st->value[0] = rank;
-      if (rank >= (uint64_t)kNone) raise_err(st, kErrOverflow);
-    }
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(kFull, incl, o);
+    if (lane >= (uint32_t)o) incl += y;
+  }
+  __syncthreads();
+  if (lane == 31) s_w[w] = incl;
+  __syncthreads();
+  uint32_t run = incl - sum, total = 0;
+  for (int ww = 0; ww < kFlT / 32; ++ww) {
+    if (ww < (int)w) run += s_w[ww];
+    total += s_w[ww];
+  }
+  for (uint32_t t = t0; t < t1; ++t) {
+    tpre[t] = run;
+    run += __ldcg(&tcnt[t]);
+  }
+  if (threadIdx.x == 0) {
+    tpre[ntiles] = total;
+    st->value[0] = total;
   }
 }
 
-__global__ void k_ids_gather(const uint32_t* __restrict__ slot_of, const uint32_t* __restrict__ slot_id, uint64_t n,
-                             uint32_t* __restrict__ ids) {
-  const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i < n) ids[i] = slot_id[slot_of[i]];
+// First occurrences before every word: one warp per tile of 64 words.
+__global__ void k_ids_wordpre(const uint32_t* __restrict__ bits, const uint32_t* __restrict__ tpre, uint32_t nwords,
+                              uint32_t* __restrict__ wpre) {
+  const uint32_t warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  const uint32_t w0 = warp * (kFlTile / 32);
+  if (w0 >= nwords) return;
+  uint32_t run = tpre[warp];
+#pragma unroll
+  for (int h = 0; h < kFlTile / 32 / 32; ++h) {
+    const uint32_t wi = w0 + h * 32 + lane;
+    const uint32_t c = wi < nwords ? __popc(bits[wi]) : 0u;
+    uint32_t incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(kFull, incl, o);
+      if (lane >= (uint32_t)o) incl += y;
+    }
+    if (wi < nwords) wpre[wi] = run + incl - c;
+    run += __shfl_sync(kFull, incl, 31);
+  }
+}
+
+__global__ void k_ids_gather(const uint32_t* __restrict__ first, const uint32_t* __restrict__ bits,
+                             const uint32_t* __restrict__ wpre, uint32_t n, uint32_t* __restrict__ ids) {
+  const uint32_t i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const uint32_t f = first[i];
+  ids[i] = f < n ? wpre[f >> 5] + __popc(bits[f >> 5] & ((1u << (f & 31)) - 1u)) : kNone;
 }
 
 // Slots for n keys at most: the full table holds 1.5 n; the first attempt
@@ -163,10 +204,11 @@ uint32_t small_table_log2(uint64_t n) { return table_log2(n / 3 + 64); }
 
 struct IdsLayout {
   DevStatus* st;
-  uint64_t* lb;
+  uint32_t* done;
   ulonglong2* table;
-  uint32_t* slot_id;
-  uint32_t* slot_of;
+  uint32_t* slot_of;  // then first[i]
+  uint32_t *bits, *wpre, *tcnt, *tpre;
+  uint32_t ntiles, nwords;
   size_t zero_bytes;
   size_t total;
   uint32_t log2m;
@@ -177,12 +219,18 @@ IdsLayout ids_layout(void* ws, uint64_t n) {
   Carver cv(ws);
   L.log2m = full_table_log2(n);
   const uint64_t m = 1ULL << L.log2m;
+  const uint64_t nn = n ? n : 1;
+  L.ntiles = ceil_div_u32(nn, kFlTile);
+  L.nwords = ceil_div_u32(nn, 32);
   L.st = cv.take<DevStatus>(1);
-  L.lb = cv.take<uint64_t>(ceil_div_u32(n, kRankTile) + 1);
+  L.done = cv.take<uint32_t>(64);
   L.zero_bytes = cv.off;
   L.table = cv.take<ulonglong2>(m);
-  L.slot_id = cv.take<uint32_t>(m);
-  L.slot_of = cv.take<uint32_t>(n ? n : 1);
+  L.slot_of = cv.take<uint32_t>(nn);
+  L.bits = cv.take<uint32_t>(L.nwords + 1);
+  L.wpre = cv.take<uint32_t>(L.nwords + 1);
+  L.tcnt = cv.take<uint32_t>(L.ntiles + 1);
+  L.tpre = cv.take<uint32_t>(L.ntiles + 1);
   L.total = cv.bytes();
   return L;
 }
@@ -263,11 +311,16 @@ extern "C" ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t*
   auto run = [&](uint32_t log2m, uint64_t probe_cap) -> bool {
     if (cudaMemsetAsync(L.table, 0xFF, sizeof(ulonglong2) << log2m, s) != cudaSuccess) return false;
     const ulonglong2* k = reinterpret_cast<const ulonglong2*>(keys);
+    const uint32_t n32 = (uint32_t)n;
     PTC_LAUNCH("k_ids_insert", s, k_ids_insert<<<ceil_div_u32(n, kInsThreads), kInsThreads, 0, s>>>(
-                                      k, n, L.table, log2m, probe_cap, L.slot_of, L.st));
-    PTC_LAUNCH("k_ids_rank", s, k_ids_rank<<<ceil_div_u32(n, kRankTile), kRankThreads, 0, s>>>(
-                                    L.table, L.slot_of, n, L.slot_id, L.lb, L.st));
-    PTC_LAUNCH("k_ids_gather", s, k_ids_gather<<<ceil_div_u32(n, 256), 256, 0, s>>>(L.slot_of, L.slot_id, n, ids_out));
+                                      k, n32, L.table, log2m, probe_cap, L.slot_of, L.st));
+    PTC_LAUNCH("k_ids_flags", s, k_ids_flags<<<L.ntiles, kFlT, 0, s>>>(L.table, L.slot_of, n32, L.ntiles, L.bits,
+                                                                       L.tcnt, L.tpre, &L.done[0], L.st));
+    PTC_LAUNCH("k_ids_wordpre", s,
+               k_ids_wordpre<<<ceil_div_u32((uint64_t)L.ntiles * 32, 256), 256, 0, s>>>(L.bits, L.tpre, L.nwords,
+                                                                                        L.wpre));
+    PTC_LAUNCH("k_ids_gather", s,
+               k_ids_gather<<<ceil_div_u32(n, 256), 256, 0, s>>>(L.slot_of, L.bits, L.wpre, n32, ids_out));
     return true;
   };
   if (n > 0) {
