@@ -119,6 +119,8 @@ def kernel_model_bytes(name, T, N, L, D):
         "k_ids_insert": 16 * N,           # keys in
         "k_ids_gather": 4 * N,            # ids out
         "k_sort_scatter": 12 * N / sort_passes(D),  # ids in, prev / next out, spread over the passes
+        "k_ir_count": 4 * N,              # ids in (sort over id-runs)
+        "k_ir_fill": 8 * N,               # prev / next out (sort over id-runs)
         "k_wm_level": per_level,          # values in, partition + bit plane out
         "k_wm_heads": (8 + L / 8) * N,    # prev in, one read of the bit planes, distances out
         "k_runs_mark": 4 * N,             # prev in (matrix over runs)
@@ -132,7 +134,9 @@ KERNEL_SOURCE = {
     "k_hash_chain": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu", "k_ids_flags": "ptc_ids.cu",
     "k_ids_wordpre": "ptc_ids.cu",
     "k_ids_gather": "ptc_ids.cu", "k_sort_count": "ptc_sort.cu", "k_sort_rowscan": "ptc_sort.cu",
-    "k_sort_scatter": "ptc_sort.cu", "k_sort_links": "ptc_sort.cu", "k_wm_count0": "ptc_wavelet.cu",
+    "k_sort_scatter": "ptc_sort.cu", "k_sort_links": "ptc_sort.cu", "k_ir_count": "ptc_reuse.cu",
+    "k_ir_mark": "ptc_reuse.cu", "k_bm_count": "ptc_reuse.cu", "k_bm_words": "ptc_reuse.cu",
+    "k_ir_inc1": "ptc_reuse.cu", "k_ir_inc2": "ptc_reuse.cu", "k_ir_fill": "ptc_reuse.cu", "k_wm_count0": "ptc_wavelet.cu",
     "k_wm_level": "ptc_wavelet.cu", "k_wm_dir": "ptc_wavelet.cu", "k_wm_heads": "ptc_wavelet.cu",
     "k_wm_propagate": "ptc_wavelet.cu", "k_runs_mark": "ptc_runs.cu", "k_runs_count": "ptc_runs.cu", "k_runs_init": "ptc_runs.cu",
     "k_runs_level": "ptc_runs.cu", "k_runs_build_cluster": "ptc_runs.cu", "k_runs_query": "ptc_runs.cu", "k_runs_expand": "ptc_runs.cu", "k_heads": "ptc_curves.cu", "k_curves_agg": "ptc_curves.cu",

@@ -150,7 +150,10 @@ ptc_status ptc_verify_ids(const uint32_t* tokens, uint64_t n_tok, const uint64_t
  * Belady's policy needs the time until each block's next access).
  *   prev_out[i] = max{ j < i : ids[j] == ids[i] }, or PTC_NONE
  *   next_out[i] = min{ j > i : ids[j] == ids[i] }, or PTC_NONE
- * Computed from a stable radix sort of (id, i) pairs.
+ * Computed from a stable radix sort: of the runs of consecutive ids, cut
+ * into pieces that every run holds whole or not at all (one piece per
+ * (interval of id-space, run)), or, when those pieces exceed a quarter of
+ * the accesses, of every (id, i) pair.
  *
  *   ids        u32[n], every value < n_distinct (PTC_ERR_INVALID_ARG otherwise)
  *   prev_out, next_out  u32[n]
@@ -158,6 +161,17 @@ ptc_status ptc_verify_ids(const uint32_t* tokens, uint64_t n_tok, const uint64_t
 size_t ptc_reuse_indices_workspace_bytes(uint64_t n, uint64_t n_distinct);
 ptc_status ptc_reuse_indices(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev_out,
                              uint32_t* next_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * ptc_reuse_indices_ex — the same outputs with the sort chosen by the caller:
+ * PTC_REUSE_SORT sorts every (id, i); PTC_REUSE_RUNS sorts the pieces of the
+ * id-runs whatever their number; PTC_REUSE_AUTO is ptc_reuse_indices.
+ * Workspace: ptc_reuse_indices_ex_workspace_bytes(n, n_distinct, method).
+ */
+enum { PTC_REUSE_AUTO = 0, PTC_REUSE_SORT = 1, PTC_REUSE_RUNS = 2 };
+size_t ptc_reuse_indices_ex_workspace_bytes(uint64_t n, uint64_t n_distinct, int method);
+ptc_status ptc_reuse_indices_ex(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev_out,
+                                uint32_t* next_out, int method, void* ws, size_t ws_bytes, void* stream);
 
 /*
  * ptc_stack_distance — LRU stack distance of every access (App. B: the stack

@@ -29,6 +29,7 @@ from . import build as _build
 PTC_NONE = 0xFFFFFFFF
 PTC_COST_UNIFORM, PTC_COST_MEASURED, PTC_COST_LINEAR = 0, 1, 2
 PTC_SD_AUTO, PTC_SD_POINTS, PTC_SD_RUNS = 0, 1, 2
+PTC_REUSE_AUTO, PTC_REUSE_SORT, PTC_REUSE_RUNS = 0, 1, 2
 F_LIN = 6_600_000_000          # 2 x 3.3e9 active parameters, FLOPs per token
 F_ATTN = 4 * 48 * 32 * 128     # per attended position: 4 x layers x heads x head_dim
 MAX_CAPACITIES = 1024
@@ -101,6 +102,10 @@ def lib():
                 L.ptc_stack_distance_workspace_bytes.argtypes = [u64]
                 L.ptc_stack_distance.restype = st
                 L.ptc_stack_distance.argtypes = [vp, u64, vp, vp, sz, vp]
+                L.ptc_reuse_indices_ex_workspace_bytes.restype = sz
+                L.ptc_reuse_indices_ex_workspace_bytes.argtypes = [u64, u64, ctypes.c_int]
+                L.ptc_reuse_indices_ex.restype = st
+                L.ptc_reuse_indices_ex.argtypes = [vp, u64, u64, vp, vp, ctypes.c_int, vp, sz, vp]
                 L.ptc_stack_distance_ex_workspace_bytes.restype = sz
                 L.ptc_stack_distance_ex_workspace_bytes.argtypes = [u64, ctypes.c_int]
                 L.ptc_stack_distance_ex.restype = st
@@ -219,15 +224,24 @@ def ptc_verify_ids(tokens, req_tok_off, req_blk_off, block_size: int, ids: torch
     _check("ptc_verify_ids", rc)
 
 
-def ptc_reuse_indices(ids: torch.Tensor, n_distinct: int, ws: torch.Tensor | None = None):
-    """Previous / next use of every access.  Returns (prev int32[N], next int32[N])."""
+def ptc_reuse_indices(ids: torch.Tensor, n_distinct: int, ws: torch.Tensor | None = None, method: int | None = None):
+    """Previous / next use of every access.  Returns (prev int32[N], next int32[N]).
+    ``method`` (PTC_REUSE_AUTO / PTC_REUSE_SORT / PTC_REUSE_RUNS) goes through
+    ptc_reuse_indices_ex; None calls ptc_reuse_indices."""
     dev = _dev(ids)
     n = ids.numel()
     prev = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
     nxt = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
-    w = _workspace(lib().ptc_reuse_indices_workspace_bytes(n, n_distinct), dev, ws)
-    rc = lib().ptc_reuse_indices(_ptr(ids), n, n_distinct, _ptr(prev), _ptr(nxt), _ptr(w), w.numel(), _stream(dev))
-    _check("ptc_reuse_indices", rc)
+    if method is None:
+        w = _workspace(lib().ptc_reuse_indices_workspace_bytes(n, n_distinct), dev, ws)
+        rc = lib().ptc_reuse_indices(_ptr(ids), n, n_distinct, _ptr(prev), _ptr(nxt), _ptr(w), w.numel(),
+                                     _stream(dev))
+        _check("ptc_reuse_indices", rc)
+    else:
+        w = _workspace(lib().ptc_reuse_indices_ex_workspace_bytes(n, n_distinct, method), dev, ws)
+        rc = lib().ptc_reuse_indices_ex(_ptr(ids), n, n_distinct, _ptr(prev), _ptr(nxt), method, _ptr(w), w.numel(),
+                                        _stream(dev))
+        _check("ptc_reuse_indices_ex", rc)
     return prev[:n], nxt[:n]
 
 

@@ -37,11 +37,10 @@ __device__ __forceinline__ ulonglong2 cas128(ulonglong2* addr, ulonglong2 cmp, u
   return old;
 }
 
+// The keys are polynomial hashes of their prefixes, spread evenly over
+// [0, 2^61 - 1), so their low bits index the table directly.
 __device__ __forceinline__ uint64_t home_slot(uint64_t h0, uint64_t h1, uint32_t log2m) {
-  uint64_t z = (h0 ^ (h1 * 0x9E3779B97F4A7C15ULL)) * 0xD6E8FEB86659FD93ULL;
-  z ^= z >> 32;
-  z *= 0xD6E8FEB86659FD93ULL;
-  return log2m ? z >> (64 - log2m) : 0;
+  return (h0 ^ (h1 >> 17)) & ((1ULL << log2m) - 1);
 }
 
 __device__ __forceinline__ ulonglong2 ld_slot(const ulonglong2* p) {
@@ -55,7 +54,7 @@ __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __
                                                             uint32_t* __restrict__ slot_of, DevStatus* st) {
   const uint32_t i = blockIdx.x * kInsThreads + threadIdx.x;
   if (i >= n) return;
-  const ulonglong2 k = keys[i];
+  const ulonglong2 k = __ldcs(&keys[i]);  // streamed once: keep L2 for the table
   if (k.x >= kP61 || k.y >= kP61) {
     raise_err(st, kErrInvalid);
     slot_of[i] = 0;
@@ -75,13 +74,13 @@ __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __
     if (cur.x == ~0ULL || cur.y == ~0ULL) {  // empty, or being filled: settle it with the CAS
       cur = cas128(&table[pos], empty, mine);
       if (cur.x == ~0ULL && cur.y == ~0ULL) {
-        slot_of[i] = (uint32_t)pos;
+        __stcs(&slot_of[i], (uint32_t)pos);
         return;
       }
     }
     if (cur.x == w0 && (uint32_t)cur.y == w1lo) {
       if ((uint32_t)(cur.y >> 32) > i) atomicMin(reinterpret_cast<uint32_t*>(&table[pos]) + 3, i);
-      slot_of[i] = (uint32_t)pos;
+      __stcs(&slot_of[i], (uint32_t)pos);
       return;
     }
     pos = (pos + 1) & mask;
@@ -103,17 +102,25 @@ __global__ void __launch_bounds__(kFlT) k_ids_flags(const ulonglong2* __restrict
   __shared__ uint32_t s_last;
   const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const uint32_t base = tile * kFlTile + w * (32 * kFlR);
+  // slots, then their first indices, then the stores: all eight loads of
+  // each kind are in flight together
+  uint32_t f[kFlR];
+#pragma unroll
+  for (int k = 0; k < kFlR; ++k) {
+    const uint32_t i = base + k * 32 + lane;
+    f[k] = i < n ? __ldcs(&slot_first[i]) : 0u;
+  }
+#pragma unroll
+  for (int k = 0; k < kFlR; ++k) {
+    const uint32_t i = base + k * 32 + lane;
+    f[k] = i < n ? reinterpret_cast<const uint32_t*>(&table[f[k]])[3] : kNone;
+  }
   uint32_t cnt = 0;
 #pragma unroll
   for (int k = 0; k < kFlR; ++k) {
     const uint32_t i = base + k * 32 + lane;
-    bool first = false;
-    if (i < n) {
-      const uint32_t f = reinterpret_cast<const uint32_t*>(&table[slot_first[i]])[3];
-      slot_first[i] = f;
-      first = f == i;
-    }
-    const uint32_t m = __ballot_sync(kFull, first);
+    if (i < n) __stcs(&slot_first[i], f[k]);
+    const uint32_t m = __ballot_sync(kFull, i < n && f[k] == i);
     if (lane == 0 && base + k * 32 < n) bits[(base + k * 32) >> 5] = m;
     cnt += __popc(m);
   }
@@ -184,7 +191,7 @@ __global__ void k_ids_gather(const uint32_t* __restrict__ first, const uint32_t*
                              const uint32_t* __restrict__ wpre, uint32_t n, uint32_t* __restrict__ ids) {
   const uint32_t i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
-  const uint32_t f = first[i];
+  const uint32_t f = __ldcs(&first[i]);
   ids[i] = f < n ? wpre[f >> 5] + __popc(bits[f >> 5] & ((1u << (f & 31)) - 1u)) : kNone;
 }
 

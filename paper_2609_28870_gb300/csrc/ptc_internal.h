@@ -63,4 +63,13 @@ size_t stack_distance_points_bytes(uint64_t n);
 ptc_status stack_distance_points(const uint32_t* prev, uint64_t n, uint32_t* dist_out, void* ws, size_t ws_bytes,
                                  cudaStream_t s);
 
+// Stage b by a radix sort of every access (ptc_sort.cu), and the same sort
+// for any (key, value) pairs; the C entry point in ptc_reuse.cu chooses.
+size_t reuse_by_sort_bytes(uint64_t n);
+ptc_status reuse_by_sort(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev_out,
+                         uint32_t* next_out, void* ws, size_t ws_bytes, cudaStream_t s);
+size_t sort_pairs_bytes(uint64_t n);
+void sort_pairs(const uint32_t* keys, const uint32_t* vals, uint32_t n, uint32_t bits, void* ws, cudaStream_t s,
+                DevStatus* st, const uint32_t** keys_sorted, const uint32_t** vals_sorted);
+
 }  // namespace ptc

@@ -1,0 +1,488 @@
+// Stage b over id-runs: previous / next use of every access, from a stable
+// sort of runs of consecutive ids rather than of single accesses.
+//
+// An id-run is a maximal stretch of accesses whose ids go up by one from
+// access to access (id-run r: positions [s_r, s_r + len_r) holding ids
+// [x_r, x_r + len_r)).  Dense ids number blocks in order of first use, so a
+// context read back block by block is a handful of id-runs: the conversational
+// traces hold about a hundred accesses per id-run.
+//
+// Cut id-space at every run's first id and one past its last id: between two
+// consecutive cuts (an elementary interval e) every id-run holds all of e or
+// none of it.  For a fixed e, the runs holding it, in time order, are the
+// successive uses of each id in e, so the previous use of id y in e by run r
+// is y's place in the run just before r in that list (and the next use, in
+// the run just after).  So one stable sort of the (e, r) incidences by e
+// (run order is time order) gives prev and next of every access; on a trace
+// without runs it is the sort of every (id, i).
+//
+//   k_ir_count     id-run starts per tile (ids < D checked); last CTA: prefixes
+//   k_ir_mark      id-run records (start, first id) and the cuts, as a bitmap
+//                  over [0, D]
+//   k_bm_count / k_bm_words   ranks of the cuts (and the cut of each rank)
+//   k_ir_inc1      elementary intervals per run; last CTA: prefixes and K
+//   k_ir_inc2      the K incidences (e, r)
+//   (sort_pairs)   stable radix sort of the incidences by e
+//   k_ir_fill      one warp per incidence writes prev / next of its accesses
+//
+// When the incidences exceed a quarter of the accesses the stage falls back
+// to sorting every access (ptc_sort.cu).
+#include "ptc_internal.h"
+
+namespace ptc {
+namespace {
+
+constexpr int kIT = 256;            // threads per tile
+constexpr int kIR = 8;              // rounds of 32 positions per warp
+constexpr int kITile = kIT * kIR;   // 2048 positions; warp w owns [256 w, 256 w + 256)
+constexpr int kBmPer = 4;           // bitmap words per thread
+constexpr int kBmTile = kIT * kBmPer;
+constexpr int kRunPer = 8;          // runs per thread in the incidence kernels
+constexpr int kRunTile = kIT * kRunPer;
+
+struct IrArgs {
+  const uint32_t* ids;
+  uint32_t n, D, ntiles;
+  uint32_t* tcnt;
+  uint32_t* tpre;     // runs before each tile; tpre[ntiles] = number of runs
+  uint32_t* done;
+  uint32_t* rec_s;    // start of each run (rec_s[R] = n)
+  uint32_t* rec_x;    // first id of each run
+  uint32_t* cut;      // bitmap over [0, D]: the cuts of id-space
+  DevStatus* st;      // value[1] <- number of runs
+};
+
+// Exclusive prefix over the threads of a 256-thread CTA (total in *all).
+__device__ __forceinline__ uint32_t cta_excl_u32(uint32_t x, uint32_t* s_w, uint32_t* all) {
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  uint32_t incl = x;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(kFull, incl, o);
+    if (lane >= (uint32_t)o) incl += y;
+  }
+  __syncthreads();
+  if (lane == 31) s_w[w] = incl;
+  __syncthreads();
+  uint32_t pre = 0, tot = 0;
+#pragma unroll
+  for (int ww = 0; ww < kIT / 32; ++ww) {
+    const uint32_t v = s_w[ww];
+    if (ww < (int)w) pre += v;
+    tot += v;
+  }
+  *all = tot;
+  return pre + incl - x;
+}
+
+// The calling CTA learns whether it is the last of the grid to get here.
+__device__ __forceinline__ bool last_cta(uint32_t* done) {
+  __shared__ uint32_t s_last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(done, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (s_last) __threadfence();
+  return s_last;
+}
+
+// Run by the last CTA: exclusive prefix of cnt[0..T) into pre, pre[T] = total.
+__device__ uint32_t tiles_prefix(const uint32_t* cnt, uint32_t* pre, uint32_t T, uint32_t* s_w) {
+  const uint32_t per = (T + kIT - 1) / kIT;
+  const uint32_t t0 = threadIdx.x * per, t1 = min(t0 + per, T);
+  uint32_t sum = 0;
+  for (uint32_t t = t0; t < t1; ++t) sum += __ldcg(&cnt[t]);
+  uint32_t total;
+  uint32_t run = cta_excl_u32(sum, s_w, &total);
+  for (uint32_t t = t0; t < t1; ++t) {
+    pre[t] = run;
+    run += __ldcg(&cnt[t]);
+  }
+  if (threadIdx.x == 0) pre[T] = total;
+  return total;
+}
+
+// Id-run starts of the warp's 8 x 32 positions from `base`, with the id left
+// of each position.
+__device__ __forceinline__ void id_starts(const IrArgs& a, uint32_t base, uint32_t lane, uint32_t (&id)[kIR],
+                                          uint32_t (&left)[kIR], uint32_t (&words)[kIR], bool& bad) {
+#pragma unroll
+  for (int k = 0; k < kIR; ++k) {
+    const uint32_t j = base + k * 32 + lane;
+    id[k] = j < a.n ? a.ids[j] : 0u;
+  }
+  uint32_t carry = (lane == 0 && base > 0 && base - 1 < a.n) ? a.ids[base - 1] : 0u;
+#pragma unroll
+  for (int k = 0; k < kIR; ++k) {
+    const uint32_t j = base + k * 32 + lane;
+    const bool valid = j < a.n;
+    if (valid && id[k] >= a.D) bad = true;
+    const uint32_t up = __shfl_up_sync(kFull, id[k], 1);
+    const uint32_t l = lane ? up : carry;
+    carry = __shfl_sync(kFull, id[k], 31);
+    left[k] = l;
+    words[k] = __ballot_sync(kFull, valid && (j == 0 || id[k] != l + 1u));
+  }
+}
+
+__global__ void __launch_bounds__(kIT) k_ir_count(IrArgs a) {
+  __shared__ uint32_t s_w[kIT / 32];
+  const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  uint32_t id[kIR], left[kIR], words[kIR];
+  bool bad = false;
+  id_starts(a, tile * kITile + w * (32 * kIR), lane, id, left, words, bad);
+  uint32_t cnt = 0;
+#pragma unroll
+  for (int k = 0; k < kIR; ++k) cnt += __popc(words[k]);
+  if (bad) raise_err(a.st, kErrInvalid);
+  uint32_t total;
+  cta_excl_u32(lane == 0 ? cnt : 0u, s_w, &total);
+  if (threadIdx.x == 0) a.tcnt[tile] = total;
+  if (!last_cta(a.done)) return;
+  const uint32_t R = tiles_prefix(a.tcnt, a.tpre, a.ntiles, s_w);
+  if (threadIdx.x == 0) a.st->value[1] = R;
+}
+
+__global__ void __launch_bounds__(kIT) k_ir_mark(IrArgs a) {
+  __shared__ uint32_t s_w[kIT / 32];
+  if (*(volatile uint32_t*)&a.st->err) return;  // ids >= D: reported, nothing is indexed by them
+  const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const uint32_t base = tile * kITile + w * (32 * kIR);
+  uint32_t id[kIR], left[kIR], words[kIR];
+  bool bad = false;
+  id_starts(a, base, lane, id, left, words, bad);
+  uint32_t cnt = 0;
+#pragma unroll
+  for (int k = 0; k < kIR; ++k) cnt += __popc(words[k]);
+  uint32_t total;
+  uint32_t run = a.tpre[tile] + cta_excl_u32(lane == 0 ? cnt : 0u, s_w, &total);
+  run = __shfl_sync(kFull, run, 0);
+#pragma unroll
+  for (int k = 0; k < kIR; ++k) {
+    const uint32_t j = base + k * 32 + lane;
+    if ((words[k] >> lane) & 1u) {
+      const uint32_t r = run + __popc(words[k] & lanemask_lt());
+      a.rec_s[r] = j;
+      a.rec_x[r] = id[k];
+      atomicOr(&a.cut[id[k] >> 5], 1u << (id[k] & 31));
+      if (j > 0) atomicOr(&a.cut[(left[k] + 1) >> 5], 1u << ((left[k] + 1) & 31));
+    }
+    if (j + 1 == a.n) {
+      atomicOr(&a.cut[(id[k] + 1) >> 5], 1u << ((id[k] + 1) & 31));
+      a.rec_s[a.tpre[a.ntiles]] = a.n;
+    }
+    run += __popc(words[k]);
+  }
+}
+
+// Ranks of the cuts: per tile of kBmTile words the set bits, then (last CTA)
+// tile prefixes; k_bm_words turns them into the cuts before every word and
+// lists the cut of every rank.
+__global__ void __launch_bounds__(kIT) k_bm_count(const uint32_t* __restrict__ bits, uint32_t nwords, uint32_t T,
+                                                  uint32_t* tcnt, uint32_t* tpre, uint32_t* done, DevStatus* st) {
+  __shared__ uint32_t s_w[kIT / 32];
+  const uint32_t w0 = blockIdx.x * kBmTile + threadIdx.x * kBmPer;
+  uint32_t c = 0;
+#pragma unroll
+  for (int k = 0; k < kBmPer; ++k)
+    if (w0 + k < nwords) c += __popc(bits[w0 + k]);
+  uint32_t total;
+  cta_excl_u32(c, s_w, &total);
+  if (threadIdx.x == 0) tcnt[blockIdx.x] = total;
+  if (!last_cta(done)) return;
+  const uint32_t M = tiles_prefix(tcnt, tpre, T, s_w);
+  if (threadIdx.x == 0) st->value[2] = M;
+}
+
+__global__ void __launch_bounds__(kIT) k_bm_words(const uint32_t* __restrict__ bits, uint32_t nwords,
+                                                  const uint32_t* __restrict__ tpre, uint32_t* __restrict__ wpre,
+                                                  uint32_t* __restrict__ cut_at) {
+  __shared__ uint32_t s_w[kIT / 32];
+  const uint32_t w0 = blockIdx.x * kBmTile + threadIdx.x * kBmPer;
+  uint32_t b[kBmPer], c = 0;
+#pragma unroll
+  for (int k = 0; k < kBmPer; ++k) {
+    b[k] = w0 + k < nwords ? bits[w0 + k] : 0u;
+    c += __popc(b[k]);
+  }
+  uint32_t total;
+  uint32_t r = tpre[blockIdx.x] + cta_excl_u32(c, s_w, &total);
+#pragma unroll
+  for (int k = 0; k < kBmPer; ++k) {
+    if (w0 + k < nwords) wpre[w0 + k] = r;
+    for (uint32_t m = b[k]; m; m &= m - 1) cut_at[r++] = (w0 + k) * 32 + (__ffs(m) - 1);
+  }
+}
+
+// Cuts at or below y, minus one: the elementary interval holding id y.
+__device__ __forceinline__ uint32_t interval_of(const uint32_t* bits, const uint32_t* wpre, uint32_t y) {
+  const uint32_t wi = y >> 5, b = y & 31;
+  const uint32_t mask_le = b == 31 ? kFull : ((2u << b) - 1u);
+  return wpre[wi] + __popc(bits[wi] & mask_le) - 1u;
+}
+
+struct IncArgs {
+  const uint32_t* rec_s;
+  const uint32_t* rec_x;
+  const uint32_t* cut;
+  const uint32_t* cwpre;
+  const DevStatus* stc;     // value[1] = number of runs
+  uint32_t* tcnt;
+  uint32_t* tpre;
+  uint32_t* done;
+  uint32_t* key;            // incidences: elementary interval
+  uint32_t* val;            //             run
+  uint32_t max_tiles;       // tiles of tcnt / tpre
+  DevStatus* st;            // value[3] <- K
+};
+
+// Intervals of run r: [first, end).
+__device__ __forceinline__ void run_intervals(const IncArgs& a, uint32_t r, uint32_t& first, uint32_t& end) {
+  const uint32_t x = a.rec_x[r], len = a.rec_s[r + 1] - a.rec_s[r];
+  first = interval_of(a.cut, a.cwpre, x);
+  end = interval_of(a.cut, a.cwpre, x + len - 1) + 1;
+}
+
+// Persistent over the run tiles (the number of runs is known on the device only).
+__global__ void __launch_bounds__(kIT) k_ir_inc1(IncArgs a) {
+  __shared__ uint32_t s_w[kIT / 32];
+  if (*(volatile const uint32_t*)&a.stc->err) return;  // the records are incomplete
+  const uint32_t R = (uint32_t)a.stc->value[1];
+  const uint32_t T = (R + kRunTile - 1) / kRunTile;
+  for (uint32_t t = blockIdx.x; t < T; t += gridDim.x) {
+    const uint32_t r0 = t * kRunTile + threadIdx.x * kRunPer;
+    uint32_t c = 0;
+#pragma unroll
+    for (int k = 0; k < kRunPer; ++k) {
+      if (r0 + k < R) {
+        uint32_t f, e;
+        run_intervals(a, r0 + k, f, e);
+        c += e - f;
+      }
+    }
+    uint32_t total;
+    cta_excl_u32(c, s_w, &total);
+    if (threadIdx.x == 0) a.tcnt[t] = total;
+  }
+  if (!last_cta(a.done)) return;
+  const uint32_t K = tiles_prefix(a.tcnt, a.tpre, T < a.max_tiles ? T : a.max_tiles, s_w);
+  if (threadIdx.x == 0) a.st->value[3] = K;
+}
+
+__global__ void __launch_bounds__(kIT) k_ir_inc2(IncArgs a, uint32_t R) {
+  __shared__ uint32_t s_w[kIT / 32];
+  const uint32_t t = blockIdx.x;
+  const uint32_t r0 = t * kRunTile + threadIdx.x * kRunPer;
+  uint32_t f[kRunPer], e[kRunPer], c = 0;
+#pragma unroll
+  for (int k = 0; k < kRunPer; ++k) {
+    f[k] = e[k] = 0;
+    if (r0 + k < R) {
+      run_intervals(a, r0 + k, f[k], e[k]);
+      c += e[k] - f[k];
+    }
+  }
+  uint32_t total;
+  uint32_t o = a.tpre[t] + cta_excl_u32(c, s_w, &total);
+#pragma unroll
+  for (int k = 0; k < kRunPer; ++k)
+    for (uint32_t iv = f[k]; iv < e[k]; ++iv) {
+      a.key[o] = iv;
+      a.val[o] = r0 + k;
+      ++o;
+    }
+}
+
+struct FillArgs {
+  const uint32_t* key;     // sorted incidences
+  const uint32_t* val;
+  uint32_t K, n;
+  const uint32_t* rec_s;
+  const uint32_t* rec_x;
+  const uint32_t* cut_at;  // id of every cut, by rank
+  uint32_t* prev;
+  uint32_t* next;
+};
+
+// One warp per incidence (e, r): the accesses of run r with ids in e take
+// their previous / next use from the runs before / after r on e.
+__global__ void __launch_bounds__(256) k_ir_fill(FillArgs a) {
+  const uint32_t lane = threadIdx.x & 31;
+  const uint32_t warps = gridDim.x * (blockDim.x >> 5);
+  for (uint32_t q = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; q < a.K; q += warps) {
+    const uint32_t e = a.key[q], r = a.val[q];
+    const bool has_pred = q > 0 && a.key[q - 1] == e;
+    const bool has_succ = q + 1 < a.K && a.key[q + 1] == e;
+    const uint32_t lo = a.cut_at[e], hi = a.cut_at[e + 1];
+    const uint32_t s0 = a.rec_s[r] + (lo - a.rec_x[r]);
+    uint32_t p0 = kNone, n0 = kNone;
+    if (has_pred) {
+      const uint32_t rp = a.val[q - 1];
+      p0 = a.rec_s[rp] + (lo - a.rec_x[rp]);
+    }
+    if (has_succ) {
+      const uint32_t rn = a.val[q + 1];
+      n0 = a.rec_s[rn] + (lo - a.rec_x[rn]);
+    }
+    for (uint32_t t = lane; t < hi - lo; t += 32) {
+      const uint32_t j = s0 + t;
+      if (j < a.n) {
+        a.prev[j] = has_pred ? p0 + t : kNone;
+        a.next[j] = has_succ ? n0 + t : kNone;
+      }
+    }
+  }
+}
+
+struct ReuseLayout {
+  DevStatus* st;
+  uint32_t* done;
+  size_t zero_bytes;
+  uint32_t *tcnt, *tpre, *rec_s, *rec_x;
+  uint32_t *cut, *cwpre, *cut_at, *btcnt, *btpre;
+  uint32_t *rtcnt, *rtpre;
+  uint32_t *key, *val;
+  void* sort_ws;
+  uint32_t ntiles, nwords, btiles, rtiles_max;
+  uint64_t kcap;
+  size_t total;
+};
+
+// Incidences the run path takes before it falls back to sorting every access
+// (all of them when the run path is forced: there are at most n).
+uint64_t incidence_cap(uint64_t n, bool forced) { return forced ? n + 64 : n / 4 + 64; }
+
+ReuseLayout reuse_layout(void* ws, uint64_t n, uint64_t D, bool forced) {
+  ReuseLayout L;
+  Carver cv(ws);
+  const uint64_t nn = n ? n : 1;
+  L.ntiles = ceil_div_u32(nn, kITile);
+  L.nwords = (uint32_t)((D + 1) / 32 + 1);
+  L.btiles = ceil_div_u32(L.nwords, kBmTile);
+  L.rtiles_max = ceil_div_u32(nn, kRunTile);
+  L.kcap = incidence_cap(nn, forced);
+  L.st = cv.take<DevStatus>(1);
+  L.done = cv.take<uint32_t>(64);
+  L.zero_bytes = cv.off;
+  L.tcnt = cv.take<uint32_t>(L.ntiles + 1);
+  L.tpre = cv.take<uint32_t>(L.ntiles + 1);
+  L.rec_s = cv.take<uint32_t>(nn + 1);
+  L.rec_x = cv.take<uint32_t>(nn);
+  L.cut = cv.take<uint32_t>(L.nwords);
+  L.cwpre = cv.take<uint32_t>(L.nwords);
+  L.cut_at = cv.take<uint32_t>(D + 3);
+  L.btcnt = cv.take<uint32_t>(L.btiles + 1);
+  L.btpre = cv.take<uint32_t>(L.btiles + 1);
+  L.rtcnt = cv.take<uint32_t>(L.rtiles_max + 1);
+  L.rtpre = cv.take<uint32_t>(L.rtiles_max + 1);
+  L.key = cv.take<uint32_t>(L.kcap);
+  L.val = cv.take<uint32_t>(L.kcap);
+  L.sort_ws = cv.take<unsigned char>(sort_pairs_bytes(L.kcap));
+  L.total = cv.bytes();
+  return L;
+}
+
+uint32_t bits_for(uint64_t v) {  // bits to hold values below v
+  uint32_t b = 1;
+  while (b < 32 && (1ULL << b) < v) ++b;
+  return b;
+}
+
+ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* prev_out, uint32_t* next_out, void* ws,
+                         size_t ws_bytes, cudaStream_t s, bool forced) {
+  const ReuseLayout L = reuse_layout(ws, n, D, forced);
+  if (!ws_ok(ws, ws_bytes, L.total)) return PTC_ERR_WORKSPACE;
+  if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
+  if (cudaMemsetAsync(L.cut, 0, sizeof(uint32_t) * L.nwords, s) != cudaSuccess) return PTC_ERR_CUDA;
+  IrArgs a;
+  a.ids = ids;
+  a.n = (uint32_t)n;
+  a.D = (uint32_t)D;
+  a.ntiles = L.ntiles;
+  a.tcnt = L.tcnt;
+  a.tpre = L.tpre;
+  a.done = &L.done[0];
+  a.rec_s = L.rec_s;
+  a.rec_x = L.rec_x;
+  a.cut = L.cut;
+  a.st = L.st;
+  PTC_LAUNCH("k_ir_count", s, k_ir_count<<<L.ntiles, kIT, 0, s>>>(a));
+  PTC_LAUNCH("k_ir_mark", s, k_ir_mark<<<L.ntiles, kIT, 0, s>>>(a));
+  PTC_LAUNCH("k_bm_count", s,
+             k_bm_count<<<L.btiles, kIT, 0, s>>>(L.cut, L.nwords, L.btiles, L.btcnt, L.btpre, &L.done[1], L.st));
+  PTC_LAUNCH("k_bm_words", s, k_bm_words<<<L.btiles, kIT, 0, s>>>(L.cut, L.nwords, L.btpre, L.cwpre, L.cut_at));
+  IncArgs ia;
+  ia.rec_s = L.rec_s;
+  ia.rec_x = L.rec_x;
+  ia.cut = L.cut;
+  ia.cwpre = L.cwpre;
+  ia.stc = L.st;
+  ia.tcnt = L.rtcnt;
+  ia.tpre = L.rtpre;
+  ia.done = &L.done[2];
+  ia.key = L.key;
+  ia.val = L.val;
+  ia.max_tiles = L.rtiles_max;
+  ia.st = L.st;
+  const uint32_t g1 = L.rtiles_max < (uint32_t)(2 * num_sms()) ? L.rtiles_max : (uint32_t)(2 * num_sms());
+  PTC_LAUNCH("k_ir_inc1", s, k_ir_inc1<<<g1, kIT, 0, s>>>(ia));
+  DevStatus h;
+  ptc_status rc = end_call(L.st, s, &h);
+  if (rc != PTC_OK) return rc;
+  const uint64_t R = h.value[1], M = h.value[2], K = h.value[3];
+  if (K > L.kcap || R == 0 || M < 2) {
+    if (forced) return PTC_ERR_WORKSPACE;  // cannot happen: K <= n
+    return reuse_by_sort(ids, n, D, prev_out, next_out, ws, ws_bytes, s);
+  }
+  PTC_LAUNCH("k_ir_inc2", s, k_ir_inc2<<<ceil_div_u32(R, kRunTile), kIT, 0, s>>>(ia, (uint32_t)R));
+  const uint32_t *skey = nullptr, *sval = nullptr;
+  sort_pairs(L.key, L.val, (uint32_t)K, bits_for(M - 1), L.sort_ws, s, L.st, &skey, &sval);
+  FillArgs f;
+  f.key = skey;
+  f.val = sval;
+  f.K = (uint32_t)K;
+  f.n = (uint32_t)n;
+  f.rec_s = L.rec_s;
+  f.rec_x = L.rec_x;
+  f.cut_at = L.cut_at;
+  f.prev = prev_out;
+  f.next = next_out;
+  const uint32_t fill_blocks = ceil_div_u32(K, 8) < (uint32_t)(16 * num_sms()) ? ceil_div_u32(K, 8)
+                                                                                : (uint32_t)(16 * num_sms());
+  PTC_LAUNCH("k_ir_fill", s, k_ir_fill<<<fill_blocks, 256, 0, s>>>(f));
+  return end_call(L.st, s, &h);
+}
+
+}  // namespace
+}  // namespace ptc
+
+using namespace ptc;
+
+extern "C" size_t ptc_reuse_indices_ex_workspace_bytes(uint64_t n, uint64_t n_distinct, int method) {
+  const uint64_t D = n_distinct ? n_distinct : (n ? n : 1);
+  const size_t by_sort = reuse_by_sort_bytes(n);
+  if (method == PTC_REUSE_SORT) return by_sort;
+  const size_t by_runs = reuse_layout(nullptr, n, D, method == PTC_REUSE_RUNS).total;
+  if (method == PTC_REUSE_RUNS) return by_runs;
+  return by_sort > by_runs ? by_sort : by_runs;
+}
+
+extern "C" size_t ptc_reuse_indices_workspace_bytes(uint64_t n, uint64_t n_distinct) {
+  return ptc_reuse_indices_ex_workspace_bytes(n, n_distinct, PTC_REUSE_AUTO);
+}
+
+extern "C" ptc_status ptc_reuse_indices_ex(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev_out,
+                                           uint32_t* next_out, int method, void* ws, size_t ws_bytes, void* stream) {
+  if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
+  if (method != PTC_REUSE_AUTO && method != PTC_REUSE_SORT && method != PTC_REUSE_RUNS) return PTC_ERR_INVALID_ARG;
+  if (n == 0) return PTC_OK;
+  if (!ids || !prev_out || !next_out || n_distinct == 0 || n_distinct > n) return PTC_ERR_INVALID_ARG;
+  cudaStream_t s = (cudaStream_t)stream;
+  if (method == PTC_REUSE_SORT) return reuse_by_sort(ids, n, n_distinct, prev_out, next_out, ws, ws_bytes, s);
+  return reuse_by_runs(ids, n, n_distinct, prev_out, next_out, ws, ws_bytes, s, method == PTC_REUSE_RUNS);
+}
+
+extern "C" ptc_status ptc_reuse_indices(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev_out,
+                                        uint32_t* next_out, void* ws, size_t ws_bytes, void* stream) {
+  return ptc_reuse_indices_ex(ids, n, n_distinct, prev_out, next_out, PTC_REUSE_AUTO, ws, ws_bytes, stream);
+}

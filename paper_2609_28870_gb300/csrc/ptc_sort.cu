@@ -337,18 +337,13 @@ SortLayout sort_layout(void* ws, uint64_t n) {
 
 using namespace ptc;
 
-extern "C" size_t ptc_reuse_indices_workspace_bytes(uint64_t n, uint64_t n_distinct) {
-  (void)n_distinct;
-  return sort_layout(nullptr, n).total;
-}
+size_t ptc::reuse_by_sort_bytes(uint64_t n) { return sort_layout(nullptr, n).total; }
 
-extern "C" ptc_status ptc_reuse_indices(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev_out,
-                                        uint32_t* next_out, void* ws, size_t ws_bytes, void* stream) {
-  if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
-  if (n == 0) return PTC_OK;
-  if (!ids || !prev_out || !next_out || n_distinct == 0 || n_distinct > n) return PTC_ERR_INVALID_ARG;
+// prev / next from a stable radix sort of every (id, i) (argument checks are
+// the caller's).
+ptc_status ptc::reuse_by_sort(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev_out,
+                              uint32_t* next_out, void* ws, size_t ws_bytes, cudaStream_t s) {
   if (!ws_ok(ws, ws_bytes, sort_layout(nullptr, n).total)) return PTC_ERR_WORKSPACE;
-  cudaStream_t s = (cudaStream_t)stream;
   const SortLayout L = sort_layout(ws, n);
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
   const uint32_t bits = key_bits(n_distinct);
@@ -398,4 +393,49 @@ extern "C" ptc_status ptc_reuse_indices(const uint32_t* ids, uint64_t n, uint64_
   }
   DevStatus h;
   return end_call(L.st, s, &h);
+}
+
+size_t ptc::sort_pairs_bytes(uint64_t n) { return sort_layout(nullptr, n).total; }
+
+// Stable LSD sort of (keys, vals) by the low `bits` bits of the keys, queued
+// on `s` without waiting; *keys_sorted / *vals_sorted point into `ws` (which
+// must hold sort_pairs_bytes(n)).  Errors go to `st`.
+void ptc::sort_pairs(const uint32_t* keys, const uint32_t* vals, uint32_t n, uint32_t bits, void* ws,
+                     cudaStream_t s, DevStatus* st, const uint32_t** keys_sorted, const uint32_t** vals_sorted) {
+  const SortLayout L = sort_layout(ws, n);
+  if (bits < 1) bits = 1;
+  const uint32_t passes = (bits + 7) / 8;
+  const uint32_t T = ceil_div_u32(n ? n : 1, kSortTile);
+  const uint32_t* kin = keys;
+  const uint32_t* vin = vals;
+  uint32_t *kout = L.k0, *vout = L.v0;
+  uint32_t shift = 0;
+  for (uint32_t p = 0; p < passes; ++p) {
+    const uint32_t width = (bits - shift + (passes - p) - 1) / (passes - p);
+    const uint32_t R = 1u << width;
+    PTC_LAUNCH("k_sort_count", s,
+               k_sort_count<<<T, kSortThreads, 0, s>>>(kin, n, shift, R, T, kNone, ((uintptr_t)kin & 15) == 0, L.cnt,
+                                                       st));
+    PTC_LAUNCH("k_sort_rowscan", s, k_sort_rowscan<<<R, kSortThreads, 0, s>>>(L.cnt, T, L.off, L.tot));
+    ScatterArgs a = {};
+    a.keys_in = kin;
+    a.vals_in = vin;
+    a.keys_out = kout;
+    a.vals_out = vout;
+    a.off = L.off;
+    a.tot = L.tot;
+    a.n = n;
+    a.T = T;
+    a.shift = shift;
+    a.R = R;
+    a.width = width;
+    PTC_LAUNCH("k_sort_scatter", s, k_sort_scatter<false><<<T, kSortThreads, 0, s>>>(a));
+    kin = kout;
+    vin = vout;
+    kout = (kout == L.k0) ? L.k1 : L.k0;
+    vout = (vout == L.v0) ? L.v1 : L.v0;
+    shift += width;
+  }
+  *keys_sorted = kin;
+  *vals_sorted = vin;
 }
