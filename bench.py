@@ -116,6 +116,7 @@ def kernel_model_bytes(name, T, N, L, D):
     per_level = ((L - 1) * 8.125 + 4.125) / L * N  # the last level writes no partition
     return {
         "k_hash_local": 4 * T + 16 * N,   # token stream in, block keys out
+        "k_hash16": 4 * T + 16 * N,       # the same, B = 16 path
         "k_ids_insert": 16 * N,           # keys in
         "k_ids_gather": 4 * N,            # ids out
         "k_sort_scatter": 12 * N / sort_passes(D),  # ids in, prev / next out, spread over the passes
@@ -131,6 +132,7 @@ def kernel_model_bytes(name, T, N, L, D):
 
 KERNEL_SOURCE = {
     "k_block_offsets": "ptc_hash.cu", "k_pow_tables": "ptc_hash.cu", "k_hash_local": "ptc_hash.cu",
+    "k_hash16": "ptc_hash.cu",
     "k_hash_chain": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu", "k_ids_flags": "ptc_ids.cu",
     "k_ids_wordpre": "ptc_ids.cu",
     "k_ids_gather": "ptc_ids.cu", "k_sort_count": "ptc_sort.cu", "k_sort_rowscan": "ptc_sort.cu",

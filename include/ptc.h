@@ -92,12 +92,13 @@ const char* ptc_version(void);
  * Request r owns tokens[req_tok_off[r] : req_tok_off[r+1]] and has
  * n_r = floor(len_r / B) full blocks; a trailing partial block is not a cache
  * object.  Block k of request r gets the key of its whole prefix
- * [0, B(k+1)): the polynomial of the sequence (1, tok_0, ..., tok_{B(k+1)-1})
- * over GF(2^61 - 1) at two bases rho_0, rho_1 drawn from `seed` with
- * SplitMix64 (rho_b = 2 + (output b) mod (2^61 - 4)).  keys_out[i].lo / .hi
- * are the values at rho_0 / rho_1.  Two different prefixes of at most m
- * tokens share a key with probability at most (m / (2^61 - 1))^2 (the
- * Schwartz-Zippel bound for each base); ptc_verify_ids checks exactly.
+ * [0, B(k+1)):  sum over t < B(k+1) of (tok_t + 1) * u^(t+1)  mod 2^61 - 1,
+ * at two bases u_0, u_1 drawn from `seed` with SplitMix64
+ * (u_b = 2 + (output b) mod (2^61 - 4)).  keys_out[i].lo / .hi are the values
+ * at u_0 / u_1.  Every coefficient tok + 1 is nonzero, so two different
+ * prefixes of at most m tokens (of equal or different length) share a key
+ * with probability at most (m / (2^61 - 1))^2 (the Schwartz-Zippel bound for
+ * each base); ptc_verify_ids checks exactly.
  *
  *   tokens          u32[n_tok]; any alignment (16-byte aligned is fastest)
  *   req_tok_off     u64[n_req + 1], non-decreasing, req_tok_off[n_req] <= n_tok

@@ -15,8 +15,8 @@ Functions and the passages they restate:
   move-to-front stack and by Bennett-Kruskal counting.
 * ``lru_curves`` — direct LRU simulation per capacity (Sec. 3.1-3.2) with
   prefix-contiguous hits (Sec. 2.2) and compute saved (Sec. 5.2, App. C).
-* ``prefix_hash`` — the polynomial prefix key the GPU path writes, evaluated
-  token by token.
+* ``prefix_hash`` — the polynomial prefix key the GPU path writes,
+  sum_t (tok_t + 1) u^(t+1) mod 2^61 - 1 at two seeded bases, token by token.
 * ``run`` — all of the above on one trace.
 """
 from __future__ import annotations

@@ -24,8 +24,9 @@
 //   * Belady's next use (Sec. 3.2, 5.2).  -> orc_reuse: previous and next
 //     access of the same block.
 // The GPU path's block keys are polynomial hashes of each block's whole
-// prefix; orc_prefix_hash evaluates that polynomial token by token (Horner)
-// so the keys themselves can be compared.
+// prefix, sum over its tokens of (tok_t + 1) u^(t+1) mod 2^61 - 1 at two
+// seeded bases u; orc_prefix_hash evaluates that sum token by token so the
+// keys themselves can be compared.
 //
 // Readings where the paper is silent (listed with the design notes): requests
 // are replayed in trace order and blocks root-first; a trailing partial block is
@@ -289,26 +290,28 @@ int orc_lru_curves(const uint32_t* ids, const uint64_t* req_blk_off, uint32_t n_
 void orc_prefix_hash(const uint32_t* tokens, const uint64_t* req_tok_off, uint32_t n_req, uint32_t B, uint64_t seed,
                      uint64_t* keys) {
   const uint64_t P = (1ULL << 61) - 1;
-  uint64_t rho[2];
+  uint64_t u[2];
   for (int b = 0; b < 2; ++b) {
     uint64_t z = seed + (uint64_t)(b + 1) * 0x9E3779B97F4A7C15ULL;
     z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
     z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
     z = z ^ (z >> 31);
-    rho[b] = 2 + z % (P - 3);
+    u[b] = 2 + z % (P - 3);
   }
   uint64_t i = 0;
   for (uint32_t r = 0; r < n_req; ++r) {
     uint64_t len = req_tok_off[r + 1] - req_tok_off[r];
     uint64_t nblk = len / B;
-    u128 h0 = 1, h1 = 1;  // the leading coefficient 1
+    u128 s0 = 0, s1 = 0, p0 = u[0], p1 = u[1];  // p_b = u_b^(t+1)
     for (uint64_t t = 0; t < nblk * B; ++t) {
-      uint64_t x = tokens[req_tok_off[r] + t];
-      h0 = (h0 * rho[0] + x) % P;
-      h1 = (h1 * rho[1] + x) % P;
+      u128 x = (u128)tokens[req_tok_off[r] + t] + 1;
+      s0 = (s0 + x * p0) % P;
+      s1 = (s1 + x * p1) % P;
+      p0 = p0 * u[0] % P;
+      p1 = p1 * u[1] % P;
       if ((t + 1) % B == 0) {
-        keys[2 * i] = (uint64_t)h0;
-        keys[2 * i + 1] = (uint64_t)h1;
+        keys[2 * i] = (uint64_t)s0;
+        keys[2 * i + 1] = (uint64_t)s1;
         ++i;
       }
     }

@@ -1,26 +1,32 @@
 // Stage a1: chained block keys (paper Sec. 2.2 block identity).
 //
-// Block k of a request covers tokens [Bk, Bk+B).  Its key is the polynomial
-// of the whole prefix sequence (1, tok_0, ..., tok_{B(k+1)-1}) over
-// GF(2^61 - 1) at two seeded bases.  Written per block:
-//     h_k = sum_{i<B} tok_{Bk+i} * rho^(B-1-i)                 (block-local)
-//     H_k = rho^(B(k+1)) * (1 + sum_{j<=k} h_j * rho^(-B(j+1)))
-// so the chain across a request is a plain segmented sum of the normalised
-// g_j = h_j * rho^(-B(j+1)) — one single-pass scan, no sequential chain.
+// Block k of a request covers tokens [Bk, Bk+B).  Its key is a polynomial of
+// the whole prefix over GF(2^61 - 1) at two seeded bases u (one per key word):
+//     S_k = sum_{t < B(k+1)} (tok_t + 1) u^(t+1)
+// Every coefficient is at least 1, so two different prefixes, of equal or of
+// different length, differ as polynomials (Karp-Rabin; a pair collides with
+// probability at most length / 2^61 per base).  Written per block:
+//     h_j = sum_{i<B} (tok_{Bj+i} + 1) u^(i+1)                 (block-local)
+//     S_k = sum_{j<=k} h_j u^(Bj)
+// so the chain across a request is a plain segmented sum of g_j = h_j u^(Bj):
+// one scan, no sequential chain, and the sum itself is the key.
 //
 // Kernels
 //   k_block_offsets  per-request block counts -> exclusive scan (look-back),
 //                    validates offsets and timestamp order, max blocks/request
-//   k_pow_tables     rho^(+-B e) for e < 2^32 as two 65,536-entry levels
+//   k_pow_tables     u^(B e) for e < 2^32 as two 65,536-entry levels
+//                    (filled up to the longest request)
+//   k_hash16         B = 16, aligned tokens: the tile's request offsets in
+//                    shared memory, one block per thread
 //   k_hash_local     tokens staged through padded shared memory with 16-byte
 //                    loads; each thread hashes 16 tokens (one "sub-chunk")
-//                    with 3 x 21-bit limbs of the powers held as constant
+//                    with 3 x 21-bit limbs of u^1..u^16 held as constant
 //                    kernel parameters; sub-chunks of one block combine by
 //                    shuffles; the segmented sum runs across the CTA.  Keys
 //                    after the tile's first request start are final; the tile
 //                    records its aggregate.  No tile depends on another.
 //   k_hash_chain     each tile's carry from its predecessors' aggregates
-//                    (all already written, so nothing waits), then the final
+//                    (all already written, so nothing waits), added to the
 //                    keys of the tile's leading blocks.
 #include "ptc_internal.h"
 
@@ -119,19 +125,23 @@ __global__ void __launch_bounds__(kOffThreads) k_block_offsets(const uint64_t* _
 }
 
 // ---------------------------------------------------------------- powers
-// tables[(b*4 + w) * 65536 + e] for base b in {0,1} and
-//   w = 0: rho_b^(B e)          w = 1: rho_b^(-B e)
-//   w = 2: rho_b^(B 65536 e)    w = 3: rho_b^(-B 65536 e)
+// tables[(b*2 + w) * 65536 + e] for base b in {0,1} and
+//   w = 0: u_b^(B e)          w = 1: u_b^(B 65536 e)
 struct PowBases {
-  uint64_t base[8];
+  uint64_t base[4];
 };
 
-__global__ void k_pow_tables(PowBases pb, uint64_t* __restrict__ tables) {
-  const uint32_t gid = blockIdx.x * blockDim.x + threadIdx.x;  // 8 tables x 1024 chunks of 64
+// Only the entries some block can use are filled: exponents e = k reach at
+// most the longest request's block count minus one (st->value[1]).
+__global__ void k_pow_tables(PowBases pb, uint64_t* __restrict__ tables, const DevStatus* st) {
+  const uint32_t gid = blockIdx.x * blockDim.x + threadIdx.x;  // 4 tables x 1024 chunks of 64
   const uint32_t t = gid >> 10, chunk = gid & 1023;
-  if (t >= 8) return;
+  if (t >= 4) return;
+  const uint64_t kmax = st->value[1];
+  const uint64_t need = (t & 1) ? (kmax >> 16) : (kmax < 65535 ? kmax : 65535);
   const uint64_t base = pb.base[t];
   const uint64_t e0 = (uint64_t)chunk * 64;
+  if (e0 > need) return;
   uint64_t v = p61_pow(base, e0);
   uint64_t* out = tables + (uint64_t)t * 65536 + e0;
   for (int i = 0; i < 64; ++i) {
@@ -150,8 +160,9 @@ __device__ __forceinline__ uint64_t pow_at(const uint64_t* __restrict__ lo, cons
 
 // ---------------------------------------------------------------- hash
 struct HashConsts {
-  uint32_t limb[2][3][16];   // 21-bit limbs of rho_b^(15 - j)
-  uint64_t sub_mul[2][32];   // rho_b^(16 q)
+  uint32_t limb[2][3][16];   // 21-bit limbs of u_b^(j + 1)
+  uint64_t csum[2][17];      // sum_{j < n} u_b^(j + 1): the "+ 1" of n tokens
+  uint64_t sub_mul[2][32];   // u_b^(16 q)
 };
 
 struct HashCarry {
@@ -193,7 +204,7 @@ __device__ __forceinline__ uint64_t mad_wide(uint32_t a, uint32_t b, uint64_t c)
   return (uint64_t)a * (uint64_t)b + c;
 }
 
-// Sum over the 16 words t[m .. m+15] of t * rho^(15 - j) for both bases, as
+// Sum over the 16 words t[m .. m+15] of t * u^(j + 1) for both bases, as
 // 21-bit limb accumulators (M is the word offset of the first token).
 template <int M>
 __device__ __forceinline__ void hash16(const uint32_t (&wd)[20], const HashConsts& c, uint64_t (&acc)[6]) {
@@ -261,14 +272,9 @@ __device__ __forceinline__ void hash_finish(const HashArgs& a, uint32_t tile, ui
   uint32_t kk = 0;
   if (valid) {
     kk = s_k[t];
-    const uint64_t e = (uint64_t)kk + 1;
-    x.v0 = p61_mul(s_h0[t], pow_at(T + 1 * 65536, T + 3 * 65536, e));
-    x.v1 = p61_mul(s_h1[t], pow_at(T + 5 * 65536, T + 7 * 65536, e));
-    if (kk == 0) {
-      x.f = 1;
-      x.v0 = p61_add(x.v0, 1);
-      x.v1 = p61_add(x.v1, 1);
-    }
+    x.v0 = p61_mul(s_h0[t], pow_at(T + 0 * 65536, T + 1 * 65536, kk));
+    x.v1 = p61_mul(s_h1[t], pow_at(T + 2 * 65536, T + 3 * 65536, kk));
+    x.f = kk == 0;
   }
   SegSumOp op;
   const uint32_t lane = t & 31, w = t >> 5;
@@ -297,21 +303,12 @@ __device__ __forceinline__ void hash_finish(const HashArgs& a, uint32_t tile, ui
   __syncthreads();
   if (w > 0) x = op(s_w[w - 1], x);
   // Blocks at or after the tile's first request start are final here; the
-  // leading blocks keep their normalised partial sum for k_hash_chain.
+  // leading blocks still lack the carry from earlier tiles (k_hash_chain).
   if (t == 0) s_first_head = TB;
   __syncthreads();
   if (valid && kk == 0) atomicMin(&s_first_head, t);
   __syncthreads();
-  if (valid) {
-    if (x.f) {
-      const uint64_t e = (uint64_t)kk + 1;
-      const uint64_t H0 = p61_mul(x.v0, pow_at(T + 0 * 65536, T + 2 * 65536, e));
-      const uint64_t H1 = p61_mul(x.v1, pow_at(T + 4 * 65536, T + 6 * 65536, e));
-      a.keys[b0 + t] = make_ulonglong2(H0, H1);
-    } else {
-      a.keys[b0 + t] = make_ulonglong2(x.v0, x.v1);
-    }
-  }
+  if (valid) a.keys[b0 + t] = make_ulonglong2(x.v0, x.v1);
   if (t == 0) {
     a.tile_agg[tile] = s_w[kHashThreads / 32 - 1];
     const uint32_t nb = (uint32_t)(b_end - b0);
@@ -383,10 +380,11 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local(HashArgs a, const _
   if (b < b_end) {
     const uint32_t r = find_request(a.blk_off, r_first, r_last, b);
     k = (uint32_t)(b - a.blk_off[r]);
-    const int64_t first = (int64_t)B - 16 * G + 16 * (int64_t)s;  // block offset of this chunk's token 0
+    const uint32_t first = 16 * s;  // block offset of this chunk's token 0
+    const uint32_t nval = first < B ? (B - first < 16 ? B - first : 16) : 0u;  // tokens of the block in the chunk
     const uint64_t bstart = a.tok_off[r] + (uint64_t)B * k;
     uint64_t a00 = 0, a01 = 0, a02 = 0, a10 = 0, a11 = 0, a12 = 0;
-    const uint64_t x0 = bstart + first;  // may wrap for the leading partial chunk; guarded below
+    const uint64_t x0 = bstart + first;
     const bool in_win = FULL && x0 >= w0 && x0 + 16 <= w_end;
     if (in_win) {
       const uint32_t rel = (uint32_t)(x0 - w0);
@@ -403,8 +401,8 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local(HashArgs a, const _
     } else {
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
-        if (FULL || first + j >= 0) {
-          const uint64_t x = bstart + (uint64_t)(first + j);
+        if (FULL || (uint32_t)j < nval) {
+          const uint64_t x = x0 + (uint64_t)j;
           uint64_t t;
           if (x >= w0 && x < w_end)
             t = s_tok[pad16((uint32_t)(x - w0))];
@@ -419,12 +417,11 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local(HashArgs a, const _
         }
       }
     }
-    h0 = limbs_to_p61(a00, a01, a02);
-    h1 = limbs_to_p61(a10, a11, a12);
-    if (G > 1) {
-      const uint32_t q = G - 1 - s;
-      h0 = p61_mul(h0, c.sub_mul[0][q]);
-      h1 = p61_mul(h1, c.sub_mul[1][q]);
+    h0 = p61_add(limbs_to_p61(a00, a01, a02), c.csum[0][FULL ? 16 : nval]);
+    h1 = p61_add(limbs_to_p61(a10, a11, a12), c.csum[1][FULL ? 16 : nval]);
+    if (G > 1 && s > 0) {
+      h0 = p61_mul(h0, c.sub_mul[0][s]);
+      h1 = p61_mul(h1, c.sub_mul[1][s]);
     }
   }
   hash_finish<G>(a, tile, b0, b_end, h0, h1, k, lb, s);
@@ -488,29 +485,141 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local_vec(HashArgs a, con
       case 2: hash16<2>(wd, c, acc); break;
       default: hash16<3>(wd, c, acc); break;
     }
-    h0 = limbs_to_p61(acc[0], acc[1], acc[2]);
-    h1 = limbs_to_p61(acc[3], acc[4], acc[5]);
-    if (G > 1) {
-      const uint32_t q = G - 1 - s;
-      h0 = p61_mul(h0, c.sub_mul[0][q]);
-      h1 = p61_mul(h1, c.sub_mul[1][q]);
+    h0 = p61_add(limbs_to_p61(acc[0], acc[1], acc[2]), c.csum[0][16]);
+    h1 = p61_add(limbs_to_p61(acc[3], acc[4], acc[5]), c.csum[1][16]);
+    if (G > 1 && s > 0) {
+      h0 = p61_mul(h0, c.sub_mul[0][s]);
+      h1 = p61_mul(h1, c.sub_mul[1][s]);
     }
   }
   hash_finish<G>(a, tile, b0, b_end, h0, h1, k, lb, s);
 }
 
+// B = 16 with 16-byte-aligned tokens: one block per thread, 512 blocks per
+// tile (as k_hash_local with G = 1).  The requests that meet the tile are
+// tile_req[tile] .. tile_req[tile + 1]; their block and token offsets are
+// loaded into shared memory once, so a thread finds its request without a
+// dependent chain of global loads, and its token loads and power-table loads
+// all go out together.  Tiles meeting more than kH16Req requests search the
+// global offsets instead.
+constexpr int kH16Req = 256;
+
+__global__ void __launch_bounds__(kHashThreads) k_hash16(HashArgs a, const __grid_constant__ HashConsts c) {
+  __shared__ uint64_t s_boff[kH16Req + 1];
+  __shared__ uint64_t s_toff[kH16Req + 1];
+  constexpr uint32_t TB = kHashThreads;
+  const uint32_t tile = blockIdx.x;
+  uint64_t N = a.st->value[0];
+  if (N > a.keys_cap) N = a.keys_cap;
+  const uint64_t b0 = (uint64_t)tile * TB;
+  if (b0 >= N) return;
+  const uint64_t b_end = b0 + TB < N ? b0 + TB : N;
+  const uint64_t ntiles = (N + TB - 1) / TB;
+  const uint32_t r_first = a.tile_req[tile];
+  const uint32_t r_last = tile + 1 < ntiles ? a.tile_req[tile + 1] : a.R - 1;  // the last request meeting the tile
+  const uint32_t nreq = r_last - r_first + 1;
+  const bool cached = nreq <= kH16Req;
+  if (cached) {
+    for (uint32_t i = threadIdx.x; i <= nreq; i += kHashThreads) {
+      s_boff[i] = a.blk_off[r_first + i];
+      s_toff[i] = a.tok_off[r_first + i];
+    }
+  }
+  __syncthreads();
+  const uint32_t t = threadIdx.x;
+  const uint64_t b = b0 + t;
+  uint64_t h0 = 0, h1 = 0;
+  uint32_t k = 0;
+  uint64_t wd_x = 0;  // token offset of this thread's block
+  if (b < b_end) {
+    uint64_t x;
+    if (cached) {  // largest i with s_boff[i] <= b
+      uint32_t lo = 0, hi = nreq - 1;
+      while (lo < hi) {
+        const uint32_t mid = (lo + hi + 1) >> 1;
+        if (s_boff[mid] <= b)
+          lo = mid;
+        else
+          hi = mid - 1;
+      }
+      k = (uint32_t)(b - s_boff[lo]);
+      x = s_toff[lo] + 16ULL * k;
+    } else {
+      const uint32_t r = find_request(a.blk_off, r_first, r_last, b);
+      k = (uint32_t)(b - a.blk_off[r]);
+      x = a.tok_off[r] + 16ULL * k;
+    }
+    wd_x = x;
+  }
+  // Each lane reads the four aligned 16-byte words that start its 16 tokens;
+  // a block that does not start on a 16-byte boundary also needs the first
+  // one to three words of the next 16, which the next lane holds when its
+  // block follows on directly (the usual case inside a request).
+  const uint32_t m = (uint32_t)(wd_x & 3);
+  const uint64_t x4 = wd_x - m;
+  uint32_t wd[20];
+  const bool live = b < b_end;
+  const bool whole = live && x4 + 16 <= a.n_tok;
+  {
+    const uint4* q4 = reinterpret_cast<const uint4*>(a.tokens + x4);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint4 v = make_uint4(0, 0, 0, 0);
+      if (whole) v = __ldcs(q4 + q);
+      wd[4 * q] = v.x;
+      wd[4 * q + 1] = v.y;
+      wd[4 * q + 2] = v.z;
+      wd[4 * q + 3] = v.w;
+    }
+    if (live && !whole) {
+#pragma unroll
+      for (int q = 0; q < 16; ++q) wd[q] = x4 + q < a.n_tok ? a.tokens[x4 + q] : 0u;
+    }
+  }
+  const uint64_t x_next = __shfl_down_sync(kFull, wd_x, 1);
+  const uint32_t n0 = __shfl_down_sync(kFull, wd[0], 1), n1 = __shfl_down_sync(kFull, wd[1], 1),
+                 n2 = __shfl_down_sync(kFull, wd[2], 1);
+  const bool follows = (threadIdx.x & 31) != 31 && x_next == wd_x + 16 && whole;
+  wd[16] = n0;
+  wd[17] = n1;
+  wd[18] = n2;
+  wd[19] = 0;
+  if (live && m && !follows) {
+    const uint64_t y = x4 + 16;
+    if (y + 4 <= a.n_tok) {
+      const uint4 v = __ldcs(reinterpret_cast<const uint4*>(a.tokens + y));
+      wd[16] = v.x;
+      wd[17] = v.y;
+      wd[18] = v.z;
+    } else {
+      wd[16] = y < a.n_tok ? a.tokens[y] : 0u;
+      wd[17] = y + 1 < a.n_tok ? a.tokens[y + 1] : 0u;
+      wd[18] = y + 2 < a.n_tok ? a.tokens[y + 2] : 0u;
+    }
+  }
+  if (live) {
+    uint64_t acc[6] = {0, 0, 0, 0, 0, 0};
+    switch (m) {
+      case 0: hash16<0>(wd, c, acc); break;
+      case 1: hash16<1>(wd, c, acc); break;
+      case 2: hash16<2>(wd, c, acc); break;
+      default: hash16<3>(wd, c, acc); break;
+    }
+    h0 = p61_add(limbs_to_p61(acc[0], acc[1], acc[2]), c.csum[0][16]);
+    h1 = p61_add(limbs_to_p61(acc[3], acc[4], acc[5]), c.csum[1][16]);
+  }
+  hash_finish<1>(a, tile, b0, b_end, h0, h1, k, t, 0);
+}
+
 // Carry of every tile = the segmented sum of the aggregates of the tiles
 // before it, back to (and including) the nearest one where a request starts.
 // All aggregates exist before this kernel starts, so nothing waits.  One warp
-// per tile: each round reads 32 predecessors; then the tile's leading blocks
-// (the tail of a request that started earlier) get the carry and their key.
+// per tile: each round reads 32 predecessors; then the carry is added to the
+// tile's leading blocks (the tail of a request that started earlier).
 constexpr int kChainWarps = 8;
 __global__ void __launch_bounds__(kChainWarps * 32) k_hash_chain(ulonglong2* __restrict__ keys,
                                                                  const HashCarry* __restrict__ tile_agg,
-                                                                 const uint32_t* __restrict__ tile_lead,
-                                                                 const uint32_t* __restrict__ tile_req,
-                                                                 const uint64_t* __restrict__ blk_off,
-                                                                 const uint64_t* tables, uint32_t TB,
+                                                                 const uint32_t* __restrict__ tile_lead, uint32_t TB,
                                                                  const DevStatus* st, uint64_t keys_cap) {
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t tile = blockIdx.x * kChainWarps + (threadIdx.x >> 5);
@@ -537,20 +646,17 @@ __global__ void __launch_bounds__(kChainWarps * 32) k_hash_chain(ulonglong2* __r
     c1 = p61_add(c1, v1);
     if (heads) break;
   }
-  const uint64_t kb = blk_off[tile_req[tile]];
   for (uint32_t i = lane; i < lead; i += 32) {
-    const uint64_t b = b0 + i;
-    const ulonglong2 k = keys[b];
-    const uint64_t e = b - kb + 1;
-    const uint64_t H0 = p61_mul(p61_add(k.x, c0), pow_at(tables + 0 * 65536, tables + 2 * 65536, e));
-    const uint64_t H1 = p61_mul(p61_add(k.y, c1), pow_at(tables + 4 * 65536, tables + 6 * 65536, e));
-    keys[b] = make_ulonglong2(H0, H1);
+    const ulonglong2 k = keys[b0 + i];
+    keys[b0 + i] = make_ulonglong2(p61_add(k.x, c0), p61_add(k.y, c1));
   }
 }
 
 template <int G>
 void launch_hash(uint32_t grid, cudaStream_t s, const HashArgs& a, const HashConsts& c, bool full) {
-  if (full && a.aligned)
+  if (G == 1 && full && a.aligned)
+    PTC_LAUNCH("k_hash16", s, k_hash16<<<grid, kHashThreads, 0, s>>>(a, c));
+  else if (full && a.aligned)
     PTC_LAUNCH("k_hash_local", s, k_hash_local_vec<G><<<grid, kHashThreads, 0, s>>>(a, c));
   else if (full)
     PTC_LAUNCH("k_hash_local", s, k_hash_local<G, true><<<grid, kHashThreads, 0, s>>>(a, c));
@@ -588,7 +694,7 @@ HashLayout hash_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   L.zero_bytes = cv.off;
   L.tile_agg = cv.take<HashCarry>(hash_tiles);
   L.tile_lead = cv.take<uint32_t>(hash_tiles);
-  L.tables = cv.take<uint64_t>(8 * 65536);
+  L.tables = cv.take<uint64_t>(4 * 65536);
   L.tile_req = cv.take<uint32_t>(hash_tiles + 1);
   L.hash_tiles = hash_tiles;
   L.total = cv.bytes();
@@ -635,22 +741,23 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
   PowBases pb;
   HashConsts hc;
   for (int b = 0; b < 2; ++b) {
-    const uint64_t rho = 2 + splitmix64_at(seed, (uint64_t)b) % (kP61 - 3);
-    const uint64_t rinv = p61_pow(rho, kP61 - 2);
-    const uint64_t rB = p61_pow(rho, block_size), riB = p61_pow(rinv, block_size);
-    pb.base[b * 4 + 0] = rB;
-    pb.base[b * 4 + 1] = riB;
-    pb.base[b * 4 + 2] = p61_pow(rB, 65536);
-    pb.base[b * 4 + 3] = p61_pow(riB, 65536);
+    const uint64_t u = 2 + splitmix64_at(seed, (uint64_t)b) % (kP61 - 3);
+    const uint64_t uB = p61_pow(u, block_size);
+    pb.base[b * 2 + 0] = uB;
+    pb.base[b * 2 + 1] = p61_pow(uB, 65536);
+    uint64_t sum = 0;
+    hc.csum[b][0] = 0;
     for (int j = 0; j < 16; ++j) {
-      const uint64_t v = p61_pow(rho, 15 - j);
+      const uint64_t v = p61_pow(u, j + 1);
       hc.limb[b][0][j] = (uint32_t)(v & 0x1FFFFF);
       hc.limb[b][1][j] = (uint32_t)((v >> 21) & 0x1FFFFF);
       hc.limb[b][2][j] = (uint32_t)(v >> 42);
+      sum = p61_add(sum, v);
+      hc.csum[b][j + 1] = sum;
     }
-    for (int q = 0; q < 32; ++q) hc.sub_mul[b][q] = p61_pow(rho, 16ULL * q);
+    for (int q = 0; q < 32; ++q) hc.sub_mul[b][q] = p61_pow(u, 16ULL * q);
   }
-  PTC_LAUNCH("k_pow_tables", s, k_pow_tables<<<(8 * 1024) / 256, 256, 0, s>>>(pb, L.tables));
+  PTC_LAUNCH("k_pow_tables", s, k_pow_tables<<<(4 * 1024) / 256, 256, 0, s>>>(pb, L.tables, L.st));
 
   HashArgs a;
   a.tokens = tokens;
@@ -680,8 +787,8 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
       default: launch_hash<32>(grid, s, a, hc, full); break;
     }
     PTC_LAUNCH("k_hash_chain", s,
-               k_hash_chain<<<ceil_div_u32(grid, kChainWarps), kChainWarps * 32, 0, s>>>(a.keys, L.tile_agg, L.tile_lead, L.tile_req, req_blk_off_out,
-                                                 L.tables, kHashThreads / G, L.st, keys_cap));
+               k_hash_chain<<<ceil_div_u32(grid, kChainWarps), kChainWarps * 32, 0, s>>>(
+                   a.keys, L.tile_agg, L.tile_lead, kHashThreads / G, L.st, keys_cap));
   }
   DevStatus h;
   ptc_status rc = end_call(L.st, s, &h);

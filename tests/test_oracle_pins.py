@@ -289,26 +289,27 @@ def test_splitmix_published_vector():
 
 @pytest.mark.parametrize("seed", [0, 1, 12345, 2**63 + 7])
 def test_prefix_hash_polynomial(seed):
-    """Keys equal the polynomial of (1, tok_0, ..., tok_{m-1}) at the two
-    seeded bases, evaluated with Python integers from the sum definition."""
+    """Keys equal sum_t (tok_t + 1) u^(t+1) mod 2^61 - 1 over the block's
+    whole prefix at the two seeded bases, evaluated with Python integers from
+    the sum definition (tokens up to 2^32 - 1 included)."""
     tr = tracegen.tiny(seed % 1000, n_sessions=4, vocab=2**32 - 1 if seed & 1 else 5)
     B = 3
     keys = oracle.prefix_hash(tr.tokens, tr.req_tok_off, B, seed)
-    rho = [2 + _splitmix(seed, b) % (P61 - 3) for b in range(2)]
+    u = [2 + _splitmix(seed, b) % (P61 - 3) for b in range(2)]
     i = 0
     for a, b in zip(tr.req_tok_off[:-1], tr.req_tok_off[1:]):
         toks = [int(x) for x in tr.tokens[int(a):int(b)]]
         for k in range(len(toks) // B):
             m = B * (k + 1)
             for base in range(2):
-                h = pow(rho[base], m, P61) + sum(toks[t] * pow(rho[base], m - 1 - t, P61) for t in range(m))
+                h = sum((toks[t] + 1) * pow(u[base], t + 1, P61) for t in range(m))
                 assert int(keys[i, base]) == h % P61
             i += 1
     assert i == keys.shape[0]
 
 
 def test_prefix_hash_separates_lengths():
-    """The leading 1 keeps a prefix and a zero-extended prefix apart."""
+    """Coefficients tok + 1 >= 1 keep a prefix and its zero-extension apart."""
     tr = tracegen.from_lists([[0, 0], [0, 0, 0, 0]])
     keys = oracle.prefix_hash(tr.tokens, tr.req_tok_off, 2, 99)
     assert not np.array_equal(keys[0], keys[2])
