@@ -257,12 +257,14 @@ __device__ __forceinline__ void hash_finish(const HashArgs& a, uint32_t tile, ui
       h1 = p61_add(h1, __shfl_xor_sync(kFull, h1, o));
     }
   }
-  if (s == 0) {
-    s_h0[lb] = h0;
-    s_h1[lb] = h1;
-    s_k[lb] = k;
+  if (G > 1) {  // one value per block: the sub-chunk holding it hands it over
+    if (s == 0) {
+      s_h0[lb] = h0;
+      s_h1[lb] = h1;
+      s_k[lb] = k;
+    }
+    __syncthreads();
   }
-  __syncthreads();
 
   // ---- phase 2: normalise, segmented sum over requests, denormalise
   const uint32_t t = threadIdx.x;
@@ -271,9 +273,9 @@ __device__ __forceinline__ void hash_finish(const HashArgs& a, uint32_t tile, ui
   HashCarry x{0, 0, 0};
   uint32_t kk = 0;
   if (valid) {
-    kk = s_k[t];
-    x.v0 = p61_mul(s_h0[t], pow_at(T + 0 * 65536, T + 1 * 65536, kk));
-    x.v1 = p61_mul(s_h1[t], pow_at(T + 2 * 65536, T + 3 * 65536, kk));
+    kk = G > 1 ? s_k[t] : k;
+    x.v0 = p61_mul(G > 1 ? s_h0[t] : h0, pow_at(T + 0 * 65536, T + 1 * 65536, kk));
+    x.v1 = p61_mul(G > 1 ? s_h1[t] : h1, pow_at(T + 2 * 65536, T + 3 * 65536, kk));
     x.f = kk == 0;
   }
   SegSumOp op;
@@ -504,7 +506,7 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local_vec(HashArgs a, con
 // global offsets instead.
 constexpr int kH16Req = 256;
 
-__global__ void __launch_bounds__(kHashThreads) k_hash16(HashArgs a, const __grid_constant__ HashConsts c) {
+__global__ void __launch_bounds__(kHashThreads, 4) k_hash16(HashArgs a, const __grid_constant__ HashConsts c) {
   __shared__ uint64_t s_boff[kH16Req + 1];
   __shared__ uint64_t s_toff[kH16Req + 1];
   constexpr uint32_t TB = kHashThreads;
