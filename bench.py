@@ -48,7 +48,11 @@ NOMINAL_HBM_GBS = 7900.0
 # Per-launch DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) from
 # the last ncu capture of each kernel, with the sha256 of the source file it
 # was taken on; a changed source reads as "no counters" (null).
-NCU_TRAFFIC: dict[str, tuple[float, str, str]] = {}
+NCU_TRAFFIC: dict[str, tuple[float, str, str]] = {
+    # 6,000-request capture (profiles/k_hash16_chat_6000req.md), scaled to the
+    # full workload by tokens
+    "k_hash16": (647.3e6, "585611a3129b3a42", "ncu --set full, first 6,000 requests, x 153.81 / 55.67"),
+}
 
 
 def parse_args():
@@ -63,6 +67,8 @@ def parse_args():
     ap.add_argument("--ref-sample", type=float, default=1.0,
                     help="fraction of requests per --impl reference step")
     ap.add_argument("--json-out", default=None)
+    ap.add_argument("--requests", type=int, default=0,
+                    help="run only the first N requests of the workload (small cases for profiling)")
     return ap.parse_args()
 
 
@@ -229,9 +235,14 @@ def run_ours(args, ws_world, rank, local):
 
     L = ptc.lib()
     # the trace, generated into pinned host memory (the end-to-end leg copies from it)
-    R, T, _ = tracegen.sizes(WORKLOAD)
-    tok_host = torch.empty(T, dtype=torch.int32, pin_memory=True)
-    tr = tracegen.make(WORKLOAD, token_buffer=tok_host.numpy().view(np.uint32))
+    if args.requests:
+        tr = tracegen.make(WORKLOAD, max_requests=args.requests)
+        T = tr.n_tok
+        tok_host = torch.from_numpy(tr.tokens.view(np.int32)).pin_memory()
+    else:
+        R, T, _ = tracegen.sizes(WORKLOAD)
+        tok_host = torch.empty(T, dtype=torch.int32, pin_memory=True)
+        tr = tracegen.make(WORKLOAD, token_buffer=tok_host.numpy().view(np.uint32))
     off_host = torch.from_numpy(tr.req_tok_off.view(np.int64)).pin_memory()
     ts_host = torch.from_numpy(tr.req_ts_us).pin_memory()
     tok = tok_host.to(dev, non_blocking=True)
@@ -336,7 +347,8 @@ def run_ours(args, ws_world, rank, local):
                                "measured-shape cost",
                    "tokens": T, "requests": tr.n_req, "accesses": N, "distinct_blocks": D, "block_size": BLOCK,
                    "capacities": G, "l2": "flushed between timed steps (256 MiB write, outside the events)",
-                   "parallelism": "replicas" if ws_world > 1 else "single GPU"},
+                   "parallelism": "replicas" if ws_world > 1 else "single GPU",
+                   "prefix_requests": args.requests or None},
         "accesses_per_s": round(acc_s, 1),
         "hbm_roofline": {"stage_model_bytes": model_total, "L": Lbits,
                          "frac_of_measured": round(model_total / (ms_per_step * 1e-3) / 1e9 / peak, 4),
