@@ -11,9 +11,21 @@
 // cost(k) = alpha + beta k, so compute saved = alpha * hits + beta * (sum of k),
 // formed exactly in 128 bits by the finalize kernel.
 //   k_heads     marks the first access of every non-empty request (bitmap)
+//   k_curves_fast  when the distances never fall inside a request (the case
+//               for any trace whose blocks are root-first: a longer prefix
+//               is never more recently used than its parent), the running
+//               max is the distance itself; bins and depths straight from
+//               the distances, request starts from a per-tile table.  A
+//               fall inside a request sets a flag, and then the scan
+//               kernels below redo the curves from scratch.
 //   k_curves    running max, bin search in shared memory, run-merged
 //               shared histograms, one global atomic per non-empty bin
-//   k_finalize  cumulative sums over bins; 128-bit saved and total cost
+//   k_curves_runs  (ptc_pipeline) the same from stage c's runs: one thread
+//               per request, one (count, depth sum) per piece of a run that
+//               lies in the request; a fall between the runs of a request
+//               sets the flag for the scan kernels
+//   k_finalize  cumulative sums over bins (a block scan); 128-bit saved and
+//               total cost
 #include "ptc_internal.h"
 
 namespace ptc {
@@ -22,10 +34,11 @@ namespace {
 constexpr int kCvThreads = 512;
 constexpr int kCvPer = 8;
 constexpr int kCvTile = kCvThreads * kCvPer;
-constexpr int kEpochCurves = 1;
 
+// Also records, for every tile of kCvTile accesses, the request holding its
+// first access (each tile has exactly one such request).
 __global__ void k_heads(const uint64_t* __restrict__ blk_off, uint32_t R, uint64_t n, uint32_t* __restrict__ bitmap,
-                        DevStatus* st) {
+                        uint32_t* __restrict__ tile_req, DevStatus* st) {
   const uint64_t r = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= R) return;
   const uint64_t a = blk_off[r], b = blk_off[r + 1];
@@ -33,7 +46,10 @@ __global__ void k_heads(const uint64_t* __restrict__ blk_off, uint32_t R, uint64
     raise_err(st, kErrInvalid);
     return;
   }
-  if (b > a) atomicOr(&bitmap[a >> 5], 1u << (a & 31));
+  if (b > a) {
+    atomicOr(&bitmap[a >> 5], 1u << (a & 31));
+    for (uint64_t t = (a + kCvTile - 1) / kCvTile; t * kCvTile < b; ++t) tile_req[t] = (uint32_t)r;
+  }
 }
 
 struct RunMax {  // (segment-start flag, running max, start index of the segment); n < 2^32 - 1
@@ -63,6 +79,10 @@ struct CurveArgs {
   unsigned long long* ksum;  // G + 1 bins
   const RunMax* tile_agg;
   DevStatus* st;
+  const uint64_t* blk_off;   // request block offsets (R + 1)
+  const uint32_t* tile_req;  // request holding each tile's first access
+  uint32_t R;
+  uint32_t* slow;            // set when a distance falls inside a request
 };
 
 // Loads the kCvPer distances of this thread and the head bits of its range,
@@ -137,8 +157,13 @@ __device__ __forceinline__ void cta_runmax_scan(RunMax& x, RunMax* s_w) {
 // last start, index of that start).  Tiles are independent.
 __global__ void __launch_bounds__(kCvThreads) k_curves_agg(const uint32_t* __restrict__ dist, uint32_t n,
                                                            const uint32_t* __restrict__ bitmap,
-                                                           RunMax* __restrict__ tile_agg) {
+                                                           RunMax* __restrict__ tile_agg, const uint32_t* slow,
+                                                           unsigned long long* cnt, unsigned long long* ksum,
+                                                           uint32_t G) {
   __shared__ RunMax s_w[kCvThreads / 32];
+  if (!*slow) return;  // k_curves_fast's bins stand
+  if (blockIdx.x == 0)  // the scan path starts the bins afresh
+    for (uint32_t g = threadIdx.x; g <= G; g += kCvThreads) cnt[g] = ksum[g] = 0;
   const uint32_t i0 = blockIdx.x * kCvTile + threadIdx.x * kCvPer;
   uint32_t e[kCvPer], st_idx[kCvPer];
   uint32_t has_head;
@@ -152,6 +177,7 @@ __global__ void __launch_bounds__(kCvThreads) k_curves_agg(const uint32_t* __res
 // and keeps its bin histograms in shared memory across them, so the global
 // bins see one atomic per CTA and bin rather than per tile.
 __global__ void __launch_bounds__(kCvThreads) k_curves(CurveArgs a) {
+  if (!*a.slow) return;
   __shared__ uint32_t s_cap[PTC_MAX_CAPACITIES];
   __shared__ uint32_t s_cnt[PTC_MAX_CAPACITIES + 1];
   __shared__ unsigned long long s_ks[PTC_MAX_CAPACITIES + 1];
@@ -277,6 +303,211 @@ __global__ void __launch_bounds__(kCvThreads) k_curves(CurveArgs a) {
   }
 }
 
+
+// Bin of e among the capacities (first capacity >= e; G for a first access).
+__device__ __forceinline__ uint32_t bin_of(const uint32_t* s_cap, uint32_t G, uint32_t e) {
+  if (e == kNone) return G;
+  uint32_t lo = 0, hi = G;
+  while (lo < hi) {
+    const uint32_t mid = (lo + hi) >> 1;
+    if (s_cap[mid] >= e)
+      hi = mid;
+    else
+      lo = mid + 1;
+  }
+  return lo;
+}
+
+constexpr int kFtReq = 128;  // requests a tile's table holds
+
+__global__ void __launch_bounds__(kCvThreads) k_curves_fast(CurveArgs a) {
+  __shared__ uint32_t s_cap[PTC_MAX_CAPACITIES];
+  __shared__ uint32_t s_cnt[PTC_MAX_CAPACITIES + 1];
+  __shared__ unsigned long long s_ks[PTC_MAX_CAPACITIES + 1];
+  __shared__ uint32_t s_off[kFtReq + 2];
+  const uint32_t G = a.G;
+  for (uint32_t g = threadIdx.x; g < G; g += kCvThreads)
+    s_cap[g] = a.caps[g] >= (uint64_t)kNone ? kNone - 1 : (uint32_t)a.caps[g];
+  for (uint32_t g = threadIdx.x; g <= G; g += kCvThreads) {
+    s_cnt[g] = 0;
+    s_ks[g] = 0;
+  }
+  const uint32_t ntiles = (a.n + kCvTile - 1) / kCvTile;
+  const uint32_t lane = threadIdx.x & 31;
+  bool fell = false;
+  for (uint32_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+    const uint32_t t0 = tile * kCvTile, t1 = min(t0 + kCvTile, a.n) - 1;  // first / last access of the tile
+    const uint32_t i0 = t0 + threadIdx.x * kCvPer;
+    uint32_t d[kCvPer];
+    if (i0 + kCvPer <= a.n && ((reinterpret_cast<uintptr_t>(a.dist) & 15) == 0)) {
+      const uint4 x = __ldg(reinterpret_cast<const uint4*>(a.dist + i0));
+      const uint4 y = __ldg(reinterpret_cast<const uint4*>(a.dist + i0 + 4));
+      d[0] = x.x; d[1] = x.y; d[2] = x.z; d[3] = x.w;
+      d[4] = y.x; d[5] = y.y; d[6] = y.z; d[7] = y.w;
+    } else {
+#pragma unroll
+      for (int j = 0; j < kCvPer; ++j) d[j] = i0 + j < a.n ? a.dist[i0 + j] : 0u;
+    }
+    (void)t1;
+    // the requests meeting the tile: from the one holding its first access to
+    // the one holding the next tile's first access
+    const uint32_t r0 = a.tile_req[tile];
+    const uint32_t r1 = tile + 1 < ntiles ? a.tile_req[tile + 1] : a.R - 1;
+    const bool cached = r1 - r0 + 1 <= kFtReq;
+    if (cached)
+      for (uint32_t k = threadIdx.x; k <= r1 - r0 + 1; k += kCvThreads) s_off[k] = (uint32_t)a.blk_off[r0 + k];
+    __syncthreads();
+    uint32_t before = __shfl_up_sync(kFull, d[kCvPer - 1], 1);  // distance of access i0 - 1
+    if (lane == 0) before = i0 > 0 && i0 - 1 < a.n ? a.dist[i0 - 1] : 0u;
+    uint32_t cur_g = 0xFFFFFFFFu, run_c = 0;
+    unsigned long long run_k = 0;
+    if (i0 < a.n) {
+      // request of access i0, then walk forward
+      uint32_t idx, start, nxt;
+      if (cached) {
+        uint32_t lo = 0, hi = r1 - r0;
+        while (lo < hi) {
+          const uint32_t mid = (lo + hi + 1) >> 1;
+          if (s_off[mid] <= i0)
+            lo = mid;
+          else
+            hi = mid - 1;
+        }
+        idx = lo;
+        start = s_off[idx];
+        nxt = s_off[idx + 1];
+      } else {
+        uint32_t lo = r0, hi = r1;
+        while (lo < hi) {
+          const uint32_t mid = (lo + hi + 1) >> 1;
+          if (a.blk_off[mid] <= i0)
+            lo = mid;
+          else
+            hi = mid - 1;
+        }
+        idx = lo;
+        start = (uint32_t)a.blk_off[idx];
+        nxt = (uint32_t)a.blk_off[idx + 1];
+      }
+      uint32_t last_e = 0xFFFFFFFEu, last_g = G;
+      uint32_t prev_d = before;
+#pragma unroll
+      for (int j = 0; j < kCvPer; ++j) {
+        const uint32_t i = i0 + j;
+        if (i >= a.n) break;
+        while (i >= nxt) {  // the next non-empty request
+          ++idx;
+          start = nxt;
+          nxt = cached ? s_off[idx + 1] : (uint32_t)a.blk_off[idx + 1];
+        }
+        const uint32_t e = d[j];
+        if (i != start && e < prev_d) fell = true;
+        prev_d = e;
+        if (e != last_e) {
+          last_g = bin_of(s_cap, G, e);
+          last_e = e;
+        }
+        const uint32_t g = last_g;
+        if (g != cur_g) {
+          if (run_c) {
+            atomicAdd(&s_cnt[cur_g], run_c);
+            atomicAdd(&s_ks[cur_g], run_k);
+          }
+          cur_g = g;
+          run_c = 0;
+          run_k = 0;
+        }
+        ++run_c;
+        run_k += i - start;
+      }
+    }
+    // the open run of every lane; inside long runs the whole warp shares one
+    // bin, so it sums across lanes and adds once
+    const uint32_t g0 = __shfl_sync(kFull, cur_g, 0);
+    if (__all_sync(kFull, cur_g == g0 || run_c == 0)) {
+      uint32_t c = run_c;
+      unsigned long long kk = run_k;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        c += __shfl_xor_sync(kFull, c, o);
+        kk += __shfl_xor_sync(kFull, kk, o);
+      }
+      if (lane == 0 && c) {
+        atomicAdd(&s_cnt[g0], c);
+        atomicAdd(&s_ks[g0], kk);
+      }
+    } else if (run_c) {
+      atomicAdd(&s_cnt[cur_g], run_c);
+      atomicAdd(&s_ks[cur_g], run_k);
+    }
+    __syncthreads();  // s_r / s_off are reused by the next tile
+  }
+  if (__syncthreads_or(fell) && threadIdx.x == 0) atomicOr(a.slow, 1u);
+  for (uint32_t g = threadIdx.x; g <= G; g += kCvThreads) {
+    if (s_cnt[g]) {
+      atomicAdd(&a.cnt[g], (unsigned long long)s_cnt[g]);
+      atomicAdd(&a.ksum[g], s_ks[g]);
+    }
+  }
+}
+
+
+// Index of the run holding access j (stage c's run-start bitmap and the runs
+// starting before each 32-access word).
+__device__ __forceinline__ uint32_t run_at(const uint32_t* bits, const uint32_t* wpre, uint32_t j) {
+  const uint32_t wi = j >> 5, b = j & 31;
+  const uint32_t mask_le = b == 31 ? kFull : ((2u << b) - 1u);
+  return wpre[wi] + __popc(bits[wi] & mask_le) - 1u;
+}
+
+struct RunsArgs {
+  const uint32_t* rec_s;
+  const uint32_t* sd;
+  const uint32_t* bits;
+  const uint32_t* wpre;
+};
+
+__global__ void __launch_bounds__(256) k_curves_runs(CurveArgs a, RunsArgs ra) {
+  __shared__ uint32_t s_cap[PTC_MAX_CAPACITIES];
+  __shared__ uint32_t s_cnt[PTC_MAX_CAPACITIES + 1];
+  __shared__ unsigned long long s_ks[PTC_MAX_CAPACITIES + 1];
+  const uint32_t G = a.G;
+  for (uint32_t g = threadIdx.x; g < G; g += blockDim.x)
+    s_cap[g] = a.caps[g] >= (uint64_t)kNone ? kNone - 1 : (uint32_t)a.caps[g];
+  for (uint32_t g = threadIdx.x; g <= G; g += blockDim.x) {
+    s_cnt[g] = 0;
+    s_ks[g] = 0;
+  }
+  __syncthreads();
+  bool fell = false;
+  for (uint32_t q = blockIdx.x * blockDim.x + threadIdx.x; q < a.R; q += gridDim.x * blockDim.x) {
+    const uint32_t start = (uint32_t)a.blk_off[q], end = (uint32_t)a.blk_off[q + 1];
+    if (end <= start || end > a.n) continue;  // empty (bad offsets are reported by k_heads)
+    const uint32_t r0 = run_at(ra.bits, ra.wpre, start), r1 = run_at(ra.bits, ra.wpre, end - 1);
+    uint32_t prev_v = 0, last_v = 0xFFFFFFFEu, g = G;
+    for (uint32_t r = r0; r <= r1; ++r) {
+      const uint32_t s0 = max(ra.rec_s[r], start), e0 = min(ra.rec_s[r + 1], end), v = ra.sd[r];
+      if (v < prev_v) fell = true;  // the running max would bind
+      prev_v = v;
+      if (v != last_v) {
+        g = bin_of(s_cap, G, v);
+        last_v = v;
+      }
+      const uint32_t c = e0 - s0;
+      const unsigned long long k0 = s0 - start;
+      atomicAdd(&s_cnt[g], c);
+      atomicAdd(&s_ks[g], (unsigned long long)c * k0 + (unsigned long long)c * (c - 1) / 2);
+    }
+  }
+  if (__syncthreads_or(fell) && threadIdx.x == 0) atomicOr(a.slow, 1u);
+  for (uint32_t g = threadIdx.x; g <= G; g += blockDim.x) {
+    if (s_cnt[g]) {
+      atomicAdd(&a.cnt[g], (unsigned long long)s_cnt[g]);
+      atomicAdd(&a.ksum[g], s_ks[g]);
+    }
+  }
+}
+
 struct U128 {
   uint64_t lo, hi;
 };
@@ -288,23 +519,43 @@ __device__ __forceinline__ U128 add_u128(U128 a, U128 b) {
   return r;
 }
 
-// out layout: hits[G] | saved[G] (lo, hi) | total (lo, hi)
-__global__ void k_finalize(const unsigned long long* __restrict__ cnt, const unsigned long long* __restrict__ ksum,
-                           uint32_t G, uint64_t alpha, uint64_t beta, uint64_t* __restrict__ out) {
-  if (threadIdx.x != 0 || blockIdx.x != 0) return;
-  uint64_t h = 0, k = 0;
-  for (uint32_t g = 0; g < G; ++g) {
-    h += cnt[g];
-    k += ksum[g];
-    const U128 s = add_u128(mul_u64(alpha, h), mul_u64(beta, k));
-    out[g] = h;
-    out[G + 2 * g] = s.lo;
-    out[G + 2 * g + 1] = s.hi;
+// out layout: hits[G] | saved[G] (lo, hi) | total (lo, hi).  One CTA of
+// 1,024 threads: an inclusive block scan of (count, depth sum) over the bins.
+__global__ void __launch_bounds__(1024) k_finalize(const unsigned long long* __restrict__ cnt,
+                                                   const unsigned long long* __restrict__ ksum, uint32_t G,
+                                                   uint64_t alpha, uint64_t beta, uint64_t* __restrict__ out) {
+  __shared__ unsigned long long s_h[32], s_k[32];
+  const uint32_t t = threadIdx.x, lane = t & 31, w = t >> 5;
+  unsigned long long h = t < G ? cnt[t] : 0ull, k = t < G ? ksum[t] : 0ull;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned long long yh = __shfl_up_sync(kFull, h, o), yk = __shfl_up_sync(kFull, k, o);
+    if (lane >= (uint32_t)o) {
+      h += yh;
+      k += yk;
+    }
   }
-  const uint64_t hn = h + cnt[G], kn = k + ksum[G];
-  const U128 t = add_u128(mul_u64(alpha, hn), mul_u64(beta, kn));
-  out[3 * G] = t.lo;
-  out[3 * G + 1] = t.hi;
+  if (lane == 31) {
+    s_h[w] = h;
+    s_k[w] = k;
+  }
+  __syncthreads();
+  for (uint32_t ww = 0; ww < w; ++ww) {
+    h += s_h[ww];
+    k += s_k[ww];
+  }
+  if (t < G) {
+    const U128 sv = add_u128(mul_u64(alpha, h), mul_u64(beta, k));
+    out[t] = h;
+    out[G + 2 * t] = sv.lo;
+    out[G + 2 * t + 1] = sv.hi;
+  }
+  if (t == G - 1) {  // G >= 1; the miss bin G joins the total
+    const uint64_t hn = h + cnt[G], kn = k + ksum[G];
+    const U128 tc = add_u128(mul_u64(alpha, hn), mul_u64(beta, kn));
+    out[3 * G] = tc.lo;
+    out[3 * G + 1] = tc.hi;
+  }
 }
 
 struct CurvesLayout {
@@ -312,6 +563,8 @@ struct CurvesLayout {
   unsigned long long* cnt;
   unsigned long long* ksum;
   uint32_t* bitmap;
+  uint32_t* slow;
+  uint32_t* tile_req;
   RunMax* lb_agg;
   uint64_t* caps;
   uint64_t* out;
@@ -327,6 +580,8 @@ CurvesLayout curves_layout(void* ws, uint64_t n, uint32_t G) {
   L.cnt = cv.take<unsigned long long>(PTC_MAX_CAPACITIES + 1);
   L.ksum = cv.take<unsigned long long>(PTC_MAX_CAPACITIES + 1);
   L.bitmap = cv.take<uint32_t>(n / 32 + 2);
+  L.slow = cv.take<uint32_t>(1);
+  L.tile_req = cv.take<uint32_t>(tiles + 1);
   L.zero_bytes = cv.off;
   L.lb_agg = cv.take<RunMax>(tiles);
   L.caps = cv.take<uint64_t>(PTC_MAX_CAPACITIES);
@@ -352,10 +607,10 @@ extern "C" size_t ptc_curves_workspace_bytes(uint64_t n, uint32_t n_req, uint32_
   return curves_layout(nullptr, n, n_cap).total;
 }
 
-extern "C" ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,
-                                 uint32_t block_size, const ptc_cost_model* cm, const uint64_t* cap_host, uint32_t n_cap,
-                                 uint64_t* hits_host_out, ptc_u128* saved_host_out, ptc_u128* total_cost_host_out,
-                                 void* ws, size_t ws_bytes, void* stream) {
+ptc_status ptc::curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,
+                            uint32_t block_size, const ptc_cost_model* cm, const uint64_t* cap_host, uint32_t n_cap,
+                            uint64_t* hits_host_out, ptc_u128* saved_host_out, ptc_u128* total_cost_host_out,
+                            void* ws, size_t ws_bytes, cudaStream_t stream, const RunsView* runs) {
   if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
   if (!cm || !cap_host || !hits_host_out || !saved_host_out || !total_cost_host_out) return PTC_ERR_INVALID_ARG;
   if (n_cap < 1 || n_cap > PTC_MAX_CAPACITIES) return PTC_ERR_INVALID_ARG;
@@ -377,13 +632,14 @@ extern "C" ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_
     return PTC_ERR_INVALID_ARG;
   }
   if (!ws_ok(ws, ws_bytes, curves_layout(nullptr, n, n_cap).total)) return PTC_ERR_WORKSPACE;
-  cudaStream_t s = (cudaStream_t)stream;
+  cudaStream_t s = stream;
   const CurvesLayout L = curves_layout(ws, n, n_cap);
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
   if (cudaMemcpyAsync(L.caps, cap_host, sizeof(uint64_t) * n_cap, cudaMemcpyHostToDevice, s) != cudaSuccess)
     return PTC_ERR_CUDA;
   if (n > 0) {
-    PTC_LAUNCH("k_heads", s, k_heads<<<ceil_div_u32(n_req, 256), 256, 0, s>>>(req_blk_off, n_req, n, L.bitmap, L.st));
+    PTC_LAUNCH("k_heads", s,
+               k_heads<<<ceil_div_u32(n_req, 256), 256, 0, s>>>(req_blk_off, n_req, n, L.bitmap, L.tile_req, L.st));
     CurveArgs a;
     a.dist = dist;
     a.n = (uint32_t)n;
@@ -394,13 +650,28 @@ extern "C" ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_
     a.ksum = L.ksum;
     a.tile_agg = L.lb_agg;
     a.st = L.st;
+    a.blk_off = req_blk_off;
+    a.tile_req = L.tile_req;
+    a.R = n_req;
+    a.slow = L.slow;
+    if (runs && runs->used) {
+      const RunsArgs ra{runs->rec_s, runs->sd, runs->bits, runs->wpre};
+      const uint32_t g_r = ceil_div_u32(n_req, 256) < (uint32_t)(2 * num_sms()) ? ceil_div_u32(n_req, 256)
+                                                                                  : (uint32_t)(2 * num_sms());
+      PTC_LAUNCH("k_curves_runs", s, k_curves_runs<<<g_r, 256, 0, s>>>(a, ra));
+    } else {
+      const uint32_t tiles0 = ceil_div_u32(n, kCvTile);
+      const uint32_t grid0 = tiles0 < (uint32_t)(3 * num_sms()) ? tiles0 : (uint32_t)(3 * num_sms());
+      PTC_LAUNCH("k_curves_fast", s, k_curves_fast<<<grid0, kCvThreads, 0, s>>>(a));
+    }
     PTC_LAUNCH("k_curves_agg", s,
-               k_curves_agg<<<ceil_div_u32(n, kCvTile), kCvThreads, 0, s>>>(dist, (uint32_t)n, L.bitmap, L.lb_agg));
+               k_curves_agg<<<ceil_div_u32(n, kCvTile), kCvThreads, 0, s>>>(dist, (uint32_t)n, L.bitmap, L.lb_agg,
+                                                                          L.slow, L.cnt, L.ksum, n_cap));
     const uint32_t tiles = ceil_div_u32(n, kCvTile);
-    const uint32_t grid = tiles < (uint32_t)(2 * num_sms()) ? tiles : (uint32_t)(2 * num_sms());
+    const uint32_t grid = tiles < (uint32_t)(3 * num_sms()) ? tiles : (uint32_t)(3 * num_sms());
     PTC_LAUNCH("k_curves", s, k_curves<<<grid, kCvThreads, 0, s>>>(a));
   }
-  PTC_LAUNCH("k_finalize", s, k_finalize<<<1, 32, 0, s>>>(L.cnt, L.ksum, n_cap, alpha, beta, L.out));
+  PTC_LAUNCH("k_finalize", s, k_finalize<<<1, 1024, 0, s>>>(L.cnt, L.ksum, n_cap, alpha, beta, L.out));
   static thread_local uint64_t host_out[3 * PTC_MAX_CAPACITIES + 2];
   if (cudaMemcpyAsync(host_out, L.out, sizeof(uint64_t) * (3 * n_cap + 2), cudaMemcpyDeviceToHost, s) != cudaSuccess)
     return PTC_ERR_CUDA;
@@ -415,6 +686,14 @@ extern "C" ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_
   total_cost_host_out->lo = host_out[3 * n_cap];
   total_cost_host_out->hi = host_out[3 * n_cap + 1];
   return PTC_OK;
+}
+
+extern "C" ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,
+                                 uint32_t block_size, const ptc_cost_model* cm, const uint64_t* cap_host, uint32_t n_cap,
+                                 uint64_t* hits_host_out, ptc_u128* saved_host_out, ptc_u128* total_cost_host_out,
+                                 void* ws, size_t ws_bytes, void* stream) {
+  return ptc::curves_impl(dist, n, req_blk_off, n_req, block_size, cm, cap_host, n_cap, hits_host_out, saved_host_out,
+                          total_cost_host_out, ws, ws_bytes, (cudaStream_t)stream, nullptr);
 }
 
 // ---------------------------------------------------------------------------

@@ -57,6 +57,25 @@ inline bool ws_ok(const void* ws, size_t ws_bytes, size_t need) {
   return ws != nullptr && ((uintptr_t)ws & 255) == 0 && ws_bytes >= need;
 }
 
+// The runs stage c leaves in its workspace when it used the matrix over runs
+// (ptc_runs.cu); the pipeline hands them to stage d.
+struct RunsView {
+  bool used = false;
+  uint32_t R = 0;
+  const uint32_t* rec_s = nullptr;  // R + 1 run starts (rec_s[R] = n)
+  const uint32_t* sd = nullptr;     // distance of every run
+  const uint32_t* bits = nullptr;   // run-start bitmap, one word per 32 accesses
+  const uint32_t* wpre = nullptr;   // runs starting before each word
+};
+ptc_status stack_distance_view(const uint32_t* prev, uint64_t n, uint32_t* dist_out, int method, void* ws,
+                               size_t ws_bytes, cudaStream_t s, RunsView* view);
+// Stage d (ptc_curves.cu); with `runs` (from stack_distance_view) the curves
+// come from the runs instead of a pass over every distance.
+ptc_status curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,
+                       uint32_t block_size, const ptc_cost_model* cm, const uint64_t* cap_host, uint32_t n_cap,
+                       uint64_t* hits_host_out, ptc_u128* saved_host_out, ptc_u128* total_cost_host_out, void* ws,
+                       size_t ws_bytes, cudaStream_t s, const RunsView* runs);
+
 // Stage c on the matrix over every access (ptc_wavelet.cu); the C entry
 // points in ptc_runs.cu choose between it and the matrix over runs.
 size_t stack_distance_points_bytes(uint64_t n);

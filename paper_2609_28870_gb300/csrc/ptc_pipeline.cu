@@ -2,7 +2,9 @@
 // needs one crossing of the C boundary.  Intermediate arrays live in caller
 // buffers when given, otherwise in the workspace; the stages' own scratch
 // reuses one region of the workspace because they run one after another on
-// the same stream.
+// the same stream.  Stage d has a region of its own: when stage c used the
+// matrix over runs, the curves come from those runs (still in stage c's
+// scratch) instead of a pass over every distance.
 #include "ptc_internal.h"
 
 namespace {
@@ -13,6 +15,8 @@ struct PipeLayout {
   uint32_t *ids, *prev, *next, *dist;
   void* scratch;
   size_t scratch_bytes;
+  void* curves;
+  size_t curves_bytes;
   size_t total;
 };
 
@@ -20,7 +24,7 @@ size_t stage_scratch_bytes(uint32_t n_req, uint64_t n_tok, uint32_t B, uint32_t 
   const uint64_t n = n_tok / B;
   size_t m = ptc_hash_blocks_workspace_bytes(n_req, n_tok, B);
   const size_t c[] = {ptc_assign_ids_workspace_bytes(n), ptc_reuse_indices_workspace_bytes(n, n),
-                      ptc_stack_distance_workspace_bytes(n), ptc_curves_workspace_bytes(n, n_req, n_cap)};
+                      ptc_stack_distance_workspace_bytes(n)};
   for (size_t x : c) m = x > m ? x : m;
   return m;
 }
@@ -38,6 +42,8 @@ PipeLayout pipe_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   L.dist = dist ? nullptr : cv.take<uint32_t>(n);
   L.scratch_bytes = stage_scratch_bytes(n_req, n_tok, B, n_cap);
   L.scratch = cv.take<unsigned char>(L.scratch_bytes);
+  L.curves_bytes = ptc_curves_workspace_bytes(n_tok / B, n_req, n_cap);
+  L.curves = cv.take<unsigned char>(L.curves_bytes);
   L.total = cv.bytes();
   return L;
 }
@@ -83,9 +89,12 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
   if (n > 0) {
     rc = ptc_reuse_indices(ids, n, d, prev, next, L.scratch, L.scratch_bytes, stream);
     if (rc != PTC_OK) return rc;
-    rc = ptc_stack_distance(prev, n, dist, L.scratch, L.scratch_bytes, stream);
+  }
+  ptc::RunsView runs;
+  if (n > 0) {
+    rc = ptc::stack_distance_view(prev, n, dist, PTC_SD_AUTO, L.scratch, L.scratch_bytes, (cudaStream_t)stream, &runs);
     if (rc != PTC_OK) return rc;
   }
-  return ptc_curves(dist, n, blk, n_req, block_size, cm, cap_host, n_cap, hits_host_out, saved_host_out,
-                    total_cost_host_out, L.scratch, L.scratch_bytes, stream);
+  return ptc::curves_impl(dist, n, blk, n_req, block_size, cm, cap_host, n_cap, hits_host_out, saved_host_out,
+                          total_cost_host_out, L.curves, L.curves_bytes, (cudaStream_t)stream, &runs);
 }

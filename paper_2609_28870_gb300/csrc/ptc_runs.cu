@@ -649,7 +649,7 @@ uint64_t runs_reserve(uint64_t n) {
 }
 
 ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_out, void* ws, size_t ws_bytes,
-                               cudaStream_t s, int method) {
+                               cudaStream_t s, int method, RunsView* view) {
   const RunsLayout M = runs_layout(ws, n, 1);
   if (!ws_ok(ws, ws_bytes, M.total)) return PTC_ERR_WORKSPACE;
   if (begin_call(ws, M.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
@@ -757,10 +757,30 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   PTC_LAUNCH("k_runs_query", s, k_runs_query<<<ceil_div_u32(R, 256), 256, 0, s>>>(q));
   PTC_LAUNCH("k_runs_expand", s,
              k_runs_expand<<<ceil_div_u32(n, 256), 256, 0, s>>>(W.bits, W.wpre, W.sd, (uint32_t)n, dist_out));
-  return end_call(W.st, s, &h);
+  const ptc_status done = end_call(W.st, s, &h);
+  if (done == PTC_OK && view) {
+    view->used = true;
+    view->R = R32;
+    view->rec_s = W.rec_s;
+    view->sd = W.sd;
+    view->bits = W.bits;
+    view->wpre = W.wpre;
+  }
+  return done;
 }
 
 }  // namespace
+
+ptc_status stack_distance_view(const uint32_t* prev, uint64_t n, uint32_t* dist_out, int method, void* ws,
+                               size_t ws_bytes, cudaStream_t s, RunsView* view) {
+  *view = RunsView{};
+  if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
+  if (n == 0) return PTC_OK;
+  if (!prev || !dist_out) return PTC_ERR_INVALID_ARG;
+  if (method == PTC_SD_POINTS) return stack_distance_points(prev, n, dist_out, ws, ws_bytes, s);
+  return stack_distance_runs(prev, n, dist_out, ws, ws_bytes, s, method, view);
+}
+
 }  // namespace ptc
 
 using namespace ptc;
@@ -785,7 +805,7 @@ extern "C" ptc_status ptc_stack_distance_ex(const uint32_t* prev, uint64_t n, ui
   if (!prev || !dist_out) return PTC_ERR_INVALID_ARG;
   cudaStream_t s = (cudaStream_t)stream;
   if (method == PTC_SD_POINTS) return stack_distance_points(prev, n, dist_out, ws, ws_bytes, s);
-  return stack_distance_runs(prev, n, dist_out, ws, ws_bytes, s, method);
+  return stack_distance_runs(prev, n, dist_out, ws, ws_bytes, s, method, nullptr);
 }
 
 extern "C" ptc_status ptc_stack_distance(const uint32_t* prev, uint64_t n, uint32_t* dist_out, void* ws,
