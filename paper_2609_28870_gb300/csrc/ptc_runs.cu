@@ -402,7 +402,6 @@ struct BuildArgs {
 __global__ void __launch_bounds__(kCT) k_runs_build_cluster(BuildArgs a) {
   extern __shared__ uint2 s_dyn[];  // two buffers of `slice` (key, weight)
   __shared__ unsigned long long s_rw[kCPer * 32];  // per (round, warp) (zeros, zero weight)
-  __shared__ unsigned long long s_warp[kCT / 32];
   __shared__ unsigned long long s_tot, s_pre, s_all;
   cg::cluster_group cl = cg::this_cluster();
   const uint32_t rank = cl.block_rank(), C = cl.num_blocks();
@@ -444,29 +443,36 @@ __global__ void __launch_bounds__(kCT) k_runs_build_cluster(BuildArgs a) {
       if (lane == 31 && k < (int)q) s_rw[k * 32 + w] = pack_zw(__popc(m), wi);
     }
     __syncthreads();
-    // exclusive scan of the (round, warp) totals in index order
-    {
-      const uint32_t t = threadIdx.x;
-      const unsigned long long x = t < q * 32 ? s_rw[t] : 0ull;
-      unsigned long long incl = x;
+    // exclusive scan of the q x 32 (round, warp) totals in index order, by
+    // warp 0: lane l sums the q consecutive entries [l q, l q + q)
+    if (w == 0) {
+      unsigned long long part[kCPer];
+      unsigned long long sum = 0;
+#pragma unroll
+      for (int k = 0; k < kCPer; ++k) {
+        part[k] = 0;
+        if (k < (int)q) {
+          part[k] = s_rw[lane * q + k];
+          sum += part[k];
+        }
+      }
+      unsigned long long incl = sum;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const unsigned long long y = __shfl_up_sync(kFull, incl, o);
         if (lane >= (uint32_t)o) incl += y;
       }
-      if (lane == 31) s_warp[w] = incl;
-      __syncthreads();
-      unsigned long long pre = 0, tot = 0;
+      unsigned long long run = incl - sum;
 #pragma unroll
-      for (int ww = 0; ww < kCT / 32; ++ww) {
-        const unsigned long long v = s_warp[ww];
-        if (ww < (int)w) pre += v;
-        tot += v;
+      for (int k = 0; k < kCPer; ++k) {
+        if (k < (int)q) {
+          s_rw[lane * q + k] = run;
+          run += part[k];
+        }
       }
-      if (t < q * 32) s_rw[t] = pre + incl - x;
-      if (t == 0) s_tot = tot;
-      __syncthreads();
+      if (lane == 31) s_tot = incl;
     }
+    __syncthreads();
     const uint32_t nz = (uint32_t)s_tot;
     // local stable partition into `cur` (every element is in registers)
 #pragma unroll
