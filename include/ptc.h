@@ -251,7 +251,8 @@ ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_
  *   cap_host, n_cap, cm, hits/saved/total outputs  as for ptc_curves
  *   n_access_host_out, n_distinct_host_out        N and D on the host
  * The workspace holds the intermediate arrays not supplied plus the largest
- * scratch of any stage (ptc_pipeline_workspace_bytes).
+ * scratch of any stage (ptc_pipeline_workspace_bytes).  Stages b and c do not
+ * wait for their own status; an error they raise is returned with stage d's.
  */
 size_t ptc_pipeline_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size, uint32_t n_cap);
 ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off, const int64_t* req_ts_us,

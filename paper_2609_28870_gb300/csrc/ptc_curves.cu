@@ -508,6 +508,11 @@ __global__ void __launch_bounds__(256) k_curves_runs(CurveArgs a, RunsArgs ra) {
   }
 }
 
+// Earlier calls' error words (deferred, see defer_status) join this call's.
+__global__ void k_carry_err(const uint32_t* err, uint32_t n, DevStatus* st) {
+  if (threadIdx.x < n && err[threadIdx.x]) atomicOr(&st->err, err[threadIdx.x]);
+}
+
 struct U128 {
   uint64_t lo, hi;
 };
@@ -610,7 +615,8 @@ extern "C" size_t ptc_curves_workspace_bytes(uint64_t n, uint32_t n_req, uint32_
 ptc_status ptc::curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,
                             uint32_t block_size, const ptc_cost_model* cm, const uint64_t* cap_host, uint32_t n_cap,
                             uint64_t* hits_host_out, ptc_u128* saved_host_out, ptc_u128* total_cost_host_out,
-                            void* ws, size_t ws_bytes, cudaStream_t stream, const RunsView* runs) {
+                            void* ws, size_t ws_bytes, cudaStream_t stream, const RunsView* runs,
+                            const uint32_t* carry_err, uint32_t n_carry) {
   if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
   if (!cm || !cap_host || !hits_host_out || !saved_host_out || !total_cost_host_out) return PTC_ERR_INVALID_ARG;
   if (n_cap < 1 || n_cap > PTC_MAX_CAPACITIES) return PTC_ERR_INVALID_ARG;
@@ -637,6 +643,7 @@ ptc_status ptc::curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* re
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
   if (cudaMemcpyAsync(L.caps, cap_host, sizeof(uint64_t) * n_cap, cudaMemcpyHostToDevice, s) != cudaSuccess)
     return PTC_ERR_CUDA;
+  if (n_carry) PTC_LAUNCH("k_carry_err", s, k_carry_err<<<1, 32, 0, s>>>(carry_err, n_carry, L.st));
   if (n > 0) {
     PTC_LAUNCH("k_heads", s,
                k_heads<<<ceil_div_u32(n_req, 256), 256, 0, s>>>(req_blk_off, n_req, n, L.bitmap, L.tile_req, L.st));

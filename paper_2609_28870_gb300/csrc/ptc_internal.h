@@ -45,6 +45,15 @@ inline ptc_status end_call(const DevStatus* dev, cudaStream_t stream, DevStatus*
   return PTC_OK;
 }
 
+// Instead of waiting for a call's status, queue a copy of its error word to
+// `slot`, for a later call that does wait to fold in (ptc_pipeline).
+inline ptc_status defer_status(const DevStatus* dev, uint32_t* slot, cudaStream_t stream) {
+  if (cudaGetLastError() != cudaSuccess) return PTC_ERR_CUDA;
+  if (cudaMemcpyAsync(slot, &dev->err, sizeof(uint32_t), cudaMemcpyDeviceToDevice, stream) != cudaSuccess)
+    return PTC_ERR_CUDA;
+  return PTC_OK;
+}
+
 // Streaming multiprocessors of the current device (persistent grids).
 inline int num_sms() {
   int dev = 0, n = 0;
@@ -68,13 +77,18 @@ struct RunsView {
   const uint32_t* wpre = nullptr;   // runs starting before each word
 };
 ptc_status stack_distance_view(const uint32_t* prev, uint64_t n, uint32_t* dist_out, int method, void* ws,
-                               size_t ws_bytes, cudaStream_t s, RunsView* view);
+                               size_t ws_bytes, cudaStream_t s, RunsView* view, uint32_t* defer_err);
+// Stage b as ptc_reuse_indices does it (ptc_reuse.cu); with `defer_err` the
+// final wait is replaced by defer_status.
+ptc_status reuse_view(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev_out, uint32_t* next_out,
+                      void* ws, size_t ws_bytes, cudaStream_t s, uint32_t* defer_err);
 // Stage d (ptc_curves.cu); with `runs` (from stack_distance_view) the curves
 // come from the runs instead of a pass over every distance.
 ptc_status curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,
                        uint32_t block_size, const ptc_cost_model* cm, const uint64_t* cap_host, uint32_t n_cap,
                        uint64_t* hits_host_out, ptc_u128* saved_host_out, ptc_u128* total_cost_host_out, void* ws,
-                       size_t ws_bytes, cudaStream_t s, const RunsView* runs);
+                       size_t ws_bytes, cudaStream_t s, const RunsView* runs, const uint32_t* carry_err = nullptr,
+                       uint32_t n_carry = 0);
 
 // Stage c on the matrix over every access (ptc_wavelet.cu); the C entry
 // points in ptc_runs.cu choose between it and the matrix over runs.

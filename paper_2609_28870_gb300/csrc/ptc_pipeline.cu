@@ -17,6 +17,7 @@ struct PipeLayout {
   size_t scratch_bytes;
   void* curves;
   size_t curves_bytes;
+  uint32_t* defer;  // error words of stages b and c, read with stage d's
   size_t total;
 };
 
@@ -44,6 +45,7 @@ PipeLayout pipe_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   L.scratch = cv.take<unsigned char>(L.scratch_bytes);
   L.curves_bytes = ptc_curves_workspace_bytes(n_tok / B, n_req, n_cap);
   L.curves = cv.take<unsigned char>(L.curves_bytes);
+  L.defer = cv.take<uint32_t>(2);
   L.total = cv.bytes();
   return L;
 }
@@ -86,15 +88,16 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
   rc = ptc_assign_ids(keys, n, ids, &d, L.scratch, L.scratch_bytes, stream);
   *n_distinct_host_out = d;
   if (rc != PTC_OK) return rc;
-  if (n > 0) {
-    rc = ptc_reuse_indices(ids, n, d, prev, next, L.scratch, L.scratch_bytes, stream);
-    if (rc != PTC_OK) return rc;
-  }
+  // stages b and c do not wait for their own status: stage d reads it
+  cudaStream_t s = (cudaStream_t)stream;
+  if (cudaMemsetAsync(L.defer, 0, 2 * sizeof(uint32_t), s) != cudaSuccess) return PTC_ERR_CUDA;
   ptc::RunsView runs;
   if (n > 0) {
-    rc = ptc::stack_distance_view(prev, n, dist, PTC_SD_AUTO, L.scratch, L.scratch_bytes, (cudaStream_t)stream, &runs);
+    rc = ptc::reuse_view(ids, n, d, prev, next, L.scratch, L.scratch_bytes, s, &L.defer[0]);
+    if (rc != PTC_OK) return rc;
+    rc = ptc::stack_distance_view(prev, n, dist, PTC_SD_AUTO, L.scratch, L.scratch_bytes, s, &runs, &L.defer[1]);
     if (rc != PTC_OK) return rc;
   }
   return ptc::curves_impl(dist, n, blk, n_req, block_size, cm, cap_host, n_cap, hits_host_out, saved_host_out,
-                          total_cost_host_out, L.curves, L.curves_bytes, (cudaStream_t)stream, &runs);
+                          total_cost_host_out, L.curves, L.curves_bytes, s, &runs, L.defer, 2);
 }

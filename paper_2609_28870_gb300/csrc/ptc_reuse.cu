@@ -389,7 +389,7 @@ uint32_t bits_for(uint64_t v) {  // bits to hold values below v
 }
 
 ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* prev_out, uint32_t* next_out, void* ws,
-                         size_t ws_bytes, cudaStream_t s, bool forced) {
+                         size_t ws_bytes, cudaStream_t s, bool forced, uint32_t* defer_err = nullptr) {
   const ReuseLayout L = reuse_layout(ws, n, D, forced);
   if (!ws_ok(ws, ws_bytes, L.total)) return PTC_ERR_WORKSPACE;
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
@@ -450,10 +450,20 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
   const uint32_t fill_blocks = ceil_div_u32(K, 8) < (uint32_t)(16 * num_sms()) ? ceil_div_u32(K, 8)
                                                                                 : (uint32_t)(16 * num_sms());
   PTC_LAUNCH("k_ir_fill", s, k_ir_fill<<<fill_blocks, 256, 0, s>>>(f));
+  if (defer_err) return defer_status(L.st, defer_err, s);
   return end_call(L.st, s, &h);
 }
 
 }  // namespace
+
+ptc_status reuse_view(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev_out, uint32_t* next_out,
+                      void* ws, size_t ws_bytes, cudaStream_t s, uint32_t* defer_err) {
+  if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
+  if (n == 0) return PTC_OK;
+  if (!ids || !prev_out || !next_out || n_distinct == 0 || n_distinct > n) return PTC_ERR_INVALID_ARG;
+  return reuse_by_runs(ids, n, n_distinct, prev_out, next_out, ws, ws_bytes, s, false, defer_err);
+}
+
 }  // namespace ptc
 
 using namespace ptc;

@@ -655,7 +655,7 @@ uint64_t runs_reserve(uint64_t n) {
 }
 
 ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_out, void* ws, size_t ws_bytes,
-                               cudaStream_t s, int method, RunsView* view) {
+                               cudaStream_t s, int method, RunsView* view, uint32_t* defer_err = nullptr) {
   const RunsLayout M = runs_layout(ws, n, 1);
   if (!ws_ok(ws, ws_bytes, M.total)) return PTC_ERR_WORKSPACE;
   if (begin_call(ws, M.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
@@ -763,7 +763,7 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   PTC_LAUNCH("k_runs_query", s, k_runs_query<<<ceil_div_u32(R, 256), 256, 0, s>>>(q));
   PTC_LAUNCH("k_runs_expand", s,
              k_runs_expand<<<ceil_div_u32(n, 256), 256, 0, s>>>(W.bits, W.wpre, W.sd, (uint32_t)n, dist_out));
-  const ptc_status done = end_call(W.st, s, &h);
+  const ptc_status done = defer_err ? defer_status(W.st, defer_err, s) : end_call(W.st, s, &h);
   if (done == PTC_OK && view) {
     view->used = true;
     view->R = R32;
@@ -778,13 +778,13 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
 }  // namespace
 
 ptc_status stack_distance_view(const uint32_t* prev, uint64_t n, uint32_t* dist_out, int method, void* ws,
-                               size_t ws_bytes, cudaStream_t s, RunsView* view) {
+                               size_t ws_bytes, cudaStream_t s, RunsView* view, uint32_t* defer_err) {
   *view = RunsView{};
   if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
   if (n == 0) return PTC_OK;
   if (!prev || !dist_out) return PTC_ERR_INVALID_ARG;
   if (method == PTC_SD_POINTS) return stack_distance_points(prev, n, dist_out, ws, ws_bytes, s);
-  return stack_distance_runs(prev, n, dist_out, ws, ws_bytes, s, method, view);
+  return stack_distance_runs(prev, n, dist_out, ws, ws_bytes, s, method, view, defer_err);
 }
 
 }  // namespace ptc
