@@ -161,6 +161,7 @@ __device__ __forceinline__ uint64_t pow_at(const uint64_t* __restrict__ lo, cons
 // ---------------------------------------------------------------- hash
 struct HashConsts {
   uint32_t limb[2][3][16];   // 21-bit limbs of u_b^(j + 1)
+  uint32_t limb2[2][2][16];  // the same split 31 + 30 bits (tokens below 2^27)
   uint64_t csum[2][17];      // sum_{j < n} u_b^(j + 1): the "+ 1" of n tokens
   uint64_t sub_mul[2][32];   // u_b^(16 q)
 };
@@ -218,6 +219,25 @@ __device__ __forceinline__ void hash16(const uint32_t (&wd)[20], const HashConst
     acc[4] = mad_wide(t, c.limb[1][1][j], acc[4]);
     acc[5] = mad_wide(t, c.limb[1][2][j], acc[5]);
   }
+}
+
+// The same sum with two limbs (31 + 30 bits), exact when every token is
+// below 2^27: 16 products of at most 2^58 stay below 2^62.
+template <int M>
+__device__ __forceinline__ void hash16_2(const uint32_t (&wd)[20], const HashConsts& c, uint64_t (&acc)[4]) {
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const uint32_t t = wd[j + M];
+    acc[0] = mad_wide(t, c.limb2[0][0][j], acc[0]);
+    acc[1] = mad_wide(t, c.limb2[0][1][j], acc[1]);
+    acc[2] = mad_wide(t, c.limb2[1][0][j], acc[2]);
+    acc[3] = mad_wide(t, c.limb2[1][1][j], acc[3]);
+  }
+}
+
+// (a0 + a1 2^31) mod p for a0, a1 < 2^62: a1 2^31 = (a1 mod 2^30) 2^31 + (a1 >> 30) 2^61
+__device__ __forceinline__ uint64_t limbs2_to_p61(uint64_t a0, uint64_t a1) {
+  return p61_fold(p61_fold(a0) + ((a1 & ((1ULL << 30) - 1)) << 31) + (a1 >> 30));
 }
 
 // (a0 + a1 2^21 + a2 2^42) mod p for a0, a1, a2 < 2^62 - 2^57 (sums of <= 32 products < 2^53)
@@ -506,7 +526,7 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local_vec(HashArgs a, con
 // global offsets instead.
 constexpr int kH16Req = 256;
 
-__global__ void __launch_bounds__(kHashThreads, 4) k_hash16(HashArgs a, const __grid_constant__ HashConsts c) {
+__global__ void __launch_bounds__(kHashThreads, 3) k_hash16(HashArgs a, const __grid_constant__ HashConsts c) {
   __shared__ uint64_t s_boff[kH16Req + 1];
   __shared__ uint64_t s_toff[kH16Req + 1];
   constexpr uint32_t TB = kHashThreads;
@@ -533,6 +553,7 @@ __global__ void __launch_bounds__(kHashThreads, 4) k_hash16(HashArgs a, const __
   uint64_t h0 = 0, h1 = 0;
   uint32_t k = 0;
   uint64_t wd_x = 0;  // token offset of this thread's block
+  uint64_t rstart = 0;  // first block of its request
   if (b < b_end) {
     uint64_t x;
     if (cached) {  // largest i with s_boff[i] <= b
@@ -544,11 +565,13 @@ __global__ void __launch_bounds__(kHashThreads, 4) k_hash16(HashArgs a, const __
         else
           hi = mid - 1;
       }
-      k = (uint32_t)(b - s_boff[lo]);
+      rstart = s_boff[lo];
+      k = (uint32_t)(b - rstart);
       x = s_toff[lo] + 16ULL * k;
     } else {
       const uint32_t r = find_request(a.blk_off, r_first, r_last, b);
-      k = (uint32_t)(b - a.blk_off[r]);
+      rstart = a.blk_off[r];
+      k = (uint32_t)(b - rstart);
       x = a.tok_off[r] + 16ULL * k;
     }
     wd_x = x;
@@ -600,17 +623,123 @@ __global__ void __launch_bounds__(kHashThreads, 4) k_hash16(HashArgs a, const __
     }
   }
   if (live) {
-    uint64_t acc[6] = {0, 0, 0, 0, 0, 0};
-    switch (m) {
-      case 0: hash16<0>(wd, c, acc); break;
-      case 1: hash16<1>(wd, c, acc); break;
-      case 2: hash16<2>(wd, c, acc); break;
-      default: hash16<3>(wd, c, acc); break;
+    uint32_t any = 0;  // bits of the block's tokens above 2^27
+#pragma unroll
+    for (int j = 0; j < 19; ++j) any |= wd[j];
+    if ((any >> 27) == 0) {  // every token fits two limbs (words outside the block only widen the test)
+      uint64_t acc[4] = {0, 0, 0, 0};
+      switch (m) {
+        case 0: hash16_2<0>(wd, c, acc); break;
+        case 1: hash16_2<1>(wd, c, acc); break;
+        case 2: hash16_2<2>(wd, c, acc); break;
+        default: hash16_2<3>(wd, c, acc); break;
+      }
+      h0 = p61_add(limbs2_to_p61(acc[0], acc[1]), c.csum[0][16]);
+      h1 = p61_add(limbs2_to_p61(acc[2], acc[3]), c.csum[1][16]);
+    } else {
+      uint64_t acc[6] = {0, 0, 0, 0, 0, 0};
+      switch (m) {
+        case 0: hash16<0>(wd, c, acc); break;
+        case 1: hash16<1>(wd, c, acc); break;
+        case 2: hash16<2>(wd, c, acc); break;
+        default: hash16<3>(wd, c, acc); break;
+      }
+      h0 = p61_add(limbs_to_p61(acc[0], acc[1], acc[2]), c.csum[0][16]);
+      h1 = p61_add(limbs_to_p61(acc[3], acc[4], acc[5]), c.csum[1][16]);
     }
-    h0 = p61_add(limbs_to_p61(acc[0], acc[1], acc[2]), c.csum[0][16]);
-    h1 = p61_add(limbs_to_p61(acc[3], acc[4], acc[5]), c.csum[1][16]);
   }
-  hash_finish<1>(a, tile, b0, b_end, h0, h1, k, t, 0);
+  // g = h u^(16 k), then a plain prefix sum over the tile; a block whose
+  // request starts inside the tile at index s subtracts the prefix before s.
+  const uint64_t* T = a.tables;
+  uint64_t v0 = 0, v1 = 0;
+  if (live) {
+    v0 = p61_mul(h0, pow_at(T + 0 * 65536, T + 1 * 65536, k));
+    v1 = p61_mul(h1, pow_at(T + 2 * 65536, T + 3 * 65536, k));
+  }
+  __shared__ uint64_t s_p0[kHashThreads], s_p1[kHashThreads];
+  __shared__ uint64_t s_w0[kHashThreads / 32], s_w1[kHashThreads / 32];
+  const uint32_t lane = t & 31, w = t >> 5;
+  // warp scan with lazy reduction: three plain steps keep sums of at most 8
+  // values below 2^64, then each step folds back below 2^62
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const uint64_t y0 = __shfl_up_sync(kFull, v0, d), y1 = __shfl_up_sync(kFull, v1, d);
+    if (lane >= (uint32_t)d) {
+      v0 += y0;
+      v1 += y1;
+    }
+    if (d >= 4) {
+      v0 = (v0 & kP61) + (v0 >> 61);
+      v1 = (v1 & kP61) + (v1 >> 61);
+    }
+  }
+  if (lane == 31) {
+    s_w0[w] = v0;
+    s_w1[w] = v1;
+  }
+  __syncthreads();
+  if (w == 0) {  // exclusive prefix of the warp totals
+    uint64_t z0 = lane < kHashThreads / 32 ? s_w0[lane] : 0, z1 = lane < kHashThreads / 32 ? s_w1[lane] : 0;
+    const uint64_t x0 = z0, x1 = z1;
+#pragma unroll
+    for (int d = 1; d < kHashThreads / 32; d <<= 1) {
+      const uint64_t y0 = __shfl_up_sync(kFull, z0, d), y1 = __shfl_up_sync(kFull, z1, d);
+      if (lane >= (uint32_t)d) {
+        z0 += y0;
+        z1 += y1;
+      }
+      z0 = (z0 & kP61) + (z0 >> 61);
+      z1 = (z1 & kP61) + (z1 >> 61);
+    }
+    if (lane < kHashThreads / 32) {
+      s_w0[lane] = p61_fold(z0 + (kP61 << 1) - x0);  // z, x < 2^62: stays positive
+      s_w1[lane] = p61_fold(z1 + (kP61 << 1) - x1);
+    }
+  }
+  __syncthreads();
+  v0 = p61_fold(v0 + s_w0[w]);
+  v1 = p61_fold(v1 + s_w1[w]);
+  s_p0[t] = v0;
+  s_p1[t] = v1;
+  __syncthreads();
+  if (live) {
+    const bool own_start = rstart >= b0;  // the request starts in this tile
+    if (own_start && rstart > b0) {
+      const uint32_t sl = (uint32_t)(rstart - b0) - 1;
+      v0 = p61_add(v0, kP61 - s_p0[sl]);
+      v1 = p61_add(v1, kP61 - s_p1[sl]);
+    }
+    a.keys[b] = make_ulonglong2(v0, v1);
+  }
+  // the tile's aggregate for k_hash_chain: the last block's sum since its
+  // request's start, and whether that start is in the tile; and the leading
+  // blocks (before the tile's first request start)
+  if (b + 1 == b_end) {
+    HashCarry agg;
+    agg.f = rstart >= b0;
+    agg.v0 = v0;
+    agg.v1 = v1;
+    a.tile_agg[tile] = agg;
+  }
+  if (t == 0) {
+    uint32_t lead = (uint32_t)(b_end - b0);
+    if (cached) {
+      for (uint32_t i = 0; i < nreq; ++i)
+        if (s_boff[i] >= b0 && s_boff[i] < b_end && s_boff[i + 1] > s_boff[i]) {
+          lead = (uint32_t)(s_boff[i] - b0);
+          break;
+        }
+    } else {
+      for (uint32_t r = r_first; r <= r_last; ++r) {
+        const uint64_t st0 = a.blk_off[r];
+        if (st0 >= b0 && st0 < b_end && a.blk_off[r + 1] > st0) {
+          lead = (uint32_t)(st0 - b0);
+          break;
+        }
+      }
+    }
+    a.tile_lead[tile] = lead;
+  }
 }
 
 // Carry of every tile = the segmented sum of the aggregates of the tiles
@@ -754,6 +883,8 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
       hc.limb[b][0][j] = (uint32_t)(v & 0x1FFFFF);
       hc.limb[b][1][j] = (uint32_t)((v >> 21) & 0x1FFFFF);
       hc.limb[b][2][j] = (uint32_t)(v >> 42);
+      hc.limb2[b][0][j] = (uint32_t)(v & 0x7FFFFFFF);
+      hc.limb2[b][1][j] = (uint32_t)(v >> 31);
       sum = p61_add(sum, v);
       hc.csum[b][j + 1] = sum;
     }

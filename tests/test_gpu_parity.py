@@ -269,3 +269,23 @@ def test_long_runs_and_run_breaks():
         ids, D = oracle.block_ids(tr.tokens, tr.req_tok_off, B)
         caps = tracegen.capacity_grid(1, D + 1, 40)
         gu.assert_same(gu.gpu_run(tr, B, caps), gu.oracle_run(tr, B, caps))
+
+
+@pytest.mark.parametrize("vocab", [2**32 - 1, 2**27 + 5])
+def test_full_range_token_values(vocab):
+    """Tokens up to 2^32 - 1 at B = 16 with 16-byte-aligned tokens: blocks
+    whose tokens all fit 27 bits and blocks that need the three-limb
+    products sit in the same warps; keys, ids and curves bit-exact."""
+    rng = np.random.default_rng(vocab & 0xFFFF)
+    reqs = []
+    for s in range(40):
+        base = [int(x) for x in rng.integers(0, vocab if s % 3 else 151936, size=int(rng.integers(16, 400)))]
+        reqs.append(base)
+        reqs.append(base + [int(x) for x in rng.integers(0, vocab, size=int(rng.integers(0, 200)))])
+    tr = tracegen.from_lists(reqs)
+    gu = _g()
+    _, D = oracle.block_ids(tr.tokens, tr.req_tok_off, 16)
+    caps = list(range(1, D + 2, max(1, D // 40)))
+    g = gu.gpu_run(tr, 16, caps, seed=77)
+    gu.assert_same(g, gu.oracle_run(tr, 16, caps))
+    assert np.array_equal(g["keys"], oracle.prefix_hash(tr.tokens, tr.req_tok_off, 16, 77))
