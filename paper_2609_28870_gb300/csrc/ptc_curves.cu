@@ -39,6 +39,7 @@ constexpr int kCvTile = kCvThreads * kCvPer;
 // first access (each tile has exactly one such request).
 __global__ void k_heads(const uint64_t* __restrict__ blk_off, uint32_t R, uint64_t n, uint32_t* __restrict__ bitmap,
                         uint32_t* __restrict__ tile_req, DevStatus* st) {
+  grid_dep_sync();
   const uint64_t r = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= R) return;
   const uint64_t a = blk_off[r], b = blk_off[r + 1];
@@ -160,6 +161,7 @@ __global__ void __launch_bounds__(kCvThreads) k_curves_agg(const uint32_t* __res
                                                            RunMax* __restrict__ tile_agg, const uint32_t* slow,
                                                            unsigned long long* cnt, unsigned long long* ksum,
                                                            uint32_t G) {
+  grid_dep_sync();
   __shared__ RunMax s_w[kCvThreads / 32];
   if (!*slow) return;  // k_curves_fast's bins stand
   if (blockIdx.x == 0)  // the scan path starts the bins afresh
@@ -177,6 +179,7 @@ __global__ void __launch_bounds__(kCvThreads) k_curves_agg(const uint32_t* __res
 // and keeps its bin histograms in shared memory across them, so the global
 // bins see one atomic per CTA and bin rather than per tile.
 __global__ void __launch_bounds__(kCvThreads) k_curves(CurveArgs a) {
+  grid_dep_sync();
   if (!*a.slow) return;
   __shared__ uint32_t s_cap[PTC_MAX_CAPACITIES];
   __shared__ uint32_t s_cnt[PTC_MAX_CAPACITIES + 1];
@@ -321,6 +324,7 @@ __device__ __forceinline__ uint32_t bin_of(const uint32_t* s_cap, uint32_t G, ui
 constexpr int kFtReq = 128;  // requests a tile's table holds
 
 __global__ void __launch_bounds__(kCvThreads) k_curves_fast(CurveArgs a) {
+  grid_dep_sync();
   __shared__ uint32_t s_cap[PTC_MAX_CAPACITIES];
   __shared__ uint32_t s_cnt[PTC_MAX_CAPACITIES + 1];
   __shared__ unsigned long long s_ks[PTC_MAX_CAPACITIES + 1];
@@ -468,6 +472,7 @@ struct RunsArgs {
 };
 
 __global__ void __launch_bounds__(256) k_curves_runs(CurveArgs a, RunsArgs ra) {
+  grid_dep_sync();
   __shared__ uint32_t s_cap[PTC_MAX_CAPACITIES];
   __shared__ uint32_t s_cnt[PTC_MAX_CAPACITIES + 1];
   __shared__ unsigned long long s_ks[PTC_MAX_CAPACITIES + 1];
@@ -510,6 +515,7 @@ __global__ void __launch_bounds__(256) k_curves_runs(CurveArgs a, RunsArgs ra) {
 
 // Earlier calls' error words (deferred, see defer_status) join this call's.
 __global__ void k_carry_err(const uint32_t* err, uint32_t n, DevStatus* st) {
+  grid_dep_sync();
   if (threadIdx.x < n && err[threadIdx.x]) atomicOr(&st->err, err[threadIdx.x]);
 }
 
@@ -529,6 +535,7 @@ __device__ __forceinline__ U128 add_u128(U128 a, U128 b) {
 __global__ void __launch_bounds__(1024) k_finalize(const unsigned long long* __restrict__ cnt,
                                                    const unsigned long long* __restrict__ ksum, uint32_t G,
                                                    uint64_t alpha, uint64_t beta, uint64_t* __restrict__ out) {
+  grid_dep_sync();
   __shared__ unsigned long long s_h[32], s_k[32];
   const uint32_t t = threadIdx.x, lane = t & 31, w = t >> 5;
   unsigned long long h = t < G ? cnt[t] : 0ull, k = t < G ? ksum[t] : 0ull;
@@ -643,10 +650,9 @@ ptc_status ptc::curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* re
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
   if (cudaMemcpyAsync(L.caps, cap_host, sizeof(uint64_t) * n_cap, cudaMemcpyHostToDevice, s) != cudaSuccess)
     return PTC_ERR_CUDA;
-  if (n_carry) PTC_LAUNCH("k_carry_err", s, k_carry_err<<<1, 32, 0, s>>>(carry_err, n_carry, L.st));
+  if (n_carry) PTC_KERNEL("k_carry_err", s, k_carry_err, 1, 32, 0, carry_err, n_carry, L.st);
   if (n > 0) {
-    PTC_LAUNCH("k_heads", s,
-               k_heads<<<ceil_div_u32(n_req, 256), 256, 0, s>>>(req_blk_off, n_req, n, L.bitmap, L.tile_req, L.st));
+    PTC_KERNEL("k_heads", s, k_heads, ceil_div_u32(n_req, 256), 256, 0, req_blk_off, n_req, n, L.bitmap, L.tile_req, L.st);
     CurveArgs a;
     a.dist = dist;
     a.n = (uint32_t)n;
@@ -665,20 +671,18 @@ ptc_status ptc::curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* re
       const RunsArgs ra{runs->rec_s, runs->sd, runs->bits, runs->wpre};
       const uint32_t g_r = ceil_div_u32(n_req, 256) < (uint32_t)(2 * num_sms()) ? ceil_div_u32(n_req, 256)
                                                                                   : (uint32_t)(2 * num_sms());
-      PTC_LAUNCH("k_curves_runs", s, k_curves_runs<<<g_r, 256, 0, s>>>(a, ra));
+      PTC_KERNEL("k_curves_runs", s, k_curves_runs, g_r, 256, 0, a, ra);
     } else {
       const uint32_t tiles0 = ceil_div_u32(n, kCvTile);
       const uint32_t grid0 = tiles0 < (uint32_t)(3 * num_sms()) ? tiles0 : (uint32_t)(3 * num_sms());
-      PTC_LAUNCH("k_curves_fast", s, k_curves_fast<<<grid0, kCvThreads, 0, s>>>(a));
+      PTC_KERNEL("k_curves_fast", s, k_curves_fast, grid0, kCvThreads, 0, a);
     }
-    PTC_LAUNCH("k_curves_agg", s,
-               k_curves_agg<<<ceil_div_u32(n, kCvTile), kCvThreads, 0, s>>>(dist, (uint32_t)n, L.bitmap, L.lb_agg,
-                                                                          L.slow, L.cnt, L.ksum, n_cap));
+    PTC_KERNEL("k_curves_agg", s, k_curves_agg, ceil_div_u32(n, kCvTile), kCvThreads, 0, dist, (uint32_t)n, L.bitmap, L.lb_agg, L.slow, L.cnt, L.ksum, n_cap);
     const uint32_t tiles = ceil_div_u32(n, kCvTile);
     const uint32_t grid = tiles < (uint32_t)(3 * num_sms()) ? tiles : (uint32_t)(3 * num_sms());
-    PTC_LAUNCH("k_curves", s, k_curves<<<grid, kCvThreads, 0, s>>>(a));
+    PTC_KERNEL("k_curves", s, k_curves, grid, kCvThreads, 0, a);
   }
-  PTC_LAUNCH("k_finalize", s, k_finalize<<<1, 1024, 0, s>>>(L.cnt, L.ksum, n_cap, alpha, beta, L.out));
+  PTC_KERNEL("k_finalize", s, k_finalize, 1, 1024, 0, L.cnt, L.ksum, n_cap, alpha, beta, L.out);
   static thread_local uint64_t host_out[3 * PTC_MAX_CAPACITIES + 2];
   if (cudaMemcpyAsync(host_out, L.out, sizeof(uint64_t) * (3 * n_cap + 2), cudaMemcpyDeviceToHost, s) != cudaSuccess)
     return PTC_ERR_CUDA;

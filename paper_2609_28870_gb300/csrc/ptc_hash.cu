@@ -77,6 +77,7 @@ __global__ void __launch_bounds__(kOffThreads) k_block_offsets(const uint64_t* _
                                                                uint64_t* __restrict__ blk_off,
                                                                uint32_t* __restrict__ tile_req, uint64_t tile_cap,
                                                                uint64_t* lb, DevStatus* st) {
+  grid_dep_sync();
   const uint32_t tile = next_tile(st, kEpochOffsets);
   const uint64_t r0 = (uint64_t)tile * kOffTile + (uint64_t)threadIdx.x * kOffPer;
   uint64_t cnt[kOffPer];
@@ -134,6 +135,7 @@ struct PowBases {
 // Only the entries some block can use are filled: exponents e = k reach at
 // most the longest request's block count minus one (st->value[1]).
 __global__ void k_pow_tables(PowBases pb, uint64_t* __restrict__ tables, const DevStatus* st) {
+  grid_dep_sync();
   const uint32_t gid = blockIdx.x * blockDim.x + threadIdx.x;  // 4 tables x 1024 chunks of 64
   const uint32_t t = gid >> 10, chunk = gid & 1023;
   if (t >= 4) return;
@@ -340,6 +342,7 @@ __device__ __forceinline__ void hash_finish(const HashArgs& a, uint32_t tile, ui
 
 template <int G, bool FULL>
 __global__ void __launch_bounds__(kHashThreads) k_hash_local(HashArgs a, const __grid_constant__ HashConsts c) {
+  grid_dep_sync();
   __shared__ uint32_t s_tok[kWinWords];
   __shared__ uint64_t s_bnd[4];
   constexpr uint32_t TB = kHashThreads / G;
@@ -456,6 +459,7 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local(HashArgs a, const _
 // request.  No shared-memory staging.
 template <int G>
 __global__ void __launch_bounds__(kHashThreads) k_hash_local_vec(HashArgs a, const __grid_constant__ HashConsts c) {
+  grid_dep_sync();
   __shared__ uint32_t s_bnd[2];
   constexpr uint32_t TB = kHashThreads / G;
   const uint32_t tile = blockIdx.x;
@@ -527,6 +531,7 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local_vec(HashArgs a, con
 constexpr int kH16Req = 256;
 
 __global__ void __launch_bounds__(kHashThreads, 3) k_hash16(HashArgs a, const __grid_constant__ HashConsts c) {
+  grid_dep_sync();
   __shared__ uint64_t s_boff[kH16Req + 1];
   __shared__ uint64_t s_toff[kH16Req + 1];
   constexpr uint32_t TB = kHashThreads;
@@ -752,6 +757,7 @@ __global__ void __launch_bounds__(kChainWarps * 32) k_hash_chain(ulonglong2* __r
                                                                  const HashCarry* __restrict__ tile_agg,
                                                                  const uint32_t* __restrict__ tile_lead, uint32_t TB,
                                                                  const DevStatus* st, uint64_t keys_cap) {
+  grid_dep_sync();
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t tile = blockIdx.x * kChainWarps + (threadIdx.x >> 5);
   uint64_t N = st->value[0];
@@ -786,13 +792,13 @@ __global__ void __launch_bounds__(kChainWarps * 32) k_hash_chain(ulonglong2* __r
 template <int G>
 void launch_hash(uint32_t grid, cudaStream_t s, const HashArgs& a, const HashConsts& c, bool full) {
   if (G == 1 && full && a.aligned)
-    PTC_LAUNCH("k_hash16", s, k_hash16<<<grid, kHashThreads, 0, s>>>(a, c));
+    PTC_KERNEL("k_hash16", s, k_hash16, grid, kHashThreads, 0, a, c);
   else if (full && a.aligned)
-    PTC_LAUNCH("k_hash_local", s, k_hash_local_vec<G><<<grid, kHashThreads, 0, s>>>(a, c));
+    PTC_KERNEL("k_hash_local", s, k_hash_local_vec<G>, grid, kHashThreads, 0, a, c);
   else if (full)
-    PTC_LAUNCH("k_hash_local", s, k_hash_local<G, true><<<grid, kHashThreads, 0, s>>>(a, c));
+    PTC_KERNEL("k_hash_local", s, (k_hash_local<G, true>), grid, kHashThreads, 0, a, c);
   else
-    PTC_LAUNCH("k_hash_local", s, k_hash_local<G, false><<<grid, kHashThreads, 0, s>>>(a, c));
+    PTC_KERNEL("k_hash_local", s, (k_hash_local<G, false>), grid, kHashThreads, 0, a, c);
 }
 
 uint32_t chunks_per_block(uint32_t B) {  // G: power of two >= ceil(B / 16)
@@ -863,10 +869,7 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
     return end_call(L.st, s, &h);
   }
   const uint32_t G = chunks_per_block(block_size);
-  PTC_LAUNCH("k_block_offsets", s,
-             k_block_offsets<<<ceil_div_u32(n_req, kOffTile), kOffThreads, 0, s>>>(
-                 req_tok_off, req_ts_us, n_req, n_tok, block_size, kHashThreads / G, req_blk_off_out, L.tile_req,
-                 L.hash_tiles, L.lb_off, L.st));
+  PTC_KERNEL("k_block_offsets", s, k_block_offsets, ceil_div_u32(n_req, kOffTile), kOffThreads, 0, req_tok_off, req_ts_us, n_req, n_tok, block_size, kHashThreads / G, req_blk_off_out, L.tile_req, L.hash_tiles, L.lb_off, L.st);
 
   // seeded bases and their derived constants
   PowBases pb;
@@ -890,7 +893,7 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
     }
     for (int q = 0; q < 32; ++q) hc.sub_mul[b][q] = p61_pow(u, 16ULL * q);
   }
-  PTC_LAUNCH("k_pow_tables", s, k_pow_tables<<<(4 * 1024) / 256, 256, 0, s>>>(pb, L.tables, L.st));
+  PTC_KERNEL("k_pow_tables", s, k_pow_tables, (4 * 1024) / 256, 256, 0, pb, L.tables, L.st);
 
   HashArgs a;
   a.tokens = tokens;
@@ -919,9 +922,7 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
       case 16: launch_hash<16>(grid, s, a, hc, full); break;
       default: launch_hash<32>(grid, s, a, hc, full); break;
     }
-    PTC_LAUNCH("k_hash_chain", s,
-               k_hash_chain<<<ceil_div_u32(grid, kChainWarps), kChainWarps * 32, 0, s>>>(
-                   a.keys, L.tile_agg, L.tile_lead, kHashThreads / G, L.st, keys_cap));
+    PTC_KERNEL("k_hash_chain", s, k_hash_chain, ceil_div_u32(grid, kChainWarps), kChainWarps * 32, 0, a.keys, L.tile_agg, L.tile_lead, kHashThreads / G, L.st, keys_cap);
   }
   DevStatus h;
   ptc_status rc = end_call(L.st, s, &h);

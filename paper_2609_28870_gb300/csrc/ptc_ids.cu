@@ -52,6 +52,7 @@ __device__ __forceinline__ ulonglong2 ld_slot(const ulonglong2* p) {
 __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __restrict__ keys, uint32_t n,
                                                             ulonglong2* table, uint32_t log2m, uint64_t probe_cap,
                                                             uint32_t* __restrict__ slot_of, DevStatus* st) {
+  grid_dep_sync();
   const uint32_t i = blockIdx.x * kInsThreads + threadIdx.x;
   if (i >= n) return;
   const ulonglong2 k = __ldcs(&keys[i]);  // streamed once: keep L2 for the table
@@ -98,6 +99,7 @@ constexpr int kFlTile = kFlT * kFlR;  // 2048 positions; warp w owns [256 w, 256
 __global__ void __launch_bounds__(kFlT) k_ids_flags(const ulonglong2* __restrict__ table, uint32_t* slot_first,
                                                    uint32_t n, uint32_t ntiles, uint32_t* __restrict__ bits,
                                                    uint32_t* tcnt, uint32_t* tpre, uint32_t* done, DevStatus* st) {
+  grid_dep_sync();
   __shared__ uint32_t s_w[kFlT / 32];
   __shared__ uint32_t s_last;
   const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -168,6 +170,7 @@ __global__ void __launch_bounds__(kFlT) k_ids_flags(const ulonglong2* __restrict
 // First occurrences before every word: one warp per tile of 64 words.
 __global__ void k_ids_wordpre(const uint32_t* __restrict__ bits, const uint32_t* __restrict__ tpre, uint32_t nwords,
                               uint32_t* __restrict__ wpre) {
+  grid_dep_sync();
   const uint32_t warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   const uint32_t w0 = warp * (kFlTile / 32);
   if (w0 >= nwords) return;
@@ -189,6 +192,7 @@ __global__ void k_ids_wordpre(const uint32_t* __restrict__ bits, const uint32_t*
 
 __global__ void k_ids_gather(const uint32_t* __restrict__ first, const uint32_t* __restrict__ bits,
                              const uint32_t* __restrict__ wpre, uint32_t n, uint32_t* __restrict__ ids) {
+  grid_dep_sync();
   const uint32_t i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   const uint32_t f = __ldcs(&first[i]);
@@ -245,6 +249,7 @@ IdsLayout ids_layout(void* ws, uint64_t n) {
 // ---------------------------------------------------------------- verify
 __global__ void k_verify_first(const uint32_t* __restrict__ ids, uint64_t n, uint64_t D, uint32_t* first,
                                DevStatus* st) {
+  grid_dep_sync();
   const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   const uint32_t id = ids[i];
@@ -271,6 +276,7 @@ __global__ void k_verify(const uint32_t* __restrict__ tokens, uint64_t n_tok, co
                          const uint64_t* __restrict__ blk_off, uint32_t R, uint32_t B,
                          const uint32_t* __restrict__ ids, uint64_t n, uint64_t D,
                          const uint32_t* __restrict__ first, DevStatus* st) {
+  grid_dep_sync();
   const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   const uint32_t id = ids[i];
@@ -319,15 +325,10 @@ extern "C" ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t*
     if (cudaMemsetAsync(L.table, 0xFF, sizeof(ulonglong2) << log2m, s) != cudaSuccess) return false;
     const ulonglong2* k = reinterpret_cast<const ulonglong2*>(keys);
     const uint32_t n32 = (uint32_t)n;
-    PTC_LAUNCH("k_ids_insert", s, k_ids_insert<<<ceil_div_u32(n, kInsThreads), kInsThreads, 0, s>>>(
-                                      k, n32, L.table, log2m, probe_cap, L.slot_of, L.st));
-    PTC_LAUNCH("k_ids_flags", s, k_ids_flags<<<L.ntiles, kFlT, 0, s>>>(L.table, L.slot_of, n32, L.ntiles, L.bits,
-                                                                       L.tcnt, L.tpre, &L.done[0], L.st));
-    PTC_LAUNCH("k_ids_wordpre", s,
-               k_ids_wordpre<<<ceil_div_u32((uint64_t)L.ntiles * 32, 256), 256, 0, s>>>(L.bits, L.tpre, L.nwords,
-                                                                                        L.wpre));
-    PTC_LAUNCH("k_ids_gather", s,
-               k_ids_gather<<<ceil_div_u32(n, 256), 256, 0, s>>>(L.slot_of, L.bits, L.wpre, n32, ids_out));
+    PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads), kInsThreads, 0, k, n32, L.table, log2m, probe_cap, L.slot_of, L.st);
+    PTC_KERNEL("k_ids_flags", s, k_ids_flags, L.ntiles, kFlT, 0, L.table, L.slot_of, n32, L.ntiles, L.bits, L.tcnt, L.tpre, &L.done[0], L.st);
+    PTC_KERNEL("k_ids_wordpre", s, k_ids_wordpre, ceil_div_u32((uint64_t)L.ntiles * 32, 256), 256, 0, L.bits, L.tpre, L.nwords, L.wpre);
+    PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, 256), 256, 0, L.slot_of, L.bits, L.wpre, n32, ids_out);
     return true;
   };
   if (n > 0) {
@@ -376,9 +377,8 @@ extern "C" ptc_status ptc_verify_ids(const uint32_t* tokens, uint64_t n_tok, con
   if (begin_call(ws, kStatusBytes, s) != PTC_OK) return PTC_ERR_CUDA;
   if (cudaMemsetAsync(first, 0xFF, sizeof(uint32_t) * (n_distinct ? n_distinct : 1), s) != cudaSuccess)
     return PTC_ERR_CUDA;
-  PTC_LAUNCH("k_verify_first", s, k_verify_first<<<ceil_div_u32(n, 256), 256, 0, s>>>(ids, n, n_distinct, first, st));
-  PTC_LAUNCH("k_verify", s, k_verify<<<ceil_div_u32(n, 256), 256, 0, s>>>(tokens, n_tok, req_tok_off, req_blk_off, n_req, block_size, ids, n,
-                                               n_distinct, first, st));
+  PTC_KERNEL("k_verify_first", s, k_verify_first, ceil_div_u32(n, 256), 256, 0, ids, n, n_distinct, first, st);
+  PTC_KERNEL("k_verify", s, k_verify, ceil_div_u32(n, 256), 256, 0, tokens, n_tok, req_tok_off, req_blk_off, n_req, block_size, ids, n, n_distinct, first, st);
   DevStatus h;
   return end_call(st, s, &h);
 }

@@ -3,6 +3,8 @@
 
 #include <cuda_runtime.h>
 
+#include <utility>
+
 #include "../../include/ptc.h"
 #include "ptc_common.cuh"
 
@@ -22,6 +24,33 @@ void timer_resolve();
     __VA_ARGS__;                                \
     ::ptc::timer_launch_end(stream);            \
   } while (0)
+
+// Launch with programmatic stream serialization: the kernel's CTAs may be
+// scheduled before the previous kernel on `s` has finished, and wait for it
+// in grid_dep_sync() (every kernel of this library starts with it).  After a
+// copy or memset the launch is ordered as usual.  A launch error is left for
+// end_call's cudaGetLastError.
+template <typename... KArgs, typename... Args>
+inline void launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args&&... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  (void)cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+// PTC_KERNEL(name, stream, kernel, grid, block, smem, args...): a counted
+// (and, while timing, bracketed) launch_pdl.  A template kernel whose
+// arguments hold a comma goes in parentheses.
+#define PTC_KERNEL(name, stream, kernel, grid, block, smem, ...) \
+  PTC_LAUNCH(name, stream, ::ptc::launch_pdl(kernel, grid, block, smem, stream, __VA_ARGS__))
 
 // Zero the status block (and any extra prefix of the workspace) on `stream`.
 inline ptc_status begin_call(void* ws, size_t zero_bytes, cudaStream_t stream) {

@@ -126,6 +126,7 @@ __device__ __forceinline__ void id_starts(const IrArgs& a, uint32_t base, uint32
 }
 
 __global__ void __launch_bounds__(kIT) k_ir_count(IrArgs a) {
+  grid_dep_sync();
   __shared__ uint32_t s_w[kIT / 32];
   const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   uint32_t id[kIR], left[kIR], words[kIR];
@@ -144,6 +145,7 @@ __global__ void __launch_bounds__(kIT) k_ir_count(IrArgs a) {
 }
 
 __global__ void __launch_bounds__(kIT) k_ir_mark(IrArgs a) {
+  grid_dep_sync();
   __shared__ uint32_t s_w[kIT / 32];
   if (*(volatile uint32_t*)&a.st->err) return;  // ids >= D: reported, nothing is indexed by them
   const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -180,6 +182,7 @@ __global__ void __launch_bounds__(kIT) k_ir_mark(IrArgs a) {
 // lists the cut of every rank.
 __global__ void __launch_bounds__(kIT) k_bm_count(const uint32_t* __restrict__ bits, uint32_t nwords, uint32_t T,
                                                   uint32_t* tcnt, uint32_t* tpre, uint32_t* done, DevStatus* st) {
+  grid_dep_sync();
   __shared__ uint32_t s_w[kIT / 32];
   const uint32_t w0 = blockIdx.x * kBmTile + threadIdx.x * kBmPer;
   uint32_t c = 0;
@@ -197,6 +200,7 @@ __global__ void __launch_bounds__(kIT) k_bm_count(const uint32_t* __restrict__ b
 __global__ void __launch_bounds__(kIT) k_bm_words(const uint32_t* __restrict__ bits, uint32_t nwords,
                                                   const uint32_t* __restrict__ tpre, uint32_t* __restrict__ wpre,
                                                   uint32_t* __restrict__ cut_at) {
+  grid_dep_sync();
   __shared__ uint32_t s_w[kIT / 32];
   const uint32_t w0 = blockIdx.x * kBmTile + threadIdx.x * kBmPer;
   uint32_t b[kBmPer], c = 0;
@@ -245,6 +249,7 @@ __device__ __forceinline__ void run_intervals(const IncArgs& a, uint32_t r, uint
 
 // Persistent over the run tiles (the number of runs is known on the device only).
 __global__ void __launch_bounds__(kIT) k_ir_inc1(IncArgs a) {
+  grid_dep_sync();
   __shared__ uint32_t s_w[kIT / 32];
   if (*(volatile const uint32_t*)&a.stc->err) return;  // the records are incomplete
   const uint32_t R = (uint32_t)a.stc->value[1];
@@ -270,6 +275,7 @@ __global__ void __launch_bounds__(kIT) k_ir_inc1(IncArgs a) {
 }
 
 __global__ void __launch_bounds__(kIT) k_ir_inc2(IncArgs a, uint32_t R) {
+  grid_dep_sync();
   __shared__ uint32_t s_w[kIT / 32];
   const uint32_t t = blockIdx.x;
   const uint32_t r0 = t * kRunTile + threadIdx.x * kRunPer;
@@ -307,6 +313,7 @@ struct FillArgs {
 // One warp per incidence (e, r): the accesses of run r with ids in e take
 // their previous / next use from the runs before / after r on e.
 __global__ void __launch_bounds__(256) k_ir_fill(FillArgs a) {
+  grid_dep_sync();
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t warps = gridDim.x * (blockDim.x >> 5);
   for (uint32_t q = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; q < a.K; q += warps) {
@@ -406,11 +413,10 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
   a.rec_x = L.rec_x;
   a.cut = L.cut;
   a.st = L.st;
-  PTC_LAUNCH("k_ir_count", s, k_ir_count<<<L.ntiles, kIT, 0, s>>>(a));
-  PTC_LAUNCH("k_ir_mark", s, k_ir_mark<<<L.ntiles, kIT, 0, s>>>(a));
-  PTC_LAUNCH("k_bm_count", s,
-             k_bm_count<<<L.btiles, kIT, 0, s>>>(L.cut, L.nwords, L.btiles, L.btcnt, L.btpre, &L.done[1], L.st));
-  PTC_LAUNCH("k_bm_words", s, k_bm_words<<<L.btiles, kIT, 0, s>>>(L.cut, L.nwords, L.btpre, L.cwpre, L.cut_at));
+  PTC_KERNEL("k_ir_count", s, k_ir_count, L.ntiles, kIT, 0, a);
+  PTC_KERNEL("k_ir_mark", s, k_ir_mark, L.ntiles, kIT, 0, a);
+  PTC_KERNEL("k_bm_count", s, k_bm_count, L.btiles, kIT, 0, L.cut, L.nwords, L.btiles, L.btcnt, L.btpre, &L.done[1], L.st);
+  PTC_KERNEL("k_bm_words", s, k_bm_words, L.btiles, kIT, 0, L.cut, L.nwords, L.btpre, L.cwpre, L.cut_at);
   IncArgs ia;
   ia.rec_s = L.rec_s;
   ia.rec_x = L.rec_x;
@@ -425,7 +431,7 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
   ia.max_tiles = L.rtiles_max;
   ia.st = L.st;
   const uint32_t g1 = L.rtiles_max < (uint32_t)(2 * num_sms()) ? L.rtiles_max : (uint32_t)(2 * num_sms());
-  PTC_LAUNCH("k_ir_inc1", s, k_ir_inc1<<<g1, kIT, 0, s>>>(ia));
+  PTC_KERNEL("k_ir_inc1", s, k_ir_inc1, g1, kIT, 0, ia);
   DevStatus h;
   ptc_status rc = end_call(L.st, s, &h);
   if (rc != PTC_OK) return rc;
@@ -434,7 +440,7 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
     if (forced) return PTC_ERR_WORKSPACE;  // cannot happen: K <= n
     return reuse_by_sort(ids, n, D, prev_out, next_out, ws, ws_bytes, s);
   }
-  PTC_LAUNCH("k_ir_inc2", s, k_ir_inc2<<<ceil_div_u32(R, kRunTile), kIT, 0, s>>>(ia, (uint32_t)R));
+  PTC_KERNEL("k_ir_inc2", s, k_ir_inc2, ceil_div_u32(R, kRunTile), kIT, 0, ia, (uint32_t)R);
   const uint32_t *skey = nullptr, *sval = nullptr;
   sort_pairs(L.key, L.val, (uint32_t)K, bits_for(M - 1), L.sort_ws, s, L.st, &skey, &sval);
   FillArgs f;
@@ -449,7 +455,7 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
   f.next = next_out;
   const uint32_t fill_blocks = ceil_div_u32(K, 8) < (uint32_t)(16 * num_sms()) ? ceil_div_u32(K, 8)
                                                                                 : (uint32_t)(16 * num_sms());
-  PTC_LAUNCH("k_ir_fill", s, k_ir_fill<<<fill_blocks, 256, 0, s>>>(f));
+  PTC_KERNEL("k_ir_fill", s, k_ir_fill, fill_blocks, 256, 0, f);
   if (defer_err) return defer_status(L.st, defer_err, s);
   return end_call(L.st, s, &h);
 }

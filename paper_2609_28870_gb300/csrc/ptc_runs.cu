@@ -111,6 +111,7 @@ __device__ __forceinline__ bool last_cta(uint32_t* done) {
 
 // Pass 1: run starts per tile; the last CTA turns them into tile prefixes.
 __global__ void __launch_bounds__(kMT) k_runs_count(MarkArgs a) {
+  grid_dep_sync();
   __shared__ uint32_t s_wcnt[kMT / 32];
   __shared__ uint32_t s_scan[kMT / 32];
   const uint32_t tile = blockIdx.x;
@@ -160,6 +161,7 @@ __global__ void __launch_bounds__(kMT) k_runs_count(MarkArgs a) {
 
 // Pass 2: bitmap, run index per word, and the (start, first value) records.
 __global__ void __launch_bounds__(kMT) k_runs_mark(MarkArgs a) {
+  grid_dep_sync();
   __shared__ uint32_t s_wcnt[kMT / 32];
   const uint32_t tile = blockIdx.x;
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -260,6 +262,7 @@ __global__ void __launch_bounds__(kRT) k_runs_init(const uint32_t* __restrict__ 
                                                   uint32_t* __restrict__ key, uint32_t* __restrict__ wt,
                                                   uint2* __restrict__ acc, uint2* __restrict__ pre, uint32_t* done,
                                                   uint32_t R, uint32_t ntiles, uint32_t shift) {
+  grid_dep_sync();
   __shared__ unsigned long long s_warp[kRT / 32];
   const uint32_t r0 = blockIdx.x * kRTile + threadIdx.x * kRPer;
   uint32_t cz = 0, cw = 0;
@@ -285,6 +288,7 @@ __global__ void __launch_bounds__(kRT) k_runs_init(const uint32_t* __restrict__ 
 }
 
 __global__ void __launch_bounds__(kRT) k_runs_level(LevelArgs a) {
+  grid_dep_sync();
   __shared__ unsigned long long s_warp[kRT / 32];
   __shared__ uint32_t s_red[4][2][kRT / 32];
   const uint32_t t = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -400,6 +404,7 @@ struct BuildArgs {
 };
 
 __global__ void __launch_bounds__(kCT) k_runs_build_cluster(BuildArgs a) {
+  grid_dep_sync();
   extern __shared__ uint2 s_dyn[];  // two buffers of `slice` (key, weight)
   __shared__ unsigned long long s_rw[kCPer * 32];  // per (round, warp) (zeros, zero weight)
   __shared__ unsigned long long s_tot, s_pre, s_all;
@@ -553,6 +558,7 @@ __device__ __forceinline__ uint32_t run_of(const uint32_t* bits, const uint32_t*
 }
 
 __global__ void __launch_bounds__(256) k_runs_query(QueryArgs a) {
+  grid_dep_sync();
   const uint32_t r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= a.R) return;
   const uint32_t x = a.rec_a[r];  // p + 1
@@ -591,6 +597,7 @@ __global__ void __launch_bounds__(256) k_runs_query(QueryArgs a) {
 __global__ void __launch_bounds__(256) k_runs_expand(const uint32_t* __restrict__ bits,
                                                     const uint32_t* __restrict__ wpre, const uint32_t* __restrict__ sd,
                                                     uint32_t n, uint32_t* __restrict__ dist) {
+  grid_dep_sync();
   const uint32_t j = blockIdx.x * blockDim.x + threadIdx.x;
   if (j >= n) return;
   dist[j] = sd[run_of(bits, wpre, j)];
@@ -671,8 +678,8 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   m.tpre = M.tpre;
   m.done = &M.done[63];
   m.st = M.st;
-  PTC_LAUNCH("k_runs_count", s, k_runs_count<<<M.mtiles, kMT, 0, s>>>(m));
-  PTC_LAUNCH("k_runs_mark", s, k_runs_mark<<<M.mtiles, kMT, 0, s>>>(m));
+  PTC_KERNEL("k_runs_count", s, k_runs_count, M.mtiles, kMT, 0, m);
+  PTC_KERNEL("k_runs_mark", s, k_runs_mark, M.mtiles, kMT, 0, m);
   DevStatus h;
   ptc_status rc = end_call(M.st, s, &h);
   if (rc != PTC_OK) return rc;
@@ -705,7 +712,7 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
     b.L = L;
     b.slice = ceil_div_u32(R, C);
     cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = C;
     attr[0].val.clusterDim.y = 1;
@@ -721,6 +728,9 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
       (void)cudaGetLastError();
       continue;
     }
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // as launch_pdl
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.numAttrs = 2;
     cudaError_t e = cudaSuccess;
     PTC_LAUNCH("k_runs_build_cluster", s, e = cudaLaunchKernelEx(&cfg, k_runs_build_cluster, b));
     if (e == cudaSuccess)
@@ -729,8 +739,7 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
       (void)cudaGetLastError();
   }
   if (!built) {
-    PTC_LAUNCH("k_runs_init", s,
-               k_runs_init<<<T, kRT, 0, s>>>(W.rec_s, W.rec_a, W.k0, W.w0, W.acc, W.pre, &W.done[0], R32, T, L - 1));
+    PTC_KERNEL("k_runs_init", s, k_runs_init, T, kRT, 0, W.rec_s, W.rec_a, W.k0, W.w0, W.acc, W.pre, &W.done[0], R32, T, L - 1);
     uint32_t* keys[2] = {W.k0, W.k1};
     uint32_t* wts[2] = {W.w0, W.w1};
     for (uint32_t l = 0; l < L; ++l) {
@@ -748,7 +757,7 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
       a.R = R32;
       a.ntiles = T;
       a.shift = L - 1 - l;
-      PTC_LAUNCH("k_runs_level", s, k_runs_level<<<T, kRT, 0, s>>>(a));
+      PTC_KERNEL("k_runs_level", s, k_runs_level, T, kRT, 0, a);
     }
   }
   QueryArgs q;
@@ -760,9 +769,8 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   q.sd = W.sd;
   q.R = R32;
   q.L = L;
-  PTC_LAUNCH("k_runs_query", s, k_runs_query<<<ceil_div_u32(R, 256), 256, 0, s>>>(q));
-  PTC_LAUNCH("k_runs_expand", s,
-             k_runs_expand<<<ceil_div_u32(n, 256), 256, 0, s>>>(W.bits, W.wpre, W.sd, (uint32_t)n, dist_out));
+  PTC_KERNEL("k_runs_query", s, k_runs_query, ceil_div_u32(R, 256), 256, 0, q);
+  PTC_KERNEL("k_runs_expand", s, k_runs_expand, ceil_div_u32(n, 256), 256, 0, W.bits, W.wpre, W.sd, (uint32_t)n, dist_out);
   const ptc_status done = defer_err ? defer_status(W.st, defer_err, s) : end_call(W.st, s, &h);
   if (done == PTC_OK && view) {
     view->used = true;

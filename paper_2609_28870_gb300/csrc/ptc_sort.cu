@@ -33,6 +33,7 @@ __global__ void __launch_bounds__(kSortThreads) k_sort_count(const uint32_t* __r
                                                              uint32_t shift, uint32_t R, uint32_t T,
                                                              uint32_t key_limit, bool vec,
                                                              uint32_t* __restrict__ cnt, DevStatus* st) {
+  grid_dep_sync();
   __shared__ uint32_t h[kSortWarps][kRadix];
   for (uint32_t x = threadIdx.x; x < kSortWarps * kRadix; x += kSortThreads) (&h[0][0])[x] = 0;
   __syncthreads();
@@ -114,6 +115,7 @@ __device__ __forceinline__ V block_excl_scan(V x, V* s_warp, V& total) {
 // tot[d] = the row's sum.
 __global__ void __launch_bounds__(kSortThreads) k_sort_rowscan(const uint32_t* __restrict__ cnt, uint32_t T,
                                                                uint32_t* __restrict__ off, uint32_t* __restrict__ tot) {
+  grid_dep_sync();
   __shared__ uint32_t s_warp[kSortWarps];
   const uint32_t d = blockIdx.x;
   const uint32_t per = (T + kSortThreads - 1) / kSortThreads;
@@ -148,6 +150,7 @@ struct ScatterArgs {
 
 template <bool LAST>
 __global__ void __launch_bounds__(kSortThreads, 3) k_sort_scatter(ScatterArgs a) {
+  grid_dep_sync();
   __shared__ uint32_t s_keys[kSortTile];
   __shared__ uint32_t s_vals[kSortTile];
   __shared__ uint32_t s_whist[kSortWarps][kRadix];
@@ -269,6 +272,7 @@ __global__ void __launch_bounds__(kSortThreads) k_sort_links(const uint32_t* __r
                                                              const uint2* __restrict__ head_kv,
                                                              const uint2* __restrict__ tail_kv, uint32_t n,
                                                              uint32_t* __restrict__ prev, uint32_t* __restrict__ next) {
+  grid_dep_sync();
   __shared__ int32_t s_last[kSortThreads];
   const uint32_t d = blockIdx.x;
   const size_t row = (size_t)d * T;
@@ -358,10 +362,8 @@ ptc_status ptc::reuse_by_sort(const uint32_t* ids, uint64_t n, uint64_t n_distin
     const uint32_t width = (bits - shift + (passes - p) - 1) / (passes - p);  // spread bits evenly
     const uint32_t R = 1u << width;
     const bool last = p + 1 == passes;
-    PTC_LAUNCH("k_sort_count", s,
-               k_sort_count<<<T, kSortThreads, 0, s>>>(kin, n32, shift, R, T, p == 0 ? (uint32_t)n_distinct : kNone,
-                                                       ((uintptr_t)kin & 15) == 0, L.cnt, L.st));
-    PTC_LAUNCH("k_sort_rowscan", s, k_sort_rowscan<<<R, kSortThreads, 0, s>>>(L.cnt, T, L.off, L.tot));
+    PTC_KERNEL("k_sort_count", s, k_sort_count, T, kSortThreads, 0, kin, n32, shift, R, T, p == 0 ? (uint32_t)n_distinct : kNone, ((uintptr_t)kin & 15) == 0, L.cnt, L.st);
+    PTC_KERNEL("k_sort_rowscan", s, k_sort_rowscan, R, kSortThreads, 0, L.cnt, T, L.off, L.tot);
     ScatterArgs a;
     a.keys_in = kin;
     a.vals_in = vin;
@@ -379,11 +381,10 @@ ptc_status ptc::reuse_by_sort(const uint32_t* ids, uint64_t n, uint64_t n_distin
     a.R = R;
     a.width = width;
     if (last) {
-      PTC_LAUNCH("k_sort_scatter", s, k_sort_scatter<true><<<T, kSortThreads, 0, s>>>(a));
-      PTC_LAUNCH("k_sort_links", s,
-                 k_sort_links<<<R, kSortThreads, 0, s>>>(L.cnt, T, L.head_kv, L.tail_kv, n32, prev_out, next_out));
+      PTC_KERNEL("k_sort_scatter", s, k_sort_scatter<true>, T, kSortThreads, 0, a);
+      PTC_KERNEL("k_sort_links", s, k_sort_links, R, kSortThreads, 0, L.cnt, T, L.head_kv, L.tail_kv, n32, prev_out, next_out);
     } else {
-      PTC_LAUNCH("k_sort_scatter", s, k_sort_scatter<false><<<T, kSortThreads, 0, s>>>(a));
+      PTC_KERNEL("k_sort_scatter", s, k_sort_scatter<false>, T, kSortThreads, 0, a);
     }
     kin = kout;
     vin = vout;
@@ -413,10 +414,8 @@ void ptc::sort_pairs(const uint32_t* keys, const uint32_t* vals, uint32_t n, uin
   for (uint32_t p = 0; p < passes; ++p) {
     const uint32_t width = (bits - shift + (passes - p) - 1) / (passes - p);
     const uint32_t R = 1u << width;
-    PTC_LAUNCH("k_sort_count", s,
-               k_sort_count<<<T, kSortThreads, 0, s>>>(kin, n, shift, R, T, kNone, ((uintptr_t)kin & 15) == 0, L.cnt,
-                                                       st));
-    PTC_LAUNCH("k_sort_rowscan", s, k_sort_rowscan<<<R, kSortThreads, 0, s>>>(L.cnt, T, L.off, L.tot));
+    PTC_KERNEL("k_sort_count", s, k_sort_count, T, kSortThreads, 0, kin, n, shift, R, T, kNone, ((uintptr_t)kin & 15) == 0, L.cnt, st);
+    PTC_KERNEL("k_sort_rowscan", s, k_sort_rowscan, R, kSortThreads, 0, L.cnt, T, L.off, L.tot);
     ScatterArgs a = {};
     a.keys_in = kin;
     a.vals_in = vin;
@@ -429,7 +428,7 @@ void ptc::sort_pairs(const uint32_t* keys, const uint32_t* vals, uint32_t n, uin
     a.shift = shift;
     a.R = R;
     a.width = width;
-    PTC_LAUNCH("k_sort_scatter", s, k_sort_scatter<false><<<T, kSortThreads, 0, s>>>(a));
+    PTC_KERNEL("k_sort_scatter", s, k_sort_scatter<false>, T, kSortThreads, 0, a);
     kin = kout;
     vin = vout;
     kout = (kout == L.k0) ? L.k1 : L.k0;

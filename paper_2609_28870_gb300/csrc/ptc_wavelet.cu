@@ -115,6 +115,7 @@ __device__ inline void finish_counts(uint32_t* done, const uint32_t* tz, uint32_
 // Level-0 zero count of every tile (bit L-1 of v = prev + 1), Z_0 and the
 // tile prefixes; also checks prev[j] < j.
 __global__ void __launch_bounds__(kLT) k_wm_count0(LevelArgs a) {
+  grid_dep_sync();
   __shared__ uint32_t s_wz[kLW];
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const uint32_t n32 = (uint32_t)a.n;
@@ -152,6 +153,7 @@ __global__ void __launch_bounds__(kLT) k_wm_count0(LevelArgs a) {
 // in (the zeros and the ones of a tile each meet at most two such tiles); the
 // CTA that finishes last turns those counts into the next level's prefixes.
 __global__ void __launch_bounds__(kLT) k_wm_level(LevelArgs a) {
+  grid_dep_sync();
   __shared__ uint32_t s_wz[kLW];
   __shared__ uint32_t s_cnt[kLW][4];
   const uint32_t t = threadIdx.x, lane = t & 31, w = t >> 5;
@@ -243,6 +245,7 @@ __global__ void __launch_bounds__(kLT) k_wm_level(LevelArgs a) {
 __global__ void __launch_bounds__(kSbPerChunk) k_wm_dir(const uint32_t* __restrict__ bits, uint64_t lw, uint32_t L,
                                                         uint32_t nsb, uint32_t nchunk, uint32_t* __restrict__ dir,
                                                         uint32_t* csum, uint32_t* __restrict__ cpre, uint32_t* done) {
+  grid_dep_sync();
   __shared__ uint32_t s_w[kSbPerChunk / 32];
   __shared__ bool s_last;
   const uint32_t t = threadIdx.x, lane = t & 31, w = t >> 5;
@@ -357,6 +360,7 @@ struct QueryArgs {
 // Pass 1: run heads query the matrix and write their distances; every tile
 // records its head bits and (last head's distance, any head).  No tile waits.
 __global__ void __launch_bounds__(kQThreads) k_wm_heads(QueryArgs a) {
+  grid_dep_sync();
   __shared__ uint32_t s_z[33];
   __shared__ RunVal s_last[kQThreads / 32];
   if (threadIdx.x < a.L) s_z[threadIdx.x] = (uint32_t)a.zcount[threadIdx.x];
@@ -417,6 +421,7 @@ __global__ void __launch_bounds__(kQThreads) k_wm_heads(QueryArgs a) {
 
 // Pass 2: every access takes the distance of the last head at or before it.
 __global__ void __launch_bounds__(kQThreads) k_wm_propagate(QueryArgs a) {
+  grid_dep_sync();
   __shared__ RunVal s_w[kQThreads / 32];
   __shared__ RunVal s_carry;
   const uint32_t tile = blockIdx.x;
@@ -583,7 +588,7 @@ ptc_status ptc::stack_distance_points(const uint32_t* prev, uint64_t n, uint32_t
   a.z_next = &W.zcount[0];
   a.done = &W.done[62];
   a.st = W.st;
-  PTC_LAUNCH("k_wm_count0", s, k_wm_count0<<<tiles, kLT, 0, s>>>(a));
+  PTC_KERNEL("k_wm_count0", s, k_wm_count0, tiles, kLT, 0, a);
   uint32_t* bufs[2] = {W.va, W.vb};
   for (uint32_t l = 0; l < W.L; ++l) {
     const bool last = l + 1 == W.L;
@@ -598,11 +603,9 @@ ptc_status ptc::stack_distance_points(const uint32_t* prev, uint64_t n, uint32_t
     a.tp_next = last ? nullptr : W.tp + (uint64_t)(l + 1) * (tiles + 1);
     a.z_next = last ? nullptr : &W.zcount[l + 1];
     a.done = &W.done[l];
-    PTC_LAUNCH("k_wm_level", s, k_wm_level<<<tiles, kLT, 0, s>>>(a));
+    PTC_KERNEL("k_wm_level", s, k_wm_level, tiles, kLT, 0, a);
   }
-  PTC_LAUNCH("k_wm_dir", s,
-             k_wm_dir<<<W.L * W.nchunk, kSbPerChunk, 0, s>>>(W.bits, W.lw, W.L, W.nsb, W.nchunk, W.dir, W.csum, W.cpre,
-                                                            &W.done[63]));
+  PTC_KERNEL("k_wm_dir", s, k_wm_dir, W.L * W.nchunk, kSbPerChunk, 0, W.bits, W.lw, W.L, W.nsb, W.nchunk, W.dir, W.csum, W.cpre, &W.done[63]);
   QueryArgs q;
   q.prev = prev;
   q.n = n;
@@ -613,8 +616,8 @@ ptc_status ptc::stack_distance_points(const uint32_t* prev, uint64_t n, uint32_t
   q.heads = W.heads;
   q.tile_agg = W.qagg;
   q.st = W.st;
-  PTC_LAUNCH("k_wm_heads", s, k_wm_heads<<<ceil_div_u32(n, kQTile), kQThreads, 0, s>>>(q));
-  PTC_LAUNCH("k_wm_propagate", s, k_wm_propagate<<<ceil_div_u32(n, kQTile), kQThreads, 0, s>>>(q));
+  PTC_KERNEL("k_wm_heads", s, k_wm_heads, ceil_div_u32(n, kQTile), kQThreads, 0, q);
+  PTC_KERNEL("k_wm_propagate", s, k_wm_propagate, ceil_div_u32(n, kQTile), kQThreads, 0, q);
   DevStatus h;
   return end_call(W.st, s, &h);
 }
