@@ -1,4 +1,5 @@
-// C-ABI entry points that belong to no stage, and the launch timer.
+// C-ABI entry points that belong to no stage, the launch timer, the host
+// staging buffers and the fill / copy kernels every stage uses.
 #include <atomic>
 #include <cstring>
 #include <map>
@@ -75,6 +76,89 @@ void timer_resolve() {
     t.pool.push_back(p.b);
   }
   t.pending.clear();
+}
+
+namespace {
+thread_local bool t_no_host_alloc = false;
+}
+NoHostAlloc::NoHostAlloc() : prev(t_no_host_alloc) { t_no_host_alloc = true; }
+NoHostAlloc::~NoHostAlloc() { t_no_host_alloc = prev; }
+
+HostStage* host_stage() {
+  static thread_local HostStage* pinned = nullptr;
+  static thread_local HostStage fallback;
+  if (!pinned) {
+    fallback.dev = nullptr;
+    if (t_no_host_alloc) return &fallback;
+    void* p = nullptr;
+    if (cudaHostAlloc(&p, sizeof(HostStage), cudaHostAllocPortable | cudaHostAllocMapped) == cudaSuccess) {
+      pinned = static_cast<HostStage*>(p);
+      void* d = nullptr;
+      pinned->dev = cudaHostGetDevicePointer(&d, p, 0) == cudaSuccess ? static_cast<HostStage*>(d) : nullptr;
+      (void)cudaGetLastError();
+    } else {
+      (void)cudaGetLastError();
+      pinned = &fallback;
+    }
+  }
+  return pinned;
+}
+
+namespace {
+__global__ void k_fill(uint32_t* __restrict__ p, uint32_t v, uint64_t words) {
+  grid_dep_sync();
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const uint64_t quads = (((uintptr_t)p & 15) == 0) ? words / 4 : 0;
+  uint4* p4 = reinterpret_cast<uint4*>(p);
+  for (uint64_t q = i; q < quads; q += stride) p4[q] = make_uint4(v, v, v, v);
+  for (uint64_t w = quads * 4 + i; w < words; w += stride) p[w] = v;
+}
+
+__global__ void k_copy_words(const uint32_t* __restrict__ src, uint32_t* dst, uint32_t words) {
+  grid_dep_sync();
+  for (uint32_t i = threadIdx.x; i < words; i += blockDim.x) dst[i] = src[i];
+}
+
+__global__ void k_copy_err(const DevStatus* st, uint32_t* slot) {
+  grid_dep_sync();
+  *slot = st->err;
+}
+}  // namespace
+
+ptc_status fill_async(void* p, uint32_t pattern, size_t bytes, cudaStream_t s) {
+  if (bytes == 0) return PTC_OK;
+  if ((bytes & 3) || ((uintptr_t)p & 3)) {
+    if (cudaMemsetAsync(p, (int)(pattern & 0xFF), bytes, s) != cudaSuccess) return PTC_ERR_CUDA;
+    return PTC_OK;
+  }
+  const uint64_t words = bytes / 4;
+  const uint64_t want = (words / 4 + 255) / 256;
+  const uint32_t cap = (uint32_t)(4 * num_sms());
+  const uint32_t grid = want < cap ? (uint32_t)(want ? want : 1) : cap;
+  PTC_KERNEL("k_fill", s, k_fill, grid, 256, 0, static_cast<uint32_t*>(p), pattern, words);
+  return PTC_OK;
+}
+
+ptc_status copy_to_host_async(void* host_dst, const void* dev_src, size_t bytes, cudaStream_t s) {
+  HostStage* hs = host_stage();
+  const char* lo = reinterpret_cast<const char*>(hs);
+  const char* d = static_cast<const char*>(host_dst);
+  const bool staged = hs->dev != nullptr && d >= lo && d + bytes <= lo + sizeof(HostStage);
+  if (staged && (bytes & 3) == 0 && ((uintptr_t)dev_src & 3) == 0 && ((uintptr_t)d & 3) == 0) {
+    uint32_t* dst = reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(hs->dev) + (d - lo));
+    PTC_KERNEL("k_copy_words", s, k_copy_words, 1, 256, 0, static_cast<const uint32_t*>(dev_src), dst,
+               (uint32_t)(bytes / 4));
+    return PTC_OK;
+  }
+  if (cudaMemcpyAsync(host_dst, dev_src, bytes, cudaMemcpyDeviceToHost, s) != cudaSuccess) return PTC_ERR_CUDA;
+  return PTC_OK;
+}
+
+ptc_status defer_status(const DevStatus* dev, uint32_t* slot, cudaStream_t stream) {
+  if (cudaGetLastError() != cudaSuccess) return PTC_ERR_CUDA;
+  PTC_KERNEL("k_copy_err", stream, k_copy_err, 1, 1, 0, dev, slot);
+  return PTC_OK;
 }
 
 }  // namespace ptc

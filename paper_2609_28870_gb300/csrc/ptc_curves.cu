@@ -74,7 +74,7 @@ struct CurveArgs {
   const uint32_t* dist;
   uint32_t n;
   const uint32_t* bitmap;
-  const uint64_t* caps;  // device copy of the grid
+  uint32_t caps[PTC_MAX_CAPACITIES];  // the grid, clamped below kNone; by value, so no copy
   uint32_t G;
   unsigned long long* cnt;   // G + 1 bins (last: miss at every capacity)
   unsigned long long* ksum;  // G + 1 bins
@@ -188,7 +188,7 @@ __global__ void __launch_bounds__(kCvThreads) k_curves(CurveArgs a) {
   __shared__ RunMax s_carry;
   const uint32_t G = a.G;
   for (uint32_t g = threadIdx.x; g < G; g += kCvThreads)
-    s_cap[g] = a.caps[g] >= (uint64_t)kNone ? kNone - 1 : (uint32_t)a.caps[g];
+    s_cap[g] = a.caps[g];
   for (uint32_t g = threadIdx.x; g <= G; g += kCvThreads) {
     s_cnt[g] = 0;
     s_ks[g] = 0;
@@ -331,7 +331,7 @@ __global__ void __launch_bounds__(kCvThreads) k_curves_fast(CurveArgs a) {
   __shared__ uint32_t s_off[kFtReq + 2];
   const uint32_t G = a.G;
   for (uint32_t g = threadIdx.x; g < G; g += kCvThreads)
-    s_cap[g] = a.caps[g] >= (uint64_t)kNone ? kNone - 1 : (uint32_t)a.caps[g];
+    s_cap[g] = a.caps[g];
   for (uint32_t g = threadIdx.x; g <= G; g += kCvThreads) {
     s_cnt[g] = 0;
     s_ks[g] = 0;
@@ -478,7 +478,7 @@ __global__ void __launch_bounds__(256) k_curves_runs(CurveArgs a, RunsArgs ra) {
   __shared__ unsigned long long s_ks[PTC_MAX_CAPACITIES + 1];
   const uint32_t G = a.G;
   for (uint32_t g = threadIdx.x; g < G; g += blockDim.x)
-    s_cap[g] = a.caps[g] >= (uint64_t)kNone ? kNone - 1 : (uint32_t)a.caps[g];
+    s_cap[g] = a.caps[g];
   for (uint32_t g = threadIdx.x; g <= G; g += blockDim.x) {
     s_cnt[g] = 0;
     s_ks[g] = 0;
@@ -578,7 +578,6 @@ struct CurvesLayout {
   uint32_t* slow;
   uint32_t* tile_req;
   RunMax* lb_agg;
-  uint64_t* caps;
   uint64_t* out;
   size_t zero_bytes;
   size_t total;
@@ -596,7 +595,6 @@ CurvesLayout curves_layout(void* ws, uint64_t n, uint32_t G) {
   L.tile_req = cv.take<uint32_t>(tiles + 1);
   L.zero_bytes = cv.off;
   L.lb_agg = cv.take<RunMax>(tiles);
-  L.caps = cv.take<uint64_t>(PTC_MAX_CAPACITIES);
   L.out = cv.take<uint64_t>(3 * PTC_MAX_CAPACITIES + 2);
   L.total = cv.bytes();
   (void)G;
@@ -648,8 +646,7 @@ ptc_status ptc::curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* re
   cudaStream_t s = stream;
   const CurvesLayout L = curves_layout(ws, n, n_cap);
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
-  if (cudaMemcpyAsync(L.caps, cap_host, sizeof(uint64_t) * n_cap, cudaMemcpyHostToDevice, s) != cudaSuccess)
-    return PTC_ERR_CUDA;
+  HostStage* hs = host_stage();
   if (n_carry) PTC_KERNEL("k_carry_err", s, k_carry_err, 1, 32, 0, carry_err, n_carry, L.st);
   if (n > 0) {
     PTC_KERNEL("k_heads", s, k_heads, ceil_div_u32(n_req, 256), 256, 0, req_blk_off, n_req, n, L.bitmap, L.tile_req, L.st);
@@ -657,7 +654,8 @@ ptc_status ptc::curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* re
     a.dist = dist;
     a.n = (uint32_t)n;
     a.bitmap = L.bitmap;
-    a.caps = L.caps;
+    for (uint32_t g = 0; g < n_cap; ++g)
+      a.caps[g] = cap_host[g] >= (uint64_t)kNone ? kNone - 1 : (uint32_t)cap_host[g];
     a.G = n_cap;
     a.cnt = L.cnt;
     a.ksum = L.ksum;
@@ -683,9 +681,8 @@ ptc_status ptc::curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* re
     PTC_KERNEL("k_curves", s, k_curves, grid, kCvThreads, 0, a);
   }
   PTC_KERNEL("k_finalize", s, k_finalize, 1, 1024, 0, L.cnt, L.ksum, n_cap, alpha, beta, L.out);
-  static thread_local uint64_t host_out[3 * PTC_MAX_CAPACITIES + 2];
-  if (cudaMemcpyAsync(host_out, L.out, sizeof(uint64_t) * (3 * n_cap + 2), cudaMemcpyDeviceToHost, s) != cudaSuccess)
-    return PTC_ERR_CUDA;
+  const uint64_t* host_out = hs->out;
+  if (copy_to_host_async(hs->out, L.out, sizeof(uint64_t) * (3 * n_cap + 2), s) != PTC_OK) return PTC_ERR_CUDA;
   DevStatus h;
   const ptc_status rc = end_call(L.st, s, &h);
   if (rc != PTC_OK) return rc;
@@ -756,6 +753,7 @@ extern "C" ptc_status ptc_curves_noalloc(const uint32_t* dist, uint64_t n, const
   const ptc_status rc = scratch_for_current_device(&scratch);
   if (rc != PTC_OK) return rc;
   // ptc_curves zeroes every part of the scratch that must start at zero.
+  const NoHostAlloc no_alloc;
   return ptc_curves(dist, n, req_blk_off, n_req, block_size, cm, cap_host, n_cap, hits_host_out, saved_host_out,
                     total_cost_host_out, scratch, kNoAllocScratchBytes, stream);
 }

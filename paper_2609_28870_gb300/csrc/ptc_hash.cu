@@ -864,7 +864,7 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
   *n_access_host_out = 0;
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
   if (n_req == 0) {
-    if (cudaMemsetAsync(req_blk_off_out, 0, sizeof(uint64_t), s) != cudaSuccess) return PTC_ERR_CUDA;
+    if (fill_async(req_blk_off_out, 0u, sizeof(uint64_t), s) != PTC_OK) return PTC_ERR_CUDA;
     DevStatus h;
     return end_call(L.st, s, &h);
   }

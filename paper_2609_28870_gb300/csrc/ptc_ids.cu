@@ -322,7 +322,7 @@ extern "C" ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t*
   const IdsLayout L = ids_layout(ws, n);
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
   auto run = [&](uint32_t log2m, uint64_t probe_cap) -> bool {
-    if (cudaMemsetAsync(L.table, 0xFF, sizeof(ulonglong2) << log2m, s) != cudaSuccess) return false;
+    if (fill_async(L.table, ~0u, sizeof(ulonglong2) << log2m, s) != PTC_OK) return false;
     const ulonglong2* k = reinterpret_cast<const ulonglong2*>(keys);
     const uint32_t n32 = (uint32_t)n;
     PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads), kInsThreads, 0, k, n32, L.table, log2m, probe_cap, L.slot_of, L.st);
@@ -375,7 +375,7 @@ extern "C" ptc_status ptc_verify_ids(const uint32_t* tokens, uint64_t n_tok, con
   DevStatus* st = cv.take<DevStatus>(1);
   uint32_t* first = cv.take<uint32_t>(n_distinct ? n_distinct : 1);
   if (begin_call(ws, kStatusBytes, s) != PTC_OK) return PTC_ERR_CUDA;
-  if (cudaMemsetAsync(first, 0xFF, sizeof(uint32_t) * (n_distinct ? n_distinct : 1), s) != cudaSuccess)
+  if (fill_async(first, ~0u, sizeof(uint32_t) * (n_distinct ? n_distinct : 1), s) != PTC_OK)
     return PTC_ERR_CUDA;
   PTC_KERNEL("k_verify_first", s, k_verify_first, ceil_div_u32(n, 256), 256, 0, ids, n, n_distinct, first, st);
   PTC_KERNEL("k_verify", s, k_verify, ceil_div_u32(n, 256), 256, 0, tokens, n_tok, req_tok_off, req_blk_off, n_req, block_size, ids, n, n_distinct, first, st);

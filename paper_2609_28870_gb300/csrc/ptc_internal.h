@@ -52,18 +52,49 @@ inline void launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 #define PTC_KERNEL(name, stream, kernel, grid, block, smem, ...) \
   PTC_LAUNCH(name, stream, ::ptc::launch_pdl(kernel, grid, block, smem, stream, __VA_ARGS__))
 
+// Fill `bytes` at `p` with the 32-bit `pattern` (0 or all ones) on `s`.  A
+// kernel (k_fill, ptc_abi.cu) rather than cudaMemsetAsync, so that it joins
+// the programmatic launch chain instead of draining the stream around it;
+// sizes or addresses that are not whole 32-bit words go to cudaMemsetAsync.
+ptc_status fill_async(void* p, uint32_t pattern, size_t bytes, cudaStream_t s);
+
 // Zero the status block (and any extra prefix of the workspace) on `stream`.
 inline ptc_status begin_call(void* ws, size_t zero_bytes, cudaStream_t stream) {
-  if (cudaMemsetAsync(ws, 0, zero_bytes, stream) != cudaSuccess) return PTC_ERR_CUDA;
-  return PTC_OK;
+  return fill_async(ws, 0u, zero_bytes, stream);
 }
+
+// Page-locked host buffers for the small copies around a call's wait, one
+// set per host thread (ptc_abi.cu).  A copy from or to pageable memory goes
+// through a driver bounce buffer and costs the wait tens of microseconds.
+// Falls back to ordinary thread-local memory if page-locked memory cannot be
+// had.  Valid until the thread's next call.
+struct HostStage {
+  DevStatus st;
+  uint64_t out[3 * PTC_MAX_CAPACITIES + 2];
+  HostStage* dev;  // the same memory as seen by kernels (mapped), or null
+};
+HostStage* host_stage();
+// Copy `bytes` from device memory to `host_dst`.  When `host_dst` lies in
+// the thread's host stage and that stage is mapped, a one-CTA kernel
+// (k_copy_words) writes it straight into host memory, which joins the launch
+// chain; otherwise cudaMemcpyAsync.
+ptc_status copy_to_host_async(void* host_dst, const void* dev_src, size_t bytes, cudaStream_t s);
+// While one is alive on a thread, host_stage() allocates nothing (the
+// allocation-free entry points): it hands out the thread-local fallback
+// unless the page-locked set already exists.
+struct NoHostAlloc {
+  NoHostAlloc();
+  ~NoHostAlloc();
+  bool prev;
+};
 
 // Wait for the call's work and translate the device status block.
 inline ptc_status end_call(const DevStatus* dev, cudaStream_t stream, DevStatus* host_copy) {
   if (cudaGetLastError() != cudaSuccess) return PTC_ERR_CUDA;
-  if (cudaMemcpyAsync(host_copy, dev, sizeof(DevStatus), cudaMemcpyDeviceToHost, stream) != cudaSuccess)
-    return PTC_ERR_CUDA;
+  DevStatus* pin = &host_stage()->st;
+  if (copy_to_host_async(pin, dev, sizeof(DevStatus), stream) != PTC_OK) return PTC_ERR_CUDA;
   if (cudaStreamSynchronize(stream) != cudaSuccess) return PTC_ERR_CUDA;
+  *host_copy = *pin;
   timer_resolve();
   uint32_t e = host_copy->err;
   if (e & kErrTimeout) return PTC_ERR_TIMEOUT;
@@ -76,12 +107,7 @@ inline ptc_status end_call(const DevStatus* dev, cudaStream_t stream, DevStatus*
 
 // Instead of waiting for a call's status, queue a copy of its error word to
 // `slot`, for a later call that does wait to fold in (ptc_pipeline).
-inline ptc_status defer_status(const DevStatus* dev, uint32_t* slot, cudaStream_t stream) {
-  if (cudaGetLastError() != cudaSuccess) return PTC_ERR_CUDA;
-  if (cudaMemcpyAsync(slot, &dev->err, sizeof(uint32_t), cudaMemcpyDeviceToDevice, stream) != cudaSuccess)
-    return PTC_ERR_CUDA;
-  return PTC_OK;
-}
+ptc_status defer_status(const DevStatus* dev, uint32_t* slot, cudaStream_t stream);
 
 // Streaming multiprocessors of the current device (persistent grids).
 inline int num_sms() {

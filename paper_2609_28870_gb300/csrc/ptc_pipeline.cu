@@ -90,7 +90,7 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
   if (rc != PTC_OK) return rc;
   // stages b and c do not wait for their own status: stage d reads it
   cudaStream_t s = (cudaStream_t)stream;
-  if (cudaMemsetAsync(L.defer, 0, 2 * sizeof(uint32_t), s) != cudaSuccess) return PTC_ERR_CUDA;
+  if (ptc::fill_async(L.defer, 0u, 2 * sizeof(uint32_t), s) != PTC_OK) return PTC_ERR_CUDA;
   ptc::RunsView runs;
   if (n > 0) {
     rc = ptc::reuse_view(ids, n, d, prev, next, L.scratch, L.scratch_bytes, s, &L.defer[0]);

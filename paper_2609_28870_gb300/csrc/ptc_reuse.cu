@@ -400,7 +400,7 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
   const ReuseLayout L = reuse_layout(ws, n, D, forced);
   if (!ws_ok(ws, ws_bytes, L.total)) return PTC_ERR_WORKSPACE;
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
-  if (cudaMemsetAsync(L.cut, 0, sizeof(uint32_t) * L.nwords, s) != cudaSuccess) return PTC_ERR_CUDA;
+  if (fill_async(L.cut, 0u, sizeof(uint32_t) * L.nwords, s) != PTC_OK) return PTC_ERR_CUDA;
   IrArgs a;
   a.ids = ids;
   a.n = (uint32_t)n;

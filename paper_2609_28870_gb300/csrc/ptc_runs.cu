@@ -43,6 +43,8 @@
 
 #include <utility>
 
+#include <atomic>
+
 #include "ptc_internal.h"
 
 namespace cg = cooperative_groups;
@@ -661,6 +663,29 @@ uint64_t runs_reserve(uint64_t n) {
   return r < (1ULL << 24) ? r : (1ULL << 24);
 }
 
+// Whether a cluster of C CTAs of k_runs_build_cluster can be resident, asked
+// once per device and cluster size with the largest shared-memory request (a
+// smaller one fits whenever that does); the occupancy query is slow next to
+// the kernels around it.
+bool cluster_fits(uint32_t C, const cudaLaunchConfig_t& cfg) {
+  constexpr int kDevs = 64;
+  static std::atomic<int8_t> known[kDevs][kCMax + 1];  // 0 unknown, 1 yes, 2 no
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kDevs || C > (uint32_t)kCMax) {
+    (void)cudaGetLastError();
+    return false;
+  }
+  const int8_t k = known[dev][C].load(std::memory_order_relaxed);
+  if (k) return k == 1;
+  cudaLaunchConfig_t q = cfg;
+  q.dynamicSmemBytes = 2 * kCSlice * sizeof(uint2);
+  int clusters = 0;
+  const bool ok = cudaOccupancyMaxActiveClusters(&clusters, k_runs_build_cluster, &q) == cudaSuccess && clusters >= 1;
+  if (!ok) (void)cudaGetLastError();
+  known[dev][C].store(ok ? 1 : 2, std::memory_order_relaxed);
+  return ok;
+}
+
 ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_out, void* ws, size_t ws_bytes,
                                cudaStream_t s, int method, RunsView* view, uint32_t* defer_err = nullptr) {
   const RunsLayout M = runs_layout(ws, n, 1);
@@ -688,8 +713,8 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   const bool fits = R >= 1 && R <= n && ws_bytes >= W.total;
   if (method == PTC_SD_AUTO && (!fits || R > n / 3)) return stack_distance_points(prev, n, dist_out, ws, ws_bytes, s);
   if (!fits) return PTC_ERR_WORKSPACE;
-  if (cudaMemsetAsync(W.acc, 0, W.acc_bytes, s) != cudaSuccess) return PTC_ERR_CUDA;
-  if (cudaMemsetAsync(W.done, 0, 64 * sizeof(uint32_t), s) != cudaSuccess) return PTC_ERR_CUDA;
+  if (fill_async(W.acc, 0u, W.acc_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
+  if (fill_async(W.done, 0u, 64 * sizeof(uint32_t), s) != PTC_OK) return PTC_ERR_CUDA;
   const uint32_t R32 = (uint32_t)R, T = W.rtiles, L = W.L;
   const size_t tstride = (size_t)T + 1;
   // one cluster when the runs fit in its shared memory, else one launch per level
@@ -723,11 +748,7 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
     cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, k_runs_build_cluster, &cfg) != cudaSuccess || clusters < 1) {
-      (void)cudaGetLastError();
-      continue;
-    }
+    if (!cluster_fits(C, cfg)) continue;
     attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // as launch_pdl
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.numAttrs = 2;

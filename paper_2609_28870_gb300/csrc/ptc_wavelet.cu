@@ -571,7 +571,7 @@ ptc_status ptc::stack_distance_points(const uint32_t* prev, uint64_t n, uint32_t
   if (!ws_ok(ws, ws_bytes, wm_layout(nullptr, n).total)) return PTC_ERR_WORKSPACE;
   const WmLayout W = wm_layout(ws, n);
   if (begin_call(ws, W.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
-  if (cudaMemsetAsync(W.bits, 0, sizeof(uint32_t) * (uint64_t)W.L * W.lw, s) != cudaSuccess) return PTC_ERR_CUDA;
+  if (fill_async(W.bits, 0u, sizeof(uint32_t) * (uint64_t)W.L * W.lw, s) != PTC_OK) return PTC_ERR_CUDA;
   const uint32_t tiles = W.ntiles;
   LevelArgs a;
   a.src = prev;
