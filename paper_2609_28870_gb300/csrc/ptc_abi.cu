@@ -120,9 +120,16 @@ __global__ void k_copy_words(const uint32_t* __restrict__ src, uint32_t* dst, ui
   for (uint32_t i = threadIdx.x; i < words; i += blockDim.x) dst[i] = src[i];
 }
 
-__global__ void k_copy_err(const DevStatus* st, uint32_t* slot) {
+// Earlier calls' error words (deferred, see defer_status) join this call's.
+__global__ void k_carry_err(const uint32_t* err, uint32_t n, DevStatus* st) {
+  grid_dep_sync();
+  if (threadIdx.x < n && err[threadIdx.x]) atomicOr(&st->err, err[threadIdx.x]);
+}
+
+__global__ void k_copy_err(const DevStatus* st, uint32_t* slot, uint64_t* value_slot, uint32_t value_index) {
   grid_dep_sync();
   *slot = st->err;
+  if (value_slot) *value_slot = st->value[value_index];
 }
 }  // namespace
 
@@ -155,9 +162,18 @@ ptc_status copy_to_host_async(void* host_dst, const void* dev_src, size_t bytes,
   return PTC_OK;
 }
 
-ptc_status defer_status(const DevStatus* dev, uint32_t* slot, cudaStream_t stream) {
+ptc_status carry_errors(const uint32_t* err, uint32_t n, DevStatus* st, cudaStream_t s) {
+  if (n == 0) return PTC_OK;
+  if (n > 32) return PTC_ERR_INVALID_ARG;
+  PTC_KERNEL("k_carry_err", s, k_carry_err, 1, 32, 0, err, n, st);
+  return PTC_OK;
+}
+
+ptc_status defer_status(const DevStatus* dev, uint32_t* slot, cudaStream_t stream, uint64_t* value_slot,
+                        uint32_t value_index) {
   if (cudaGetLastError() != cudaSuccess) return PTC_ERR_CUDA;
-  PTC_KERNEL("k_copy_err", stream, k_copy_err, 1, 1, 0, dev, slot);
+  if (value_index >= 8) return PTC_ERR_INVALID_ARG;
+  PTC_KERNEL("k_copy_err", stream, k_copy_err, 1, 1, 0, dev, slot, value_slot, value_index);
   return PTC_OK;
 }
 

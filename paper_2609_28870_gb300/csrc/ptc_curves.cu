@@ -513,11 +513,6 @@ __global__ void __launch_bounds__(256) k_curves_runs(CurveArgs a, RunsArgs ra) {
   }
 }
 
-// Earlier calls' error words (deferred, see defer_status) join this call's.
-__global__ void k_carry_err(const uint32_t* err, uint32_t n, DevStatus* st) {
-  grid_dep_sync();
-  if (threadIdx.x < n && err[threadIdx.x]) atomicOr(&st->err, err[threadIdx.x]);
-}
 
 struct U128 {
   uint64_t lo, hi;
@@ -647,7 +642,7 @@ ptc_status ptc::curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* re
   const CurvesLayout L = curves_layout(ws, n, n_cap);
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
   HostStage* hs = host_stage();
-  if (n_carry) PTC_KERNEL("k_carry_err", s, k_carry_err, 1, 32, 0, carry_err, n_carry, L.st);
+  if (n_carry && carry_errors(carry_err, n_carry, L.st, s) != PTC_OK) return PTC_ERR_CUDA;
   if (n > 0) {
     PTC_KERNEL("k_heads", s, k_heads, ceil_div_u32(n_req, 256), 256, 0, req_blk_off, n_req, n, L.bitmap, L.tile_req, L.st);
     CurveArgs a;

@@ -848,16 +848,17 @@ extern "C" size_t ptc_hash_blocks_workspace_bytes(uint32_t n_req, uint64_t n_tok
   return hash_layout(nullptr, n_req, n_tok, block_size, ~0ULL).total;
 }
 
-extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off,
-                                      const int64_t* req_ts_us, uint32_t n_req, uint32_t block_size, uint64_t seed,
-                                      ptc_u128* keys_out, uint64_t keys_cap, uint64_t* req_blk_off_out,
-                                      uint64_t* n_access_host_out, void* ws, size_t ws_bytes, void* stream) {
+ptc_status ptc::hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off,
+                         const int64_t* req_ts_us, uint32_t n_req, uint32_t block_size, uint64_t seed,
+                         ptc_u128* keys_out, uint64_t keys_cap, uint64_t* req_blk_off_out,
+                         uint64_t* n_access_host_out, void* ws, size_t ws_bytes, cudaStream_t s, uint64_t* n_slot,
+                         uint32_t* err_slot) {
   if (block_size < 1 || block_size > PTC_MAX_BLOCK_SIZE) return PTC_ERR_INVALID_ARG;
   if (req_tok_off == nullptr || req_blk_off_out == nullptr || n_access_host_out == nullptr)
     return PTC_ERR_INVALID_ARG;
   if (n_tok > 0 && tokens == nullptr) return PTC_ERR_INVALID_ARG;
   if (keys_cap > 0 && keys_out == nullptr) return PTC_ERR_INVALID_ARG;
-  cudaStream_t s = (cudaStream_t)stream;
+  const bool deferred = n_slot != nullptr && err_slot != nullptr;
   const HashLayout need = hash_layout(nullptr, n_req, n_tok, block_size, ~0ULL);
   if (!ws_ok(ws, ws_bytes, need.total)) return PTC_ERR_WORKSPACE;
   const HashLayout L = hash_layout(ws, n_req, n_tok, block_size, ~0ULL);
@@ -865,6 +866,7 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
   if (n_req == 0) {
     if (fill_async(req_blk_off_out, 0u, sizeof(uint64_t), s) != PTC_OK) return PTC_ERR_CUDA;
+    if (deferred) return defer_status(L.st, err_slot, s, n_slot, 0);
     DevStatus h;
     return end_call(L.st, s, &h);
   }
@@ -924,10 +926,19 @@ extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, co
     }
     PTC_KERNEL("k_hash_chain", s, k_hash_chain, ceil_div_u32(grid, kChainWarps), kChainWarps * 32, 0, a.keys, L.tile_agg, L.tile_lead, kHashThreads / G, L.st, keys_cap);
   }
+  if (deferred) return defer_status(L.st, err_slot, s, n_slot, 0);
   DevStatus h;
   ptc_status rc = end_call(L.st, s, &h);
   *n_access_host_out = h.value[0];
   if (rc != PTC_OK) return rc;
   if (h.value[0] > keys_cap) return PTC_ERR_INVALID_ARG;
   return PTC_OK;
+}
+
+extern "C" ptc_status ptc_hash_blocks(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off,
+                                      const int64_t* req_ts_us, uint32_t n_req, uint32_t block_size, uint64_t seed,
+                                      ptc_u128* keys_out, uint64_t keys_cap, uint64_t* req_blk_off_out,
+                                      uint64_t* n_access_host_out, void* ws, size_t ws_bytes, void* stream) {
+  return ptc::hash_impl(tokens, n_tok, req_tok_off, req_ts_us, n_req, block_size, seed, keys_out, keys_cap,
+                        req_blk_off_out, n_access_host_out, ws, ws_bytes, (cudaStream_t)stream, nullptr, nullptr);
 }

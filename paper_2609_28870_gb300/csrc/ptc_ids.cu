@@ -49,12 +49,21 @@ __device__ __forceinline__ ulonglong2 ld_slot(const ulonglong2* p) {
   return v;
 }
 
-__global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __restrict__ keys, uint32_t n,
-                                                            ulonglong2* table, uint32_t log2m, uint64_t probe_cap,
-                                                            uint32_t* __restrict__ slot_of, DevStatus* st) {
+// The number of keys: n, or min(*n_dev, n) when the count is only known on
+// the device (the pipeline does not wait for stage a1).
+__device__ __forceinline__ uint32_t keys_used(uint32_t n, const uint64_t* n_dev) {
+  if (!n_dev) return n;
+  const uint64_t v = *n_dev;
+  return v < n ? (uint32_t)v : n;
+}
+
+__global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __restrict__ keys, uint32_t n_ub,
+                                                            const uint64_t* n_dev, ulonglong2* table, uint32_t log2m,
+                                                            uint64_t probe_cap, uint32_t* __restrict__ slot_of,
+                                                            DevStatus* st) {
   grid_dep_sync();
   const uint32_t i = blockIdx.x * kInsThreads + threadIdx.x;
-  if (i >= n) return;
+  if (i >= keys_used(n_ub, n_dev)) return;
   const ulonglong2 k = __ldcs(&keys[i]);  // streamed once: keep L2 for the table
   if (k.x >= kP61 || k.y >= kP61) {
     raise_err(st, kErrInvalid);
@@ -95,11 +104,15 @@ constexpr int kFlR = 8;               // rounds of 32 positions per warp
 constexpr int kFlTile = kFlT * kFlR;  // 2048 positions; warp w owns [256 w, 256 w + 256)
 
 // first[i] (in place of slot_of[i]) and the first-occurrence bitmap; tile
-// counts, and the last CTA's tile prefixes (tpre[ntiles] = D).
+// counts, and the last CTA's tile prefixes (tpre[ntiles] = D).  Bitmap words
+// past the keys used but inside the n_ub the grid covers are written as 0.
+// The last CTA also reports D (value[0]) and the key count (value[1]).
 __global__ void __launch_bounds__(kFlT) k_ids_flags(const ulonglong2* __restrict__ table, uint32_t* slot_first,
-                                                   uint32_t n, uint32_t ntiles, uint32_t* __restrict__ bits,
-                                                   uint32_t* tcnt, uint32_t* tpre, uint32_t* done, DevStatus* st) {
+                                                   uint32_t n_ub, const uint64_t* n_dev, uint32_t ntiles,
+                                                   uint32_t* __restrict__ bits, uint32_t* tcnt, uint32_t* tpre,
+                                                   uint32_t* done, DevStatus* st) {
   grid_dep_sync();
+  const uint32_t n = keys_used(n_ub, n_dev);
   __shared__ uint32_t s_w[kFlT / 32];
   __shared__ uint32_t s_last;
   const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -123,7 +136,7 @@ __global__ void __launch_bounds__(kFlT) k_ids_flags(const ulonglong2* __restrict
     const uint32_t i = base + k * 32 + lane;
     if (i < n) __stcs(&slot_first[i], f[k]);
     const uint32_t m = __ballot_sync(kFull, i < n && f[k] == i);
-    if (lane == 0 && base + k * 32 < n) bits[(base + k * 32) >> 5] = m;
+    if (lane == 0 && base + k * 32 < n_ub) bits[(base + k * 32) >> 5] = m;
     cnt += __popc(m);
   }
   if (lane == 0) s_w[w] = cnt;
@@ -164,6 +177,8 @@ __global__ void __launch_bounds__(kFlT) k_ids_flags(const ulonglong2* __restrict
   if (threadIdx.x == 0) {
     tpre[ntiles] = total;
     st->value[0] = total;
+    st->value[1] = n_dev ? *n_dev : n;
+    if (n_dev && *n_dev > n_ub) raise_err(st, kErrInvalid);  // more blocks than the keys buffer holds
   }
 }
 
@@ -191,9 +206,11 @@ __global__ void k_ids_wordpre(const uint32_t* __restrict__ bits, const uint32_t*
 }
 
 __global__ void k_ids_gather(const uint32_t* __restrict__ first, const uint32_t* __restrict__ bits,
-                             const uint32_t* __restrict__ wpre, uint32_t n, uint32_t* __restrict__ ids) {
+                             const uint32_t* __restrict__ wpre, uint32_t n_ub, const uint64_t* n_dev,
+                             uint32_t* __restrict__ ids) {
   grid_dep_sync();
   const uint32_t i = blockIdx.x * blockDim.x + threadIdx.x;
+  const uint32_t n = keys_used(n_ub, n_dev);
   if (i >= n) return;
   const uint32_t f = __ldcs(&first[i]);
   ids[i] = f < n ? wpre[f >> 5] + __popc(bits[f >> 5] & ((1u << (f & 31)) - 1u)) : kNone;
@@ -311,46 +328,60 @@ using namespace ptc;
 
 extern "C" size_t ptc_assign_ids_workspace_bytes(uint64_t n) { return ids_layout(nullptr, n).total; }
 
-extern "C" ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t* ids_out, uint64_t* n_distinct_host_out,
-                                     void* ws, size_t ws_bytes, void* stream) {
+ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev, uint32_t* ids_out,
+                        uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
+                        cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry) {
   if (n_distinct_host_out == nullptr) return PTC_ERR_INVALID_ARG;
   *n_distinct_host_out = 0;
+  if (n_used_host_out) *n_used_host_out = 0;
   if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
   if (n > 0 && (keys == nullptr || ids_out == nullptr)) return PTC_ERR_INVALID_ARG;
   if (!ws_ok(ws, ws_bytes, ids_layout(nullptr, n).total)) return PTC_ERR_WORKSPACE;
-  cudaStream_t s = (cudaStream_t)stream;
   const IdsLayout L = ids_layout(ws, n);
-  if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
+  auto start = [&]() -> bool {
+    return begin_call(ws, L.zero_bytes, s) == PTC_OK && carry_errors(carry_err, n_carry, L.st, s) == PTC_OK;
+  };
   auto run = [&](uint32_t log2m, uint64_t probe_cap) -> bool {
     if (fill_async(L.table, ~0u, sizeof(ulonglong2) << log2m, s) != PTC_OK) return false;
     const ulonglong2* k = reinterpret_cast<const ulonglong2*>(keys);
     const uint32_t n32 = (uint32_t)n;
-    PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads), kInsThreads, 0, k, n32, L.table, log2m, probe_cap, L.slot_of, L.st);
-    PTC_KERNEL("k_ids_flags", s, k_ids_flags, L.ntiles, kFlT, 0, L.table, L.slot_of, n32, L.ntiles, L.bits, L.tcnt, L.tpre, &L.done[0], L.st);
-    PTC_KERNEL("k_ids_wordpre", s, k_ids_wordpre, ceil_div_u32((uint64_t)L.ntiles * 32, 256), 256, 0, L.bits, L.tpre, L.nwords, L.wpre);
-    PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, 256), 256, 0, L.slot_of, L.bits, L.wpre, n32, ids_out);
+    PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads), kInsThreads, 0, k, n32, n_dev, L.table,
+               log2m, probe_cap, L.slot_of, L.st);
+    PTC_KERNEL("k_ids_flags", s, k_ids_flags, L.ntiles, kFlT, 0, L.table, L.slot_of, n32, n_dev, L.ntiles, L.bits,
+               L.tcnt, L.tpre, &L.done[0], L.st);
+    PTC_KERNEL("k_ids_wordpre", s, k_ids_wordpre, ceil_div_u32((uint64_t)L.ntiles * 32, 256), 256, 0, L.bits, L.tpre,
+               L.nwords, L.wpre);
+    PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, 256), 256, 0, L.slot_of, L.bits, L.wpre, n32, n_dev,
+               ids_out);
     return true;
   };
+  if (!start()) return PTC_ERR_CUDA;
+  DevStatus h{};
   if (n > 0) {
     const uint32_t small = small_table_log2(n);
     if (!run(small, small < L.log2m ? kSmallProbeCap : ~0ULL)) return PTC_ERR_CUDA;
     if (small < L.log2m) {
-      DevStatus h1;
-      const ptc_status rc1 = end_call(L.st, s, &h1);
-      if (rc1 == PTC_OK) {
-        *n_distinct_host_out = h1.value[0];
-        return PTC_OK;
+      const ptc_status rc1 = end_call(L.st, s, &h);
+      // anything but a probe sequence outrunning the small table is final
+      if (rc1 == PTC_OK || h.err != kErrTableFull) {
+        *n_distinct_host_out = h.value[0];
+        if (n_used_host_out) *n_used_host_out = h.value[1];
+        return rc1;
       }
-      if (!(h1.err & kErrTableFull)) return rc1;
       // the small table overflowed: redo with the full one
-      if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
-      if (!run(L.log2m, ~0ULL)) return PTC_ERR_CUDA;
+      if (!start() || !run(L.log2m, ~0ULL)) return PTC_ERR_CUDA;
     }
   }
-  DevStatus h;
   const ptc_status rc = end_call(L.st, s, &h);
   *n_distinct_host_out = n ? h.value[0] : 0;
+  if (n_used_host_out) *n_used_host_out = n ? h.value[1] : 0;
   return rc;
+}
+
+extern "C" ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t* ids_out, uint64_t* n_distinct_host_out,
+                                     void* ws, size_t ws_bytes, void* stream) {
+  return ptc::ids_impl(keys, n, nullptr, ids_out, nullptr, n_distinct_host_out, ws, ws_bytes, (cudaStream_t)stream,
+                       nullptr, 0);
 }
 
 extern "C" size_t ptc_verify_ids_workspace_bytes(uint64_t n, uint64_t n_distinct) {

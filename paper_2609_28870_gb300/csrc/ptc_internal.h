@@ -107,7 +107,11 @@ inline ptc_status end_call(const DevStatus* dev, cudaStream_t stream, DevStatus*
 
 // Instead of waiting for a call's status, queue a copy of its error word to
 // `slot`, for a later call that does wait to fold in (ptc_pipeline).
-ptc_status defer_status(const DevStatus* dev, uint32_t* slot, cudaStream_t stream);
+// OR the n (at most 32) deferred error words at `err` into st->err.
+ptc_status carry_errors(const uint32_t* err, uint32_t n, DevStatus* st, cudaStream_t s);
+// With `value_slot`, value[value_index] of the status block is copied there too.
+ptc_status defer_status(const DevStatus* dev, uint32_t* slot, cudaStream_t stream, uint64_t* value_slot = nullptr,
+                        uint32_t value_index = 0);
 
 // Streaming multiprocessors of the current device (persistent grids).
 inline int num_sms() {
@@ -131,6 +135,19 @@ struct RunsView {
   const uint32_t* bits = nullptr;   // run-start bitmap, one word per 32 accesses
   const uint32_t* wpre = nullptr;   // runs starting before each word
 };
+// Stage a1 (ptc_hash.cu).  With `n_slot` and `err_slot` (device memory) the
+// final wait is replaced by defer_status: N goes to *n_slot, the error word
+// to *err_slot, and *n_access_host_out is left 0.
+ptc_status hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off, const int64_t* req_ts_us,
+                     uint32_t n_req, uint32_t block_size, uint64_t seed, ptc_u128* keys_out, uint64_t keys_cap,
+                     uint64_t* req_blk_off_out, uint64_t* n_access_host_out, void* ws, size_t ws_bytes,
+                     cudaStream_t s, uint64_t* n_slot, uint32_t* err_slot);
+// Stage a2 (ptc_ids.cu) over n_ub keys, of which the first min(*n_dev, n_ub)
+// are used when `n_dev` (device memory) is given.  Error words at
+// `carry_err` join the call's own.  Reports the number used and D.
+ptc_status ids_impl(const ptc_u128* keys, uint64_t n_ub, const uint64_t* n_dev, uint32_t* ids_out,
+                    uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
+                    cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry);
 ptc_status stack_distance_view(const uint32_t* prev, uint64_t n, uint32_t* dist_out, int method, void* ws,
                                size_t ws_bytes, cudaStream_t s, RunsView* view, uint32_t* defer_err);
 // Stage b as ptc_reuse_indices does it (ptc_reuse.cu); with `defer_err` the

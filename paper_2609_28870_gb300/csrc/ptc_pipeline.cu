@@ -17,7 +17,8 @@ struct PipeLayout {
   size_t scratch_bytes;
   void* curves;
   size_t curves_bytes;
-  uint32_t* defer;  // error words of stages b and c, read with stage d's
+  uint32_t* defer;  // error words of stages a1, b and c, read with a later stage's
+  uint64_t* n_slot;  // N as stage a1 left it, for stage a2
   size_t total;
 };
 
@@ -45,7 +46,8 @@ PipeLayout pipe_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   L.scratch = cv.take<unsigned char>(L.scratch_bytes);
   L.curves_bytes = ptc_curves_workspace_bytes(n_tok / B, n_req, n_cap);
   L.curves = cv.take<unsigned char>(L.curves_bytes);
-  L.defer = cv.take<uint32_t>(2);
+  L.defer = cv.take<uint32_t>(3);
+  L.n_slot = cv.take<uint64_t>(1);
   L.total = cv.bytes();
   return L;
 }
@@ -79,25 +81,28 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
   uint32_t* next = next_out ? next_out : L.next;
   uint32_t* dist = dist_out ? dist_out : L.dist;
   const uint64_t cap = n_tok / block_size ? n_tok / block_size : 1;
-  uint64_t n = 0, d = 0;
-  ptc_status rc = ptc_hash_blocks(tokens, n_tok, req_tok_off, req_ts_us, n_req, block_size, seed, keys, cap, blk, &n,
-                                  L.scratch, L.scratch_bytes, stream);
-  *n_access_host_out = n;
+  uint64_t n = 0, d = 0, unused = 0;
+  *n_access_host_out = 0;
   *n_distinct_host_out = 0;
+  cudaStream_t s = (cudaStream_t)stream;
+  // Stages a1, b and c do not wait for their own status: a1's error word and
+  // N go to device slots that stage a2 reads (its grids cover N's upper
+  // bound, n_tok / B); b's and c's error words are read with stage d's.
+  if (ptc::fill_async(L.defer, 0u, 3 * sizeof(uint32_t), s) != PTC_OK) return PTC_ERR_CUDA;
+  ptc_status rc = ptc::hash_impl(tokens, n_tok, req_tok_off, req_ts_us, n_req, block_size, seed, keys, cap, blk,
+                                 &unused, L.scratch, L.scratch_bytes, s, L.n_slot, &L.defer[0]);
   if (rc != PTC_OK) return rc;
-  rc = ptc_assign_ids(keys, n, ids, &d, L.scratch, L.scratch_bytes, stream);
+  rc = ptc::ids_impl(keys, cap, L.n_slot, ids, &n, &d, L.scratch, L.scratch_bytes, s, &L.defer[0], 1);
+  *n_access_host_out = n;
   *n_distinct_host_out = d;
   if (rc != PTC_OK) return rc;
-  // stages b and c do not wait for their own status: stage d reads it
-  cudaStream_t s = (cudaStream_t)stream;
-  if (ptc::fill_async(L.defer, 0u, 2 * sizeof(uint32_t), s) != PTC_OK) return PTC_ERR_CUDA;
   ptc::RunsView runs;
   if (n > 0) {
-    rc = ptc::reuse_view(ids, n, d, prev, next, L.scratch, L.scratch_bytes, s, &L.defer[0]);
+    rc = ptc::reuse_view(ids, n, d, prev, next, L.scratch, L.scratch_bytes, s, &L.defer[1]);
     if (rc != PTC_OK) return rc;
-    rc = ptc::stack_distance_view(prev, n, dist, PTC_SD_AUTO, L.scratch, L.scratch_bytes, s, &runs, &L.defer[1]);
+    rc = ptc::stack_distance_view(prev, n, dist, PTC_SD_AUTO, L.scratch, L.scratch_bytes, s, &runs, &L.defer[2]);
     if (rc != PTC_OK) return rc;
   }
   return ptc::curves_impl(dist, n, blk, n_req, block_size, cm, cap_host, n_cap, hits_host_out, saved_host_out,
-                          total_cost_host_out, L.curves, L.curves_bytes, s, &runs, L.defer, 2);
+                          total_cost_host_out, L.curves, L.curves_bytes, s, &runs, &L.defer[1], 2);
 }

@@ -113,3 +113,29 @@ def test_pipeline_rejects_bad_arguments():
                         hits.ctypes.data, saved.ctypes.data, ctypes.byref(total), small.data_ptr(), 256,
                         torch.cuda.current_stream().cuda_stream)
     assert ptc.STATUS[rc] == "PTC_ERR_WORKSPACE"
+
+
+def test_pipeline_reports_stage_a1_errors():
+    """Stage a1 does not wait for its own status inside ptc_pipeline: its
+    error word reaches the caller through stage a2's wait, and stage a2 must
+    stay inside the keys buffer whatever N stage a1 left."""
+    import paper_2609_28870_gb300 as ptc
+    from tests import gpu_util as gu
+    tr = tracegen.tiny(1, n_sessions=4)
+    tok, off, ts = gu.to_gpu(tr)
+    bad_off = off.clone()
+    bad_off[-1] = tr.tokens.size + 100  # the last request runs past the tokens
+    with pytest.raises(ptc.PtcError) as e:
+        ptc.ptc_pipeline(tok, bad_off, ts, 2, [1, 2])
+    assert e.value.name == "PTC_ERR_INVALID_ARG"
+    bad_ts = ts.flip(0).contiguous()
+    with pytest.raises(ptc.PtcError) as e:
+        ptc.ptc_pipeline(tok, off, bad_ts, 2, [1, 2])
+    assert e.value.name == "PTC_ERR_UNSORTED"
+    bad_off = off.clone()
+    bad_off[1] = bad_off[2] + 5  # offsets that go backwards
+    with pytest.raises(ptc.PtcError) as e:
+        ptc.ptc_pipeline(tok, bad_off, ts, 2, [1, 2])
+    assert e.value.name == "PTC_ERR_INVALID_ARG"
+    # and a good call afterwards still matches the oracle (nothing stale in the slots)
+    gu.assert_same(_run(tr, 2, [1, 2]), gu.oracle_run(tr, 2, [1, 2]))
