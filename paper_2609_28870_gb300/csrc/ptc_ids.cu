@@ -57,30 +57,22 @@ __device__ __forceinline__ uint32_t keys_used(uint32_t n, const uint64_t* n_dev)
   return v < n ? (uint32_t)v : n;
 }
 
-__global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __restrict__ keys, uint32_t n_ub,
-                                                            const uint64_t* n_dev, ulonglong2* table, uint32_t log2m,
-                                                            uint64_t probe_cap, uint32_t* __restrict__ slot_of,
-                                                            DevStatus* st) {
-  grid_dep_sync();
-  const uint32_t i = blockIdx.x * kInsThreads + threadIdx.x;
-  if (i >= keys_used(n_ub, n_dev)) return;
-  const ulonglong2 k = __ldcs(&keys[i]);  // streamed once: keep L2 for the table
-  if (k.x >= kP61 || k.y >= kP61) {
-    raise_err(st, kErrInvalid);
-    slot_of[i] = 0;
-    return;
-  }
-  // 96 key bits: all of h0 (61) + 35 bits of h1.  Word 0 is never all-ones
-  // because h0 < 2^61 - 1, and word 1 of a filled slot holds an index below
-  // 2^32 - 1, so an all-ones word marks an empty or half-written slot.
+constexpr int kInsK = 1;  // keys per thread: their key and slot loads are in flight together
+
+// Settle the key k of access i, whose home slot `pos` was read as `cur`:
+// claim an empty (or half-written) slot with one 128-bit CAS, or find the
+// key's slot and lower its stored index to i if it is above; linear probing.
+// 96 key bits: all of h0 (61) + 35 bits of h1.  Word 0 is never all-ones
+// because h0 < 2^61 - 1, and word 1 of a filled slot holds an index below
+// 2^32 - 1, so an all-ones word marks an empty or half-written slot.
+__device__ __forceinline__ void settle(ulonglong2* table, uint64_t mask, uint64_t probe_cap, uint32_t i,
+                                       ulonglong2 k, uint64_t pos, ulonglong2 cur, uint32_t* __restrict__ slot_of,
+                                       DevStatus* st) {
   const uint64_t w0 = k.x | ((k.y & 7ULL) << 61);
   const uint32_t w1lo = (uint32_t)(k.y >> 3);
   const ulonglong2 mine = make_ulonglong2(w0, (uint64_t)w1lo | ((uint64_t)i << 32));
   const ulonglong2 empty = make_ulonglong2(~0ULL, ~0ULL);
-  const uint64_t mask = (1ULL << log2m) - 1;
-  uint64_t pos = home_slot(k.x, k.y, log2m);
-  for (uint64_t probe = 0; probe <= mask && probe < probe_cap; ++probe) {
-    ulonglong2 cur = ld_slot(&table[pos]);
+  for (uint64_t probe = 0;;) {
     if (cur.x == ~0ULL || cur.y == ~0ULL) {  // empty, or being filled: settle it with the CAS
       cur = cas128(&table[pos], empty, mine);
       if (cur.x == ~0ULL && cur.y == ~0ULL) {
@@ -93,10 +85,47 @@ __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __
       __stcs(&slot_of[i], (uint32_t)pos);
       return;
     }
+    if (++probe > mask || probe >= probe_cap) break;
     pos = (pos + 1) & mask;
+    cur = ld_slot(&table[pos]);
   }
   raise_err(st, kErrTableFull);
   slot_of[i] = 0;
+}
+
+// kInsK keys per thread, kInsThreads apart: all their key loads, then all
+// their home-slot loads, go out before any is settled.
+__global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __restrict__ keys, uint32_t n_ub,
+                                                            const uint64_t* n_dev, ulonglong2* table, uint32_t log2m,
+                                                            uint64_t probe_cap, uint32_t* __restrict__ slot_of,
+                                                            DevStatus* st) {
+  grid_dep_sync();
+  const uint32_t n = keys_used(n_ub, n_dev);
+  const uint32_t i0 = blockIdx.x * (kInsThreads * kInsK) + threadIdx.x;
+  const uint64_t mask = (1ULL << log2m) - 1;
+  ulonglong2 k[kInsK], cur[kInsK];
+  uint64_t pos[kInsK];
+#pragma unroll
+  for (int j = 0; j < kInsK; ++j) {
+    const uint32_t i = i0 + j * kInsThreads;
+    k[j] = i < n ? __ldcs(&keys[i]) : make_ulonglong2(~0ULL, ~0ULL);  // streamed once: keep L2 for the table
+  }
+#pragma unroll
+  for (int j = 0; j < kInsK; ++j) {
+    pos[j] = home_slot(k[j].x, k[j].y, log2m);
+    cur[j] = k[j].x < kP61 && k[j].y < kP61 ? ld_slot(&table[pos[j]]) : make_ulonglong2(0, 0);
+  }
+#pragma unroll
+  for (int j = 0; j < kInsK; ++j) {
+    const uint32_t i = i0 + j * kInsThreads;
+    if (i >= n) continue;
+    if (k[j].x >= kP61 || k[j].y >= kP61) {
+      raise_err(st, kErrInvalid);
+      slot_of[i] = 0;
+      continue;
+    }
+    settle(table, mask, probe_cap, i, k[j], pos[j], cur[j], slot_of, st);
+  }
 }
 
 constexpr int kFlT = 256;             // flags: threads per tile
@@ -345,7 +374,7 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
     if (fill_async(L.table, ~0u, sizeof(ulonglong2) << log2m, s) != PTC_OK) return false;
     const ulonglong2* k = reinterpret_cast<const ulonglong2*>(keys);
     const uint32_t n32 = (uint32_t)n;
-    PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads), kInsThreads, 0, k, n32, n_dev, L.table,
+    PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads * kInsK), kInsThreads, 0, k, n32, n_dev, L.table,
                log2m, probe_cap, L.slot_of, L.st);
     PTC_KERNEL("k_ids_flags", s, k_ids_flags, L.ntiles, kFlT, 0, L.table, L.slot_of, n32, n_dev, L.ntiles, L.bits,
                L.tcnt, L.tpre, &L.done[0], L.st);
