@@ -46,17 +46,16 @@ constexpr uint32_t kSpinCap = 1u << 20;
 
 __device__ __forceinline__ void raise_err(DevStatus* st, uint32_t f) { atomicOr(&st->err, f); }
 
-// Programmatic dependent launch.  Kernels are launched so that their CTAs may
-// be scheduled while the previous kernel on the stream is still finishing;
-// every kernel calls this first, before it touches global memory: it waits
-// until that kernel has completed and its writes are visible (a no-op for a
-// launch without the attribute), then lets the next kernel be scheduled in
-// turn.  Because each kernel waits for its predecessor before it lets its own
-// dependent start, the chain stays ordered end to end.
-__device__ __forceinline__ void grid_dep_sync() {
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
+// Programmatic dependent launch.  Kernels are launched so that the next one
+// on the stream is set up while the previous one is still running; every
+// kernel calls this first, before it touches global memory: it waits until
+// the previous kernel has completed and its writes are visible (a no-op for a
+// launch without the attribute).  No kernel signals early completion
+// (griddepcontrol.launch_dependents): measured over the whole pipeline,
+// letting the next grid's CTAs in while the last wave of many short CTAs
+// still runs cost more than it saved.  Each kernel waits for its predecessor,
+// so the chain stays ordered end to end.
+__device__ __forceinline__ void grid_dep_sync() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 __device__ __forceinline__ uint32_t next_tile(DevStatus* st, int epoch) {
   __shared__ uint32_t s_tile;
