@@ -93,6 +93,66 @@ __device__ __forceinline__ uint64_t warp_sum_u64(uint64_t v) {
 }
 
 // ---------------------------------------------------------------------------
+// Exclusive prefix of the per-tile counts cnt[0, T) into pre[0, T), with
+// pre[T] = the total, which it also returns.  Run by every thread of ONE CTA
+// (the last of a grid to finish, after last-CTA fencing; blockDim.x a
+// multiple of 32).  Warp w owns a contiguous range of rows of 32 tiles and
+// reads kTpRows rows per round with coalesced loads that are all in flight
+// together, so the scan costs a few memory round trips rather than one per
+// tile and thread.
+// ---------------------------------------------------------------------------
+constexpr int kTpRows = 8;
+__device__ inline uint32_t cta_tiles_prefix(const uint32_t* cnt, uint32_t* pre, uint32_t T) {
+  __shared__ uint32_t s_tp[32];
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const uint32_t rows = (T + 31) / 32, rpw = (rows + nw - 1) / nw;
+  const uint32_t r0 = w * rpw < rows ? w * rpw : rows, r1 = r0 + rpw < rows ? r0 + rpw : rows;
+  uint32_t sum = 0;
+  for (uint32_t r = r0; r < r1; r += kTpRows) {
+    uint32_t v[kTpRows];
+#pragma unroll
+    for (int u = 0; u < kTpRows; ++u) {
+      const uint32_t t = (r + u) * 32 + lane;
+      v[u] = (r + u < r1 && t < T) ? __ldcg(&cnt[t]) : 0u;
+    }
+#pragma unroll
+    for (int u = 0; u < kTpRows; ++u) sum += v[u];
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(kFull, sum, o);
+  if (lane == 0) s_tp[w] = sum;
+  __syncthreads();
+  uint32_t base = 0, total = 0;
+  for (uint32_t i = 0; i < nw; ++i) {
+    const uint32_t x = s_tp[i];
+    if (i < w) base += x;
+    total += x;
+  }
+  for (uint32_t r = r0; r < r1; r += kTpRows) {
+    uint32_t v[kTpRows];
+#pragma unroll
+    for (int u = 0; u < kTpRows; ++u) {
+      const uint32_t t = (r + u) * 32 + lane;
+      v[u] = (r + u < r1 && t < T) ? __ldcg(&cnt[t]) : 0u;
+    }
+#pragma unroll
+    for (int u = 0; u < kTpRows; ++u) {
+      uint32_t incl = v[u];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(kFull, incl, o);
+        if (lane >= (uint32_t)o) incl += y;
+      }
+      const uint32_t t = (r + u) * 32 + lane;
+      if (r + u < r1 && t < T) pre[t] = base + incl - v[u];
+      base += __shfl_sync(kFull, incl, 31);
+    }
+  }
+  if (threadIdx.x == 0) pre[T] = total;
+  return total;
+}
+
+// ---------------------------------------------------------------------------
 // Packed look-back for sums below 2^56: word = epoch(6) | flag(2) | value(56).
 // flag 1 = aggregate, 2 = inclusive prefix.  Called by all 32 lanes of ONE
 // warp; returns the exclusive prefix of `tile` (0 if the wait gave up, with

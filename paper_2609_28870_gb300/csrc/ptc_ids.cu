@@ -181,30 +181,8 @@ __global__ void __launch_bounds__(kFlT) k_ids_flags(const ulonglong2* __restrict
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  const uint32_t per = (ntiles + kFlT - 1) / kFlT;
-  const uint32_t t0 = threadIdx.x * per, t1 = min(t0 + per, ntiles);
-  uint32_t sum = 0;
-  for (uint32_t t = t0; t < t1; ++t) sum += __ldcg(&tcnt[t]);
-  uint32_t incl = sum;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t y = __shfl_up_sync(kFull, incl, o);
-    if (lane >= (uint32_t)o) incl += y;
-  }
-  __syncthreads();
-  if (lane == 31) s_w[w] = incl;
-  __syncthreads();
-  uint32_t run = incl - sum, total = 0;
-  for (int ww = 0; ww < kFlT / 32; ++ww) {
-    if (ww < (int)w) run += s_w[ww];
-    total += s_w[ww];
-  }
-  for (uint32_t t = t0; t < t1; ++t) {
-    tpre[t] = run;
-    run += __ldcg(&tcnt[t]);
-  }
+  const uint32_t total = cta_tiles_prefix(tcnt, tpre, ntiles);
   if (threadIdx.x == 0) {
-    tpre[ntiles] = total;
     st->value[0] = total;
     st->value[1] = n_dev ? *n_dev : n;
     if (n_dev && *n_dev > n_ub) raise_err(st, kErrInvalid);  // more blocks than the keys buffer holds
@@ -234,15 +212,34 @@ __global__ void k_ids_wordpre(const uint32_t* __restrict__ bits, const uint32_t*
   }
 }
 
-__global__ void k_ids_gather(const uint32_t* __restrict__ first, const uint32_t* __restrict__ bits,
-                             const uint32_t* __restrict__ wpre, uint32_t n_ub, const uint64_t* n_dev,
-                             uint32_t* __restrict__ ids) {
+// kGaPer accesses per thread, kGaThreads apart, their loads in flight together.
+constexpr int kGaThreads = 256;
+constexpr int kGaPer = 8;
+__global__ void __launch_bounds__(kGaThreads) k_ids_gather(const uint32_t* __restrict__ first,
+                                                          const uint32_t* __restrict__ bits,
+                                                          const uint32_t* __restrict__ wpre, uint32_t n_ub,
+                                                          const uint64_t* n_dev, uint32_t* __restrict__ ids) {
   grid_dep_sync();
-  const uint32_t i = blockIdx.x * blockDim.x + threadIdx.x;
   const uint32_t n = keys_used(n_ub, n_dev);
-  if (i >= n) return;
-  const uint32_t f = __ldcs(&first[i]);
-  ids[i] = f < n ? wpre[f >> 5] + __popc(bits[f >> 5] & ((1u << (f & 31)) - 1u)) : kNone;
+  const uint32_t i0 = blockIdx.x * (kGaThreads * kGaPer) + threadIdx.x;
+  uint32_t f[kGaPer];
+#pragma unroll
+  for (int k = 0; k < kGaPer; ++k) {
+    const uint32_t i = i0 + k * kGaThreads;
+    f[k] = i < n ? __ldcs(&first[i]) : kNone;
+  }
+  uint32_t wp[kGaPer], bw[kGaPer];
+#pragma unroll
+  for (int k = 0; k < kGaPer; ++k) {
+    const bool ok = f[k] < n;
+    wp[k] = ok ? wpre[f[k] >> 5] : 0u;
+    bw[k] = ok ? bits[f[k] >> 5] : 0u;
+  }
+#pragma unroll
+  for (int k = 0; k < kGaPer; ++k) {
+    const uint32_t i = i0 + k * kGaThreads;
+    if (i < n) ids[i] = f[k] < n ? wp[k] + __popc(bw[k] & ((1u << (f[k] & 31)) - 1u)) : kNone;
+  }
 }
 
 // Slots for n keys at most: the full table holds 1.5 n; the first attempt
@@ -380,7 +377,7 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
                L.tcnt, L.tpre, &L.done[0], L.st);
     PTC_KERNEL("k_ids_wordpre", s, k_ids_wordpre, ceil_div_u32((uint64_t)L.ntiles * 32, 256), 256, 0, L.bits, L.tpre,
                L.nwords, L.wpre);
-    PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, 256), 256, 0, L.slot_of, L.bits, L.wpre, n32, n_dev,
+    PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of, L.bits, L.wpre, n32, n_dev,
                ids_out);
     return true;
   };

@@ -88,18 +88,8 @@ __device__ __forceinline__ bool last_cta(uint32_t* done) {
 
 // Run by the last CTA: exclusive prefix of cnt[0..T) into pre, pre[T] = total.
 __device__ uint32_t tiles_prefix(const uint32_t* cnt, uint32_t* pre, uint32_t T, uint32_t* s_w) {
-  const uint32_t per = (T + kIT - 1) / kIT;
-  const uint32_t t0 = threadIdx.x * per, t1 = min(t0 + per, T);
-  uint32_t sum = 0;
-  for (uint32_t t = t0; t < t1; ++t) sum += __ldcg(&cnt[t]);
-  uint32_t total;
-  uint32_t run = cta_excl_u32(sum, s_w, &total);
-  for (uint32_t t = t0; t < t1; ++t) {
-    pre[t] = run;
-    run += __ldcg(&cnt[t]);
-  }
-  if (threadIdx.x == 0) pre[T] = total;
-  return total;
+  (void)s_w;
+  return cta_tiles_prefix(cnt, pre, T);
 }
 
 // Id-run starts of the warp's 8 x 32 positions from `base`, with the id left

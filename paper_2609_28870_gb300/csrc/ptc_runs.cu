@@ -115,7 +115,6 @@ __device__ __forceinline__ bool last_cta(uint32_t* done) {
 __global__ void __launch_bounds__(kMT) k_runs_count(MarkArgs a) {
   grid_dep_sync();
   __shared__ uint32_t s_wcnt[kMT / 32];
-  __shared__ uint32_t s_scan[kMT / 32];
   const uint32_t tile = blockIdx.x;
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   uint32_t pv[kMR], words[kMR];
@@ -133,32 +132,8 @@ __global__ void __launch_bounds__(kMT) k_runs_count(MarkArgs a) {
     a.tcnt[tile] = t;
   }
   if (!last_cta(a.done)) return;
-  // exclusive prefix of the tile counts
-  const uint32_t T = a.ntiles, per = (T + kMT - 1) / kMT;
-  const uint32_t t0 = threadIdx.x * per, t1 = min(t0 + per, T);
-  uint32_t sum = 0;
-  for (uint32_t t = t0; t < t1; ++t) sum += __ldcg(&a.tcnt[t]);
-  uint32_t incl = sum;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t y = __shfl_up_sync(kFull, incl, o);
-    if (lane >= (uint32_t)o) incl += y;
-  }
-  if (lane == 31) s_scan[w] = incl;
-  __syncthreads();
-  uint32_t run = incl - sum, total = 0;
-  for (int ww = 0; ww < kMT / 32; ++ww) {
-    if (ww < (int)w) run += s_scan[ww];
-    total += s_scan[ww];
-  }
-  for (uint32_t t = t0; t < t1; ++t) {
-    a.tpre[t] = run;
-    run += __ldcg(&a.tcnt[t]);
-  }
-  if (threadIdx.x == 0) {
-    a.tpre[T] = total;
-    a.st->value[1] = total;
-  }
+  const uint32_t total = cta_tiles_prefix(a.tcnt, a.tpre, a.ntiles);  // exclusive prefix of the tile counts
+  if (threadIdx.x == 0) a.st->value[1] = total;
 }
 
 // Pass 2: bitmap, run index per word, and the (start, first value) records.
@@ -596,13 +571,27 @@ __global__ void __launch_bounds__(256) k_runs_query(QueryArgs a) {
   a.sd[r] = 1u + partial + cnt;
 }
 
-__global__ void __launch_bounds__(256) k_runs_expand(const uint32_t* __restrict__ bits,
-                                                    const uint32_t* __restrict__ wpre, const uint32_t* __restrict__ sd,
-                                                    uint32_t n, uint32_t* __restrict__ dist) {
+// kExpPer accesses per thread, kExpThreads apart: each thread's dependent
+// loads (word, then distance) for all of them are in flight together.
+constexpr int kExpThreads = 256;
+constexpr int kExpPer = 8;
+__global__ void __launch_bounds__(kExpThreads) k_runs_expand(const uint32_t* __restrict__ bits,
+                                                            const uint32_t* __restrict__ wpre,
+                                                            const uint32_t* __restrict__ sd, uint32_t n,
+                                                            uint32_t* __restrict__ dist) {
   grid_dep_sync();
-  const uint32_t j = blockIdx.x * blockDim.x + threadIdx.x;
-  if (j >= n) return;
-  dist[j] = sd[run_of(bits, wpre, j)];
+  const uint32_t j0 = blockIdx.x * (kExpThreads * kExpPer) + threadIdx.x;
+  uint32_t r[kExpPer];
+#pragma unroll
+  for (int k = 0; k < kExpPer; ++k) {
+    const uint32_t j = j0 + k * kExpThreads;
+    r[k] = j < n ? run_of(bits, wpre, j) : 0u;
+  }
+#pragma unroll
+  for (int k = 0; k < kExpPer; ++k) {
+    const uint32_t j = j0 + k * kExpThreads;
+    if (j < n) __stcs(&dist[j], __ldg(&sd[r[k]]));
+  }
 }
 
 uint32_t key_bits_n(uint64_t n) {  // keys and thresholds lie in [0, n]
@@ -791,7 +780,7 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   q.R = R32;
   q.L = L;
   PTC_KERNEL("k_runs_query", s, k_runs_query, ceil_div_u32(R, 256), 256, 0, q);
-  PTC_KERNEL("k_runs_expand", s, k_runs_expand, ceil_div_u32(n, 256), 256, 0, W.bits, W.wpre, W.sd, (uint32_t)n, dist_out);
+  PTC_KERNEL("k_runs_expand", s, k_runs_expand, ceil_div_u32(n, kExpThreads * kExpPer), kExpThreads, 0, W.bits, W.wpre, W.sd, (uint32_t)n, dist_out);
   const ptc_status done = defer_err ? defer_status(W.st, defer_err, s) : end_call(W.st, s, &h);
   if (done == PTC_OK && view) {
     view->used = true;
