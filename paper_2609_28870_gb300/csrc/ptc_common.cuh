@@ -183,7 +183,11 @@ __device__ inline uint64_t lookback_sum(uint64_t* words, uint32_t tile, uint64_t
       f = ((uint32_t)(w >> 58) == epoch) ? (uint32_t)((w >> 56) & 3) : 0u;
       v = w & kLbValMask;
     }
-    if (__any_sync(kFull, f == 0)) {
+    // only the tiles after the nearest published prefix must be ready
+    const uint32_t incl = __ballot_sync(kFull, f == 2);
+    const uint32_t first = incl ? (uint32_t)(__ffs(incl) - 1) : 31u;
+    const uint32_t upto = first == 31u ? kFull : ((2u << first) - 1u);
+    if (__ballot_sync(kFull, f == 0) & upto) {
       if (++spins > kSpinCap) {
         if (lane == 0) raise_err(st, kErrTimeout);
         return 0;
@@ -192,9 +196,7 @@ __device__ inline uint64_t lookback_sum(uint64_t* words, uint32_t tile, uint64_t
       if (ns < 1000) ns += ns;
       continue;
     }
-    uint32_t incl = __ballot_sync(kFull, f == 2);
     if (incl) {
-      uint32_t first = __ffs(incl) - 1;
       if (lane > first) v = 0;
       excl += warp_sum_u64(v);
       break;
@@ -393,7 +395,13 @@ __device__ inline uint64_t lookback_sum_cta(uint64_t* words, uint32_t tile, uint
       f = ((uint32_t)(wv >> 58) == epoch) ? (uint32_t)((wv >> 56) & 3) : 0u;
       v = wv & kLbValMask;
     }
-    if (__syncthreads_or(f == 0)) {
+    // the nearest published prefix; only the tiles after it must be ready
+    if (t == 0) s_first = 0xFFFFFFFFu;
+    __syncthreads();
+    if (f == 2) atomicMin(&s_first, t);
+    __syncthreads();
+    const uint32_t first = s_first;
+    if (__syncthreads_or(f == 0 && t < first)) {
       if (++spins > kSpinCap) {
         if (t == 0) {
           raise_err(st, kErrTimeout);
@@ -405,11 +413,6 @@ __device__ inline uint64_t lookback_sum_cta(uint64_t* words, uint32_t tile, uint
       if (ns < 500) ns += ns;
       continue;
     }
-    if (t == 0) s_first = 0xFFFFFFFFu;
-    __syncthreads();
-    if (f == 2) atomicMin(&s_first, t);
-    __syncthreads();
-    const uint32_t first = s_first;
     if (t > first) v = 0;
     v = warp_sum_u64(v);
     if (lane == 0) s_part[wid] = v;

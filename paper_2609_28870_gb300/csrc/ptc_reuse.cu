@@ -33,8 +33,8 @@ namespace ptc {
 namespace {
 
 constexpr int kIT = 256;            // threads per tile
-constexpr int kIR = 8;              // rounds of 32 positions per warp
-constexpr int kITile = kIT * kIR;   // 2048 positions; warp w owns [256 w, 256 w + 256)
+constexpr int kIR = 16;             // rounds of 32 positions per warp
+constexpr int kITile = kIT * kIR;   // 4096 positions; warp w owns [512 w, 512 w + 512)
 constexpr int kBmPer = 4;           // bitmap words per thread
 constexpr int kBmTile = kIT * kBmPer;
 constexpr int kRunPer = 8;          // runs per thread in the incidence kernels

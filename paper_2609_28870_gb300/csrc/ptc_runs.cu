@@ -53,8 +53,8 @@ namespace ptc {
 namespace {
 
 constexpr int kMT = 256;           // run marking: threads per tile
-constexpr int kMR = 8;             // rounds of 32 positions per warp
-constexpr int kMTile = kMT * kMR;  // 2048 positions; warp w owns [256 w, 256 w + 256)
+constexpr int kMR = 16;            // rounds of 32 positions per warp
+constexpr int kMTile = kMT * kMR;  // 4096 positions; warp w owns [512 w, 512 w + 512)
 constexpr int kRT = 256;           // level tiles: threads
 constexpr int kRPer = 8;           // runs per thread (consecutive)
 constexpr int kRTile = kRT * kRPer;
