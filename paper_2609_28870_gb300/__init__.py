@@ -318,30 +318,59 @@ def pipeline(tokens, req_tok_off, req_ts_us, block_size: int, caps_for, kind: in
     return out
 
 
+class PipelinePlan:
+    """ptc_pipeline with its arguments marshalled once, for running the same
+    call again and again (a serving loop, a benchmark): ``run()`` is one C
+    call.  The device tensors given here are read at every run, so a new
+    trace of the same shape is run by refilling them in place.  The stream is
+    the current stream of the tensors' device when the plan is made.
+    ``outputs`` may map any of keys / req_blk_off / ids / prev / next / dist to
+    preallocated CUDA tensors that receive those arrays.  After ``run()``,
+    ``hits`` (uint64, one per capacity) and ``saved`` (uint64 pairs lo, hi)
+    hold the curves, and ``result()`` converts them as ptc_pipeline returns
+    them."""
+
+    def __init__(self, tokens, req_tok_off, req_ts_us, block_size: int, caps, kind: int = PTC_COST_MEASURED,
+                 seed: int = 0, f_lin: int = F_LIN, f_attn: int = F_ATTN, ws: torch.Tensor | None = None,
+                 outputs: dict | None = None):
+        dev = _dev(req_tok_off)
+        n_req = req_tok_off.numel() - 1
+        n_tok = tokens.numel()
+        self.caps = np.ascontiguousarray(caps, dtype=np.uint64)
+        G = self.caps.shape[0]
+        self.ws = _workspace(lib().ptc_pipeline_workspace_bytes(n_req, n_tok, block_size, G), dev, ws)
+        o = outputs or {}
+        self.hits = np.zeros(G, dtype=np.uint64)
+        self.saved = np.zeros(2 * G, dtype=np.uint64)
+        self.total = U128()
+        self.n, self.d = ctypes.c_uint64(0), ctypes.c_uint64(0)
+        self.cm = CostModel(int(f_lin), int(f_attn), int(kind))
+        self._keep = (tokens, req_tok_off, req_ts_us, o)  # the pointers below stay valid
+        self._fn = lib().ptc_pipeline
+        self._args = (_ptr(tokens), n_tok, _ptr(req_tok_off), _ptr(req_ts_us), n_req, block_size,
+                      int(seed) & (2**64 - 1), ctypes.byref(self.cm), self.caps.ctypes.data, G, _ptr(o.get("keys")),
+                      _ptr(o.get("req_blk_off")), _ptr(o.get("ids")), _ptr(o.get("prev")), _ptr(o.get("next")),
+                      _ptr(o.get("dist")), ctypes.byref(self.n), ctypes.byref(self.d), self.hits.ctypes.data,
+                      self.saved.ctypes.data, ctypes.byref(self.total), _ptr(self.ws), self.ws.numel(), _stream(dev))
+
+    def run(self) -> "PipelinePlan":
+        rc = self._fn(*self._args)
+        if rc != 0:
+            raise PtcError("ptc_pipeline", rc)
+        return self
+
+    def result(self) -> dict:
+        G = self.hits.shape[0]
+        return {"n_access": int(self.n.value), "n_distinct": int(self.d.value), "hits": [int(h) for h in self.hits],
+                "saved": [int(self.saved[2 * g + 1]) << 64 | int(self.saved[2 * g]) for g in range(G)],
+                "total_cost": int(self.total.hi) << 64 | int(self.total.lo)}
+
+
 def ptc_pipeline(tokens, req_tok_off, req_ts_us, block_size: int, caps, kind: int = PTC_COST_MEASURED, seed: int = 0,
                  f_lin: int = F_LIN, f_attn: int = F_ATTN, ws: torch.Tensor | None = None, outputs: dict | None = None):
     """All five stages in one C call (trace already on the GPU).  ``outputs``
     may map any of keys / req_blk_off / ids / prev / next / dist to
     preallocated CUDA tensors that receive those arrays.  Returns the curves
     with N and D."""
-    dev = _dev(req_tok_off)
-    n_req = req_tok_off.numel() - 1
-    n_tok = tokens.numel()
-    caps = np.ascontiguousarray(caps, dtype=np.uint64)
-    G = caps.shape[0]
-    w = _workspace(lib().ptc_pipeline_workspace_bytes(n_req, n_tok, block_size, G), dev, ws)
-    o = outputs or {}
-    hits = np.zeros(G, dtype=np.uint64)
-    saved = np.zeros(2 * G, dtype=np.uint64)
-    total = U128()
-    n, d = ctypes.c_uint64(0), ctypes.c_uint64(0)
-    cm = CostModel(int(f_lin), int(f_attn), int(kind))
-    rc = lib().ptc_pipeline(_ptr(tokens), n_tok, _ptr(req_tok_off), _ptr(req_ts_us), n_req, block_size,
-                            int(seed) & (2**64 - 1), ctypes.byref(cm), caps.ctypes.data, G, _ptr(o.get("keys")),
-                            _ptr(o.get("req_blk_off")), _ptr(o.get("ids")), _ptr(o.get("prev")), _ptr(o.get("next")),
-                            _ptr(o.get("dist")), ctypes.byref(n), ctypes.byref(d), hits.ctypes.data,
-                            saved.ctypes.data, ctypes.byref(total), _ptr(w), w.numel(), _stream(dev))
-    _check("ptc_pipeline", rc)
-    return {"n_access": int(n.value), "n_distinct": int(d.value), "hits": [int(h) for h in hits],
-            "saved": [int(saved[2 * g + 1]) << 64 | int(saved[2 * g]) for g in range(G)],
-            "total_cost": int(total.hi) << 64 | int(total.lo)}
+    return PipelinePlan(tokens, req_tok_off, req_ts_us, block_size, caps, kind, seed, f_lin, f_attn, ws,
+                        outputs).run().result()

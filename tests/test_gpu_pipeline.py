@@ -139,3 +139,31 @@ def test_pipeline_reports_stage_a1_errors():
     assert e.value.name == "PTC_ERR_INVALID_ARG"
     # and a good call afterwards still matches the oracle (nothing stale in the slots)
     gu.assert_same(_run(tr, 2, [1, 2]), gu.oracle_run(tr, 2, [1, 2]))
+
+
+def test_pipeline_plan_runs_again_and_on_refilled_buffers():
+    """PipelinePlan marshals ptc_pipeline's arguments once: repeated runs give
+    the same curves, and refilling its device buffers with another trace of
+    the same shape gives that trace's curves."""
+    import numpy as np
+    import paper_2609_28870_gb300 as ptc
+    from tests import gpu_util as gu
+    tr_a = tracegen.tiny(5, n_sessions=6, max_turns=4, vocab=5, max_seg=30)
+    rng = np.random.default_rng(12)
+    tr_b = tracegen.from_lists([list(rng.integers(0, 5, size=int(tr_a.req_tok_off[r + 1] - tr_a.req_tok_off[r])))
+                                for r in range(tr_a.n_req)])
+    assert tr_b.tokens.size == tr_a.tokens.size and np.array_equal(tr_b.req_tok_off, tr_a.req_tok_off)
+    B = 3
+    caps = [1, 2, 4, 8, 16, 1000]
+    tok, off, ts = gu.to_gpu(tr_a)
+    tok = tok[: tr_a.tokens.size]
+    plan = ptc.PipelinePlan(tok, off, None, B, caps)
+    keys = ("n_access", "n_distinct", "hits", "saved", "total_cost")
+    first = plan.run().result()
+    o = gu.oracle_run(tr_a, B, caps)
+    assert {k: first[k] for k in keys} == {k: o[k] for k in keys}
+    assert plan.run().result() == first
+    tok.copy_(ptc.to_device_u32(tr_b.tokens))
+    second = plan.run().result()
+    o = gu.oracle_run(tr_b, B, caps)
+    assert {k: second[k] for k in keys} == {k: o[k] for k in keys}
