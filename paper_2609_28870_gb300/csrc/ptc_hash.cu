@@ -242,6 +242,21 @@ __device__ __forceinline__ uint64_t limbs2_to_p61(uint64_t a0, uint64_t a1) {
   return p61_fold(p61_fold(a0) + ((a1 & ((1ULL << 30) - 1)) << 31) + (a1 >> 30));
 }
 
+// Congruent to (a0 + a1 2^31) mod p and below 2^61 + 3, for a0, a1 < 2^62.
+__device__ __forceinline__ uint64_t limbs2_lazy(uint64_t a0, uint64_t a1) {
+  const uint64_t x = (a0 & kP61) + (a0 >> 61) + ((a1 & ((1ULL << 30) - 1)) << 31) + (a1 >> 30);  // < 2^62 + 2^33
+  return (x & kP61) + (x >> 61);
+}
+
+// a b mod p, reduced only below 2^61 + 5, for a < 2^63 and b < p: the
+// product is below 2^124, so hi << 3 < 2^63 and the first sum stays below
+// 2^63 + 2^61 + 8.
+__device__ __forceinline__ uint64_t p61_mul_lazy(uint64_t a, uint64_t b) {
+  const uint64_t lo = a * b, hi = __umul64hi(a, b);
+  const uint64_t r = (lo & kP61) + (lo >> 61) + (hi << 3);
+  return (r & kP61) + (r >> 61);
+}
+
 // (a0 + a1 2^21 + a2 2^42) mod p for a0, a1, a2 < 2^62 - 2^57 (sums of <= 32 products < 2^53)
 __device__ __forceinline__ uint64_t limbs_to_p61(uint64_t a0, uint64_t a1, uint64_t a2) {
   uint64_t x = a0 + ((a1 & ((1ULL << 40) - 1)) << 21) + (a1 >> 40) + ((a2 & ((1ULL << 19) - 1)) << 42) + (a2 >> 19);
@@ -639,8 +654,9 @@ __global__ void __launch_bounds__(kHashThreads, 3) k_hash16(HashArgs a, const __
         case 2: hash16_2<2>(wd, c, acc); break;
         default: hash16_2<3>(wd, c, acc); break;
       }
-      h0 = p61_add(limbs2_to_p61(acc[0], acc[1]), c.csum[0][16]);
-      h1 = p61_add(limbs2_to_p61(acc[2], acc[3]), c.csum[1][16]);
+      // lazily reduced (below 2^62 + 3); p61_mul_lazy takes it as it is
+      h0 = limbs2_lazy(acc[0], acc[1]) + c.csum[0][16];
+      h1 = limbs2_lazy(acc[2], acc[3]) + c.csum[1][16];
     } else {
       uint64_t acc[6] = {0, 0, 0, 0, 0, 0};
       switch (m) {
@@ -656,16 +672,18 @@ __global__ void __launch_bounds__(kHashThreads, 3) k_hash16(HashArgs a, const __
   // g = h u^(16 k), then a plain prefix sum over the tile; a block whose
   // request starts inside the tile at index s subtracts the prefix before s.
   const uint64_t* T = a.tables;
-  uint64_t v0 = 0, v1 = 0;
+  uint64_t v0 = 0, v1 = 0;  // below 2^61 + 5
   if (live) {
-    v0 = p61_mul(h0, pow_at(T + 0 * 65536, T + 1 * 65536, k));
-    v1 = p61_mul(h1, pow_at(T + 2 * 65536, T + 3 * 65536, k));
+    v0 = p61_mul_lazy(h0, pow_at(T + 0 * 65536, T + 1 * 65536, k));
+    v1 = p61_mul_lazy(h1, pow_at(T + 2 * 65536, T + 3 * 65536, k));
   }
   __shared__ uint64_t s_p0[kHashThreads], s_p1[kHashThreads];
   __shared__ uint64_t s_w0[kHashThreads / 32], s_w1[kHashThreads / 32];
   const uint32_t lane = t & 31, w = t >> 5;
-  // warp scan with lazy reduction: three plain steps keep sums of at most 8
-  // values below 2^64, then each step folds back below 2^62
+  // warp scan with lazy reduction: from values below 2^61 + 5, two plain
+  // steps stay below 2^63 + 20; a fold (x & p) + (x >> 61) brings such a sum
+  // back below 2^61 + 4, so folding after d = 2 and d = 8 keeps every sum
+  // below 2^64 and leaves the result below 2^62 + 8
 #pragma unroll
   for (int d = 1; d < 32; d <<= 1) {
     const uint64_t y0 = __shfl_up_sync(kFull, v0, d), y1 = __shfl_up_sync(kFull, v1, d);
@@ -673,7 +691,7 @@ __global__ void __launch_bounds__(kHashThreads, 3) k_hash16(HashArgs a, const __
       v0 += y0;
       v1 += y1;
     }
-    if (d >= 4) {
+    if (d == 2 || d == 8) {
       v0 = (v0 & kP61) + (v0 >> 61);
       v1 = (v1 & kP61) + (v1 >> 61);
     }
@@ -697,8 +715,8 @@ __global__ void __launch_bounds__(kHashThreads, 3) k_hash16(HashArgs a, const __
       z1 = (z1 & kP61) + (z1 >> 61);
     }
     if (lane < kHashThreads / 32) {
-      s_w0[lane] = p61_fold(z0 + (kP61 << 1) - x0);  // z, x < 2^62: stays positive
-      s_w1[lane] = p61_fold(z1 + (kP61 << 1) - x1);
+      s_w0[lane] = p61_fold(z0 + (kP61 << 2) - x0);  // z < 2^61 + 4, x < 2^62 + 8: stays in (0, 2^64)
+      s_w1[lane] = p61_fold(z1 + (kP61 << 2) - x1);
     }
   }
   __syncthreads();
