@@ -807,6 +807,47 @@ __global__ void __launch_bounds__(kChainWarps * 32) k_hash_chain(ulonglong2* __r
   }
 }
 
+// The same carries as k_hash_chain, left for the keys' reader instead of
+// added to the keys (a pipeline that does not return the keys saves the
+// pass over them): carry[t] and lead[t] per tile, 0 where no key needs one.
+__global__ void __launch_bounds__(kChainWarps * 32) k_hash_carry(const HashCarry* __restrict__ tile_agg,
+                                                                 const uint32_t* __restrict__ tile_lead, uint32_t TB,
+                                                                 const DevStatus* st, uint64_t keys_cap,
+                                                                 uint32_t ntiles, ulonglong2* __restrict__ carry,
+                                                                 uint32_t* __restrict__ lead_out) {
+  grid_dep_sync();
+  const uint32_t lane = threadIdx.x & 31;
+  const uint32_t tile = blockIdx.x * kChainWarps + (threadIdx.x >> 5);
+  if (tile >= ntiles) return;
+  uint64_t N = st->value[0];
+  if (N > keys_cap) N = keys_cap;
+  const uint64_t b0 = (uint64_t)tile * TB;
+  const uint32_t lead = (b0 >= N || tile == 0) ? 0u : tile_lead[tile];
+  uint64_t c0 = 0, c1 = 0;
+  if (lead) {
+    for (int64_t base = (int64_t)tile - 1; base >= 0; base -= 32) {
+      const int64_t idx = base - (int64_t)lane;
+      HashCarry g{0, 0, 0};
+      if (idx >= 0) g = tile_agg[idx];
+      const uint32_t heads = __ballot_sync(kFull, idx >= 0 && g.f);
+      const uint32_t first = heads ? (uint32_t)(__ffs(heads) - 1) : 31u;
+      uint64_t v0 = lane <= first ? g.v0 : 0, v1 = lane <= first ? g.v1 : 0;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        v0 = p61_add(v0, __shfl_xor_sync(kFull, v0, o));
+        v1 = p61_add(v1, __shfl_xor_sync(kFull, v1, o));
+      }
+      c0 = p61_add(c0, v0);
+      c1 = p61_add(c1, v1);
+      if (heads) break;
+    }
+  }
+  if (lane == 0) {
+    carry[tile] = make_ulonglong2(c0, c1);
+    lead_out[tile] = lead;
+  }
+}
+
 template <int G>
 void launch_hash(uint32_t grid, cudaStream_t s, const HashArgs& a, const HashConsts& c, bool full) {
   if (G == 1 && full && a.aligned)
@@ -861,6 +902,11 @@ HashLayout hash_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
 
 using namespace ptc;
 
+uint64_t ptc::hash_carry_tiles(uint64_t n_tok, uint32_t block_size) {
+  if (block_size == 0) block_size = 1;
+  return ceil_div_u32(n_tok / block_size, kHashThreads / chunks_per_block(block_size)) + 1;
+}
+
 extern "C" size_t ptc_hash_blocks_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size) {
   if (block_size == 0) block_size = 1;
   return hash_layout(nullptr, n_req, n_tok, block_size, ~0ULL).total;
@@ -870,7 +916,7 @@ ptc_status ptc::hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t
                          const int64_t* req_ts_us, uint32_t n_req, uint32_t block_size, uint64_t seed,
                          ptc_u128* keys_out, uint64_t keys_cap, uint64_t* req_blk_off_out,
                          uint64_t* n_access_host_out, void* ws, size_t ws_bytes, cudaStream_t s, uint64_t* n_slot,
-                         uint32_t* err_slot) {
+                         uint32_t* err_slot, KeyCarry* carry) {
   if (block_size < 1 || block_size > PTC_MAX_BLOCK_SIZE) return PTC_ERR_INVALID_ARG;
   if (req_tok_off == nullptr || req_blk_off_out == nullptr || n_access_host_out == nullptr)
     return PTC_ERR_INVALID_ARG;
@@ -942,7 +988,14 @@ ptc_status ptc::hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t
       case 16: launch_hash<16>(grid, s, a, hc, full); break;
       default: launch_hash<32>(grid, s, a, hc, full); break;
     }
-    PTC_KERNEL("k_hash_chain", s, k_hash_chain, ceil_div_u32(grid, kChainWarps), kChainWarps * 32, 0, a.keys, L.tile_agg, L.tile_lead, kHashThreads / G, L.st, keys_cap);
+    if (carry) {
+      PTC_KERNEL("k_hash_carry", s, k_hash_carry, ceil_div_u32(grid, kChainWarps), kChainWarps * 32, 0, L.tile_agg,
+                 L.tile_lead, kHashThreads / G, L.st, keys_cap, grid, carry->carry, carry->lead);
+      carry->tile_blocks = kHashThreads / G;
+    } else {
+      PTC_KERNEL("k_hash_chain", s, k_hash_chain, ceil_div_u32(grid, kChainWarps), kChainWarps * 32, 0, a.keys,
+                 L.tile_agg, L.tile_lead, kHashThreads / G, L.st, keys_cap);
+    }
   }
   if (deferred) return defer_status(L.st, err_slot, s, n_slot, 0);
   DevStatus h;

@@ -95,10 +95,18 @@ __device__ __forceinline__ void settle(ulonglong2* table, uint64_t mask, uint64_
 
 // kInsK keys per thread, kInsThreads apart: all their key loads, then all
 // their home-slot loads, go out before any is settled.
+// Keys read by the insert; with kc.carry set they still lack the carry from
+// earlier tiles, which is added here (both words are below p, so p61_add).
+struct InsCarry {
+  const ulonglong2* carry;
+  const uint32_t* lead;
+  uint32_t tile_blocks;
+};
+
 __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __restrict__ keys, uint32_t n_ub,
                                                             const uint64_t* n_dev, ulonglong2* table, uint32_t log2m,
                                                             uint64_t probe_cap, uint32_t* __restrict__ slot_of,
-                                                            DevStatus* st) {
+                                                            DevStatus* st, InsCarry kc) {
   grid_dep_sync();
   const uint32_t n = keys_used(n_ub, n_dev);
   const uint32_t i0 = blockIdx.x * (kInsThreads * kInsK) + threadIdx.x;
@@ -109,6 +117,13 @@ __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __
   for (int j = 0; j < kInsK; ++j) {
     const uint32_t i = i0 + j * kInsThreads;
     k[j] = i < n ? __ldcs(&keys[i]) : make_ulonglong2(~0ULL, ~0ULL);  // streamed once: keep L2 for the table
+    if (kc.carry && i < n) {
+      const uint32_t t = i / kc.tile_blocks;
+      if (i - t * kc.tile_blocks < __ldg(&kc.lead[t]) && k[j].x < kP61 && k[j].y < kP61) {
+        const ulonglong2 c = __ldg(&kc.carry[t]);
+        k[j] = make_ulonglong2(p61_add(k[j].x, c.x), p61_add(k[j].y, c.y));
+      }
+    }
   }
 #pragma unroll
   for (int j = 0; j < kInsK; ++j) {
@@ -356,7 +371,8 @@ extern "C" size_t ptc_assign_ids_workspace_bytes(uint64_t n) { return ids_layout
 
 ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev, uint32_t* ids_out,
                         uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
-                        cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry) {
+                        cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc) {
+  const InsCarry ic = kc ? InsCarry{kc->carry, kc->lead, kc->tile_blocks} : InsCarry{nullptr, nullptr, 1};
   if (n_distinct_host_out == nullptr) return PTC_ERR_INVALID_ARG;
   *n_distinct_host_out = 0;
   if (n_used_host_out) *n_used_host_out = 0;
@@ -372,7 +388,7 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
     const ulonglong2* k = reinterpret_cast<const ulonglong2*>(keys);
     const uint32_t n32 = (uint32_t)n;
     PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads * kInsK), kInsThreads, 0, k, n32, n_dev, L.table,
-               log2m, probe_cap, L.slot_of, L.st);
+               log2m, probe_cap, L.slot_of, L.st, ic);
     PTC_KERNEL("k_ids_flags", s, k_ids_flags, L.ntiles, kFlT, 0, L.table, L.slot_of, n32, n_dev, L.ntiles, L.bits,
                L.tcnt, L.tpre, &L.done[0], L.st);
     PTC_KERNEL("k_ids_wordpre", s, k_ids_wordpre, ceil_div_u32((uint64_t)L.ntiles * 32, 256), 256, 0, L.bits, L.tpre,

@@ -135,19 +135,32 @@ struct RunsView {
   const uint32_t* bits = nullptr;   // run-start bitmap, one word per 32 accesses
   const uint32_t* wpre = nullptr;   // runs starting before each word
 };
+// Keys left without the carry from earlier tiles (stage a1 skips its
+// chain pass): block i of tile t = i / tile_blocks still needs carry[t] added
+// (mod p, per word) when i - t tile_blocks < lead[t].  Device arrays of
+// hash_carry_tiles() entries, owned by the caller.
+struct KeyCarry {
+  ulonglong2* carry;
+  uint32_t* lead;
+  uint32_t tile_blocks;
+};
+uint64_t hash_carry_tiles(uint64_t n_tok, uint32_t block_size);
+
 // Stage a1 (ptc_hash.cu).  With `n_slot` and `err_slot` (device memory) the
 // final wait is replaced by defer_status: N goes to *n_slot, the error word
-// to *err_slot, and *n_access_host_out is left 0.
+// to *err_slot, and *n_access_host_out is left 0.  With `carry` the keys are
+// left without the cross-tile carry, which goes to carry's arrays instead.
 ptc_status hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off, const int64_t* req_ts_us,
                      uint32_t n_req, uint32_t block_size, uint64_t seed, ptc_u128* keys_out, uint64_t keys_cap,
                      uint64_t* req_blk_off_out, uint64_t* n_access_host_out, void* ws, size_t ws_bytes,
-                     cudaStream_t s, uint64_t* n_slot, uint32_t* err_slot);
+                     cudaStream_t s, uint64_t* n_slot, uint32_t* err_slot, KeyCarry* carry = nullptr);
 // Stage a2 (ptc_ids.cu) over n_ub keys, of which the first min(*n_dev, n_ub)
 // are used when `n_dev` (device memory) is given.  Error words at
-// `carry_err` join the call's own.  Reports the number used and D.
+// `carry_err` join the call's own.  Reports the number used and D.  With
+// `kc` each key gets its tile's carry as it is read.
 ptc_status ids_impl(const ptc_u128* keys, uint64_t n_ub, const uint64_t* n_dev, uint32_t* ids_out,
                     uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
-                    cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry);
+                    cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc = nullptr);
 ptc_status stack_distance_view(const uint32_t* prev, uint64_t n, uint32_t* dist_out, int method, void* ws,
                                size_t ws_bytes, cudaStream_t s, RunsView* view, uint32_t* defer_err);
 // Stage b as ptc_reuse_indices does it (ptc_reuse.cu); with `defer_err` the

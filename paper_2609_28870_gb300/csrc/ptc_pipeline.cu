@@ -19,6 +19,8 @@ struct PipeLayout {
   size_t curves_bytes;
   uint32_t* defer;  // error words of stages a1, b and c, read with a later stage's
   uint64_t* n_slot;  // N as stage a1 left it, for stage a2
+  ulonglong2* carry;  // per hash tile: the carry stage a2 adds to the keys (when they are not returned)
+  uint32_t* lead;
   size_t total;
 };
 
@@ -48,6 +50,9 @@ PipeLayout pipe_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   L.curves = cv.take<unsigned char>(L.curves_bytes);
   L.defer = cv.take<uint32_t>(3);
   L.n_slot = cv.take<uint64_t>(1);
+  const uint64_t ct = keys ? 1 : ptc::hash_carry_tiles(n_tok, B);
+  L.carry = cv.take<ulonglong2>(ct);
+  L.lead = cv.take<uint32_t>(ct);
   L.total = cv.bytes();
   return L;
 }
@@ -89,10 +94,14 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
   // N go to device slots that stage a2 reads (its grids cover N's upper
   // bound, n_tok / B); b's and c's error words are read with stage d's.
   if (ptc::fill_async(L.defer, 0u, 3 * sizeof(uint32_t), s) != PTC_OK) return PTC_ERR_CUDA;
+  // keys the caller does not take skip their carry pass: stage a2 adds the
+  // carry as it reads them
+  ptc::KeyCarry kc{L.carry, L.lead, 1};
+  ptc::KeyCarry* kcp = keys_out ? nullptr : &kc;
   ptc_status rc = ptc::hash_impl(tokens, n_tok, req_tok_off, req_ts_us, n_req, block_size, seed, keys, cap, blk,
-                                 &unused, L.scratch, L.scratch_bytes, s, L.n_slot, &L.defer[0]);
+                                 &unused, L.scratch, L.scratch_bytes, s, L.n_slot, &L.defer[0], kcp);
   if (rc != PTC_OK) return rc;
-  rc = ptc::ids_impl(keys, cap, L.n_slot, ids, &n, &d, L.scratch, L.scratch_bytes, s, &L.defer[0], 1);
+  rc = ptc::ids_impl(keys, cap, L.n_slot, ids, &n, &d, L.scratch, L.scratch_bytes, s, &L.defer[0], 1, kcp);
   *n_access_host_out = n;
   *n_distinct_host_out = d;
   if (rc != PTC_OK) return rc;

@@ -54,6 +54,29 @@ def test_pipeline_tiny_random(seed):
     o = gu.oracle_run(tr, B, caps, kind)
     gu.assert_same(g, o)
     assert np.array_equal(g["keys"], oracle.prefix_hash(tr.tokens, tr.req_tok_off, B, seed))
+    # without caller arrays the keys skip their carry pass (stage a2 adds it)
+    bare = _run(tr, B, caps, kind, seed, with_outputs=False)
+    for k in ("n_access", "n_distinct", "hits", "saved", "total_cost"):
+        assert bare[k] == o[k]
+
+
+@pytest.mark.parametrize("B", [1, 5, 16])
+def test_pipeline_without_outputs_across_hash_tiles(B):
+    """Requests of thousands of blocks, so most keys take a carry from an
+    earlier tile; the pipeline without caller arrays adds it in stage a2."""
+    from tests import gpu_util as gu
+    rng = np.random.default_rng(400 + B)
+    base = list(rng.integers(0, 6, size=3000 * B))
+    reqs = [base[: 1700 * B + 3], base[: 2600 * B], list(rng.integers(0, 6, size=900 * B)), base[: 3000 * B - 1],
+            base[: 40 * B]]
+    tr = tracegen.from_lists(reqs)
+    _, D = oracle.block_ids(tr.tokens, tr.req_tok_off, B)
+    caps = [1, 7, 64, 500, D + 1]
+    o = gu.oracle_run(tr, B, caps)
+    for with_outputs in (True, False):
+        g = _run(tr, B, caps, with_outputs=with_outputs)
+        for k in ("n_access", "n_distinct", "hits", "saved", "total_cost"):
+            assert g[k] == o[k], (k, with_outputs)
 
 
 def test_pipeline_conversational_matches_oracle_and_separate_calls():
