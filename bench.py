@@ -150,7 +150,8 @@ KERNEL_SOURCE = {
     "k_runs_level": "ptc_runs.cu", "k_runs_build_cluster": "ptc_runs.cu", "k_runs_query": "ptc_runs.cu", "k_runs_expand": "ptc_runs.cu", "k_heads": "ptc_curves.cu", "k_curves_agg": "ptc_curves.cu",
     "k_curves": "ptc_curves.cu", "k_finalize": "ptc_curves.cu", "k_curves_fast": "ptc_curves.cu",
     "k_curves_runs": "ptc_curves.cu", "k_fill": "ptc_abi.cu", "k_copy_words": "ptc_abi.cu",
-    "k_copy_err": "ptc_abi.cu", "k_carry_err": "ptc_abi.cu",
+    "k_copy_err": "ptc_abi.cu", "k_carry_err": "ptc_abi.cu", "k_hash_carry": "ptc_hash.cu",
+    "k_keys_count": "ptc_runs.cu", "k_keys_pre": "ptc_runs.cu",
 }
 
 

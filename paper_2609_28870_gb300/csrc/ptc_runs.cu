@@ -34,6 +34,11 @@
 //   k_runs_count   run starts per tile; the last CTA scans the tile counts
 //   k_runs_mark    run starts again: bitmap, run index per 32-position word,
 //                  run (start, first value) records
+//   k_keys_count,  the runs' keys (marked by k_runs_mark in a bitmap over
+//   k_keys_pre     [0, n]) counted per word: the matrix holds each key's rank
+//                  among the distinct keys, so it has ceil(log2(R + 2))
+//                  levels instead of ceil(log2(n + 1)), and a query's
+//                  threshold x becomes the number of keys below x
 //   k_runs_init    level-0 keys and weights, per-tile zero counts / weights
 //   k_runs_level   one level: (Z, W), stable partition, the next level's
 //                  per-tile zero counts (four atomics per tile)
@@ -72,13 +77,14 @@ struct MarkArgs {
   uint32_t* tcnt;     // run starts in each tile
   uint32_t* tpre;     // runs starting before each tile; tpre[ntiles] = R
   uint32_t* done;
+  uint32_t* kbits;    // bitmap of the runs' keys (largest values) over [0, n]
   DevStatus* st;      // value[1] <- R
 };
 
 // Run-start bits of the warp's 8 x 32 positions from `base` (the previous
 // access decides whether one continues a run).
 __device__ __forceinline__ void start_words(const MarkArgs& a, uint32_t base, uint32_t lane, uint32_t (&pv)[kMR],
-                                            uint32_t (&words)[kMR], bool& bad) {
+                                            uint32_t (&words)[kMR], bool& bad, uint32_t* left = nullptr) {
 #pragma unroll
   for (int k = 0; k < kMR; ++k) {
     const uint32_t j = base + k * 32 + lane;
@@ -97,6 +103,7 @@ __device__ __forceinline__ void start_words(const MarkArgs& a, uint32_t base, ui
     carry = __shfl_sync(kFull, v, 31);
     const bool cont = j > 0 && ((v == vl + 1 && vl != 0) || (v == 0 && vl == 0));
     words[k] = __ballot_sync(kFull, valid && !cont);
+    if (left) left[k] = vl;
   }
 }
 
@@ -143,13 +150,28 @@ __global__ void __launch_bounds__(kMT) k_runs_mark(MarkArgs a) {
   const uint32_t tile = blockIdx.x;
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const uint32_t base = tile * kMTile + w * (32 * kMR);
-  uint32_t pv[kMR], words[kMR];
+  uint32_t pv[kMR], words[kMR], left[kMR];
   bool bad = false;
-  start_words(a, base, lane, pv, words, bad);
+  start_words(a, base, lane, pv, words, bad, left);
   uint32_t cnt = 0;
 #pragma unroll
   for (int k = 0; k < kMR; ++k) cnt += __popc(words[k]);
   if (lane == 0) s_wcnt[w] = cnt;
+  // The runs' keys for rank compression: a run's largest value is its last
+  // one (values along a context run rise by one; a first-access run is all
+  // zeros), i.e. the value left of the next run's start, or the last
+  // access's.  Nonzero keys are distinct (each access is the previous use of
+  // at most one other); 0 is always entered, once.
+#pragma unroll
+  for (int k = 0; k < kMR; ++k) {
+    const uint32_t j = base + k * 32 + lane;
+    if (j < a.n) {
+      if (((words[k] >> lane) & 1u) && j > 0 && left[k] != 0) atomicOr(&a.kbits[left[k] >> 5], 1u << (left[k] & 31));
+      const uint32_t v = vval(pv[k]);
+      if (j + 1 == a.n && v != 0) atomicOr(&a.kbits[v >> 5], 1u << (v & 31));
+    }
+  }
+  if (tile == 0 && threadIdx.x == 0) atomicOr(&a.kbits[0], 1u);
   __syncthreads();
   uint32_t run = a.tpre[tile];
   for (int ww = 0; ww < (int)w; ++ww) run += s_wcnt[ww];
@@ -168,6 +190,70 @@ __global__ void __launch_bounds__(kMT) k_runs_mark(MarkArgs a) {
     run += __popc(words[k]);
   }
   if (tile == a.ntiles - 1 && threadIdx.x == 0) a.rec_s[a.tpre[a.ntiles]] = a.n;
+}
+
+// Rank compression of the keys: keys set before every word of the key
+// bitmap, so that a key's rank among the distinct keys, and the number of
+// distinct keys below a query's threshold, are one lookup each.  Per tile of
+// kKTile words the set bits, the last CTA's tile prefixes, then per word.
+constexpr int kKT = 256;
+constexpr int kKPer = 8;
+constexpr int kKTile = kKT * kKPer;
+__global__ void __launch_bounds__(kKT) k_keys_count(const uint32_t* __restrict__ kbits, uint32_t nwords,
+                                                   uint32_t ntiles, uint32_t* tcnt, uint32_t* tpre, uint32_t* done) {
+  grid_dep_sync();
+  __shared__ uint32_t s_w[kKT / 32];
+  const uint32_t w0 = blockIdx.x * kKTile + threadIdx.x;
+  uint32_t c = 0;
+#pragma unroll
+  for (int k = 0; k < kKPer; ++k)
+    if (w0 + k * kKT < nwords) c += __popc(kbits[w0 + k * kKT]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(kFull, c, o);
+  if ((threadIdx.x & 31) == 0) s_w[threadIdx.x >> 5] = c;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t t = 0;
+    for (int i = 0; i < kKT / 32; ++i) t += s_w[i];
+    tcnt[blockIdx.x] = t;
+  }
+  if (!last_cta(done)) return;
+  cta_tiles_prefix(tcnt, tpre, ntiles);
+}
+
+__global__ void __launch_bounds__(kKT) k_keys_pre(const uint32_t* __restrict__ kbits, uint32_t nwords,
+                                                 const uint32_t* __restrict__ tpre, uint32_t* __restrict__ kpre) {
+  grid_dep_sync();
+  __shared__ uint32_t s_w[kKT / 32];
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const uint32_t w0 = blockIdx.x * kKTile + threadIdx.x * kKPer;  // consecutive words per thread
+  uint32_t c[kKPer], sum = 0;
+#pragma unroll
+  for (int k = 0; k < kKPer; ++k) {
+    c[k] = w0 + k < nwords ? __popc(kbits[w0 + k]) : 0u;
+    sum += c[k];
+  }
+  uint32_t incl = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(kFull, incl, o);
+    if (lane >= (uint32_t)o) incl += y;
+  }
+  if (lane == 31) s_w[w] = incl;
+  __syncthreads();
+  uint32_t run = tpre[blockIdx.x] + incl - sum;
+  for (int i = 0; i < (int)w; ++i) run += s_w[i];
+#pragma unroll
+  for (int k = 0; k < kKPer; ++k) {
+    if (w0 + k < nwords) kpre[w0 + k] = run;
+    run += c[k];
+  }
+}
+
+// Keys in the bitmap below v: the rank of v when v is a key.
+__device__ __forceinline__ uint32_t key_rank(const uint32_t* __restrict__ kbits, const uint32_t* __restrict__ kpre,
+                                             uint32_t v) {
+  return __ldg(&kpre[v >> 5]) + __popc(__ldg(&kbits[v >> 5]) & ((1u << (v & 31)) - 1u));
 }
 
 // Exclusive scan over the threads of a 256-thread CTA.
@@ -236,6 +322,7 @@ struct LevelArgs {
 // Level-0 keys (largest value of each run) and weights (lengths) and the
 // per-tile zero counts of level 0.
 __global__ void __launch_bounds__(kRT) k_runs_init(const uint32_t* __restrict__ rec_s, const uint32_t* __restrict__ rec_a,
+                                                  const uint32_t* __restrict__ kbits, const uint32_t* __restrict__ kpre,
                                                   uint32_t* __restrict__ key, uint32_t* __restrict__ wt,
                                                   uint2* __restrict__ acc, uint2* __restrict__ pre, uint32_t* done,
                                                   uint32_t R, uint32_t ntiles, uint32_t shift) {
@@ -249,7 +336,7 @@ __global__ void __launch_bounds__(kRT) k_runs_init(const uint32_t* __restrict__ 
     if (r < R) {
       const uint32_t s = rec_s[r], e = rec_s[r + 1], a0 = rec_a[r];
       const uint32_t len = e - s;
-      const uint32_t kv = a0 ? a0 + len - 1 : 0u;
+      const uint32_t kv = key_rank(kbits, kpre, a0 ? a0 + len - 1 : 0u);
       key[r] = kv;
       wt[r] = len;
       if (!((kv >> shift) & 1u)) {
@@ -376,6 +463,8 @@ constexpr int kCMax = 16;           // largest cluster (above 8 needs the non-po
 struct BuildArgs {
   const uint32_t* rec_s;
   const uint32_t* rec_a;
+  const uint32_t* kbits;  // keys enter the matrix as their ranks (key_rank)
+  const uint32_t* kpre;
   uint2* zw;
   uint32_t R, L, slice;
 };
@@ -396,7 +485,7 @@ __global__ void __launch_bounds__(kCT) k_runs_build_cluster(BuildArgs a) {
     const uint32_t r = base + i;
     const uint32_t st = a.rec_s[r], e = a.rec_s[r + 1], a0 = a.rec_a[r];
     const uint32_t len = e - st;
-    s_dyn[i] = make_uint2(a0 ? a0 + len - 1 : 0u, len);
+    s_dyn[i] = make_uint2(key_rank(a.kbits, a.kpre, a0 ? a0 + len - 1 : 0u), len);
   }
   cl.sync();
   for (uint32_t l = 0; l < a.L; ++l) {
@@ -522,6 +611,8 @@ struct QueryArgs {
   const uint32_t* rec_a;
   const uint32_t* bits;
   const uint32_t* wpre;
+  const uint32_t* kbits;  // the matrix holds key ranks: thresholds go through key_rank too
+  const uint32_t* kpre;
   const uint2* zw;      // level l at zw + l * (R + 1)
   uint32_t* sd;         // distance of each run
   uint32_t R, L;
@@ -555,10 +646,12 @@ __global__ void __launch_bounds__(256) k_runs_query(QueryArgs a) {
   }
   uint32_t hi = r, cnt = 0;
   const uint32_t stride = a.R + 1;
+  // keys below x are the keys whose rank is below the number of keys below x
+  const uint32_t xr = key_rank(a.kbits, a.kpre, x);
   for (uint32_t l = 0; l < a.L && lo < hi; ++l) {
     const uint2* zl = a.zw + (size_t)l * stride;
     const uint2 zlo = zl[lo], zhi = zl[hi];
-    if ((x >> (a.L - 1 - l)) & 1u) {
+    if ((xr >> (a.L - 1 - l)) & 1u) {
       const uint32_t Zc = zl[a.R].x;
       cnt += zhi.y - zlo.y;
       lo = Zc + (lo - zlo.x);
@@ -605,7 +698,10 @@ uint32_t key_bits_n(uint64_t n) {  // keys and thresholds lie in [0, n]
 struct RunsLayout {
   DevStatus* st;
   uint32_t* done;
+  uint32_t* kbits;  // key bitmap over [0, n] (zeroed with the status)
   uint32_t *tcnt, *tpre;
+  uint32_t *kpre, *ktcnt, *ktpre;
+  uint32_t kwords, ktiles;
   size_t zero_bytes;
   uint32_t *bits, *wpre, *rec_s, *rec_a;
   uint32_t *sd, *k0, *k1, *w0, *w1;
@@ -619,14 +715,20 @@ RunsLayout runs_layout(void* ws, uint64_t n, uint64_t R) {
   RunsLayout W;
   Carver cv(ws);
   const uint64_t nn = n ? n : 1, rr = R ? R : 1;
-  W.L = key_bits_n(n);
+  W.L = key_bits_n(rr + 1);  // key ranks and thresholds lie in [0, R + 1]
   W.mtiles = ceil_div_u32(nn, kMTile);
   W.rtiles = ceil_div_u32(rr, kRTile);
+  W.kwords = (uint32_t)(nn / 32 + 2);  // keys and thresholds lie in [0, n]
+  W.ktiles = ceil_div_u32(W.kwords, kKTile);
   W.st = cv.take<DevStatus>(1);
   W.done = cv.take<uint32_t>(64);
+  W.kbits = cv.take<uint32_t>(W.kwords);
   W.zero_bytes = cv.off;
   W.tcnt = cv.take<uint32_t>(W.mtiles + 1);
   W.tpre = cv.take<uint32_t>(W.mtiles + 1);
+  W.kpre = cv.take<uint32_t>(W.kwords);
+  W.ktcnt = cv.take<uint32_t>(W.ktiles + 1);
+  W.ktpre = cv.take<uint32_t>(W.ktiles + 1);
   W.bits = cv.take<uint32_t>(nn / 32 + 2);
   W.wpre = cv.take<uint32_t>(nn / 32 + 2);
   W.rec_s = cv.take<uint32_t>(nn + 1);
@@ -691,9 +793,13 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   m.tcnt = M.tcnt;
   m.tpre = M.tpre;
   m.done = &M.done[63];
+  m.kbits = M.kbits;
   m.st = M.st;
   PTC_KERNEL("k_runs_count", s, k_runs_count, M.mtiles, kMT, 0, m);
   PTC_KERNEL("k_runs_mark", s, k_runs_mark, M.mtiles, kMT, 0, m);
+  PTC_KERNEL("k_keys_count", s, k_keys_count, M.ktiles, kKT, 0, M.kbits, M.kwords, M.ktiles, M.ktcnt, M.ktpre,
+             &M.done[62]);
+  PTC_KERNEL("k_keys_pre", s, k_keys_pre, M.ktiles, kKT, 0, M.kbits, M.kwords, M.ktpre, M.kpre);
   DevStatus h;
   ptc_status rc = end_call(M.st, s, &h);
   if (rc != PTC_OK) return rc;
@@ -721,6 +827,8 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
     BuildArgs b;
     b.rec_s = W.rec_s;
     b.rec_a = W.rec_a;
+    b.kbits = W.kbits;
+    b.kpre = W.kpre;
     b.zw = W.zw;
     b.R = R32;
     b.L = L;
@@ -749,7 +857,8 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
       (void)cudaGetLastError();
   }
   if (!built) {
-    PTC_KERNEL("k_runs_init", s, k_runs_init, T, kRT, 0, W.rec_s, W.rec_a, W.k0, W.w0, W.acc, W.pre, &W.done[0], R32, T, L - 1);
+    PTC_KERNEL("k_runs_init", s, k_runs_init, T, kRT, 0, W.rec_s, W.rec_a, W.kbits, W.kpre, W.k0, W.w0, W.acc, W.pre,
+               &W.done[0], R32, T, L - 1);
     uint32_t* keys[2] = {W.k0, W.k1};
     uint32_t* wts[2] = {W.w0, W.w1};
     for (uint32_t l = 0; l < L; ++l) {
@@ -775,6 +884,8 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   q.rec_a = W.rec_a;
   q.bits = W.bits;
   q.wpre = W.wpre;
+  q.kbits = W.kbits;
+  q.kpre = W.kpre;
   q.zw = W.zw;
   q.sd = W.sd;
   q.R = R32;
