@@ -139,8 +139,7 @@ def kernel_model_bytes(name, T, N, L, D):
 KERNEL_SOURCE = {
     "k_block_offsets": "ptc_hash.cu", "k_pow_tables": "ptc_hash.cu", "k_hash_local": "ptc_hash.cu",
     "k_hash16": "ptc_hash.cu",
-    "k_hash_chain": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu", "k_ids_flags": "ptc_ids.cu",
-    "k_ids_wordpre": "ptc_ids.cu",
+    "k_hash_chain": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu", "k_ids_mark": "ptc_ids.cu",
     "k_ids_gather": "ptc_ids.cu", "k_sort_count": "ptc_sort.cu", "k_sort_rowscan": "ptc_sort.cu",
     "k_sort_scatter": "ptc_sort.cu", "k_sort_links": "ptc_sort.cu", "k_ir_count": "ptc_reuse.cu",
     "k_ir_mark": "ptc_reuse.cu", "k_bm_count": "ptc_reuse.cu", "k_bm_words": "ptc_reuse.cu",
@@ -151,7 +150,7 @@ KERNEL_SOURCE = {
     "k_curves": "ptc_curves.cu", "k_finalize": "ptc_curves.cu", "k_curves_fast": "ptc_curves.cu",
     "k_curves_runs": "ptc_curves.cu", "k_fill": "ptc_abi.cu", "k_copy_words": "ptc_abi.cu",
     "k_copy_err": "ptc_abi.cu", "k_carry_err": "ptc_abi.cu", "k_hash_carry": "ptc_hash.cu",
-    "k_keys_count": "ptc_runs.cu", "k_keys_pre": "ptc_runs.cu",
+    "k_rank_count": "ptc_abi.cu", "k_rank_words": "ptc_abi.cu",
 }
 
 

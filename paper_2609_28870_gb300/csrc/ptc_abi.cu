@@ -162,6 +162,84 @@ ptc_status copy_to_host_async(void* host_dst, const void* dev_src, size_t bytes,
   return PTC_OK;
 }
 
+namespace {
+constexpr int kRkThreads = 256;
+constexpr int kRkPer = kRankTile / kRkThreads;  // consecutive words per thread
+static_assert(kRkPer * kRkThreads == (int)kRankTile, "rank tile");
+
+__device__ __forceinline__ bool rank_last_cta(uint32_t* done) {
+  __shared__ uint32_t s_last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(done, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (s_last) __threadfence();
+  return s_last;
+}
+
+__global__ void __launch_bounds__(kRkThreads) k_rank_count(const uint32_t* __restrict__ bits, uint32_t nwords,
+                                                          uint32_t ntiles, uint32_t* tcnt, uint32_t* tpre,
+                                                          uint32_t* done, uint64_t* total) {
+  grid_dep_sync();
+  __shared__ uint32_t s_w[kRkThreads / 32];
+  const uint32_t w0 = blockIdx.x * kRankTile + threadIdx.x;
+  uint32_t c = 0;
+#pragma unroll
+  for (int k = 0; k < kRkPer; ++k)
+    if (w0 + k * kRkThreads < nwords) c += __popc(bits[w0 + k * kRkThreads]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(kFull, c, o);
+  if ((threadIdx.x & 31) == 0) s_w[threadIdx.x >> 5] = c;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t t = 0;
+    for (int i = 0; i < kRkThreads / 32; ++i) t += s_w[i];
+    tcnt[blockIdx.x] = t;
+  }
+  if (!rank_last_cta(done)) return;
+  const uint32_t all = cta_tiles_prefix(tcnt, tpre, ntiles);
+  if (total && threadIdx.x == 0) *total = all;
+}
+
+__global__ void __launch_bounds__(kRkThreads) k_rank_words(const uint32_t* __restrict__ bits, uint32_t nwords,
+                                                          const uint32_t* __restrict__ tpre, uint32_t* __restrict__ pre) {
+  grid_dep_sync();
+  __shared__ uint32_t s_w[kRkThreads / 32];
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const uint32_t w0 = blockIdx.x * kRankTile + threadIdx.x * kRkPer;
+  uint32_t c[kRkPer], sum = 0;
+#pragma unroll
+  for (int k = 0; k < kRkPer; ++k) {
+    c[k] = w0 + k < nwords ? __popc(bits[w0 + k]) : 0u;
+    sum += c[k];
+  }
+  uint32_t incl = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(kFull, incl, o);
+    if (lane >= (uint32_t)o) incl += y;
+  }
+  if (lane == 31) s_w[w] = incl;
+  __syncthreads();
+  uint32_t run = tpre[blockIdx.x] + incl - sum;
+  for (int i = 0; i < (int)w; ++i) run += s_w[i];
+#pragma unroll
+  for (int k = 0; k < kRkPer; ++k) {
+    if (w0 + k < nwords) pre[w0 + k] = run;
+    run += c[k];
+  }
+}
+}  // namespace
+
+ptc_status bitmap_ranks(const uint32_t* bits, uint32_t nwords, uint32_t* pre, uint32_t* tcnt, uint32_t* tpre,
+                        uint32_t* done, uint64_t* total, cudaStream_t s) {
+  if (nwords == 0) return PTC_OK;
+  const uint32_t T = rank_tiles(nwords);
+  PTC_KERNEL("k_rank_count", s, k_rank_count, T, kRkThreads, 0, bits, nwords, T, tcnt, tpre, done, total);
+  PTC_KERNEL("k_rank_words", s, k_rank_words, T, kRkThreads, 0, bits, nwords, tpre, pre);
+  return PTC_OK;
+}
+
 ptc_status carry_errors(const uint32_t* err, uint32_t n, DevStatus* st, cudaStream_t s) {
   if (n == 0) return PTC_OK;
   if (n > 32) return PTC_ERR_INVALID_ARG;

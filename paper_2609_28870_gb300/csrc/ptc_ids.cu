@@ -7,11 +7,11 @@
 //                  empty (or half-written) slot is claimed with one 128-bit
 //                  CAS, and a stored index above i is lowered with atomicMin.
 //                  Linear probing.
-//   k_ids_flags    first[i] = index stored in i's slot; access i is a first
-//                  occurrence iff first[i] == i: a bitmap of those, counts
-//                  per tile, and (last CTA) the tile prefixes
-//   k_ids_wordpre  first occurrences before every 32-position word
-//   k_ids_gather   ids[i] = rank of first[i] among the first occurrences.
+//   k_ids_mark     one pass over the slots: each filled slot's index is a
+//                  first occurrence; a bitmap of those over positions
+//   bitmap_ranks   first occurrences before every 32-position word, and D
+//   k_ids_gather   ids[i] = rank, among the first occurrences, of the index
+//                  stored in i's slot.
 // ptc_verify_ids
 //   k_verify_first first access of every id (atomicMin)
 //   k_verify       compares every access's B tokens and parent id with those
@@ -143,94 +143,44 @@ __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __
   }
 }
 
-constexpr int kFlT = 256;             // flags: threads per tile
-constexpr int kFlR = 8;               // rounds of 32 positions per warp
-constexpr int kFlTile = kFlT * kFlR;  // 2048 positions; warp w owns [256 w, 256 w + 256)
-
-// first[i] (in place of slot_of[i]) and the first-occurrence bitmap; tile
-// counts, and the last CTA's tile prefixes (tpre[ntiles] = D).  Bitmap words
-// past the keys used but inside the n_ub the grid covers are written as 0.
-// The last CTA also reports D (value[0]) and the key count (value[1]).
-__global__ void __launch_bounds__(kFlT) k_ids_flags(const ulonglong2* __restrict__ table, uint32_t* slot_first,
-                                                   uint32_t n_ub, const uint64_t* n_dev, uint32_t ntiles,
-                                                   uint32_t* __restrict__ bits, uint32_t* tcnt, uint32_t* tpre,
-                                                   uint32_t* done, DevStatus* st) {
+// First occurrences from the table itself: every filled slot holds the
+// smallest access index of its key, so one pass over the slots (coalesced,
+// mostly in L2) marks the first-occurrence bitmap over access positions.
+// Block 0 also reports the number of keys used (value[1]).
+constexpr int kMkThreads = 256;
+constexpr int kMkPer = 8;
+__global__ void __launch_bounds__(kMkThreads) k_ids_mark(const ulonglong2* __restrict__ table, uint64_t m,
+                                                        uint32_t* __restrict__ bits, uint32_t n_ub,
+                                                        const uint64_t* n_dev, DevStatus* st) {
   grid_dep_sync();
-  const uint32_t n = keys_used(n_ub, n_dev);
-  __shared__ uint32_t s_w[kFlT / 32];
-  __shared__ uint32_t s_last;
-  const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  const uint32_t base = tile * kFlTile + w * (32 * kFlR);
-  // slots, then their first indices, then the stores: all eight loads of
-  // each kind are in flight together
-  uint32_t f[kFlR];
-#pragma unroll
-  for (int k = 0; k < kFlR; ++k) {
-    const uint32_t i = base + k * 32 + lane;
-    f[k] = i < n ? __ldcs(&slot_first[i]) : 0u;
-  }
-#pragma unroll
-  for (int k = 0; k < kFlR; ++k) {
-    const uint32_t i = base + k * 32 + lane;
-    f[k] = i < n ? reinterpret_cast<const uint32_t*>(&table[f[k]])[3] : kNone;
-  }
-  uint32_t cnt = 0;
-#pragma unroll
-  for (int k = 0; k < kFlR; ++k) {
-    const uint32_t i = base + k * 32 + lane;
-    if (i < n) __stcs(&slot_first[i], f[k]);
-    const uint32_t m = __ballot_sync(kFull, i < n && f[k] == i);
-    if (lane == 0 && base + k * 32 < n_ub) bits[(base + k * 32) >> 5] = m;
-    cnt += __popc(m);
-  }
-  if (lane == 0) s_w[w] = cnt;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    uint32_t t = 0;
-    for (int ww = 0; ww < kFlT / 32; ++ww) t += s_w[ww];
-    tcnt[tile] = t;
-  }
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) s_last = atomicAdd(done, 1u) == gridDim.x - 1;
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  const uint32_t total = cta_tiles_prefix(tcnt, tpre, ntiles);
-  if (threadIdx.x == 0) {
-    st->value[0] = total;
-    st->value[1] = n_dev ? *n_dev : n;
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    st->value[1] = n_dev ? *n_dev : n_ub;
     if (n_dev && *n_dev > n_ub) raise_err(st, kErrInvalid);  // more blocks than the keys buffer holds
   }
-}
-
-// First occurrences before every word: one warp per tile of 64 words.
-__global__ void k_ids_wordpre(const uint32_t* __restrict__ bits, const uint32_t* __restrict__ tpre, uint32_t nwords,
-                              uint32_t* __restrict__ wpre) {
-  grid_dep_sync();
-  const uint32_t warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
-  const uint32_t w0 = warp * (kFlTile / 32);
-  if (w0 >= nwords) return;
-  uint32_t run = tpre[warp];
+  const uint64_t s0 = (uint64_t)blockIdx.x * (kMkThreads * kMkPer) + threadIdx.x;
+  ulonglong2 v[kMkPer];
 #pragma unroll
-  for (int h = 0; h < kFlTile / 32 / 32; ++h) {
-    const uint32_t wi = w0 + h * 32 + lane;
-    const uint32_t c = wi < nwords ? __popc(bits[wi]) : 0u;
-    uint32_t incl = c;
+  for (int k = 0; k < kMkPer; ++k) {
+    const uint64_t sl = s0 + (uint64_t)k * kMkThreads;
+    v[k] = sl < m ? __ldg(&table[sl]) : make_ulonglong2(~0ULL, ~0ULL);  // the gather reads it again
+  }
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t y = __shfl_up_sync(kFull, incl, o);
-      if (lane >= (uint32_t)o) incl += y;
+  for (int k = 0; k < kMkPer; ++k) {
+    if (v[k].x != ~0ULL && v[k].y != ~0ULL) {
+      const uint32_t f = (uint32_t)(v[k].y >> 32);
+      atomicOr(&bits[f >> 5], 1u << (f & 31));
     }
-    if (wi < nwords) wpre[wi] = run + incl - c;
-    run += __shfl_sync(kFull, incl, 31);
   }
 }
 
-// kGaPer accesses per thread, kGaThreads apart, their loads in flight together.
+// ids[i] = rank of the first occurrence of i's key among all first
+// occurrences: the slot gives the first occurrence, the bitmap's word
+// prefixes its rank.  kGaPer accesses per thread, kGaThreads apart, their
+// dependent loads in flight together.
 constexpr int kGaThreads = 256;
 constexpr int kGaPer = 8;
-__global__ void __launch_bounds__(kGaThreads) k_ids_gather(const uint32_t* __restrict__ first,
+__global__ void __launch_bounds__(kGaThreads) k_ids_gather(const uint32_t* __restrict__ slot_of,
+                                                          const ulonglong2* __restrict__ table,
                                                           const uint32_t* __restrict__ bits,
                                                           const uint32_t* __restrict__ wpre, uint32_t n_ub,
                                                           const uint64_t* n_dev, uint32_t* __restrict__ ids) {
@@ -241,7 +191,12 @@ __global__ void __launch_bounds__(kGaThreads) k_ids_gather(const uint32_t* __res
 #pragma unroll
   for (int k = 0; k < kGaPer; ++k) {
     const uint32_t i = i0 + k * kGaThreads;
-    f[k] = i < n ? __ldcs(&first[i]) : kNone;
+    f[k] = i < n ? __ldcs(&slot_of[i]) : 0u;
+  }
+#pragma unroll
+  for (int k = 0; k < kGaPer; ++k) {
+    const uint32_t i = i0 + k * kGaThreads;
+    f[k] = i < n ? __ldg(reinterpret_cast<const uint32_t*>(&table[f[k]]) + 3) : kNone;
   }
   uint32_t wp[kGaPer], bw[kGaPer];
 #pragma unroll
@@ -275,9 +230,9 @@ struct IdsLayout {
   DevStatus* st;
   uint32_t* done;
   ulonglong2* table;
-  uint32_t* slot_of;  // then first[i]
-  uint32_t *bits, *wpre, *tcnt, *tpre;
-  uint32_t ntiles, nwords;
+  uint32_t* slot_of;
+  uint32_t *bits, *wpre, *tcnt, *tpre;  // first-occurrence bitmap and its ranks
+  uint32_t nwords;
   size_t zero_bytes;
   size_t total;
   uint32_t log2m;
@@ -289,7 +244,6 @@ IdsLayout ids_layout(void* ws, uint64_t n) {
   L.log2m = full_table_log2(n);
   const uint64_t m = 1ULL << L.log2m;
   const uint64_t nn = n ? n : 1;
-  L.ntiles = ceil_div_u32(nn, kFlTile);
   L.nwords = ceil_div_u32(nn, 32);
   L.st = cv.take<DevStatus>(1);
   L.done = cv.take<uint32_t>(64);
@@ -298,8 +252,8 @@ IdsLayout ids_layout(void* ws, uint64_t n) {
   L.slot_of = cv.take<uint32_t>(nn);
   L.bits = cv.take<uint32_t>(L.nwords + 1);
   L.wpre = cv.take<uint32_t>(L.nwords + 1);
-  L.tcnt = cv.take<uint32_t>(L.ntiles + 1);
-  L.tpre = cv.take<uint32_t>(L.ntiles + 1);
+  L.tcnt = cv.take<uint32_t>(rank_tiles(L.nwords) + 1);
+  L.tpre = cv.take<uint32_t>(rank_tiles(L.nwords) + 1);
   L.total = cv.bytes();
   return L;
 }
@@ -389,12 +343,13 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
     const uint32_t n32 = (uint32_t)n;
     PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads * kInsK), kInsThreads, 0, k, n32, n_dev, L.table,
                log2m, probe_cap, L.slot_of, L.st, ic);
-    PTC_KERNEL("k_ids_flags", s, k_ids_flags, L.ntiles, kFlT, 0, L.table, L.slot_of, n32, n_dev, L.ntiles, L.bits,
-               L.tcnt, L.tpre, &L.done[0], L.st);
-    PTC_KERNEL("k_ids_wordpre", s, k_ids_wordpre, ceil_div_u32((uint64_t)L.ntiles * 32, 256), 256, 0, L.bits, L.tpre,
-               L.nwords, L.wpre);
-    PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of, L.bits, L.wpre, n32, n_dev,
-               ids_out);
+    const uint64_t m = 1ULL << log2m;
+    if (fill_async(L.bits, 0u, sizeof(uint32_t) * L.nwords, s) != PTC_OK) return false;
+    PTC_KERNEL("k_ids_mark", s, k_ids_mark, ceil_div_u32(m, kMkThreads * kMkPer), kMkThreads, 0, L.table, m, L.bits,
+               n32, n_dev, L.st);
+    if (bitmap_ranks(L.bits, L.nwords, L.wpre, L.tcnt, L.tpre, &L.done[0], &L.st->value[0], s) != PTC_OK) return false;
+    PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of,
+               L.table, L.bits, L.wpre, n32, n_dev, ids_out);
     return true;
   };
   if (!start()) return PTC_ERR_CUDA;

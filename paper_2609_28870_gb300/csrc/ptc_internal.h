@@ -107,6 +107,16 @@ inline ptc_status end_call(const DevStatus* dev, cudaStream_t stream, DevStatus*
 
 // Instead of waiting for a call's status, queue a copy of its error word to
 // `slot`, for a later call that does wait to fold in (ptc_pipeline).
+// Ranks over a bitmap (ptc_abi.cu): pre[w] = set bits in words [0, w) for
+// w < nwords, by a count per tile of kRankTile words, the last CTA's prefix
+// over the tiles, then a pass per word.  Scratch: tcnt and tpre of
+// rank_tiles(nwords) + 1 entries, and a zeroed counter *done.  With `total`
+// the number of set bits is stored there (device memory).
+constexpr uint32_t kRankTile = 2048;
+inline uint32_t rank_tiles(uint32_t nwords) { return (nwords + kRankTile - 1) / kRankTile; }
+ptc_status bitmap_ranks(const uint32_t* bits, uint32_t nwords, uint32_t* pre, uint32_t* tcnt, uint32_t* tpre,
+                        uint32_t* done, uint64_t* total, cudaStream_t s);
+
 // OR the n (at most 32) deferred error words at `err` into st->err.
 ptc_status carry_errors(const uint32_t* err, uint32_t n, DevStatus* st, cudaStream_t s);
 // With `value_slot`, value[value_index] of the status block is copied there too.

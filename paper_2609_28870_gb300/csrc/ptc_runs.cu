@@ -34,8 +34,8 @@
 //   k_runs_count   run starts per tile; the last CTA scans the tile counts
 //   k_runs_mark    run starts again: bitmap, run index per 32-position word,
 //                  run (start, first value) records
-//   k_keys_count,  the runs' keys (marked by k_runs_mark in a bitmap over
-//   k_keys_pre     [0, n]) counted per word: the matrix holds each key's rank
+//   bitmap_ranks   the runs' keys (marked by k_runs_mark in a bitmap over
+//                  [0, n]) counted per word: the matrix holds each key's rank
 //                  among the distinct keys, so it has ceil(log2(R + 2))
 //                  levels instead of ceil(log2(n + 1)), and a query's
 //                  threshold x becomes the number of keys below x
@@ -190,64 +190,6 @@ __global__ void __launch_bounds__(kMT) k_runs_mark(MarkArgs a) {
     run += __popc(words[k]);
   }
   if (tile == a.ntiles - 1 && threadIdx.x == 0) a.rec_s[a.tpre[a.ntiles]] = a.n;
-}
-
-// Rank compression of the keys: keys set before every word of the key
-// bitmap, so that a key's rank among the distinct keys, and the number of
-// distinct keys below a query's threshold, are one lookup each.  Per tile of
-// kKTile words the set bits, the last CTA's tile prefixes, then per word.
-constexpr int kKT = 256;
-constexpr int kKPer = 8;
-constexpr int kKTile = kKT * kKPer;
-__global__ void __launch_bounds__(kKT) k_keys_count(const uint32_t* __restrict__ kbits, uint32_t nwords,
-                                                   uint32_t ntiles, uint32_t* tcnt, uint32_t* tpre, uint32_t* done) {
-  grid_dep_sync();
-  __shared__ uint32_t s_w[kKT / 32];
-  const uint32_t w0 = blockIdx.x * kKTile + threadIdx.x;
-  uint32_t c = 0;
-#pragma unroll
-  for (int k = 0; k < kKPer; ++k)
-    if (w0 + k * kKT < nwords) c += __popc(kbits[w0 + k * kKT]);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(kFull, c, o);
-  if ((threadIdx.x & 31) == 0) s_w[threadIdx.x >> 5] = c;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    uint32_t t = 0;
-    for (int i = 0; i < kKT / 32; ++i) t += s_w[i];
-    tcnt[blockIdx.x] = t;
-  }
-  if (!last_cta(done)) return;
-  cta_tiles_prefix(tcnt, tpre, ntiles);
-}
-
-__global__ void __launch_bounds__(kKT) k_keys_pre(const uint32_t* __restrict__ kbits, uint32_t nwords,
-                                                 const uint32_t* __restrict__ tpre, uint32_t* __restrict__ kpre) {
-  grid_dep_sync();
-  __shared__ uint32_t s_w[kKT / 32];
-  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  const uint32_t w0 = blockIdx.x * kKTile + threadIdx.x * kKPer;  // consecutive words per thread
-  uint32_t c[kKPer], sum = 0;
-#pragma unroll
-  for (int k = 0; k < kKPer; ++k) {
-    c[k] = w0 + k < nwords ? __popc(kbits[w0 + k]) : 0u;
-    sum += c[k];
-  }
-  uint32_t incl = sum;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t y = __shfl_up_sync(kFull, incl, o);
-    if (lane >= (uint32_t)o) incl += y;
-  }
-  if (lane == 31) s_w[w] = incl;
-  __syncthreads();
-  uint32_t run = tpre[blockIdx.x] + incl - sum;
-  for (int i = 0; i < (int)w; ++i) run += s_w[i];
-#pragma unroll
-  for (int k = 0; k < kKPer; ++k) {
-    if (w0 + k < nwords) kpre[w0 + k] = run;
-    run += c[k];
-  }
 }
 
 // Keys in the bitmap below v: the rank of v when v is a key.
@@ -719,7 +661,7 @@ RunsLayout runs_layout(void* ws, uint64_t n, uint64_t R) {
   W.mtiles = ceil_div_u32(nn, kMTile);
   W.rtiles = ceil_div_u32(rr, kRTile);
   W.kwords = (uint32_t)(nn / 32 + 2);  // keys and thresholds lie in [0, n]
-  W.ktiles = ceil_div_u32(W.kwords, kKTile);
+  W.ktiles = rank_tiles(W.kwords);
   W.st = cv.take<DevStatus>(1);
   W.done = cv.take<uint32_t>(64);
   W.kbits = cv.take<uint32_t>(W.kwords);
@@ -797,9 +739,7 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   m.st = M.st;
   PTC_KERNEL("k_runs_count", s, k_runs_count, M.mtiles, kMT, 0, m);
   PTC_KERNEL("k_runs_mark", s, k_runs_mark, M.mtiles, kMT, 0, m);
-  PTC_KERNEL("k_keys_count", s, k_keys_count, M.ktiles, kKT, 0, M.kbits, M.kwords, M.ktiles, M.ktcnt, M.ktpre,
-             &M.done[62]);
-  PTC_KERNEL("k_keys_pre", s, k_keys_pre, M.ktiles, kKT, 0, M.kbits, M.kwords, M.ktpre, M.kpre);
+  if (bitmap_ranks(M.kbits, M.kwords, M.kpre, M.ktcnt, M.ktpre, &M.done[62], nullptr, s) != PTC_OK) return PTC_ERR_CUDA;
   DevStatus h;
   ptc_status rc = end_call(M.st, s, &h);
   if (rc != PTC_OK) return rc;
