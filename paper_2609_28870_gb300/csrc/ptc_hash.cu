@@ -37,14 +37,14 @@ constexpr int kOffThreads = 512;
 constexpr int kOffPer = 8;
 constexpr int kOffTile = kOffThreads * kOffPer;
 
-constexpr int kHashThreads = 512;
+constexpr int kHashThreads = 256;
 constexpr int kWinTokens = 8192 + 256;
 constexpr int kWinWords = kWinTokens + kWinTokens / 16;
 
 constexpr int kEpochOffsets = 1;
 
 // ---------------------------------------------------------------- block scans
-// Exclusive sum over a CTA of 512 threads; returns the CTA total in *total.
+// Exclusive sum over a CTA of kOffThreads (512) threads; returns the CTA total in *total.
 __device__ __forceinline__ uint64_t cta_exclusive_sum(uint64_t v, uint64_t* total) {
   __shared__ uint64_t s_w[kOffThreads / 32];
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -536,8 +536,9 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local_vec(HashArgs a, con
   hash_finish<G>(a, tile, b0, b_end, h0, h1, k, lb, s);
 }
 
-// B = 16 with 16-byte-aligned tokens: one block per thread, 512 blocks per
-// tile (as k_hash_local with G = 1).  The requests that meet the tile are
+// B = 16 with 16-byte-aligned tokens: one block per thread, kHashThreads =
+// 256 blocks per tile (as k_hash_local with G = 1), six CTAs per SM, so that
+// a CTA waiting at one of its barriers leaves five others to issue.  The requests that meet the tile are
 // tile_req[tile] .. tile_req[tile + 1]; their block and token offsets are
 // loaded into shared memory once, so a thread finds its request without a
 // dependent chain of global loads, and its token loads and power-table loads
@@ -545,7 +546,7 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local_vec(HashArgs a, con
 // global offsets instead.
 constexpr int kH16Req = 256;
 
-__global__ void __launch_bounds__(kHashThreads, 3) k_hash16(HashArgs a, const __grid_constant__ HashConsts c) {
+__global__ void __launch_bounds__(kHashThreads, 6) k_hash16(HashArgs a, const __grid_constant__ HashConsts c) {
   grid_dep_sync();
   __shared__ uint64_t s_boff[kH16Req + 1];
   __shared__ uint64_t s_toff[kH16Req + 1];
