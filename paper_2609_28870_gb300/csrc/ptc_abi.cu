@@ -126,10 +126,12 @@ __global__ void k_carry_err(const uint32_t* err, uint32_t n, DevStatus* st) {
   if (threadIdx.x < n && err[threadIdx.x]) atomicOr(&st->err, err[threadIdx.x]);
 }
 
-__global__ void k_copy_err(const DevStatus* st, uint32_t* slot, uint64_t* value_slot, uint32_t value_index) {
+__global__ void k_copy_err(const DevStatus* st, uint32_t* slot, uint64_t* value_slot, uint32_t value_index,
+                           uint32_t value_count) {
   grid_dep_sync();
   *slot = st->err;
-  if (value_slot) *value_slot = st->value[value_index];
+  if (value_slot)
+    for (uint32_t i = 0; i < value_count; ++i) value_slot[i] = st->value[value_index + i];
 }
 }  // namespace
 
@@ -248,10 +250,10 @@ ptc_status carry_errors(const uint32_t* err, uint32_t n, DevStatus* st, cudaStre
 }
 
 ptc_status defer_status(const DevStatus* dev, uint32_t* slot, cudaStream_t stream, uint64_t* value_slot,
-                        uint32_t value_index) {
+                        uint32_t value_index, uint32_t value_count) {
   if (cudaGetLastError() != cudaSuccess) return PTC_ERR_CUDA;
-  if (value_index >= 8) return PTC_ERR_INVALID_ARG;
-  PTC_KERNEL("k_copy_err", stream, k_copy_err, 1, 1, 0, dev, slot, value_slot, value_index);
+  if (value_index + value_count > 8) return PTC_ERR_INVALID_ARG;
+  PTC_KERNEL("k_copy_err", stream, k_copy_err, 1, 1, 0, dev, slot, value_slot, value_index, value_count);
   return PTC_OK;
 }
 

@@ -325,7 +325,8 @@ extern "C" size_t ptc_assign_ids_workspace_bytes(uint64_t n) { return ids_layout
 
 ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev, uint32_t* ids_out,
                         uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
-                        cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc) {
+                        cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc,
+                        uint64_t* nd_slot, uint32_t* err_slot, bool full_table) {
   const InsCarry ic = kc ? InsCarry{kc->carry, kc->lead, kc->tile_blocks} : InsCarry{nullptr, nullptr, 1};
   if (n_distinct_host_out == nullptr) return PTC_ERR_INVALID_ARG;
   *n_distinct_host_out = 0;
@@ -354,8 +355,13 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
   };
   if (!start()) return PTC_ERR_CUDA;
   DevStatus h{};
+  if (nd_slot && err_slot) {  // one attempt, nothing waits
+    const uint32_t lg = full_table ? L.log2m : small_table_log2(n);
+    if (n > 0 && !run(lg, lg < L.log2m ? kSmallProbeCap : ~0ULL)) return PTC_ERR_CUDA;
+    return defer_status(L.st, err_slot, s, nd_slot, 0, 2);
+  }
   if (n > 0) {
-    const uint32_t small = small_table_log2(n);
+    const uint32_t small = full_table ? L.log2m : small_table_log2(n);
     if (!run(small, small < L.log2m ? kSmallProbeCap : ~0ULL)) return PTC_ERR_CUDA;
     if (small < L.log2m) {
       const ptc_status rc1 = end_call(L.st, s, &h);

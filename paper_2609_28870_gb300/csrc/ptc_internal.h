@@ -89,6 +89,16 @@ struct NoHostAlloc {
 };
 
 // Wait for the call's work and translate the device status block.
+// The status a device error word stands for.
+inline ptc_status status_of(uint32_t e) {
+  if (e & kErrTimeout) return PTC_ERR_TIMEOUT;
+  if (e & kErrUnsorted) return PTC_ERR_UNSORTED;
+  if (e & kErrOverflow) return PTC_ERR_OVERFLOW;
+  if (e & kErrCollision) return PTC_ERR_HASH_COLLISION;
+  if (e & (kErrInvalid | kErrTableFull)) return PTC_ERR_INVALID_ARG;
+  return PTC_OK;
+}
+
 inline ptc_status end_call(const DevStatus* dev, cudaStream_t stream, DevStatus* host_copy) {
   if (cudaGetLastError() != cudaSuccess) return PTC_ERR_CUDA;
   DevStatus* pin = &host_stage()->st;
@@ -96,13 +106,7 @@ inline ptc_status end_call(const DevStatus* dev, cudaStream_t stream, DevStatus*
   if (cudaStreamSynchronize(stream) != cudaSuccess) return PTC_ERR_CUDA;
   *host_copy = *pin;
   timer_resolve();
-  uint32_t e = host_copy->err;
-  if (e & kErrTimeout) return PTC_ERR_TIMEOUT;
-  if (e & kErrUnsorted) return PTC_ERR_UNSORTED;
-  if (e & kErrOverflow) return PTC_ERR_OVERFLOW;
-  if (e & kErrCollision) return PTC_ERR_HASH_COLLISION;
-  if (e & (kErrInvalid | kErrTableFull)) return PTC_ERR_INVALID_ARG;
-  return PTC_OK;
+  return status_of(host_copy->err);
 }
 
 // Instead of waiting for a call's status, queue a copy of its error word to
@@ -119,9 +123,10 @@ ptc_status bitmap_ranks(const uint32_t* bits, uint32_t nwords, uint32_t* pre, ui
 
 // OR the n (at most 32) deferred error words at `err` into st->err.
 ptc_status carry_errors(const uint32_t* err, uint32_t n, DevStatus* st, cudaStream_t s);
-// With `value_slot`, value[value_index] of the status block is copied there too.
+// With `value_slot`, value[value_index .. value_index + value_count) of the
+// status block is copied there too.
 ptc_status defer_status(const DevStatus* dev, uint32_t* slot, cudaStream_t stream, uint64_t* value_slot = nullptr,
-                        uint32_t value_index = 0);
+                        uint32_t value_index = 0, uint32_t value_count = 1);
 
 // Streaming multiprocessors of the current device (persistent grids).
 inline int num_sms() {
@@ -168,15 +173,34 @@ ptc_status hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req
 // are used when `n_dev` (device memory) is given.  Error words at
 // `carry_err` join the call's own.  Reports the number used and D.  With
 // `kc` each key gets its tile's carry as it is read.
+// With `nd_slot` and `err_slot` (device memory) the call does not wait: it
+// makes one attempt with the small table and leaves D in nd_slot[0], the
+// number of keys used in nd_slot[1] and its error word in *err_slot (a
+// probe sequence that outran the small table shows as exactly
+// kErrTableFull; redo the stage then with `full_table`).
 ptc_status ids_impl(const ptc_u128* keys, uint64_t n_ub, const uint64_t* n_dev, uint32_t* ids_out,
                     uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
-                    cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc = nullptr);
+                    cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc = nullptr,
+                    uint64_t* nd_slot = nullptr, uint32_t* err_slot = nullptr, bool full_table = false);
 ptc_status stack_distance_view(const uint32_t* prev, uint64_t n, uint32_t* dist_out, int method, void* ws,
                                size_t ws_bytes, cudaStream_t s, RunsView* view, uint32_t* defer_err);
 // Stage b as ptc_reuse_indices does it (ptc_reuse.cu); with `defer_err` the
-// final wait is replaced by defer_status.
+// final wait is replaced by defer_status.  With `din`, stage a2 has not
+// waited: n and n_distinct are upper bounds, the kernels before this stage's
+// own wait read the real ones from din->nd (nd[0] = D, nd[1] = accesses),
+// and that wait reports them, with stage a2's error word, in *hout.  If that
+// word is not 0 the call returns PTC_OK at once and its results are void.
+struct ReuseDevIn {
+  const uint64_t* nd;
+  const uint32_t* ids_err;
+};
+struct ReuseHostOut {
+  uint64_t n = 0, D = 0;
+  uint32_t ids_err = 0;
+};
 ptc_status reuse_view(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev_out, uint32_t* next_out,
-                      void* ws, size_t ws_bytes, cudaStream_t s, uint32_t* defer_err);
+                      void* ws, size_t ws_bytes, cudaStream_t s, uint32_t* defer_err, const ReuseDevIn* din = nullptr,
+                      ReuseHostOut* hout = nullptr);
 // Stage d (ptc_curves.cu); with `runs` (from stack_distance_view) the curves
 // come from the runs instead of a pass over every distance.
 ptc_status curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,

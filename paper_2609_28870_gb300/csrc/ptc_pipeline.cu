@@ -17,8 +17,9 @@ struct PipeLayout {
   size_t scratch_bytes;
   void* curves;
   size_t curves_bytes;
-  uint32_t* defer;  // error words of stages a1, b and c, read with a later stage's
+  uint32_t* defer;  // error words of stages a1, b, c and a2, read with a later stage's
   uint64_t* n_slot;  // N as stage a1 left it, for stage a2
+  uint64_t* nd_slot;  // D and N as stage a2 left them, for stage b
   ulonglong2* carry;  // per hash tile: the carry stage a2 adds to the keys (when they are not returned)
   uint32_t* lead;
   size_t total;
@@ -48,8 +49,9 @@ PipeLayout pipe_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   L.scratch = cv.take<unsigned char>(L.scratch_bytes);
   L.curves_bytes = ptc_curves_workspace_bytes(n_tok / B, n_req, n_cap);
   L.curves = cv.take<unsigned char>(L.curves_bytes);
-  L.defer = cv.take<uint32_t>(3);
+  L.defer = cv.take<uint32_t>(4);
   L.n_slot = cv.take<uint64_t>(1);
+  L.nd_slot = cv.take<uint64_t>(2);
   const uint64_t ct = keys ? 1 : ptc::hash_carry_tiles(n_tok, B);
   L.carry = cv.take<ulonglong2>(ct);
   L.lead = cv.take<uint32_t>(ct);
@@ -90,10 +92,12 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
   *n_access_host_out = 0;
   *n_distinct_host_out = 0;
   cudaStream_t s = (cudaStream_t)stream;
-  // Stages a1, b and c do not wait for their own status: a1's error word and
-  // N go to device slots that stage a2 reads (its grids cover N's upper
-  // bound, n_tok / B); b's and c's error words are read with stage d's.
-  if (ptc::fill_async(L.defer, 0u, 3 * sizeof(uint32_t), s) != PTC_OK) return PTC_ERR_CUDA;
+  // Stages a1, a2, b and c do not wait for their own status.  a1's error
+  // word and N go to device slots that stage a2 reads (its grids cover N's
+  // upper bound, n_tok / B); a2's error word, N and D go to slots that stage
+  // b's first kernels read, and reach the host with stage b's own wait; b's
+  // and c's error words are read with stage d's.
+  if (ptc::fill_async(L.defer, 0u, 4 * sizeof(uint32_t), s) != PTC_OK) return PTC_ERR_CUDA;
   // keys the caller does not take skip their carry pass: stage a2 adds the
   // carry as it reads them
   ptc::KeyCarry kc{L.carry, L.lead, 1};
@@ -101,14 +105,29 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
   ptc_status rc = ptc::hash_impl(tokens, n_tok, req_tok_off, req_ts_us, n_req, block_size, seed, keys, cap, blk,
                                  &unused, L.scratch, L.scratch_bytes, s, L.n_slot, &L.defer[0], kcp);
   if (rc != PTC_OK) return rc;
-  rc = ptc::ids_impl(keys, cap, L.n_slot, ids, &n, &d, L.scratch, L.scratch_bytes, s, &L.defer[0], 1, kcp);
-  *n_access_host_out = n;
-  *n_distinct_host_out = d;
+  rc = ptc::ids_impl(keys, cap, L.n_slot, ids, &n, &d, L.scratch, L.scratch_bytes, s, &L.defer[0], 1, kcp,
+                     L.nd_slot, &L.defer[3]);
   if (rc != PTC_OK) return rc;
+  const ptc::ReuseDevIn din{L.nd_slot, &L.defer[3]};
+  ptc::ReuseHostOut hout;
+  rc = ptc::reuse_view(ids, cap, cap, prev, next, L.scratch, L.scratch_bytes, s, &L.defer[1], &din, &hout);
+  *n_access_host_out = n = hout.n;
+  *n_distinct_host_out = d = hout.D;
+  if (rc != PTC_OK) return rc;
+  if (hout.ids_err) {
+    // stage a2's small table overflowed (or a1 / a2 failed): redo a2 with the
+    // full table, waiting for it, then stage b with the host's N and D
+    if (hout.ids_err != ptc::kErrTableFull) return ptc::status_of(hout.ids_err);
+    rc = ptc::ids_impl(keys, cap, L.n_slot, ids, &n, &d, L.scratch, L.scratch_bytes, s, &L.defer[0], 1, kcp, nullptr,
+                       nullptr, true);
+    *n_access_host_out = n;
+    *n_distinct_host_out = d;
+    if (rc != PTC_OK) return rc;
+    if (n > 0) rc = ptc::reuse_view(ids, n, d, prev, next, L.scratch, L.scratch_bytes, s, &L.defer[1]);
+    if (rc != PTC_OK) return rc;
+  }
   ptc::RunsView runs;
   if (n > 0) {
-    rc = ptc::reuse_view(ids, n, d, prev, next, L.scratch, L.scratch_bytes, s, &L.defer[1]);
-    if (rc != PTC_OK) return rc;
     rc = ptc::stack_distance_view(prev, n, dist, PTC_SD_AUTO, L.scratch, L.scratch_bytes, s, &runs, &L.defer[2]);
     if (rc != PTC_OK) return rc;
   }

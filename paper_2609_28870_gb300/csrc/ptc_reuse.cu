@@ -42,7 +42,9 @@ constexpr int kRunTile = kIT * kRunPer;
 
 struct IrArgs {
   const uint32_t* ids;
-  uint32_t n, D, ntiles;
+  uint32_t n, D, ntiles;  // with nd: n is an upper bound, and D and the used n come from nd
+  const uint64_t* nd;     // device: nd[0] = D, nd[1] = accesses (stage a2 did not wait), or null
+  const uint32_t* ext_err;  // device: stage a2's error word, reported in value[6], or null
   uint32_t* tcnt;
   uint32_t* tpre;     // runs before each tile; tpre[ntiles] = number of runs
   uint32_t* done;
@@ -115,9 +117,26 @@ __device__ __forceinline__ void id_starts(const IrArgs& a, uint32_t base, uint32
   }
 }
 
-__global__ void __launch_bounds__(kIT) k_ir_count(IrArgs a) {
+// n and D from the device when stage a2 did not wait for them.
+__device__ __forceinline__ IrArgs resolved(const IrArgs& in) {
+  IrArgs a = in;
+  if (a.nd) {
+    const uint64_t nn = a.nd[1], d = a.nd[0];
+    a.n = nn < a.n ? (uint32_t)nn : a.n;
+    a.D = d < a.n ? (uint32_t)d : a.n;
+  }
+  return a;
+}
+
+__global__ void __launch_bounds__(kIT) k_ir_count(IrArgs a0) {
   grid_dep_sync();
   __shared__ uint32_t s_w[kIT / 32];
+  const IrArgs a = resolved(a0);
+  if (a0.nd && blockIdx.x == 0 && threadIdx.x == 0) {
+    a.st->value[4] = a0.nd[1];
+    a.st->value[5] = a0.nd[0];
+    a.st->value[6] = a0.ext_err ? *a0.ext_err : 0u;
+  }
   const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   uint32_t id[kIR], left[kIR], words[kIR];
   bool bad = false;
@@ -134,9 +153,10 @@ __global__ void __launch_bounds__(kIT) k_ir_count(IrArgs a) {
   if (threadIdx.x == 0) a.st->value[1] = R;
 }
 
-__global__ void __launch_bounds__(kIT) k_ir_mark(IrArgs a) {
+__global__ void __launch_bounds__(kIT) k_ir_mark(IrArgs a0) {
   grid_dep_sync();
   __shared__ uint32_t s_w[kIT / 32];
+  const IrArgs a = resolved(a0);
   if (*(volatile uint32_t*)&a.st->err) return;  // ids >= D: reported, nothing is indexed by them
   const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const uint32_t base = tile * kITile + w * (32 * kIR);
@@ -386,7 +406,8 @@ uint32_t bits_for(uint64_t v) {  // bits to hold values below v
 }
 
 ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* prev_out, uint32_t* next_out, void* ws,
-                         size_t ws_bytes, cudaStream_t s, bool forced, uint32_t* defer_err = nullptr) {
+                         size_t ws_bytes, cudaStream_t s, bool forced, uint32_t* defer_err = nullptr,
+                         const ReuseDevIn* din = nullptr, ReuseHostOut* hout = nullptr) {
   const ReuseLayout L = reuse_layout(ws, n, D, forced);
   if (!ws_ok(ws, ws_bytes, L.total)) return PTC_ERR_WORKSPACE;
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
@@ -403,6 +424,8 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
   a.rec_x = L.rec_x;
   a.cut = L.cut;
   a.st = L.st;
+  a.nd = din ? din->nd : nullptr;
+  a.ext_err = din ? din->ids_err : nullptr;
   PTC_KERNEL("k_ir_count", s, k_ir_count, L.ntiles, kIT, 0, a);
   PTC_KERNEL("k_ir_mark", s, k_ir_mark, L.ntiles, kIT, 0, a);
   PTC_KERNEL("k_bm_count", s, k_bm_count, L.btiles, kIT, 0, L.cut, L.nwords, L.btiles, L.btcnt, L.btpre, &L.done[1], L.st);
@@ -422,8 +445,18 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
   ia.st = L.st;
   const uint32_t g1 = L.rtiles_max < (uint32_t)(2 * num_sms()) ? L.rtiles_max : (uint32_t)(2 * num_sms());
   PTC_KERNEL("k_ir_inc1", s, k_ir_inc1, g1, kIT, 0, ia);
-  DevStatus h;
+  DevStatus h{};
   ptc_status rc = end_call(L.st, s, &h);
+  if (din) {  // n and D were bounds: the real ones, and stage a2's status, arrive with this wait
+    hout->n = h.value[4];
+    hout->D = h.value[5];
+    hout->ids_err = (uint32_t)h.value[6];
+    if (rc == PTC_ERR_CUDA) return rc;
+    if (hout->ids_err) return PTC_OK;  // this stage's results are void; the caller redoes a2 and b
+    n = hout->n;
+    D = hout->D;
+    if (rc == PTC_OK && (n == 0 || D == 0)) return PTC_OK;  // no accesses: nothing to link
+  }
   if (rc != PTC_OK) return rc;
   const uint64_t R = h.value[1], M = h.value[2], K = h.value[3];
   if (K > L.kcap || R == 0 || M < 2) {
@@ -453,11 +486,13 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
 }  // namespace
 
 ptc_status reuse_view(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev_out, uint32_t* next_out,
-                      void* ws, size_t ws_bytes, cudaStream_t s, uint32_t* defer_err) {
+                      void* ws, size_t ws_bytes, cudaStream_t s, uint32_t* defer_err, const ReuseDevIn* din,
+                      ReuseHostOut* hout) {
   if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
   if (n == 0) return PTC_OK;
   if (!ids || !prev_out || !next_out || n_distinct == 0 || n_distinct > n) return PTC_ERR_INVALID_ARG;
-  return reuse_by_runs(ids, n, n_distinct, prev_out, next_out, ws, ws_bytes, s, false, defer_err);
+  if (din && !hout) return PTC_ERR_INVALID_ARG;
+  return reuse_by_runs(ids, n, n_distinct, prev_out, next_out, ws, ws_bytes, s, false, defer_err, din, hout);
 }
 
 }  // namespace ptc

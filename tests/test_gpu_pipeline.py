@@ -190,3 +190,24 @@ def test_pipeline_plan_runs_again_and_on_refilled_buffers():
     second = plan.run().result()
     o = gu.oracle_run(tr_b, B, caps)
     assert {k: second[k] for k in keys} == {k: o[k] for k in keys}
+
+
+def test_pipeline_redoes_stage_a2_when_the_small_table_overflows():
+    """ptc_pipeline does not wait for stage a2: its first attempt uses the
+    small table (N/3 slots); when every block is distinct that table
+    overflows, stage b's wait reports it, and the pipeline redoes a2 with the
+    full table and b with the host's N and D."""
+    from tests import gpu_util as gu
+    rng = np.random.default_rng(77)
+    reqs = [list(rng.integers(0, 2**31, size=16 * 500)) for _ in range(40)]
+    tr = tracegen.from_lists(reqs)
+    B = 16
+    caps = [1, 100, 5000, 30000]
+    o = gu.oracle_run(tr, B, caps)
+    assert o["n_distinct"] == o["n_access"] == 20000
+    for with_outputs in (True, False):
+        g = _run(tr, B, caps, with_outputs=with_outputs)
+        for k in ("n_access", "n_distinct", "hits", "saved", "total_cost"):
+            assert g[k] == o[k], (k, with_outputs)
+        if with_outputs:
+            gu.assert_same(g, o)
