@@ -33,8 +33,8 @@
 namespace ptc {
 namespace {
 
-constexpr int kOffThreads = 512;
-constexpr int kOffPer = 8;
+constexpr int kOffThreads = 256;  // one request per thread: the grid spreads over many SMs
+constexpr int kOffPer = 1;
 constexpr int kOffTile = kOffThreads * kOffPer;
 
 constexpr int kHashThreads = 256;
@@ -44,7 +44,7 @@ constexpr int kWinWords = kWinTokens + kWinTokens / 16;
 constexpr int kEpochOffsets = 1;
 
 // ---------------------------------------------------------------- block scans
-// Exclusive sum over a CTA of kOffThreads (512) threads; returns the CTA total in *total.
+// Exclusive sum over a CTA of kOffThreads threads; returns the CTA total in *total.
 __device__ __forceinline__ uint64_t cta_exclusive_sum(uint64_t v, uint64_t* total) {
   __shared__ uint64_t s_w[kOffThreads / 32];
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -100,7 +100,15 @@ __global__ void __launch_bounds__(kOffThreads) k_block_offsets(const uint64_t* _
     }
   }
   if (err) raise_err(st, err);
-  if (kmax) atomicMax((unsigned long long*)&st->value[1], (unsigned long long)kmax);
+  {  // the longest request: one atomic per warp
+    uint64_t m = kmax;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const uint64_t y = __shfl_xor_sync(kFull, m, o);
+      m = y > m ? y : m;
+    }
+    if ((threadIdx.x & 31) == 0 && m) atomicMax((unsigned long long*)&st->value[1], (unsigned long long)m);
+  }
   uint64_t total;
   uint64_t excl = cta_exclusive_sum(local, &total);
   const uint64_t base = lookback_sum_cta(lb, tile, total, kEpochOffsets, st);
@@ -128,6 +136,8 @@ __global__ void __launch_bounds__(kOffThreads) k_block_offsets(const uint64_t* _
 // ---------------------------------------------------------------- powers
 // tables[(b*2 + w) * 65536 + e] for base b in {0,1} and
 //   w = 0: u_b^(B e)          w = 1: u_b^(B 65536 e)
+constexpr int kPowChunk = 8;  // powers per thread: short dependent chains
+
 struct PowBases {
   uint64_t base[4];
 };
@@ -136,17 +146,17 @@ struct PowBases {
 // most the longest request's block count minus one (st->value[1]).
 __global__ void k_pow_tables(PowBases pb, uint64_t* __restrict__ tables, const DevStatus* st) {
   grid_dep_sync();
-  const uint32_t gid = blockIdx.x * blockDim.x + threadIdx.x;  // 4 tables x 1024 chunks of 64
-  const uint32_t t = gid >> 10, chunk = gid & 1023;
+  const uint32_t gid = blockIdx.x * blockDim.x + threadIdx.x;  // 4 tables x 8192 chunks of kPowChunk
+  const uint32_t t = gid >> 13, chunk = gid & 8191;
   if (t >= 4) return;
   const uint64_t kmax = st->value[1];
   const uint64_t need = (t & 1) ? (kmax >> 16) : (kmax < 65535 ? kmax : 65535);
   const uint64_t base = pb.base[t];
-  const uint64_t e0 = (uint64_t)chunk * 64;
+  const uint64_t e0 = (uint64_t)chunk * kPowChunk;
   if (e0 > need) return;
   uint64_t v = p61_pow(base, e0);
   uint64_t* out = tables + (uint64_t)t * 65536 + e0;
-  for (int i = 0; i < 64; ++i) {
+  for (int i = 0; i < kPowChunk; ++i) {
     out[i] = v;
     v = p61_mul(v, base);
   }
@@ -960,7 +970,7 @@ ptc_status ptc::hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t
     }
     for (int q = 0; q < 32; ++q) hc.sub_mul[b][q] = p61_pow(u, 16ULL * q);
   }
-  PTC_KERNEL("k_pow_tables", s, k_pow_tables, (4 * 1024) / 256, 256, 0, pb, L.tables, L.st);
+  PTC_KERNEL("k_pow_tables", s, k_pow_tables, (4 * 8192) / 256, 256, 0, pb, L.tables, L.st);
 
   HashArgs a;
   a.tokens = tokens;
