@@ -821,6 +821,10 @@ __global__ void __launch_bounds__(kChainWarps * 32) k_hash_chain(ulonglong2* __r
 // The same carries as k_hash_chain, left for the keys' reader instead of
 // added to the keys (a pipeline that does not return the keys saves the
 // pass over them): carry[t] and lead[t] per tile, 0 where no key needs one.
+// A warp takes kCarryPer consecutive tiles: the carry into the first from a
+// look-back over the aggregates before it (all written, so nothing waits),
+// then a segmented scan of its own tiles' aggregates across kCarryPer lanes.
+constexpr int kCarryPer = 8;
 __global__ void __launch_bounds__(kChainWarps * 32) k_hash_carry(const HashCarry* __restrict__ tile_agg,
                                                                  const uint32_t* __restrict__ tile_lead, uint32_t TB,
                                                                  const DevStatus* st, uint64_t keys_cap,
@@ -828,15 +832,15 @@ __global__ void __launch_bounds__(kChainWarps * 32) k_hash_carry(const HashCarry
                                                                  uint32_t* __restrict__ lead_out) {
   grid_dep_sync();
   const uint32_t lane = threadIdx.x & 31;
-  const uint32_t tile = blockIdx.x * kChainWarps + (threadIdx.x >> 5);
-  if (tile >= ntiles) return;
+  const uint32_t t0 = (blockIdx.x * kChainWarps + (threadIdx.x >> 5)) * kCarryPer;
+  if (t0 >= ntiles) return;
   uint64_t N = st->value[0];
   if (N > keys_cap) N = keys_cap;
-  const uint64_t b0 = (uint64_t)tile * TB;
-  const uint32_t lead = (b0 >= N || tile == 0) ? 0u : tile_lead[tile];
-  uint64_t c0 = 0, c1 = 0;
-  if (lead) {
-    for (int64_t base = (int64_t)tile - 1; base >= 0; base -= 32) {
+  const uint64_t live = (N + TB - 1) / TB;  // tiles that hold blocks
+  const SegSumOp op;
+  HashCarry cin{0, 0, 0};
+  if (t0 > 0 && t0 < live) {
+    for (int64_t base = (int64_t)t0 - 1; base >= 0; base -= 32) {
       const int64_t idx = base - (int64_t)lane;
       HashCarry g{0, 0, 0};
       if (idx >= 0) g = tile_agg[idx];
@@ -848,14 +852,33 @@ __global__ void __launch_bounds__(kChainWarps * 32) k_hash_carry(const HashCarry
         v0 = p61_add(v0, __shfl_xor_sync(kFull, v0, o));
         v1 = p61_add(v1, __shfl_xor_sync(kFull, v1, o));
       }
-      c0 = p61_add(c0, v0);
-      c1 = p61_add(c1, v1);
+      cin.v0 = p61_add(cin.v0, v0);
+      cin.v1 = p61_add(cin.v1, v1);
       if (heads) break;
     }
   }
-  if (lane == 0) {
-    carry[tile] = make_ulonglong2(c0, c1);
-    lead_out[tile] = lead;
+  const uint32_t t = t0 + lane;
+  HashCarry g{0, 0, 0};
+  if (lane < kCarryPer && t < live) g = tile_agg[t];
+#pragma unroll
+  for (int o = 1; o < kCarryPer; o <<= 1) {  // inclusive segmented sums over lanes 0 .. kCarryPer - 1
+    HashCarry y;
+    y.v0 = __shfl_up_sync(kFull, g.v0, o);
+    y.v1 = __shfl_up_sync(kFull, g.v1, o);
+    y.f = __shfl_up_sync(kFull, g.f, o);
+    if (lane >= (uint32_t)o) g = op(y, g);
+  }
+  HashCarry before;  // this warp's tiles before tile t
+  before.v0 = __shfl_up_sync(kFull, g.v0, 1);
+  before.v1 = __shfl_up_sync(kFull, g.v1, 1);
+  before.f = __shfl_up_sync(kFull, g.f, 1);
+  if (lane == 0) before = HashCarry{0, 0, 0};
+  const HashCarry c = op(cin, before);
+  if (lane < kCarryPer && t < ntiles) {
+    const uint64_t b0 = (uint64_t)t * TB;
+    const uint32_t lead = (b0 >= N || t == 0) ? 0u : tile_lead[t];
+    carry[t] = lead ? make_ulonglong2(c.v0, c.v1) : make_ulonglong2(0, 0);
+    lead_out[t] = lead;
   }
 }
 
@@ -1000,7 +1023,7 @@ ptc_status ptc::hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t
       default: launch_hash<32>(grid, s, a, hc, full); break;
     }
     if (carry) {
-      PTC_KERNEL("k_hash_carry", s, k_hash_carry, ceil_div_u32(grid, kChainWarps), kChainWarps * 32, 0, L.tile_agg,
+      PTC_KERNEL("k_hash_carry", s, k_hash_carry, ceil_div_u32(grid, kChainWarps * kCarryPer), kChainWarps * 32, 0, L.tile_agg,
                  L.tile_lead, kHashThreads / G, L.st, keys_cap, grid, carry->carry, carry->lead);
       carry->tile_blocks = kHashThreads / G;
     } else {
