@@ -15,6 +15,9 @@ Functions and the passages they restate:
   move-to-front stack and by Bennett-Kruskal counting.
 * ``lru_curves`` — direct LRU simulation per capacity (Sec. 3.1-3.2) with
   prefix-contiguous hits (Sec. 2.2) and compute saved (Sec. 5.2, App. C).
+* ``trace_stats`` — Sec. 4.1-4.3 and App. B: per-category block counts,
+  frequency, lifetime and reuse-interval histograms, session lengths and
+  durations, and reuses reachable within each capacity.
 * ``prefix_hash`` — the polynomial prefix key the GPU path writes,
   sum_t (tok_t + 1) u^(t+1) mod 2^61 - 1 at two seeded bases, token by token.
 * ``run`` — all of the above on one trace.
@@ -73,6 +76,8 @@ def _load():
         lib.orc_lru_curves.restype = i32
         lib.orc_lru_curves.argtypes = [vp, vp, u32, u32, i32, u64, u64, vp, u32, i32, vp, vp, vp, vp, vp]
         lib.orc_prefix_hash.argtypes = [vp, vp, u32, u32, u64, vp]
+        lib.orc_trace_stats.restype = i32
+        lib.orc_trace_stats.argtypes = [vp, u64, u64, vp, vp, vp, u32, u64, vp, vp, u32] + [vp] * 13
         _lib = lib
     return _lib
 
@@ -150,6 +155,45 @@ def prefix_hash(tokens, req_tok_off, B: int, seed: int) -> np.ndarray:
     keys = np.empty((n, 2), dtype=np.uint64)
     _load().orc_prefix_hash(_p(tok), _p(off), off.shape[0] - 1, int(B), int(seed) & (2**64 - 1), _p(keys))
     return keys
+
+
+# Shapes of the trace statistics: category-major histograms have 3 rows
+# (0 shared across sessions, 1 session history, 2 single-turn); log2 bins are
+# the bit length of the value (65 bins); freq has 256 exact bins with the
+# blocks used 256 times or more in bin 0.
+STAT_SHAPES = dict(blocks=(3,), accesses=(3,), freq=(3, 256), freq_log2=(3, 65), reuse_us=(3, 65),
+                   lifetime_us=(3, 65), reuse_by_freq=(65, 65), lifetime_by_freq=(65, 65), dist_log2=(65,),
+                   sess_requests=(65,), sess_duration_us=(65,))
+STAT_SCALARS = ("n_access", "n_distinct", "n_reuse", "n_sessions", "n_multi_sessions")
+
+
+def trace_stats(ids, n_distinct: int, req_blk_off, req_ts_us, req_session, n_session: int, dist=None,
+                caps=None) -> dict:
+    """Trace statistics of Sec. 4.1-4.3 and App. B (see orc_trace_stats):
+    uint64 histograms named as in STAT_SHAPES, the STAT_SCALARS, and
+    ``reach`` (reuses with stack distance <= caps[g]) when dist is given."""
+    ids, bo = _c(ids, np.uint32), _c(req_blk_off, np.uint64)
+    ts, ses = _c(req_ts_us, np.int64), _c(req_session, np.uint64)
+    caps = _c([] if caps is None else caps, np.uint64)
+    out = {k: np.zeros(v, dtype=np.uint64) for k, v in STAT_SHAPES.items()}
+    reach = np.zeros(max(caps.shape[0], 1), dtype=np.uint64)
+    scal = np.zeros(len(STAT_SCALARS), dtype=np.uint64)
+    dptr = None
+    if dist is not None:
+        dist = _c(dist, np.uint32)
+        dptr = _p(dist)
+    rc = _load().orc_trace_stats(_p(ids), ids.shape[0], int(n_distinct), _p(bo), _p(ts), _p(ses),
+                                 bo.shape[0] - 1, int(n_session), dptr, _p(caps), caps.shape[0],
+                                 *[_p(out[k]) for k in list(STAT_SHAPES)[:9]], _p(reach),
+                                 _p(out["sess_requests"]), _p(out["sess_duration_us"]), _p(scal))
+    if rc == 1:
+        raise ValueError("malformed trace (ids, sessions or offsets)")
+    if rc == 2:
+        raise ValueError("request timestamps decrease")
+    out.update({k: int(v) for k, v in zip(STAT_SCALARS, scal)})
+    if dist is not None:
+        out["reach"] = reach[: caps.shape[0]]
+    return out
 
 
 def run(tokens, req_tok_off, B: int, caps, kind: int = COST_MEASURED, f_lin: int = F_LIN, f_attn: int = F_ATTN,

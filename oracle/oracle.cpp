@@ -23,6 +23,10 @@
 //        orc_sd_fenwick (Bennett & Kruskal 1975 counting), two independent ways.
 //   * Belady's next use (Sec. 3.2, 5.2).  -> orc_reuse: previous and next
 //     access of the same block.
+//   * Sec. 4.1-4.3 and App. B: block lifetimes, frequencies, reuse intervals,
+//     block categories, session lengths and reuses reachable within a
+//     capacity.  -> orc_trace_stats: two passes over the access stream with
+//        per-block arrays, then loops over blocks and sessions.
 // The GPU path's block keys are polynomial hashes of each block's whole
 // prefix, sum over its tokens of (tok_t + 1) u^(t+1) mod 2^61 - 1 at two
 // seeded bases u; orc_prefix_hash evaluates that sum token by token so the
@@ -316,6 +320,155 @@ void orc_prefix_hash(const uint32_t* tokens, const uint64_t* req_tok_off, uint32
       }
     }
   }
+}
+
+}  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Trace characterization (Sec. 4.1-4.3; App. B).  Each access of block d in
+// request r happens at the request's arrival time ts[r] and belongs to the
+// request's session sess[r].  Per block d: its frequency (number of
+// accesses), its lifetime (time of its last access minus time of its first,
+// zero for a block used once), and its category.  Per reuse (every access but
+// a block's first): the reuse interval, its time minus the time of the
+// previous access of the same block.  Per session: its request count and its
+// duration (last minus first request time).
+//
+// Categories (Sec. 4.1 names three, by message role, which a token trace does
+// not carry; the reading used here classifies by the sessions a block appears
+// in):
+//   0  shared across sessions: the block appears in two or more sessions and
+//      at least one of them has two or more requests (system prompts reused
+//      across conversations);
+//   1  session history: the block appears in exactly one session, and that
+//      session has two or more requests;
+//   2  single-turn: every session the block appears in has one request.
+// Histograms bin a value x >= 0 by the bit length of x (0 for x = 0, else
+// floor(log2 x) + 1), 65 bins.  freq[c][k] counts blocks used exactly k times
+// for 1 <= k < 256, and freq[c][0] those used 256 times or more.
+// reach[g] counts reuses whose LRU stack distance is at most cap[g] (App. B:
+// reuses reachable within a cache of cap[g] blocks); dist may be NULL.
+// Returns 0, or 1 for malformed input (an id >= D, a session label >=
+// n_session, offsets that are not a partition of [0, n)), or 2 if the
+// timestamps decrease.
+// ---------------------------------------------------------------------------
+namespace {
+int bit_length(uint64_t x) {
+  int b = 0;
+  while (x != 0) {
+    ++b;
+    x >>= 1;
+  }
+  return b;
+}
+}  // namespace
+
+extern "C" {
+
+int orc_trace_stats(const uint32_t* ids, uint64_t n, uint64_t D, const uint64_t* req_blk_off, const int64_t* ts,
+                    const uint64_t* sess, uint32_t n_req, uint64_t n_session, const uint32_t* dist,
+                    const uint64_t* caps, uint32_t n_cap, uint64_t* blocks, uint64_t* accesses, uint64_t* freq,
+                    uint64_t* freq_log2, uint64_t* reuse_us, uint64_t* lifetime_us, uint64_t* reuse_by_freq,
+                    uint64_t* lifetime_by_freq, uint64_t* dist_log2, uint64_t* reach, uint64_t* sess_requests,
+                    uint64_t* sess_duration_us, uint64_t* scalars) {
+  // inputs
+  if (req_blk_off[0] != 0 || req_blk_off[n_req] != n) return 1;
+  for (uint32_t r = 0; r < n_req; ++r) {
+    if (req_blk_off[r + 1] < req_blk_off[r] || sess[r] >= n_session) return 1;
+    if (r > 0 && ts[r] < ts[r - 1]) return 2;
+  }
+  for (uint64_t i = 0; i < n; ++i)
+    if (ids[i] >= D) return 1;
+
+  // sessions: request count, first and last request time
+  std::vector<uint64_t> s_req(n_session, 0);
+  std::vector<int64_t> s_first(n_session, 0), s_last(n_session, 0);
+  for (uint32_t r = 0; r < n_req; ++r) {
+    uint64_t s = sess[r];
+    if (s_req[s] == 0) s_first[s] = ts[r];
+    s_last[s] = ts[r];
+    ++s_req[s];
+  }
+
+  // first pass over the accesses in stream order: frequency, first and last
+  // access time, the first session seen, and the two category conditions
+  std::vector<uint64_t> cnt(D, 0);
+  std::vector<int64_t> t_first(D, 0), t_last(D, 0);
+  std::vector<uint64_t> first_sess(D, 0);
+  std::vector<char> in_multi(D, 0), in_two(D, 0);
+  for (uint32_t r = 0; r < n_req; ++r) {
+    for (uint64_t i = req_blk_off[r]; i < req_blk_off[r + 1]; ++i) {
+      uint32_t d = ids[i];
+      if (cnt[d] == 0) {
+        t_first[d] = ts[r];
+        first_sess[d] = sess[r];
+      } else if (first_sess[d] != sess[r]) {
+        in_two[d] = 1;
+      }
+      t_last[d] = ts[r];
+      if (s_req[sess[r]] >= 2) in_multi[d] = 1;
+      ++cnt[d];
+    }
+  }
+  auto category = [&](uint32_t d) { return in_multi[d] ? (in_two[d] ? 0 : 1) : 2; };
+
+  // per block
+  for (uint64_t d = 0; d < D; ++d) {
+    if (cnt[d] == 0) return 1;  // ids must be dense
+    int c = category((uint32_t)d);
+    uint64_t life = (uint64_t)(t_last[d] - t_first[d]);
+    blocks[c] += 1;
+    accesses[c] += cnt[d];
+    freq[c * 256 + (cnt[d] < 256 ? cnt[d] : 0)] += 1;
+    freq_log2[c * 65 + bit_length(cnt[d])] += 1;
+    lifetime_us[c * 65 + bit_length(life)] += 1;
+    lifetime_by_freq[bit_length(cnt[d]) * 65 + bit_length(life)] += 1;
+  }
+
+  // second pass: reuse intervals, binned by the category and the frequency of
+  // the block (both final after the first pass)
+  std::vector<char> seen(D, 0);
+  std::vector<int64_t> t_prev(D, 0);
+  uint64_t n_reuse = 0;
+  for (uint32_t r = 0; r < n_req; ++r) {
+    for (uint64_t i = req_blk_off[r]; i < req_blk_off[r + 1]; ++i) {
+      uint32_t d = ids[i];
+      if (seen[d]) {
+        uint64_t gap = (uint64_t)(ts[r] - t_prev[d]);
+        reuse_us[category(d) * 65 + bit_length(gap)] += 1;
+        reuse_by_freq[bit_length(cnt[d]) * 65 + bit_length(gap)] += 1;
+        ++n_reuse;
+      }
+      seen[d] = 1;
+      t_prev[d] = ts[r];
+    }
+  }
+
+  // stack distances of the reuses
+  if (dist != nullptr) {
+    for (uint64_t i = 0; i < n; ++i) {
+      if (dist[i] == NONE) continue;
+      dist_log2[bit_length(dist[i])] += 1;
+      for (uint32_t g = 0; g < n_cap; ++g)
+        if (dist[i] <= caps[g]) reach[g] += 1;
+    }
+  }
+
+  // per session
+  uint64_t used = 0, multi = 0;
+  for (uint64_t s = 0; s < n_session; ++s) {
+    if (s_req[s] == 0) continue;
+    ++used;
+    if (s_req[s] >= 2) ++multi;
+    sess_requests[bit_length(s_req[s])] += 1;
+    sess_duration_us[bit_length((uint64_t)(s_last[s] - s_first[s]))] += 1;
+  }
+  scalars[0] = n;
+  scalars[1] = D;
+  scalars[2] = n_reuse;
+  scalars[3] = used;
+  scalars[4] = multi;
+  return 0;
 }
 
 }  // extern "C"
