@@ -11,6 +11,10 @@
  *     -> ptc_reuse_indices   previous / next use of each block Sec. 3.2, 5.2 (Belady's next access)
  *     -> ptc_stack_distance  LRU stack distance of each access App. B ("reuses reachable within C")
  *     -> ptc_curves          hits and compute saved per C      Sec. 3.2 (hit ratio), Sec. 5.2 (compute savings)
+ *   and, over the same arrays,
+ *        ptc_trace_stats     lifetimes, reuse intervals, frequency, block categories,
+ *                            session lengths, reuses reachable within C
+ *                                                              Sec. 4.1-4.3, App. B
  *
  * Conventions shared by every call
  *   - Pointers are caller-owned DEVICE memory unless the name ends in _host.
@@ -262,6 +266,77 @@ ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const uint64_t* 
                         uint64_t* n_access_host_out, uint64_t* n_distinct_host_out, uint64_t* hits_host_out,
                         ptc_u128* saved_host_out, ptc_u128* total_cost_host_out, void* ws, size_t ws_bytes,
                         void* stream);
+
+/*
+ * ptc_trace_stats — trace characterization over the arrays of the path
+ * (Sec. 4.1 block lifetimes, categories and the one-hit share; Sec. 4.2 reuse
+ * intervals; Sec. 4.3 frequency, reuse interval and lifetime against
+ * frequency, requests per session; App. B reuses reachable within a cache of
+ * C blocks).  Access i of request r happens at req_ts_us[r] in session
+ * req_session[r].  For a block d:
+ *   frequency f_d    its number of accesses
+ *   lifetime         time of its last access minus time of its first (0 if used once)
+ *   category c_d     0 shared across sessions: d appears in two or more sessions,
+ *                      at least one of which has two or more requests
+ *                    1 session history: d appears in exactly one session, and
+ *                      that session has two or more requests
+ *                    2 single-turn: every session d appears in has one request
+ *                    (the paper's three categories are by message role, which a
+ *                    token trace does not carry; sessions stand in for roles)
+ * and for a reuse (an access with a previous access of its block) the reuse
+ * interval, its time minus the time of that previous access.  bin(x) is the
+ * bit length of x: 0 for x = 0, else floor(log2 x) + 1, in [0, 64].
+ * Every field of ptc_trace_summary counts:
+ *   blocks[c], accesses[c]   blocks of category c and their accesses
+ *   freq[c][k]               blocks of category c used exactly k times, 1 <= k < 256;
+ *                            freq[c][0]: those used 256 times or more
+ *   freq_log2[c][b]          blocks of category c with bin(f) = b
+ *   lifetime_us[c][b]        blocks of category c with bin(lifetime) = b
+ *   reuse_us[c][b]           reuses of category-c blocks with bin(interval) = b
+ *   reuse_by_freq[bf][b]     reuses whose block has bin(f) = bf, with bin(interval) = b
+ *   lifetime_by_freq[bf][b]  blocks with bin(f) = bf and bin(lifetime) = b
+ *   dist_log2[b]             reuses with bin(stack distance) = b (zero without dist)
+ *   sess_requests[b]         sessions with at least one request, by bin(request count)
+ *   sess_duration_us[b]      the same sessions by bin(last minus first request time)
+ *   n_access = n, n_distinct, n_reuse = n - n_distinct, n_sessions (with at least
+ *   one request), n_multi_sessions (with two or more)
+ *
+ *   ids, prev, next  u32[n] from ptc_assign_ids and ptc_reuse_indices; every id
+ *                    below n_distinct and every id used (PTC_ERR_INVALID_ARG
+ *                    otherwise, as for prev[i] >= i or next[i] <= i)
+ *   dist             u32[n] from ptc_stack_distance, or NULL
+ *   req_blk_off      u64[n_req + 1] from ptc_hash_blocks, req_blk_off[n_req] == n
+ *   req_ts_us        i64[n_req], non-decreasing (PTC_ERR_UNSORTED otherwise)
+ *   req_session      u32[n_req], labels below n_session (PTC_ERR_INVALID_ARG otherwise)
+ *   cap_host         u64[n_cap] capacities, strictly ascending and >= 1, host
+ *                    memory; n_cap <= PTC_MAX_CAPACITIES, 0 allowed (then NULL)
+ *   reach_host_out   u64[n_cap] (host): reuses with stack distance <= cap_host[g];
+ *                    needs dist when n > 0 and n_cap > 0
+ *   stats_host_out   host memory
+ */
+#define PTC_STAT_CATEGORIES 3
+#define PTC_STAT_BINS 65
+#define PTC_STAT_FREQ_EXACT 256
+typedef struct {
+  uint64_t blocks[PTC_STAT_CATEGORIES];
+  uint64_t accesses[PTC_STAT_CATEGORIES];
+  uint64_t freq[PTC_STAT_CATEGORIES][PTC_STAT_FREQ_EXACT];
+  uint64_t freq_log2[PTC_STAT_CATEGORIES][PTC_STAT_BINS];
+  uint64_t reuse_us[PTC_STAT_CATEGORIES][PTC_STAT_BINS];
+  uint64_t lifetime_us[PTC_STAT_CATEGORIES][PTC_STAT_BINS];
+  uint64_t reuse_by_freq[PTC_STAT_BINS][PTC_STAT_BINS];
+  uint64_t lifetime_by_freq[PTC_STAT_BINS][PTC_STAT_BINS];
+  uint64_t dist_log2[PTC_STAT_BINS];
+  uint64_t sess_requests[PTC_STAT_BINS];
+  uint64_t sess_duration_us[PTC_STAT_BINS];
+  uint64_t n_access, n_distinct, n_reuse, n_sessions, n_multi_sessions;
+} ptc_trace_summary;
+size_t ptc_trace_stats_workspace_bytes(uint64_t n, uint64_t n_distinct, uint32_t n_req, uint32_t n_session);
+ptc_status ptc_trace_stats(const uint32_t* ids, const uint32_t* prev, const uint32_t* next, const uint32_t* dist,
+                           uint64_t n, uint64_t n_distinct, const uint64_t* req_blk_off, const int64_t* req_ts_us,
+                           const uint32_t* req_session, uint32_t n_req, uint32_t n_session, const uint64_t* cap_host,
+                           uint32_t n_cap, uint64_t* reach_host_out, ptc_trace_summary* stats_host_out, void* ws,
+                           size_t ws_bytes, void* stream);
 
 /*
  * ptc_curves_noalloc — ptc_curves for callers that cannot allocate device

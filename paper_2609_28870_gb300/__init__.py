@@ -121,6 +121,11 @@ def lib():
                 L.ptc_pipeline.argtypes = [vp, u64, vp, vp, u32, u32, u64, ctypes.POINTER(CostModel), vp, u32,
                                            vp, vp, vp, vp, vp, vp, ctypes.POINTER(u64), ctypes.POINTER(u64), vp, vp,
                                            ctypes.POINTER(U128), vp, sz, vp]
+                L.ptc_trace_stats_workspace_bytes.restype = sz
+                L.ptc_trace_stats_workspace_bytes.argtypes = [u64, u64, u32, u32]
+                L.ptc_trace_stats.restype = st
+                L.ptc_trace_stats.argtypes = [vp, vp, vp, vp, u64, u64, vp, vp, vp, u32, u32, vp, u32, vp, vp, vp,
+                                              sz, vp]
                 L.ptc_timer_enable.restype = None
                 L.ptc_timer_enable.argtypes = [ctypes.c_int]
                 L.ptc_timer_reset.restype = None
@@ -285,6 +290,50 @@ def ptc_curves(dist: torch.Tensor, req_blk_off: torch.Tensor, block_size: int, c
     return {"hits": [int(h) for h in hits],
             "saved": [int(saved[2 * g + 1]) << 64 | int(saved[2 * g]) for g in range(G)],
             "total_cost": int(total.hi) << 64 | int(total.lo)}
+
+
+# ptc_trace_summary, field by field (all uint64, in declaration order):
+# category-major histograms have 3 rows (0 shared across sessions, 1 session
+# history, 2 single-turn), log2 histograms 65 bins (the bit length of the
+# value), freq 256 exact bins with the blocks used 256 times or more in bin 0.
+STAT_FIELDS = (("blocks", (3,)), ("accesses", (3,)), ("freq", (3, 256)), ("freq_log2", (3, 65)),
+               ("reuse_us", (3, 65)), ("lifetime_us", (3, 65)), ("reuse_by_freq", (65, 65)),
+               ("lifetime_by_freq", (65, 65)), ("dist_log2", (65,)), ("sess_requests", (65,)),
+               ("sess_duration_us", (65,)))
+STAT_SCALARS = ("n_access", "n_distinct", "n_reuse", "n_sessions", "n_multi_sessions")
+STAT_WORDS = sum(int(np.prod(sh)) for _, sh in STAT_FIELDS) + len(STAT_SCALARS)
+
+
+def ptc_trace_stats(ids: torch.Tensor, prev: torch.Tensor, nxt: torch.Tensor, n_distinct: int,
+                    req_blk_off: torch.Tensor, req_ts_us: torch.Tensor, req_session: torch.Tensor, n_session: int,
+                    dist: torch.Tensor | None = None, caps=None, ws: torch.Tensor | None = None) -> dict:
+    """Trace statistics (block categories, frequency, lifetime, reuse-interval
+    and session histograms; reuses reachable within each of ``caps``).
+    ``req_session`` is an int32 tensor of session labels below ``n_session``.
+    Returns numpy uint64 arrays named as in STAT_FIELDS, the STAT_SCALARS as
+    ints, and ``reach`` when ``caps`` is given (it needs ``dist``)."""
+    dev = _dev(ids)
+    n = ids.numel()
+    n_req = req_blk_off.numel() - 1
+    caps = np.ascontiguousarray([] if caps is None else caps, dtype=np.uint64)
+    G = caps.shape[0]
+    reach = np.zeros(max(G, 1), dtype=np.uint64)
+    buf = np.zeros(STAT_WORDS, dtype=np.uint64)
+    w = _workspace(lib().ptc_trace_stats_workspace_bytes(n, n_distinct, n_req, n_session), dev, ws)
+    rc = lib().ptc_trace_stats(_ptr(ids), _ptr(prev), _ptr(nxt), _ptr(dist), n, n_distinct, _ptr(req_blk_off),
+                               _ptr(req_ts_us), _ptr(req_session), n_req, n_session,
+                               caps.ctypes.data if G else None, G, reach.ctypes.data if G else None,
+                               buf.ctypes.data, _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_trace_stats", rc)
+    out, at = {}, 0
+    for name, shape in STAT_FIELDS:
+        size = int(np.prod(shape))
+        out[name] = buf[at: at + size].reshape(shape).copy()
+        at += size
+    out.update({k: int(v) for k, v in zip(STAT_SCALARS, buf[at:])})
+    if G:
+        out["reach"] = reach[:G]
+    return out
 
 
 def workspace_bytes(n_req: int, n_tok: int, block_size: int, n: int | None = None, n_cap: int = MAX_CAPACITIES) -> int:

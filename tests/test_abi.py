@@ -74,3 +74,56 @@ def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(ptc._build, "LIB", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="not built"):
         ptc.lib()
+
+
+def test_trace_summary_layout_matches_binding(tmp_path):
+    """The binding reads ptc_trace_summary as a flat uint64 array: every
+    field's offset and the struct's size, as a C compiler lays them out."""
+    import subprocess
+    import numpy as np
+    import paper_2609_28870_gb300 as ptc
+    fields = [n for n, _ in ptc.STAT_FIELDS] + list(ptc.STAT_SCALARS)
+    src = tmp_path / "layout.c"
+    src.write_text("#include <stdio.h>\n#include <stddef.h>\n#include \"ptc.h\"\nint main(void) {\n"
+                   + "".join(f'  printf("%zu\\n", offsetof(ptc_trace_summary, {f}));\n' for f in fields)
+                   + '  printf("%zu\\n", sizeof(ptc_trace_summary));\n  return 0;\n}\n')
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-std=c99", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)], check=True)
+    got = [int(x) for x in subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()]
+    want, at = [], 0
+    for _, shape in ptc.STAT_FIELDS:
+        want.append(8 * at)
+        at += int(np.prod(shape))
+    for _ in ptc.STAT_SCALARS:
+        want.append(8 * at)
+        at += 1
+    assert got == want + [8 * ptc.STAT_WORDS]
+
+
+def test_trace_stats_host_checks_need_no_gpu(libptc):
+    """ptc_trace_stats rejects bad arguments before any CUDA call."""
+    import numpy as np
+    import paper_2609_28870_gb300 as ptc
+    L = ptc.lib()
+    buf = np.zeros(ptc.STAT_WORDS, dtype=np.uint64)
+    caps = np.array([4, 2], dtype=np.uint64)
+    reach = np.zeros(2, dtype=np.uint64)
+    fake = 256  # never dereferenced: the checks below fail first
+    # no output
+    assert L.ptc_trace_stats(fake, fake, fake, fake, 10, 5, fake, fake, fake, 2, 2, None, 0, None, None,
+                             fake, 1 << 20, None) == 1
+    # capacities not ascending
+    assert L.ptc_trace_stats(fake, fake, fake, fake, 10, 5, fake, fake, fake, 2, 2, caps.ctypes.data, 2,
+                             reach.ctypes.data, buf.ctypes.data, fake, 1 << 20, None) == 1
+    # capacities without distances
+    caps2 = np.array([2, 4], dtype=np.uint64)
+    assert L.ptc_trace_stats(fake, fake, fake, None, 10, 5, fake, fake, fake, 2, 2, caps2.ctypes.data, 2,
+                             reach.ctypes.data, buf.ctypes.data, fake, 1 << 20, None) == 1
+    # more distinct blocks than accesses; N at the marker
+    assert L.ptc_trace_stats(fake, fake, fake, None, 10, 11, fake, fake, fake, 2, 2, None, 0, None,
+                             buf.ctypes.data, fake, 1 << 20, None) == 1
+    assert L.ptc_trace_stats(fake, fake, fake, None, 0xFFFFFFFF, 5, fake, fake, fake, 2, 2, None, 0, None,
+                             buf.ctypes.data, fake, 1 << 20, None) == 3
+    # workspace too small
+    assert L.ptc_trace_stats(fake, fake, fake, None, 10, 5, fake, fake, fake, 2, 2, None, 0, None,
+                             buf.ctypes.data, fake, 16, None) == 4
