@@ -117,7 +117,11 @@ __global__ void k_fill(uint32_t* __restrict__ p, uint32_t v, uint64_t words) {
 
 __global__ void k_copy_words(const uint32_t* __restrict__ src, uint32_t* dst, uint32_t words) {
   grid_dep_sync();
-  for (uint32_t i = threadIdx.x; i < words; i += blockDim.x) dst[i] = src[i];
+  const uint32_t tid = blockIdx.x * blockDim.x + threadIdx.x, nth = gridDim.x * blockDim.x;
+  const uint32_t quads = (((uintptr_t)src | (uintptr_t)dst) & 15) == 0 ? words / 4 : 0;
+  for (uint32_t q = tid; q < quads; q += nth)
+    reinterpret_cast<uint4*>(dst)[q] = reinterpret_cast<const uint4*>(src)[q];
+  for (uint32_t i = quads * 4 + tid; i < words; i += nth) dst[i] = src[i];
 }
 
 // Earlier calls' error words (deferred, see defer_status) join this call's.
@@ -156,8 +160,9 @@ ptc_status copy_to_host_async(void* host_dst, const void* dev_src, size_t bytes,
   const bool staged = hs->dev != nullptr && d >= lo && d + bytes <= lo + sizeof(HostStage);
   if (staged && (bytes & 3) == 0 && ((uintptr_t)dev_src & 3) == 0 && ((uintptr_t)d & 3) == 0) {
     uint32_t* dst = reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(hs->dev) + (d - lo));
-    PTC_KERNEL("k_copy_words", s, k_copy_words, 1, 256, 0, static_cast<const uint32_t*>(dev_src), dst,
-               (uint32_t)(bytes / 4));
+    const uint32_t words = (uint32_t)(bytes / 4);
+    const uint32_t grid = words <= 1024 ? 1u : (words / 1024 < 16 ? words / 1024 : 16u);
+    PTC_KERNEL("k_copy_words", s, k_copy_words, grid, 256, 0, static_cast<const uint32_t*>(dev_src), dst, words);
     return PTC_OK;
   }
   if (cudaMemcpyAsync(host_dst, dev_src, bytes, cudaMemcpyDeviceToHost, s) != cudaSuccess) return PTC_ERR_CUDA;

@@ -63,6 +63,8 @@ inline ptc_status begin_call(void* ws, size_t zero_bytes, cudaStream_t stream) {
   return fill_async(ws, 0u, zero_bytes, stream);
 }
 
+// Words of ptc_trace_stats's results: the summary and the reach bins.
+constexpr size_t kStatsHostWords = sizeof(ptc_trace_summary) / 8 + PTC_MAX_CAPACITIES + 1;
 // Page-locked host buffers for the small copies around a call's wait, one
 // set per host thread (ptc_abi.cu).  A copy from or to pageable memory goes
 // through a driver bounce buffer and costs the wait tens of microseconds.
@@ -71,6 +73,7 @@ inline ptc_status begin_call(void* ws, size_t zero_bytes, cudaStream_t stream) {
 struct HostStage {
   DevStatus st;
   uint64_t out[3 * PTC_MAX_CAPACITIES + 2];
+  alignas(16) uint64_t stats[kStatsHostWords];
   HostStage* dev;  // the same memory as seen by kernels (mapped), or null
 };
 HostStage* host_stage();

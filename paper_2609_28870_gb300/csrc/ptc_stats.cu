@@ -6,37 +6,39 @@
 //   k_st_req     one thread per request: timestamp order, offsets, session
 //                labels; per session its request count and first / last request
 //   k_st_access  tiles of accesses: the request of every access (req_of), the
-//                per-block word (frequency; "in a session with two or more
-//                requests"; "in two or more sessions", decided against the
-//                first session that claims the block's tag), the first and
-//                last request of every block, and the stack-distance and
-//                reach bins
-//   k_st_blocks  one thread per block: category, frequency and lifetime bins
+//                frequency and flags of every block ("in two or more
+//                sessions", decided against the first session that claims
+//                the block's tag; "in a session with two or more requests"),
+//                the first and last request of every block, and the
+//                stack-distance and reach bins
+//   k_st_blocks  one thread per block: category, frequency and lifetime bins,
+//                and a class byte (category, frequency bin) per block; then
+//                one thread per session: request-count and duration bins
 //   k_st_reuse   tiles of accesses: the interval of every reuse, binned by the
-//                category and frequency of its block
-//   k_st_sess    one thread per session: request-count and duration bins
+//                category and frequency of its block (its class byte)
 //
 // Every histogram is counted in shared memory, one update per distinct bin of
 // a warp (__match_any_sync), and added to the u64 totals once per CTA.
+#include <cstring>
+
 #include "ptc_internal.h"
 
 namespace ptc {
 namespace {
 
 constexpr int kStThreads = 256;
-constexpr int kStPer = 8;
+constexpr int kStPer = 4;
 constexpr uint32_t kStTile = kStThreads * kStPer;
 constexpr uint32_t kBins = PTC_STAT_BINS;
 constexpr uint32_t kCats = PTC_STAT_CATEGORIES;
 constexpr uint32_t kFreqExact = PTC_STAT_FREQ_EXACT;
-// The per-block word: frequency in the low 32 bits, then two flags.
-constexpr unsigned long long kMulti = 1ull << 32;  // appears in a session with >= 2 requests
-constexpr unsigned long long kCross = 1ull << 33;  // appears in >= 2 sessions
+// Per-block flags.
+constexpr uint32_t kFlagMulti = 1u;  // appears in a session with >= 2 requests
+constexpr uint32_t kFlagCross = 2u;  // appears in >= 2 sessions
 
 typedef unsigned long long ull;
 
 __device__ __forceinline__ uint32_t bit_len(uint64_t x) { return 64u - (uint32_t)__clzll((long long)x); }
-__device__ __forceinline__ uint32_t category_of(ull w) { return (w & kMulti) ? ((w & kCross) ? 0u : 1u) : 2u; }
 __host__ __device__ __forceinline__ ull* U(uint64_t* p) { return reinterpret_cast<ull*>(p); }
 __device__ __forceinline__ uint32_t cdiv(uint32_t a, uint32_t b) { return a / b + (a % b != 0); }
 
@@ -76,6 +78,8 @@ struct ReqArgs {
   uint32_t* s_cnt;
   uint32_t* s_first;
   uint32_t* s_last;
+  uint32_t* tile_req;  // request holding the first access of each access tile; [tiles] = n_req - 1
+  uint32_t tiles;
   DevStatus* st;
 };
 
@@ -86,6 +90,9 @@ __global__ void __launch_bounds__(kStThreads) k_st_req(ReqArgs a) {
   const uint64_t lo = a.off[r], hi = a.off[r + 1];
   if (hi < lo || hi > a.n || (r == 0 && lo != 0) || (r + 1 == a.n_req && hi != a.n)) raise_err(a.st, kErrInvalid);
   if (r > 0 && a.ts[r] < a.ts[r - 1]) raise_err(a.st, kErrUnsorted);
+  if (hi > lo && hi <= a.n)
+    for (uint64_t t = (lo + kStTile - 1) / kStTile; t * kStTile < hi; ++t) a.tile_req[t] = r;
+  if (r + 1 == a.n_req) a.tile_req[a.tiles] = r;
   const uint32_t s = a.sess[r];
   if (s >= a.n_session) {
     raise_err(a.st, kErrInvalid);
@@ -108,10 +115,12 @@ struct AccArgs {
   const uint32_t* s_cnt;
   uint32_t n_req;
   uint32_t n_session;
+  const uint32_t* tile_req;
   uint32_t* req_of;
-  ull* blk;
-  uint32_t* tag;  // first session seen for each block, kNone before
-  uint2* fl;      // (first request, last request) of each block
+  uint32_t* cnt;    // accesses of each block
+  uint32_t* flg;    // kFlagMulti / kFlagCross of each block
+  uint32_t* tag;    // 1 + the first session that claimed the block, 0 before
+  uint2* fl;        // (first request, last request) of each block
   ull* dist_bins;   // kBins
   ull* reach_bins;  // G + 1: reuses first reachable at grid point g (G: at none)
   ull* n_reuse;
@@ -120,30 +129,48 @@ struct AccArgs {
   uint32_t caps[PTC_MAX_CAPACITIES];  // clamped below kNone
 };
 
-__global__ void __launch_bounds__(kStThreads) k_st_access(const __grid_constant__ AccArgs a) {
+// Access pass.  The two-sessions test: a block's tag is claimed once, by the
+// first session whose access gets to it; an access of any other session sees
+// a different tag and marks the block as crossing sessions (and, if its own
+// session has two or more requests, as appearing in such a session; the
+// claiming session's request count is looked up in the block pass).  The tag
+// only ever changes from 0 to its final value, so any nonzero value read,
+// even a stale one, is final.  Loads are issued for all of a thread's
+// accesses before any result is used.
+__global__ void __launch_bounds__(kStThreads, 6) k_st_access(const __grid_constant__ AccArgs a) {
   __shared__ uint32_t s_caps[PTC_MAX_CAPACITIES];
   __shared__ uint32_t s_reach[PTC_MAX_CAPACITIES + 1];
   __shared__ uint32_t s_dist[kBins];
-  __shared__ uint32_t s_r[2];
+  __shared__ uint32_t s_oct[34];  // s_oct[b]: first grid point with cap >= 2^(b-1) (b >= 1)
   grid_dep_sync();
   for (uint32_t j = threadIdx.x; j < a.G; j += blockDim.x) s_caps[j] = a.caps[j];
   for (uint32_t j = threadIdx.x; j <= a.G; j += blockDim.x) s_reach[j] = 0;
   for (uint32_t j = threadIdx.x; j < kBins; j += blockDim.x) s_dist[j] = 0;
+  if (threadIdx.x < 34) {
+    const uint64_t x = threadIdx.x == 0 ? 0 : 1ull << (threadIdx.x - 1);
+    uint32_t lo = 0, hi = a.G;
+    while (lo < hi) {
+      const uint32_t mid = (lo + hi) >> 1;
+      if ((uint64_t)a.caps[mid] < x) lo = mid + 1;
+      else hi = mid;
+    }
+    s_oct[threadIdx.x] = lo;
+  }
+  __syncthreads();
   const bool with_dist = a.dist != nullptr;
   uint32_t reuses = 0;
   const uint32_t tiles = cdiv(a.n, kStTile);
   for (uint32_t t = blockIdx.x; t < tiles; t += gridDim.x) {
     const uint32_t i0 = t * kStTile;
     const uint32_t iend = a.n - i0 < kStTile ? a.n : i0 + kStTile;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      const uint32_t r0 = req_search(a.off, 0, a.n_req - 1, i0);
-      s_r[0] = r0;
-      s_r[1] = req_search(a.off, r0, a.n_req - 1, iend - 1);
-    }
-    __syncthreads();
-    const uint32_t r0 = s_r[0], r1 = s_r[1];
-    uint32_t id[kStPer], pv[kStPer], nx[kStPer], dv[kStPer];
+    // requests of the tile: from the one holding its first access to the one
+    // holding the next tile's first access (clamped: malformed offsets have
+    // raised an error already)
+    uint32_t r0 = __ldg(a.tile_req + t), r1 = __ldg(a.tile_req + t + 1);
+    r0 = r0 < a.n_req ? r0 : a.n_req - 1;
+    r1 = r1 < a.n_req ? (r1 > r0 ? r1 : r0) : a.n_req - 1;
+    uint32_t id[kStPer], pv[kStPer], nx[kStPer], dv[kStPer], rq[kStPer], ss[kStPer], tg[kStPer];
+    bool ok[kStPer];
 #pragma unroll
     for (int k = 0; k < kStPer; ++k) {
       const uint32_t i = i0 + k * kStThreads + threadIdx.x;
@@ -152,49 +179,63 @@ __global__ void __launch_bounds__(kStThreads) k_st_access(const __grid_constant_
       pv[k] = in ? __ldg(a.prev + i) : kNone;
       nx[k] = in ? __ldg(a.next + i) : 0u;
       dv[k] = in && with_dist ? __ldg(a.dist + i) : kNone;
+      ok[k] = in;
     }
 #pragma unroll
     for (int k = 0; k < kStPer; ++k) {
       const uint32_t i = i0 + k * kStThreads + threadIdx.x;
-      bool ok = (uint64_t)i0 + k * kStThreads + threadIdx.x < iend;
-      uint32_t key = kNone;
-      if (ok) {
-        const uint32_t r = req_search(a.off, r0, r1, i);
-        a.req_of[i] = r;
+      rq[k] = 0;
+      ss[k] = kNone;
+      if (ok[k]) {
+        rq[k] = req_search(a.off, r0, r1, i);
+        a.req_of[i] = rq[k];
         const uint32_t d = id[k], p = pv[k], x = nx[k];
         if (d >= a.D || (p != kNone && p >= i) || (x != kNone && (x <= i || x >= a.n))) {
           raise_err(a.st, kErrInvalid);
-          ok = false;
+          ok[k] = false;
+        } else {
+          ss[k] = __ldg(a.sess + rq[k]);
         }
-        const uint32_t s = ok ? __ldg(a.sess + r) : kNone;
-        if (ok && s < a.n_session) {
-          const ull w = atomicAdd(&a.blk[d], 1ull);
-          ull set = 0;
-          if (!(w & kMulti) && __ldg(a.s_cnt + s) >= 2u) set |= kMulti;
-          if (!(w & kCross)) {
-            // The tag only ever changes from kNone to one session, so any
-            // other value read (even a stale one) is final.
-            uint32_t v = a.tag[d];
-            if (v == kNone) v = atomicCAS(&a.tag[d], kNone, s);
-            if (v != kNone && v != s) set |= kCross;
-          }
-          if (set) atomicOr(&a.blk[d], set);
-        }
-        if (ok) {
-          if (p == kNone) a.fl[d].x = r;
-          if (x == kNone) a.fl[d].y = r;
-          if (p != kNone) {
-            ++reuses;
-            if (with_dist) {
-              const uint32_t dd = dv[k];
-              uint32_t lo = 0, hi = a.G;  // first grid point with cap >= dd
-              while (lo < hi) {
-                const uint32_t mid = (lo + hi) >> 1;
-                if (s_caps[mid] < dd) lo = mid + 1;
-                else hi = mid;
-              }
-              key = bit_len(dd) | (lo << 7);
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < kStPer; ++k) {
+      tg[k] = 0;
+      if (ok[k] && ss[k] < a.n_session) {
+        atomicAdd(&a.cnt[id[k]], 1u);
+        tg[k] = a.tag[id[k]];
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < kStPer; ++k) {
+      if (ok[k] && ss[k] < a.n_session) {
+        const uint32_t mine = ss[k] + 1;
+        uint32_t v = tg[k];
+        if (v == 0) v = atomicCAS(&a.tag[id[k]], 0u, mine);
+        if (v != 0 && v != mine)
+          atomicOr(&a.flg[id[k]], kFlagCross | (__ldg(a.s_cnt + ss[k]) >= 2u ? kFlagMulti : 0u));
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < kStPer; ++k) {
+      uint32_t key = kNone;
+      if (ok[k]) {
+        const uint32_t d = id[k], p = pv[k];
+        if (p == kNone) a.fl[d].x = rq[k];
+        if (nx[k] == kNone) a.fl[d].y = rq[k];
+        if (p != kNone) {
+          ++reuses;
+          if (with_dist) {
+            // first grid point with cap >= dd: between those of the powers
+            // of two around dd (2^(b-1) <= dd < 2^b, b = bit length of dd)
+            const uint32_t dd = dv[k], b = bit_len(dd);
+            uint32_t lo = s_oct[b], hi = s_oct[b < 33 ? b + 1 : 33];
+            while (lo < hi) {
+              const uint32_t mid = (lo + hi) >> 1;
+              if (s_caps[mid] < dd) lo = mid + 1;
+              else hi = mid;
             }
+            key = b | (lo << 7);
           }
         }
       }
@@ -212,56 +253,105 @@ __global__ void __launch_bounds__(kStThreads) k_st_access(const __grid_constant_
 }
 
 struct BlkArgs {
-  const ull* blk;
+  const uint32_t* cnt;
+  const uint32_t* flg;
+  const uint32_t* tag;
   const uint2* fl;
   const int64_t* ts;
+  const uint32_t* s_cnt;
+  const uint32_t* s_first;
+  const uint32_t* s_last;
+  uint8_t* cls;  // category | bit_len(frequency) << 2, for the reuse pass
   uint32_t D;
   uint32_t n_req;
+  uint32_t n_session;
   ptc_trace_summary* out;
   DevStatus* st;
 };
 
+constexpr int kBlkPer = 4;
+
+// Block pass (categories, frequency and lifetime bins, the class byte of
+// every block), then the session bins.
 __global__ void __launch_bounds__(kStThreads) k_st_blocks(const __grid_constant__ BlkArgs a) {
   __shared__ uint32_t s_freq[kCats * kFreqExact];
   __shared__ uint32_t s_flog[kCats * kBins];
   __shared__ uint32_t s_life[kCats * kBins];
   __shared__ uint32_t s_lbf[kBins * kBins];
+  __shared__ uint32_t s_req[kBins];
+  __shared__ uint32_t s_dur[kBins];
   grid_dep_sync();
   for (uint32_t j = threadIdx.x; j < kCats * kFreqExact; j += blockDim.x) s_freq[j] = 0;
   for (uint32_t j = threadIdx.x; j < kCats * kBins; j += blockDim.x) s_flog[j] = s_life[j] = 0;
   for (uint32_t j = threadIdx.x; j < kBins * kBins; j += blockDim.x) s_lbf[j] = 0;
+  for (uint32_t j = threadIdx.x; j < kBins; j += blockDim.x) s_req[j] = s_dur[j] = 0;
   __syncthreads();
   uint32_t nblk[kCats] = {0, 0, 0};
   ull nacc[kCats] = {0, 0, 0};
-  const uint32_t stride = gridDim.x * blockDim.x;
-  const uint32_t rounds = cdiv(a.D, stride);
+  const uint32_t chunk = gridDim.x * blockDim.x * kBlkPer;
+  const uint32_t rounds = cdiv(a.D, chunk);
   for (uint32_t round = 0; round < rounds; ++round) {
-    const uint32_t d = round * stride + blockIdx.x * blockDim.x + threadIdx.x;
-    uint32_t key = kNone;
-    if (d < a.D) {
-      const ull w = a.blk[d];
-      const uint2 fl = a.fl[d];
-      const uint32_t f = (uint32_t)w;
-      if (f == 0 || fl.x >= a.n_req || fl.y >= a.n_req) {
-        raise_err(a.st, kErrInvalid);
-      } else {
-        const uint32_t c = category_of(w);
-        const uint64_t life = (uint64_t)(__ldg(a.ts + fl.y) - __ldg(a.ts + fl.x));
-        const uint32_t fe = f < kFreqExact ? f : 0u;
-        key = c | (fe << 2) | (bit_len(life) << 10) | (bit_len(f) << 17);
+    const uint64_t base = (uint64_t)round * chunk + (uint64_t)blockIdx.x * blockDim.x * kBlkPer + threadIdx.x;
+    uint32_t f[kBlkPer], fg[kBlkPer], tg[kBlkPer];
+    uint2 fl[kBlkPer];
 #pragma unroll
-        for (uint32_t cc = 0; cc < kCats; ++cc) {
-          nblk[cc] += cc == c;
-          nacc[cc] += cc == c ? f : 0u;
+    for (int k = 0; k < kBlkPer; ++k) {
+      const uint64_t d = base + (uint64_t)k * blockDim.x;
+      const bool in = d < a.D;
+      f[k] = in ? a.cnt[d] : 0u;
+      fg[k] = in ? a.flg[d] : 0u;
+      tg[k] = in ? a.tag[d] : 0u;
+      fl[k] = in ? a.fl[d] : make_uint2(kNone, kNone);
+    }
+#pragma unroll
+    for (int k = 0; k < kBlkPer; ++k) {
+      const uint64_t d = base + (uint64_t)k * blockDim.x;
+      uint32_t key = kNone;
+      if (d < a.D) {
+        if (f[k] == 0 || fl[k].x >= a.n_req || fl[k].y >= a.n_req || tg[k] == 0 || tg[k] > a.n_session) {
+          raise_err(a.st, kErrInvalid);
+        } else {
+          const bool multi = (fg[k] & kFlagMulti) || __ldg(a.s_cnt + tg[k] - 1) >= 2u;
+          const uint32_t c = multi ? ((fg[k] & kFlagCross) ? 0u : 1u) : 2u;
+          const uint64_t life = (uint64_t)(__ldg(a.ts + fl[k].y) - __ldg(a.ts + fl[k].x));
+          const uint32_t fe = f[k] < kFreqExact ? f[k] : 0u, bf = bit_len(f[k]);
+          a.cls[d] = (uint8_t)(c | (bf << 2));
+          key = c | (fe << 2) | (bit_len(life) << 10) | (bf << 17);
+#pragma unroll
+          for (uint32_t cc = 0; cc < kCats; ++cc) {
+            nblk[cc] += cc == c;
+            nacc[cc] += cc == c ? f[k] : 0u;
+          }
         }
+      }
+      warp_bin(key, [&](uint32_t kk, uint32_t cnt) {
+        const uint32_t c = kk & 3u, fe = (kk >> 2) & 255u, bl = (kk >> 10) & 127u, bf = kk >> 17;
+        atomicAdd(&s_freq[c * kFreqExact + fe], cnt);
+        atomicAdd(&s_flog[c * kBins + bf], cnt);
+        atomicAdd(&s_life[c * kBins + bl], cnt);
+        atomicAdd(&s_lbf[bf * kBins + bl], cnt);
+      });
+    }
+  }
+  // sessions
+  uint32_t used = 0, multi_s = 0;
+  const uint32_t stride = gridDim.x * blockDim.x;
+  const uint32_t srounds = cdiv(a.n_session, stride);
+  for (uint32_t round = 0; round < srounds; ++round) {
+    const uint32_t s = round * stride + blockIdx.x * blockDim.x + threadIdx.x;
+    uint32_t key = kNone;
+    if (s < a.n_session) {
+      const uint32_t c = a.s_cnt[s];
+      const uint32_t fr = a.s_first[s], lr = a.s_last[s];
+      if (c > 0 && fr < a.n_req && lr < a.n_req) {
+        ++used;
+        multi_s += c >= 2u;
+        key = bit_len(c) | (bit_len((uint64_t)(__ldg(a.ts + lr) - __ldg(a.ts + fr))) << 7);
       }
     }
     warp_bin(key, [&](uint32_t kk, uint32_t cnt) {
-      const uint32_t c = kk & 3u, fe = (kk >> 2) & 255u, bl = (kk >> 10) & 127u, bf = kk >> 17;
-      atomicAdd(&s_freq[c * kFreqExact + fe], cnt);
-      atomicAdd(&s_flog[c * kBins + bf], cnt);
-      atomicAdd(&s_life[c * kBins + bl], cnt);
-      atomicAdd(&s_lbf[bf * kBins + bl], cnt);
+      atomicAdd(&s_req[kk & 127u], cnt);
+      atomicAdd(&s_dur[kk >> 7], cnt);
     });
   }
   __syncthreads();
@@ -270,15 +360,22 @@ __global__ void __launch_bounds__(kStThreads) k_st_blocks(const __grid_constant_
   flush(s_flog, U(&o->freq_log2[0][0]), kCats * kBins);
   flush(s_life, U(&o->lifetime_us[0][0]), kCats * kBins);
   flush(s_lbf, U(&o->lifetime_by_freq[0][0]), kBins * kBins);
+  flush(s_req, U(&o->sess_requests[0]), kBins);
+  flush(s_dur, U(&o->sess_duration_us[0]), kBins);
 #pragma unroll
   for (uint32_t c = 0; c < kCats; ++c) {
     const uint32_t b = __reduce_add_sync(kFull, nblk[c]);
-    ull s = nacc[c];
-    for (int o2 = 16; o2 > 0; o2 >>= 1) s += __shfl_xor_sync(kFull, s, o2);
+    ull sum = nacc[c];
+    for (int o2 = 16; o2 > 0; o2 >>= 1) sum += __shfl_xor_sync(kFull, sum, o2);
     if ((threadIdx.x & 31) == 0) {
       if (b) atomicAdd(U(&o->blocks[c]), (ull)b);
-      if (s) atomicAdd(U(&o->accesses[c]), s);
+      if (sum) atomicAdd(U(&o->accesses[c]), sum);
     }
+  }
+  const uint32_t u = __reduce_add_sync(kFull, used), m = __reduce_add_sync(kFull, multi_s);
+  if ((threadIdx.x & 31) == 0) {
+    if (u) atomicAdd(U(&o->n_sessions), (ull)u);
+    if (m) atomicAdd(U(&o->n_multi_sessions), (ull)m);
   }
 }
 
@@ -286,13 +383,17 @@ struct ReuseArgs {
   const uint32_t* ids;
   const uint32_t* prev;
   const uint32_t* req_of;
-  const ull* blk;
+  const uint8_t* cls;
   const int64_t* ts;
   uint32_t n;
   uint32_t D;
   ptc_trace_summary* out;
 };
 
+// Reuse pass: the interval of every reuse, binned by its block's category
+// and frequency (the class byte).  The random loads (the previous access's
+// request, the class byte, two arrival times) are issued for all of a
+// thread's accesses before any is used.
 __global__ void __launch_bounds__(kStThreads) k_st_reuse(const __grid_constant__ ReuseArgs a) {
   __shared__ uint32_t s_ru[kCats * kBins];
   __shared__ uint32_t s_rbf[kBins * kBins];
@@ -303,25 +404,29 @@ __global__ void __launch_bounds__(kStThreads) k_st_reuse(const __grid_constant__
   const uint32_t tiles = cdiv(a.n, kStTile);
   for (uint32_t t = blockIdx.x; t < tiles; t += gridDim.x) {
     const uint32_t i0 = t * kStTile;
-    uint32_t pv[kStPer];
+    uint32_t pv[kStPer], id[kStPer], ri[kStPer], rp[kStPer], cl[kStPer];
+    bool use[kStPer];
 #pragma unroll
     for (int k = 0; k < kStPer; ++k) {
       const uint64_t i = (uint64_t)i0 + k * kStThreads + threadIdx.x;
-      pv[k] = i < a.n ? __ldg(a.prev + i) : kNone;
+      const bool in = i < a.n;
+      pv[k] = in ? __ldg(a.prev + i) : kNone;
+      id[k] = in ? __ldg(a.ids + i) : 0u;
+      ri[k] = in ? __ldg(a.req_of + i) : 0u;
+      // out-of-range ids or prev were reported by the access pass; skip them
+      use[k] = in && pv[k] < i && id[k] < a.D;
     }
 #pragma unroll
     for (int k = 0; k < kStPer; ++k) {
-      const uint64_t i = (uint64_t)i0 + k * kStThreads + threadIdx.x;
-      const uint32_t p = pv[k];
+      rp[k] = use[k] ? __ldg(a.req_of + pv[k]) : 0u;
+      cl[k] = use[k] ? (uint32_t)__ldg(a.cls + id[k]) : 0u;
+    }
+#pragma unroll
+    for (int k = 0; k < kStPer; ++k) {
       uint32_t key = kNone;
-      // out-of-range ids or prev were reported by k_st_access; skip them here
-      if (p < i && i < a.n) {
-        const uint32_t d = __ldg(a.ids + i);
-        if (d < a.D) {
-          const ull w = a.blk[d];
-          const uint64_t gap = (uint64_t)(__ldg(a.ts + __ldg(a.req_of + i)) - __ldg(a.ts + __ldg(a.req_of + p)));
-          key = category_of(w) | (bit_len(gap) << 2) | (bit_len((uint32_t)w) << 9);
-        }
+      if (use[k]) {
+        const uint64_t gap = (uint64_t)(__ldg(a.ts + ri[k]) - __ldg(a.ts + rp[k]));
+        key = (cl[k] & 3u) | (bit_len(gap) << 2) | ((cl[k] >> 2) << 9);
       }
       warp_bin(key, [&](uint32_t kk, uint32_t cnt) {
         const uint32_t c = kk & 3u, bg = (kk >> 2) & 127u, bf = kk >> 9;
@@ -335,84 +440,55 @@ __global__ void __launch_bounds__(kStThreads) k_st_reuse(const __grid_constant__
   flush(s_rbf, U(&a.out->reuse_by_freq[0][0]), kBins * kBins);
 }
 
-struct SessArgs {
-  const uint32_t* s_cnt;
-  const uint32_t* s_first;
-  const uint32_t* s_last;
-  const int64_t* ts;
-  uint32_t n_session;
-  uint32_t n_req;
-  ptc_trace_summary* out;
-};
-
-__global__ void __launch_bounds__(kStThreads) k_st_sess(SessArgs a) {
-  __shared__ uint32_t s_req[kBins];
-  __shared__ uint32_t s_dur[kBins];
-  grid_dep_sync();
-  for (uint32_t j = threadIdx.x; j < kBins; j += blockDim.x) s_req[j] = s_dur[j] = 0;
-  __syncthreads();
-  uint32_t used = 0, multi = 0;
-  const uint32_t stride = gridDim.x * blockDim.x;
-  const uint32_t rounds = cdiv(a.n_session, stride);
-  for (uint32_t round = 0; round < rounds; ++round) {
-    const uint32_t s = round * stride + blockIdx.x * blockDim.x + threadIdx.x;
-    uint32_t key = kNone;
-    if (s < a.n_session) {
-      const uint32_t c = a.s_cnt[s];
-      const uint32_t f = a.s_first[s], l = a.s_last[s];
-      if (c > 0 && f < a.n_req && l < a.n_req) {
-        ++used;
-        multi += c >= 2u;
-        key = bit_len(c) | (bit_len((uint64_t)(__ldg(a.ts + l) - __ldg(a.ts + f))) << 7);
-      }
-    }
-    warp_bin(key, [&](uint32_t kk, uint32_t cnt) {
-      atomicAdd(&s_req[kk & 127u], cnt);
-      atomicAdd(&s_dur[kk >> 7], cnt);
-    });
-  }
-  __syncthreads();
-  flush(s_req, U(&a.out->sess_requests[0]), kBins);
-  flush(s_dur, U(&a.out->sess_duration_us[0]), kBins);
-  const uint32_t u = __reduce_add_sync(kFull, used), m = __reduce_add_sync(kFull, multi);
-  if ((threadIdx.x & 31) == 0) {
-    if (u) atomicAdd(U(&a.out->n_sessions), (ull)u);
-    if (m) atomicAdd(U(&a.out->n_multi_sessions), (ull)m);
-  }
-}
-
 struct StatsLayout {
   DevStatus* st;
-  ptc_trace_summary* out;
+  ptc_trace_summary* out;  // the summary, then the reach bins right after it
   ull* reach_bins;
   uint32_t* s_cnt;
   uint32_t* s_last;
-  ull* blk;
-  size_t zero_bytes;   // [0, zero_bytes) starts at zero
-  uint32_t* s_first;   // these three start at all ones
+  uint32_t* cnt;
+  uint32_t* flg;
   uint32_t* tag;
+  size_t zero_bytes;   // [0, zero_bytes) starts at zero
+  uint32_t* s_first;   // these two start at all ones
   uint2* fl;
   size_t ones_from, ones_bytes;
+  uint8_t* cls;
   uint32_t* req_of;
+  uint32_t* tile_req;
   size_t total;
 };
+
+// One wave of CTAs (as many as fit on every SM at once), or fewer if there
+// is less work: the kernels above loop over their tiles.
+template <class K>
+uint32_t persistent_grid(K kernel, int threads, int sms, uint32_t work) {
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, 0) != cudaSuccess || per_sm < 1)
+    per_sm = 1;
+  const uint32_t wave = (uint32_t)(per_sm * sms);
+  return work < wave ? (work ? work : 1u) : wave;
+}
 
 StatsLayout stats_layout(void* ws, uint64_t n, uint64_t D, uint32_t n_session) {
   StatsLayout L;
   Carver cv(ws);
   L.st = cv.take<DevStatus>(1);
   L.out = cv.take<ptc_trace_summary>(1);
-  L.reach_bins = cv.take<ull>(PTC_MAX_CAPACITIES + 1);
+  L.reach_bins = cv.take<ull>(PTC_MAX_CAPACITIES + 1, 8);
   L.s_cnt = cv.take<uint32_t>(n_session);
   L.s_last = cv.take<uint32_t>(n_session);
-  L.blk = cv.take<ull>(D);
+  L.cnt = cv.take<uint32_t>(D);
+  L.flg = cv.take<uint32_t>(D);
+  L.tag = cv.take<uint32_t>(D);
   L.zero_bytes = cv.off;
   L.ones_from = cv.bytes();
   L.s_first = cv.take<uint32_t>(n_session);
-  L.tag = cv.take<uint32_t>(D);
   L.fl = cv.take<uint2>(D);
   L.ones_bytes = cv.off - L.ones_from;
+  L.cls = cv.take<uint8_t>(D);
   L.req_of = cv.take<uint32_t>(n);
+  L.tile_req = cv.take<uint32_t>((n + kStTile - 1) / kStTile + 1);
   L.total = cv.bytes();
   return L;
 }
@@ -449,12 +525,14 @@ extern "C" ptc_status ptc_trace_stats(const uint32_t* ids, const uint32_t* prev,
   if (fill_async((char*)ws + L.ones_from, 0xFFFFFFFFu, L.ones_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
   const int sms = num_sms();
   if (n_req > 0) {
-    const ReqArgs ra{req_blk_off, req_ts_us, req_session, n, n_req, n_session, L.s_cnt, L.s_first, L.s_last, L.st};
+    const ReqArgs ra{req_blk_off, req_ts_us, req_session, n, n_req, n_session, L.s_cnt, L.s_first, L.s_last,
+                     L.tile_req, ceil_div_u32(n, kStTile), L.st};
     PTC_KERNEL("k_st_req", s, k_st_req, ceil_div_u32(n_req, kStThreads), kStThreads, 0, ra);
   }
+  const uint32_t tiles = ceil_div_u32(n, kStTile);
+  const uint32_t grid_acc = persistent_grid(k_st_access, kStThreads, sms, tiles);
+  const uint32_t grid_reuse = persistent_grid(k_st_reuse, kStThreads, sms, tiles);
   if (n > 0) {
-    const uint32_t tiles = ceil_div_u32(n, kStTile);
-    const uint32_t grid = tiles < (uint32_t)(4 * sms) ? tiles : (uint32_t)(4 * sms);
     AccArgs aa;
     aa.ids = ids;
     aa.prev = prev;
@@ -467,8 +545,10 @@ extern "C" ptc_status ptc_trace_stats(const uint32_t* ids, const uint32_t* prev,
     aa.s_cnt = L.s_cnt;
     aa.n_req = n_req;
     aa.n_session = n_session;
+    aa.tile_req = L.tile_req;
     aa.req_of = L.req_of;
-    aa.blk = L.blk;
+    aa.cnt = L.cnt;
+    aa.flg = L.flg;
     aa.tag = L.tag;
     aa.fl = L.fl;
     aa.dist_bins = U(&L.out->dist_log2[0]);
@@ -477,32 +557,32 @@ extern "C" ptc_status ptc_trace_stats(const uint32_t* ids, const uint32_t* prev,
     aa.st = L.st;
     aa.G = n_cap;
     for (uint32_t g = 0; g < n_cap; ++g) aa.caps[g] = cap_host[g] >= (uint64_t)kNone ? kNone - 1 : (uint32_t)cap_host[g];
-    PTC_KERNEL("k_st_access", s, k_st_access, grid, kStThreads, 0, aa);
-    const BlkArgs ba{L.blk, L.fl, req_ts_us, (uint32_t)n_distinct, n_req, L.out, L.st};
-    const uint32_t bgrid0 = ceil_div_u32(n_distinct, kStThreads);
-    const uint32_t bgrid = bgrid0 < (uint32_t)(4 * sms) ? bgrid0 : (uint32_t)(4 * sms);
+    PTC_KERNEL("k_st_access", s, k_st_access, grid_acc, kStThreads, 0, aa);
+  }
+  if (n_req > 0) {  // blocks (if any), then sessions
+    const BlkArgs ba{L.cnt, L.flg, L.tag, L.fl, req_ts_us, L.s_cnt, L.s_first, L.s_last, L.cls,
+                     (uint32_t)n_distinct, n_req, n_session, L.out, L.st};
+    const uint64_t want = n_distinct / kBlkPer > n_session ? n_distinct / kBlkPer : n_session;
+    const uint32_t bgrid = persistent_grid(k_st_blocks, kStThreads, sms, ceil_div_u32(want ? want : 1, kStThreads));
     PTC_KERNEL("k_st_blocks", s, k_st_blocks, bgrid, kStThreads, 0, ba);
-    const ReuseArgs rua{ids, prev, L.req_of, L.blk, req_ts_us, (uint32_t)n, (uint32_t)n_distinct, L.out};
-    PTC_KERNEL("k_st_reuse", s, k_st_reuse, grid, kStThreads, 0, rua);
   }
-  if (n_session > 0 && n_req > 0) {
-    const uint32_t sgrid0 = ceil_div_u32(n_session, kStThreads);
-    const uint32_t sgrid = sgrid0 < (uint32_t)(2 * sms) ? sgrid0 : (uint32_t)(2 * sms);
-    const SessArgs sa{L.s_cnt, L.s_first, L.s_last, req_ts_us, n_session, n_req, L.out};
-    PTC_KERNEL("k_st_sess", s, k_st_sess, sgrid, kStThreads, 0, sa);
+  if (n > 0) {
+    const ReuseArgs rua{ids, prev, L.req_of, L.cls, req_ts_us, (uint32_t)n, (uint32_t)n_distinct, L.out};
+    PTC_KERNEL("k_st_reuse", s, k_st_reuse, grid_reuse, kStThreads, 0, rua);
   }
-  if (cudaMemcpyAsync(stats_host_out, L.out, sizeof(ptc_trace_summary), cudaMemcpyDeviceToHost, s) != cudaSuccess)
-    return PTC_ERR_CUDA;
-  uint64_t* bins = nullptr;
-  if (n_cap > 0) {
-    bins = host_stage()->out;  // PTC_MAX_CAPACITIES + 1 <= 3 * PTC_MAX_CAPACITIES + 2 entries
-    if (copy_to_host_async(bins, L.reach_bins, sizeof(uint64_t) * (n_cap + 1), s) != PTC_OK) return PTC_ERR_CUDA;
-  }
+  // the summary and the reach bins (contiguous in the workspace) in one copy
+  HostStage* hs = host_stage();
+  const size_t words = sizeof(ptc_trace_summary) / 8 + (n_cap ? n_cap + 1 : 0);
+  static_assert(sizeof(ptc_trace_summary) % 8 == 0, "summary of u64 fields");
+  if ((const char*)L.reach_bins != (const char*)L.out + sizeof(ptc_trace_summary)) return PTC_ERR_CUDA;
+  if (copy_to_host_async(hs->stats, L.out, 8 * words, s) != PTC_OK) return PTC_ERR_CUDA;
   DevStatus h;
   const ptc_status rc = end_call(L.st, s, &h);
   if (rc != PTC_OK) return rc;
+  std::memcpy(stats_host_out, hs->stats, sizeof(ptc_trace_summary));
   stats_host_out->n_access = n;
   stats_host_out->n_distinct = n_distinct;
+  const uint64_t* bins = hs->stats + sizeof(ptc_trace_summary) / 8;
   uint64_t run = 0;
   for (uint32_t g = 0; g < n_cap; ++g) reach_host_out[g] = (run += bins[g]);
   return PTC_OK;
