@@ -322,6 +322,24 @@ def run_ours(args, ws_world, rank, local):
     h2d = 4 * T + 8 * (tr.n_req + 1) + 8 * tr.n_req
     d2h = 8 * G + 16 * G + 16 + 8 + 8  # hits, saved (u128), total cost, N, D
 
+    # ---- trace statistics (Sec. 4.1-4.3, App. B) over the pipeline's own
+    # per-access arrays: one pipeline run that keeps them, then K timed calls
+    outs = {k: torch.empty(max(N, 1), dtype=torch.int32, device=dev) for k in ("ids", "prev", "next", "dist")}
+    outs["req_blk_off"] = torch.empty(tr.n_req + 1, dtype=torch.int64, device=dev)
+    ptc.PipelinePlan(tok, off, ts, BLOCK, caps, ws=ws, outputs=outs).run()
+    ses = torch.from_numpy(tr.req_session.astype(np.uint32).view(np.int32)).to(dev)
+    splan = ptc.TraceStatsPlan(outs["ids"][:N], outs["prev"][:N], outs["next"][:N], D, outs["req_blk_off"], ts, ses,
+                               tr.n_sessions, dist=outs["dist"][:N], caps=caps)
+    stats = splan.run().result()
+    assert stats["n_reuse"] == N - D and int(stats["blocks"].sum()) == D and int(stats["accesses"].sum()) == N
+    assert int(stats["reuse_us"].sum()) == N - D and int(stats["reach"][-1]) <= N - D
+    L.ptc_timer_reset()
+    L.ptc_timer_enable(1)
+    splan.run()
+    L.ptc_timer_enable(0)
+    st_kernels = {name: round(tot, 4) for name, _, tot in read_timer(ptc)}
+    st_ms = max_over_ranks(sum(timed(args.steps, splan.run))) / args.steps
+
     # ---- roofline
     peak, peak_kind = measured_peaks()
     stages, Lbits = stage_model_bytes(T, N)
@@ -370,9 +388,28 @@ def run_ours(args, ws_world, rank, local):
                 "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_total / args.steps, 4)},
         "gpu_launches": launches,
         "clocks": clk,
+        "trace_stats": {
+            "call": "ptc_trace_stats on the step's ids, prev, next and stack distances, 64-point reach grid",
+            "ms": round(st_ms, 4), "accesses_per_s": round(ws_world * N / (st_ms * 1e-3), 1),
+            "roofline": {"bound": "hbm", "bytes_model": "16 N: ids, prev, next, dist read once",
+                         "achieved": round(16 * N / (st_ms * 1e-3) / 1e9, 1), "peak": peak, "unit": "GB/s",
+                         "frac": round(16 * N / (st_ms * 1e-3) / 1e9 / peak, 4), "traffic": None},
+            "kernels_ms": st_kernels,
+            "categories": {"blocks": stats["blocks"].tolist(), "accesses": stats["accesses"].tolist(),
+                           "one_hit_blocks": [int(stats["freq"][c, 1]) for c in range(3)]},
+        },
     }
     if rank == 0 and ws_world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(tr, args.cpu_sample)
+        line["cpu_baseline"], orc = cpu_baseline(tr, args.cpu_sample, stats=True)
+        ost, odt = oracle_trace_stats(tr, orc)
+        same = None
+        if orc["n_req"] == tr.n_req:  # the sample is the whole trace: the oracle's statistics must match
+            same = all(np.array_equal(np.asarray(ost[k]), np.asarray(stats[k])) for k in ost)
+            assert same, "trace statistics differ from the oracle"
+        line["trace_stats"]["cpu_baseline"] = {
+            "value": round(orc["n"] / odt, 1), "unit": "accesses/s", "cores": 1, "kind": "oracle",
+            "sample": f"orc_trace_stats on the oracle's own ids and distances of the first {orc['n_req']} requests "
+                      f"({orc['n']} accesses); {odt:.2f} s", "parity_with_gpu": same}
     if rank == 0:
         s = json.dumps(line)
         print(s, flush=True)
@@ -400,7 +437,7 @@ def read_timer(ptc):
 
 
 # ---------------------------------------------------------------- CPU oracle
-def oracle_on_sample(tr, fraction, threads):
+def oracle_on_sample(tr, fraction, threads, keep=False):
     import oracle
     import tracegen
     n_req = max(1, int(tr.n_req * fraction))
@@ -409,20 +446,34 @@ def oracle_on_sample(tr, fraction, threads):
     ids, D = oracle.block_ids(sub.tokens, sub.req_tok_off, BLOCK)
     off = oracle.block_offsets(sub.req_tok_off, BLOCK)
     prev, nxt = oracle.reuse(ids, D)
-    oracle.sd_fenwick(prev)
+    sd = oracle.sd_fenwick(prev)
     caps = tracegen.workload_grid(WORKLOAD, D)
     oracle.lru_curves(ids, off, BLOCK, caps, oracle.COST_MEASURED, threads=threads)
     dt = time.perf_counter() - t0
-    return sub, dt
+    kept = dict(sub=sub, ids=ids, D=D, off=off, sd=sd, n=int(ids.size), n_req=n_req) if keep else None
+    return sub, dt, kept
 
 
-def cpu_baseline(tr, fraction):
+def cpu_baseline(tr, fraction, stats=False):
     threads = os.cpu_count() or 1
-    sub, dt = oracle_on_sample(tr, fraction, threads)
-    return {"value": round(sub.n_tok / dt, 1), "unit": "tokens/s", "cores": threads, "kind": "oracle",
+    sub, dt, kept = oracle_on_sample(tr, fraction, threads, keep=stats)
+    line = {"value": round(sub.n_tok / dt, 1), "unit": "tokens/s", "cores": threads, "kind": "oracle",
             "sample": f"first {sub.n_req} of {tr.n_req} requests ({sub.n_tok} tokens) of the same workload; "
                       f"exact trie ids, prev/next, Fenwick stack distances, direct LRU simulation at all 64 "
                       f"capacities on {threads} threads; {dt:.2f} s"}
+    return (line, kept) if stats else line
+
+
+def oracle_trace_stats(tr, kept):
+    """The oracle's trace statistics on its own arrays of the sample, timed."""
+    import oracle
+    import tracegen
+    sub = kept["sub"]
+    caps = tracegen.workload_grid(WORKLOAD, kept["D"]) if kept["n_req"] == tr.n_req else None
+    t0 = time.perf_counter()
+    st = oracle.trace_stats(kept["ids"], kept["D"], kept["off"], sub.req_ts_us, sub.req_session, tr.n_sessions,
+                            kept["sd"], caps)
+    return st, time.perf_counter() - t0
 
 
 def run_reference(args, ws_world, rank):
@@ -432,11 +483,11 @@ def run_reference(args, ws_world, rank):
     tr = tracegen.make(WORKLOAD)
     threads = os.cpu_count() or 1
     for _ in range(max(args.warmup, 0)):
-        oracle_on_sample(tr, args.ref_sample, threads)
+        oracle_on_sample(tr, args.ref_sample, threads)[:2]
     times = []
     sub = None
     for _ in range(args.steps):
-        sub, dt = oracle_on_sample(tr, args.ref_sample, threads)
+        sub, dt, _ = oracle_on_sample(tr, args.ref_sample, threads)
         times.append(dt)
     total = sum(times)
     value = sub.n_tok * args.steps / total

@@ -304,36 +304,57 @@ STAT_SCALARS = ("n_access", "n_distinct", "n_reuse", "n_sessions", "n_multi_sess
 STAT_WORDS = sum(int(np.prod(sh)) for _, sh in STAT_FIELDS) + len(STAT_SCALARS)
 
 
+class TraceStatsPlan:
+    """ptc_trace_stats with its arguments marshalled once: ``run()`` is one C
+    call that rereads the given device arrays, ``result()`` converts the
+    summary.  ``req_session`` is an int32 tensor of session labels below
+    ``n_session``; ``caps`` needs ``dist``."""
+
+    def __init__(self, ids: torch.Tensor, prev: torch.Tensor, nxt: torch.Tensor, n_distinct: int,
+                 req_blk_off: torch.Tensor, req_ts_us: torch.Tensor, req_session: torch.Tensor, n_session: int,
+                 dist: torch.Tensor | None = None, caps=None, ws: torch.Tensor | None = None):
+        dev = _dev(req_blk_off)
+        n = ids.numel()
+        n_req = req_blk_off.numel() - 1
+        self.caps = np.ascontiguousarray([] if caps is None else caps, dtype=np.uint64)
+        G = self.caps.shape[0]
+        self.reach = np.zeros(max(G, 1), dtype=np.uint64)
+        self.buf = np.zeros(STAT_WORDS, dtype=np.uint64)
+        self.ws = _workspace(lib().ptc_trace_stats_workspace_bytes(n, n_distinct, n_req, n_session), dev, ws)
+        self._keep = (ids, prev, nxt, req_blk_off, req_ts_us, req_session, dist)
+        self._fn = lib().ptc_trace_stats
+        self._args = (_ptr(ids), _ptr(prev), _ptr(nxt), _ptr(dist), n, n_distinct, _ptr(req_blk_off),
+                      _ptr(req_ts_us), _ptr(req_session), n_req, n_session, self.caps.ctypes.data if G else None, G,
+                      self.reach.ctypes.data if G else None, self.buf.ctypes.data, _ptr(self.ws), self.ws.numel(),
+                      _stream(dev))
+
+    def run(self) -> "TraceStatsPlan":
+        rc = self._fn(*self._args)
+        if rc != 0:
+            raise PtcError("ptc_trace_stats", rc)
+        return self
+
+    def result(self) -> dict:
+        out, at = {}, 0
+        for name, shape in STAT_FIELDS:
+            size = int(np.prod(shape))
+            out[name] = self.buf[at: at + size].reshape(shape).copy()
+            at += size
+        out.update({k: int(v) for k, v in zip(STAT_SCALARS, self.buf[at:])})
+        if self.caps.shape[0]:
+            out["reach"] = self.reach[: self.caps.shape[0]].copy()
+        return out
+
+
 def ptc_trace_stats(ids: torch.Tensor, prev: torch.Tensor, nxt: torch.Tensor, n_distinct: int,
                     req_blk_off: torch.Tensor, req_ts_us: torch.Tensor, req_session: torch.Tensor, n_session: int,
                     dist: torch.Tensor | None = None, caps=None, ws: torch.Tensor | None = None) -> dict:
     """Trace statistics (block categories, frequency, lifetime, reuse-interval
     and session histograms; reuses reachable within each of ``caps``).
-    ``req_session`` is an int32 tensor of session labels below ``n_session``.
     Returns numpy uint64 arrays named as in STAT_FIELDS, the STAT_SCALARS as
     ints, and ``reach`` when ``caps`` is given (it needs ``dist``)."""
-    dev = _dev(ids)
-    n = ids.numel()
-    n_req = req_blk_off.numel() - 1
-    caps = np.ascontiguousarray([] if caps is None else caps, dtype=np.uint64)
-    G = caps.shape[0]
-    reach = np.zeros(max(G, 1), dtype=np.uint64)
-    buf = np.zeros(STAT_WORDS, dtype=np.uint64)
-    w = _workspace(lib().ptc_trace_stats_workspace_bytes(n, n_distinct, n_req, n_session), dev, ws)
-    rc = lib().ptc_trace_stats(_ptr(ids), _ptr(prev), _ptr(nxt), _ptr(dist), n, n_distinct, _ptr(req_blk_off),
-                               _ptr(req_ts_us), _ptr(req_session), n_req, n_session,
-                               caps.ctypes.data if G else None, G, reach.ctypes.data if G else None,
-                               buf.ctypes.data, _ptr(w), w.numel(), _stream(dev))
-    _check("ptc_trace_stats", rc)
-    out, at = {}, 0
-    for name, shape in STAT_FIELDS:
-        size = int(np.prod(shape))
-        out[name] = buf[at: at + size].reshape(shape).copy()
-        at += size
-    out.update({k: int(v) for k, v in zip(STAT_SCALARS, buf[at:])})
-    if G:
-        out["reach"] = reach[:G]
-    return out
+    return TraceStatsPlan(ids, prev, nxt, n_distinct, req_blk_off, req_ts_us, req_session, n_session, dist, caps,
+                          ws).run().result()
 
 
 def workspace_bytes(n_req: int, n_tok: int, block_size: int, n: int | None = None, n_cap: int = MAX_CAPACITIES) -> int:
