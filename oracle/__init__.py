@@ -15,6 +15,9 @@ Functions and the passages they restate:
   move-to-front stack and by Bennett-Kruskal counting.
 * ``lru_curves`` — direct LRU simulation per capacity (Sec. 3.1-3.2) with
   prefix-contiguous hits (Sec. 2.2) and compute saved (Sec. 5.2, App. C).
+* ``lru_curves_variant``, ``sd_variant`` — Sec. 3.1: leaf-first touch order
+  and whole-request residency (every block looked up at the request's
+  arrival), by direct LRU per capacity, Fenwick counting and Mattson's list.
 * ``trace_stats`` — Sec. 4.1-4.3 and App. B: per-category block counts,
   frequency, lifetime and reuse-interval histograms, session lengths and
   durations, and reuses reachable within each capacity.
@@ -76,6 +79,12 @@ def _load():
         lib.orc_lru_curves.restype = i32
         lib.orc_lru_curves.argtypes = [vp, vp, u32, u32, i32, u64, u64, vp, u32, i32, vp, vp, vp, vp, vp]
         lib.orc_prefix_hash.argtypes = [vp, vp, u32, u32, u64, vp]
+        lib.orc_lru_curves_variant.restype = i32
+        lib.orc_lru_curves_variant.argtypes = [vp, vp, u32, u32, i32, u64, u64, vp, u32, i32, i32, i32, vp, vp, vp]
+        lib.orc_sd_variant.restype = i32
+        lib.orc_sd_variant.argtypes = [vp, u64, vp, u32, i32, i32, vp]
+        lib.orc_sd_variant_mattson.restype = i32
+        lib.orc_sd_variant_mattson.argtypes = [vp, vp, u32, i32, i32, vp]
         lib.orc_trace_stats.restype = i32
         lib.orc_trace_stats.argtypes = [vp, u64, u64, vp, vp, vp, u32, u64, vp, vp, u32] + [vp] * 13
         _lib = lib
@@ -155,6 +164,43 @@ def prefix_hash(tokens, req_tok_off, B: int, seed: int) -> np.ndarray:
     keys = np.empty((n, 2), dtype=np.uint64)
     _load().orc_prefix_hash(_p(tok), _p(off), off.shape[0] - 1, int(B), int(seed) & (2**64 - 1), _p(keys))
     return keys
+
+
+# Semantics variants (Sec. 3.1): the order a request's blocks are touched in,
+# and whether they are looked up one by one or all at the request's arrival.
+ROOT_FIRST, LEAF_FIRST = 0, 1
+RES_BLOCK, RES_REQUEST = 0, 1
+
+
+def lru_curves_variant(ids, req_blk_off, B: int, caps, order: int, residency: int, kind: int = COST_MEASURED,
+                       f_lin: int = F_LIN, f_attn: int = F_ATTN, threads: int | None = None):
+    """Direct LRU simulation per capacity under a touch order and a
+    residency rule.  Returns (hits list[int], saved list[int])."""
+    ids, bo, caps = _c(ids, np.uint32), _c(req_blk_off, np.uint64), _c(caps, np.uint64)
+    G = caps.shape[0]
+    hits = np.zeros(G, dtype=np.uint64)
+    slo = np.zeros(G, dtype=np.uint64)
+    shi = np.zeros(G, dtype=np.uint64)
+    nthreads = threads or max(1, min(G, os.cpu_count() or 1))
+    rc = _load().orc_lru_curves_variant(_p(ids), _p(bo), bo.shape[0] - 1, int(B), int(kind), int(f_lin), int(f_attn),
+                                        _p(caps), G, int(order), int(residency), nthreads, _p(hits), _p(slo), _p(shi))
+    if rc != 0:
+        raise ValueError("bad capacity grid or variant")
+    return [int(h) for h in hits], [int(h) << 64 | int(l) for l, h in zip(slo, shi)]
+
+
+def sd_variant(ids, n_distinct: int, req_blk_off, order: int, residency: int, mattson: bool = False) -> np.ndarray:
+    """Stack distance of every access under a variant, in depth order."""
+    ids, bo = _c(ids, np.uint32), _c(req_blk_off, np.uint64)
+    sd = np.empty_like(ids)
+    if mattson:
+        rc = _load().orc_sd_variant_mattson(_p(ids), _p(bo), bo.shape[0] - 1, int(order), int(residency), _p(sd))
+    else:
+        rc = _load().orc_sd_variant(_p(ids), int(n_distinct), _p(bo), bo.shape[0] - 1, int(order), int(residency),
+                                    _p(sd))
+    if rc != 0:
+        raise ValueError("bad variant")
+    return sd
 
 
 # Shapes of the trace statistics: category-major histograms have 3 rows

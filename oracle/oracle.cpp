@@ -23,6 +23,11 @@
 //        orc_sd_fenwick (Bennett & Kruskal 1975 counting), two independent ways.
 //   * Belady's next use (Sec. 3.2, 5.2).  -> orc_reuse: previous and next
 //     access of the same block.
+//   * Sec. 3.1 (the paper's simulator keeps a whole request resident and
+//     makes room for it up front) and the order a request's blocks are
+//     touched in.  -> orc_lru_curves_variant (direct LRU per capacity),
+//        orc_sd_variant (Fenwick counting) and orc_sd_variant_mattson
+//        (move-to-front list).
 //   * Sec. 4.1-4.3 and App. B: block lifetimes, frequencies, reuse intervals,
 //     block categories, session lengths and reuses reachable within a
 //     capacity.  -> orc_trace_stats: two passes over the access stream with
@@ -468,6 +473,156 @@ int orc_trace_stats(const uint32_t* ids, uint64_t n, uint64_t D, const uint64_t*
   scalars[2] = n_reuse;
   scalars[3] = used;
   scalars[4] = multi;
+  return 0;
+}
+
+}  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Semantics variants (Sec. 3.1: the paper's simulator makes room for a whole
+// request before its prefill, so every block of a request is resident at
+// once; engines differ in the order they touch a request's blocks).
+//   order      0: root-first (depth 0, 1, ...), the hot path's order
+//              1: leaf-first (deepest block first, the root last)
+//   residency  0: per block: each block is looked up when it is touched
+//              1: per request: every block of the request is looked up at the
+//                 request's arrival, before any of them is touched; then all
+//                 are touched in `order`
+// A block counts as a hit iff it and every shallower block of its request
+// were found resident (prefix reuse, Sec. 2.2).  (order 0, residency 0) is
+// orc_lru_curves.
+// ---------------------------------------------------------------------------
+extern "C" {
+
+// Direct LRU simulation per capacity under a variant; arguments and outputs
+// as for orc_lru_curves (without the total cost).  Returns 0, or -1 on a bad
+// argument.
+int orc_lru_curves_variant(const uint32_t* ids, const uint64_t* req_blk_off, uint32_t n_req, uint32_t B, int kind,
+                           uint64_t f_lin, uint64_t f_attn, const uint64_t* caps, uint32_t G, int order,
+                           int residency, int threads, uint64_t* hits, uint64_t* saved_lo, uint64_t* saved_hi) {
+  if ((order != 0 && order != 1) || (residency != 0 && residency != 1)) return -1;
+  for (uint32_t g = 0; g < G; ++g)
+    if (caps[g] == 0) return -1;
+  std::atomic<uint32_t> next_cap{0};
+  auto simulate = [&]() {
+    for (;;) {
+      uint32_t g = next_cap.fetch_add(1);
+      if (g >= G) return;
+      uint64_t C = caps[g];
+      std::list<uint32_t> recency;  // front = most recent
+      std::unordered_map<uint32_t, std::list<uint32_t>::iterator> where;
+      auto touch = [&](uint32_t id) {
+        auto it = where.find(id);
+        if (it != where.end()) {
+          recency.splice(recency.begin(), recency, it->second);
+        } else {
+          recency.push_front(id);
+          where[id] = recency.begin();
+          if (recency.size() > C) {
+            where.erase(recency.back());
+            recency.pop_back();
+          }
+        }
+      };
+      uint64_t h = 0;
+      u128 saved = 0;
+      std::vector<char> resident;
+      for (uint32_t r = 0; r < n_req; ++r) {
+        const uint64_t a = req_blk_off[r], n = req_blk_off[r + 1] - a;
+        resident.assign(n, 0);
+        if (residency == 1)
+          for (uint64_t k = 0; k < n; ++k) resident[k] = where.count(ids[a + k]) != 0;
+        for (uint64_t s = 0; s < n; ++s) {
+          const uint64_t k = order == 0 ? s : n - 1 - s;  // the s-th block touched
+          if (residency == 0) resident[k] = where.count(ids[a + k]) != 0;
+          touch(ids[a + k]);
+        }
+        for (uint64_t k = 0; k < n && resident[k]; ++k) {
+          ++h;
+          saved += cost_of(k, B, kind, f_lin, f_attn);
+        }
+      }
+      hits[g] = h;
+      saved_lo[g] = (uint64_t)saved;
+      saved_hi[g] = (uint64_t)(saved >> 64);
+    }
+  };
+  if (threads < 1) threads = 1;
+  std::vector<std::thread> pool;
+  for (int t = 1; t < threads; ++t) pool.emplace_back(simulate);
+  simulate();
+  for (auto& th : pool) th.join();
+  return 0;
+}
+
+// Stack distance under a variant: the block's depth in the LRU stack (1 =
+// most recent) when it is looked up, i.e. 1 + the number of distinct blocks
+// touched since its own last touch; 0xFFFFFFFF for a block never seen.  Per
+// block it is looked up when touched, per request at the request's arrival.
+// Written in depth order (index req_blk_off[r] + k).  Counting as in
+// orc_sd_fenwick: positions are numbered in touch order, and a Fenwick tree
+// marks the position of every block's latest touch.
+int orc_sd_variant(const uint32_t* ids, uint64_t n_distinct, const uint64_t* req_blk_off, uint32_t n_req, int order,
+                   int residency, uint32_t* sd) {
+  if ((order != 0 && order != 1) || (residency != 0 && residency != 1)) return -1;
+  const uint64_t n = req_blk_off[n_req];
+  std::vector<uint32_t> tree(n + 1, 0);
+  auto add = [&](uint64_t pos, int32_t v) {
+    for (uint64_t x = pos + 1; x <= n; x += x & (~x + 1)) tree[x] += (uint32_t)v;
+  };
+  auto prefix = [&](uint64_t cnt) {  // marks in positions [0, cnt)
+    uint64_t s = 0;
+    for (uint64_t x = cnt; x > 0; x -= x & (~x + 1)) s += tree[x];
+    return s;
+  };
+  std::vector<uint64_t> last(n_distinct, UINT64_MAX);
+  auto depth = [&](uint32_t id, uint64_t now) -> uint32_t {
+    if (last[id] == UINT64_MAX) return NONE;
+    return (uint32_t)(1 + prefix(now) - prefix(last[id] + 1));
+  };
+  uint64_t t = 0;  // touches so far
+  for (uint32_t r = 0; r < n_req; ++r) {
+    const uint64_t a = req_blk_off[r], m = req_blk_off[r + 1] - a;
+    if (residency == 1)
+      for (uint64_t k = 0; k < m; ++k) sd[a + k] = depth(ids[a + k], t);
+    for (uint64_t s = 0; s < m; ++s) {
+      const uint64_t k = order == 0 ? s : m - 1 - s;
+      const uint32_t id = ids[a + k];
+      if (residency == 0) sd[a + k] = depth(id, t);
+      if (last[id] != UINT64_MAX) add(last[id], -1);
+      add(t, +1);
+      last[id] = t++;
+    }
+  }
+  return 0;
+}
+
+// The same distances by a move-to-front list (Mattson et al. 1970): O(N * D),
+// tiny inputs only.
+int orc_sd_variant_mattson(const uint32_t* ids, const uint64_t* req_blk_off, uint32_t n_req, int order,
+                           int residency, uint32_t* sd) {
+  if ((order != 0 && order != 1) || (residency != 0 && residency != 1)) return -1;
+  std::vector<uint32_t> stack;  // stack[0] is the most recent
+  auto find = [&](uint32_t id) -> uint32_t {
+    for (size_t pos = 0; pos < stack.size(); ++pos)
+      if (stack[pos] == id) return (uint32_t)(pos + 1);
+    return NONE;
+  };
+  auto touch = [&](uint32_t id) {
+    uint32_t d = find(id);
+    if (d != NONE) stack.erase(stack.begin() + (d - 1));
+    stack.insert(stack.begin(), id);
+  };
+  for (uint32_t r = 0; r < n_req; ++r) {
+    const uint64_t a = req_blk_off[r], m = req_blk_off[r + 1] - a;
+    if (residency == 1)
+      for (uint64_t k = 0; k < m; ++k) sd[a + k] = find(ids[a + k]);
+    for (uint64_t s = 0; s < m; ++s) {
+      const uint64_t k = order == 0 ? s : m - 1 - s;
+      if (residency == 0) sd[a + k] = find(ids[a + k]);
+      touch(ids[a + k]);
+    }
+  }
   return 0;
 }
 
