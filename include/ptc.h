@@ -11,6 +11,8 @@
  *     -> ptc_reuse_indices   previous / next use of each block Sec. 3.2, 5.2 (Belady's next access)
  *     -> ptc_stack_distance  LRU stack distance of each access App. B ("reuses reachable within C")
  *     -> ptc_curves          hits and compute saved per C      Sec. 3.2 (hit ratio), Sec. 5.2 (compute savings)
+ *   with, for the semantics variants (touch order, whole-request residency),
+ *        ptc_stack_distance_variant                           Sec. 3.1 (simulator)
  *   and, over the same arrays,
  *        ptc_trace_stats     lifetimes, reuse intervals, frequency, block categories,
  *                            session lengths, reuses reachable within C
@@ -216,6 +218,53 @@ enum { PTC_SD_AUTO = 0, PTC_SD_POINTS = 1, PTC_SD_RUNS = 2 };
 size_t ptc_stack_distance_ex_workspace_bytes(uint64_t n, int method);
 ptc_status ptc_stack_distance_ex(const uint32_t* prev, uint64_t n, uint32_t* dist_out, int method, void* ws,
                                  size_t ws_bytes, void* stream);
+
+/*
+ * ptc_stack_distance_variant — stack distances under the semantics variants
+ * of Sec. 3.1 (the paper's simulator keeps a whole request resident, making
+ * room for it before its prefill) and of the order a request's blocks are
+ * touched in.  The result feeds ptc_curves unchanged: block k of a request
+ * counts at capacity C iff the largest distance over its depths 0..k is <= C.
+ *   touch_order  PTC_TOUCH_ROOT_FIRST: depth 0, 1, ... (the hot path's order)
+ *                PTC_TOUCH_LEAF_FIRST: the deepest block first, the root last
+ *   residency    PTC_RESIDENCY_BLOCK:   each block is looked up when touched;
+ *                                       its distance is its LRU stack depth then
+ *                PTC_RESIDENCY_REQUEST: every block of a request is looked up at
+ *                                       the request's arrival, before any is
+ *                                       touched; its distance is its stack depth
+ *                                       at arrival (1 + distinct blocks touched
+ *                                       since its last touch and before the
+ *                                       request)
+ * Every request's blocks are then touched in touch_order.  (ROOT_FIRST, BLOCK)
+ * is ptc_stack_distance.
+ *   prev         u32[n] from ptc_reuse_indices (root-first access order)
+ *   req_blk_off  u64[n_req + 1] from ptc_hash_blocks, req_blk_off[n_req] == n
+ *   dist_out     u32[n] in root-first access order; PTC_NONE for a first access
+ * PTC_ERR_INVALID_ARG for other touch_order / residency values, malformed
+ * offsets, or prev[i] >= i.  Workspace:
+ * ptc_stack_distance_variant_workspace_bytes(n, n_req, touch_order, residency).
+ */
+enum { PTC_TOUCH_ROOT_FIRST = 0, PTC_TOUCH_LEAF_FIRST = 1 };
+enum { PTC_RESIDENCY_BLOCK = 0, PTC_RESIDENCY_REQUEST = 1 };
+size_t ptc_stack_distance_variant_workspace_bytes(uint64_t n, uint32_t n_req, int touch_order, int residency);
+ptc_status ptc_stack_distance_variant(const uint32_t* prev, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,
+                                      int touch_order, int residency, uint32_t* dist_out, void* ws, size_t ws_bytes,
+                                      void* stream);
+/*
+ * ptc_stack_distance_variant_ex — the same, with the route for per-request
+ * residency chosen by the caller.  Per request, dist = the per-block distance
+ * on the touch stream minus the number of the request's own earlier touches
+ * whose previous touch precedes this block's (a block touched after the
+ * request began is new to the shorter window iff that holds).  PTC_SD_RUNS
+ * counts them over the request's runs (prev growing by one, or first
+ * accesses), O(runs of the request) per access; PTC_SD_POINTS answers the
+ * window ending at the request's start on the matrix over every access;
+ * PTC_SD_AUTO takes the runs when they are at most a third of the accesses.
+ * Per-block residency ignores the method.  Same workspace size.
+ */
+ptc_status ptc_stack_distance_variant_ex(const uint32_t* prev, uint64_t n, const uint64_t* req_blk_off,
+                                         uint32_t n_req, int touch_order, int residency, uint32_t* dist_out,
+                                         int method, void* ws, size_t ws_bytes, void* stream);
 
 /*
  * ptc_curves — hit and compute-saved curves for every capacity at once

@@ -30,6 +30,8 @@ PTC_NONE = 0xFFFFFFFF
 PTC_COST_UNIFORM, PTC_COST_MEASURED, PTC_COST_LINEAR = 0, 1, 2
 PTC_SD_AUTO, PTC_SD_POINTS, PTC_SD_RUNS = 0, 1, 2
 PTC_REUSE_AUTO, PTC_REUSE_SORT, PTC_REUSE_RUNS = 0, 1, 2
+PTC_TOUCH_ROOT_FIRST, PTC_TOUCH_LEAF_FIRST = 0, 1
+PTC_RESIDENCY_BLOCK, PTC_RESIDENCY_REQUEST = 0, 1
 F_LIN = 6_600_000_000          # 2 x 3.3e9 active parameters, FLOPs per token
 F_ATTN = 4 * 48 * 32 * 128     # per attended position: 4 x layers x heads x head_dim
 MAX_CAPACITIES = 1024
@@ -121,6 +123,13 @@ def lib():
                 L.ptc_pipeline.argtypes = [vp, u64, vp, vp, u32, u32, u64, ctypes.POINTER(CostModel), vp, u32,
                                            vp, vp, vp, vp, vp, vp, ctypes.POINTER(u64), ctypes.POINTER(u64), vp, vp,
                                            ctypes.POINTER(U128), vp, sz, vp]
+                L.ptc_stack_distance_variant_workspace_bytes.restype = sz
+                L.ptc_stack_distance_variant_workspace_bytes.argtypes = [u64, u32, ctypes.c_int, ctypes.c_int]
+                L.ptc_stack_distance_variant.restype = st
+                L.ptc_stack_distance_variant.argtypes = [vp, u64, vp, u32, ctypes.c_int, ctypes.c_int, vp, vp, sz, vp]
+                L.ptc_stack_distance_variant_ex.restype = st
+                L.ptc_stack_distance_variant_ex.argtypes = [vp, u64, vp, u32, ctypes.c_int, ctypes.c_int, vp,
+                                                            ctypes.c_int, vp, sz, vp]
                 L.ptc_trace_stats_workspace_bytes.restype = sz
                 L.ptc_trace_stats_workspace_bytes.argtypes = [u64, u64, u32, u32]
                 L.ptc_trace_stats.restype = st
@@ -265,6 +274,27 @@ def ptc_stack_distance(prev: torch.Tensor, ws: torch.Tensor | None = None, metho
         w = _workspace(lib().ptc_stack_distance_ex_workspace_bytes(n, method), dev, ws)
         rc = lib().ptc_stack_distance_ex(_ptr(prev), n, _ptr(dist), method, _ptr(w), w.numel(), _stream(dev))
         _check("ptc_stack_distance_ex", rc)
+    return dist[:n]
+
+
+def ptc_stack_distance_variant(prev: torch.Tensor, req_blk_off: torch.Tensor, touch_order: int, residency: int,
+                               ws: torch.Tensor | None = None, method: int | None = None) -> torch.Tensor:
+    """Stack distances under a touch order (PTC_TOUCH_*) and a residency rule
+    (PTC_RESIDENCY_*), in root-first access order, ready for ptc_curves.
+    ``method`` (PTC_SD_AUTO / PTC_SD_POINTS / PTC_SD_RUNS) picks the route for
+    per-request residency through ptc_stack_distance_variant_ex."""
+    dev = _dev(req_blk_off)
+    n = prev.numel()
+    n_req = req_blk_off.numel() - 1
+    dist = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
+    w = _workspace(lib().ptc_stack_distance_variant_workspace_bytes(n, n_req, touch_order, residency), dev, ws)
+    if method is None:
+        rc = lib().ptc_stack_distance_variant(_ptr(prev), n, _ptr(req_blk_off), n_req, touch_order, residency,
+                                              _ptr(dist), _ptr(w), w.numel(), _stream(dev))
+    else:
+        rc = lib().ptc_stack_distance_variant_ex(_ptr(prev), n, _ptr(req_blk_off), n_req, touch_order, residency,
+                                                 _ptr(dist), method, _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_stack_distance_variant", rc)
     return dist[:n]
 
 

@@ -57,6 +57,18 @@ __device__ __forceinline__ void raise_err(DevStatus* st, uint32_t f) { atomicOr(
 // so the chain stays ordered end to end.
 __device__ __forceinline__ void grid_dep_sync() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
+// The request of access i: the largest r in [lo, hi] with off[r] <= i
+// (request block offsets, non-decreasing).
+__device__ __forceinline__ uint32_t req_search(const uint64_t* __restrict__ off, uint32_t lo, uint32_t hi,
+                                               uint64_t i) {
+  while (lo < hi) {
+    const uint32_t mid = lo + (hi - lo + 1) / 2;
+    if (__ldg(off + mid) <= i) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
 __device__ __forceinline__ uint32_t next_tile(DevStatus* st, int epoch) {
   __shared__ uint32_t s_tile;
   if (threadIdx.x == 0) s_tile = atomicAdd(&st->tile_ctr[epoch], 1u);

@@ -213,10 +213,12 @@ ptc_status curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* req_blk
                        uint32_t n_carry = 0);
 
 // Stage c on the matrix over every access (ptc_wavelet.cu); the C entry
-// points in ptc_runs.cu choose between it and the matrix over runs.
+// points in ptc_runs.cu choose between it and the matrix over runs.  With
+// `wend` (device, one entry per access) the window of access i ends at
+// wend[i] <= i instead of at i: dist = 1 + distinct values in (prev[i], wend[i]).
 size_t stack_distance_points_bytes(uint64_t n);
 ptc_status stack_distance_points(const uint32_t* prev, uint64_t n, uint32_t* dist_out, void* ws, size_t ws_bytes,
-                                 cudaStream_t s);
+                                 cudaStream_t s, const uint32_t* wend = nullptr);
 
 // Stage b by a radix sort of every access (ptc_sort.cu), and the same sort
 // for any (key, value) pairs; the C entry point in ptc_reuse.cu chooses.

@@ -57,17 +57,6 @@ __device__ __forceinline__ void flush(const uint32_t* s, ull* g, uint32_t len) {
     if (s[j]) atomicAdd(g + j, (ull)s[j]);
 }
 
-// Largest r in [lo, hi] with off[r] <= i.
-__device__ __forceinline__ uint32_t req_search(const uint64_t* __restrict__ off, uint32_t lo, uint32_t hi,
-                                               uint64_t i) {
-  while (lo < hi) {
-    const uint32_t mid = lo + (hi - lo + 1) / 2;
-    if (__ldg(off + mid) <= i) lo = mid;
-    else hi = mid - 1;
-  }
-  return lo;
-}
-
 struct ReqArgs {
   const uint64_t* off;
   const int64_t* ts;

@@ -347,6 +347,7 @@ struct RunValOp {
 
 struct QueryArgs {
   const uint32_t* prev;
+  const uint32_t* wend;  // window end of every access (null: the access itself)
   uint64_t n;
   uint32_t L;
   RankView rv;
@@ -378,6 +379,14 @@ __global__ void __launch_bounds__(kQThreads) k_wm_heads(QueryArgs a) {
     for (int j = 0; j < kQPer; ++j) p[j] = i0 + j < a.n ? a.prev[i0 + j] : kNone;
   }
   const uint32_t before = (i0 > 0 && i0 - 1 < a.n) ? a.prev[i0 - 1] : kNone;
+  // window ends: a run continues only within one window end (with window
+  // ends the distance then falls by one per access, see k_wm_propagate)
+  uint32_t we[kQPer + 1];
+#pragma unroll
+  for (int j = 0; j <= kQPer; ++j) {
+    const uint64_t i = i0 + j - 1;
+    we[j] = (a.wend && j + i0 > 0 && i < a.n) ? __ldg(a.wend + i) : 0u;
+  }
   RunVal loc{0, 0};
   uint32_t hbits = 0;
   bool bad = false;
@@ -386,18 +395,19 @@ __global__ void __launch_bounds__(kQThreads) k_wm_heads(QueryArgs a) {
     const uint64_t i = i0 + j;
     const uint32_t pj = p[j];
     const uint32_t pb = j ? p[j - 1] : before;
-    const bool member = pj != kNone && pb != kNone && pb + 1u == pj;
+    const bool member = pj != kNone && pb != kNone && pb + 1u == pj && we[j + 1] == we[j];
     if (i < a.n && !member) {
       uint32_t d = kNone;
       if (pj != kNone) {
-        if ((uint64_t)pj >= i)
+        const uint64_t e = a.wend ? (uint64_t)we[j + 1] : i;
+        if ((uint64_t)pj >= e || e > i)
           bad = true;
         else
-          d = 1 + range_count_less(a.rv, s_z, a.L, nmax, pj + 1, pj + 1, (uint32_t)i);
+          d = 1 + range_count_less(a.rv, s_z, a.L, nmax, pj + 1, pj + 1, (uint32_t)e);
       }
       a.dist[i] = d;
       hbits |= 1u << j;
-      loc = RunVal{d, 1};
+      loc = RunVal{(uint64_t)d + (a.wend ? i : 0), 1};  // the form k_wm_propagate carries
     }
   }
   if (bad) raise_err(a.st, kErrInvalid);
@@ -438,13 +448,17 @@ __global__ void __launch_bounds__(kQThreads) k_wm_propagate(QueryArgs a) {
     for (int j = 0; j < kQPer; ++j) d[j] = i0 + j < a.n ? a.dist[i0 + j] : 0u;
   }
   const uint32_t hbits = i0 < a.n ? a.heads[i0 / kQPer] : 0u;
+  // With window ends a run's distance falls by one per access (the window
+  // keeps its end and loses its first position), so the carried value is the
+  // head's distance plus the head's index, and access i takes it minus i.
+  const bool shift = a.wend != nullptr;
   RunVal loc{0, 0};
-  uint32_t val[kQPer];
+  uint64_t val[kQPer];
   uint32_t covered = 0;
 #pragma unroll
   for (int j = 0; j < kQPer; ++j) {
-    if ((hbits >> j) & 1u) loc = RunVal{d[j], 1};
-    val[j] = (uint32_t)loc.v;
+    if ((hbits >> j) & 1u) loc = RunVal{(uint64_t)d[j] + (shift ? i0 + j : 0), 1};
+    val[j] = loc.v;
     if (loc.f) covered |= 1u << j;
   }
   RunValOp op;
@@ -494,7 +508,8 @@ __global__ void __launch_bounds__(kQThreads) k_wm_propagate(QueryArgs a) {
   }
   uint32_t out[kQPer];
 #pragma unroll
-  for (int j = 0; j < kQPer; ++j) out[j] = ((covered >> j) & 1u) ? val[j] : (uint32_t)pre.v;
+  for (int j = 0; j < kQPer; ++j)
+    out[j] = (uint32_t)((((covered >> j) & 1u) ? val[j] : pre.v) - (shift ? i0 + j : 0));
   if (vec) {
     reinterpret_cast<uint4*>(a.dist + i0)[0] = make_uint4(out[0], out[1], out[2], out[3]);
     reinterpret_cast<uint4*>(a.dist + i0)[1] = make_uint4(out[4], out[5], out[6], out[7]);
@@ -567,7 +582,7 @@ size_t ptc::stack_distance_points_bytes(uint64_t n) { return wm_layout(nullptr, 
 
 // The matrix over every access (argument checks are the caller's).
 ptc_status ptc::stack_distance_points(const uint32_t* prev, uint64_t n, uint32_t* dist_out, void* ws,
-                                      size_t ws_bytes, cudaStream_t s) {
+                                      size_t ws_bytes, cudaStream_t s, const uint32_t* wend) {
   if (!ws_ok(ws, ws_bytes, wm_layout(nullptr, n).total)) return PTC_ERR_WORKSPACE;
   const WmLayout W = wm_layout(ws, n);
   if (begin_call(ws, W.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
@@ -608,6 +623,7 @@ ptc_status ptc::stack_distance_points(const uint32_t* prev, uint64_t n, uint32_t
   PTC_KERNEL("k_wm_dir", s, k_wm_dir, W.L * W.nchunk, kSbPerChunk, 0, W.bits, W.lw, W.L, W.nsb, W.nchunk, W.dir, W.csum, W.cpre, &W.done[63]);
   QueryArgs q;
   q.prev = prev;
+  q.wend = wend;
   q.n = n;
   q.L = W.L;
   q.rv = RankView{W.bits, W.lw, W.dir, W.cpre, W.nsb, W.nchunk};
