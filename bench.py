@@ -55,6 +55,9 @@ NCU_TRAFFIC: dict[str, tuple[float, str, str]] = {
 }
 
 
+VARIANTS = (("leaf_first", 1, 0), ("request_residency", 0, 1), ("leaf_first_request_residency", 1, 1))
+
+
 def parse_args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -340,6 +343,33 @@ def run_ours(args, ws_world, rank, local):
     st_kernels = {name: round(tot, 4) for name, _, tot in read_timer(ptc)}
     st_ms = max_over_ranks(sum(timed(args.steps, splan.run))) / args.steps
 
+    # ---- semantics variants (Sec. 3.1): stack distances under leaf-first
+    # touch order and whole-request residency from the step's prev, then the
+    # curves on them
+    variants, vdists = {}, {}
+    prev_t, rbo = outs["prev"][:N], outs["req_blk_off"]
+    mid = [0, G // 2, G - 1]
+    for vname, order, res in VARIANTS:
+        vws = torch.empty(L.ptc_stack_distance_variant_workspace_bytes(N, tr.n_req, order, res), dtype=torch.uint8,
+                          device=dev)
+        vdist = torch.empty(max(N, 1), dtype=torch.int32, device=dev)
+        vargs = (prev_t.data_ptr(), N, rbo.data_ptr(), tr.n_req, order, res, vdist.data_ptr(), vws.data_ptr(),
+                 vws.numel(), stream.cuda_stream)
+
+        def vrun(vargs=vargs):
+            rc = L.ptc_stack_distance_variant(*vargs)
+            assert rc == 0, rc
+
+        vrun()
+        v_ms = max_over_ranks(sum(timed(args.steps, vrun))) / args.steps
+        cur = ptc.ptc_curves(vdist[:N], rbo, BLOCK, caps)
+        variants[vname] = {"touch_order": "leaf-first" if order else "root-first",
+                           "residency": "per request" if res else "per block", "ms": round(v_ms, 4),
+                           "achieved_gbs_8n": round(8 * N / (v_ms * 1e-3) / 1e9, 1),
+                           "hit_ratio_at": {str(int(caps[g])): round(cur["hits"][g] / N, 5) for g in mid}}
+        vdists[vname] = (order, res, vdist[:N])
+        del vws
+
     # ---- roofline
     peak, peak_kind = measured_peaks()
     stages, Lbits = stage_model_bytes(T, N)
@@ -398,6 +428,9 @@ def run_ours(args, ws_world, rank, local):
             "categories": {"blocks": stats["blocks"].tolist(), "accesses": stats["accesses"].tolist(),
                            "one_hit_blocks": [int(stats["freq"][c, 1]) for c in range(3)]},
         },
+        "variants": {"call": "ptc_stack_distance_variant on the step's prev (distances in depth order for ptc_curves)",
+                     "bytes_model": "8 N: prev read, dist written", "hot_path_hit_ratio_at":
+                         {str(int(caps[g])): round(int(plan.hits[g]) / N, 5) for g in mid}, **variants},
     }
     if rank == 0 and ws_world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"], orc = cpu_baseline(tr, args.cpu_sample, stats=True)
@@ -406,6 +439,17 @@ def run_ours(args, ws_world, rank, local):
         if orc["n_req"] == tr.n_req:  # the sample is the whole trace: the oracle's statistics must match
             same = all(np.array_equal(np.asarray(ost[k]), np.asarray(stats[k])) for k in ost)
             assert same, "trace statistics differ from the oracle"
+        if orc["n_req"] == tr.n_req:  # the oracle's distances under every variant must match
+            import oracle
+            for vname, (order, res, vd) in vdists.items():
+                t0 = time.perf_counter()
+                want = oracle.sd_variant(orc["ids"], orc["D"], orc["off"], order, res)
+                dt = time.perf_counter() - t0
+                same_v = bool(np.array_equal(ptc.u32(vd), want))
+                assert same_v, f"variant {vname} differs from the oracle"
+                line["variants"][vname]["cpu_baseline"] = {
+                    "value": round(N / dt, 1), "unit": "accesses/s", "cores": 1, "kind": "oracle",
+                    "sample": f"orc_sd_variant (Fenwick) on the whole trace; {dt:.2f} s", "parity_with_gpu": same_v}
         line["trace_stats"]["cpu_baseline"] = {
             "value": round(orc["n"] / odt, 1), "unit": "accesses/s", "cores": 1, "kind": "oracle",
             "sample": f"orc_trace_stats on the oracle's own ids and distances of the first {orc['n_req']} requests "

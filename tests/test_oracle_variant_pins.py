@@ -166,3 +166,20 @@ def test_bad_variant_rejected():
         oracle.sd_variant(ids, 1, off, 2, 0)
     with pytest.raises(ValueError):
         oracle.lru_curves_variant(ids, off, 1, [1], 0, 3)
+
+
+@pytest.mark.parametrize("seed", range(10))
+def test_root_first_residency_leaves_hits_unchanged(seed):
+    """Root-first, whole-request residency counts the same hits as per-block
+    lookups.  Either way a counted block's shallower blocks were all found
+    resident, so touching them root-first only moved them to the front and
+    evicted nothing: the block's residency when touched is its residency at
+    arrival."""
+    rng = np.random.default_rng(8800 + seed)
+    B = int(rng.integers(1, 4))
+    tr = tracegen.tiny(seed, n_sessions=int(rng.integers(2, 9)), vocab=int(rng.integers(2, 5)))
+    ids, D, off = _setup(tr, B)
+    caps = list(range(1, D + 2))
+    per_block = oracle.lru_curves_variant(ids, off, B, caps, oracle.ROOT_FIRST, oracle.RES_BLOCK)
+    per_request = oracle.lru_curves_variant(ids, off, B, caps, oracle.ROOT_FIRST, oracle.RES_REQUEST)
+    assert per_block == per_request
