@@ -212,19 +212,27 @@ __global__ void __launch_bounds__(kGaThreads) k_ids_gather(const uint32_t* __res
   }
 }
 
-// Slots for n keys at most: the full table holds 1.5 n; the first attempt
-// holds n / 3 (real traces repeat most blocks, so it is rarely more than 40%
-// full and, at this size, stays in L2).  If a probe sequence of the first
-// attempt runs past kSmallProbeCap slots, the call redoes the stage with the
-// full table.
+// Slots for n keys at most: the full table holds 1.5 n.  The first attempt
+// holds n / 3 while that is at most 2^22 slots (64 MB, half of L2): traces
+// that repeat most blocks fill it well below half, and it stays in L2.  A
+// larger table lives in DRAM whatever its size, so there the first attempt
+// takes 3n / 4 slots instead: a trace that repeats few blocks (an agentic
+// trace, D near n / 2) then probes a table at most about half full rather
+// than one near 90% full, whose linear probe runs are tens of slots long.  If
+// a probe sequence of the first attempt runs past kSmallProbeCap slots, the
+// call redoes the stage with the full table.
 constexpr uint64_t kSmallProbeCap = 4096;
+constexpr uint32_t kL2TableLog2 = 22;
 uint32_t table_log2(uint64_t want) {
   uint32_t l = 10;
   while ((1ULL << l) < want) ++l;
   return l;
 }
 uint32_t full_table_log2(uint64_t n) { return table_log2(n + n / 2 + 64); }
-uint32_t small_table_log2(uint64_t n) { return table_log2(n / 3 + 64); }
+uint32_t small_table_log2(uint64_t n) {
+  const uint32_t l = table_log2(n / 3 + 64);
+  return l <= kL2TableLog2 ? l : table_log2(n / 4 * 3 + 64);
+}
 
 struct IdsLayout {
   DevStatus* st;
