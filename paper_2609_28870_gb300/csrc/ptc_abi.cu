@@ -115,6 +115,26 @@ __global__ void k_fill(uint32_t* __restrict__ p, uint32_t v, uint64_t words) {
   for (uint64_t w = quads * 4 + i; w < words; w += stride) p[w] = v;
 }
 
+struct FillMany {
+  uint32_t* p[kFillRanges];
+  uint64_t words[kFillRanges];
+  uint32_t v[kFillRanges];
+};
+
+__global__ void k_fill_many(FillMany a) {
+  grid_dep_sync();
+  const uint32_t r = blockIdx.y;
+  uint32_t* p = a.p[r];
+  const uint32_t v = a.v[r];
+  const uint64_t words = a.words[r];
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const uint64_t quads = (((uintptr_t)p & 15) == 0) ? words / 4 : 0;
+  uint4* p4 = reinterpret_cast<uint4*>(p);
+  for (uint64_t q = i; q < quads; q += stride) p4[q] = make_uint4(v, v, v, v);
+  for (uint64_t w = quads * 4 + i; w < words; w += stride) p[w] = v;
+}
+
 __global__ void k_copy_words(const uint32_t* __restrict__ src, uint32_t* dst, uint32_t words) {
   grid_dep_sync();
   const uint32_t tid = blockIdx.x * blockDim.x + threadIdx.x, nth = gridDim.x * blockDim.x;
@@ -150,6 +170,30 @@ ptc_status fill_async(void* p, uint32_t pattern, size_t bytes, cudaStream_t s) {
   const uint32_t cap = (uint32_t)(4 * num_sms());
   const uint32_t grid = want < cap ? (uint32_t)(want ? want : 1) : cap;
   PTC_KERNEL("k_fill", s, k_fill, grid, 256, 0, static_cast<uint32_t*>(p), pattern, words);
+  return PTC_OK;
+}
+
+ptc_status fill_many_async(const FillRange* r, int n, cudaStream_t s) {
+  FillMany a{};
+  uint32_t m = 0;
+  uint64_t most = 0;
+  for (int i = 0; i < n; ++i) {
+    if (r[i].bytes == 0) continue;
+    if ((r[i].bytes & 3) || ((uintptr_t)r[i].p & 3) || m == (uint32_t)kFillRanges) {
+      if (fill_async(r[i].p, r[i].pattern, r[i].bytes, s) != PTC_OK) return PTC_ERR_CUDA;
+      continue;
+    }
+    a.p[m] = static_cast<uint32_t*>(r[i].p);
+    a.words[m] = r[i].bytes / 4;
+    a.v[m] = r[i].pattern;
+    most = a.words[m] > most ? a.words[m] : most;
+    ++m;
+  }
+  if (m == 0) return PTC_OK;
+  const uint64_t want = (most / 4 + 255) / 256;
+  const uint32_t cap = (uint32_t)(4 * num_sms());
+  const uint32_t gx = want < cap ? (uint32_t)(want ? want : 1) : cap;
+  PTC_KERNEL("k_fill_many", s, k_fill_many, dim3(gx, m), 256, 0, a);
   return PTC_OK;
 }
 

@@ -18,7 +18,11 @@
 //                    (filled up to the longest request)
 //   k_hash16         B = 16, aligned tokens: the tile's request offsets in
 //                    shared memory, one block per thread
-//   k_hash_local     tokens staged through padded shared memory with 16-byte
+//   k_hash_tile      B any multiple of 16, aligned tokens: one block per
+//                    thread, its 16-token chunks hashed one after another
+//                    with two-limb products, 256-block tiles whatever B
+//   k_hash_local     any other B or tokens not 16-byte aligned: tokens
+//                    staged through padded shared memory with 16-byte
 //                    loads; each thread hashes 16 tokens (one "sub-chunk")
 //                    with 3 x 21-bit limbs of u^1..u^16 held as constant
 //                    kernel parameters; sub-chunks of one block combine by
@@ -219,8 +223,9 @@ __device__ __forceinline__ uint64_t mad_wide(uint32_t a, uint32_t b, uint64_t c)
 
 // Sum over the 16 words t[m .. m+15] of t * u^(j + 1) for both bases, as
 // 21-bit limb accumulators (M is the word offset of the first token).
-template <int M>
-__device__ __forceinline__ void hash16(const uint32_t (&wd)[20], const HashConsts& c, uint64_t (&acc)[6]) {
+template <int M, int NW>
+__device__ __forceinline__ void hash16(const uint32_t (&wd)[NW], const HashConsts& c, uint64_t (&acc)[6]) {
+  static_assert(M + 16 <= NW, "chunk words out of range");
 #pragma unroll
   for (int j = 0; j < 16; ++j) {
     const uint32_t t = wd[j + M];
@@ -235,8 +240,9 @@ __device__ __forceinline__ void hash16(const uint32_t (&wd)[20], const HashConst
 
 // The same sum with two limbs (31 + 30 bits), exact when every token is
 // below 2^27: 16 products of at most 2^58 stay below 2^62.
-template <int M>
-__device__ __forceinline__ void hash16_2(const uint32_t (&wd)[20], const HashConsts& c, uint64_t (&acc)[4]) {
+template <int M, int NW>
+__device__ __forceinline__ void hash16_2(const uint32_t (&wd)[NW], const HashConsts& c, uint64_t (&acc)[4]) {
+  static_assert(M + 16 <= NW, "chunk words out of range");
 #pragma unroll
   for (int j = 0; j < 16; ++j) {
     const uint32_t t = wd[j + M];
@@ -245,11 +251,6 @@ __device__ __forceinline__ void hash16_2(const uint32_t (&wd)[20], const HashCon
     acc[2] = mad_wide(t, c.limb2[1][0][j], acc[2]);
     acc[3] = mad_wide(t, c.limb2[1][1][j], acc[3]);
   }
-}
-
-// (a0 + a1 2^31) mod p for a0, a1 < 2^62: a1 2^31 = (a1 mod 2^30) 2^31 + (a1 >> 30) 2^61
-__device__ __forceinline__ uint64_t limbs2_to_p61(uint64_t a0, uint64_t a1) {
-  return p61_fold(p61_fold(a0) + ((a1 & ((1ULL << 30) - 1)) << 31) + (a1 >> 30));
 }
 
 // Congruent to (a0 + a1 2^31) mod p and below 2^61 + 3, for a0, a1 < 2^62.
@@ -469,75 +470,6 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local(HashArgs a, const _
     }
     h0 = p61_add(limbs_to_p61(a00, a01, a02), c.csum[0][FULL ? 16 : nval]);
     h1 = p61_add(limbs_to_p61(a10, a11, a12), c.csum[1][FULL ? 16 : nval]);
-    if (G > 1 && s > 0) {
-      h0 = p61_mul(h0, c.sub_mul[0][s]);
-      h1 = p61_mul(h1, c.sub_mul[1][s]);
-    }
-  }
-  hash_finish<G>(a, tile, b0, b_end, h0, h1, k, lb, s);
-}
-
-// Fast path for 16-byte-aligned tokens and B a multiple of 16: every thread
-// reads its 16 tokens with four or five 16-byte loads straight from global
-// memory (a warp's loads cover consecutive 64-byte runs, so each line is
-// fetched once) and realigns them by a word offset that is uniform over a
-// request.  No shared-memory staging.
-template <int G>
-__global__ void __launch_bounds__(kHashThreads) k_hash_local_vec(HashArgs a, const __grid_constant__ HashConsts c) {
-  grid_dep_sync();
-  __shared__ uint32_t s_bnd[2];
-  constexpr uint32_t TB = kHashThreads / G;
-  const uint32_t tile = blockIdx.x;
-  uint64_t N = a.st->value[0];
-  if (N > a.keys_cap) N = a.keys_cap;
-  const uint64_t b0 = (uint64_t)tile * TB;
-  if (b0 >= N) return;
-  const uint64_t b_end = b0 + TB < N ? b0 + TB : N;
-  if (threadIdx.x == 0) {
-    const uint64_t ntiles = (N + TB - 1) / TB;
-    const uint32_t r0 = a.tile_req[tile];
-    const uint32_t rh = tile + 1 < ntiles ? a.tile_req[tile + 1] : a.R - 1;
-    s_bnd[0] = r0;
-    s_bnd[1] = find_request(a.blk_off, r0, rh, b_end - 1);
-  }
-  __syncthreads();
-  const uint32_t r_first = s_bnd[0], r_last = s_bnd[1];
-  const uint32_t lb = threadIdx.x / G, s = threadIdx.x % G;
-  const uint64_t b = b0 + lb;
-  uint64_t h0 = 0, h1 = 0;
-  uint32_t k = 0;
-  if (b < b_end) {
-    const uint32_t r = find_request(a.blk_off, r_first, r_last, b);
-    k = (uint32_t)(b - a.blk_off[r]);
-    const uint64_t x = a.tok_off[r] + (uint64_t)a.B * k + 16ULL * s;
-    const uint32_t m = (uint32_t)(x & 3);
-    const uint64_t x4 = x - m;
-    uint32_t wd[20];
-    const uint4* p = reinterpret_cast<const uint4*>(a.tokens + x4);
-    const uint32_t nv = m ? 5u : 4u;
-    if (x4 + 4 * nv <= a.n_tok) {
-#pragma unroll
-      for (int q = 0; q < 5; ++q) {
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if ((uint32_t)q < nv) v = __ldg(p + q);
-        wd[4 * q] = v.x;
-        wd[4 * q + 1] = v.y;
-        wd[4 * q + 2] = v.z;
-        wd[4 * q + 3] = v.w;
-      }
-    } else {
-#pragma unroll
-      for (int q = 0; q < 20; ++q) wd[q] = x4 + q < a.n_tok ? a.tokens[x4 + q] : 0u;
-    }
-    uint64_t acc[6] = {0, 0, 0, 0, 0, 0};
-    switch (m) {
-      case 0: hash16<0>(wd, c, acc); break;
-      case 1: hash16<1>(wd, c, acc); break;
-      case 2: hash16<2>(wd, c, acc); break;
-      default: hash16<3>(wd, c, acc); break;
-    }
-    h0 = p61_add(limbs_to_p61(acc[0], acc[1], acc[2]), c.csum[0][16]);
-    h1 = p61_add(limbs_to_p61(acc[3], acc[4], acc[5]), c.csum[1][16]);
     if (G > 1 && s > 0) {
       h0 = p61_mul(h0, c.sub_mul[0][s]);
       h1 = p61_mul(h1, c.sub_mul[1][s]);
@@ -776,6 +708,299 @@ __global__ void __launch_bounds__(kHashThreads, 6) k_hash16(HashArgs a, const __
   }
 }
 
+// B a multiple of 16 (g = B / 16 chunks of 16 tokens) with 16-byte-aligned
+// tokens: P consecutive blocks per thread (one here; two would suit B = 16,
+// which k_hash16 takes), tiles of kHashThreads = 256 blocks whatever B,
+// kHashThreads / P threads per CTA, 64 registers.
+// The requests that meet the tile are tile_req[tile] .. tile_req[tile + 1];
+// their block and token offsets are loaded into shared memory once, so a
+// thread finds its request without a dependent chain of global loads.  A
+// thread hashes its P g chunks one after another in one loop (four or five
+// 16-byte loads each), so the code of the chunk product exists once and the
+// registers of one chunk are live at a time: h_b = sum over chunks s of
+// h_(b,s) u^(16 s).  The prefix sum then runs over one value per thread.
+// Tiles meeting more than kH16Req requests search the global offsets.
+// The 20 words x4 .. x4 + 19 of a 16-token chunk whose first token is word
+// m of them (the fifth 16-byte load only when m > 0).
+__device__ __forceinline__ void load_chunk(const HashArgs& a, uint64_t x4, uint32_t m, uint32_t (&wd)[20]) {
+  if (x4 + 20 <= a.n_tok) {
+    const uint4* q4 = reinterpret_cast<const uint4*>(a.tokens + x4);
+#pragma unroll
+    for (int q = 0; q < 5; ++q) {
+      uint4 v = make_uint4(0, 0, 0, 0);
+      if (q < 4 || m != 0) v = __ldcs(q4 + q);
+      wd[4 * q] = v.x;
+      wd[4 * q + 1] = v.y;
+      wd[4 * q + 2] = v.z;
+      wd[4 * q + 3] = v.w;
+    }
+  } else {  // within 20 words of the end of the token array
+#pragma unroll
+    for (int q = 0; q < 20; ++q) wd[q] = x4 + q < a.n_tok ? a.tokens[x4 + q] : 0u;
+  }
+}
+
+// h of the 16 tokens wd[M .. M+15] for both bases, every token below 2^27:
+// below 2^62 + 2.
+template <int M>
+__device__ __forceinline__ void chunk_narrow(const uint32_t (&wd)[20], const HashConsts& c, uint64_t& e0, uint64_t& e1) {
+  uint64_t acc[4] = {0, 0, 0, 0};
+  hash16_2<M>(wd, c, acc);
+  e0 = limbs2_lazy(acc[0], acc[1]) + c.csum[0][16];
+  e1 = limbs2_lazy(acc[2], acc[3]) + c.csum[1][16];
+}
+
+// The same for any 32-bit tokens (three limbs), fully reduced.
+template <int M>
+__device__ __forceinline__ void chunk_wide(const uint32_t (&wd)[20], const HashConsts& c, uint64_t& e0, uint64_t& e1) {
+  uint64_t acc[6] = {0, 0, 0, 0, 0, 0};
+  hash16<M>(wd, c, acc);
+  e0 = p61_add(limbs_to_p61(acc[0], acc[1], acc[2]), c.csum[0][16]);
+  e1 = p61_add(limbs_to_p61(acc[3], acc[4], acc[5]), c.csum[1][16]);
+}
+
+// Chunk s of block j (A or B) into the block's h: h_(b,s) u^(16 s), kept
+// below 2^62 + 2 by one fold.
+__device__ __forceinline__ void chunk_add(const HashConsts& c, uint32_t j, uint32_t s, uint64_t e0, uint64_t e1,
+                                          uint64_t& hA0, uint64_t& hA1, uint64_t& hB0, uint64_t& hB1) {
+  if (s > 0) {
+    e0 = p61_mul_lazy(e0, c.sub_mul[0][s]);
+    e1 = p61_mul_lazy(e1, c.sub_mul[1][s]);
+    hA0 += e0;
+    hA1 += e1;
+    hA0 = (hA0 & kP61) + (hA0 >> 61);
+    hA1 = (hA1 & kP61) + (hA1 >> 61);
+  } else if (j == 0) {
+    hA0 = e0;
+    hA1 = e1;
+  } else {
+    hB0 = e0;
+    hB1 = e1;
+  }
+}
+
+constexpr int kTileReq = 256;
+
+template <int P>
+__global__ void __launch_bounds__(kHashThreads / P, 8 / (3 - P)) k_hash_tile(HashArgs a,
+                                                                              const __grid_constant__ HashConsts c) {
+  constexpr int NT = kHashThreads / P;
+  constexpr uint32_t TB = kHashThreads;
+  grid_dep_sync();
+  __shared__ uint64_t s_boff[kTileReq + 1];
+  __shared__ uint64_t s_toff[kTileReq + 1];
+  __shared__ uint64_t s_p0[TB], s_p1[TB];
+  __shared__ uint64_t s_w0[NT / 32], s_w1[NT / 32];
+  const uint32_t tile = blockIdx.x;
+  uint64_t N = a.st->value[0];
+  if (N > a.keys_cap) N = a.keys_cap;
+  const uint64_t b0 = (uint64_t)tile * TB;
+  if (b0 >= N) return;
+  const uint64_t b_end = b0 + TB < N ? b0 + TB : N;
+  const uint64_t ntiles = (N + TB - 1) / TB;
+  const uint32_t r_first = a.tile_req[tile];
+  const uint32_t r_last = tile + 1 < ntiles ? a.tile_req[tile + 1] : a.R - 1;  // the last request meeting the tile
+  const uint32_t nreq = r_last - r_first + 1;
+  const bool cached = nreq <= kTileReq;
+  if (cached) {
+    for (uint32_t i = threadIdx.x; i <= nreq; i += NT) {
+      s_boff[i] = a.blk_off[r_first + i];
+      s_toff[i] = a.tok_off[r_first + i];
+    }
+  }
+  __syncthreads();
+  const uint32_t t = threadIdx.x, lane = t & 31, w = t >> 5;
+  const uint32_t g = a.B / 16;
+  const uint64_t bA = b0 + (uint64_t)P * t, bB = bA + 1;
+  const bool liveA = bA < b_end, liveB = P == 2 && bB < b_end;
+  // block A's request starts at block rsA, its tokens at xA; likewise B
+  uint64_t rsA = 0, rsB = 0, xA = 0, xB = 0;
+  if (liveA) {
+    if (cached) {  // largest i with s_boff[i] <= bA, then the same for bB
+      uint32_t lo = 0, hi = nreq - 1;
+      while (lo < hi) {
+        const uint32_t mid = (lo + hi + 1) >> 1;
+        if (s_boff[mid] <= bA)
+          lo = mid;
+        else
+          hi = mid - 1;
+      }
+      rsA = s_boff[lo];
+      xA = s_toff[lo] + (uint64_t)a.B * (bA - rsA);
+      if (P == 2) {
+        while (lo + 1 < nreq && s_boff[lo + 1] <= bB) ++lo;
+        rsB = s_boff[lo];
+        xB = s_toff[lo] + (uint64_t)a.B * (bB - rsB);
+      }
+    } else {
+      uint32_t r = find_request(a.blk_off, r_first, r_last, bA);
+      rsA = a.blk_off[r];
+      xA = a.tok_off[r] + (uint64_t)a.B * (bA - rsA);
+      if (P == 2) {
+        while (r < r_last && a.blk_off[r + 1] <= bB) ++r;
+        rsB = a.blk_off[r];
+        xB = a.tok_off[r] + (uint64_t)a.B * (bB - rsB);
+      }
+    }
+  }
+  // h of A and B: chunk s of block j at x_j + 16 s, below 2^62 + 2.  The
+  // loop takes every chunk with two-limb products; a thread that meets a
+  // token of 2^27 or more redoes all its chunks with three limbs in a second
+  // loop (never taken over a real vocabulary), so the two paths' registers
+  // are not live together.
+  uint64_t hA0 = 0, hA1 = 0, hB0 = 0, hB1 = 0;
+  bool wide = false;
+#pragma unroll 1
+  for (uint32_t ci = 0; ci < P * g; ++ci) {
+    const uint32_t j = P == 2 ? ci : 0u, s = P == 2 ? 0u : ci;
+    if (!(j == 0 ? liveA : liveB)) continue;
+    const uint64_t x = (j == 0 ? xA : xB) + 16ULL * s;
+    const uint32_t m = (uint32_t)(x & 3);
+    uint32_t wd[20];
+    load_chunk(a, x - m, m, wd);
+    uint32_t any = 0;  // words outside the chunk only widen the test
+#pragma unroll
+    for (int q = 0; q < 20; ++q) any |= wd[q];
+    if (any >> 27) {
+      wide = true;
+      continue;
+    }
+    uint64_t e0, e1;
+    switch (m) {
+      case 0: chunk_narrow<0>(wd, c, e0, e1); break;
+      case 1: chunk_narrow<1>(wd, c, e0, e1); break;
+      case 2: chunk_narrow<2>(wd, c, e0, e1); break;
+      default: chunk_narrow<3>(wd, c, e0, e1); break;
+    }
+    chunk_add(c, j, s, e0, e1, hA0, hA1, hB0, hB1);
+  }
+  if (wide) {
+#pragma unroll 1
+    for (uint32_t ci = 0; ci < P * g; ++ci) {
+      const uint32_t j = P == 2 ? ci : 0u, s = P == 2 ? 0u : ci;
+      if (!(j == 0 ? liveA : liveB)) continue;
+      const uint64_t x = (j == 0 ? xA : xB) + 16ULL * s;
+      const uint32_t m = (uint32_t)(x & 3);
+      uint32_t wd[20];
+      load_chunk(a, x - m, m, wd);
+      uint64_t e0, e1;
+      switch (m) {
+        case 0: chunk_wide<0>(wd, c, e0, e1); break;
+        case 1: chunk_wide<1>(wd, c, e0, e1); break;
+        case 2: chunk_wide<2>(wd, c, e0, e1); break;
+        default: chunk_wide<3>(wd, c, e0, e1); break;
+      }
+      chunk_add(c, j, s, e0, e1, hA0, hA1, hB0, hB1);
+    }
+  }
+  // g = h u^(B k) per block (the tables hold u^(B e)), below 2^61 + 5
+  const uint64_t* T = a.tables;
+  uint64_t vA0 = 0, vA1 = 0, vB0 = 0, vB1 = 0;
+  if (liveA) {
+    const uint32_t kA = (uint32_t)(bA - rsA);
+    vA0 = p61_mul_lazy(hA0, pow_at(T + 0 * 65536, T + 1 * 65536, kA));
+    vA1 = p61_mul_lazy(hA1, pow_at(T + 2 * 65536, T + 3 * 65536, kA));
+  }
+  if (liveB) {
+    const uint32_t kB = (uint32_t)(bB - rsB);
+    vB0 = p61_mul_lazy(hB0, pow_at(T + 0 * 65536, T + 1 * 65536, kB));
+    vB1 = p61_mul_lazy(hB1, pow_at(T + 2 * 65536, T + 3 * 65536, kB));
+  }
+  uint64_t v0 = vA0 + vB0, v1 = vA1 + vB1;  // below 2^62 + 10
+  v0 = (v0 & kP61) + (v0 >> 61);            // below 2^61 + 2
+  v1 = (v1 & kP61) + (v1 >> 61);
+  // warp scan with lazy reduction: from values below 2^61 + 5, two plain
+  // steps stay below 2^63 + 20; a fold (x & p) + (x >> 61) brings such a sum
+  // back below 2^61 + 4, so folding after d = 2 and d = 8 keeps every sum
+  // below 2^64 and leaves the result below 2^62 + 8
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const uint64_t y0 = __shfl_up_sync(kFull, v0, d), y1 = __shfl_up_sync(kFull, v1, d);
+    if (lane >= (uint32_t)d) {
+      v0 += y0;
+      v1 += y1;
+    }
+    if (d == 2 || d == 8) {
+      v0 = (v0 & kP61) + (v0 >> 61);
+      v1 = (v1 & kP61) + (v1 >> 61);
+    }
+  }
+  if (lane == 31) {
+    s_w0[w] = v0;
+    s_w1[w] = v1;
+  }
+  __syncthreads();
+  if (w == 0) {  // exclusive prefix of the warp totals
+    constexpr int NW = NT / 32;
+    uint64_t z0 = lane < NW ? s_w0[lane] : 0, z1 = lane < NW ? s_w1[lane] : 0;
+    const uint64_t o0 = z0, o1 = z1;
+#pragma unroll
+    for (int d = 1; d < NW; d <<= 1) {
+      const uint64_t y0 = __shfl_up_sync(kFull, z0, d), y1 = __shfl_up_sync(kFull, z1, d);
+      if (lane >= (uint32_t)d) {
+        z0 += y0;
+        z1 += y1;
+      }
+      z0 = (z0 & kP61) + (z0 >> 61);
+      z1 = (z1 & kP61) + (z1 >> 61);
+    }
+    if (lane < NW) {
+      s_w0[lane] = p61_fold(z0 + (kP61 << 2) - o0);  // z < 2^61 + 4, o < 2^62 + 8: stays in (0, 2^64)
+      s_w1[lane] = p61_fold(z1 + (kP61 << 2) - o1);
+    }
+  }
+  __syncthreads();
+  // inclusive prefix through this thread's last block (reduced), and through
+  // A when the thread holds two: that minus B's g
+  const uint64_t iB0 = p61_fold(v0 + s_w0[w]), iB1 = p61_fold(v1 + s_w1[w]);
+  const uint64_t iA0 = P == 2 ? p61_fold(iB0 + 2 * kP61 - vB0) : iB0;
+  const uint64_t iA1 = P == 2 ? p61_fold(iB1 + 2 * kP61 - vB1) : iB1;
+  s_p0[P * t] = iA0;
+  s_p1[P * t] = iA1;
+  if (P == 2) {
+    s_p0[P * t + 1] = iB0;
+    s_p1[P * t + 1] = iB1;
+  }
+  __syncthreads();
+  uint64_t kA0 = iA0, kA1 = iA1, kB0 = iB0, kB1 = iB1;
+  if (liveA && rsA > b0) {  // A's request starts inside the tile, after its first block
+    const uint32_t sl = (uint32_t)(rsA - b0) - 1;
+    kA0 = p61_add(kA0, kP61 - s_p0[sl]);
+    kA1 = p61_add(kA1, kP61 - s_p1[sl]);
+  }
+  if (liveB && rsB > b0) {
+    const uint32_t sl = (uint32_t)(rsB - b0) - 1;
+    kB0 = p61_add(kB0, kP61 - s_p0[sl]);
+    kB1 = p61_add(kB1, kP61 - s_p1[sl]);
+  }
+  if (liveA) a.keys[bA] = make_ulonglong2(kA0, kA1);
+  if (liveB) a.keys[bB] = make_ulonglong2(kB0, kB1);
+  // the tile's aggregate for the carry: the last block's sum since its
+  // request's start, and whether that start is in the tile; and the leading
+  // blocks (before the tile's first request start)
+  if (liveA && bA + 1 == b_end) a.tile_agg[tile] = HashCarry{kA0, kA1, rsA >= b0};
+  if (liveB && bB + 1 == b_end) a.tile_agg[tile] = HashCarry{kB0, kB1, rsB >= b0};
+  if (t == 0) {
+    uint32_t lead = (uint32_t)(b_end - b0);
+    if (cached) {
+      for (uint32_t i = 0; i < nreq; ++i)
+        if (s_boff[i] >= b0 && s_boff[i] < b_end && s_boff[i + 1] > s_boff[i]) {
+          lead = (uint32_t)(s_boff[i] - b0);
+          break;
+        }
+    } else {
+      for (uint32_t r = r_first; r <= r_last; ++r) {
+        const uint64_t st0 = a.blk_off[r];
+        if (st0 >= b0 && st0 < b_end && a.blk_off[r + 1] > st0) {
+          lead = (uint32_t)(st0 - b0);
+          break;
+        }
+      }
+    }
+    a.tile_lead[tile] = lead;
+  }
+}
+
 // Carry of every tile = the segmented sum of the aggregates of the tiles
 // before it, back to (and including) the nearest one where a request starts.
 // All aggregates exist before this kernel starts, so nothing waits.  One warp
@@ -886,8 +1111,8 @@ template <int G>
 void launch_hash(uint32_t grid, cudaStream_t s, const HashArgs& a, const HashConsts& c, bool full) {
   if (G == 1 && full && a.aligned)
     PTC_KERNEL("k_hash16", s, k_hash16, grid, kHashThreads, 0, a, c);
-  else if (full && a.aligned)
-    PTC_KERNEL("k_hash_local", s, k_hash_local_vec<G>, grid, kHashThreads, 0, a, c);
+  else if (a.aligned && a.B % 16 == 0)
+    PTC_KERNEL("k_hash_tile", s, k_hash_tile<1>, grid, kHashThreads, 0, a, c);
   else if (full)
     PTC_KERNEL("k_hash_local", s, (k_hash_local<G, true>), grid, kHashThreads, 0, a, c);
   else
@@ -899,6 +1124,15 @@ uint32_t chunks_per_block(uint32_t B) {  // G: power of two >= ceil(B / 16)
   while (g < need) g <<= 1;
   return g;
 }
+
+// Blocks per hash tile: kHashThreads for k_hash16 and k_hash_tile (B a
+// multiple of 16 over 16-byte-aligned tokens), one CTA's kHashThreads / G for
+// k_hash_local.  Arrays sized per tile take the smaller (the alignment of the
+// tokens is not known there).
+uint32_t tile_blocks(uint32_t B, bool aligned) {
+  return aligned && B % 16 == 0 ? (uint32_t)kHashThreads : kHashThreads / chunks_per_block(B);
+}
+uint32_t min_tile_blocks(uint32_t B) { return tile_blocks(B, false); }
 
 struct HashLayout {
   DevStatus* st;
@@ -917,7 +1151,7 @@ HashLayout hash_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   Carver cv(ws);
   const uint32_t off_tiles = ceil_div_u32(n_req, kOffTile) + 1;
   const uint64_t nb = n_tok / B < keys_cap ? n_tok / B : keys_cap;
-  const uint32_t tb = kHashThreads / chunks_per_block(B);
+  const uint32_t tb = min_tile_blocks(B);
   const uint32_t hash_tiles = ceil_div_u32(nb, tb) + 1;
   L.st = cv.take<DevStatus>(1);
   L.lb_off = cv.take<uint64_t>(off_tiles);
@@ -938,7 +1172,7 @@ using namespace ptc;
 
 uint64_t ptc::hash_carry_tiles(uint64_t n_tok, uint32_t block_size) {
   if (block_size == 0) block_size = 1;
-  return ceil_div_u32(n_tok / block_size, kHashThreads / chunks_per_block(block_size)) + 1;
+  return ceil_div_u32(n_tok / block_size, min_tile_blocks(block_size)) + 1;
 }
 
 extern "C" size_t ptc_hash_blocks_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size) {
@@ -969,7 +1203,9 @@ ptc_status ptc::hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t
     return end_call(L.st, s, &h);
   }
   const uint32_t G = chunks_per_block(block_size);
-  PTC_KERNEL("k_block_offsets", s, k_block_offsets, ceil_div_u32(n_req, kOffTile), kOffThreads, 0, req_tok_off, req_ts_us, n_req, n_tok, block_size, kHashThreads / G, req_blk_off_out, L.tile_req, L.hash_tiles, L.lb_off, L.st);
+  const bool aligned = (((uintptr_t)tokens) & 15) == 0;
+  const uint32_t tb = tile_blocks(block_size, aligned);
+  PTC_KERNEL("k_block_offsets", s, k_block_offsets, ceil_div_u32(n_req, kOffTile), kOffThreads, 0, req_tok_off, req_ts_us, n_req, n_tok, block_size, tb, req_blk_off_out, L.tile_req, L.hash_tiles, L.lb_off, L.st);
 
   // seeded bases and their derived constants
   PowBases pb;
@@ -1009,10 +1245,10 @@ ptc_status ptc::hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t
   a.tile_agg = L.tile_agg;
   a.tile_lead = L.tile_lead;
   a.st = L.st;
-  a.aligned = (((uintptr_t)tokens) & 15) == 0;
+  a.aligned = aligned;
   const bool full = block_size == 16 * G;
   const uint64_t nb = n_tok / block_size < keys_cap ? n_tok / block_size : keys_cap;
-  const uint32_t grid = ceil_div_u32(nb, kHashThreads / G);
+  const uint32_t grid = ceil_div_u32(nb, tb);
   if (grid > 0) {
     switch (G) {
       case 1: launch_hash<1>(grid, s, a, hc, full); break;
@@ -1024,11 +1260,11 @@ ptc_status ptc::hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t
     }
     if (carry) {
       PTC_KERNEL("k_hash_carry", s, k_hash_carry, ceil_div_u32(grid, kChainWarps * kCarryPer), kChainWarps * 32, 0, L.tile_agg,
-                 L.tile_lead, kHashThreads / G, L.st, keys_cap, grid, carry->carry, carry->lead);
-      carry->tile_blocks = kHashThreads / G;
+                 L.tile_lead, tb, L.st, keys_cap, grid, carry->carry, carry->lead);
+      carry->tile_blocks = tb;
     } else {
       PTC_KERNEL("k_hash_chain", s, k_hash_chain, ceil_div_u32(grid, kChainWarps), kChainWarps * 32, 0, a.keys,
-                 L.tile_agg, L.tile_lead, kHashThreads / G, L.st, keys_cap);
+                 L.tile_agg, L.tile_lead, tb, L.st, keys_cap);
     }
   }
   if (deferred) return defer_status(L.st, err_slot, s, n_slot, 0);

@@ -100,7 +100,7 @@ __device__ __forceinline__ void settle(ulonglong2* table, uint64_t mask, uint64_
 struct InsCarry {
   const ulonglong2* carry;
   const uint32_t* lead;
-  uint32_t tile_blocks;
+  uint32_t tile_shift;  // log2 of the blocks per hash tile (a power of two)
 };
 
 __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __restrict__ keys, uint32_t n_ub,
@@ -108,21 +108,34 @@ __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __
                                                             uint64_t probe_cap, uint32_t* __restrict__ slot_of,
                                                             DevStatus* st, InsCarry kc) {
   grid_dep_sync();
-  const uint32_t n = keys_used(n_ub, n_dev);
   const uint32_t i0 = blockIdx.x * (kInsThreads * kInsK) + threadIdx.x;
   const uint64_t mask = (1ULL << log2m) - 1;
-  ulonglong2 k[kInsK], cur[kInsK];
+  ulonglong2 k[kInsK], cur[kInsK], cy[kInsK];
+  uint32_t lead[kInsK];
   uint64_t pos[kInsK];
+  // Every load that does not depend on a key goes out first, together: the
+  // keys (the buffer holds n_ub of them, so reading up to n_ub stays inside
+  // it), their tiles' carries, and the key count.
 #pragma unroll
   for (int j = 0; j < kInsK; ++j) {
     const uint32_t i = i0 + j * kInsThreads;
-    k[j] = i < n ? __ldcs(&keys[i]) : make_ulonglong2(~0ULL, ~0ULL);  // streamed once: keep L2 for the table
-    if (kc.carry && i < n) {
-      const uint32_t t = i / kc.tile_blocks;
-      if (i - t * kc.tile_blocks < __ldg(&kc.lead[t]) && k[j].x < kP61 && k[j].y < kP61) {
-        const ulonglong2 c = __ldg(&kc.carry[t]);
-        k[j] = make_ulonglong2(p61_add(k[j].x, c.x), p61_add(k[j].y, c.y));
-      }
+    k[j] = i < n_ub ? __ldcs(&keys[i]) : make_ulonglong2(~0ULL, ~0ULL);  // streamed once: keep L2 for the table
+    lead[j] = 0;
+    cy[j] = make_ulonglong2(0, 0);
+    if (kc.carry && i < n_ub) {
+      const uint32_t t = i >> kc.tile_shift;
+      lead[j] = __ldg(&kc.lead[t]);
+      cy[j] = __ldg(&kc.carry[t]);
+    }
+  }
+  const uint32_t n = keys_used(n_ub, n_dev);
+#pragma unroll
+  for (int j = 0; j < kInsK; ++j) {
+    const uint32_t i = i0 + j * kInsThreads;
+    if (i >= n) {
+      k[j] = make_ulonglong2(~0ULL, ~0ULL);
+    } else if ((i & ((1u << kc.tile_shift) - 1u)) < lead[j] && k[j].x < kP61 && k[j].y < kP61) {
+      k[j] = make_ulonglong2(p61_add(k[j].x, cy[j].x), p61_add(k[j].y, cy[j].y));
     }
   }
 #pragma unroll
@@ -335,7 +348,9 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
                         uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
                         cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc,
                         uint64_t* nd_slot, uint32_t* err_slot, bool full_table) {
-  const InsCarry ic = kc ? InsCarry{kc->carry, kc->lead, kc->tile_blocks} : InsCarry{nullptr, nullptr, 1};
+  if (kc && (kc->tile_blocks == 0 || (kc->tile_blocks & (kc->tile_blocks - 1)) != 0)) return PTC_ERR_INVALID_ARG;
+  const InsCarry ic = kc ? InsCarry{kc->carry, kc->lead, (uint32_t)__builtin_ctz(kc->tile_blocks)}
+                        : InsCarry{nullptr, nullptr, 0};
   if (n_distinct_host_out == nullptr) return PTC_ERR_INVALID_ARG;
   *n_distinct_host_out = 0;
   if (n_used_host_out) *n_used_host_out = 0;
@@ -343,17 +358,20 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
   if (n > 0 && (keys == nullptr || ids_out == nullptr)) return PTC_ERR_INVALID_ARG;
   if (!ws_ok(ws, ws_bytes, ids_layout(nullptr, n).total)) return PTC_ERR_WORKSPACE;
   const IdsLayout L = ids_layout(ws, n);
-  auto start = [&]() -> bool {
-    return begin_call(ws, L.zero_bytes, s) == PTC_OK && carry_errors(carry_err, n_carry, L.st, s) == PTC_OK;
+  // the status block, the table (all ones: empty) and the first-occurrence
+  // bitmap are cleared by one launch
+  auto start = [&](uint32_t log2m) -> bool {
+    const FillRange zf[3] = {{ws, L.zero_bytes, 0u},
+                            {L.table, n > 0 ? sizeof(ulonglong2) << log2m : 0, ~0u},
+                            {L.bits, n > 0 ? sizeof(uint32_t) * L.nwords : 0, 0u}};
+    return fill_many_async(zf, 3, s) == PTC_OK && carry_errors(carry_err, n_carry, L.st, s) == PTC_OK;
   };
   auto run = [&](uint32_t log2m, uint64_t probe_cap) -> bool {
-    if (fill_async(L.table, ~0u, sizeof(ulonglong2) << log2m, s) != PTC_OK) return false;
     const ulonglong2* k = reinterpret_cast<const ulonglong2*>(keys);
     const uint32_t n32 = (uint32_t)n;
     PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads * kInsK), kInsThreads, 0, k, n32, n_dev, L.table,
                log2m, probe_cap, L.slot_of, L.st, ic);
     const uint64_t m = 1ULL << log2m;
-    if (fill_async(L.bits, 0u, sizeof(uint32_t) * L.nwords, s) != PTC_OK) return false;
     PTC_KERNEL("k_ids_mark", s, k_ids_mark, ceil_div_u32(m, kMkThreads * kMkPer), kMkThreads, 0, L.table, m, L.bits,
                n32, n_dev, L.st);
     if (bitmap_ranks(L.bits, L.nwords, L.wpre, L.tcnt, L.tpre, &L.done[0], &L.st->value[0], s) != PTC_OK) return false;
@@ -361,15 +379,16 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
                L.table, L.bits, L.wpre, n32, n_dev, ids_out);
     return true;
   };
-  if (!start()) return PTC_ERR_CUDA;
+  const uint32_t first_log2m = full_table ? L.log2m : small_table_log2(n);
+  if (!start(first_log2m)) return PTC_ERR_CUDA;
   DevStatus h{};
   if (nd_slot && err_slot) {  // one attempt, nothing waits
-    const uint32_t lg = full_table ? L.log2m : small_table_log2(n);
+    const uint32_t lg = first_log2m;
     if (n > 0 && !run(lg, lg < L.log2m ? kSmallProbeCap : ~0ULL)) return PTC_ERR_CUDA;
     return defer_status(L.st, err_slot, s, nd_slot, 0, 2);
   }
   if (n > 0) {
-    const uint32_t small = full_table ? L.log2m : small_table_log2(n);
+    const uint32_t small = first_log2m;
     if (!run(small, small < L.log2m ? kSmallProbeCap : ~0ULL)) return PTC_ERR_CUDA;
     if (small < L.log2m) {
       const ptc_status rc1 = end_call(L.st, s, &h);
@@ -380,7 +399,7 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
         return rc1;
       }
       // the small table overflowed: redo with the full one
-      if (!start() || !run(L.log2m, ~0ULL)) return PTC_ERR_CUDA;
+      if (!start(L.log2m) || !run(L.log2m, ~0ULL)) return PTC_ERR_CUDA;
     }
   }
   const ptc_status rc = end_call(L.st, s, &h);

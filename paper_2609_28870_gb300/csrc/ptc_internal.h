@@ -58,6 +58,17 @@ inline void launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 // sizes or addresses that are not whole 32-bit words go to cudaMemsetAsync.
 ptc_status fill_async(void* p, uint32_t pattern, size_t bytes, cudaStream_t s);
 
+// Several fills in one launch (one kernel, one grid row per range), for the
+// regions a call clears before its first kernel; a range that is not whole
+// 32-bit words goes to fill_async on its own.
+struct FillRange {
+  void* p;
+  size_t bytes;
+  uint32_t pattern;
+};
+constexpr int kFillRanges = 4;
+ptc_status fill_many_async(const FillRange* r, int n, cudaStream_t s);
+
 // Zero the status block (and any extra prefix of the workspace) on `stream`.
 inline ptc_status begin_call(void* ws, size_t zero_bytes, cudaStream_t stream) {
   return fill_async(ws, 0u, zero_bytes, stream);
@@ -155,7 +166,8 @@ struct RunsView {
 };
 // Keys left without the carry from earlier tiles (stage a1 skips its
 // chain pass): block i of tile t = i / tile_blocks still needs carry[t] added
-// (mod p, per word) when i - t tile_blocks < lead[t].  Device arrays of
+// (mod p, per word) when i - t tile_blocks < lead[t]; tile_blocks is a power
+// of two.  Device arrays of
 // hash_carry_tiles() entries, owned by the caller.
 struct KeyCarry {
   ulonglong2* carry;

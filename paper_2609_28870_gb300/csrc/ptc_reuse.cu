@@ -410,8 +410,8 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
                          const ReuseDevIn* din = nullptr, ReuseHostOut* hout = nullptr) {
   const ReuseLayout L = reuse_layout(ws, n, D, forced);
   if (!ws_ok(ws, ws_bytes, L.total)) return PTC_ERR_WORKSPACE;
-  if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
-  if (fill_async(L.cut, 0u, sizeof(uint32_t) * L.nwords, s) != PTC_OK) return PTC_ERR_CUDA;
+  const FillRange zf[2] = {{ws, L.zero_bytes, 0u}, {L.cut, sizeof(uint32_t) * L.nwords, 0u}};
+  if (fill_many_async(zf, 2, s) != PTC_OK) return PTC_ERR_CUDA;
   IrArgs a;
   a.ids = ids;
   a.n = (uint32_t)n;

@@ -748,8 +748,8 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   const bool fits = R >= 1 && R <= n && ws_bytes >= W.total;
   if (method == PTC_SD_AUTO && (!fits || R > n / 3)) return stack_distance_points(prev, n, dist_out, ws, ws_bytes, s);
   if (!fits) return PTC_ERR_WORKSPACE;
-  if (fill_async(W.acc, 0u, W.acc_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
-  if (fill_async(W.done, 0u, 64 * sizeof(uint32_t), s) != PTC_OK) return PTC_ERR_CUDA;
+  const FillRange zf[2] = {{W.acc, W.acc_bytes, 0u}, {W.done, 64 * sizeof(uint32_t), 0u}};
+  if (fill_many_async(zf, 2, s) != PTC_OK) return PTC_ERR_CUDA;
   const uint32_t R32 = (uint32_t)R, T = W.rtiles, L = W.L;
   const size_t tstride = (size_t)T + 1;
   // one cluster when the runs fit in its shared memory, else one launch per level
