@@ -51,7 +51,7 @@ NOMINAL_HBM_GBS = 7900.0
 NCU_TRAFFIC: dict[str, tuple[float, str, str]] = {
     # 6,000-request capture (profiles/k_hash16_chat_6000req.md), scaled to the
     # full workload by tokens
-    "k_hash16": (639.5e6, "7183762f6db4895e", "ncu --set full, first 6,000 requests, x 153.81 / 55.67"),
+    "k_hash16": (640.0e6, "10d7d4bebd635899", "ncu --set full, first 6,000 requests, x 153.81 / 55.67"),
 }
 
 
@@ -141,7 +141,7 @@ def kernel_model_bytes(name, T, N, L, D):
 
 KERNEL_SOURCE = {
     "k_block_offsets": "ptc_hash.cu", "k_pow_tables": "ptc_hash.cu", "k_hash_local": "ptc_hash.cu",
-    "k_hash16": "ptc_hash.cu",
+    "k_hash16": "ptc_hash.cu", "k_hash_tile": "ptc_hash.cu", "k_fill_many": "ptc_abi.cu",
     "k_hash_chain": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu", "k_ids_mark": "ptc_ids.cu",
     "k_ids_gather": "ptc_ids.cu", "k_sort_count": "ptc_sort.cu", "k_sort_rowscan": "ptc_sort.cu",
     "k_sort_scatter": "ptc_sort.cu", "k_sort_links": "ptc_sort.cu", "k_ir_count": "ptc_reuse.cu",
