@@ -51,7 +51,7 @@ NOMINAL_HBM_GBS = 7900.0
 NCU_TRAFFIC: dict[str, tuple[float, str, str]] = {
     # 6,000-request capture (profiles/k_hash16_chat_6000req.md), scaled to the
     # full workload by tokens
-    "k_hash16": (640.0e6, "10d7d4bebd635899", "ncu --set full, first 6,000 requests, x 153.81 / 55.67"),
+    "k_hash16": (645.6e6, "35e274868498a45b", "ncu --set full, first 6,000 requests, x 153.81 / 55.67"),
 }
 
 

@@ -479,8 +479,10 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local(HashArgs a, const _
 }
 
 // B = 16 with 16-byte-aligned tokens: one block per thread, kHashThreads =
-// 256 blocks per tile (as k_hash_local with G = 1), six CTAs per SM, so that
-// a CTA waiting at one of its barriers leaves five others to issue.  The requests that meet the tile are
+// 256 blocks per tile (as k_hash_local with G = 1), eight CTAs per SM (32
+// registers; a few values spill to L1, which measured faster than six CTAs
+// at 40 registers), so that a CTA waiting at one of its barriers leaves seven
+// others to issue.  The requests that meet the tile are
 // tile_req[tile] .. tile_req[tile + 1]; their block and token offsets are
 // loaded into shared memory once, so a thread finds its request without a
 // dependent chain of global loads, and its token loads and power-table loads
@@ -488,7 +490,7 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local(HashArgs a, const _
 // global offsets instead.
 constexpr int kH16Req = 256;
 
-__global__ void __launch_bounds__(kHashThreads, 6) k_hash16(HashArgs a, const __grid_constant__ HashConsts c) {
+__global__ void __launch_bounds__(kHashThreads, 8) k_hash16(HashArgs a, const __grid_constant__ HashConsts c) {
   grid_dep_sync();
   __shared__ uint64_t s_boff[kH16Req + 1];
   __shared__ uint64_t s_toff[kH16Req + 1];
@@ -759,38 +761,40 @@ __device__ __forceinline__ void chunk_wide(const uint32_t (&wd)[20], const HashC
   e1 = p61_add(limbs_to_p61(acc[3], acc[4], acc[5]), c.csum[1][16]);
 }
 
-// Chunk s of block j (A or B) into the block's h: h_(b,s) u^(16 s), kept
-// below 2^62 + 2 by one fold.
-__device__ __forceinline__ void chunk_add(const HashConsts& c, uint32_t j, uint32_t s, uint64_t e0, uint64_t e1,
-                                          uint64_t& hA0, uint64_t& hA1, uint64_t& hB0, uint64_t& hB1) {
-  if (s > 0) {
-    e0 = p61_mul_lazy(e0, c.sub_mul[0][s]);
-    e1 = p61_mul_lazy(e1, c.sub_mul[1][s]);
-    hA0 += e0;
-    hA1 += e1;
-    hA0 = (hA0 & kP61) + (hA0 >> 61);
-    hA1 = (hA1 & kP61) + (hA1 >> 61);
-  } else if (j == 0) {
-    hA0 = e0;
-    hA1 = e1;
-  } else {
-    hB0 = e0;
-    hB1 = e1;
+// Chunk s of a block into its h: h_s u^(16 s) added to the chunks before,
+// kept below 2^62 + 2 by one fold (the first chunk is taken as it is).
+__device__ __forceinline__ void chunk_add(const HashConsts& c, uint32_t s, uint64_t e0, uint64_t e1, uint64_t& h0,
+                                          uint64_t& h1) {
+  if (s == 0) {
+    h0 = e0;
+    h1 = e1;
+    return;
   }
+  h0 += p61_mul_lazy(e0, c.sub_mul[0][s]);
+  h1 += p61_mul_lazy(e1, c.sub_mul[1][s]);
+  h0 = (h0 & kP61) + (h0 >> 61);
+  h1 = (h1 & kP61) + (h1 >> 61);
 }
 
+// B a multiple of 16 (g = B / 16 chunks of 16 tokens) with 16-byte-aligned
+// tokens, B > 16: one block per thread, tiles of kHashThreads = 256 blocks
+// whatever B, four CTAs per SM (64 registers).  The requests that meet the
+// tile are tile_req[tile] .. tile_req[tile + 1]; their block and token
+// offsets are loaded into shared memory once, so a thread finds its request
+// without a dependent chain of global loads.  A thread hashes its block's g
+// chunks one after another in one loop (four or five 16-byte loads each), so
+// the code of the chunk product exists once and the registers of one chunk
+// are live at a time: h = sum over chunks s of h_s u^(16 s).  Tiles meeting
+// more than kTileReq requests search the global offsets.
 constexpr int kTileReq = 256;
 
-template <int P>
-__global__ void __launch_bounds__(kHashThreads / P, 8 / (3 - P)) k_hash_tile(HashArgs a,
-                                                                              const __grid_constant__ HashConsts c) {
-  constexpr int NT = kHashThreads / P;
+__global__ void __launch_bounds__(kHashThreads, 4) k_hash_tile(HashArgs a, const __grid_constant__ HashConsts c) {
   constexpr uint32_t TB = kHashThreads;
   grid_dep_sync();
   __shared__ uint64_t s_boff[kTileReq + 1];
   __shared__ uint64_t s_toff[kTileReq + 1];
   __shared__ uint64_t s_p0[TB], s_p1[TB];
-  __shared__ uint64_t s_w0[NT / 32], s_w1[NT / 32];
+  __shared__ uint64_t s_w0[TB / 32], s_w1[TB / 32];
   const uint32_t tile = blockIdx.x;
   uint64_t N = a.st->value[0];
   if (N > a.keys_cap) N = a.keys_cap;
@@ -803,7 +807,7 @@ __global__ void __launch_bounds__(kHashThreads / P, 8 / (3 - P)) k_hash_tile(Has
   const uint32_t nreq = r_last - r_first + 1;
   const bool cached = nreq <= kTileReq;
   if (cached) {
-    for (uint32_t i = threadIdx.x; i <= nreq; i += NT) {
+    for (uint32_t i = threadIdx.x; i <= nreq; i += TB) {
       s_boff[i] = a.blk_off[r_first + i];
       s_toff[i] = a.tok_off[r_first + i];
     }
@@ -811,75 +815,65 @@ __global__ void __launch_bounds__(kHashThreads / P, 8 / (3 - P)) k_hash_tile(Has
   __syncthreads();
   const uint32_t t = threadIdx.x, lane = t & 31, w = t >> 5;
   const uint32_t g = a.B / 16;
-  const uint64_t bA = b0 + (uint64_t)P * t, bB = bA + 1;
-  const bool liveA = bA < b_end, liveB = P == 2 && bB < b_end;
-  // block A's request starts at block rsA, its tokens at xA; likewise B
-  uint64_t rsA = 0, rsB = 0, xA = 0, xB = 0;
-  if (liveA) {
-    if (cached) {  // largest i with s_boff[i] <= bA, then the same for bB
+  const uint64_t b = b0 + t;
+  const bool live = b < b_end;
+  // the block's request starts at block rs, the block's tokens at xb
+  uint64_t rs = 0, xb = 0;
+  if (live) {
+    if (cached) {  // largest i with s_boff[i] <= b
       uint32_t lo = 0, hi = nreq - 1;
       while (lo < hi) {
         const uint32_t mid = (lo + hi + 1) >> 1;
-        if (s_boff[mid] <= bA)
+        if (s_boff[mid] <= b)
           lo = mid;
         else
           hi = mid - 1;
       }
-      rsA = s_boff[lo];
-      xA = s_toff[lo] + (uint64_t)a.B * (bA - rsA);
-      if (P == 2) {
-        while (lo + 1 < nreq && s_boff[lo + 1] <= bB) ++lo;
-        rsB = s_boff[lo];
-        xB = s_toff[lo] + (uint64_t)a.B * (bB - rsB);
-      }
+      rs = s_boff[lo];
+      xb = s_toff[lo] + (uint64_t)a.B * (b - rs);
     } else {
-      uint32_t r = find_request(a.blk_off, r_first, r_last, bA);
-      rsA = a.blk_off[r];
-      xA = a.tok_off[r] + (uint64_t)a.B * (bA - rsA);
-      if (P == 2) {
-        while (r < r_last && a.blk_off[r + 1] <= bB) ++r;
-        rsB = a.blk_off[r];
-        xB = a.tok_off[r] + (uint64_t)a.B * (bB - rsB);
-      }
+      const uint32_t r = find_request(a.blk_off, r_first, r_last, b);
+      rs = a.blk_off[r];
+      xb = a.tok_off[r] + (uint64_t)a.B * (b - rs);
     }
   }
-  // h of A and B: chunk s of block j at x_j + 16 s, below 2^62 + 2.  The
-  // loop takes every chunk with two-limb products; a thread that meets a
-  // token of 2^27 or more redoes all its chunks with three limbs in a second
-  // loop (never taken over a real vocabulary), so the two paths' registers
-  // are not live together.
-  uint64_t hA0 = 0, hA1 = 0, hB0 = 0, hB1 = 0;
+  // h of the block, below 2^62 + 2.  The loop takes every chunk with
+  // two-limb products; a block with a token of 2^27 or more is redone with
+  // three limbs in a second loop (never taken over a real vocabulary), so
+  // the two paths' registers are not live together.  (Loop bounds rather than
+  // an enclosing branch, and the first loop running to its end: this shape
+  // spills the fewest registers at 64.)
+  uint64_t h0 = 0, h1 = 0;
   bool wide = false;
+  const uint32_t gl = live ? g : 0u;
+  {
 #pragma unroll 1
-  for (uint32_t ci = 0; ci < P * g; ++ci) {
-    const uint32_t j = P == 2 ? ci : 0u, s = P == 2 ? 0u : ci;
-    if (!(j == 0 ? liveA : liveB)) continue;
-    const uint64_t x = (j == 0 ? xA : xB) + 16ULL * s;
-    const uint32_t m = (uint32_t)(x & 3);
-    uint32_t wd[20];
-    load_chunk(a, x - m, m, wd);
-    uint32_t any = 0;  // words outside the chunk only widen the test
+    for (uint32_t s = 0; s < gl; ++s) {
+      const uint64_t x = xb + 16ULL * s;
+      const uint32_t m = (uint32_t)(x & 3);
+      uint32_t wd[20];
+      load_chunk(a, x - m, m, wd);
+      uint32_t any = 0;  // words outside the chunk only widen the test
 #pragma unroll
-    for (int q = 0; q < 20; ++q) any |= wd[q];
-    if (any >> 27) {
-      wide = true;
-      continue;
+      for (int q = 0; q < 20; ++q) any |= wd[q];
+      if (any >> 27) {
+        wide = true;
+        continue;
+      }
+      uint64_t e0, e1;
+      switch (m) {
+        case 0: chunk_narrow<0>(wd, c, e0, e1); break;
+        case 1: chunk_narrow<1>(wd, c, e0, e1); break;
+        case 2: chunk_narrow<2>(wd, c, e0, e1); break;
+        default: chunk_narrow<3>(wd, c, e0, e1); break;
+      }
+      chunk_add(c, s, e0, e1, h0, h1);
     }
-    uint64_t e0, e1;
-    switch (m) {
-      case 0: chunk_narrow<0>(wd, c, e0, e1); break;
-      case 1: chunk_narrow<1>(wd, c, e0, e1); break;
-      case 2: chunk_narrow<2>(wd, c, e0, e1); break;
-      default: chunk_narrow<3>(wd, c, e0, e1); break;
-    }
-    chunk_add(c, j, s, e0, e1, hA0, hA1, hB0, hB1);
   }
   if (wide) {
 #pragma unroll 1
-    for (uint32_t ci = 0; ci < P * g; ++ci) {
-      const uint32_t j = P == 2 ? ci : 0u, s = P == 2 ? 0u : ci;
-      if (!(j == 0 ? liveA : liveB)) continue;
-      const uint64_t x = (j == 0 ? xA : xB) + 16ULL * s;
+    for (uint32_t s = 0; s < g; ++s) {
+      const uint64_t x = xb + 16ULL * s;
       const uint32_t m = (uint32_t)(x & 3);
       uint32_t wd[20];
       load_chunk(a, x - m, m, wd);
@@ -890,25 +884,19 @@ __global__ void __launch_bounds__(kHashThreads / P, 8 / (3 - P)) k_hash_tile(Has
         case 2: chunk_wide<2>(wd, c, e0, e1); break;
         default: chunk_wide<3>(wd, c, e0, e1); break;
       }
-      chunk_add(c, j, s, e0, e1, hA0, hA1, hB0, hB1);
+      chunk_add(c, s, e0, e1, h0, h1);
     }
   }
-  // g = h u^(B k) per block (the tables hold u^(B e)), below 2^61 + 5
+  // g = h u^(B k) for the block's depth k (the tables hold u^(B e)), below
+  // 2^61 + 5, then a plain prefix sum over the tile; a block whose request
+  // starts inside the tile at index s subtracts the prefix before s.
   const uint64_t* T = a.tables;
-  uint64_t vA0 = 0, vA1 = 0, vB0 = 0, vB1 = 0;
-  if (liveA) {
-    const uint32_t kA = (uint32_t)(bA - rsA);
-    vA0 = p61_mul_lazy(hA0, pow_at(T + 0 * 65536, T + 1 * 65536, kA));
-    vA1 = p61_mul_lazy(hA1, pow_at(T + 2 * 65536, T + 3 * 65536, kA));
+  uint64_t v0 = 0, v1 = 0;
+  if (live) {
+    const uint32_t k = (uint32_t)(b - rs);
+    v0 = p61_mul_lazy(h0, pow_at(T + 0 * 65536, T + 1 * 65536, k));
+    v1 = p61_mul_lazy(h1, pow_at(T + 2 * 65536, T + 3 * 65536, k));
   }
-  if (liveB) {
-    const uint32_t kB = (uint32_t)(bB - rsB);
-    vB0 = p61_mul_lazy(hB0, pow_at(T + 0 * 65536, T + 1 * 65536, kB));
-    vB1 = p61_mul_lazy(hB1, pow_at(T + 2 * 65536, T + 3 * 65536, kB));
-  }
-  uint64_t v0 = vA0 + vB0, v1 = vA1 + vB1;  // below 2^62 + 10
-  v0 = (v0 & kP61) + (v0 >> 61);            // below 2^61 + 2
-  v1 = (v1 & kP61) + (v1 >> 61);
   // warp scan with lazy reduction: from values below 2^61 + 5, two plain
   // steps stay below 2^63 + 20; a fold (x & p) + (x >> 61) brings such a sum
   // back below 2^61 + 4, so folding after d = 2 and d = 8 keeps every sum
@@ -931,7 +919,7 @@ __global__ void __launch_bounds__(kHashThreads / P, 8 / (3 - P)) k_hash_tile(Has
   }
   __syncthreads();
   if (w == 0) {  // exclusive prefix of the warp totals
-    constexpr int NW = NT / 32;
+    constexpr int NW = TB / 32;
     uint64_t z0 = lane < NW ? s_w0[lane] : 0, z1 = lane < NW ? s_w1[lane] : 0;
     const uint64_t o0 = z0, o1 = z1;
 #pragma unroll
@@ -950,36 +938,21 @@ __global__ void __launch_bounds__(kHashThreads / P, 8 / (3 - P)) k_hash_tile(Has
     }
   }
   __syncthreads();
-  // inclusive prefix through this thread's last block (reduced), and through
-  // A when the thread holds two: that minus B's g
-  const uint64_t iB0 = p61_fold(v0 + s_w0[w]), iB1 = p61_fold(v1 + s_w1[w]);
-  const uint64_t iA0 = P == 2 ? p61_fold(iB0 + 2 * kP61 - vB0) : iB0;
-  const uint64_t iA1 = P == 2 ? p61_fold(iB1 + 2 * kP61 - vB1) : iB1;
-  s_p0[P * t] = iA0;
-  s_p1[P * t] = iA1;
-  if (P == 2) {
-    s_p0[P * t + 1] = iB0;
-    s_p1[P * t + 1] = iB1;
-  }
+  v0 = p61_fold(v0 + s_w0[w]);
+  v1 = p61_fold(v1 + s_w1[w]);
+  s_p0[t] = v0;
+  s_p1[t] = v1;
   __syncthreads();
-  uint64_t kA0 = iA0, kA1 = iA1, kB0 = iB0, kB1 = iB1;
-  if (liveA && rsA > b0) {  // A's request starts inside the tile, after its first block
-    const uint32_t sl = (uint32_t)(rsA - b0) - 1;
-    kA0 = p61_add(kA0, kP61 - s_p0[sl]);
-    kA1 = p61_add(kA1, kP61 - s_p1[sl]);
+  if (live && rs > b0) {  // the request starts inside the tile, after its first block
+    const uint32_t sl = (uint32_t)(rs - b0) - 1;
+    v0 = p61_add(v0, kP61 - s_p0[sl]);
+    v1 = p61_add(v1, kP61 - s_p1[sl]);
   }
-  if (liveB && rsB > b0) {
-    const uint32_t sl = (uint32_t)(rsB - b0) - 1;
-    kB0 = p61_add(kB0, kP61 - s_p0[sl]);
-    kB1 = p61_add(kB1, kP61 - s_p1[sl]);
-  }
-  if (liveA) a.keys[bA] = make_ulonglong2(kA0, kA1);
-  if (liveB) a.keys[bB] = make_ulonglong2(kB0, kB1);
+  if (live) a.keys[b] = make_ulonglong2(v0, v1);
   // the tile's aggregate for the carry: the last block's sum since its
   // request's start, and whether that start is in the tile; and the leading
   // blocks (before the tile's first request start)
-  if (liveA && bA + 1 == b_end) a.tile_agg[tile] = HashCarry{kA0, kA1, rsA >= b0};
-  if (liveB && bB + 1 == b_end) a.tile_agg[tile] = HashCarry{kB0, kB1, rsB >= b0};
+  if (live && b + 1 == b_end) a.tile_agg[tile] = HashCarry{v0, v1, rs >= b0};
   if (t == 0) {
     uint32_t lead = (uint32_t)(b_end - b0);
     if (cached) {
@@ -1112,7 +1085,7 @@ void launch_hash(uint32_t grid, cudaStream_t s, const HashArgs& a, const HashCon
   if (G == 1 && full && a.aligned)
     PTC_KERNEL("k_hash16", s, k_hash16, grid, kHashThreads, 0, a, c);
   else if (a.aligned && a.B % 16 == 0)
-    PTC_KERNEL("k_hash_tile", s, k_hash_tile<1>, grid, kHashThreads, 0, a, c);
+    PTC_KERNEL("k_hash_tile", s, k_hash_tile, grid, kHashThreads, 0, a, c);
   else if (full)
     PTC_KERNEL("k_hash_local", s, (k_hash_local<G, true>), grid, kHashThreads, 0, a, c);
   else
