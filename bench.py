@@ -126,6 +126,7 @@ def kernel_model_bytes(name, T, N, L, D):
     return {
         "k_hash_local": 4 * T + 16 * N,   # token stream in, block keys out
         "k_hash16": 4 * T + 16 * N,       # the same, B = 16 path
+        "k_hash_tile": 4 * T + 16 * N,    # the same, other multiples of 16
         "k_ids_insert": 16 * N,           # keys in
         "k_ids_gather": 4 * N,            # ids out
         "k_sort_scatter": 12 * N / sort_passes(D),  # ids in, prev / next out, spread over the passes
