@@ -83,6 +83,25 @@ def dist_env():
     return ws, rank, local
 
 
+def max_over_ranks(x, world, device=None):
+    """The largest x over the ranks of the default process group: the slowest
+    replica's time.  x itself on one rank (no process group)."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_step, steps, world, total_ms):
+    """Units per second of the whole job: every replica processes the same
+    units each step (weak scaling), and the job lasts as long as its slowest
+    replica (total_ms, already the max over ranks)."""
+    return world * units_per_step * steps / (total_ms * 1e-3)
+
+
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -231,13 +250,8 @@ def run_ours(args, ws_world, rank, local):
             import torch.distributed as dist
             dist.barrier()
 
-    def max_over_ranks(x):
-        if ws_world == 1:
-            return x
-        import torch.distributed as dist
-        t = torch.tensor([x], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+    def slowest(x):
+        return max_over_ranks(x, ws_world, dev)
 
     L = ptc.lib()
     # the trace, generated into pinned host memory (the end-to-end leg copies from it)
@@ -301,7 +315,7 @@ def run_ours(args, ws_world, rank, local):
     launches = L.ptc_launch_count() - launches0
     barrier()
     clk = clocks.stop()
-    total_ms = max_over_ranks(sum(step_ms))
+    total_ms = slowest(sum(step_ms))
     ms_per_step = total_ms / args.steps
 
     # ---- per-kernel durations: the same K steps again with CUDA events
@@ -322,7 +336,7 @@ def run_ours(args, ws_world, rank, local):
         ts.copy_(ts_host, non_blocking=True)
         return step()
 
-    e2e_total = max_over_ranks(sum(timed(args.steps, e2e_body)))
+    e2e_total = slowest(sum(timed(args.steps, e2e_body)))
     h2d = 4 * T + 8 * (tr.n_req + 1) + 8 * tr.n_req
     d2h = 8 * G + 16 * G + 16 + 8 + 8  # hits, saved (u128), total cost, N, D
 
@@ -342,7 +356,7 @@ def run_ours(args, ws_world, rank, local):
     splan.run()
     L.ptc_timer_enable(0)
     st_kernels = {name: round(tot, 4) for name, _, tot in read_timer(ptc)}
-    st_ms = max_over_ranks(sum(timed(args.steps, splan.run))) / args.steps
+    st_ms = slowest(sum(timed(args.steps, splan.run))) / args.steps
 
     # ---- semantics variants (Sec. 3.1): stack distances under leaf-first
     # touch order and whole-request residency from the step's prev, then the
@@ -362,7 +376,7 @@ def run_ours(args, ws_world, rank, local):
             assert rc == 0, rc
 
         vrun()
-        v_ms = max_over_ranks(sum(timed(args.steps, vrun))) / args.steps
+        v_ms = slowest(sum(timed(args.steps, vrun))) / args.steps
         cur = ptc.ptc_curves(vdist[:N], rbo, BLOCK, caps)
         variants[vname] = {"touch_order": "leaf-first" if order else "root-first",
                            "residency": "per request" if res else "per block", "ms": round(v_ms, 4),
@@ -392,9 +406,9 @@ def run_ours(args, ws_world, rank, local):
                 "unit": "GB/s", "frac": round(dom["achieved_gbs"] / peak, 4), "traffic": traffic,
                 "peak_source": f"{peak_kind} hbm_gbs"}
 
-    value = ws_world * T * args.steps / (total_ms * 1e-3)
-    acc_s = ws_world * N * args.steps / (total_ms * 1e-3)
-    e2e_value = ws_world * T * args.steps / (e2e_total * 1e-3)
+    value = whole_job_rate(T, args.steps, ws_world, total_ms)
+    acc_s = whole_job_rate(N, args.steps, ws_world, total_ms)
+    e2e_value = whole_job_rate(T, args.steps, ws_world, e2e_total)
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": ws_world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True, "scaling": "weak",
