@@ -3,13 +3,17 @@
 
 One step is the whole path — block hashing, dense ids, reuse indices, stack
 distances, curves — in one ptc_pipeline call over one synthetic trace
-resident in HBM: the conversational chat workload (~154M tokens, ~9.6M block
-accesses, 16-token blocks, 64 log-spaced capacities from 64 blocks to all
-distinct blocks, measured-shape cost model).  The metric is trace tokens per
-second; the JSON line also carries block accesses per second and the fraction
-of the HBM roofline for the path's stage-byte model.
+resident in HBM.  The headline workload is the largest one that fits one GPU:
+the mixed 24-hour trace (~10B tokens, ~624M block accesses, 16-token blocks,
+128 log-spaced capacities from 0.1% to 100% of the distinct blocks,
+measured-shape cost model).  The metric is trace tokens per second; the JSON
+line also carries block accesses per second, the fraction of the HBM
+roofline for the stage-byte model and for the path's own bytes, the dominant
+kernel's roofline, the end-to-end rate through the host-buffer C call, and the
+conversational chat trace (~154M tokens) as an extra key.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload 0-3] [--requests R]
 
 Timing: W untimed warm-up steps, then K steps, each bracketed by CUDA events
 on the launching stream, with a 256 MiB write between steps to flush L2
@@ -19,9 +23,11 @@ second pass of K steps with events around every launch.
 With N > 1 (torchrun) every rank runs an independent replica (the path has
 no cross-GPU exchange): value = tokens of all replicas / slowest rank's time.
 
---impl reference times the CPU oracle (the plain restatement used as the
-parity reference) on the host cores, on a bounded sample of the same
-workload; rank 0 alone runs it.
+The CPU oracle (the plain restatement used as the parity reference) runs on
+a bounded prefix of the same workload on the host cores, and the GPU path
+runs on that prefix too: their curves must be equal (cpu_baseline).
+--impl reference times that oracle alone, per step, on the prefix; rank 0
+alone runs it.
 """
 from __future__ import annotations
 
@@ -41,17 +47,17 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "trace tokens/s to all-capacity LRU hit+compute-saved curves; % of HBM roofline"
-WORKLOAD = 1
+WORKLOAD = 3   # the mixed 24-hour trace
+CHAT = 1       # the conversational chat trace, reported as an extra key
 BLOCK = 16
 NOMINAL_HBM_GBS = 7900.0
 
 # Per-launch DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) from
-# the last ncu capture of each kernel, with the sha256 of the source file it
-# was taken on; a changed source reads as "no counters" (null).
-NCU_TRAFFIC: dict[str, tuple[float, str, str]] = {
-    # 6,000-request capture (profiles/k_hash16_chat_6000req.md), scaled to the
-    # full workload by tokens
-    "k_hash16": (645.6e6, "35e274868498a45b", "ncu --set full, first 6,000 requests, x 153.81 / 55.67"),
+# the last ncu capture of each kernel, keyed by (kernel, workload), with the
+# sha256 prefix of the source file it was taken on (a changed source reads as
+# "no counters", null) and how the capture was scaled to a full launch.
+NCU_TRAFFIC: dict[tuple[str, int], tuple[float, str, str]] = {
+    ("k_hash16", 1): (645.6e6, "35e274868498a45b", "ncu --set full, first 6,000 requests, x 153.81 / 55.67"),
 }
 
 
@@ -65,10 +71,13 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-sample", type=float, default=1.0,
-                    help="fraction of the workload's requests (a prefix in time) the CPU oracle runs on")
-    ap.add_argument("--ref-sample", type=float, default=1.0,
-                    help="fraction of requests per --impl reference step")
+    ap.add_argument("--workload", type=int, choices=[0, 1, 2, 3], default=WORKLOAD,
+                    help="0 tiny, 1 chat, 2 agentic, 3 mixed 24 h (the headline)")
+    ap.add_argument("--cpu-sample", type=float, default=None,
+                    help="fraction of the workload's requests (a prefix in time) the CPU oracle runs on "
+                         "(default: all of workloads 0-1, 5%% of 2-3)")
+    ap.add_argument("--ref-sample", type=float, default=None,
+                    help="fraction of requests per --impl reference step (default as --cpu-sample)")
     ap.add_argument("--json-out", default=None)
     ap.add_argument("--requests", type=int, default=0,
                     help="run only the first N requests of the workload (small cases for profiling)")
@@ -147,6 +156,7 @@ def kernel_model_bytes(name, T, N, L, D):
         "k_hash16": 4 * T + 16 * N,       # the same, B = 16 path
         "k_hash_tile": 4 * T + 16 * N,    # the same, other multiples of 16
         "k_ids_insert": 16 * N,           # keys in
+        "k_ids_insert_prior": 16 * N,     # keys in (the same stage, prior-request hint)
         "k_ids_gather": 4 * N,            # ids out
         "k_sort_scatter": 12 * N / sort_passes(D),  # ids in, prev / next out, spread over the passes
         "k_ir_count": 4 * N,              # ids in (sort over id-runs)
@@ -165,7 +175,8 @@ KERNEL_SOURCE = {
     "k_part_count": "ptc_ids.cu", "k_part_scan": "ptc_ids.cu", "k_part_scatter": "ptc_ids.cu",
     "k_ids_insert_part": "ptc_ids.cu", "k_ids_gather_part": "ptc_ids.cu",
     "k_hash_chain": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu", "k_ids_mark": "ptc_ids.cu",
-    "k_ids_gather": "ptc_ids.cu", "k_sort_count": "ptc_sort.cu", "k_sort_rowscan": "ptc_sort.cu",
+    "k_ids_gather": "ptc_ids.cu", "k_ids_insert_prior": "ptc_ids.cu", "k_ids_follow": "ptc_ids.cu",
+    "k_tile_req": "ptc_ids.cu", "k_session_prior": "ptc_ids.cu", "k_sort_count": "ptc_sort.cu", "k_sort_rowscan": "ptc_sort.cu",
     "k_sort_scatter": "ptc_sort.cu", "k_sort_links": "ptc_sort.cu", "k_ir_count": "ptc_reuse.cu",
     "k_ir_mark": "ptc_reuse.cu", "k_bm_count": "ptc_reuse.cu", "k_bm_words": "ptc_reuse.cu",
     "k_ir_inc1": "ptc_reuse.cu", "k_ir_inc2": "ptc_reuse.cu", "k_ir_fill": "ptc_reuse.cu", "k_wm_count0": "ptc_wavelet.cu",
@@ -234,6 +245,133 @@ class Clocks:
 
 
 # ---------------------------------------------------------------- our arm
+WORKLOAD_NAMES = {
+    0: "tiny conversational trace (workload 0, seed 0): 444 sessions, 16-point capacity grid",
+    1: "conversational chat trace (workload 1, seed 1): 5,600 sessions, 60% single-turn, LN(300)/LN(600) turns, "
+       "50 Zipf system prompts, B=16, 64-point capacity grid, measured-shape cost",
+    2: "agentic coding trace (workload 2, seed 2): 560 sessions, Zipf(1.2) turns <= 400, 131,072-token cap, B=16, "
+       "64-point capacity grid, measured-shape cost",
+    3: "mixed 24 h trace (workload 3, seed 3): 50/50 token mix of the chat and agentic generators, diurnal arrivals "
+       "(3x peak/trough), ~10B tokens, ~624M block accesses, fully resident, B=16, 128-point capacity grid from "
+       "0.1% to 100% of distinct blocks, measured-shape cost",
+}
+GOLDEN = os.path.join(ROOT, "tests", "golden", "big_configs.json")
+
+
+def load_trace(workload, requests, dev):
+    """The workload generated into page-locked host memory (the end-to-end leg
+    copies from it) and copied once to the device."""
+    import numpy as np
+    import torch
+    import tracegen
+    if requests:
+        tr = tracegen.make(workload, max_requests=requests)
+        tok_host = torch.from_numpy(tr.tokens.view(np.int32)).pin_memory()
+    else:
+        _, T, _ = tracegen.sizes(workload)
+        tok_host = torch.empty(T, dtype=torch.int32, pin_memory=True)
+        tr = tracegen.make(workload, token_buffer=tok_host.numpy().view(np.uint32))
+    off_host = torch.from_numpy(tr.req_tok_off.view(np.int64)).pin_memory()
+    ts_host = torch.from_numpy(tr.req_ts_us).pin_memory()
+    ses_host = torch.from_numpy(np.ascontiguousarray(tr.req_session, dtype=np.uint32).view(np.int32)).pin_memory()
+    dev_t = (tok_host.to(dev, non_blocking=True), off_host.to(dev, non_blocking=True),
+             ts_host.to(dev, non_blocking=True), ses_host.to(dev, non_blocking=True))
+    torch.cuda.synchronize(dev)
+    return tr, (tok_host, off_host, ts_host, ses_host), dev_t
+
+
+def grid_for(ptc, tracegen, workload, dev_t, n_req, T):
+    """D is a property of the trace, taken once before timing; the grid spans
+    the workload's range over it."""
+    import torch
+    tok, off, ts, _ = dev_t
+    ws = torch.empty(ptc.workspace_bytes(n_req, T, BLOCK, n_cap=1), dtype=torch.uint8, device=tok.device)
+    D = ptc.pipeline(tok, off, ts, BLOCK, lambda d: [1], ws=ws, keep=False)["n_distinct"]
+    del ws
+    return D, tracegen.workload_grid(workload, D)
+
+
+class Timer:
+    """CUDA events on the launch stream around each step, an L2 flush (a
+    256 MiB write) between steps outside the events, and a check that every
+    step returns the warm-up's curves."""
+
+    def __init__(self, dev, stream):
+        import torch
+        self.flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+        self.stream = stream
+
+    def run(self, k_steps, body, plan=None, ref=None):
+        import numpy as np
+        import torch
+        ms = []
+        for k in range(k_steps):
+            self.flush.fill_(k & 0xFF)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(self.stream)
+            body()
+            e1.record(self.stream)
+            e1.synchronize()
+            ms.append(e0.elapsed_time(e1))
+            if plan is not None:
+                assert np.array_equal(plan.hits, ref[0]) and np.array_equal(plan.saved, ref[1])
+        return ms
+
+
+def kernel_table(ktimes, steps, T, N, D, Lbits):
+    kernels = []
+    for name, launches_k, tot_ms in ktimes:
+        per = tot_ms / max(launches_k, 1)
+        mb = kernel_model_bytes(name, T, N, Lbits, D)
+        kernels.append({"name": name, "launches_per_step": launches_k / steps, "ms_per_step": tot_ms / steps,
+                        "avg_launch_ms": per, "model_bytes_per_launch": mb,
+                        "achieved_gbs": (mb / (per * 1e-3) / 1e9) if per > 0 else 0.0})
+    kernels.sort(key=lambda x: -x["ms_per_step"])
+    return kernels
+
+
+def roofline_of(kernels, peak, peak_kind, workload):
+    """The dominant kernel's algorithmic bytes over its average launch time."""
+    if not kernels:
+        return None
+    dom = kernels[0]
+    tr_entry = NCU_TRAFFIC.get((dom["name"], workload))
+    traffic = tr_entry[0] if tr_entry and tr_entry[1] == source_sha(dom["name"]) else None
+    return {"kernel": dom["name"], "bound": "hbm", "achieved": round(dom["achieved_gbs"], 1), "peak": peak,
+            "unit": "GB/s", "frac": round(dom["achieved_gbs"] / peak, 4), "traffic": traffic,
+            "traffic_source": tr_entry[2] if traffic is not None else None,
+            "peak_source": f"{peak_kind} hbm_gbs"}
+
+
+def hbm_fractions(T, N, ms, peak):
+    stages, Lbits = stage_model_bytes(T, N)
+    model_total = sum(stages.values())
+    own = 4 * T + 60 * N
+    sec = ms * 1e-3
+    return {"stage_model_bytes": model_total, "L": Lbits,
+            "frac_of_measured": round(model_total / sec / 1e9 / peak, 4),
+            "frac_of_nominal_7900": round(model_total / sec / 1e9 / NOMINAL_HBM_GBS, 4),
+            "path_bytes_4T_60N": own, "path_frac_of_measured": round(own / sec / 1e9 / peak, 4),
+            "stages_bytes": stages}, Lbits
+
+
+def golden_parity(workload, N, D, hits, saved, caps):
+    """The full-size headline curves against the oracle's stored results
+    (tests/golden/big_configs.json, written by a script that runs the oracle
+    alone), where an entry for this workload exists."""
+    key = {3: "mixed_B16", 2: "agentic_B16"}.get(workload)
+    if key is None or not os.path.exists(GOLDEN):
+        return None
+    with open(GOLDEN) as f:
+        g = json.load(f).get(key)
+    if g is None:
+        return None
+    same = (g["N"] == N and g["D"] == D and g["caps"] == [int(c) for c in caps]
+            and g["hits"] == [int(h) for h in hits] and g["saved"] == [str(int(s)) for s in saved])
+    return {"golden": f"tests/golden/big_configs.json[{key}]", "equal": bool(same)}
+
+
 def run_ours(args, ws_world, rank, local):
     import numpy as np
     import torch
@@ -256,55 +394,25 @@ def run_ours(args, ws_world, rank, local):
         return max_over_ranks(x, ws_world, dev)
 
     L = ptc.lib()
-    # the trace, generated into pinned host memory (the end-to-end leg copies from it)
-    if args.requests:
-        tr = tracegen.make(WORKLOAD, max_requests=args.requests)
-        T = tr.n_tok
-        tok_host = torch.from_numpy(tr.tokens.view(np.int32)).pin_memory()
-    else:
-        R, T, _ = tracegen.sizes(WORKLOAD)
-        tok_host = torch.empty(T, dtype=torch.int32, pin_memory=True)
-        tr = tracegen.make(WORKLOAD, token_buffer=tok_host.numpy().view(np.uint32))
-    off_host = torch.from_numpy(tr.req_tok_off.view(np.int64)).pin_memory()
-    ts_host = torch.from_numpy(tr.req_ts_us).pin_memory()
-    tok = tok_host.to(dev, non_blocking=True)
-    off = off_host.to(dev, non_blocking=True)
-    ts = ts_host.to(dev, non_blocking=True)
-    torch.cuda.synchronize(dev)
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
-    # the capacity grid spans 64 blocks .. D; D is a property of the trace, taken once before timing
-    ws_probe = torch.empty(ptc.workspace_bytes(tr.n_req, T, BLOCK, n_cap=64), dtype=torch.uint8, device=dev)
-    D = ptc.pipeline(tok, off, ts, BLOCK, lambda d: [1], ws=ws_probe, keep=False)["n_distinct"]
-    del ws_probe
-    caps = tracegen.workload_grid(WORKLOAD, D)
-    G = len(caps)
-    ws = torch.empty(L.ptc_pipeline_workspace_bytes(tr.n_req, T, BLOCK, G), dtype=torch.uint8, device=dev)
-
-    # the call a serving loop makes: arguments marshalled once, one C call per step
-    plan = ptc.PipelinePlan(tok, off, ts, BLOCK, caps, kind=ptc.PTC_COST_MEASURED, seed=0, ws=ws)
-
-    def step():
-        return plan.run()
-
-    for _ in range(max(args.warmup, 0)):
-        step()
-    N = plan.n.value
-    ref_hits, ref_saved = plan.hits.copy(), plan.saved.copy()
+    W = args.workload
     stream = torch.cuda.current_stream(dev)
+    timer = Timer(dev, stream)
+    peak, peak_kind = measured_peaks()
 
-    def timed(k_steps, body):
-        ms = []
-        for k in range(k_steps):
-            flush.fill_(k & 0xFF)
-            e0 = torch.cuda.Event(enable_timing=True)
-            e1 = torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            body()
-            e1.record(stream)
-            e1.synchronize()
-            ms.append(e0.elapsed_time(e1))
-            assert np.array_equal(plan.hits, ref_hits) and np.array_equal(plan.saved, ref_saved)
-        return ms
+    # ================================================= the headline workload
+    tr, host_t, dev_t = load_trace(W, args.requests, dev)
+    T, R = tr.n_tok, tr.n_req
+    D, caps = grid_for(ptc, tracegen, W, dev_t, R, T)
+    G = len(caps)
+    tok, off, ts, ses = dev_t
+    ws = torch.empty(L.ptc_pipeline_workspace_bytes(R, T, BLOCK, G), dtype=torch.uint8, device=dev)
+    # the call a serving loop makes: arguments marshalled once, one C call per step
+    plan = ptc.PipelinePlan(tok, off, ts, BLOCK, caps, kind=ptc.PTC_COST_MEASURED, seed=0, ws=ws,
+                            req_session=ses, n_session=tr.n_sessions)
+    for _ in range(max(args.warmup, 0)):
+        plan.run()
+    N = plan.n.value
+    ref = (plan.hits.copy(), plan.saved.copy())
 
     # ---- timed region (inputs resident in HBM)
     clocks = Clocks(local)
@@ -312,7 +420,7 @@ def run_ours(args, ws_world, rank, local):
     torch.cuda.synchronize(dev)
     clocks.start()
     launches0 = L.ptc_launch_count()
-    step_ms = timed(args.steps, step)
+    step_ms = timer.run(args.steps, plan.run, plan, ref)
     torch.cuda.synchronize(dev)
     launches = L.ptc_launch_count() - launches0
     barrier()
@@ -325,88 +433,28 @@ def run_ours(args, ws_world, rank, local):
     # this pass is separate from the timed one)
     L.ptc_timer_reset()
     L.ptc_timer_enable(1)
-    inst_ms = timed(args.steps, step)
+    inst_ms = timer.run(args.steps, plan.run, plan, ref)
     L.ptc_timer_enable(0)
     ktimes = read_timer(ptc)
+    hbm, Lbits = hbm_fractions(T, N, ms_per_step, peak)
+    kernels = kernel_table(ktimes, args.steps, T, N, D, Lbits)
+    roof = roofline_of(kernels, peak, peak_kind, W)
+    gold = golden_parity(W, N, D, plan.hits, plan.result()["saved"], caps) if not args.requests else None
+    del plan, ws, tok, off, ts, ses, dev_t
+    torch.cuda.empty_cache()
 
-    # ---- end to end through the public API: each step copies its trace from
-    # pinned host memory into the plan's device buffers, then runs the plan
-    # (the curves come back to host memory inside the call)
-    def e2e_body():
-        tok.copy_(tok_host, non_blocking=True)
-        off.copy_(off_host, non_blocking=True)
-        ts.copy_(ts_host, non_blocking=True)
-        return step()
-
-    e2e_total = slowest(sum(timed(args.steps, e2e_body)))
-    h2d = 4 * T + 8 * (tr.n_req + 1) + 8 * tr.n_req
+    # ---- end to end through the C ABI with HOST buffers: each step copies
+    # the trace from page-locked host memory to the device inside the call,
+    # runs the path and returns the curves to host memory
+    hplan = ptc.HostPipelinePlan(*host_t[:3], BLOCK, caps, kind=ptc.PTC_COST_MEASURED, seed=0, device=dev,
+                                 req_session=host_t[3], n_session=tr.n_sessions)
+    hplan.run()
+    assert np.array_equal(hplan.hits, ref[0]) and np.array_equal(hplan.saved, ref[1])
+    e2e_total = slowest(sum(timer.run(args.steps, hplan.run, hplan, ref)))
+    h2d = 4 * T + 8 * (R + 1) + 8 * R + 4 * R
     d2h = 8 * G + 16 * G + 16 + 8 + 8  # hits, saved (u128), total cost, N, D
-
-    # ---- trace statistics (Sec. 4.1-4.3, App. B) over the pipeline's own
-    # per-access arrays: one pipeline run that keeps them, then K timed calls
-    outs = {k: torch.empty(max(N, 1), dtype=torch.int32, device=dev) for k in ("ids", "prev", "next", "dist")}
-    outs["req_blk_off"] = torch.empty(tr.n_req + 1, dtype=torch.int64, device=dev)
-    ptc.PipelinePlan(tok, off, ts, BLOCK, caps, ws=ws, outputs=outs).run()
-    ses = torch.from_numpy(tr.req_session.astype(np.uint32).view(np.int32)).to(dev)
-    splan = ptc.TraceStatsPlan(outs["ids"][:N], outs["prev"][:N], outs["next"][:N], D, outs["req_blk_off"], ts, ses,
-                               tr.n_sessions, dist=outs["dist"][:N], caps=caps)
-    stats = splan.run().result()
-    assert stats["n_reuse"] == N - D and int(stats["blocks"].sum()) == D and int(stats["accesses"].sum()) == N
-    assert int(stats["reuse_us"].sum()) == N - D and int(stats["reach"][-1]) <= N - D
-    L.ptc_timer_reset()
-    L.ptc_timer_enable(1)
-    splan.run()
-    L.ptc_timer_enable(0)
-    st_kernels = {name: round(tot, 4) for name, _, tot in read_timer(ptc)}
-    st_ms = slowest(sum(timed(args.steps, splan.run))) / args.steps
-
-    # ---- semantics variants (Sec. 3.1): stack distances under leaf-first
-    # touch order and whole-request residency from the step's prev, then the
-    # curves on them
-    variants, vdists = {}, {}
-    prev_t, rbo = outs["prev"][:N], outs["req_blk_off"]
-    mid = [0, G // 2, G - 1]
-    for vname, order, res in VARIANTS:
-        vws = torch.empty(L.ptc_stack_distance_variant_workspace_bytes(N, tr.n_req, order, res), dtype=torch.uint8,
-                          device=dev)
-        vdist = torch.empty(max(N, 1), dtype=torch.int32, device=dev)
-        vargs = (prev_t.data_ptr(), N, rbo.data_ptr(), tr.n_req, order, res, vdist.data_ptr(), vws.data_ptr(),
-                 vws.numel(), stream.cuda_stream)
-
-        def vrun(vargs=vargs):
-            rc = L.ptc_stack_distance_variant(*vargs)
-            assert rc == 0, rc
-
-        vrun()
-        v_ms = slowest(sum(timed(args.steps, vrun))) / args.steps
-        cur = ptc.ptc_curves(vdist[:N], rbo, BLOCK, caps)
-        variants[vname] = {"touch_order": "leaf-first" if order else "root-first",
-                           "residency": "per request" if res else "per block", "ms": round(v_ms, 4),
-                           "achieved_gbs_8n": round(8 * N / (v_ms * 1e-3) / 1e9, 1),
-                           "hit_ratio_at": {str(int(caps[g])): round(cur["hits"][g] / N, 5) for g in mid}}
-        vdists[vname] = (order, res, vdist[:N])
-        del vws
-
-    # ---- roofline
-    peak, peak_kind = measured_peaks()
-    stages, Lbits = stage_model_bytes(T, N)
-    model_total = sum(stages.values())
-    kernels = []
-    for name, launches_k, tot_ms in ktimes:
-        per = tot_ms / max(launches_k, 1)
-        mb = kernel_model_bytes(name, T, N, Lbits, D)
-        kernels.append({"name": name, "launches_per_step": launches_k / args.steps, "ms_per_step": tot_ms / args.steps,
-                        "avg_launch_ms": per, "model_bytes_per_launch": mb,
-                        "achieved_gbs": (mb / (per * 1e-3) / 1e9) if per > 0 else 0.0})
-    kernels.sort(key=lambda x: -x["ms_per_step"])
-    dom = kernels[0] if kernels else None
-    roof = None
-    if dom:
-        tr_entry = NCU_TRAFFIC.get(dom["name"])
-        traffic = tr_entry[0] if tr_entry and tr_entry[1] == source_sha(dom["name"]) else None
-        roof = {"kernel": dom["name"], "bound": "hbm", "achieved": round(dom["achieved_gbs"], 1), "peak": peak,
-                "unit": "GB/s", "frac": round(dom["achieved_gbs"] / peak, 4), "traffic": traffic,
-                "peak_source": f"{peak_kind} hbm_gbs"}
+    del hplan
+    torch.cuda.empty_cache()
 
     value = whole_job_rate(T, args.steps, ws_world, total_ms)
     acc_s = whole_job_rate(N, args.steps, ws_world, total_ms)
@@ -415,62 +463,40 @@ def run_ours(args, ws_world, rank, local):
         "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": ws_world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "u32/u64 integer", "data": "synthetic",
-        "config": {"workload": "conversational chat trace (workload 1, seed 1): 5,600 sessions, 60% single-turn, "
-                               "LN(300)/LN(600) turns, 50 Zipf system prompts, B=16, 64-point capacity grid, "
-                               "measured-shape cost",
-                   "tokens": T, "requests": tr.n_req, "accesses": N, "distinct_blocks": D, "block_size": BLOCK,
-                   "capacities": G, "l2": "flushed between timed steps (256 MiB write, outside the events)",
+        "config": {"workload": WORKLOAD_NAMES[W], "tokens": T, "requests": R, "accesses": N, "distinct_blocks": D,
+                   "block_size": BLOCK, "capacities": G,
+                   "l2": "inputs larger than L2; also flushed between timed steps (256 MiB write, outside the events)",
                    "parallelism": "replicas" if ws_world > 1 else "single GPU",
                    "prefix_requests": args.requests or None},
         "accesses_per_s": round(acc_s, 1),
-        "hbm_roofline": {"stage_model_bytes": model_total, "L": Lbits,
-                         "frac_of_measured": round(model_total / (ms_per_step * 1e-3) / 1e9 / peak, 4),
-                         "frac_of_nominal_7900": round(model_total / (ms_per_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS, 4),
-                         "stages_bytes": stages},
+        "hbm_roofline": hbm,
         "roofline": roof,
         "kernels": [{k: (round(v, 5) if isinstance(v, float) else v) for k, v in x.items()} for x in kernels],
         "kernel_timing": {"how": "separate pass of the same K steps with CUDA events around every launch",
                           "ms_per_step": round(sum(inst_ms) / len(inst_ms), 4)},
         "e2e": {"value": round(e2e_value, 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_total / args.steps, 4)},
+                "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_total / args.steps, 4),
+                "call": "ptc_pipeline_host: trace in page-locked host memory, copied inside the call; curves "
+                        "returned to host memory"},
         "gpu_launches": launches,
         "clocks": clk,
-        "trace_stats": {
-            "call": "ptc_trace_stats on the step's ids, prev, next and stack distances, 64-point reach grid",
-            "ms": round(st_ms, 4), "accesses_per_s": round(ws_world * N / (st_ms * 1e-3), 1),
-            "roofline": {"bound": "hbm", "bytes_model": "16 N: ids, prev, next, dist read once",
-                         "achieved": round(16 * N / (st_ms * 1e-3) / 1e9, 1), "peak": peak, "unit": "GB/s",
-                         "frac": round(16 * N / (st_ms * 1e-3) / 1e9 / peak, 4), "traffic": None},
-            "kernels_ms": st_kernels,
-            "categories": {"blocks": stats["blocks"].tolist(), "accesses": stats["accesses"].tolist(),
-                           "one_hit_blocks": [int(stats["freq"][c, 1]) for c in range(3)]},
-        },
-        "variants": {"call": "ptc_stack_distance_variant on the step's prev (distances in depth order for ptc_curves)",
-                     "bytes_model": "8 N: prev read, dist written", "hot_path_hit_ratio_at":
-                         {str(int(caps[g])): round(int(plan.hits[g]) / N, 5) for g in mid}, **variants},
+        "parity_with_oracle_golden": gold,
     }
+
+    # ---- the oracle on a bounded prefix of the same workload, and the GPU
+    # on that same prefix: the curves must be equal
     if rank == 0 and ws_world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"], orc = cpu_baseline(tr, args.cpu_sample, stats=True)
-        ost, odt = oracle_trace_stats(tr, orc)
-        same = None
-        if orc["n_req"] == tr.n_req:  # the sample is the whole trace: the oracle's statistics must match
-            same = all(np.array_equal(np.asarray(ost[k]), np.asarray(stats[k])) for k in ost)
-            assert same, "trace statistics differ from the oracle"
-        if orc["n_req"] == tr.n_req:  # the oracle's distances under every variant must match
-            import oracle
-            for vname, (order, res, vd) in vdists.items():
-                t0 = time.perf_counter()
-                want = oracle.sd_variant(orc["ids"], orc["D"], orc["off"], order, res)
-                dt = time.perf_counter() - t0
-                same_v = bool(np.array_equal(ptc.u32(vd), want))
-                assert same_v, f"variant {vname} differs from the oracle"
-                line["variants"][vname]["cpu_baseline"] = {
-                    "value": round(N / dt, 1), "unit": "accesses/s", "cores": 1, "kind": "oracle",
-                    "sample": f"orc_sd_variant (Fenwick) on the whole trace; {dt:.2f} s", "parity_with_gpu": same_v}
-        line["trace_stats"]["cpu_baseline"] = {
-            "value": round(orc["n"] / odt, 1), "unit": "accesses/s", "cores": 1, "kind": "oracle",
-            "sample": f"orc_trace_stats on the oracle's own ids and distances of the first {orc['n_req']} requests "
-                      f"({orc['n']} accesses); {odt:.2f} s", "parity_with_gpu": same}
+        frac = args.cpu_sample if args.cpu_sample is not None else (1.0 if W in (0, 1) else 0.05)
+        cb, orc = cpu_baseline(tr, frac, W)
+        cb["parity_with_gpu"] = gpu_matches_oracle(ptc, orc, dev)
+        assert cb["parity_with_gpu"], "the GPU's curves differ from the oracle's on the sample"
+        line["cpu_baseline"] = cb
+    del tr, host_t
+    torch.cuda.empty_cache()
+
+    # ================================================= the chat trace (an extra key)
+    if W != CHAT and not args.requests:
+        line["chat"] = chat_extras(args, ptc, tracegen, dev, timer, slowest, peak, peak_kind, rank, ws_world)
     if rank == 0:
         s = json.dumps(line)
         print(s, flush=True)
@@ -480,6 +506,139 @@ def run_ours(args, ws_world, rank, local):
     if ws_world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def gpu_matches_oracle(ptc, orc, dev):
+    """Run the GPU path on the oracle's sample trace and compare N, D, the
+    curves and the total cost with the oracle's."""
+    import numpy as np
+    import torch
+    sub = orc["sub"]
+    tok = torch.from_numpy(sub.tokens.view(np.int32)).to(dev)
+    off = torch.from_numpy(sub.req_tok_off.view(np.int64)).to(dev)
+    ts = torch.from_numpy(sub.req_ts_us).to(dev)
+    ses = torch.from_numpy(np.ascontiguousarray(sub.req_session, dtype=np.uint32).view(np.int32)).to(dev)
+    g = ptc.ptc_pipeline(tok, off, ts, BLOCK, orc["caps"], kind=ptc.PTC_COST_MEASURED, req_session=ses,
+                         n_session=sub.n_sessions)
+    return bool(g["n_access"] == orc["n"] and g["n_distinct"] == orc["D"] and g["hits"] == orc["hits"]
+                and g["saved"] == orc["saved"] and g["total_cost"] == orc["total"])
+
+
+def chat_extras(args, ptc, tracegen, dev, timer, slowest, peak, peak_kind, rank, ws_world):
+    """The conversational chat trace (~154M tokens) through the same path,
+    its oracle parity on the whole trace, and the trace statistics and
+    semantics variants over its per-access arrays."""
+    import numpy as np
+    import torch
+    L = ptc.lib()
+    tr, host_t, dev_t = load_trace(CHAT, 0, dev)
+    T, R = tr.n_tok, tr.n_req
+    D, caps = grid_for(ptc, tracegen, CHAT, dev_t, R, T)
+    G = len(caps)
+    tok, off, ts, ses_d = dev_t
+    ws = torch.empty(L.ptc_pipeline_workspace_bytes(R, T, BLOCK, G), dtype=torch.uint8, device=dev)
+    plan = ptc.PipelinePlan(tok, off, ts, BLOCK, caps, kind=ptc.PTC_COST_MEASURED, seed=0, ws=ws,
+                            req_session=ses_d, n_session=tr.n_sessions)
+    for _ in range(max(args.warmup, 0)):
+        plan.run()
+    N = plan.n.value
+    ref = (plan.hits.copy(), plan.saved.copy())
+    ms = slowest(sum(timer.run(args.steps, plan.run, plan, ref))) / args.steps
+    L.ptc_timer_reset()
+    L.ptc_timer_enable(1)
+    timer.run(args.steps, plan.run, plan, ref)
+    L.ptc_timer_enable(0)
+    hbm, Lbits = hbm_fractions(T, N, ms, peak)
+    kernels = kernel_table(read_timer(ptc), args.steps, T, N, D, Lbits)
+    out = {"workload": WORKLOAD_NAMES[CHAT], "tokens": T, "requests": R, "accesses": N, "distinct_blocks": D,
+           "capacities": G, "ms_per_step": round(ms, 4), "tokens_per_s": round(ws_world * T / (ms * 1e-3), 1),
+           "accesses_per_s": round(ws_world * N / (ms * 1e-3), 1), "hbm_roofline": hbm,
+           "roofline": roofline_of(kernels, peak, peak_kind, CHAT),
+           "kernels_top": [{"name": k["name"], "ms_per_step": round(k["ms_per_step"], 4)} for k in kernels[:8]]}
+    # ---- trace statistics (Sec. 4.1-4.3, App. B) over the path's own
+    # per-access arrays: one pipeline run that keeps them, then K timed calls
+    outs = {k: torch.empty(max(N, 1), dtype=torch.int32, device=dev) for k in ("ids", "prev", "next", "dist")}
+    outs["req_blk_off"] = torch.empty(R + 1, dtype=torch.int64, device=dev)
+    ptc.PipelinePlan(tok, off, ts, BLOCK, caps, ws=ws, outputs=outs, req_session=ses_d,
+                     n_session=tr.n_sessions).run()
+    ses = torch.from_numpy(tr.req_session.astype(np.uint32).view(np.int32)).to(dev)
+    splan = ptc.TraceStatsPlan(outs["ids"][:N], outs["prev"][:N], outs["next"][:N], D, outs["req_blk_off"], ts, ses,
+                               tr.n_sessions, dist=outs["dist"][:N], caps=caps)
+    stats = splan.run().result()
+    assert stats["n_reuse"] == N - D and int(stats["blocks"].sum()) == D and int(stats["accesses"].sum()) == N
+    L.ptc_timer_reset()
+    L.ptc_timer_enable(1)
+    splan.run()
+    L.ptc_timer_enable(0)
+    st_kernels = {name: round(tot, 4) for name, _, tot in read_timer(ptc)}
+    st_ms = slowest(sum(timer.run(args.steps, splan.run))) / args.steps
+    out["trace_stats"] = {
+        "call": "ptc_trace_stats on the step's ids, prev, next and stack distances, 64-point reach grid",
+        "ms": round(st_ms, 4), "accesses_per_s": round(ws_world * N / (st_ms * 1e-3), 1),
+        "roofline": {"bound": "hbm", "bytes_model": "16 N: ids, prev, next, dist read once",
+                     "achieved": round(16 * N / (st_ms * 1e-3) / 1e9, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(16 * N / (st_ms * 1e-3) / 1e9 / peak, 4), "traffic": None},
+        "kernels_ms": st_kernels,
+        "categories": {"blocks": stats["blocks"].tolist(), "accesses": stats["accesses"].tolist(),
+                       "one_hit_blocks": [int(stats["freq"][c, 1]) for c in range(3)]},
+    }
+    # ---- semantics variants (Sec. 3.1): stack distances under leaf-first
+    # touch order and whole-request residency from the step's prev, then the
+    # curves on them
+    variants, vdists = {}, {}
+    prev_t, rbo = outs["prev"][:N], outs["req_blk_off"]
+    mid = [0, G // 2, G - 1]
+    for vname, order, res in VARIANTS:
+        vws = torch.empty(L.ptc_stack_distance_variant_workspace_bytes(N, R, order, res), dtype=torch.uint8,
+                          device=dev)
+        vdist = torch.empty(max(N, 1), dtype=torch.int32, device=dev)
+        vargs = (prev_t.data_ptr(), N, rbo.data_ptr(), R, order, res, vdist.data_ptr(), vws.data_ptr(),
+                 vws.numel(), timer.stream.cuda_stream)
+
+        def vrun(vargs=vargs):
+            rc = L.ptc_stack_distance_variant(*vargs)
+            assert rc == 0, rc
+
+        vrun()
+        v_ms = slowest(sum(timer.run(args.steps, vrun))) / args.steps
+        cur = ptc.ptc_curves(vdist[:N], rbo, BLOCK, caps)
+        variants[vname] = {"touch_order": "leaf-first" if order else "root-first",
+                           "residency": "per request" if res else "per block", "ms": round(v_ms, 4),
+                           "achieved_gbs_8n": round(8 * N / (v_ms * 1e-3) / 1e9, 1),
+                           "hit_ratio_at": {str(int(caps[g])): round(cur["hits"][g] / N, 5) for g in mid}}
+        vdists[vname] = (order, res, vdist[:N])
+        del vws
+    out["variants"] = {"call": "ptc_stack_distance_variant on the step's prev (distances in depth order for "
+                               "ptc_curves)", "bytes_model": "8 N: prev read, dist written",
+                       "hot_path_hit_ratio_at": {str(int(caps[g])): round(int(plan.hits[g]) / N, 5) for g in mid},
+                       **variants}
+    if rank == 0 and ws_world == 1 and not args.no_cpu_baseline:
+        # the oracle on the whole chat trace: curves, statistics and variant distances must match
+        cb, orc = cpu_baseline(tr, 1.0, CHAT, keep_sd=True)
+        g_res = plan.result()
+        same = (orc["n"] == N and orc["D"] == D and orc["hits"] == g_res["hits"] and orc["saved"] == g_res["saved"]
+                and orc["total"] == g_res["total_cost"])
+        assert same, "the chat trace's curves differ from the oracle's"
+        cb["parity_with_gpu"] = same
+        out["cpu_baseline"] = cb
+        ost, odt = oracle_trace_stats(tr, orc)
+        same_st = all(np.array_equal(np.asarray(ost[k]), np.asarray(stats[k])) for k in ost)
+        assert same_st, "trace statistics differ from the oracle"
+        out["trace_stats"]["cpu_baseline"] = {
+            "value": round(orc["n"] / odt, 1), "unit": "accesses/s", "cores": 1, "kind": "oracle",
+            "sample": f"orc_trace_stats on the oracle's own ids and distances of the whole trace "
+                      f"({orc['n']} accesses); {odt:.2f} s", "parity_with_gpu": same_st}
+        import oracle
+        for vname, (order, res, vd) in vdists.items():
+            t0 = time.perf_counter()
+            want = oracle.sd_variant(orc["ids"], orc["D"], orc["off"], order, res)
+            dt = time.perf_counter() - t0
+            same_v = bool(np.array_equal(ptc.u32(vd), want))
+            assert same_v, f"variant {vname} differs from the oracle"
+            out["variants"][vname]["cpu_baseline"] = {
+                "value": round(N / dt, 1), "unit": "accesses/s", "cores": 1, "kind": "oracle",
+                "sample": f"orc_sd_variant (Fenwick) on the whole trace; {dt:.2f} s", "parity_with_gpu": same_v}
+    return out
 
 
 def read_timer(ptc):
@@ -498,7 +657,10 @@ def read_timer(ptc):
 
 
 # ---------------------------------------------------------------- CPU oracle
-def oracle_on_sample(tr, fraction, threads, keep=False):
+def oracle_on_sample(tr, fraction, threads, workload, keep=False):
+    """The oracle as it stands on the first `fraction` of the requests:
+    exact trie ids, prev / next, Fenwick stack distances, direct LRU
+    simulation at every capacity of the workload's grid over the sample's D."""
     import oracle
     import tracegen
     n_req = max(1, int(tr.n_req * fraction))
@@ -508,29 +670,31 @@ def oracle_on_sample(tr, fraction, threads, keep=False):
     off = oracle.block_offsets(sub.req_tok_off, BLOCK)
     prev, nxt = oracle.reuse(ids, D)
     sd = oracle.sd_fenwick(prev)
-    caps = tracegen.workload_grid(WORKLOAD, D)
-    oracle.lru_curves(ids, off, BLOCK, caps, oracle.COST_MEASURED, threads=threads)
+    caps = tracegen.workload_grid(workload, D)
+    hits, saved, total = oracle.lru_curves(ids, off, BLOCK, caps, oracle.COST_MEASURED, threads=threads)
     dt = time.perf_counter() - t0
-    kept = dict(sub=sub, ids=ids, D=D, off=off, sd=sd, n=int(ids.size), n_req=n_req) if keep else None
-    return sub, dt, kept
+    res = dict(sub=sub, D=D, n=int(ids.size), n_req=n_req, caps=caps, hits=hits, saved=saved, total=total)
+    if keep:
+        res.update(ids=ids, off=off, sd=sd)
+    return sub, dt, res
 
 
-def cpu_baseline(tr, fraction, stats=False):
+def cpu_baseline(tr, fraction, workload, keep_sd=False):
     threads = os.cpu_count() or 1
-    sub, dt, kept = oracle_on_sample(tr, fraction, threads, keep=stats)
+    sub, dt, res = oracle_on_sample(tr, fraction, threads, workload, keep=keep_sd)
     line = {"value": round(sub.n_tok / dt, 1), "unit": "tokens/s", "cores": threads, "kind": "oracle",
-            "sample": f"first {sub.n_req} of {tr.n_req} requests ({sub.n_tok} tokens) of the same workload; "
-                      f"exact trie ids, prev/next, Fenwick stack distances, direct LRU simulation at all 64 "
-                      f"capacities on {threads} threads; {dt:.2f} s"}
-    return (line, kept) if stats else line
+            "sample": f"first {sub.n_req} of {tr.n_req} requests ({sub.n_tok} tokens, {res['n']} accesses) of the "
+                      f"same workload; exact trie ids, prev/next, Fenwick stack distances, direct LRU simulation "
+                      f"at all {len(res['caps'])} capacities of the workload's grid over the sample's D on "
+                      f"{threads} threads; {dt:.2f} s"}
+    return line, res
 
 
 def oracle_trace_stats(tr, kept):
     """The oracle's trace statistics on its own arrays of the sample, timed."""
     import oracle
-    import tracegen
     sub = kept["sub"]
-    caps = tracegen.workload_grid(WORKLOAD, kept["D"]) if kept["n_req"] == tr.n_req else None
+    caps = kept["caps"] if kept["n_req"] == tr.n_req else None
     t0 = time.perf_counter()
     st = oracle.trace_stats(kept["ids"], kept["D"], kept["off"], sub.req_ts_us, sub.req_session, tr.n_sessions,
                             kept["sd"], caps)
@@ -541,14 +705,16 @@ def run_reference(args, ws_world, rank):
     if rank != 0:
         return
     import tracegen
-    tr = tracegen.make(WORKLOAD)
+    W = args.workload
+    frac = args.ref_sample if args.ref_sample is not None else (1.0 if W in (0, 1) else 0.05)
+    tr = tracegen.make(W, max_requests=max(1, int(tracegen.sizes(W)[0] * frac)))
     threads = os.cpu_count() or 1
     for _ in range(max(args.warmup, 0)):
-        oracle_on_sample(tr, args.ref_sample, threads)[:2]
+        oracle_on_sample(tr, 1.0, threads, W)
     times = []
     sub = None
     for _ in range(args.steps):
-        sub, dt, _ = oracle_on_sample(tr, args.ref_sample, threads)
+        sub, dt, _ = oracle_on_sample(tr, 1.0, threads, W)
         times.append(dt)
     total = sum(times)
     value = sub.n_tok * args.steps / total
@@ -557,10 +723,11 @@ def run_reference(args, ws_world, rank):
         "warmup": args.warmup, "ms_per_step": round(1e3 * total / args.steps, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u32/u64/u128 integer", "data": "synthetic",
         "impl": "reference",
-        "config": {"workload": "conversational chat trace (workload 1, seed 1), B=16, 64-point capacity grid",
-                   "sample_requests": sub.n_req, "sample_tokens": sub.n_tok},
+        "config": {"workload": WORKLOAD_NAMES[W], "sample_requests": sub.n_req, "sample_tokens": sub.n_tok},
         "cpu_baseline": {"value": round(value, 1), "unit": "tokens/s", "cores": threads, "kind": "oracle",
-                         "sample": f"first {sub.n_req} of {tr.n_req} requests per step"},
+                         "sample": f"first {sub.n_req} requests ({sub.n_tok} tokens) of the workload per step: "
+                                   f"exact trie ids, prev/next, Fenwick stack distances, direct LRU at every "
+                                   f"capacity of the grid"},
         "e2e": {"value": round(value, 1), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     s = json.dumps(line)

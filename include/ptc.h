@@ -11,6 +11,8 @@
  *     -> ptc_reuse_indices   previous / next use of each block Sec. 3.2, 5.2 (Belady's next access)
  *     -> ptc_stack_distance  LRU stack distance of each access App. B ("reuses reachable within C")
  *     -> ptc_curves          hits and compute saved per C      Sec. 3.2 (hit ratio), Sec. 5.2 (compute savings)
+ *   with Belady's offline optimum from the same reuse indices,
+ *        ptc_belady_curves                                     Sec. 3.2 (offline ceiling)
  *   with, for the semantics variants (touch order, whole-request residency),
  *        ptc_stack_distance_variant                           Sec. 3.1 (simulator)
  *   and, over the same arrays,
@@ -153,6 +155,37 @@ enum { PTC_IDS_AUTO = 0, PTC_IDS_DIRECT = 1, PTC_IDS_GROUPED = 2 };
 size_t ptc_assign_ids_ex_workspace_bytes(uint64_t n, int method);
 ptc_status ptc_assign_ids_ex(const ptc_u128* keys, uint64_t n, uint32_t* ids_out, uint64_t* n_distinct_host_out,
                              int method, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * ptc_assign_ids_prior — the ids of ptc_assign_ids, with a prior-request hint
+ * that saves table probes.  Sec. 2.3: a turn of a multi-turn session sends
+ * the whole context again, so request r usually repeats every block of an
+ * earlier request of its session and appends to it.  req_prior[r] names such
+ * an earlier request (or PTC_NONE).  An access whose key equals that of the
+ * same depth of req_prior[r] is a repeat: it is not inserted into the table
+ * and takes its id from the prior request's chain; only the other accesses
+ * are inserted.  The ids are exactly those of ptc_assign_ids for ANY hint
+ * with req_prior[r] < r or PTC_NONE (a poor hint only costs probes);
+ * req_prior[r] >= r is PTC_ERR_INVALID_ARG.
+ *   keys         ptc_u128[n] as for ptc_assign_ids
+ *   req_blk_off  u64[n_req + 1] from ptc_hash_blocks (req_blk_off[n_req] == n)
+ *   req_prior    u32[n_req]
+ */
+size_t ptc_assign_ids_prior_workspace_bytes(uint64_t n, uint32_t n_req);
+ptc_status ptc_assign_ids_prior(const ptc_u128* keys, uint64_t n, const uint64_t* req_blk_off, const uint32_t* req_prior,
+                                uint32_t n_req, uint32_t* ids_out, uint64_t* n_distinct_host_out, void* ws,
+                                size_t ws_bytes, void* stream);
+
+/*
+ * ptc_session_prior — the hint above from session labels (Sec. 2.3,
+ * sessions): prior_out[r] = the latest request before r with the same label,
+ * or PTC_NONE for a session's first request.  req_session u32[n_req], labels
+ * below n_session (PTC_ERR_INVALID_ARG otherwise); prior_out u32[n_req].
+ * A stable radix sort of the requests by label, then one pass.
+ */
+size_t ptc_session_prior_workspace_bytes(uint32_t n_req);
+ptc_status ptc_session_prior(const uint32_t* req_session, uint32_t n_req, uint32_t n_session, uint32_t* prior_out,
+                             void* ws, size_t ws_bytes, void* stream);
 
 /*
  * ptc_verify_ids — exact check of the ids (Sec. 2.2 identity, without hashing):
@@ -312,6 +345,33 @@ ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_
                       size_t ws_bytes, void* stream);
 
 /*
+ * ptc_belady_curves — Belady's offline optimum (Sec. 3.2: the offline ceiling
+ * the paper sets every eviction policy against) at every capacity of the
+ * grid: the block hit and compute-saved curves of Belady's MIN, which on a
+ * miss with a full cache evicts the resident block, other than the one just
+ * brought in, whose next access lies farthest (never again counts as
+ * farthest); every accessed block is admitted.  Block k of a request counts
+ * as a hit iff blocks 0..k of that request were all resident (the prefix rule
+ * of ptc_curves), and compute saved sums the cost model over those hits.
+ * MIN's hits are computed from the reuse intervals (prev[i], i): they are the
+ * intervals an earliest-end-first greedy with best-fit tracks keeps with at
+ * most C - 1 of them spanning any access.
+ *   prev            u32[n] from ptc_reuse_indices (prev[i] < i or PTC_NONE,
+ *                   PTC_ERR_INVALID_ARG otherwise)
+ *   req_blk_off, n_req, block_size, cm, cap_host, n_cap   as for ptc_curves
+ *   hits_host_out   u64[n_cap], saved_host_out ptc_u128[n_cap] (host)
+ *   raw_hits_host_out  u64[n_cap] (host) or NULL: resident accesses at each
+ *                   capacity without the prefix rule
+ * One warp per capacity replays the runs of consecutive re-reads in order;
+ * the time grows with the number of runs, not of accesses.
+ */
+size_t ptc_belady_curves_workspace_bytes(uint64_t n, uint32_t n_req, uint32_t n_cap);
+ptc_status ptc_belady_curves(const uint32_t* prev, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,
+                             uint32_t block_size, const ptc_cost_model* cm, const uint64_t* cap_host, uint32_t n_cap,
+                             uint64_t* hits_host_out, ptc_u128* saved_host_out, uint64_t* raw_hits_host_out, void* ws,
+                             size_t ws_bytes, void* stream);
+
+/*
  * ptc_pipeline — the five calls in order (hash, ids, reuse, stack distance,
  * curves) in one call, for a trace already on the device.  Semantics, limits
  * and errors are those of the individual calls; the first error stops the
@@ -322,18 +382,49 @@ ptc_status ptc_curves(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_
  *       floor(n_tok / block_size) entries
  *   cap_host, n_cap, cm, hits/saved/total outputs  as for ptc_curves
  *   n_access_host_out, n_distinct_host_out        N and D on the host
+ *   req_session, n_session   optional (NULL, 0): u32[n_req] session label of
+ *       each request, below n_session (PTC_ERR_INVALID_ARG otherwise).  With
+ *       them, stage a2 takes the previous request of each request's session
+ *       as its prior-request hint (ptc_session_prior, ptc_assign_ids_prior):
+ *       a turn of a session re-sends that request's context (Sec. 2.3), so
+ *       most of its blocks need no table probe.  The results do not depend
+ *       on the sessions; only the time does.
  * The workspace holds the intermediate arrays not supplied plus the largest
  * scratch of any stage (ptc_pipeline_workspace_bytes).  Stages b and c do not
  * wait for their own status; an error they raise is returned with stage d's.
  */
 size_t ptc_pipeline_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size, uint32_t n_cap);
 ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off, const int64_t* req_ts_us,
-                        uint32_t n_req, uint32_t block_size, uint64_t seed, const ptc_cost_model* cm,
+                        const uint32_t* req_session, uint32_t n_session, uint32_t n_req, uint32_t block_size, uint64_t seed, const ptc_cost_model* cm,
                         const uint64_t* cap_host, uint32_t n_cap, ptc_u128* keys_out, uint64_t* req_blk_off_out,
                         uint32_t* ids_out, uint32_t* prev_out, uint32_t* next_out, uint32_t* dist_out,
                         uint64_t* n_access_host_out, uint64_t* n_distinct_host_out, uint64_t* hits_host_out,
                         ptc_u128* saved_host_out, ptc_u128* total_cost_host_out, void* ws, size_t ws_bytes,
                         void* stream);
+
+/*
+ * ptc_pipeline_host — ptc_pipeline for a trace held in HOST memory: the call
+ * a user with a trace on the host makes.  tokens_host (u32[n_tok]),
+ * req_tok_off_host (u64[n_req + 1]), req_ts_us_host (i64[n_req], or NULL
+ * to skip the order check) and req_session_host (u32[n_req] labels below
+ * n_session, or NULL) are host pointers; they are copied on `stream`
+ * into the front of the workspace (page-locked host memory copies
+ * asynchronously at full link speed, pageable memory is staged by the
+ * driver), then the whole path runs on the copy exactly as ptc_pipeline.
+ * The curves, N and D come back in host memory as for ptc_pipeline; the
+ * per-access arrays stay in the workspace and are not returned.
+ * Workspace: ptc_pipeline_host_workspace_bytes, which is
+ * ptc_pipeline_workspace_bytes plus room for the copied trace.  The caller
+ * keeps the host buffers unchanged until the call returns.
+ */
+size_t ptc_pipeline_host_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size, uint32_t n_cap);
+ptc_status ptc_pipeline_host(const uint32_t* tokens_host, uint64_t n_tok, const uint64_t* req_tok_off_host,
+                             const int64_t* req_ts_us_host, const uint32_t* req_session_host, uint32_t n_session,
+                             uint32_t n_req, uint32_t block_size, uint64_t seed,
+                             const ptc_cost_model* cm, const uint64_t* cap_host, uint32_t n_cap,
+                             uint64_t* n_access_host_out, uint64_t* n_distinct_host_out, uint64_t* hits_host_out,
+                             ptc_u128* saved_host_out, ptc_u128* total_cost_host_out, void* ws, size_t ws_bytes,
+                             void* stream);
 
 /*
  * ptc_trace_stats — trace characterization over the arrays of the path

@@ -15,6 +15,10 @@ Functions and the passages they restate:
   move-to-front stack and by Bennett-Kruskal counting.
 * ``lru_curves`` — direct LRU simulation per capacity (Sec. 3.1-3.2) with
   prefix-contiguous hits (Sec. 2.2) and compute saved (Sec. 5.2, App. C).
+* ``curves_from_dist`` — the same curves from stack distances by Mattson
+  inclusion (App. B).
+* ``belady_curves`` — Belady's offline optimum (Sec. 3.2): direct MIN
+  simulation per capacity, same prefix rule and costs.
 * ``lru_curves_variant``, ``sd_variant`` — Sec. 3.1: leaf-first touch order
   and whole-request residency (every block looked up at the request's
   arrival), by direct LRU per capacity, Fenwick counting and Mattson's list.
@@ -79,6 +83,10 @@ def _load():
         lib.orc_lru_curves.restype = i32
         lib.orc_lru_curves.argtypes = [vp, vp, u32, u32, i32, u64, u64, vp, u32, i32, vp, vp, vp, vp, vp]
         lib.orc_prefix_hash.argtypes = [vp, vp, u32, u32, u64, vp]
+        lib.orc_belady_curves.restype = i32
+        lib.orc_belady_curves.argtypes = [vp, vp, u32, u32, i32, u64, u64, vp, u32, i32, vp, vp, vp, vp]
+        lib.orc_curves_from_dist.restype = i32
+        lib.orc_curves_from_dist.argtypes = [vp, vp, u32, u32, i32, u64, u64, vp, u32, vp, vp, vp]
         lib.orc_lru_curves_variant.restype = i32
         lib.orc_lru_curves_variant.argtypes = [vp, vp, u32, u32, i32, u64, u64, vp, u32, i32, i32, i32, vp, vp, vp]
         lib.orc_sd_variant.restype = i32
@@ -155,6 +163,43 @@ def lru_curves(ids, req_blk_off, B: int, caps, kind: int = COST_MEASURED, f_lin:
         raise ValueError("bad capacity grid (capacities must be >= 1)")
     saved = [int(h) << 64 | int(l) for l, h in zip(slo, shi)]
     return [int(h) for h in hits], saved, int(thi[0]) << 64 | int(tlo[0])
+
+
+def belady_curves(ids, req_blk_off, B: int, caps, kind: int = COST_MEASURED, f_lin: int = F_LIN,
+                  f_attn: int = F_ATTN, threads: int | None = None):
+    """Belady's MIN simulated directly at each capacity (evict the resident
+    block, other than the one just brought in, whose next access is farthest;
+    every access admitted), with the prefix rule.  Returns (hits list[int],
+    saved list[int], raw_hits list[int]); raw hits ignore the prefix rule."""
+    ids, bo, caps = _c(ids, np.uint32), _c(req_blk_off, np.uint64), _c(caps, np.uint64)
+    G = caps.shape[0]
+    hits = np.zeros(G, dtype=np.uint64)
+    raw = np.zeros(G, dtype=np.uint64)
+    slo = np.zeros(G, dtype=np.uint64)
+    shi = np.zeros(G, dtype=np.uint64)
+    nthreads = threads or max(1, min(G, os.cpu_count() or 1))
+    rc = _load().orc_belady_curves(_p(ids), _p(bo), bo.shape[0] - 1, int(B), int(kind), int(f_lin), int(f_attn),
+                                   _p(caps), G, nthreads, _p(hits), _p(slo), _p(shi), _p(raw))
+    if rc != 0:
+        raise ValueError("bad capacity grid (capacities must be >= 1)")
+    return [int(h) for h in hits], [int(h) << 64 | int(l) for l, h in zip(slo, shi)], [int(x) for x in raw]
+
+
+def curves_from_dist(sd, req_blk_off, B: int, caps, kind: int = COST_MEASURED, f_lin: int = F_LIN,
+                     f_attn: int = F_ATTN):
+    """Hits and compute saved per capacity from stack distances by Mattson
+    inclusion (running maximum per request, root-first).  Returns (hits
+    list[int], saved list[int]); caps strictly ascending."""
+    sd, bo, caps = _c(sd, np.uint32), _c(req_blk_off, np.uint64), _c(caps, np.uint64)
+    G = caps.shape[0]
+    hits = np.zeros(G, dtype=np.uint64)
+    slo = np.zeros(G, dtype=np.uint64)
+    shi = np.zeros(G, dtype=np.uint64)
+    rc = _load().orc_curves_from_dist(_p(sd), _p(bo), bo.shape[0] - 1, int(B), int(kind), int(f_lin), int(f_attn),
+                                      _p(caps), G, _p(hits), _p(slo), _p(shi))
+    if rc != 0:
+        raise ValueError("bad capacity grid (capacities must be >= 1 and strictly ascending)")
+    return [int(h) for h in hits], [int(h) << 64 | int(l) for l, h in zip(slo, shi)]
 
 
 def prefix_hash(tokens, req_tok_off, B: int, seed: int) -> np.ndarray:

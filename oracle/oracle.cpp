@@ -23,6 +23,9 @@
 //        orc_sd_fenwick (Bennett & Kruskal 1975 counting), two independent ways.
 //   * Belady's next use (Sec. 3.2, 5.2).  -> orc_reuse: previous and next
 //     access of the same block.
+//   * Sec. 3.2: Belady's optimum as the offline ceiling.  -> orc_belady_curves:
+//     one direct MIN simulation (evict the farthest next access) per capacity,
+//     with the same prefix rule as the LRU curves.
 //   * Sec. 3.1 (the paper's simulator keeps a whole request resident and
 //     makes room for it up front) and the order a request's blocks are
 //     touched in.  -> orc_lru_curves_variant (direct LRU per capacity),
@@ -45,7 +48,9 @@
 #include <atomic>
 #include <cstdint>
 #include <cstring>
+#include <iterator>
 #include <list>
+#include <set>
 #include <thread>
 #include <unordered_map>
 #include <vector>
@@ -287,15 +292,138 @@ int orc_lru_curves(const uint32_t* ids, const uint64_t* req_blk_off, uint32_t n_
   return 0;
 }
 
+// Belady's offline optimum (Belady 1966), the paper's offline ceiling
+// (Sec. 3.2, and the headroom in App. A-B), simulated directly, one capacity
+// at a time.  For capacity C: replay requests in trace order and their blocks
+// root-first; a resident block stays (a hit); a missing block is brought in
+// and, if the cache then holds more than C blocks, the resident block other
+// than the one just brought in whose next access lies farthest in the future
+// (never again counts as farthest) is evicted.  Every accessed block is
+// admitted: the demand-paging MIN that Mattson et al. (1970) show to be a
+// stack algorithm.  Block k of a request counts as a hit iff blocks 0..k of
+// that request were all resident when touched (Sec. 2.2 prefix reuse), as in
+// orc_lru_curves; raw_hits[g] counts every resident access, without the
+// prefix rule.  Next accesses come from a backward pass over the ids.
+// Outputs per capacity as orc_lru_curves.  Returns 0, or -1 on a capacity
+// of 0.
+int orc_belady_curves(const uint32_t* ids, const uint64_t* req_blk_off, uint32_t n_req, uint32_t B, int kind,
+                      uint64_t f_lin, uint64_t f_attn, const uint64_t* caps, uint32_t G, int threads, uint64_t* hits,
+                      uint64_t* saved_lo, uint64_t* saved_hi, uint64_t* raw_hits) {
+  for (uint32_t g = 0; g < G; ++g)
+    if (caps[g] == 0) return -1;
+  const uint64_t n = req_blk_off[n_req];
+  uint32_t D = 0;
+  for (uint64_t i = 0; i < n; ++i)
+    if (ids[i] + 1 > D) D = ids[i] + 1;
+  std::vector<uint32_t> nxt(n, NONE), last(D, NONE);
+  for (uint64_t i = n; i-- > 0;) {
+    nxt[i] = last[ids[i]];
+    last[ids[i]] = (uint32_t)i;
+  }
+  const uint64_t kNever = 1ULL << 63;  // "never again": beyond every access index, ties broken by id
+  const uint64_t kOut = ~0ULL;         // not resident
+  std::atomic<uint32_t> next_cap{0};
+  auto simulate = [&]() {
+    for (;;) {
+      uint32_t g = next_cap.fetch_add(1);
+      if (g >= G) return;
+      uint64_t C = caps[g];
+      std::set<std::pair<uint64_t, uint32_t>> by_next;  // resident blocks by (next access, id)
+      std::vector<uint64_t> key(D, kOut);                // each resident block's next access
+      uint64_t h = 0, raw = 0;
+      u128 saved = 0;
+      for (uint32_t r = 0; r < n_req; ++r) {
+        bool prefix_ok = true;
+        for (uint64_t k = 0; k < req_blk_off[r + 1] - req_blk_off[r]; ++k) {
+          uint64_t i = req_blk_off[r] + k;
+          uint32_t id = ids[i];
+          uint64_t nu = nxt[i] == NONE ? kNever + id : nxt[i];
+          bool resident = key[id] != kOut;
+          if (resident) by_next.erase({key[id], id});
+          by_next.insert({nu, id});
+          key[id] = nu;
+          if (!resident && by_next.size() > C) {
+            auto victim = std::prev(by_next.end());
+            if (victim->second == id) victim = std::prev(victim);  // the block just brought in stays
+            key[victim->second] = kOut;
+            by_next.erase(victim);
+          }
+          raw += resident;
+          prefix_ok = prefix_ok && resident;
+          if (prefix_ok) {
+            ++h;
+            saved += cost_of(k, B, kind, f_lin, f_attn);
+          }
+        }
+      }
+      hits[g] = h;
+      raw_hits[g] = raw;
+      saved_lo[g] = (uint64_t)saved;
+      saved_hi[g] = (uint64_t)(saved >> 64);
+    }
+  };
+  if (threads < 1) threads = 1;
+  std::vector<std::thread> pool;
+  for (int t = 1; t < threads; ++t) pool.emplace_back(simulate);
+  simulate();
+  for (auto& th : pool) th.join();
+  return 0;
+}
+
+// Curves from stack distances by Mattson inclusion (Mattson et al. 1970;
+// App. B "reuses reachable within C"): LRU is a stack algorithm, so the
+// access with stack distance sd is resident in every cache of at least sd
+// blocks.  With the prefix rule of Sec. 2.2, block k of a request counts at
+// capacity C iff the distances of blocks 0..k of that request are all at most
+// C, i.e. iff e_k = max(sd_0, .., sd_k) <= C (sd = NONE never counts).  For
+// each capacity: hits[g] = #{accesses with e <= caps[g]} and saved[g] = the
+// 128-bit sum of their costs.  The same outputs as orc_lru_curves, reached
+// through the distances instead of a cache simulation.  caps must be strictly
+// ascending.  Returns 0, or -1 on a capacity of 0 or an unsorted grid.
+int orc_curves_from_dist(const uint32_t* sd, const uint64_t* req_blk_off, uint32_t n_req, uint32_t B, int kind,
+                         uint64_t f_lin, uint64_t f_attn, const uint64_t* caps, uint32_t G, uint64_t* hits,
+                         uint64_t* saved_lo, uint64_t* saved_hi) {
+  for (uint32_t g = 0; g < G; ++g)
+    if (caps[g] == 0) return -1;
+  for (uint32_t g = 1; g < G; ++g)
+    if (caps[g] <= caps[g - 1]) return -1;
+  // An access with running maximum e counts at every capacity from the
+  // first grid point >= e on: add it to that point, then sum over the grid.
+  std::vector<uint64_t> h(G, 0);
+  std::vector<u128> saved(G, 0);
+  for (uint32_t r = 0; r < n_req; ++r) {
+    uint64_t e = 0;  // running maximum of the distances, NONE as 2^32 - 1
+    for (uint64_t k = 0; k < req_blk_off[r + 1] - req_blk_off[r]; ++k) {
+      uint32_t d = sd[req_blk_off[r] + k];
+      if (d > e) e = d;
+      if (e == NONE) continue;  // a cold block, or a deeper block of a request with one
+      uint32_t g = (uint32_t)(std::lower_bound(caps, caps + G, e) - caps);
+      if (g == G) continue;  // beyond the largest capacity
+      ++h[g];
+      saved[g] += cost_of(k, B, kind, f_lin, f_attn);
+    }
+  }
+  uint64_t hs = 0;
+  u128 ss = 0;
+  for (uint32_t g = 0; g < G; ++g) {
+    hs += h[g];
+    ss += saved[g];
+    hits[g] = hs;
+    saved_lo[g] = (uint64_t)ss;
+    saved_hi[g] = (uint64_t)(ss >> 64);
+  }
+  return 0;
+}
+
 // Polynomial prefix hash over GF(p), p = 2^61 - 1, evaluated token by token:
 // the prefix tok_0 .. tok_{m-1} of a request maps to
-//     H(m) = rho^m + sum_{t<m} tok_t * rho^(m-1-t)   (mod p),
-// i.e. the polynomial of the sequence (1, tok_0, ..., tok_{m-1}); the leading 1
-// keeps prefixes of different lengths apart.  For each block k of each request
-// the key is (H(B(k+1)) with rho_0, H(B(k+1)) with rho_1), written as
-// keys[2i], keys[2i+1].  The two bases come from `seed` by SplitMix64
-// (Steele, Lea, Flood 2014): rho_b = 2 + (output b of the stream seeded `seed`)
-// mod (p - 3).
+//     S(m) = sum_{t<m} (tok_t + 1) * u^(t+1)   (mod p).
+// Every coefficient tok_t + 1 is at least 1, so a prefix and any longer
+// prefix are different polynomials and no leading term is needed to keep
+// lengths apart.  For each block k of each request the key is
+// (S(B(k+1)) at u_0, S(B(k+1)) at u_1), written as keys[2i], keys[2i+1].
+// The two bases come from `seed` by SplitMix64 (Steele, Lea, Flood 2014):
+// u_b = 2 + (output b of the stream seeded `seed`) mod (p - 3).
 void orc_prefix_hash(const uint32_t* tokens, const uint64_t* req_tok_off, uint32_t n_req, uint32_t B, uint64_t seed,
                      uint64_t* keys) {
   const uint64_t P = (1ULL << 61) - 1;

@@ -125,9 +125,29 @@ def lib():
                 L.ptc_pipeline_workspace_bytes.restype = sz
                 L.ptc_pipeline_workspace_bytes.argtypes = [u32, u64, u32, u32]
                 L.ptc_pipeline.restype = st
-                L.ptc_pipeline.argtypes = [vp, u64, vp, vp, u32, u32, u64, ctypes.POINTER(CostModel), vp, u32,
+                L.ptc_pipeline.argtypes = [vp, u64, vp, vp, vp, u32, u32, u32, u64, ctypes.POINTER(CostModel), vp, u32,
                                            vp, vp, vp, vp, vp, vp, ctypes.POINTER(u64), ctypes.POINTER(u64), vp, vp,
                                            ctypes.POINTER(U128), vp, sz, vp]
+                L.ptc_pipeline_host_workspace_bytes.restype = sz
+                L.ptc_pipeline_host_workspace_bytes.argtypes = [u32, u64, u32, u32]
+                L.ptc_pipeline_host.restype = st
+                L.ptc_pipeline_host.argtypes = [vp, u64, vp, vp, vp, u32, u32, u32, u64, ctypes.POINTER(CostModel),
+                                                vp, u32,
+                                                ctypes.POINTER(u64), ctypes.POINTER(u64), vp, vp, ctypes.POINTER(U128),
+                                                vp, sz, vp]
+                L.ptc_belady_curves_workspace_bytes.restype = sz
+                L.ptc_belady_curves_workspace_bytes.argtypes = [u64, u32, u32]
+                L.ptc_belady_curves.restype = st
+                L.ptc_belady_curves.argtypes = [vp, u64, vp, u32, u32, ctypes.POINTER(CostModel), vp, u32, vp, vp, vp,
+                                                vp, sz, vp]
+                L.ptc_assign_ids_prior_workspace_bytes.restype = sz
+                L.ptc_assign_ids_prior_workspace_bytes.argtypes = [u64, u32]
+                L.ptc_assign_ids_prior.restype = st
+                L.ptc_assign_ids_prior.argtypes = [vp, u64, vp, vp, u32, vp, ctypes.POINTER(u64), vp, sz, vp]
+                L.ptc_session_prior_workspace_bytes.restype = sz
+                L.ptc_session_prior_workspace_bytes.argtypes = [u32]
+                L.ptc_session_prior.restype = st
+                L.ptc_session_prior.argtypes = [vp, u32, u32, vp, vp, sz, vp]
                 L.ptc_stack_distance_variant_workspace_bytes.restype = sz
                 L.ptc_stack_distance_variant_workspace_bytes.argtypes = [u64, u32, ctypes.c_int, ctypes.c_int]
                 L.ptc_stack_distance_variant.restype = st
@@ -238,6 +258,57 @@ def ptc_assign_ids(keys: torch.Tensor, ws: torch.Tensor | None = None, method: i
                                      _stream(dev))
         _check("ptc_assign_ids_ex", rc)
     return ids[:n], int(d.value)
+
+
+def ptc_belady_curves(prev: torch.Tensor, req_blk_off: torch.Tensor, block_size: int, caps,
+                      kind: int = PTC_COST_MEASURED, f_lin: int = F_LIN, f_attn: int = F_ATTN,
+                      ws: torch.Tensor | None = None) -> dict:
+    """Belady's MIN curves from the reuse indices.  Returns hits, saved
+    (Python ints, exact) and raw_hits (without the prefix rule) per capacity."""
+    dev = _dev(req_blk_off)
+    n = prev.numel()
+    R = req_blk_off.numel() - 1
+    caps = np.ascontiguousarray(caps, dtype=np.uint64)
+    G = caps.shape[0]
+    w = _workspace(lib().ptc_belady_curves_workspace_bytes(n, R, G), dev, ws)
+    hits = np.zeros(G, dtype=np.uint64)
+    raw = np.zeros(G, dtype=np.uint64)
+    saved = np.zeros(2 * G, dtype=np.uint64)
+    cm = CostModel(int(f_lin), int(f_attn), int(kind))
+    rc = lib().ptc_belady_curves(_ptr(prev), n, _ptr(req_blk_off), R, block_size, ctypes.byref(cm), caps.ctypes.data,
+                                 G, hits.ctypes.data, saved.ctypes.data, raw.ctypes.data, _ptr(w), w.numel(),
+                                 _stream(dev))
+    _check("ptc_belady_curves", rc)
+    return {"hits": [int(h) for h in hits], "raw_hits": [int(x) for x in raw],
+            "saved": [int(saved[2 * g + 1]) << 64 | int(saved[2 * g]) for g in range(G)]}
+
+
+def ptc_assign_ids_prior(keys: torch.Tensor, req_blk_off: torch.Tensor, req_prior: torch.Tensor,
+                         ws: torch.Tensor | None = None):
+    """Dense ids with a prior-request hint (req_prior[r] < r or PTC_NONE, int32
+    CUDA tensor).  Returns (ids int32[N], D); the same ids as ptc_assign_ids."""
+    dev = _dev(keys)
+    n = keys.shape[0]
+    R = req_prior.numel()
+    ids = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
+    d = ctypes.c_uint64(0)
+    w = _workspace(lib().ptc_assign_ids_prior_workspace_bytes(n, R), dev, ws)
+    rc = lib().ptc_assign_ids_prior(_ptr(keys), n, _ptr(req_blk_off), _ptr(req_prior), R, _ptr(ids), ctypes.byref(d),
+                                    _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_assign_ids_prior", rc)
+    return ids[:n], int(d.value)
+
+
+def ptc_session_prior(req_session: torch.Tensor, n_session: int, ws: torch.Tensor | None = None) -> torch.Tensor:
+    """The previous request of each request's session (PTC_NONE for a
+    session's first): int32 CUDA tensor of req_session's length."""
+    dev = _dev(req_session)
+    R = req_session.numel()
+    out = torch.empty(max(R, 1), dtype=torch.int32, device=dev)
+    w = _workspace(lib().ptc_session_prior_workspace_bytes(R), dev, ws)
+    rc = lib().ptc_session_prior(_ptr(req_session), R, int(n_session), _ptr(out), _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_session_prior", rc)
+    return out[:R]
 
 
 def ptc_verify_ids(tokens, req_tok_off, req_blk_off, block_size: int, ids: torch.Tensor, n_distinct: int,
@@ -445,7 +516,7 @@ class PipelinePlan:
 
     def __init__(self, tokens, req_tok_off, req_ts_us, block_size: int, caps, kind: int = PTC_COST_MEASURED,
                  seed: int = 0, f_lin: int = F_LIN, f_attn: int = F_ATTN, ws: torch.Tensor | None = None,
-                 outputs: dict | None = None):
+                 outputs: dict | None = None, req_session: torch.Tensor | None = None, n_session: int = 0):
         dev = _dev(req_tok_off)
         n_req = req_tok_off.numel() - 1
         n_tok = tokens.numel()
@@ -458,9 +529,10 @@ class PipelinePlan:
         self.total = U128()
         self.n, self.d = ctypes.c_uint64(0), ctypes.c_uint64(0)
         self.cm = CostModel(int(f_lin), int(f_attn), int(kind))
-        self._keep = (tokens, req_tok_off, req_ts_us, o)  # the pointers below stay valid
+        self._keep = (tokens, req_tok_off, req_ts_us, req_session, o)  # the pointers below stay valid
         self._fn = lib().ptc_pipeline
-        self._args = (_ptr(tokens), n_tok, _ptr(req_tok_off), _ptr(req_ts_us), n_req, block_size,
+        self._args = (_ptr(tokens), n_tok, _ptr(req_tok_off), _ptr(req_ts_us), _ptr(req_session),
+                      int(n_session) if req_session is not None else 0, n_req, block_size,
                       int(seed) & (2**64 - 1), ctypes.byref(self.cm), self.caps.ctypes.data, G, _ptr(o.get("keys")),
                       _ptr(o.get("req_blk_off")), _ptr(o.get("ids")), _ptr(o.get("prev")), _ptr(o.get("next")),
                       _ptr(o.get("dist")), ctypes.byref(self.n), ctypes.byref(self.d), self.hits.ctypes.data,
@@ -479,11 +551,66 @@ class PipelinePlan:
                 "total_cost": int(self.total.hi) << 64 | int(self.total.lo)}
 
 
+class HostPipelinePlan:
+    """ptc_pipeline_host with its arguments marshalled once: the trace is in
+    host memory (numpy arrays or CPU tensors; page-locked memory copies at
+    full speed) and every ``run()`` copies it to the device and runs the whole
+    path in one C call on the current stream of ``device``.  The workspace
+    (device memory, which also holds the copied trace) is made once.  After
+    ``run()`` the fields are those of PipelinePlan."""
+
+    def __init__(self, tokens, req_tok_off, req_ts_us, block_size: int, caps, kind: int = PTC_COST_MEASURED,
+                 seed: int = 0, f_lin: int = F_LIN, f_attn: int = F_ATTN, device="cuda",
+                 ws: torch.Tensor | None = None, req_session=None, n_session: int = 0):
+        dev = torch.device(device)
+        if dev.index is None:
+            dev = torch.device("cuda", torch.cuda.current_device())
+
+        def host_ptr(a, dt):
+            if a is None:
+                return None, None
+            if isinstance(a, torch.Tensor):
+                if a.is_cuda:
+                    raise ValueError("HostPipelinePlan takes host buffers")
+                return a, a.data_ptr()
+            a = np.ascontiguousarray(a, dtype=dt)
+            return a, a.ctypes.data
+
+        tok, tp = host_ptr(tokens, np.uint32)
+        off, op = host_ptr(req_tok_off, np.uint64)
+        ts, sp = host_ptr(req_ts_us, np.int64)
+        ses, sep = host_ptr(req_session, np.uint32)
+        n_req = (off.numel() if isinstance(off, torch.Tensor) else off.shape[0]) - 1
+        n_tok = tok.numel() if isinstance(tok, torch.Tensor) else tok.shape[0]
+        self.caps = np.ascontiguousarray(caps, dtype=np.uint64)
+        G = self.caps.shape[0]
+        self.ws = _workspace(lib().ptc_pipeline_host_workspace_bytes(n_req, n_tok, block_size, G), dev, ws)
+        self.hits = np.zeros(G, dtype=np.uint64)
+        self.saved = np.zeros(2 * G, dtype=np.uint64)
+        self.total = U128()
+        self.n, self.d = ctypes.c_uint64(0), ctypes.c_uint64(0)
+        self.cm = CostModel(int(f_lin), int(f_attn), int(kind))
+        self._keep = (tok, off, ts, ses)
+        self._fn = lib().ptc_pipeline_host
+        self._args = (tp, n_tok, op, sp, sep, int(n_session) if ses is not None else 0, n_req, block_size, int(seed) & (2**64 - 1), ctypes.byref(self.cm),
+                      self.caps.ctypes.data, G, ctypes.byref(self.n), ctypes.byref(self.d), self.hits.ctypes.data,
+                      self.saved.ctypes.data, ctypes.byref(self.total), _ptr(self.ws), self.ws.numel(), _stream(dev))
+
+    def run(self) -> "HostPipelinePlan":
+        rc = self._fn(*self._args)
+        if rc != 0:
+            raise PtcError("ptc_pipeline_host", rc)
+        return self
+
+    result = PipelinePlan.result
+
+
 def ptc_pipeline(tokens, req_tok_off, req_ts_us, block_size: int, caps, kind: int = PTC_COST_MEASURED, seed: int = 0,
-                 f_lin: int = F_LIN, f_attn: int = F_ATTN, ws: torch.Tensor | None = None, outputs: dict | None = None):
+                 f_lin: int = F_LIN, f_attn: int = F_ATTN, ws: torch.Tensor | None = None, outputs: dict | None = None,
+                 req_session: torch.Tensor | None = None, n_session: int = 0):
     """All five stages in one C call (trace already on the GPU).  ``outputs``
     may map any of keys / req_blk_off / ids / prev / next / dist to
     preallocated CUDA tensors that receive those arrays.  Returns the curves
     with N and D."""
     return PipelinePlan(tokens, req_tok_off, req_ts_us, block_size, caps, kind, seed, f_lin, f_attn, ws,
-                        outputs).run().result()
+                        outputs, req_session, n_session).run().result()

@@ -612,6 +612,24 @@ extern "C" size_t ptc_curves_workspace_bytes(uint64_t n, uint32_t n_req, uint32_
   return curves_layout(nullptr, n, n_cap).total;
 }
 
+ptc_status ptc::cost_coeffs(const ptc_cost_model* cm, uint32_t block_size, uint64_t* alpha_out, uint64_t* beta_out) {
+  const uint64_t B = block_size;
+  uint64_t alpha = 0, beta = 0, lin = 0, attn0 = 0;
+  if (cm->kind == PTC_COST_UNIFORM) {
+    alpha = 1;
+  } else if (cm->kind == PTC_COST_MEASURED || cm->kind == PTC_COST_LINEAR) {
+    if (!mul_ok(cm->f_attn, B * (B + 1) / 2, &attn0) || !mul_ok(cm->f_attn, B * B, &beta)) return PTC_ERR_OVERFLOW;
+    if (cm->kind == PTC_COST_MEASURED && !mul_ok(cm->f_lin, B, &lin)) return PTC_ERR_OVERFLOW;
+    alpha = lin + attn0;
+    if (alpha < lin) return PTC_ERR_OVERFLOW;
+  } else {
+    return PTC_ERR_INVALID_ARG;
+  }
+  *alpha_out = alpha;
+  *beta_out = beta;
+  return PTC_OK;
+}
+
 ptc_status ptc::curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,
                             uint32_t block_size, const ptc_cost_model* cm, const uint64_t* cap_host, uint32_t n_cap,
                             uint64_t* hits_host_out, ptc_u128* saved_host_out, ptc_u128* total_cost_host_out,
@@ -625,18 +643,9 @@ ptc_status ptc::curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* re
   for (uint32_t g = 0; g < n_cap; ++g)
     if (cap_host[g] < 1 || (g && cap_host[g] <= cap_host[g - 1])) return PTC_ERR_INVALID_ARG;
   // cost(k) = alpha + beta k
-  const uint64_t B = block_size;
-  uint64_t alpha = 0, beta = 0, lin = 0, attn0 = 0;
-  if (cm->kind == PTC_COST_UNIFORM) {
-    alpha = 1;
-  } else if (cm->kind == PTC_COST_MEASURED || cm->kind == PTC_COST_LINEAR) {
-    if (!mul_ok(cm->f_attn, B * (B + 1) / 2, &attn0) || !mul_ok(cm->f_attn, B * B, &beta)) return PTC_ERR_OVERFLOW;
-    if (cm->kind == PTC_COST_MEASURED && !mul_ok(cm->f_lin, B, &lin)) return PTC_ERR_OVERFLOW;
-    alpha = lin + attn0;
-    if (alpha < lin) return PTC_ERR_OVERFLOW;
-  } else {
-    return PTC_ERR_INVALID_ARG;
-  }
+  uint64_t alpha = 0, beta = 0;
+  const ptc_status crc = cost_coeffs(cm, block_size, &alpha, &beta);
+  if (crc != PTC_OK) return crc;
   if (!ws_ok(ws, ws_bytes, curves_layout(nullptr, n, n_cap).total)) return PTC_ERR_WORKSPACE;
   cudaStream_t s = stream;
   const CurvesLayout L = curves_layout(ws, n, n_cap);

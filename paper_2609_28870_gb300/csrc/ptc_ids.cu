@@ -197,6 +197,8 @@ __global__ void __launch_bounds__(kMkThreads) k_ids_mark(const ulonglong2* __res
 // dependent loads in flight together.
 constexpr int kGaThreads = 256;
 constexpr int kGaPer = 8;
+// slot_of of an access that the prior-request hint matched (no slot)
+constexpr uint32_t kMatchedSlot = 0xFFFFFFFFu;
 __global__ void __launch_bounds__(kGaThreads) k_ids_gather(const uint32_t* __restrict__ slot_of,
                                                           const ulonglong2* __restrict__ table,
                                                           const uint32_t* __restrict__ bits,
@@ -214,7 +216,7 @@ __global__ void __launch_bounds__(kGaThreads) k_ids_gather(const uint32_t* __res
 #pragma unroll
   for (int k = 0; k < kGaPer; ++k) {
     const uint32_t i = i0 + k * kGaThreads;
-    f[k] = i < n ? __ldg(reinterpret_cast<const uint32_t*>(&table[f[k]]) + 3) : kNone;
+    f[k] = i < n && f[k] != kMatchedSlot ? __ldg(reinterpret_cast<const uint32_t*>(&table[f[k]]) + 3) : kMatchedSlot;
   }
   uint32_t wp[kGaPer], bw[kGaPer];
 #pragma unroll
@@ -223,10 +225,11 @@ __global__ void __launch_bounds__(kGaThreads) k_ids_gather(const uint32_t* __res
     wp[k] = ok ? wpre[f[k] >> 5] : 0u;
     bw[k] = ok ? bits[f[k] >> 5] : 0u;
   }
+  // a matched access (prior-request hint) gets its id from k_ids_follow
 #pragma unroll
   for (int k = 0; k < kGaPer; ++k) {
     const uint32_t i = i0 + k * kGaThreads;
-    if (i < n) ids[i] = f[k] < n ? wp[k] + __popc(bw[k] & ((1u << (f[k] & 31)) - 1u)) : kNone;
+    if (i < n && f[k] != kMatchedSlot) ids[i] = f[k] < n ? wp[k] + __popc(bw[k] & ((1u << (f[k] & 31)) - 1u)) : kNone;
   }
 }
 
@@ -412,6 +415,148 @@ __global__ void __launch_bounds__(kGaThreads) k_ids_gather_part(const uint32_t* 
   }
 }
 
+// ---------------------------------------------------------------- prior-request hint
+// A request usually re-sends the whole context of an earlier request of its
+// session and appends to it (Sec. 2.3: the turns of a multi-turn session
+// extend one context).  Given a hint prior[r] (an earlier request, or none),
+// access (r, k) is "matched" when its key equals that of block k of request
+// prior[r]: its prefix occurred earlier, so it is not a first occurrence and
+// is not inserted.  Equal keys mean equal prefixes, so the matched blocks of
+// r are its depths k < lam[r].  A first occurrence is never matched, so the
+// table of the unmatched keys still holds every key with its smallest access
+// index.  A matched access takes the id of block k of the nearest request on
+// its prior chain whose depth k is unmatched (k_ids_follow).  The ids do not
+// depend on the hint: any prior[r] < r gives the same ids, only the number of
+// table probes changes.
+constexpr uint32_t kMatched = kMatchedSlot;  // slot_of of a matched access
+
+struct PriorHint {
+  const uint64_t* blk_off;  // n_req + 1 access offsets of the requests
+  const uint32_t* prior;    // n_req: an earlier request, or kNone
+  uint32_t n_req;
+  uint32_t* lam;            // n_req: first unmatched depth, kNone if none (cleared to kNone)
+  uint32_t* tile_req;       // request of the first access of every kReqTile accesses, and n_req - 1 last
+};
+constexpr uint32_t kReqTileLog2 = 11;  // 2048 accesses per entry of tile_req
+
+// The last request r in [lo, hi] with off[r] <= i (requests without blocks
+// are skipped because a later offset equals theirs).
+__device__ __forceinline__ uint32_t req_at(const uint64_t* __restrict__ off, uint32_t lo, uint32_t hi, uint64_t i) {
+  while (lo < hi) {
+    const uint32_t mid = (lo + hi + 1) >> 1;
+    if (__ldg(&off[mid]) <= i)
+      lo = mid;
+    else
+      hi = mid - 1;
+  }
+  return lo;
+}
+
+// tile_req[t] = the request of access t * 2048 (one binary search per entry),
+// and tile_req[T] = n_req - 1, so accesses of tile t lie in requests
+// [tile_req[t], tile_req[t + 1]].
+__global__ void k_tile_req(PriorHint ph, uint32_t n_ub, const uint64_t* n_dev) {
+  grid_dep_sync();
+  const uint32_t n = keys_used(n_ub, n_dev);
+  const uint32_t T = (n + (1u << kReqTileLog2) - 1) >> kReqTileLog2;
+  const uint32_t t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t < T) ph.tile_req[t] = req_at(ph.blk_off, 0, ph.n_req - 1, (uint64_t)t << kReqTileLog2);
+  if (t == T) ph.tile_req[t] = ph.n_req - 1;
+}
+
+// One key per thread.  Each access finds its request by binary search among
+// the few requests its 2048-access tile spans (tile_req).
+// A matched access writes kMatched and stops; an unmatched one lowers its
+// request's lam (one atomic per group of lanes in one request) and settles
+// its key in the table as k_ids_insert does.
+__global__ void __launch_bounds__(kInsThreads) k_ids_insert_prior(const ulonglong2* __restrict__ keys, uint32_t n_ub,
+                                                                  const uint64_t* n_dev, ulonglong2* table,
+                                                                  uint32_t log2m, uint64_t probe_cap,
+                                                                  uint32_t* __restrict__ slot_of, DevStatus* st,
+                                                                  InsCarry kc, PriorHint ph) {
+  grid_dep_sync();
+  const uint32_t n = keys_used(n_ub, n_dev);
+  const uint32_t i = blockIdx.x * kInsThreads + threadIdx.x;
+  if (i >= n) return;
+  const ulonglong2 k = carried_key(keys, i, n, kc);
+  const uint32_t t = i >> kReqTileLog2;
+  const uint32_t r0 = __ldg(&ph.tile_req[t]), r1 = __ldg(&ph.tile_req[t + 1]);
+  if (k.x >= kP61 || k.y >= kP61) {
+    raise_err(st, kErrInvalid);
+    slot_of[i] = 0;
+    return;
+  }
+  const uint32_t r = req_at(ph.blk_off, r0, r1, i);
+  const uint64_t depth = i - __ldg(&ph.blk_off[r]);
+  const uint32_t p = __ldg(&ph.prior[r]);
+  bool matched = false;
+  if (p != kNone) {
+    if (p >= r) {
+      raise_err(st, kErrInvalid);  // a hint must point to an earlier request
+    } else {
+      const uint64_t pb = __ldg(&ph.blk_off[p]), pn = __ldg(&ph.blk_off[p + 1]) - pb;
+      if (depth < pn && pb + depth < n) {
+        const ulonglong2 q = carried_key(keys, (uint32_t)(pb + depth), n, kc);
+        matched = q.x == k.x && q.y == k.y;
+      }
+    }
+  }
+  if (matched) {
+    __stcs(&slot_of[i], kMatched);
+    return;
+  }
+  const unsigned grp = __match_any_sync(__activemask(), r);
+  const uint32_t lo = __reduce_min_sync(grp, (uint32_t)depth);
+  if ((threadIdx.x & 31) == (uint32_t)(__ffs(grp) - 1)) atomicMin(&ph.lam[r], lo);
+  const uint64_t pos = home_slot(k.x, k.y, log2m);
+  settle(table, (1ULL << log2m) - 1, probe_cap, i, k, pos, ld_slot(&table[pos]), &slot_of[i], st);
+}
+
+// ids of the matched accesses, one warp per request r: its depths below
+// lam[r] equal those of prior[r]; walking the prior chain t = prior[r],
+// prior[t], ..., the depths in [lam[t], hi) are unmatched in t (their ids
+// come from the table) and are copied, and hi drops to lam[t], until no
+// depth is left.  A chain that does not strictly descend, or that ends while
+// depths are left, is malformed input.
+constexpr int kFoThreads = 256;
+__global__ void __launch_bounds__(kFoThreads) k_ids_follow(PriorHint ph, uint32_t* __restrict__ ids, DevStatus* st) {
+  grid_dep_sync();
+  const uint32_t lane = threadIdx.x & 31;
+  const uint32_t r = blockIdx.x * (kFoThreads / 32) + (threadIdx.x >> 5);
+  if (r >= ph.n_req) return;
+  const uint64_t b = ph.blk_off[r], nr = ph.blk_off[r + 1] - b;
+  const uint32_t lr = ph.lam[r];
+  uint64_t hi = lr < nr ? lr : nr;
+  uint32_t cur = r, t = ph.prior[r];
+  while (hi > 0) {
+    if (t == kNone || t >= cur) {
+      if (lane == 0) raise_err(st, kErrInvalid);
+      return;
+    }
+    const uint64_t tb = ph.blk_off[t];
+    const uint64_t lo = ph.lam[t];  // kNone (no unmatched depth) is above every hi
+    if (lo < hi) {
+      for (uint64_t d = lo + lane; d < hi; d += 32) ids[b + d] = ids[tb + d];
+      hi = lo;
+    }
+    cur = t;
+    t = ph.prior[t];
+  }
+}
+
+// prior[r] = the previous request of r's session, from the requests sorted
+// stably by session label: neighbours in that order with the same label.
+__global__ void k_session_prior(const uint32_t* __restrict__ ses_sorted, const uint32_t* __restrict__ req_sorted,
+                                const uint32_t* __restrict__ ses, uint32_t n_req, uint32_t n_session,
+                                uint32_t* __restrict__ prior, uint32_t* err) {
+  grid_dep_sync();
+  const uint32_t j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j >= n_req) return;
+  if (ses[j] >= n_session) atomicOr(err, kErrInvalid);  // the sort sees only the label's low bits
+  const uint32_t sj = ses_sorted[j];
+  prior[req_sorted[j]] = (j > 0 && ses_sorted[j - 1] == sj) ? req_sorted[j - 1] : kNone;
+}
+
 // Slots for n keys at most: the full table holds 1.5 n.  The first attempt
 // holds n / 3 while that is at most 2^22 slots (64 MB, half of L2): traces
 // that repeat most blocks fill it well below half, and it stays in L2.  A
@@ -454,13 +599,15 @@ struct IdsLayout {
   uint32_t *pcount, *pcursor;  // grouped: keys per partition, next place in each
   ulonglong2* pkey;            // grouped: the keys, carry added, partition by partition
   uint32_t* pidx;              // grouped: their access indices
+  uint32_t* lam;               // prior hint: first unmatched depth of each request
+  uint32_t* tile_req;          // prior hint: request of every 2048th access
   uint32_t nwords;
   size_t zero_bytes;
   size_t total;
   uint32_t log2m;
 };
 
-IdsLayout ids_layout(void* ws, uint64_t n, bool grouped) {
+IdsLayout ids_layout(void* ws, uint64_t n, bool grouped, uint32_t n_req_hint = 0) {
   IdsLayout L;
   Carver cv(ws);
   L.log2m = full_table_log2(n);
@@ -484,6 +631,8 @@ IdsLayout ids_layout(void* ws, uint64_t n, bool grouped) {
     L.pkey = cv.take<ulonglong2>(nn);
     L.pidx = cv.take<uint32_t>(nn);
   }
+  L.lam = n_req_hint ? cv.take<uint32_t>(n_req_hint) : nullptr;
+  L.tile_req = n_req_hint ? cv.take<uint32_t>((nn >> kReqTileLog2) + 2) : nullptr;
   L.total = cv.bytes();
   return L;
 }
@@ -562,8 +711,10 @@ extern "C" size_t ptc_assign_ids_ex_workspace_bytes(uint64_t n, int method) {
 ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev, uint32_t* ids_out,
                         uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
                         cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc,
-                        uint64_t* nd_slot, uint32_t* err_slot, bool full_table, int method) {
+                        uint64_t* nd_slot, uint32_t* err_slot, bool full_table, int method, const IdsHint* hint) {
   if (method != PTC_IDS_AUTO && method != PTC_IDS_DIRECT && method != PTC_IDS_GROUPED) return PTC_ERR_INVALID_ARG;
+  if (hint && (method == PTC_IDS_GROUPED || hint->n_req == 0 || !hint->blk_off || !hint->prior))
+    return PTC_ERR_INVALID_ARG;
   if (kc && (kc->tile_blocks == 0 || (kc->tile_blocks & (kc->tile_blocks - 1)) != 0)) return PTC_ERR_INVALID_ARG;
   const InsCarry ic = kc ? InsCarry{kc->carry, kc->lead, (uint32_t)__builtin_ctz(kc->tile_blocks)}
                         : InsCarry{nullptr, nullptr, 0};
@@ -573,15 +724,21 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
   if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
   if (n > 0 && (keys == nullptr || ids_out == nullptr)) return PTC_ERR_INVALID_ARG;
   const bool grouped = ids_grouped(n, method);
-  if (!ws_ok(ws, ws_bytes, ids_layout(nullptr, n, grouped).total)) return PTC_ERR_WORKSPACE;
-  const IdsLayout L = ids_layout(ws, n, grouped);
+  const uint32_t hreq = hint ? hint->n_req : 0;
+  if (!ws_ok(ws, ws_bytes, ids_layout(nullptr, n, grouped, hreq).total)) return PTC_ERR_WORKSPACE;
+  const IdsLayout L = ids_layout(ws, n, grouped, hreq);
+  const PriorHint ph = hint ? PriorHint{hint->blk_off, hint->prior, hint->n_req, L.lam, L.tile_req}
+                            : PriorHint{nullptr, nullptr, 0, nullptr, nullptr};
   // the status block, the table (all ones: empty), the first-occurrence
   // bitmap and the partition counts are cleared by one launch
   auto start = [&](uint32_t log2m) -> bool {
     const FillRange zf[4] = {{ws, L.zero_bytes, 0u},
                             {L.table, n > 0 ? sizeof(ulonglong2) << log2m : 0, ~0u},
                             {L.bits, n > 0 ? sizeof(uint32_t) * L.nwords : 0, 0u},
-                            {L.pcount, grouped && n > 0 ? sizeof(uint32_t) << kMaxPartsLog2 : 0, 0u}};
+                            {grouped ? (void*)L.pcount : (void*)L.lam,
+                             grouped ? (n > 0 ? sizeof(uint32_t) << kMaxPartsLog2 : 0)
+                                     : (hint && n > 0 ? sizeof(uint32_t) * hreq : 0),
+                             grouped ? 0u : ~0u}};
     return fill_many_async(zf, 4, s) == PTC_OK && carry_errors(carry_err, n_carry, L.st, s) == PTC_OK;
   };
   auto run = [&](uint32_t log2m, uint64_t probe_cap) -> bool {
@@ -600,6 +757,10 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
                  L.pcursor, L.pkey, L.pidx);
       PTC_KERNEL("k_ids_insert_part", s, k_ids_insert_part, ceil_div_u32(n, kInsThreads), kInsThreads, 0, L.pkey, L.pidx,
                  n32, n_dev, L.table, log2m, probe_cap, L.slot_of, L.st);
+    } else if (hint) {
+      PTC_KERNEL("k_tile_req", s, k_tile_req, ceil_div_u32((n >> kReqTileLog2) + 2, 256), 256, 0, ph, n32, n_dev);
+      PTC_KERNEL("k_ids_insert_prior", s, k_ids_insert_prior, ceil_div_u32(n, kInsThreads), kInsThreads, 0, k, n32,
+                 n_dev, L.table, log2m, probe_cap, L.slot_of, L.st, ic, ph);
     } else {
       PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads * kInsK), kInsThreads, 0, k, n32, n_dev,
                  L.table, log2m, probe_cap, L.slot_of, L.st, ic);
@@ -614,6 +775,9 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
     else
       PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of,
                  L.table, L.bits, L.wpre, n32, n_dev, ids_out);
+    if (hint)
+      PTC_KERNEL("k_ids_follow", s, k_ids_follow, ceil_div_u32(hint->n_req, kFoThreads / 32), kFoThreads, 0, ph,
+                 ids_out, L.st);
     return true;
   };
   const uint32_t first_log2m = full_table ? L.log2m : small_table_log2(n);
@@ -656,6 +820,72 @@ extern "C" ptc_status ptc_assign_ids_ex(const ptc_u128* keys, uint64_t n, uint32
                                         void* stream) {
   return ptc::ids_impl(keys, n, nullptr, ids_out, nullptr, n_distinct_host_out, ws, ws_bytes, (cudaStream_t)stream,
                        nullptr, 0, nullptr, nullptr, nullptr, false, method);
+}
+
+bool ptc::ids_table_in_dram(uint64_t n) { return n / 3 + 64 > (1ULL << kL2TableLog2); }
+
+size_t ptc::ids_ws_bytes(uint64_t n, uint32_t n_req_hint) { return ids_layout(nullptr, n, false, n_req_hint).total; }
+
+extern "C" size_t ptc_assign_ids_prior_workspace_bytes(uint64_t n, uint32_t n_req) {
+  return ids_layout(nullptr, n, false, n_req ? n_req : 1).total;
+}
+
+extern "C" ptc_status ptc_assign_ids_prior(const ptc_u128* keys, uint64_t n, const uint64_t* req_blk_off,
+                                           const uint32_t* req_prior, uint32_t n_req, uint32_t* ids_out,
+                                           uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes, void* stream) {
+  if (n > 0 && (n_req == 0 || !req_blk_off || !req_prior)) return PTC_ERR_INVALID_ARG;
+  if (n == 0 || n_req == 0)
+    return ptc::ids_impl(keys, n, nullptr, ids_out, nullptr, n_distinct_host_out, ws, ws_bytes,
+                         (cudaStream_t)stream, nullptr, 0);
+  const IdsHint h{req_blk_off, req_prior, n_req};
+  return ptc::ids_impl(keys, n, nullptr, ids_out, nullptr, n_distinct_host_out, ws, ws_bytes, (cudaStream_t)stream,
+                       nullptr, 0, nullptr, nullptr, nullptr, false, PTC_IDS_AUTO, &h);
+}
+
+size_t ptc::session_prior_bytes(uint32_t n_req) {
+  Carver cv(nullptr);
+  cv.take<DevStatus>(1);
+  cv.take<unsigned char>(sort_pairs_bytes(n_req ? n_req : 1));
+  return cv.bytes();
+}
+
+// prior[r] = the previous request of r's session (kNone for a session's
+// first request): a stable sort of the requests by session label, then one
+// pass over neighbours.  Queued on `s`; a label >= n_session raises
+// kErrInvalid into *err.
+void ptc::session_prior(const uint32_t* req_session, uint32_t n_req, uint32_t n_session, uint32_t* prior, void* ws,
+                        cudaStream_t s, uint32_t* err) {
+  Carver cv(ws);
+  DevStatus* st = cv.take<DevStatus>(1);  // the sort has no bound to check and raises nothing
+  void* sws = cv.take<unsigned char>(sort_pairs_bytes(n_req ? n_req : 1));
+  uint32_t bits = 1;
+  while (bits < 32 && (1ULL << bits) < n_session) ++bits;
+  const uint32_t *ks = nullptr, *vs = nullptr;
+  sort_pairs(req_session, nullptr, n_req, bits, sws, s, st, &ks, &vs);
+  PTC_KERNEL("k_session_prior", s, k_session_prior, ceil_div_u32(n_req, 256), 256, 0, ks, vs, req_session, n_req,
+             n_session, prior, err);
+}
+
+extern "C" size_t ptc_session_prior_workspace_bytes(uint32_t n_req) {
+  Carver cv(nullptr);
+  cv.take<DevStatus>(1);
+  cv.take<unsigned char>(session_prior_bytes(n_req));
+  return cv.bytes();
+}
+
+extern "C" ptc_status ptc_session_prior(const uint32_t* req_session, uint32_t n_req, uint32_t n_session,
+                                        uint32_t* prior_out, void* ws, size_t ws_bytes, void* stream) {
+  if (n_req == 0) return PTC_OK;
+  if (!req_session || !prior_out || n_session == 0) return PTC_ERR_INVALID_ARG;
+  if (!ws_ok(ws, ws_bytes, ptc_session_prior_workspace_bytes(n_req))) return PTC_ERR_WORKSPACE;
+  cudaStream_t s = (cudaStream_t)stream;
+  Carver cv(ws);
+  DevStatus* st = cv.take<DevStatus>(1);
+  void* sws = cv.take<unsigned char>(session_prior_bytes(n_req));
+  if (begin_call(ws, kStatusBytes, s) != PTC_OK) return PTC_ERR_CUDA;
+  session_prior(req_session, n_req, n_session, prior_out, sws, s, &st->err);
+  DevStatus h;
+  return end_call(st, s, &h);
 }
 
 extern "C" size_t ptc_verify_ids_workspace_bytes(uint64_t n, uint64_t n_distinct) {

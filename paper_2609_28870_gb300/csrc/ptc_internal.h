@@ -193,11 +193,28 @@ ptc_status hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req
 // number of keys used in nd_slot[1] and its error word in *err_slot (a
 // probe sequence that outran the small table shows as exactly
 // kErrTableFull; redo the stage then with `full_table`).
+// The prior-request hint of stage a2 (ptc_assign_ids_prior): prior[r] is an
+// earlier request whose blocks request r is likely to repeat, or PTC_NONE.
+struct IdsHint {
+  const uint64_t* blk_off;  // n_req + 1 (device)
+  const uint32_t* prior;    // n_req (device)
+  uint32_t n_req;
+};
+size_t ids_ws_bytes(uint64_t n, uint32_t n_req_hint);
+// Whether the id table for n keys is larger than the part of L2 it may take:
+// only then do the table probes the prior-request hint saves cost DRAM
+// traffic; an L2-resident table probes faster than the hint's extra reads.
+bool ids_table_in_dram(uint64_t n);
+// The previous request of each request's session (ptc_session_prior),
+// queued on `s` without waiting; scratch of session_prior_bytes(n_req).
+size_t session_prior_bytes(uint32_t n_req);
+void session_prior(const uint32_t* req_session, uint32_t n_req, uint32_t n_session, uint32_t* prior, void* ws,
+                   cudaStream_t s, uint32_t* err);
 ptc_status ids_impl(const ptc_u128* keys, uint64_t n_ub, const uint64_t* n_dev, uint32_t* ids_out,
                     uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
                     cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc = nullptr,
                     uint64_t* nd_slot = nullptr, uint32_t* err_slot = nullptr, bool full_table = false,
-                    int method = PTC_IDS_AUTO);
+                    int method = PTC_IDS_AUTO, const IdsHint* hint = nullptr);
 ptc_status stack_distance_view(const uint32_t* prev, uint64_t n, uint32_t* dist_out, int method, void* ws,
                                size_t ws_bytes, cudaStream_t s, RunsView* view, uint32_t* defer_err);
 // Stage b as ptc_reuse_indices does it (ptc_reuse.cu); with `defer_err` the
@@ -217,6 +234,10 @@ struct ReuseHostOut {
 ptc_status reuse_view(const uint32_t* ids, uint64_t n, uint64_t n_distinct, uint32_t* prev_out, uint32_t* next_out,
                       void* ws, size_t ws_bytes, cudaStream_t s, uint32_t* defer_err, const ReuseDevIn* din = nullptr,
                       ReuseHostOut* hout = nullptr);
+// The per-block cost as cost(k) = alpha + beta k for block size B (R7: every
+// cost kind is affine in the depth k); PTC_ERR_OVERFLOW if a coefficient
+// exceeds 64 bits, PTC_ERR_INVALID_ARG for an unknown kind (ptc_curves.cu).
+ptc_status cost_coeffs(const ptc_cost_model* cm, uint32_t block_size, uint64_t* alpha, uint64_t* beta);
 // Stage d (ptc_curves.cu); with `runs` (from stack_distance_view) the curves
 // come from the runs instead of a pass over every distance.
 ptc_status curves_impl(const uint32_t* dist, uint64_t n, const uint64_t* req_blk_off, uint32_t n_req,

@@ -1,20 +1,25 @@
 """Parity at the full sizes of the agentic (2.08B tokens, 130M accesses),
 agentic-at-other-block-sizes and mixed 24-hour (10.0B tokens, 624M accesses)
 workloads, in the launch configuration the bench times (ptc_pipeline, one C
-call, caller arrays for every intermediate).
+call, session labels given, caller arrays for every intermediate).
 
-Where the oracle finishes in a couple of minutes (the agentic trace at every
-block size) every per-access array is compared with it element by element.
-The mixed trace is too large for the oracle's exact trie in test time, so it
-is checked through what holds at any size:
-  * dense ids number blocks by first occurrence, so the ids, prev and stack
-    distances of the first accesses depend on the trace up to them only: the
-    oracle run on a prefix of the requests must match the full run there;
+The agentic trace at B = 16 is compared with the oracle run live, element by
+element.  The other block sizes and the mixed trace are compared with the
+oracle's stored results (tests/golden/big_configs.json, written by
+tests/golden/make_big_goldens.py, which runs the oracle alone): SHA-256 of
+every per-access array (ids, prev, next, stack distances), N and D, hits and
+128-bit compute saved at every grid point, the total cost, and the direct
+per-capacity LRU simulation at several grid points.  On top of that, what
+holds at any size is checked from the GPU's own arrays:
   * sampled accesses against the definitions themselves (same id iff same
     prefix, by token comparison; prev is the last earlier access with the id;
     the stack distance is one plus the distinct ids strictly between);
   * the identities of the method (next[prev[i]] = i, D first accesses,
     Mattson inclusion for every grid point, the cost totals in closed form)."""
+import hashlib
+import json
+import os
+
 import numpy as np
 import pytest
 
@@ -32,7 +37,48 @@ def _gpu():
         pytest.skip("no CUDA device")
 
 
-def _pipeline(tok, off, ts, n_tok, n_req, B, caps):
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "big_configs.json")
+
+
+def _sha(a):
+    h = hashlib.sha256()
+    mv = memoryview(np.ascontiguousarray(a)).cast("B")
+    for i in range(0, len(mv), 1 << 28):
+        h.update(mv[i:i + (1 << 28)])
+    return h.hexdigest()
+
+
+def _golden(key):
+    if not os.path.exists(GOLDEN):
+        pytest.fail("tests/golden/big_configs.json is missing: run tests/golden/make_big_goldens.py")
+    with open(GOLDEN) as f:
+        g = json.load(f)
+    if key not in g:
+        pytest.fail(f"{key} is missing from tests/golden/big_configs.json")
+    return g[key]
+
+
+def _against_golden(g, gold, tr, caps):
+    """Every output of the GPU run against the oracle's stored results."""
+    assert _sha(tr.tokens) == gold["tokens_sha256"] and _sha(tr.req_tok_off) == gold["req_tok_off_sha256"]
+    assert g["n_access"] == gold["N"] and g["n_distinct"] == gold["D"]
+    for k in ("ids", "prev", "next", "dist"):
+        assert _sha(g[k]) == gold[k + "_sha256"], k
+    assert [int(c) for c in caps] == gold["caps"]
+    assert g["hits"] == gold["hits"]
+    assert [str(x) for x in g["saved"]] == gold["saved"]
+    assert str(g["total_cost"]) == gold["total_cost"]
+    d = gold["direct"]
+    for idx, h, s in zip(d["index"], d["hits"], d["saved"]):
+        assert g["hits"][idx] == h and str(g["saved"][idx]) == s
+
+
+def _sessions(tr):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(tr.req_session, dtype=np.uint32).view(np.int32)).cuda()
+
+
+def _pipeline(tok, off, ts, n_tok, n_req, B, caps, ses=None, n_session=0):
     """ptc_pipeline with caller arrays for every intermediate; numpy results."""
     import torch
     import paper_2609_28870_gb300 as ptc
@@ -40,7 +86,7 @@ def _pipeline(tok, off, ts, n_tok, n_req, B, caps):
     outs = {k: torch.empty(nmax, dtype=torch.int32, device="cuda") for k in ("ids", "prev", "next", "dist")}
     outs["keys"] = torch.empty(2 * nmax, dtype=torch.int64, device="cuda")
     outs["req_blk_off"] = torch.empty(n_req + 1, dtype=torch.int64, device="cuda")
-    res = ptc.ptc_pipeline(tok, off, ts, B, caps, outputs=outs)
+    res = ptc.ptc_pipeline(tok, off, ts, B, caps, outputs=outs, req_session=ses, n_session=n_session)
     n = res["n_access"]
     for k in ("ids", "prev", "next", "dist"):
         res[k] = outs[k][:n].cpu().numpy().view(np.uint32)
@@ -146,22 +192,23 @@ def _sampled_definitions(g, tr, B, off, rng, n_samples=300, window_cap=2_000_000
 def agentic():
     tr = tracegen.make(2)
     dev = _to_gpu(tr)
+    ses = _sessions(tr)
     # D at B = 16 sets the token-denominated grid of the other block sizes
     # (the value itself is pinned by test_agentic_full_size)
     d16 = _pipeline(*dev, tr.tokens.size, tr.n_req, 16, [1])["n_distinct"]
-    return tr, dev, d16
+    return tr, dev, ses, d16
 
 
 def test_agentic_full_size(agentic):
-    """Agentic workload, B = 16, at full size: every per-access array against
-    the oracle, the curves by direct LRU simulation at two capacities and by
-    inclusion at all 64."""
-    tr, (tok, off_d, ts), d16 = agentic
+    """Agentic workload, B = 16, at full size, with and without session
+    labels: every per-access array against the oracle run here, the curves by
+    direct LRU simulation at two capacities and by inclusion at all 64."""
+    tr, (tok, off_d, ts), ses, d16 = agentic
     B = 16
     ids, D = oracle.block_ids(tr.tokens, tr.req_tok_off, B)
     assert D == d16
     caps = tracegen.workload_grid(2, D)
-    g = _pipeline(tok, off_d, ts, tr.tokens.size, tr.n_req, B, caps)
+    g = _pipeline(tok, off_d, ts, tr.tokens.size, tr.n_req, B, caps, ses, tr.n_sessions)
     assert g["n_distinct"] == D and np.array_equal(g["ids"], ids)
     prev, nxt = oracle.reuse(ids, D)
     assert np.array_equal(g["prev"], prev) and np.array_equal(g["next"], nxt)
@@ -173,50 +220,42 @@ def test_agentic_full_size(agentic):
     assert [g["hits"][p] for p in pick] == h and [g["saved"][p] for p in pick] == s
     assert g["total_cost"] == t
     _sampled_definitions(g, tr, B, off, np.random.default_rng(2), n_samples=100)
+    # without sessions (every key through the table): the same results
+    g2 = _pipeline(tok, off_d, ts, tr.tokens.size, tr.n_req, B, caps)
+    for k in ("ids", "prev", "next", "dist"):
+        assert np.array_equal(g2[k], g[k]), k
+    assert g2["hits"] == g["hits"] and g2["saved"] == g["saved"]
 
 
-@pytest.mark.parametrize("B", [32, 64, 256])
-def test_agentic_other_block_sizes_full_size(agentic, B):
-    """The agentic trace re-blocked at B = 32, 64, 256 (the block-size study)
-    with the token-denominated capacity grid: ids, prev, next and stack
-    distances against the oracle, the curves by inclusion."""
-    tr, (tok, off_d, ts), d16 = agentic
-    ids, D = oracle.block_ids(tr.tokens, tr.req_tok_off, B)
+@pytest.mark.parametrize("B", [16, 32, 64, 256])
+def test_agentic_block_sizes_against_golden(agentic, B):
+    """The agentic trace re-blocked at B = 16, 32, 64, 256 (the block-size
+    study) with the token-denominated capacity grid, against the oracle's
+    stored results: every per-access array, the curves at all grid points and
+    the direct LRU simulation at four of them."""
+    tr, (tok, off_d, ts), ses, d16 = agentic
+    gold = _golden(f"agentic_B{B}")
     # capacities in tokens: 16 x a mixed-style grid over D at B = 16, as blocks of B
     base = tracegen.capacity_grid(max(1, round(0.001 * d16)), d16, 128).astype(np.uint64)
     caps = np.unique(np.maximum(np.uint64(1), (np.uint64(16) * base) // np.uint64(B)))
-    g = _pipeline(tok, off_d, ts, tr.tokens.size, tr.n_req, B, caps)
-    assert g["n_distinct"] == D and np.array_equal(g["ids"], ids)
-    prev, nxt = oracle.reuse(ids, D)
-    assert np.array_equal(g["prev"], prev) and np.array_equal(g["next"], nxt)
-    assert np.array_equal(g["dist"], oracle.sd_fenwick(prev))
+    g = _pipeline(tok, off_d, ts, tr.tokens.size, tr.n_req, B, caps, ses, tr.n_sessions)
+    _against_golden(g, gold, tr, caps)
     _identities(g, B, caps, tr)
 
 
 def test_mixed_full_size():
-    """Mixed 24-hour workload (10.0B tokens) at full size, B = 16, 128-point
-    grid: the oracle on the first 30,000 requests must match the full run
-    there; sampled accesses against the definitions; the identities over all
-    624M accesses."""
+    """Mixed 24-hour workload (10.0B tokens, 624M accesses) at full size,
+    B = 16, 128-point grid, with session labels as the bench runs it: every
+    output against the oracle's stored results; sampled accesses against the
+    definitions; the identities over all accesses."""
     tr = tracegen.make(3)
+    gold = _golden("mixed_B16")
     tok, off_d, ts = _to_gpu(tr)
+    ses = _sessions(tr)
     B = 16
-    head = tr.head(30000)
-    ids_h, D_h = oracle.block_ids(head.tokens, head.req_tok_off, B)
-    n_h = ids_h.size
-    # the grid: the workload's 128 points over D of the full trace
-    g0 = _pipeline(tok, off_d, ts, tr.tokens.size, tr.n_req, B, [1])
-    caps = tracegen.workload_grid(3, g0["n_distinct"])
-    del g0
-    g = _pipeline(tok, off_d, ts, tr.tokens.size, tr.n_req, B, caps)
-    del tok, off_d, ts
-    assert np.array_equal(g["ids"][:n_h], ids_h)
-    prev_h, next_h = oracle.reuse(ids_h, D_h)
-    assert np.array_equal(g["prev"][:n_h], prev_h)
-    # a next use inside the prefix is the same; none there means later or none
-    inside = next_h != NONE
-    assert np.array_equal(g["next"][:n_h][inside], next_h[inside])
-    assert np.all((g["next"][:n_h][~inside] == NONE) | (g["next"][:n_h][~inside] >= n_h))
-    assert np.array_equal(g["dist"][:n_h], oracle.sd_fenwick(prev_h))
+    caps = tracegen.workload_grid(3, gold["D"])
+    g = _pipeline(tok, off_d, ts, tr.tokens.size, tr.n_req, B, caps, ses, tr.n_sessions)
+    del tok, off_d, ts, ses
+    _against_golden(g, gold, tr, caps)
     off = _identities(g, B, caps, tr)
     _sampled_definitions(g, tr, B, off, np.random.default_rng(3), n_samples=200)

@@ -131,7 +131,7 @@ def test_pipeline_rejects_bad_arguments():
     hits, saved, total = np.zeros(1, np.uint64), np.zeros(2, np.uint64), ptc.U128()
     caps = np.array([1], np.uint64)
     cm = ptc.CostModel(ptc.F_LIN, ptc.F_ATTN, ptc.PTC_COST_MEASURED)
-    rc = L.ptc_pipeline(tok.data_ptr(), 32, off.data_ptr(), ts.data_ptr(), 1, 16, 0, ctypes.byref(cm),
+    rc = L.ptc_pipeline(tok.data_ptr(), 32, off.data_ptr(), ts.data_ptr(), None, 0, 1, 16, 0, ctypes.byref(cm),
                         caps.ctypes.data, 1, None, None, None, None, None, None, ctypes.byref(n), ctypes.byref(d),
                         hits.ctypes.data, saved.ctypes.data, ctypes.byref(total), small.data_ptr(), 256,
                         torch.cuda.current_stream().cuda_stream)

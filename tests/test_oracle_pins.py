@@ -314,3 +314,39 @@ def test_prefix_hash_separates_lengths():
     keys = oracle.prefix_hash(tr.tokens, tr.req_tok_off, 2, 99)
     assert not np.array_equal(keys[0], keys[2])
     assert np.array_equal(keys[0], keys[1])
+
+
+# ---------------------------------------------------------------- curves by inclusion
+@pytest.mark.parametrize("seed", range(12))
+def test_curves_from_dist_bruteforce(seed):
+    """orc_curves_from_dist (the inclusion route the GPU takes) against the
+    plain-Python OrderedDict LRU at every capacity from 1 to D + 2, with
+    distances from window sets, under all three cost kinds."""
+    tr = tracegen.tiny(500 + seed, n_sessions=5, vocab=2)
+    B = 1 + seed % 3
+    reqs = [list(tr.tokens[int(tr.req_tok_off[r]):int(tr.req_tok_off[r + 1])]) for r in range(tr.n_req)]
+    ids, D, off = bf_ids(reqs, B)
+    sd = np.asarray(bf_sd(ids), dtype=np.uint32)
+    caps = np.arange(1, D + 3, dtype=np.uint64)
+    for kind, f_lin, f_attn in ((0, 0, 0), (1, 5, 3), (2, 0, 7)):
+        hits, saved = oracle.curves_from_dist(sd, off, B, caps, kind, f_lin, f_attn)
+        for C, h, s in zip(caps, hits, saved):
+            assert (h, s) == bf_lru(ids, off, B, int(C), kind, f_lin, f_attn)
+
+
+def test_curves_from_dist_equals_direct_lru(small_conv):
+    """On the tiny conversational workload: the inclusion route equals the
+    oracle's direct per-capacity LRU simulation (Mattson inclusion), hits and
+    128-bit compute saved, on a grid that includes capacities past D."""
+    tr, B, off, ids, D, prev, nxt, sd = small_conv
+    caps = tracegen.capacity_grid(1, D + 5, 20)
+    hits, saved, _ = oracle.lru_curves(ids, off, B, caps)
+    h2, s2 = oracle.curves_from_dist(sd, off, B, caps)
+    assert hits == h2 and saved == s2
+
+
+def test_curves_from_dist_rejects_bad_grid():
+    with pytest.raises(ValueError):
+        oracle.curves_from_dist(np.zeros(1, np.uint32), np.array([0, 1], np.uint64), 1, np.array([3, 3], np.uint64))
+    with pytest.raises(ValueError):
+        oracle.curves_from_dist(np.zeros(1, np.uint32), np.array([0, 1], np.uint64), 1, np.array([0], np.uint64))

@@ -351,7 +351,7 @@ tg_trace* tg_make(int cfg, uint64_t seed, int64_t sessions_a, int64_t sessions_b
       c.window_s = a.window_s = 86400.0;
       c.diurnal = a.diurnal = true;
       gen_conv(*tr, c, derive(root, 31), 0);
-      gen_agent(*tr, a, derive(root, 32), 1ULL << 40);
+      gen_agent(*tr, a, derive(root, 32), c.n_sessions);  // labels stay dense: 0 .. sessions - 1
       break;
     }
     default:
