@@ -612,6 +612,21 @@ def chat_extras(args, ptc, tracegen, dev, timer, slowest, peak, peak_kind, rank,
                                "ptc_curves)", "bytes_model": "8 N: prev read, dist written",
                        "hot_path_hit_ratio_at": {str(int(caps[g])): round(int(plan.hits[g]) / N, 5) for g in mid},
                        **variants}
+    # ---- Belady's offline optimum (Sec. 3.2) from the step's prev, every grid capacity
+    bws = torch.empty(L.ptc_belady_curves_workspace_bytes(N, R, G), dtype=torch.uint8, device=dev)
+    bel = ptc.ptc_belady_curves(prev_t, rbo, BLOCK, caps, ws=bws)
+    L.ptc_timer_reset()
+    L.ptc_timer_enable(1)
+    ptc.ptc_belady_curves(prev_t, rbo, BLOCK, caps, ws=bws)
+    L.ptc_timer_enable(0)
+    bel_kernels = {name: round(tot, 4) for name, _, tot in read_timer(ptc)}
+    bel_ms = slowest(sum(timer.run(args.steps, lambda: ptc.ptc_belady_curves(prev_t, rbo, BLOCK, caps, ws=bws)))) \
+        / args.steps
+    del bws
+    out["belady"] = {"call": "ptc_belady_curves on the step's prev: MIN curves at every grid capacity, one warp per "
+                             "capacity over runs of re-reads", "ms": round(bel_ms, 3), "kernels_ms": bel_kernels,
+                     "hit_ratio_at": {str(int(caps[g])): round(bel["hits"][g] / N, 5) for g in mid},
+                     "lru_hit_ratio_at": {str(int(caps[g])): round(int(plan.hits[g]) / N, 5) for g in mid}}
     if rank == 0 and ws_world == 1 and not args.no_cpu_baseline:
         # the oracle on the whole chat trace: curves, statistics and variant distances must match
         cb, orc = cpu_baseline(tr, 1.0, CHAT, keep_sd=True)
@@ -638,6 +653,16 @@ def chat_extras(args, ptc, tracegen, dev, timer, slowest, peak, peak_kind, rank,
             out["variants"][vname]["cpu_baseline"] = {
                 "value": round(N / dt, 1), "unit": "accesses/s", "cores": 1, "kind": "oracle",
                 "sample": f"orc_sd_variant (Fenwick) on the whole trace; {dt:.2f} s", "parity_with_gpu": same_v}
+        threads = os.cpu_count() or 1
+        t0 = time.perf_counter()
+        bh, bs, braw = oracle.belady_curves(orc["ids"], orc["off"], BLOCK, caps, threads=threads)
+        dt = time.perf_counter() - t0
+        same_b = bh == bel["hits"] and bs == bel["saved"] and braw == bel["raw_hits"]
+        assert same_b, "Belady curves differ from the oracle"
+        out["belady"]["cpu_baseline"] = {
+            "value": round(N / dt, 1), "unit": "accesses/s", "cores": threads, "kind": "oracle",
+            "sample": f"orc_belady_curves (direct MIN per capacity) on the whole trace, all {G} capacities; "
+                      f"{dt:.2f} s", "parity_with_gpu": same_b}
     return out
 
 
