@@ -81,6 +81,9 @@ def parse_args():
     ap.add_argument("--json-out", default=None)
     ap.add_argument("--requests", type=int, default=0,
                     help="run only the first N requests of the workload (small cases for profiling)")
+    ap.add_argument("--profile-one-step", action="store_true",
+                    help="set up, run one warm-up step, then exactly one step between cudaProfilerStart and "
+                         "cudaProfilerStop (for ncu --profile-from-start off), and exit")
     return ap.parse_args()
 
 
@@ -413,6 +416,18 @@ def run_ours(args, ws_world, rank, local):
         plan.run()
     N = plan.n.value
     ref = (plan.hits.copy(), plan.saved.copy())
+    if args.profile_one_step:
+        torch.cuda.synchronize(dev)
+        launches0 = L.ptc_launch_count()
+        torch.cuda.profiler.start()
+        plan.run()
+        torch.cuda.synchronize(dev)
+        torch.cuda.profiler.stop()
+        assert np.array_equal(plan.hits, ref[0]) and np.array_equal(plan.saved, ref[1])
+        if rank == 0:
+            print(json.dumps({"profiled_step": WORKLOAD_NAMES[W], "tokens": T, "accesses": N,
+                              "launches": L.ptc_launch_count() - launches0}), flush=True)
+        return
 
     # ---- timed region (inputs resident in HBM)
     clocks = Clocks(local)
@@ -627,6 +642,19 @@ def chat_extras(args, ptc, tracegen, dev, timer, slowest, peak, peak_kind, rank,
                              "capacity over runs of re-reads", "ms": round(bel_ms, 3), "kernels_ms": bel_kernels,
                      "hit_ratio_at": {str(int(caps[g])): round(bel["hits"][g] / N, 5) for g in mid},
                      "lru_hit_ratio_at": {str(int(caps[g])): round(int(plan.hits[g]) / N, 5) for g in mid}}
+    # ---- session-level eviction (Sec. 5.3) on the step's ids, every grid capacity
+    ses_t = ses
+    sws = torch.empty(L.ptc_session_lru_curves_workspace_bytes(D, tr.n_sessions, G), dtype=torch.uint8, device=dev)
+    ids_t = outs["ids"][:N]
+    sesc = ptc.ptc_session_lru_curves(ids_t, D, rbo, ses_t, tr.n_sessions, BLOCK, caps, ws=sws)
+    ses_ms = slowest(sum(timer.run(args.steps, lambda: ptc.ptc_session_lru_curves(
+        ids_t, D, rbo, ses_t, tr.n_sessions, BLOCK, caps, ws=sws)))) / args.steps
+    del sws
+    out["session_eviction"] = {
+        "call": "ptc_session_lru_curves on the step's ids: session-level LRU at every grid capacity, one warp per "
+                "capacity", "ms": round(ses_ms, 3),
+        "hit_ratio_at": {str(int(caps[g])): round(sesc["hits"][g] / N, 5) for g in mid},
+        "block_level_hit_ratio_at": {str(int(caps[g])): round(int(plan.hits[g]) / N, 5) for g in mid}}
     if rank == 0 and ws_world == 1 and not args.no_cpu_baseline:
         # the oracle on the whole chat trace: curves, statistics and variant distances must match
         cb, orc = cpu_baseline(tr, 1.0, CHAT, keep_sd=True)
@@ -659,6 +687,16 @@ def chat_extras(args, ptc, tracegen, dev, timer, slowest, peak, peak_kind, rank,
         dt = time.perf_counter() - t0
         same_b = bh == bel["hits"] and bs == bel["saved"] and braw == bel["raw_hits"]
         assert same_b, "Belady curves differ from the oracle"
+        t0 = time.perf_counter()
+        sh_, ss_ = oracle.session_lru_curves(orc["ids"], orc["off"], tr.req_session.astype(np.uint32), tr.n_sessions,
+                                             BLOCK, caps, threads=threads)
+        dts = time.perf_counter() - t0
+        same_s = sh_ == sesc["hits"] and ss_ == sesc["saved"]
+        assert same_s, "session-level curves differ from the oracle"
+        out["session_eviction"]["cpu_baseline"] = {
+            "value": round(N / dts, 1), "unit": "accesses/s", "cores": threads, "kind": "oracle",
+            "sample": f"orc_session_lru_curves (direct simulation per capacity) on the whole trace, all {G} "
+                      f"capacities; {dts:.2f} s", "parity_with_gpu": same_s}
         out["belady"]["cpu_baseline"] = {
             "value": round(N / dt, 1), "unit": "accesses/s", "cores": threads, "kind": "oracle",
             "sample": f"orc_belady_curves (direct MIN per capacity) on the whole trace, all {G} capacities; "

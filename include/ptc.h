@@ -13,6 +13,8 @@
  *     -> ptc_curves          hits and compute saved per C      Sec. 3.2 (hit ratio), Sec. 5.2 (compute savings)
  *   with Belady's offline optimum from the same reuse indices,
  *        ptc_belady_curves                                     Sec. 3.2 (offline ceiling)
+ *   and session-level instead of block-level eviction,
+ *        ptc_session_lru_curves                                Sec. 5.3 (eviction granularity)
  *   with, for the semantics variants (touch order, whole-request residency),
  *        ptc_stack_distance_variant                           Sec. 3.1 (simulator)
  *   and, over the same arrays,
@@ -22,9 +24,18 @@
  *
  * Conventions shared by every call
  *   - Pointers are caller-owned DEVICE memory unless the name ends in _host.
- *     The library allocates nothing: each call takes a device workspace `ws`
- *     of at least ptc_<call>_workspace_bytes(...) bytes, 256-byte aligned.
- *     The workspace holds no state between calls.
+ *     The library allocates no device memory: each call takes a device
+ *     workspace `ws` of at least ptc_<call>_workspace_bytes(...) bytes,
+ *     256-byte aligned.  The workspace holds no state between calls.
+ *   - Host staging: the first call made by a host thread allocates one small
+ *     page-locked, device-mapped block for that thread (cudaHostAlloc, about
+ *     110 KB), through which status words and results reach the host without
+ *     a copy-engine transfer.  It lives until ptc_release_host_staging() is
+ *     called on that thread (the next call allocates it again).  Like any
+ *     cudaHostAlloc, that first allocation may synchronize the device, so a
+ *     serving loop should make one call before it starts.  If page-locked
+ *     memory cannot be had, ordinary thread-local memory is used instead.
+ *     ptc_curves_noalloc never allocates it.
  *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Work is
  *     enqueued on it.  Every call returns after reading its device status
  *     word, so it synchronizes `stream` once before returning; outputs are
@@ -62,7 +73,8 @@ typedef enum {
   PTC_ERR_CUDA = 5,           /* a CUDA runtime call failed */
   PTC_ERR_TIMEOUT = 6,        /* a device-side wait gave up (bounded spin); no result */
   PTC_ERR_HASH_COLLISION = 7, /* ptc_verify_ids found two different prefixes under one id */
-  PTC_ERR_NOT_IMPLEMENTED = 8
+  PTC_ERR_NOT_IMPLEMENTED = 8,
+  PTC_ERR_BOUNDS = 9          /* checked build only: an index read from data fell outside its array */
 } ptc_status;
 
 /* Unsigned 128-bit integer, little-endian halves. */
@@ -372,6 +384,35 @@ ptc_status ptc_belady_curves(const uint32_t* prev, uint64_t n, const uint64_t* r
                              size_t ws_bytes, void* stream);
 
 /*
+ * ptc_session_lru_curves — session-level LRU eviction (Sec. 5.3: evicting
+ * whole sessions instead of blocks, the eviction-granularity study) at every
+ * capacity of the grid, with the prefix rule and cost model of ptc_curves.
+ * Rules (the paper states none; these are this library's reading):
+ *   - a block belongs to the session whose request brought it into the cache
+ *     until it is evicted; hits by other sessions do not change that, so
+ *     evicting a session also drops shared prompts it brought in;
+ *   - sessions are ordered by the arrival of their latest request (a session
+ *     is touched when its request arrives, before its blocks);
+ *   - while more than C blocks are resident, every block of the least
+ *     recently touched session other than the current one is evicted;
+ *   - a session that alone holds more than C blocks keeps only the block
+ *     just brought in.
+ * Not a stack algorithm: each capacity is replayed on its own (one warp per
+ * capacity), so the time grows with n, not with the number of runs.
+ *   ids          u32[n] from ptc_assign_ids, each below n_distinct
+ *   req_session  u32[n_req] labels below n_session
+ *   req_blk_off, n_req, block_size, cm, cap_host, n_cap, hits/saved  as ptc_curves
+ * Workspace: ptc_session_lru_curves_workspace_bytes (n_cap x n_distinct x 8
+ * bytes for block ownership, plus per-session state).
+ */
+size_t ptc_session_lru_curves_workspace_bytes(uint64_t n_distinct, uint32_t n_session, uint32_t n_cap);
+ptc_status ptc_session_lru_curves(const uint32_t* ids, uint64_t n, uint64_t n_distinct, const uint64_t* req_blk_off,
+                                  const uint32_t* req_session, uint32_t n_req, uint32_t n_session,
+                                  uint32_t block_size, const ptc_cost_model* cm, const uint64_t* cap_host,
+                                  uint32_t n_cap, uint64_t* hits_host_out, ptc_u128* saved_host_out, void* ws,
+                                  size_t ws_bytes, void* stream);
+
+/*
  * ptc_pipeline — the five calls in order (hash, ids, reuse, stack distance,
  * curves) in one call, for a trace already on the device.  Semantics, limits
  * and errors are those of the individual calls; the first error stops the
@@ -510,7 +551,10 @@ ptc_status ptc_trace_stats(const uint32_t* ids, const uint32_t* prev, const uint
  *     PTC_MAX_CAPACITIES.
  *   - The first call on each device looks up the array's device address
  *     (cudaGetSymbolAddress) with that device current; make that first call
- *     before any stream capture.
+ *     before any stream capture.  The address is kept for the life of the
+ *     process: after cudaDeviceReset on a device (which unloads the
+ *     library's device code there) do not call this entry point on that
+ *     device again in the same process.
  *   - Every call on a device shares the one array, and each call leaves its
  *     contents behind (the next call re-zeroes what must start at zero).
  *     Calls whose work overlaps on the GPU (for example on two streams) race
@@ -521,6 +565,23 @@ ptc_status ptc_curves_noalloc(const uint32_t* dist, uint64_t n, const uint64_t* 
                               uint32_t block_size, const ptc_cost_model* cm, const uint64_t* cap_host,
                               uint32_t n_cap, uint64_t* hits_host_out, ptc_u128* saved_host_out,
                               ptc_u128* total_cost_host_out, void* stream);
+
+/* Frees the calling thread's page-locked staging block (see the
+ * conventions above); safe to call at any time between calls. */
+void ptc_release_host_staging(void);
+
+/*
+ * ptc_test_wait_polls — test hook for the bounded waits (no counterpart in
+ * the paper: failure detection).  Kernels that wait on other CTAs (the
+ * decoupled look-back of stage a1's block offsets) poll a bounded number of
+ * times and then give up with PTC_ERR_TIMEOUT instead of hanging.  With
+ * polls > 0, every later ptc_hash_blocks / ptc_pipeline call in the process
+ * makes those waits see no predecessor as ready (a flag that nothing sets)
+ * and give up after `polls` polls, so a test can drive the give-up path: the
+ * call must return PTC_ERR_TIMEOUT and leave the device usable.  polls = 0
+ * restores normal waits.  Process-wide; not for production use.
+ */
+void ptc_test_wait_polls(uint32_t polls);
 
 /*
  * Measurement hooks (no counterpart in the paper: instrumentation for the

@@ -19,6 +19,8 @@ Functions and the passages they restate:
   inclusion (App. B).
 * ``belady_curves`` — Belady's offline optimum (Sec. 3.2): direct MIN
   simulation per capacity, same prefix rule and costs.
+* ``session_lru_curves`` — session-level LRU eviction (Sec. 5.3): direct
+  simulation per capacity, evicting the least recent session's blocks whole.
 * ``lru_curves_variant``, ``sd_variant`` — Sec. 3.1: leaf-first touch order
   and whole-request residency (every block looked up at the request's
   arrival), by direct LRU per capacity, Fenwick counting and Mattson's list.
@@ -83,6 +85,8 @@ def _load():
         lib.orc_lru_curves.restype = i32
         lib.orc_lru_curves.argtypes = [vp, vp, u32, u32, i32, u64, u64, vp, u32, i32, vp, vp, vp, vp, vp]
         lib.orc_prefix_hash.argtypes = [vp, vp, u32, u32, u64, vp]
+        lib.orc_session_lru_curves.restype = i32
+        lib.orc_session_lru_curves.argtypes = [vp, vp, vp, u32, u32, u32, i32, u64, u64, vp, u32, i32, vp, vp, vp]
         lib.orc_belady_curves.restype = i32
         lib.orc_belady_curves.argtypes = [vp, vp, u32, u32, i32, u64, u64, vp, u32, i32, vp, vp, vp, vp]
         lib.orc_curves_from_dist.restype = i32
@@ -163,6 +167,27 @@ def lru_curves(ids, req_blk_off, B: int, caps, kind: int = COST_MEASURED, f_lin:
         raise ValueError("bad capacity grid (capacities must be >= 1)")
     saved = [int(h) << 64 | int(l) for l, h in zip(slo, shi)]
     return [int(h) for h in hits], saved, int(thi[0]) << 64 | int(tlo[0])
+
+
+def session_lru_curves(ids, req_blk_off, req_session, n_session: int, B: int, caps, kind: int = COST_MEASURED,
+                       f_lin: int = F_LIN, f_attn: int = F_ATTN, threads: int | None = None):
+    """Session-level LRU (Sec. 5.3) simulated directly at each capacity: a
+    block belongs to the session that brought it in; the least recently
+    touched other session is evicted whole while more than C blocks are
+    resident; a session alone above C keeps only the block just brought in.
+    Prefix rule and costs as lru_curves.  Returns (hits, saved)."""
+    ids, bo, caps = _c(ids, np.uint32), _c(req_blk_off, np.uint64), _c(caps, np.uint64)
+    ses = _c(req_session, np.uint32)
+    G = caps.shape[0]
+    hits = np.zeros(G, dtype=np.uint64)
+    slo = np.zeros(G, dtype=np.uint64)
+    shi = np.zeros(G, dtype=np.uint64)
+    nthreads = threads or max(1, min(G, os.cpu_count() or 1))
+    rc = _load().orc_session_lru_curves(_p(ids), _p(bo), _p(ses), bo.shape[0] - 1, int(n_session), int(B), int(kind),
+                                        int(f_lin), int(f_attn), _p(caps), G, nthreads, _p(hits), _p(slo), _p(shi))
+    if rc != 0:
+        raise ValueError("bad capacity grid or session label")
+    return [int(h) for h in hits], [int(h) << 64 | int(l) for l, h in zip(slo, shi)]
 
 
 def belady_curves(ids, req_blk_off, B: int, caps, kind: int = COST_MEASURED, f_lin: int = F_LIN,

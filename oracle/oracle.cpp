@@ -23,6 +23,9 @@
 //        orc_sd_fenwick (Bennett & Kruskal 1975 counting), two independent ways.
 //   * Belady's next use (Sec. 3.2, 5.2).  -> orc_reuse: previous and next
 //     access of the same block.
+//   * Sec. 5.3: session-level instead of block-level eviction.
+//     -> orc_session_lru_curves: one direct simulation per capacity that evicts
+//        the least recently touched session's blocks together.
 //   * Sec. 3.2: Belady's optimum as the offline ceiling.  -> orc_belady_curves:
 //     one direct MIN simulation (evict the farthest next access) per capacity,
 //     with the same prefix rule as the LRU curves.
@@ -358,6 +361,94 @@ int orc_belady_curves(const uint32_t* ids, const uint64_t* req_blk_off, uint32_t
       }
       hits[g] = h;
       raw_hits[g] = raw;
+      saved_lo[g] = (uint64_t)saved;
+      saved_hi[g] = (uint64_t)(saved >> 64);
+    }
+  };
+  if (threads < 1) threads = 1;
+  std::vector<std::thread> pool;
+  for (int t = 1; t < threads; ++t) pool.emplace_back(simulate);
+  simulate();
+  for (auto& th : pool) th.join();
+  return 0;
+}
+
+// Session-level LRU eviction (Sec. 5.3: evicting whole sessions instead of
+// blocks), one capacity at a time.  Readings (the paper gives no rules):
+//   * a block brought in by a request belongs to that request's session until
+//     it is evicted, even when other sessions hit it later (so evicting a
+//     session also drops the shared prompts it brought in, as Sec. 5.3 notes);
+//   * sessions are ordered by the arrival of their latest request; a session
+//     is touched when its request arrives, before its blocks;
+//   * a miss brings the block in; while more than C blocks are resident, all
+//     blocks of the least recently touched session other than the current
+//     one are evicted;
+//   * if the current session is then the only one holding blocks and the
+//     cache still holds more than C, all its blocks except the one just
+//     brought in are evicted (a session larger than the cache restarts).
+// Block k of a request counts as a hit iff blocks 0..k of that request were
+// all resident (Sec. 2.2 prefix reuse); costs as in orc_lru_curves.
+// req_session[r] < n_session.  Returns 0, or -1 on a bad argument.
+int orc_session_lru_curves(const uint32_t* ids, const uint64_t* req_blk_off, const uint32_t* req_session,
+                           uint32_t n_req, uint32_t n_session, uint32_t B, int kind, uint64_t f_lin, uint64_t f_attn,
+                           const uint64_t* caps, uint32_t G, int threads, uint64_t* hits, uint64_t* saved_lo,
+                           uint64_t* saved_hi) {
+  for (uint32_t g = 0; g < G; ++g)
+    if (caps[g] == 0) return -1;
+  for (uint32_t r = 0; r < n_req; ++r)
+    if (req_session[r] >= n_session) return -1;
+  std::atomic<uint32_t> next_cap{0};
+  auto simulate = [&]() {
+    for (;;) {
+      uint32_t g = next_cap.fetch_add(1);
+      if (g >= G) return;
+      uint64_t C = caps[g];
+      std::unordered_map<uint32_t, uint32_t> owner;     // resident block -> its session
+      std::vector<std::vector<uint32_t>> owned(n_session);  // each session's resident blocks
+      std::list<uint32_t> order;                        // sessions, most recently touched first
+      std::vector<std::list<uint32_t>::iterator> pos(n_session, order.end());
+      uint64_t total = 0, h = 0;
+      u128 saved = 0;
+      for (uint32_t r = 0; r < n_req; ++r) {
+        uint32_t s = req_session[r];
+        if (pos[s] != order.end()) order.erase(pos[s]);
+        order.push_front(s);
+        pos[s] = order.begin();
+        bool prefix_ok = true;
+        for (uint64_t k = 0; k < req_blk_off[r + 1] - req_blk_off[r]; ++k) {
+          uint32_t id = ids[req_blk_off[r] + k];
+          bool resident = owner.count(id) != 0;
+          if (!resident) {
+            owner[id] = s;
+            owned[s].push_back(id);
+            ++total;
+            while (total > C) {
+              uint32_t victim = s;
+              for (auto it = order.rbegin(); it != order.rend(); ++it)
+                if (*it != s && !owned[*it].empty()) {
+                  victim = *it;
+                  break;
+                }
+              if (victim != s) {
+                for (uint32_t b : owned[victim]) owner.erase(b);
+                total -= owned[victim].size();
+                owned[victim].clear();
+              } else {  // only the current session holds blocks
+                for (uint32_t b : owned[s])
+                  if (b != id) owner.erase(b);
+                total = 1;
+                owned[s].assign(1, id);
+              }
+            }
+          }
+          prefix_ok = prefix_ok && resident;
+          if (prefix_ok) {
+            ++h;
+            saved += cost_of(k, B, kind, f_lin, f_attn);
+          }
+        }
+      }
+      hits[g] = h;
       saved_lo[g] = (uint64_t)saved;
       saved_hi[g] = (uint64_t)(saved >> 64);
     }

@@ -44,7 +44,7 @@ _lib = None
 STATUS = {
     0: "PTC_OK", 1: "PTC_ERR_INVALID_ARG", 2: "PTC_ERR_UNSORTED", 3: "PTC_ERR_OVERFLOW",
     4: "PTC_ERR_WORKSPACE", 5: "PTC_ERR_CUDA", 6: "PTC_ERR_TIMEOUT", 7: "PTC_ERR_HASH_COLLISION",
-    8: "PTC_ERR_NOT_IMPLEMENTED",
+    8: "PTC_ERR_NOT_IMPLEMENTED", 9: "PTC_ERR_BOUNDS",
 }
 
 
@@ -63,8 +63,22 @@ class U128(ctypes.Structure):
     _fields_ = [("lo", ctypes.c_uint64), ("hi", ctypes.c_uint64)]
 
 
+_lib_path = None
+
+
 def library_path() -> str:
-    return _build.LIB
+    return _lib_path or _build.LIB
+
+
+def use_checked_build() -> str:
+    """Load the checked build (``build(checked=True)``: every index read from
+    data is checked, PTC_ERR_BOUNDS on a miss) instead of the normal one.  Must
+    come before the first call into the library in this process."""
+    global _lib_path
+    if _lib is not None:
+        raise RuntimeError("the library is already loaded in this process")
+    _lib_path = _build.LIB_CHECKED
+    return _lib_path
 
 
 def lib():
@@ -73,7 +87,7 @@ def lib():
     if _lib is None:
         with _lock:
             if _lib is None:
-                path = _build.LIB
+                path = library_path()
                 if not os.path.exists(path):
                     raise RuntimeError(f"libptc.so is not built ({path}); run "
                                        "`python -c 'import __graft_entry__ as g; g.build()'`")
@@ -135,6 +149,11 @@ def lib():
                                                 vp, u32,
                                                 ctypes.POINTER(u64), ctypes.POINTER(u64), vp, vp, ctypes.POINTER(U128),
                                                 vp, sz, vp]
+                L.ptc_session_lru_curves_workspace_bytes.restype = sz
+                L.ptc_session_lru_curves_workspace_bytes.argtypes = [u64, u32, u32]
+                L.ptc_session_lru_curves.restype = st
+                L.ptc_session_lru_curves.argtypes = [vp, u64, u64, vp, vp, u32, u32, u32, ctypes.POINTER(CostModel),
+                                                     vp, u32, vp, vp, vp, sz, vp]
                 L.ptc_belady_curves_workspace_bytes.restype = sz
                 L.ptc_belady_curves_workspace_bytes.argtypes = [u64, u32, u32]
                 L.ptc_belady_curves.restype = st
@@ -160,6 +179,10 @@ def lib():
                 L.ptc_trace_stats.restype = st
                 L.ptc_trace_stats.argtypes = [vp, vp, vp, vp, u64, u64, vp, vp, vp, u32, u32, vp, u32, vp, vp, vp,
                                               sz, vp]
+                L.ptc_release_host_staging.restype = None
+                L.ptc_release_host_staging.argtypes = []
+                L.ptc_test_wait_polls.restype = None
+                L.ptc_test_wait_polls.argtypes = [u32]
                 L.ptc_timer_enable.restype = None
                 L.ptc_timer_enable.argtypes = [ctypes.c_int]
                 L.ptc_timer_reset.restype = None
@@ -280,6 +303,27 @@ def ptc_belady_curves(prev: torch.Tensor, req_blk_off: torch.Tensor, block_size:
                                  _stream(dev))
     _check("ptc_belady_curves", rc)
     return {"hits": [int(h) for h in hits], "raw_hits": [int(x) for x in raw],
+            "saved": [int(saved[2 * g + 1]) << 64 | int(saved[2 * g]) for g in range(G)]}
+
+
+def ptc_session_lru_curves(ids: torch.Tensor, n_distinct: int, req_blk_off: torch.Tensor, req_session: torch.Tensor,
+                           n_session: int, block_size: int, caps, kind: int = PTC_COST_MEASURED, f_lin: int = F_LIN,
+                           f_attn: int = F_ATTN, ws: torch.Tensor | None = None) -> dict:
+    """Session-level LRU curves.  Returns hits and saved (Python ints, exact)."""
+    dev = _dev(req_blk_off)
+    n = ids.numel()
+    R = req_blk_off.numel() - 1
+    caps = np.ascontiguousarray(caps, dtype=np.uint64)
+    G = caps.shape[0]
+    w = _workspace(lib().ptc_session_lru_curves_workspace_bytes(n_distinct, n_session, G), dev, ws)
+    hits = np.zeros(G, dtype=np.uint64)
+    saved = np.zeros(2 * G, dtype=np.uint64)
+    cm = CostModel(int(f_lin), int(f_attn), int(kind))
+    rc = lib().ptc_session_lru_curves(_ptr(ids), n, int(n_distinct), _ptr(req_blk_off), _ptr(req_session), R,
+                                      int(n_session), block_size, ctypes.byref(cm), caps.ctypes.data, G,
+                                      hits.ctypes.data, saved.ctypes.data, _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_session_lru_curves", rc)
+    return {"hits": [int(h) for h in hits],
             "saved": [int(saved[2 * g + 1]) << 64 | int(saved[2 * g]) for g in range(G)]}
 
 

@@ -84,9 +84,17 @@ thread_local bool t_no_host_alloc = false;
 NoHostAlloc::NoHostAlloc() : prev(t_no_host_alloc) { t_no_host_alloc = true; }
 NoHostAlloc::~NoHostAlloc() { t_no_host_alloc = prev; }
 
+namespace {
+thread_local HostStage* t_pinned = nullptr;
+thread_local HostStage t_fallback;
+}  // namespace
+
+// The calling thread's staging block: page-locked and mapped, allocated on
+// the thread's first call (ptc_release_host_staging frees it), or ordinary
+// thread-local memory when page-locked memory cannot be had.
 HostStage* host_stage() {
-  static thread_local HostStage* pinned = nullptr;
-  static thread_local HostStage fallback;
+  HostStage*& pinned = t_pinned;
+  HostStage& fallback = t_fallback;
   if (!pinned) {
     fallback.dev = nullptr;
     if (t_no_host_alloc) return &fallback;
@@ -349,8 +357,31 @@ extern "C" const char* ptc_strerror(ptc_status s) {
     case PTC_ERR_TIMEOUT: return "a bounded device-side wait gave up";
     case PTC_ERR_HASH_COLLISION: return "two different prefixes share one block id";
     case PTC_ERR_NOT_IMPLEMENTED: return "not implemented";
+    case PTC_ERR_BOUNDS: return "checked build: an index read from data fell outside its array";
   }
   return "unknown status";
 }
 
+#ifdef PTC_CHECKED
+extern "C" const char* ptc_version(void) { return "ptc 0.1.0 (sm_103a, checked)"; }
+#else
 extern "C" const char* ptc_version(void) { return "ptc 0.1.0 (sm_103a)"; }
+#endif
+
+namespace {
+std::atomic<uint32_t> g_wait_polls{0};
+}  // namespace
+
+uint32_t ptc::test_wait_polls() { return g_wait_polls.load(std::memory_order_relaxed); }
+
+void ptc::release_host_stage() {
+  if (t_pinned && t_pinned != &t_fallback) {
+    (void)cudaFreeHost(t_pinned);
+    (void)cudaGetLastError();
+  }
+  t_pinned = nullptr;
+}
+
+extern "C" void ptc_release_host_staging(void) { ptc::release_host_stage(); }
+
+extern "C" void ptc_test_wait_polls(uint32_t polls) { g_wait_polls.store(polls, std::memory_order_relaxed); }

@@ -27,8 +27,9 @@
 // run with gap < L is cut into pieces of length gap, which meet that case.
 //
 // One warp simulates one capacity: the free times are a bitmap over access
-// positions with two summary levels (a bit per word that may be nonzero,
-// kept as a superset and cleaned while searching); runs go in order, up to
+// positions with three summary levels (a bit per nonzero word, kept exact as
+// words fill and empty) and a lower bound on the smallest free time, so a run
+// with nothing free below p learns it at once; runs go in order, up to
 // 1024 steps at a time, one 32-step word per lane.  Hits count with the
 // prefix rule (Sec. 2.2): a request's accesses before its first miss.
 #include "ptc_internal.h"
@@ -107,25 +108,43 @@ struct BelArgs {
   const uint32_t* rec_p;
   const uint8_t* rec_rs;
   const uint64_t* nruns;
-  uint32_t *lv0, *lv1, *lv2;  // free-time bitmap and its summaries, one slice per capacity
-  uint64_t s0, s1, s2;        // words per slice
+  uint32_t *lv0, *lv1, *lv2, *lv3;  // free-time bitmap and its summaries, one slice per capacity
+  uint64_t s0, s1, s2, s3;          // words per slice
   uint32_t G;
   uint64_t alpha, beta;
   uint64_t* out;  // hits[G] | saved[G] (lo, hi) | raw hits[G]
+  const DevStatus* st;
 };
 
-// One capacity's free-time bitmap.
+// One capacity's free-time bitmap: level 0 one bit per access position,
+// level k + 1 one bit per nonzero word of level k.  `low` is a lower bound on
+// every set position (raised when a search finds nothing below a point).
 struct FreeBits {
-  uint32_t *l0, *l1, *l2;
+  uint32_t *l0, *l1, *l2, *l3;
+  uint64_t low;
+  uint64_t words;     // level-0 words of the slice
+  const DevStatus* st;
 
   __device__ void set_word(uint64_t w, uint32_t m) {
-    if (!m) return;
+    if (!m || !in_bounds(st, w, words)) return;
     atomicOr(&l0[w], m);
     atomicOr(&l1[w >> 5], 1u << (w & 31));
     atomicOr(&l2[w >> 10], 1u << ((w >> 5) & 31));
+    atomicOr(&l3[w >> 15], 1u << ((w >> 10) & 31));
   }
+  // Clear bits m of word w; a word that becomes empty clears its summary
+  // bit, and an emptied summary word its bit above (sets and clears of one
+  // warp never overlap, so exactly one lane sees each word empty out).
   __device__ void clear_word(uint64_t w, uint32_t m) {
-    if (m) atomicAnd(&l0[w], ~m);
+    if (!m || !in_bounds(st, w, words)) return;
+    const uint32_t old = atomicAnd(&l0[w], ~m);
+    if (old == 0 || (old & ~m) != 0) return;
+    const uint32_t b1 = 1u << (w & 31);
+    const uint32_t o1 = atomicAnd(&l1[w >> 5], ~b1);
+    if (o1 == 0 || (o1 & ~b1) != 0) return;
+    const uint32_t b2 = 1u << ((w >> 5) & 31);
+    const uint32_t o2 = atomicAnd(&l2[w >> 10], ~b2);
+    if (o2 != 0 && (o2 & ~b2) == 0) atomicAnd(&l3[w >> 15], ~(1u << ((w >> 10) & 31)));
   }
   // The highest set bit in words below w0, or -1.  Summary bits of words
   // found empty are cleared on the way.
@@ -144,10 +163,17 @@ struct FreeBits {
       uint64_t w2 = w1 >> 5;
       uint32_t m2 = __ldcg(&l2[w2]) & mask_lt((uint32_t)(w1 & 31));
       for (;;) {
-        while (!m2) {
-          if (w2 == 0) return -1;
-          --w2;
+        while (!m2) {  // the next nonzero level-2 word below w2, through level 3
+          uint64_t w3 = w2 >> 5;
+          uint32_t m3 = __ldcg(&l3[w3]) & mask_lt((uint32_t)(w2 & 31));
+          while (!m3) {
+            if (w3 == 0) return -1;
+            --w3;
+            m3 = __ldcg(&l3[w3]);
+          }
+          w2 = w3 * 32 + hi_bit(m3);
           m2 = __ldcg(&l2[w2]);
+          if (!m2) atomicAnd(&l3[w3], ~(1u << (w2 & 31)));
         }
         const uint32_t b2 = hi_bit(m2);
         const uint64_t c1 = w2 * 32 + b2;
@@ -166,13 +192,16 @@ struct FreeBits {
   // there were (fewer if the bitmap runs out).
   __device__ uint32_t pop_below(uint64_t pos, uint32_t need) {
     uint32_t got = 0;
-    while (got < need && pos > 0) {
+    while (got < need && pos > low) {
       const uint64_t w = (pos - 1) >> 5;
       uint32_t v = __ldcg(&l0[w]) & mask_le((uint32_t)((pos - 1) & 31));
       uint64_t ww = w;
       if (!v) {
         const int64_t b = below_word(w);
-        if (b < 0) break;
+        if (b < 0) {  // nothing set below pos (and appends only go above p0)
+          low = low > pos ? low : pos;
+          break;
+        }
         ww = (uint64_t)b >> 5;
         v = __ldcg(&l0[ww]);
       }
@@ -203,7 +232,7 @@ __global__ void __launch_bounds__(32) k_bel_sim(BelArgs a, BelCaps caps) {
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t g = blockIdx.x;
   if (g >= a.G) return;
-  FreeBits fb{a.lv0 + g * a.s0, a.lv1 + g * a.s1, a.lv2 + g * a.s2};
+  FreeBits fb{a.lv0 + g * a.s0, a.lv1 + g * a.s1, a.lv2 + g * a.s2, a.lv3 + g * a.s3, 0, a.s0, a.st};
   uint64_t free_inf = caps.c[g] - 1;  // never-used tracks (lane 0's copy is the one used)
   uint64_t hits = 0, raw = 0, sv_lo = 0, sv_hi = 0;
   uint32_t req_start = 0;
@@ -248,7 +277,7 @@ __global__ void __launch_bounds__(32) k_bel_sim(BelArgs a, BelCaps caps) {
         const uint64_t q = (uint64_t)p + k0, w = q >> 5;
         const uint32_t sh = (uint32_t)(q & 31);
         uint32_t Bk = 0;
-        if (valid) {
+        if (valid && in_bounds(a.st, w + (sh ? 1 : 0), a.s0)) {
           const uint32_t lo = __ldcg(&fb.l0[w]);
           const uint32_t hi = sh ? __ldcg(&fb.l0[w + 1]) : 0u;
           Bk = (sh ? (lo >> sh) | (hi << (32 - sh)) : lo) & valid;
@@ -340,8 +369,8 @@ struct BelLayout {
   uint64_t* nruns;
   uint32_t *rec_start, *rec_p;
   uint8_t* rec_rs;
-  uint32_t *lv0, *lv1, *lv2;
-  uint64_t s0, s1, s2;
+  uint32_t *lv0, *lv1, *lv2, *lv3;
+  uint64_t s0, s1, s2, s3;
   uint64_t* out;
   size_t zero_bytes, bits_bytes;
   uint32_t nwords;
@@ -369,10 +398,12 @@ BelLayout bel_layout(void* ws, uint64_t n, uint32_t n_cap) {
   L.s0 = (uint64_t)L.nwords + 2;
   L.s1 = (L.s0 + 31) / 32 + 1;
   L.s2 = (L.s1 + 31) / 32 + 1;
-  L.lv0 = cv.take<uint32_t>((L.s0 + L.s1 + L.s2) * G);
+  L.s3 = (L.s2 + 31) / 32 + 1;
+  L.lv0 = cv.take<uint32_t>((L.s0 + L.s1 + L.s2 + L.s3) * G);
   L.lv1 = L.lv0 + L.s0 * G;
   L.lv2 = L.lv1 + L.s1 * G;
-  L.bits_bytes = sizeof(uint32_t) * (L.s0 + L.s1 + L.s2) * G;
+  L.lv3 = L.lv2 + L.s2 * G;
+  L.bits_bytes = sizeof(uint32_t) * (L.s0 + L.s1 + L.s2 + L.s3) * G;
   L.out = cv.take<uint64_t>(4 * G);
   L.total = cv.bytes();
   return L;
@@ -431,13 +462,16 @@ extern "C" ptc_status ptc_belady_curves(const uint32_t* prev, uint64_t n, const 
   a.lv0 = L.lv0;
   a.lv1 = L.lv1;
   a.lv2 = L.lv2;
+  a.lv3 = L.lv3;
   a.s0 = L.s0;
   a.s1 = L.s1;
   a.s2 = L.s2;
+  a.s3 = L.s3;
   a.G = n_cap;
   a.alpha = alpha;
   a.beta = beta;
   a.out = L.out;
+  a.st = L.st;
   BelCaps caps;
   for (uint32_t g = 0; g < n_cap; ++g) caps.c[g] = cap_host[g];
   PTC_KERNEL("k_bel_sim", s, k_bel_sim, n_cap, 32, 0, a, caps);

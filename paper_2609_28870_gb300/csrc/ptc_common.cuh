@@ -28,13 +28,17 @@ enum : uint32_t {
   kErrOverflow = 8u,
   kErrCollision = 16u,
   kErrTableFull = 32u,
+  kErrBounds = 64u,  // the checked build caught an index outside its array
 };
 
 constexpr int kMaxEpochs = 64;
 
 struct DevStatus {
   uint32_t err;
-  uint32_t pad0;
+  // 0 normally.  Otherwise a test has asked the look-back waits of this call
+  // to see no predecessor as ready (a flag nothing sets) and to give up after
+  // this many polls: the bounded-wait path, forced (ptc_test_wait_polls).
+  uint32_t wait_test;
   uint64_t value[8];              // per-call results (N, D, max depth ...)
   uint32_t tile_ctr[kMaxEpochs];  // dynamic tile counter of each launch
 };
@@ -45,6 +49,24 @@ constexpr size_t kStatusBytes = 512;
 constexpr uint32_t kSpinCap = 1u << 20;
 
 __device__ __forceinline__ void raise_err(DevStatus* st, uint32_t f) { atomicOr(&st->err, f); }
+
+// The checked build (compiled with -DPTC_CHECKED; paper_2609_28870_gb300
+// build(checked=True)): an index that comes from data another stage or the
+// caller wrote is checked before it is used; a failed check raises
+// kErrBounds in the call's status word (PTC_ERR_BOUNDS) and the access is
+// skipped, never trapped.  In the normal build the check compiles away.
+__device__ __forceinline__ bool in_bounds(const DevStatus* st, uint64_t i, uint64_t bound) {
+#ifdef PTC_CHECKED
+  if (i < bound) return true;
+  atomicOr(const_cast<uint32_t*>(&st->err), kErrBounds);
+  return false;
+#else
+  (void)st;
+  (void)i;
+  (void)bound;
+  return true;
+#endif
+}
 
 // Programmatic dependent launch.  Kernels are launched so that the next one
 // on the stream is set up while the previous one is still running; every
@@ -165,138 +187,15 @@ __device__ inline uint32_t cta_tiles_prefix(const uint32_t* cnt, uint32_t* pre, 
 }
 
 // ---------------------------------------------------------------------------
-// Packed look-back for sums below 2^56: word = epoch(6) | flag(2) | value(56).
-// flag 1 = aggregate, 2 = inclusive prefix.  Called by all 32 lanes of ONE
-// warp; returns the exclusive prefix of `tile` (0 if the wait gave up, with
-// kErrTimeout raised).
+// Packed look-back words for sums below 2^56: epoch(6) | flag(2) | value(56);
+// flag 1 = aggregate, 2 = inclusive prefix.
 // ---------------------------------------------------------------------------
 constexpr uint64_t kLbValMask = (1ULL << 56) - 1;
 __device__ __forceinline__ uint64_t lb_pack(uint32_t epoch, uint32_t flag, uint64_t v) {
   return ((uint64_t)epoch << 58) | ((uint64_t)flag << 56) | (v & kLbValMask);
 }
 
-__device__ inline uint64_t lookback_sum(uint64_t* words, uint32_t tile, uint64_t agg, uint32_t epoch,
-                                        DevStatus* st) {
-  const uint32_t lane = threadIdx.x & 31;
-  if (tile == 0) {
-    if (lane == 0) st_relaxed_u64(&words[0], lb_pack(epoch, 2, agg));
-    return 0;
-  }
-  if (lane == 0) st_relaxed_u64(&words[tile], lb_pack(epoch, 1, agg));
-  uint64_t excl = 0;
-  int64_t base = (int64_t)tile - 1;
-  uint32_t spins = 0, ns = 20;
-  for (;;) {
-    int64_t idx = base - (int64_t)lane;
-    uint32_t f = 2;
-    uint64_t v = 0;
-    if (idx >= 0) {
-      uint64_t w = ld_relaxed_u64(&words[idx]);
-      f = ((uint32_t)(w >> 58) == epoch) ? (uint32_t)((w >> 56) & 3) : 0u;
-      v = w & kLbValMask;
-    }
-    // only the tiles after the nearest published prefix must be ready
-    const uint32_t incl = __ballot_sync(kFull, f == 2);
-    const uint32_t first = incl ? (uint32_t)(__ffs(incl) - 1) : 31u;
-    const uint32_t upto = first == 31u ? kFull : ((2u << first) - 1u);
-    if (__ballot_sync(kFull, f == 0) & upto) {
-      if (++spins > kSpinCap) {
-        if (lane == 0) raise_err(st, kErrTimeout);
-        return 0;
-      }
-      __nanosleep(ns);
-      if (ns < 1000) ns += ns;
-      continue;
-    }
-    if (incl) {
-      if (lane > first) v = 0;
-      excl += warp_sum_u64(v);
-      break;
-    }
-    excl += warp_sum_u64(v);
-    base -= 32;
-  }
-  if (lane == 0) st_relaxed_u64(&words[tile], lb_pack(epoch, 2, excl + agg));
-  return excl;
-}
-
-// ---------------------------------------------------------------------------
-// Generic look-back for a payload T with an associative operator `op` and a
-// two-sided identity.  Status word per tile: epoch << 2 | flag.  Payloads go
-// to separate aggregate / inclusive arrays, published before the flag with a
-// fence.  Called by ONE thread.
-// ---------------------------------------------------------------------------
-template <class T>
-struct LbArrays {
-  uint32_t* status;
-  T* agg;
-  T* incl;
-};
-
-template <class T>
-__device__ __forceinline__ void lb_store(T* dst, const T& v) {
-  volatile uint64_t* d = reinterpret_cast<volatile uint64_t*>(dst);
-  const uint64_t* s = reinterpret_cast<const uint64_t*>(&v);
-#pragma unroll
-  for (int i = 0; i < (int)(sizeof(T) / 8); ++i) d[i] = s[i];
-}
-template <class T>
-__device__ __forceinline__ T lb_load(const T* src) {
-  T v;
-  const volatile uint64_t* s = reinterpret_cast<const volatile uint64_t*>(src);
-  uint64_t* d = reinterpret_cast<uint64_t*>(&v);
-#pragma unroll
-  for (int i = 0; i < (int)(sizeof(T) / 8); ++i) d[i] = s[i];
-  return v;
-}
-
-template <class T, class Op>
-__device__ inline T lookback_generic(LbArrays<T> a, uint32_t tile, const T& agg, const T& identity, Op op,
-                                     uint32_t epoch, DevStatus* st) {
-  static_assert(sizeof(T) % 8 == 0, "payload must be a multiple of 8 bytes");
-  if (tile == 0) {
-    lb_store(&a.incl[0], agg);
-    __threadfence();
-    st_relaxed_u32(&a.status[0], (epoch << 2) | 2u);
-    return identity;
-  }
-  lb_store(&a.agg[tile], agg);
-  __threadfence();
-  st_relaxed_u32(&a.status[tile], (epoch << 2) | 1u);
-  T acc = identity;
-  int64_t j = (int64_t)tile - 1;
-  uint32_t spins = 0, ns = 20;
-  while (j >= 0) {
-    uint32_t s = ld_relaxed_u32(&a.status[j]);
-    uint32_t f = ((s >> 2) == epoch) ? (s & 3u) : 0u;
-    if (f == 0) {
-      if (++spins > kSpinCap) {
-        raise_err(st, kErrTimeout);
-        return identity;
-      }
-      __nanosleep(ns);
-      if (ns < 1000) ns += ns;
-      continue;
-    }
-    __threadfence();
-    if (f == 2) {
-      acc = op(lb_load(&a.incl[j]), acc);
-      break;
-    }
-    acc = op(lb_load(&a.agg[j]), acc);
-    --j;
-  }
-  T inc = op(acc, agg);
-  lb_store(&a.incl[tile], inc);
-  __threadfence();
-  st_relaxed_u32(&a.status[tile], (epoch << 2) | 2u);
-  return acc;
-}
-
-// Warp-parallel variant of lookback_generic: called by all 32 lanes of ONE
-// warp; each round inspects 32 predecessors at once and folds them in order
-// (a higher lane holds an earlier tile, so it is the left operand).  Returns
-// the exclusive prefix in every lane.
+// Shuffles of a payload of 8-byte words across a warp.
 template <class T>
 __device__ __forceinline__ T shfl_down_payload(const T& v, int o) {
   T r;
@@ -314,66 +213,6 @@ __device__ __forceinline__ T shfl_payload(const T& v, int src) {
 #pragma unroll
   for (int i = 0; i < (int)(sizeof(T) / 8); ++i) d[i] = __shfl_sync(kFull, s[i], src);
   return r;
-}
-
-template <class T, class Op>
-__device__ inline T lookback_warp(LbArrays<T> a, uint32_t tile, const T& agg, const T& identity, Op op,
-                                  uint32_t epoch, DevStatus* st) {
-  static_assert(sizeof(T) % 8 == 0, "payload must be a multiple of 8 bytes");
-  const uint32_t lane = threadIdx.x & 31;
-  if (tile == 0) {
-    if (lane == 0) {
-      lb_store(&a.incl[0], agg);
-      __threadfence();
-      st_relaxed_u32(&a.status[0], (epoch << 2) | 2u);
-    }
-    return identity;
-  }
-  if (lane == 0) {
-    lb_store(&a.agg[tile], agg);
-    __threadfence();
-    st_relaxed_u32(&a.status[tile], (epoch << 2) | 1u);
-  }
-  T acc = identity;
-  int64_t base = (int64_t)tile - 1;
-  uint32_t spins = 0, ns = 20;
-  for (;;) {
-    const int64_t idx = base - (int64_t)lane;
-    uint32_t f = 2;
-    if (idx >= 0) {
-      const uint32_t s = ld_relaxed_u32(&a.status[idx]);
-      f = ((s >> 2) == epoch) ? (s & 3u) : 0u;
-    }
-    if (__any_sync(kFull, f == 0)) {
-      if (++spins > kSpinCap) {
-        if (lane == 0) raise_err(st, kErrTimeout);
-        return identity;
-      }
-      __nanosleep(ns);
-      if (ns < 1000) ns += ns;
-      continue;
-    }
-    __threadfence();
-    const uint32_t incl = __ballot_sync(kFull, f == 2);
-    const uint32_t first = incl ? (uint32_t)(__ffs(incl) - 1) : 31u;
-    T x = identity;
-    if (idx >= 0 && lane <= first) x = (f == 2) ? lb_load(&a.incl[idx]) : lb_load(&a.agg[idx]);
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const T y = shfl_down_payload(x, o);
-      if (lane + o < 32) x = op(y, x);
-    }
-    acc = op(shfl_payload(x, 0), acc);
-    if (incl) break;
-    base -= 32;
-  }
-  if (lane == 0) {
-    const T inc = op(acc, agg);
-    lb_store(&a.incl[tile], inc);
-    __threadfence();
-    st_relaxed_u32(&a.status[tile], (epoch << 2) | 2u);
-  }
-  return acc;
 }
 
 // ---------------------------------------------------------------------------
@@ -398,6 +237,8 @@ __device__ inline uint64_t lookback_sum_cta(uint64_t* words, uint32_t tile, uint
   }
   int64_t base = (int64_t)tile - 1;
   uint32_t spins = 0, ns = 20;
+  const uint32_t wait_test = ld_relaxed_u32(&st->wait_test);
+  const uint32_t cap = wait_test ? wait_test : kSpinCap;
   for (;;) {
     const int64_t idx = base - (int64_t)t;
     uint32_t f = 2;
@@ -406,6 +247,7 @@ __device__ inline uint64_t lookback_sum_cta(uint64_t* words, uint32_t tile, uint
       const uint64_t wv = ld_relaxed_u64(&words[idx]);
       f = ((uint32_t)(wv >> 58) == epoch) ? (uint32_t)((wv >> 56) & 3) : 0u;
       v = wv & kLbValMask;
+      if (wait_test) f = 0;
     }
     // the nearest published prefix; only the tiles after it must be ready
     if (t == 0) s_first = 0xFFFFFFFFu;
@@ -414,7 +256,7 @@ __device__ inline uint64_t lookback_sum_cta(uint64_t* words, uint32_t tile, uint
     __syncthreads();
     const uint32_t first = s_first;
     if (__syncthreads_or(f == 0 && t < first)) {
-      if (++spins > kSpinCap) {
+      if (++spins > cap) {
         if (t == 0) {
           raise_err(st, kErrTimeout);
           s_excl = 0;
@@ -441,125 +283,6 @@ __device__ inline uint64_t lookback_sum_cta(uint64_t* words, uint32_t tile, uint
   if (t == 0) st_relaxed_u64(&words[tile], lb_pack(epoch, 2, s_excl + agg));
   __syncthreads();
   return s_excl;
-}
-
-template <class T, class Op>
-__device__ inline T lookback_cta(LbArrays<T> a, uint32_t tile, const T& agg, const T& identity, Op op,
-                                 uint32_t epoch, DevStatus* st) {
-  static_assert(sizeof(T) % 8 == 0, "payload must be a multiple of 8 bytes");
-  __shared__ T s_wres[32];
-  __shared__ T s_acc;
-  __shared__ uint32_t s_first;
-  const uint32_t t = threadIdx.x, lane = t & 31, wid = t >> 5, nw = blockDim.x >> 5;
-  if (tile == 0) {
-    if (t == 0) {
-      lb_store(&a.incl[0], agg);
-      __threadfence();
-      st_relaxed_u32(&a.status[0], (epoch << 2) | 2u);
-    }
-    return identity;
-  }
-  if (t == 0) {
-    lb_store(&a.agg[tile], agg);
-    __threadfence();
-    st_relaxed_u32(&a.status[tile], (epoch << 2) | 1u);
-    s_acc = identity;
-  }
-  int64_t base = (int64_t)tile - 1;
-  uint32_t spins = 0, ns = 20;
-  for (;;) {
-    const int64_t idx = base - (int64_t)t;
-    uint32_t f = 2;
-    if (idx >= 0) {
-      const uint32_t sv = ld_relaxed_u32(&a.status[idx]);
-      f = ((sv >> 2) == epoch) ? (sv & 3u) : 0u;
-    }
-    if (__syncthreads_or(f == 0)) {
-      if (++spins > kSpinCap) {
-        if (t == 0) {
-          raise_err(st, kErrTimeout);
-          s_acc = identity;
-        }
-        break;
-      }
-      __nanosleep(ns);
-      if (ns < 500) ns += ns;
-      continue;
-    }
-    __threadfence();
-    if (t == 0) s_first = 0xFFFFFFFFu;
-    __syncthreads();
-    if (f == 2 && idx >= 0) atomicMin(&s_first, t);
-    __syncthreads();
-    const uint32_t first = s_first;
-    T x = identity;
-    if (idx >= 0 && t <= first) x = (f == 2) ? lb_load(&a.incl[idx]) : lb_load(&a.agg[idx]);
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const T y = shfl_down_payload(x, o);
-      if (lane + o < 32) x = op(y, x);
-    }
-    if (lane == 0) s_wres[wid] = x;
-    __syncthreads();
-    if (t == 0) {
-      T r = identity;
-      for (int k = (int)nw - 1; k >= 0; --k) r = op(r, s_wres[k]);
-      s_acc = op(r, s_acc);
-    }
-    __syncthreads();
-    // a window reaching past tile 0 counts as complete (idx < 0 reads as inclusive)
-    if (first != 0xFFFFFFFFu || base < (int64_t)blockDim.x) break;
-    base -= (int64_t)blockDim.x;
-  }
-  if (t == 0) {
-    const T inc = op(s_acc, agg);
-    lb_store(&a.incl[tile], inc);
-    __threadfence();
-    st_relaxed_u32(&a.status[tile], (epoch << 2) | 2u);
-  }
-  __syncthreads();
-  return s_acc;
-}
-
-// ---------------------------------------------------------------------------
-// Bulk (TMA) copies global -> shared with mbarrier completion (sm_90+).
-// The source and destination must be 16-byte aligned and the size a multiple
-// of 16 bytes.  Waits are bounded: on give-up the caller raises kErrTimeout.
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_init_fence() {
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                   smem_addr(dst)),
-               "l"(src), "r"(bytes), "r"(smem_addr(bar))
-               : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t phase) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(smem_addr(bar)), "r"(phase)
-      : "memory");
-  return ok != 0;
-}
-// Wait for phase `phase` of `bar`; false if the bounded wait gave up.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t phase) {
-  for (uint32_t i = 0; i < (1u << 22); ++i)
-    if (mbar_try_wait(bar, phase)) return true;
-  return false;
 }
 
 // ---------------------------------------------------------------------------

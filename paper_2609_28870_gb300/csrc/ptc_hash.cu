@@ -148,6 +148,15 @@ struct PowBases {
 
 // Only the entries some block can use are filled: exponents e = k reach at
 // most the longest request's block count minus one (st->value[1]).
+// Blocks the key kernels may touch: N as the offsets kernel left it, or none
+// if its look-back gave up (then the offsets are not a prefix sum and must
+// not steer any read; the call reports PTC_ERR_TIMEOUT).
+__device__ __forceinline__ uint64_t blocks_live(const DevStatus* st, uint64_t keys_cap) {
+  if (ld_relaxed_u32(&st->err) & kErrTimeout) return 0;
+  const uint64_t N = st->value[0];
+  return N < keys_cap ? N : keys_cap;
+}
+
 __global__ void k_pow_tables(PowBases pb, uint64_t* __restrict__ tables, const DevStatus* st) {
   grid_dep_sync();
   const uint32_t gid = blockIdx.x * blockDim.x + threadIdx.x;  // 4 tables x 8192 chunks of kPowChunk
@@ -374,8 +383,7 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local(HashArgs a, const _
   constexpr uint32_t TB = kHashThreads / G;
 
   const uint32_t tile = blockIdx.x;
-  uint64_t N = a.st->value[0];
-  if (N > a.keys_cap) N = a.keys_cap;
+  const uint64_t N = blocks_live(a.st, a.keys_cap);
   const uint64_t b0 = (uint64_t)tile * TB;
   if (b0 >= N) return;
   const uint64_t b_end = b0 + TB < N ? b0 + TB : N;
@@ -496,8 +504,7 @@ __global__ void __launch_bounds__(kHashThreads, 8) k_hash16(HashArgs a, const __
   __shared__ uint64_t s_toff[kH16Req + 1];
   constexpr uint32_t TB = kHashThreads;
   const uint32_t tile = blockIdx.x;
-  uint64_t N = a.st->value[0];
-  if (N > a.keys_cap) N = a.keys_cap;
+  const uint64_t N = blocks_live(a.st, a.keys_cap);
   const uint64_t b0 = (uint64_t)tile * TB;
   if (b0 >= N) return;
   const uint64_t b_end = b0 + TB < N ? b0 + TB : N;
@@ -796,8 +803,7 @@ __global__ void __launch_bounds__(kHashThreads, 4) k_hash_tile(HashArgs a, const
   __shared__ uint64_t s_p0[TB], s_p1[TB];
   __shared__ uint64_t s_w0[TB / 32], s_w1[TB / 32];
   const uint32_t tile = blockIdx.x;
-  uint64_t N = a.st->value[0];
-  if (N > a.keys_cap) N = a.keys_cap;
+  const uint64_t N = blocks_live(a.st, a.keys_cap);
   const uint64_t b0 = (uint64_t)tile * TB;
   if (b0 >= N) return;
   const uint64_t b_end = b0 + TB < N ? b0 + TB : N;
@@ -987,12 +993,11 @@ __global__ void __launch_bounds__(kChainWarps * 32) k_hash_chain(ulonglong2* __r
   grid_dep_sync();
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t tile = blockIdx.x * kChainWarps + (threadIdx.x >> 5);
-  uint64_t N = st->value[0];
-  if (N > keys_cap) N = keys_cap;
+  const uint64_t N = blocks_live(st, keys_cap);
   const uint64_t b0 = (uint64_t)tile * TB;
   if (b0 >= N || tile == 0) return;
   const uint32_t lead = tile_lead[tile];
-  if (lead == 0) return;
+  if (lead == 0 || !in_bounds(st, b0 + lead - 1, keys_cap)) return;
   uint64_t c0 = 0, c1 = 0;
   for (int64_t base = (int64_t)tile - 1; base >= 0; base -= 32) {
     const int64_t idx = base - (int64_t)lane;
@@ -1032,8 +1037,7 @@ __global__ void __launch_bounds__(kChainWarps * 32) k_hash_carry(const HashCarry
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t t0 = (blockIdx.x * kChainWarps + (threadIdx.x >> 5)) * kCarryPer;
   if (t0 >= ntiles) return;
-  uint64_t N = st->value[0];
-  if (N > keys_cap) N = keys_cap;
+  const uint64_t N = blocks_live(st, keys_cap);
   const uint64_t live = (N + TB - 1) / TB;  // tiles that hold blocks
   const SegSumOp op;
   HashCarry cin{0, 0, 0};
@@ -1169,6 +1173,8 @@ ptc_status ptc::hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t
   const HashLayout L = hash_layout(ws, n_req, n_tok, block_size, ~0ULL);
   *n_access_host_out = 0;
   if (begin_call(ws, L.zero_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
+  const uint32_t wait_test = test_wait_polls();
+  if (wait_test && fill_async(&L.st->wait_test, wait_test, sizeof(uint32_t), s) != PTC_OK) return PTC_ERR_CUDA;
   if (n_req == 0) {
     if (fill_async(req_blk_off_out, 0u, sizeof(uint64_t), s) != PTC_OK) return PTC_ERR_CUDA;
     if (deferred) return defer_status(L.st, err_slot, s, n_slot, 0);

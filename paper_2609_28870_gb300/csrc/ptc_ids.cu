@@ -186,7 +186,7 @@ __global__ void __launch_bounds__(kMkThreads) k_ids_mark(const ulonglong2* __res
   for (int k = 0; k < kMkPer; ++k) {
     if (v[k].x != ~0ULL && v[k].y != ~0ULL) {
       const uint32_t f = (uint32_t)(v[k].y >> 32);
-      atomicOr(&bits[f >> 5], 1u << (f & 31));
+      if (in_bounds(st, f, n_ub)) atomicOr(&bits[f >> 5], 1u << (f & 31));
     }
   }
 }
@@ -200,10 +200,11 @@ constexpr int kGaPer = 8;
 // slot_of of an access that the prior-request hint matched (no slot)
 constexpr uint32_t kMatchedSlot = 0xFFFFFFFFu;
 __global__ void __launch_bounds__(kGaThreads) k_ids_gather(const uint32_t* __restrict__ slot_of,
-                                                          const ulonglong2* __restrict__ table,
+                                                          const ulonglong2* __restrict__ table, uint64_t m,
                                                           const uint32_t* __restrict__ bits,
                                                           const uint32_t* __restrict__ wpre, uint32_t n_ub,
-                                                          const uint64_t* n_dev, uint32_t* __restrict__ ids) {
+                                                          const uint64_t* n_dev, uint32_t* __restrict__ ids,
+                                                          const DevStatus* st) {
   grid_dep_sync();
   const uint32_t n = keys_used(n_ub, n_dev);
   const uint32_t i0 = blockIdx.x * (kGaThreads * kGaPer) + threadIdx.x;
@@ -216,7 +217,9 @@ __global__ void __launch_bounds__(kGaThreads) k_ids_gather(const uint32_t* __res
 #pragma unroll
   for (int k = 0; k < kGaPer; ++k) {
     const uint32_t i = i0 + k * kGaThreads;
-    f[k] = i < n && f[k] != kMatchedSlot ? __ldg(reinterpret_cast<const uint32_t*>(&table[f[k]]) + 3) : kMatchedSlot;
+    f[k] = i < n && f[k] != kMatchedSlot && in_bounds(st, f[k], m)
+               ? __ldg(reinterpret_cast<const uint32_t*>(&table[f[k]]) + 3)
+               : kMatchedSlot;
   }
   uint32_t wp[kGaPer], bw[kGaPer];
 #pragma unroll
@@ -464,11 +467,15 @@ __global__ void k_tile_req(PriorHint ph, uint32_t n_ub, const uint64_t* n_dev) {
   if (t == T) ph.tile_req[t] = ph.n_req - 1;
 }
 
-// One key per thread.  Each access finds its request by binary search among
-// the few requests its 2048-access tile spans (tile_req).
-// A matched access writes kMatched and stops; an unmatched one lowers its
-// request's lam (one atomic per group of lanes in one request) and settles
-// its key in the table as k_ids_insert does.
+// kPriorK keys per thread, kInsThreads apart.  Each access finds its request
+// by binary search among the few requests its 2048-access tile spans
+// (tile_req).  A matched access writes kMatched and stops; an unmatched one
+// lowers its request's lam (one atomic per group of lanes in one request) and
+// settles its key in the table as k_ids_insert does.  The keys' loads, then
+// the previous requests' keys, then the slot loads of all unmatched keys go
+// out together, so a thread has kPriorK independent probes in flight.
+constexpr int kPriorK = 1;
+template <int K>
 __global__ void __launch_bounds__(kInsThreads) k_ids_insert_prior(const ulonglong2* __restrict__ keys, uint32_t n_ub,
                                                                   const uint64_t* n_dev, ulonglong2* table,
                                                                   uint32_t log2m, uint64_t probe_cap,
@@ -476,40 +483,65 @@ __global__ void __launch_bounds__(kInsThreads) k_ids_insert_prior(const ulonglon
                                                                   InsCarry kc, PriorHint ph) {
   grid_dep_sync();
   const uint32_t n = keys_used(n_ub, n_dev);
-  const uint32_t i = blockIdx.x * kInsThreads + threadIdx.x;
-  if (i >= n) return;
-  const ulonglong2 k = carried_key(keys, i, n, kc);
-  const uint32_t t = i >> kReqTileLog2;
-  const uint32_t r0 = __ldg(&ph.tile_req[t]), r1 = __ldg(&ph.tile_req[t + 1]);
-  if (k.x >= kP61 || k.y >= kP61) {
-    raise_err(st, kErrInvalid);
-    slot_of[i] = 0;
-    return;
+  const uint32_t base = blockIdx.x * (kInsThreads * K) + threadIdx.x;
+  if (blockIdx.x * (kInsThreads * K) >= n) return;  // the whole CTA
+  ulonglong2 k[K], q[K];
+  uint32_t r[K];
+  uint64_t depth[K];
+  bool live[K], unm[K];
+#pragma unroll
+  for (int j = 0; j < K; ++j) {
+    const uint32_t i = base + j * kInsThreads;
+    live[j] = i < n;
+    k[j] = carried_key(keys, i, n, kc);
   }
-  const uint32_t r = req_at(ph.blk_off, r0, r1, i);
-  const uint64_t depth = i - __ldg(&ph.blk_off[r]);
-  const uint32_t p = __ldg(&ph.prior[r]);
-  bool matched = false;
-  if (p != kNone) {
-    if (p >= r) {
-      raise_err(st, kErrInvalid);  // a hint must point to an earlier request
-    } else {
-      const uint64_t pb = __ldg(&ph.blk_off[p]), pn = __ldg(&ph.blk_off[p + 1]) - pb;
-      if (depth < pn && pb + depth < n) {
-        const ulonglong2 q = carried_key(keys, (uint32_t)(pb + depth), n, kc);
-        matched = q.x == k.x && q.y == k.y;
-      }
+#pragma unroll
+  for (int j = 0; j < K; ++j) {
+    const uint32_t i = base + j * kInsThreads;
+    r[j] = 0;
+    depth[j] = 0;
+    q[j] = make_ulonglong2(~0ULL, ~0ULL);
+    unm[j] = live[j];
+    if (!live[j]) continue;
+    if (k[j].x >= kP61 || k[j].y >= kP61) {
+      raise_err(st, kErrInvalid);
+      slot_of[i] = 0;
+      live[j] = unm[j] = false;
+      continue;
     }
+    const uint32_t t = i >> kReqTileLog2;
+    r[j] = req_at(ph.blk_off, __ldg(&ph.tile_req[t]), __ldg(&ph.tile_req[t + 1]), i);
+    depth[j] = i - __ldg(&ph.blk_off[r[j]]);
+    const uint32_t p = __ldg(&ph.prior[r[j]]);
+    if (p == kNone) continue;
+    if (p >= r[j]) {
+      raise_err(st, kErrInvalid);  // a hint must point to an earlier request
+      continue;
+    }
+    const uint64_t pb = __ldg(&ph.blk_off[p]), pn = __ldg(&ph.blk_off[p + 1]) - pb;
+    if (depth[j] < pn && pb + depth[j] < n) q[j] = carried_key(keys, (uint32_t)(pb + depth[j]), n, kc);
   }
-  if (matched) {
-    __stcs(&slot_of[i], kMatched);
-    return;
+  ulonglong2 cur[K];
+  uint64_t pos[K];
+#pragma unroll
+  for (int j = 0; j < K; ++j) {
+    if (live[j] && q[j].x == k[j].x && q[j].y == k[j].y) {
+      __stcs(&slot_of[base + j * kInsThreads], kMatched);
+      unm[j] = false;
+    }
+    pos[j] = home_slot(k[j].x, k[j].y, log2m);
+    cur[j] = unm[j] ? ld_slot(&table[pos[j]]) : make_ulonglong2(0, 0);
   }
-  const unsigned grp = __match_any_sync(__activemask(), r);
-  const uint32_t lo = __reduce_min_sync(grp, (uint32_t)depth);
-  if ((threadIdx.x & 31) == (uint32_t)(__ffs(grp) - 1)) atomicMin(&ph.lam[r], lo);
-  const uint64_t pos = home_slot(k.x, k.y, log2m);
-  settle(table, (1ULL << log2m) - 1, probe_cap, i, k, pos, ld_slot(&table[pos]), &slot_of[i], st);
+#pragma unroll
+  for (int j = 0; j < K; ++j) {
+    const uint32_t am = __ballot_sync(kFull, unm[j]);
+    if (!unm[j]) continue;
+    const unsigned grp = __match_any_sync(am, r[j]);
+    const uint32_t lo = __reduce_min_sync(grp, (uint32_t)depth[j]);
+    if ((threadIdx.x & 31) == (uint32_t)(__ffs(grp) - 1)) atomicMin(&ph.lam[r[j]], lo);
+    settle(table, (1ULL << log2m) - 1, probe_cap, base + j * kInsThreads, k[j], pos[j], cur[j],
+           &slot_of[base + j * kInsThreads], st);
+  }
 }
 
 // ids of the matched accesses, one warp per request r: its depths below
@@ -536,6 +568,7 @@ __global__ void __launch_bounds__(kFoThreads) k_ids_follow(PriorHint ph, uint32_
     const uint64_t tb = ph.blk_off[t];
     const uint64_t lo = ph.lam[t];  // kNone (no unmatched depth) is above every hi
     if (lo < hi) {
+      if (!in_bounds(st, tb + hi - 1, b) || !in_bounds(st, b + hi - 1, ph.blk_off[ph.n_req])) return;
       for (uint64_t d = lo + lane; d < hi; d += 32) ids[b + d] = ids[tb + d];
       hi = lo;
     }
@@ -759,8 +792,8 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
                  n32, n_dev, L.table, log2m, probe_cap, L.slot_of, L.st);
     } else if (hint) {
       PTC_KERNEL("k_tile_req", s, k_tile_req, ceil_div_u32((n >> kReqTileLog2) + 2, 256), 256, 0, ph, n32, n_dev);
-      PTC_KERNEL("k_ids_insert_prior", s, k_ids_insert_prior, ceil_div_u32(n, kInsThreads), kInsThreads, 0, k, n32,
-                 n_dev, L.table, log2m, probe_cap, L.slot_of, L.st, ic, ph);
+      PTC_KERNEL("k_ids_insert_prior", s, k_ids_insert_prior<kPriorK>, ceil_div_u32(n, kInsThreads * kPriorK),
+                 kInsThreads, 0, k, n32, n_dev, L.table, log2m, probe_cap, L.slot_of, L.st, ic, ph);
     } else {
       PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads * kInsK), kInsThreads, 0, k, n32, n_dev,
                  L.table, log2m, probe_cap, L.slot_of, L.st, ic);
@@ -768,13 +801,14 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
     const uint64_t m = 1ULL << log2m;
     PTC_KERNEL("k_ids_mark", s, k_ids_mark, ceil_div_u32(m, kMkThreads * kMkPer), kMkThreads, 0, L.table, m, L.bits,
                n32, n_dev, L.st);
-    if (bitmap_ranks(L.bits, L.nwords, L.wpre, L.tcnt, L.tpre, &L.done[0], &L.st->value[0], s) != PTC_OK) return false;
+    if (bitmap_ranks(L.bits, L.nwords, L.wpre, L.tcnt, L.tpre, &L.done[0], &L.st->value[0], s) != PTC_OK)
+      return false;
     if (grouped)
       PTC_KERNEL("k_ids_gather_part", s, k_ids_gather_part, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of,
                  L.pidx, L.table, L.bits, L.wpre, n32, n_dev, ids_out);
     else
       PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of,
-                 L.table, L.bits, L.wpre, n32, n_dev, ids_out);
+                 L.table, m, L.bits, L.wpre, n32, n_dev, ids_out, L.st);
     if (hint)
       PTC_KERNEL("k_ids_follow", s, k_ids_follow, ceil_div_u32(hint->n_req, kFoThreads / 32), kFoThreads, 0, ph,
                  ids_out, L.st);

@@ -74,6 +74,10 @@ inline ptc_status begin_call(void* ws, size_t zero_bytes, cudaStream_t stream) {
   return fill_async(ws, 0u, zero_bytes, stream);
 }
 
+// The poll count set by ptc_test_wait_polls (0: normal waits), read by the
+// calls whose kernels wait on each other (stage a1's look-back).
+uint32_t test_wait_polls();
+
 // Words of ptc_trace_stats's results: the summary and the reach bins.
 constexpr size_t kStatsHostWords = sizeof(ptc_trace_summary) / 8 + PTC_MAX_CAPACITIES + 1;
 // Page-locked host buffers for the small copies around a call's wait, one
@@ -88,6 +92,7 @@ struct HostStage {
   HostStage* dev;  // the same memory as seen by kernels (mapped), or null
 };
 HostStage* host_stage();
+void release_host_stage();  // frees the calling thread's page-locked block
 // Copy `bytes` from device memory to `host_dst`.  When `host_dst` lies in
 // the thread's host stage and that stage is mapped, a one-CTA kernel
 // (k_copy_words) writes it straight into host memory, which joins the launch
@@ -105,6 +110,7 @@ struct NoHostAlloc {
 // Wait for the call's work and translate the device status block.
 // The status a device error word stands for.
 inline ptc_status status_of(uint32_t e) {
+  if (e & kErrBounds) return PTC_ERR_BOUNDS;
   if (e & kErrTimeout) return PTC_ERR_TIMEOUT;
   if (e & kErrUnsorted) return PTC_ERR_UNSORTED;
   if (e & kErrOverflow) return PTC_ERR_OVERFLOW;

@@ -318,6 +318,7 @@ struct FillArgs {
   const uint32_t* cut_at;  // id of every cut, by rank
   uint32_t* prev;
   uint32_t* next;
+  const DevStatus* st;     // for the checked build's bounds checks
 };
 
 // One warp per incidence (e, r): the accesses of run r with ids in e take
@@ -343,7 +344,7 @@ __global__ void __launch_bounds__(256) k_ir_fill(FillArgs a) {
     }
     for (uint32_t t = lane; t < hi - lo; t += 32) {
       const uint32_t j = s0 + t;
-      if (j < a.n) {
+      if (in_bounds(a.st, j, a.n)) {
         a.prev[j] = has_pred ? p0 + t : kNone;
         a.next[j] = has_succ ? n0 + t : kNone;
       }
@@ -476,6 +477,7 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
   f.cut_at = L.cut_at;
   f.prev = prev_out;
   f.next = next_out;
+  f.st = L.st;
   const uint32_t fill_blocks = ceil_div_u32(K, 8) < (uint32_t)(16 * num_sms()) ? ceil_div_u32(K, 8)
                                                                                 : (uint32_t)(16 * num_sms());
   PTC_KERNEL("k_ir_fill", s, k_ir_fill, fill_blocks, 256, 0, f);

@@ -613,7 +613,8 @@ constexpr int kExpPer = 8;
 __global__ void __launch_bounds__(kExpThreads) k_runs_expand(const uint32_t* __restrict__ bits,
                                                             const uint32_t* __restrict__ wpre,
                                                             const uint32_t* __restrict__ sd, uint32_t n,
-                                                            uint32_t* __restrict__ dist) {
+                                                            uint32_t* __restrict__ dist, uint32_t nruns,
+                                                            const DevStatus* st) {
   grid_dep_sync();
   const uint32_t j0 = blockIdx.x * (kExpThreads * kExpPer) + threadIdx.x;
   uint32_t r[kExpPer];
@@ -625,7 +626,7 @@ __global__ void __launch_bounds__(kExpThreads) k_runs_expand(const uint32_t* __r
 #pragma unroll
   for (int k = 0; k < kExpPer; ++k) {
     const uint32_t j = j0 + k * kExpThreads;
-    if (j < n) __stcs(&dist[j], __ldg(&sd[r[k]]));
+    if (j < n && in_bounds(st, r[k], nruns)) __stcs(&dist[j], __ldg(&sd[r[k]]));
   }
 }
 
@@ -831,7 +832,7 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   q.R = R32;
   q.L = L;
   PTC_KERNEL("k_runs_query", s, k_runs_query, ceil_div_u32(R, 256), 256, 0, q);
-  PTC_KERNEL("k_runs_expand", s, k_runs_expand, ceil_div_u32(n, kExpThreads * kExpPer), kExpThreads, 0, W.bits, W.wpre, W.sd, (uint32_t)n, dist_out);
+  PTC_KERNEL("k_runs_expand", s, k_runs_expand, ceil_div_u32(n, kExpThreads * kExpPer), kExpThreads, 0, W.bits, W.wpre, W.sd, (uint32_t)n, dist_out, R32, W.st);
   const ptc_status done = defer_err ? defer_status(W.st, defer_err, s) : end_call(W.st, s, &h);
   if (done == PTC_OK && view) {
     view->used = true;

@@ -146,6 +146,7 @@ struct ScatterArgs {
   const uint32_t* off;      // this pass's tile prefixes, digit-major
   const uint32_t* tot;      // this pass's digit totals
   uint32_t n, T, shift, R, width;
+  const DevStatus* st;      // for the checked build's bounds checks
 };
 
 template <bool LAST>
@@ -231,7 +232,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) k_sort_scatter(ScatterArgs a)
       const uint32_t k = s_keys[p];
       const uint32_t dd = (k >> a.shift) & dmask;
       const uint32_t dst = s_gbase[dd] + (p - s_start[dd]);
-      if (dst < a.n) {
+      if (in_bounds(a.st, dst, a.n)) {
         a.keys_out[dst] = k;
         a.vals_out[dst] = s_vals[p];
       }
@@ -241,7 +242,7 @@ __global__ void __launch_bounds__(kSortThreads, 3) k_sort_scatter(ScatterArgs a)
       const uint32_t k = s_keys[p], v = s_vals[p];
       const uint32_t dd = (k >> a.shift) & dmask;
       const uint32_t lo = s_start[dd], hi = s_start[dd + 1];
-      if (v < a.n) {
+      if (in_bounds(a.st, v, a.n)) {
         if (p > lo) a.prev[v] = s_keys[p - 1] == k ? s_vals[p - 1] : kNone;
         if (p + 1 < hi) a.next[v] = s_keys[p + 1] == k ? s_vals[p + 1] : kNone;
       }
@@ -380,6 +381,7 @@ ptc_status ptc::reuse_by_sort(const uint32_t* ids, uint64_t n, uint64_t n_distin
     a.shift = shift;
     a.R = R;
     a.width = width;
+    a.st = L.st;
     if (last) {
       PTC_KERNEL("k_sort_scatter", s, k_sort_scatter<true>, T, kSortThreads, 0, a);
       PTC_KERNEL("k_sort_links", s, k_sort_links, R, kSortThreads, 0, L.cnt, T, L.head_kv, L.tail_kv, n32, prev_out, next_out);
@@ -428,6 +430,7 @@ void ptc::sort_pairs(const uint32_t* keys, const uint32_t* vals, uint32_t n, uin
     a.shift = shift;
     a.R = R;
     a.width = width;
+    a.st = st;
     PTC_KERNEL("k_sort_scatter", s, k_sort_scatter<false>, T, kSortThreads, 0, a);
     kin = kout;
     vin = vout;
