@@ -150,25 +150,6 @@ ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t* ids_out, u
                           void* ws, size_t ws_bytes, void* stream);
 
 /*
- * ptc_assign_ids_ex — the same ids with the order of the table inserts chosen
- * by the caller (the ids do not depend on it).  PTC_IDS_DIRECT inserts the
- * keys in access order.  PTC_IDS_GROUPED first groups them by the partition
- * of the table their home slot lies in (2^21 slots, 32 MB, per partition;
- * 16 partitions when the table is smaller than 2^25 slots), then inserts
- * and reads back the slots partition by partition, so that the table slice
- * being probed stays in L2; this costs 20 n bytes of workspace, two more
- * passes over the keys and a scattered write of the ids, and on one GB300 it
- * was slower over the whole stage even where the table exceeds L2.
- * PTC_IDS_AUTO (ptc_assign_ids) inserts in access order.
- * Workspace: ptc_assign_ids_ex_workspace_bytes(n, method); an unknown
- * method returns PTC_ERR_INVALID_ARG.
- */
-enum { PTC_IDS_AUTO = 0, PTC_IDS_DIRECT = 1, PTC_IDS_GROUPED = 2 };
-size_t ptc_assign_ids_ex_workspace_bytes(uint64_t n, int method);
-ptc_status ptc_assign_ids_ex(const ptc_u128* keys, uint64_t n, uint32_t* ids_out, uint64_t* n_distinct_host_out,
-                             int method, void* ws, size_t ws_bytes, void* stream);
-
-/*
  * ptc_assign_ids_prior — the ids of ptc_assign_ids, with a prior-request hint
  * that saves table probes.  Sec. 2.3: a turn of a multi-turn session sends
  * the whole context again, so request r usually repeats every block of an

@@ -30,7 +30,6 @@ PTC_NONE = 0xFFFFFFFF
 PTC_COST_UNIFORM, PTC_COST_MEASURED, PTC_COST_LINEAR = 0, 1, 2
 PTC_SD_AUTO, PTC_SD_POINTS, PTC_SD_RUNS = 0, 1, 2
 PTC_REUSE_AUTO, PTC_REUSE_SORT, PTC_REUSE_RUNS = 0, 1, 2
-PTC_IDS_AUTO, PTC_IDS_DIRECT, PTC_IDS_GROUPED = 0, 1, 2
 PTC_TOUCH_ROOT_FIRST, PTC_TOUCH_LEAF_FIRST = 0, 1
 PTC_RESIDENCY_BLOCK, PTC_RESIDENCY_REQUEST = 0, 1
 F_LIN = 6_600_000_000          # 2 x 3.3e9 active parameters, FLOPs per token
@@ -107,10 +106,6 @@ def lib():
                 L.ptc_assign_ids_workspace_bytes.argtypes = [u64]
                 L.ptc_assign_ids.restype = st
                 L.ptc_assign_ids.argtypes = [vp, u64, vp, ctypes.POINTER(u64), vp, sz, vp]
-                L.ptc_assign_ids_ex_workspace_bytes.restype = sz
-                L.ptc_assign_ids_ex_workspace_bytes.argtypes = [u64, ctypes.c_int]
-                L.ptc_assign_ids_ex.restype = st
-                L.ptc_assign_ids_ex.argtypes = [vp, u64, vp, ctypes.POINTER(u64), ctypes.c_int, vp, sz, vp]
                 L.ptc_verify_ids_workspace_bytes.restype = sz
                 L.ptc_verify_ids_workspace_bytes.argtypes = [u64, u64]
                 L.ptc_verify_ids.restype = st
@@ -263,23 +258,15 @@ def ptc_hash_blocks(tokens: torch.Tensor, req_tok_off: torch.Tensor, req_ts_us: 
     return keys[: n.value], blk_off, int(n.value)
 
 
-def ptc_assign_ids(keys: torch.Tensor, ws: torch.Tensor | None = None, method: int | None = None):
-    """Dense ids in first-occurrence order.  Returns (ids int32[N], D).
-    ``method`` (PTC_IDS_AUTO / PTC_IDS_DIRECT / PTC_IDS_GROUPED) goes through
-    ptc_assign_ids_ex; None calls ptc_assign_ids."""
+def ptc_assign_ids(keys: torch.Tensor, ws: torch.Tensor | None = None):
+    """Dense ids in first-occurrence order.  Returns (ids int32[N], D)."""
     dev = _dev(keys)
     n = keys.shape[0]
     ids = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
     d = ctypes.c_uint64(0)
-    if method is None:
-        w = _workspace(lib().ptc_assign_ids_workspace_bytes(n), dev, ws)
-        rc = lib().ptc_assign_ids(_ptr(keys), n, _ptr(ids), ctypes.byref(d), _ptr(w), w.numel(), _stream(dev))
-        _check("ptc_assign_ids", rc)
-    else:
-        w = _workspace(lib().ptc_assign_ids_ex_workspace_bytes(n, method), dev, ws)
-        rc = lib().ptc_assign_ids_ex(_ptr(keys), n, _ptr(ids), ctypes.byref(d), method, _ptr(w), w.numel(),
-                                     _stream(dev))
-        _check("ptc_assign_ids_ex", rc)
+    w = _workspace(lib().ptc_assign_ids_workspace_bytes(n), dev, ws)
+    rc = lib().ptc_assign_ids(_ptr(keys), n, _ptr(ids), ctypes.byref(d), _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_assign_ids", rc)
     return ids[:n], int(d.value)
 
 

@@ -12,10 +12,6 @@
 //   bitmap_ranks   first occurrences before every 32-position word, and D
 //   k_ids_gather   ids[i] = rank, among the first occurrences, of the index
 //                  stored in i's slot.
-//   grouped (on request, ptc_assign_ids_ex): k_part_count, k_part_scan and
-//   k_part_scatter group the keys by the partition of the table their home
-//   slot lies in; k_ids_insert_part and k_ids_gather_part then work
-//   partition by partition, each partition's slice of the table in L2.
 // ptc_verify_ids
 //   k_verify_first first access of every id (atomicMin)
 //   k_verify       compares every access's B tokens and parent id with those
@@ -236,21 +232,6 @@ __global__ void __launch_bounds__(kGaThreads) k_ids_gather(const uint32_t* __res
   }
 }
 
-// ---------------------------------------------------------------- partitioned
-// A table larger than L2 is filled partition by partition: the keys are first
-// grouped by the top bits of their home slot (2^pshift slots of table per
-// partition), then inserted in that order, so that the inserts running at any
-// time probe one partition's slice of the table, which stays in L2, instead
-// of random DRAM sectors.  The slot of every grouped key goes to slot_of in
-// grouped order, and the gather, also in grouped order, reads the slots of
-// one slice at a time before writing each id to its access.  The order of
-// the inserts does not change the table's contents: each filled slot holds
-// its key and the smallest index of that key whatever the order.
-constexpr int kPtThreads = 256;
-constexpr int kPtPer = 4;           // keys per thread in the count and scatter passes
-constexpr uint32_t kPartSliceLog2 = 21;  // 2^21 slots = 32 MB of table per partition
-constexpr uint32_t kMaxPartsLog2 = 12;   // tables of at most 2^33 slots
-
 // Key i with the carry of its hash tile added (as k_ids_insert does), or
 // all-ones past the buffer.
 __device__ __forceinline__ ulonglong2 carried_key(const ulonglong2* __restrict__ keys, uint32_t i, uint32_t n_ub,
@@ -265,157 +246,6 @@ __device__ __forceinline__ ulonglong2 carried_key(const ulonglong2* __restrict__
     }
   }
   return k;
-}
-
-// The partition of a key: its home slot's top bits; a key that is not a
-// field element (an error the insert reports) goes to partition 0.
-__device__ __forceinline__ uint32_t part_of(ulonglong2 k, uint32_t log2m, uint32_t pshift) {
-  if (k.x >= kP61 || k.y >= kP61) return 0;
-  return (uint32_t)(home_slot(k.x, k.y, log2m) >> pshift);
-}
-
-// Keys per partition: a shared-memory histogram per CTA, added to count[].
-__global__ void __launch_bounds__(kPtThreads) k_part_count(const ulonglong2* __restrict__ keys, uint32_t n_ub,
-                                                           const uint64_t* n_dev, InsCarry kc, uint32_t log2m,
-                                                           uint32_t pshift, uint32_t nparts,
-                                                           uint32_t* __restrict__ count) {
-  __shared__ uint32_t s_cnt[1u << kMaxPartsLog2];
-  grid_dep_sync();
-  for (uint32_t q = threadIdx.x; q < nparts; q += kPtThreads) s_cnt[q] = 0;
-  __syncthreads();
-  const uint32_t n = keys_used(n_ub, n_dev);
-  const uint32_t i0 = blockIdx.x * (kPtThreads * kPtPer) + threadIdx.x;
-#pragma unroll
-  for (int j = 0; j < kPtPer; ++j) {
-    const uint32_t i = i0 + j * kPtThreads;
-    const ulonglong2 k = carried_key(keys, i, n_ub, kc);
-    if (i < n) atomicAdd(&s_cnt[part_of(k, log2m, pshift)], 1u);
-  }
-  __syncthreads();
-  for (uint32_t q = threadIdx.x; q < nparts; q += kPtThreads)
-    if (s_cnt[q]) atomicAdd(&count[q], s_cnt[q]);
-}
-
-// Exclusive prefix of the partition counts into cursor[] (one warp; nparts
-// is at most 2^kMaxPartsLog2, so each lane sums a run of at most 128).
-__global__ void __launch_bounds__(32) k_part_scan(const uint32_t* __restrict__ count, uint32_t nparts,
-                                                  uint32_t* __restrict__ cursor) {
-  grid_dep_sync();
-  const uint32_t lane = threadIdx.x;
-  const uint32_t per = (nparts + 31) / 32, q0 = lane * per, q1 = q0 + per < nparts ? q0 + per : nparts;
-  uint32_t sum = 0;
-  for (uint32_t q = q0; q < q1; ++q) sum += count[q];
-  uint32_t x = sum;
-#pragma unroll
-  for (int d = 1; d < 32; d <<= 1) {
-    const uint32_t y = __shfl_up_sync(kFull, x, d);
-    if (lane >= (uint32_t)d) x += y;
-  }
-  uint32_t run = x - sum;
-  for (uint32_t q = q0; q < q1; ++q) {
-    cursor[q] = run;
-    run += count[q];
-  }
-}
-
-// Each key (carry added) and its index to its partition's next places: a
-// CTA counts its keys per partition, reserves one range per partition with
-// one atomic each, and places its keys inside the ranges.
-__global__ void __launch_bounds__(kPtThreads) k_part_scatter(const ulonglong2* __restrict__ keys, uint32_t n_ub,
-                                                             const uint64_t* n_dev, InsCarry kc, uint32_t log2m,
-                                                             uint32_t pshift, uint32_t nparts,
-                                                             uint32_t* __restrict__ cursor,
-                                                             ulonglong2* __restrict__ pkey,
-                                                             uint32_t* __restrict__ pidx) {
-  __shared__ uint32_t s_cnt[1u << kMaxPartsLog2];
-  grid_dep_sync();
-  for (uint32_t q = threadIdx.x; q < nparts; q += kPtThreads) s_cnt[q] = 0;
-  __syncthreads();
-  const uint32_t n = keys_used(n_ub, n_dev);
-  const uint32_t i0 = blockIdx.x * (kPtThreads * kPtPer) + threadIdx.x;
-  ulonglong2 k[kPtPer];
-  uint32_t part[kPtPer];
-#pragma unroll
-  for (int j = 0; j < kPtPer; ++j) {
-    const uint32_t i = i0 + j * kPtThreads;
-    k[j] = carried_key(keys, i, n_ub, kc);
-    part[j] = part_of(k[j], log2m, pshift);
-    if (i < n) atomicAdd(&s_cnt[part[j]], 1u);
-  }
-  __syncthreads();
-  for (uint32_t q = threadIdx.x; q < nparts; q += kPtThreads)  // this CTA's range in each partition
-    if (s_cnt[q]) s_cnt[q] = atomicAdd(&cursor[q], s_cnt[q]);
-  __syncthreads();
-#pragma unroll
-  for (int j = 0; j < kPtPer; ++j) {
-    const uint32_t i = i0 + j * kPtThreads;
-    if (i < n) {
-      const uint32_t at = atomicAdd(&s_cnt[part[j]], 1u);
-      pkey[at] = k[j];
-      pidx[at] = i;
-    }
-  }
-}
-
-// The insert in grouped order: place j holds key pkey[j] of access pidx[j];
-// its slot goes to slot_of[j].
-__global__ void __launch_bounds__(kInsThreads) k_ids_insert_part(const ulonglong2* __restrict__ pkey,
-                                                                 const uint32_t* __restrict__ pidx, uint32_t n_ub,
-                                                                 const uint64_t* n_dev, ulonglong2* table,
-                                                                 uint32_t log2m, uint64_t probe_cap,
-                                                                 uint32_t* __restrict__ slot_of, DevStatus* st) {
-  grid_dep_sync();
-  const uint32_t j = blockIdx.x * kInsThreads + threadIdx.x;
-  if (j >= n_ub) return;
-  const ulonglong2 k = __ldcs(&pkey[j]);
-  const uint32_t i = __ldcs(&pidx[j]);
-  const uint32_t n = keys_used(n_ub, n_dev);
-  if (j >= n) return;
-  if (k.x >= kP61 || k.y >= kP61) {
-    raise_err(st, kErrInvalid);
-    slot_of[j] = 0;
-    return;
-  }
-  const uint64_t mask = (1ULL << log2m) - 1;
-  const uint64_t pos = home_slot(k.x, k.y, log2m);
-  settle(table, mask, probe_cap, i, k, pos, ld_slot(&table[pos]), &slot_of[j], st);
-}
-
-// ids in grouped order: place j's slot gives the first occurrence of its
-// key, the bitmap's ranks its id, written to access pidx[j].
-__global__ void __launch_bounds__(kGaThreads) k_ids_gather_part(const uint32_t* __restrict__ slot_of,
-                                                               const uint32_t* __restrict__ pidx,
-                                                               const ulonglong2* __restrict__ table,
-                                                               const uint32_t* __restrict__ bits,
-                                                               const uint32_t* __restrict__ wpre, uint32_t n_ub,
-                                                               const uint64_t* n_dev, uint32_t* __restrict__ ids) {
-  grid_dep_sync();
-  const uint32_t n = keys_used(n_ub, n_dev);
-  const uint32_t j0 = blockIdx.x * (kGaThreads * kGaPer) + threadIdx.x;
-  uint32_t f[kGaPer], at[kGaPer];
-#pragma unroll
-  for (int q = 0; q < kGaPer; ++q) {
-    const uint32_t j = j0 + q * kGaThreads;
-    f[q] = j < n ? __ldcs(&slot_of[j]) : 0u;
-    at[q] = j < n ? __ldcs(&pidx[j]) : 0u;
-  }
-#pragma unroll
-  for (int q = 0; q < kGaPer; ++q) {
-    const uint32_t j = j0 + q * kGaThreads;
-    f[q] = j < n ? __ldg(reinterpret_cast<const uint32_t*>(&table[f[q]]) + 3) : kNone;
-  }
-  uint32_t wp[kGaPer], bw[kGaPer];
-#pragma unroll
-  for (int q = 0; q < kGaPer; ++q) {
-    const bool ok = f[q] < n;
-    wp[q] = ok ? wpre[f[q] >> 5] : 0u;
-    bw[q] = ok ? bits[f[q] >> 5] : 0u;
-  }
-#pragma unroll
-  for (int q = 0; q < kGaPer; ++q) {
-    const uint32_t j = j0 + q * kGaThreads;
-    if (j < n && at[q] < n) ids[at[q]] = f[q] < n ? wp[q] + __popc(bw[q] & ((1u << (f[q] & 31)) - 1u)) : kNone;
-  }
 }
 
 // ---------------------------------------------------------------- prior-request hint
@@ -612,26 +442,12 @@ uint32_t small_table_log2(uint64_t n) {
   return l <= kL2TableLog2 ? l : table_log2(n / 4 * 3 + 64);
 }
 
-// Whether the keys are grouped by table partition before the insert: only
-// when the caller asks.  Grouping keeps the probed slice of a DRAM-sized
-// table in L2 (the insert of the 130M-key agentic trace: 4.9 -> 2.8 ms), but
-// placing the keys and writing the ids back to access order cost more than
-// that (the whole stage: 7.9 -> 12.1 ms), so PTC_IDS_AUTO inserts in access
-// order.
-bool ids_grouped(uint64_t n, int method) {
-  (void)n;
-  return method == PTC_IDS_GROUPED;
-}
-
 struct IdsLayout {
   DevStatus* st;
   uint32_t* done;
   ulonglong2* table;
-  uint32_t* slot_of;  // per access, or per grouped place
+  uint32_t* slot_of;  // per access: its slot, or kMatched
   uint32_t *bits, *wpre, *tcnt, *tpre;  // first-occurrence bitmap and its ranks
-  uint32_t *pcount, *pcursor;  // grouped: keys per partition, next place in each
-  ulonglong2* pkey;            // grouped: the keys, carry added, partition by partition
-  uint32_t* pidx;              // grouped: their access indices
   uint32_t* lam;               // prior hint: first unmatched depth of each request
   uint32_t* tile_req;          // prior hint: request of every 2048th access
   uint32_t nwords;
@@ -640,7 +456,7 @@ struct IdsLayout {
   uint32_t log2m;
 };
 
-IdsLayout ids_layout(void* ws, uint64_t n, bool grouped, uint32_t n_req_hint = 0) {
+IdsLayout ids_layout(void* ws, uint64_t n, uint32_t n_req_hint = 0) {
   IdsLayout L;
   Carver cv(ws);
   L.log2m = full_table_log2(n);
@@ -656,14 +472,6 @@ IdsLayout ids_layout(void* ws, uint64_t n, bool grouped, uint32_t n_req_hint = 0
   L.wpre = cv.take<uint32_t>(L.nwords + 1);
   L.tcnt = cv.take<uint32_t>(rank_tiles(L.nwords) + 1);
   L.tpre = cv.take<uint32_t>(rank_tiles(L.nwords) + 1);
-  L.pcount = L.pcursor = L.pidx = nullptr;
-  L.pkey = nullptr;
-  if (grouped) {
-    L.pcount = cv.take<uint32_t>(1u << kMaxPartsLog2);
-    L.pcursor = cv.take<uint32_t>(1u << kMaxPartsLog2);
-    L.pkey = cv.take<ulonglong2>(nn);
-    L.pidx = cv.take<uint32_t>(nn);
-  }
   L.lam = n_req_hint ? cv.take<uint32_t>(n_req_hint) : nullptr;
   L.tile_req = n_req_hint ? cv.take<uint32_t>((nn >> kReqTileLog2) + 2) : nullptr;
   L.total = cv.bytes();
@@ -733,21 +541,13 @@ __global__ void k_verify(const uint32_t* __restrict__ tokens, uint64_t n_tok, co
 
 using namespace ptc;
 
-extern "C" size_t ptc_assign_ids_workspace_bytes(uint64_t n) {
-  return ids_layout(nullptr, n, ids_grouped(n, PTC_IDS_AUTO)).total;
-}
-
-extern "C" size_t ptc_assign_ids_ex_workspace_bytes(uint64_t n, int method) {
-  return ids_layout(nullptr, n, ids_grouped(n, method)).total;
-}
+extern "C" size_t ptc_assign_ids_workspace_bytes(uint64_t n) { return ids_layout(nullptr, n).total; }
 
 ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev, uint32_t* ids_out,
                         uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
                         cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc,
-                        uint64_t* nd_slot, uint32_t* err_slot, bool full_table, int method, const IdsHint* hint) {
-  if (method != PTC_IDS_AUTO && method != PTC_IDS_DIRECT && method != PTC_IDS_GROUPED) return PTC_ERR_INVALID_ARG;
-  if (hint && (method == PTC_IDS_GROUPED || hint->n_req == 0 || !hint->blk_off || !hint->prior))
-    return PTC_ERR_INVALID_ARG;
+                        uint64_t* nd_slot, uint32_t* err_slot, bool full_table, const IdsHint* hint) {
+  if (hint && (hint->n_req == 0 || !hint->blk_off || !hint->prior)) return PTC_ERR_INVALID_ARG;
   if (kc && (kc->tile_blocks == 0 || (kc->tile_blocks & (kc->tile_blocks - 1)) != 0)) return PTC_ERR_INVALID_ARG;
   const InsCarry ic = kc ? InsCarry{kc->carry, kc->lead, (uint32_t)__builtin_ctz(kc->tile_blocks)}
                         : InsCarry{nullptr, nullptr, 0};
@@ -756,41 +556,24 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
   if (n_used_host_out) *n_used_host_out = 0;
   if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
   if (n > 0 && (keys == nullptr || ids_out == nullptr)) return PTC_ERR_INVALID_ARG;
-  const bool grouped = ids_grouped(n, method);
   const uint32_t hreq = hint ? hint->n_req : 0;
-  if (!ws_ok(ws, ws_bytes, ids_layout(nullptr, n, grouped, hreq).total)) return PTC_ERR_WORKSPACE;
-  const IdsLayout L = ids_layout(ws, n, grouped, hreq);
+  if (!ws_ok(ws, ws_bytes, ids_layout(nullptr, n, hreq).total)) return PTC_ERR_WORKSPACE;
+  const IdsLayout L = ids_layout(ws, n, hreq);
   const PriorHint ph = hint ? PriorHint{hint->blk_off, hint->prior, hint->n_req, L.lam, L.tile_req}
                             : PriorHint{nullptr, nullptr, 0, nullptr, nullptr};
   // the status block, the table (all ones: empty), the first-occurrence
-  // bitmap and the partition counts are cleared by one launch
+  // bitmap and the hint's first unmatched depths are cleared by one launch
   auto start = [&](uint32_t log2m) -> bool {
     const FillRange zf[4] = {{ws, L.zero_bytes, 0u},
                             {L.table, n > 0 ? sizeof(ulonglong2) << log2m : 0, ~0u},
                             {L.bits, n > 0 ? sizeof(uint32_t) * L.nwords : 0, 0u},
-                            {grouped ? (void*)L.pcount : (void*)L.lam,
-                             grouped ? (n > 0 ? sizeof(uint32_t) << kMaxPartsLog2 : 0)
-                                     : (hint && n > 0 ? sizeof(uint32_t) * hreq : 0),
-                             grouped ? 0u : ~0u}};
+                            {L.lam, hint && n > 0 ? sizeof(uint32_t) * hreq : 0, ~0u}};
     return fill_many_async(zf, 4, s) == PTC_OK && carry_errors(carry_err, n_carry, L.st, s) == PTC_OK;
   };
   auto run = [&](uint32_t log2m, uint64_t probe_cap) -> bool {
     const ulonglong2* k = reinterpret_cast<const ulonglong2*>(keys);
     const uint32_t n32 = (uint32_t)n;
-    if (grouped) {
-      // 2^21-slot partitions (32 MB of table each), or 16 partitions of a
-      // table of at most 2^25 slots (log2m is at least 10)
-      const uint32_t pshift = log2m > kPartSliceLog2 + 4 ? kPartSliceLog2 : log2m - 4;
-      const uint32_t nparts = 1u << (log2m - pshift);
-      const uint32_t pgrid = ceil_div_u32(n, kPtThreads * kPtPer);
-      PTC_KERNEL("k_part_count", s, k_part_count, pgrid, kPtThreads, 0, k, n32, n_dev, ic, log2m, pshift, nparts,
-                 L.pcount);
-      PTC_KERNEL("k_part_scan", s, k_part_scan, 1, 32, 0, L.pcount, nparts, L.pcursor);
-      PTC_KERNEL("k_part_scatter", s, k_part_scatter, pgrid, kPtThreads, 0, k, n32, n_dev, ic, log2m, pshift, nparts,
-                 L.pcursor, L.pkey, L.pidx);
-      PTC_KERNEL("k_ids_insert_part", s, k_ids_insert_part, ceil_div_u32(n, kInsThreads), kInsThreads, 0, L.pkey, L.pidx,
-                 n32, n_dev, L.table, log2m, probe_cap, L.slot_of, L.st);
-    } else if (hint) {
+    if (hint) {
       PTC_KERNEL("k_tile_req", s, k_tile_req, ceil_div_u32((n >> kReqTileLog2) + 2, 256), 256, 0, ph, n32, n_dev);
       PTC_KERNEL("k_ids_insert_prior", s, k_ids_insert_prior<kPriorK>, ceil_div_u32(n, kInsThreads * kPriorK),
                  kInsThreads, 0, k, n32, n_dev, L.table, log2m, probe_cap, L.slot_of, L.st, ic, ph);
@@ -803,11 +586,7 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
                n32, n_dev, L.st);
     if (bitmap_ranks(L.bits, L.nwords, L.wpre, L.tcnt, L.tpre, &L.done[0], &L.st->value[0], s) != PTC_OK)
       return false;
-    if (grouped)
-      PTC_KERNEL("k_ids_gather_part", s, k_ids_gather_part, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of,
-                 L.pidx, L.table, L.bits, L.wpre, n32, n_dev, ids_out);
-    else
-      PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of,
+    PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of,
                  L.table, m, L.bits, L.wpre, n32, n_dev, ids_out, L.st);
     if (hint)
       PTC_KERNEL("k_ids_follow", s, k_ids_follow, ceil_div_u32(hint->n_req, kFoThreads / 32), kFoThreads, 0, ph,
@@ -849,19 +628,12 @@ extern "C" ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t*
                        nullptr, 0);
 }
 
-extern "C" ptc_status ptc_assign_ids_ex(const ptc_u128* keys, uint64_t n, uint32_t* ids_out,
-                                        uint64_t* n_distinct_host_out, int method, void* ws, size_t ws_bytes,
-                                        void* stream) {
-  return ptc::ids_impl(keys, n, nullptr, ids_out, nullptr, n_distinct_host_out, ws, ws_bytes, (cudaStream_t)stream,
-                       nullptr, 0, nullptr, nullptr, nullptr, false, method);
-}
-
 bool ptc::ids_table_in_dram(uint64_t n) { return n / 3 + 64 > (1ULL << kL2TableLog2); }
 
-size_t ptc::ids_ws_bytes(uint64_t n, uint32_t n_req_hint) { return ids_layout(nullptr, n, false, n_req_hint).total; }
+size_t ptc::ids_ws_bytes(uint64_t n, uint32_t n_req_hint) { return ids_layout(nullptr, n, n_req_hint).total; }
 
 extern "C" size_t ptc_assign_ids_prior_workspace_bytes(uint64_t n, uint32_t n_req) {
-  return ids_layout(nullptr, n, false, n_req ? n_req : 1).total;
+  return ids_layout(nullptr, n, n_req ? n_req : 1).total;
 }
 
 extern "C" ptc_status ptc_assign_ids_prior(const ptc_u128* keys, uint64_t n, const uint64_t* req_blk_off,
@@ -873,7 +645,7 @@ extern "C" ptc_status ptc_assign_ids_prior(const ptc_u128* keys, uint64_t n, con
                          (cudaStream_t)stream, nullptr, 0);
   const IdsHint h{req_blk_off, req_prior, n_req};
   return ptc::ids_impl(keys, n, nullptr, ids_out, nullptr, n_distinct_host_out, ws, ws_bytes, (cudaStream_t)stream,
-                       nullptr, 0, nullptr, nullptr, nullptr, false, PTC_IDS_AUTO, &h);
+                       nullptr, 0, nullptr, nullptr, nullptr, false, &h);
 }
 
 size_t ptc::session_prior_bytes(uint32_t n_req) {

@@ -220,7 +220,7 @@ ptc_status ids_impl(const ptc_u128* keys, uint64_t n_ub, const uint64_t* n_dev, 
                     uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
                     cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc = nullptr,
                     uint64_t* nd_slot = nullptr, uint32_t* err_slot = nullptr, bool full_table = false,
-                    int method = PTC_IDS_AUTO, const IdsHint* hint = nullptr);
+                    const IdsHint* hint = nullptr);
 ptc_status stack_distance_view(const uint32_t* prev, uint64_t n, uint32_t* dist_out, int method, void* ws,
                                size_t ws_bytes, cudaStream_t s, RunsView* view, uint32_t* defer_err);
 // Stage b as ptc_reuse_indices does it (ptc_reuse.cu); with `defer_err` the

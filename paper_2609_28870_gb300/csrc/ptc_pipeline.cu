@@ -119,7 +119,7 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
                                  &unused, L.scratch, L.scratch_bytes, s, L.n_slot, &L.defer[0], kcp);
   if (rc != PTC_OK) return rc;
   rc = ptc::ids_impl(keys, cap, L.n_slot, ids, &n, &d, L.scratch, L.scratch_bytes, s, &L.defer[0], 2, kcp,
-                     L.nd_slot, &L.defer[4], false, PTC_IDS_AUTO, hp);
+                     L.nd_slot, &L.defer[4], false, hp);
   if (rc != PTC_OK) return rc;
   const ptc::ReuseDevIn din{L.nd_slot, &L.defer[4]};
   ptc::ReuseHostOut hout;
@@ -132,7 +132,7 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
     // full table, waiting for it, then stage b with the host's N and D
     if (hout.ids_err != ptc::kErrTableFull) return ptc::status_of(hout.ids_err);
     rc = ptc::ids_impl(keys, cap, L.n_slot, ids, &n, &d, L.scratch, L.scratch_bytes, s, &L.defer[0], 2, kcp, nullptr,
-                       nullptr, true, PTC_IDS_AUTO, hp);
+                       nullptr, true, hp);
     *n_access_host_out = n;
     *n_distinct_host_out = d;
     if (rc != PTC_OK) return rc;

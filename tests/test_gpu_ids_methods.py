@@ -1,7 +1,7 @@
-"""Both insert orders of the id stage (keys in access order, and keys grouped
-by the table partition of their home slot) against the oracle's exact ids,
-bit-exact.  The keys come from the oracle's own prefix hash, so this checks
-the id stage alone."""
+"""The id stage (ptc_assign_ids) against the oracle's exact ids, bit-exact.
+The keys come from the oracle's own prefix hash, so this checks the id stage
+alone: tiny traces, workload prefixes, all-distinct keys (the table's largest
+fill), one key repeated, and a key that is not a field element."""
 import numpy as np
 import pytest
 
@@ -29,10 +29,9 @@ def _check_all(tr, B, seed=0):
     import paper_2609_28870_gb300 as ptc
     want, D = oracle.block_ids(tr.tokens, tr.req_tok_off, B)
     keys = _keys(oracle.prefix_hash(tr.tokens, tr.req_tok_off, B, seed)).view(-1, 2)
-    for m in (None, ptc.PTC_IDS_AUTO, ptc.PTC_IDS_DIRECT, ptc.PTC_IDS_GROUPED):
-        ids, d = ptc.ptc_assign_ids(keys, method=m)
-        assert d == D, m
-        assert np.array_equal(ptc.u32(ids), want), m
+    ids, d = ptc.ptc_assign_ids(keys)
+    assert d == D
+    assert np.array_equal(ptc.u32(ids), want)
 
 
 @pytest.mark.parametrize("seed", range(12))
@@ -56,23 +55,18 @@ def test_all_distinct_and_all_equal_keys():
     distinct = rng.integers(0, (1 << 61) - 1, size=(20000, 2), dtype=np.uint64)
     same = np.repeat(distinct[:1], 5000, axis=0)
     for k, want_d in ((distinct, 20000), (same, 1)):
-        for m in (ptc.PTC_IDS_DIRECT, ptc.PTC_IDS_GROUPED):
-            ids, d = ptc.ptc_assign_ids(_keys(k).view(-1, 2), method=m)
-            assert d == want_d
-            got = ptc.u32(ids)
-            if want_d == 1:
-                assert not got.any()
-            else:
-                assert np.array_equal(got, np.arange(20000, dtype=np.uint32))
+        ids, d = ptc.ptc_assign_ids(_keys(k).view(-1, 2))
+        assert d == want_d
+        got = ptc.u32(ids)
+        if want_d == 1:
+            assert not got.any()
+        else:
+            assert np.array_equal(got, np.arange(20000, dtype=np.uint32))
 
 
-def test_invalid_method_and_invalid_key():
+def test_invalid_key():
     import paper_2609_28870_gb300 as ptc
-    keys = _keys(np.array([[1, 2], [3, 4]], dtype=np.uint64)).view(-1, 2)
-    with pytest.raises(ptc.PtcError) as e:
-        ptc.ptc_assign_ids(keys, method=7)
-    assert e.value.name == "PTC_ERR_INVALID_ARG"
     bad = _keys(np.array([[1, 2], [(1 << 61) - 1, 4]], dtype=np.uint64)).view(-1, 2)  # not a field element
     with pytest.raises(ptc.PtcError) as e:
-        ptc.ptc_assign_ids(bad, method=ptc.PTC_IDS_GROUPED)
+        ptc.ptc_assign_ids(bad)
     assert e.value.name == "PTC_ERR_INVALID_ARG"
