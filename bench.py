@@ -175,9 +175,9 @@ def kernel_model_bytes(name, T, N, L, D):
 KERNEL_SOURCE = {
     "k_block_offsets": "ptc_hash.cu", "k_pow_tables": "ptc_hash.cu", "k_hash_local": "ptc_hash.cu",
     "k_hash16": "ptc_hash.cu", "k_hash_tile": "ptc_hash.cu", "k_fill_many": "ptc_abi.cu",
-    "k_hash_chain": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu", "k_ids_mark": "ptc_ids.cu",
+    "k_hash_chain": "ptc_hash.cu", "k_ids_insert": "ptc_ids.cu",
     "k_ids_gather": "ptc_ids.cu", "k_ids_insert_prior": "ptc_ids.cu", "k_ids_follow": "ptc_ids.cu",
-    "k_tile_req": "ptc_ids.cu", "k_session_prior": "ptc_ids.cu", "k_sort_count": "ptc_sort.cu", "k_sort_rowscan": "ptc_sort.cu",
+    "k_tile_req": "ptc_ids.cu", "k_ids_lam": "ptc_ids.cu", "k_session_prior": "ptc_ids.cu", "k_sort_count": "ptc_sort.cu", "k_sort_rowscan": "ptc_sort.cu",
     "k_sort_scatter": "ptc_sort.cu", "k_sort_links": "ptc_sort.cu", "k_ir_count": "ptc_reuse.cu",
     "k_ir_mark": "ptc_reuse.cu", "k_bm_count": "ptc_reuse.cu", "k_bm_words": "ptc_reuse.cu",
     "k_ir_inc1": "ptc_reuse.cu", "k_ir_inc2": "ptc_reuse.cu", "k_ir_fill": "ptc_reuse.cu", "k_wm_count0": "ptc_wavelet.cu",

@@ -154,13 +154,19 @@ ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t* ids_out, u
  * that saves table probes.  Sec. 2.3: a turn of a multi-turn session sends
  * the whole context again, so request r usually repeats every block of an
  * earlier request of its session and appends to it.  req_prior[r] names such
- * an earlier request (or PTC_NONE).  An access whose key equals that of the
- * same depth of req_prior[r] is a repeat: it is not inserted into the table
- * and takes its id from the prior request's chain; only the other accesses
- * are inserted.  The ids are exactly those of ptc_assign_ids for ANY hint
- * with req_prior[r] < r or PTC_NONE (a poor hint only costs probes);
- * req_prior[r] >= r is PTC_ERR_INVALID_ARG.
- *   keys         ptc_u128[n] as for ptc_assign_ids
+ * an earlier request (or PTC_NONE).  The leading depths of r whose keys
+ * equal those of the same depths of req_prior[r] are repeats: they are not
+ * inserted into the table and take their ids from the prior request's chain;
+ * only the other accesses are inserted.  The keys must be prefix keys as
+ * ptc_hash_blocks writes them (equal keys at depth k imply equal keys at
+ * every depth below k), so the end of that leading run is found by a binary
+ * search over the depths, reading about 2 log2(n_r) keys per request rather
+ * than the prior request's key of every access.  The ids are then exactly
+ * those of ptc_assign_ids for ANY hint with req_prior[r] < r or PTC_NONE (a
+ * poor hint only costs probes); req_prior[r] >= r is PTC_ERR_INVALID_ARG.
+ * A key that is not a field element is reported when it is inserted; the
+ * keys of repeated depths are only compared.
+ *   keys         ptc_u128[n] as for ptc_assign_ids, prefix keys
  *   req_blk_off  u64[n_req + 1] from ptc_hash_blocks (req_blk_off[n_req] == n)
  *   req_prior    u32[n_req]
  */

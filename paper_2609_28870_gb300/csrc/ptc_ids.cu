@@ -6,12 +6,16 @@
 //                  smallest access index seen.  A slot is read first; only an
 //                  empty (or half-written) slot is claimed with one 128-bit
 //                  CAS, and a stored index above i is lowered with atomicMin.
-//                  Linear probing.
-//   k_ids_mark     one pass over the slots: each filled slot's index is a
-//                  first occurrence; a bitmap of those over positions
+//                  Linear probing.  Each claim and each lowering toggles bits
+//                  of the first-occurrence bitmap over positions, which ends
+//                  with exactly the smallest index of every key set.
 //   bitmap_ranks   first occurrences before every 32-position word, and D
-//   k_ids_gather   ids[i] = rank, among the first occurrences, of the index
-//                  stored in i's slot.
+//   k_ids_gather   ids[i] = rank, among the first occurrences, of i itself
+//                  if its bit is set, else of the index stored in i's slot.
+// With a prior-request hint (ptc_assign_ids_prior), k_ids_lam finds the
+// leading depths of each request that repeat the hinted request, which skip
+// the table (k_ids_insert_prior) and take their ids along the hint chain
+// (k_ids_follow).
 // ptc_verify_ids
 //   k_verify_first first access of every id (atomicMin)
 //   k_verify       compares every access's B tokens and parent id with those
@@ -57,18 +61,36 @@ __device__ __forceinline__ uint32_t keys_used(uint32_t n, const uint64_t* n_dev)
   return v < n ? (uint32_t)v : n;
 }
 
+// Block 0 reports the number of keys used (value[1]); a count above the
+// keys buffer is malformed input.
+__device__ __forceinline__ void report_keys_used(uint32_t n_ub, const uint64_t* n_dev, DevStatus* st) {
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    st->value[1] = n_dev ? *n_dev : n_ub;
+    if (n_dev && *n_dev > n_ub) raise_err(st, kErrInvalid);
+  }
+}
+
 constexpr int kInsK = 1;  // keys per thread: their key and slot loads are in flight together
 
 // Settle the key k of access i, whose home slot `pos` was read as `cur`:
 // claim an empty (or half-written) slot with one 128-bit CAS, or find the
 // key's slot and lower its stored index to i if it is above; linear probing.
 // The slot goes to *slot_out.
+// The first-occurrence bitmap is kept as the table changes: every index that
+// becomes a slot's stored index toggles its bit, and so does every index that
+// an atomicMin replaces (the atomicMin's return value names it, to one thread
+// only).  An index that is stored and later replaced is toggled twice, the
+// final one once, and XOR does not depend on the order in which the toggles
+// land, so once all keys are settled the set bits are exactly the smallest
+// index of every key.
 // 96 key bits: all of h0 (61) + 35 bits of h1.  Word 0 is never all-ones
 // because h0 < 2^61 - 1, and word 1 of a filled slot holds an index below
 // 2^32 - 1, so an all-ones word marks an empty or half-written slot.
+__device__ __forceinline__ void toggle(uint32_t* bits, uint32_t i) { atomicXor(&bits[i >> 5], 1u << (i & 31)); }
+
 __device__ __forceinline__ void settle(ulonglong2* table, uint64_t mask, uint64_t probe_cap, uint32_t i,
                                        ulonglong2 k, uint64_t pos, ulonglong2 cur, uint32_t* __restrict__ slot_out,
-                                       DevStatus* st) {
+                                       uint32_t* bits, DevStatus* st) {
   const uint64_t w0 = k.x | ((k.y & 7ULL) << 61);
   const uint32_t w1lo = (uint32_t)(k.y >> 3);
   const ulonglong2 mine = make_ulonglong2(w0, (uint64_t)w1lo | ((uint64_t)i << 32));
@@ -77,12 +99,19 @@ __device__ __forceinline__ void settle(ulonglong2* table, uint64_t mask, uint64_
     if (cur.x == ~0ULL || cur.y == ~0ULL) {  // empty, or being filled: settle it with the CAS
       cur = cas128(&table[pos], empty, mine);
       if (cur.x == ~0ULL && cur.y == ~0ULL) {
+        toggle(bits, i);
         __stcs(slot_out, (uint32_t)pos);
         return;
       }
     }
     if (cur.x == w0 && (uint32_t)cur.y == w1lo) {
-      if ((uint32_t)(cur.y >> 32) > i) atomicMin(reinterpret_cast<uint32_t*>(&table[pos]) + 3, i);
+      if ((uint32_t)(cur.y >> 32) > i) {
+        const uint32_t old = atomicMin(reinterpret_cast<uint32_t*>(&table[pos]) + 3, i);
+        if (old > i) {
+          toggle(bits, i);
+          toggle(bits, old);
+        }
+      }
       __stcs(slot_out, (uint32_t)pos);
       return;
     }
@@ -107,8 +136,9 @@ struct InsCarry {
 __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __restrict__ keys, uint32_t n_ub,
                                                             const uint64_t* n_dev, ulonglong2* table, uint32_t log2m,
                                                             uint64_t probe_cap, uint32_t* __restrict__ slot_of,
-                                                            DevStatus* st, InsCarry kc) {
+                                                            uint32_t* bits, DevStatus* st, InsCarry kc) {
   grid_dep_sync();
+  report_keys_used(n_ub, n_dev, st);
   const uint32_t i0 = blockIdx.x * (kInsThreads * kInsK) + threadIdx.x;
   const uint64_t mask = (1ULL << log2m) - 1;
   ulonglong2 k[kInsK], cur[kInsK], cy[kInsK];
@@ -153,44 +183,16 @@ __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __
       slot_of[i] = 0;
       continue;
     }
-    settle(table, mask, probe_cap, i, k[j], pos[j], cur[j], &slot_of[i], st);
-  }
-}
-
-// First occurrences from the table itself: every filled slot holds the
-// smallest access index of its key, so one pass over the slots (coalesced,
-// mostly in L2) marks the first-occurrence bitmap over access positions.
-// Block 0 also reports the number of keys used (value[1]).
-constexpr int kMkThreads = 256;
-constexpr int kMkPer = 8;
-__global__ void __launch_bounds__(kMkThreads) k_ids_mark(const ulonglong2* __restrict__ table, uint64_t m,
-                                                        uint32_t* __restrict__ bits, uint32_t n_ub,
-                                                        const uint64_t* n_dev, DevStatus* st) {
-  grid_dep_sync();
-  if (blockIdx.x == 0 && threadIdx.x == 0) {
-    st->value[1] = n_dev ? *n_dev : n_ub;
-    if (n_dev && *n_dev > n_ub) raise_err(st, kErrInvalid);  // more blocks than the keys buffer holds
-  }
-  const uint64_t s0 = (uint64_t)blockIdx.x * (kMkThreads * kMkPer) + threadIdx.x;
-  ulonglong2 v[kMkPer];
-#pragma unroll
-  for (int k = 0; k < kMkPer; ++k) {
-    const uint64_t sl = s0 + (uint64_t)k * kMkThreads;
-    v[k] = sl < m ? __ldg(&table[sl]) : make_ulonglong2(~0ULL, ~0ULL);  // the gather reads it again
-  }
-#pragma unroll
-  for (int k = 0; k < kMkPer; ++k) {
-    if (v[k].x != ~0ULL && v[k].y != ~0ULL) {
-      const uint32_t f = (uint32_t)(v[k].y >> 32);
-      if (in_bounds(st, f, n_ub)) atomicOr(&bits[f >> 5], 1u << (f & 31));
-    }
+    settle(table, mask, probe_cap, i, k[j], pos[j], cur[j], &slot_of[i], bits, st);
   }
 }
 
 // ids[i] = rank of the first occurrence of i's key among all first
-// occurrences: the slot gives the first occurrence, the bitmap's word
-// prefixes its rank.  kGaPer accesses per thread, kGaThreads apart, their
-// dependent loads in flight together.
+// occurrences, the bitmap's word prefixes giving ranks.  A first occurrence
+// finds its own bit set and is its own first occurrence, with no table read
+// (its bitmap word is shared with its neighbours, so the read is coalesced);
+// a later occurrence reads its slot's stored index.  kGaPer accesses per
+// thread, kGaThreads apart, their dependent loads in flight together.
 constexpr int kGaThreads = 256;
 constexpr int kGaPer = 8;
 // slot_of of an access that the prior-request hint matched (no slot)
@@ -204,25 +206,29 @@ __global__ void __launch_bounds__(kGaThreads) k_ids_gather(const uint32_t* __res
   grid_dep_sync();
   const uint32_t n = keys_used(n_ub, n_dev);
   const uint32_t i0 = blockIdx.x * (kGaThreads * kGaPer) + threadIdx.x;
-  uint32_t f[kGaPer];
+  uint32_t f[kGaPer], own[kGaPer];
 #pragma unroll
   for (int k = 0; k < kGaPer; ++k) {
     const uint32_t i = i0 + k * kGaThreads;
-    f[k] = i < n ? __ldcs(&slot_of[i]) : 0u;
+    f[k] = i < n ? __ldcs(&slot_of[i]) : kMatchedSlot;
+    own[k] = i < n ? bits[i >> 5] : 0u;
   }
 #pragma unroll
   for (int k = 0; k < kGaPer; ++k) {
     const uint32_t i = i0 + k * kGaThreads;
-    f[k] = i < n && f[k] != kMatchedSlot && in_bounds(st, f[k], m)
-               ? __ldg(reinterpret_cast<const uint32_t*>(&table[f[k]]) + 3)
-               : kMatchedSlot;
+    if (f[k] == kMatchedSlot) continue;
+    if ((own[k] >> (i & 31)) & 1u)
+      f[k] = i;
+    else
+      f[k] = in_bounds(st, f[k], m) ? __ldg(reinterpret_cast<const uint32_t*>(&table[f[k]]) + 3) : kNone;
   }
   uint32_t wp[kGaPer], bw[kGaPer];
 #pragma unroll
   for (int k = 0; k < kGaPer; ++k) {
+    const uint32_t i = i0 + k * kGaThreads;
     const bool ok = f[k] < n;
     wp[k] = ok ? wpre[f[k] >> 5] : 0u;
-    bw[k] = ok ? bits[f[k] >> 5] : 0u;
+    bw[k] = f[k] == i ? own[k] : ok ? bits[f[k] >> 5] : 0u;
   }
   // a matched access (prior-request hint) gets its id from k_ids_follow
 #pragma unroll
@@ -255,7 +261,7 @@ __device__ __forceinline__ ulonglong2 carried_key(const ulonglong2* __restrict__
 // access (r, k) is "matched" when its key equals that of block k of request
 // prior[r]: its prefix occurred earlier, so it is not a first occurrence and
 // is not inserted.  Equal keys mean equal prefixes, so the matched blocks of
-// r are its depths k < lam[r].  A first occurrence is never matched, so the
+// r are its depths k < lam[r] (k_ids_lam).  A first occurrence is never matched, so the
 // table of the unmatched keys still holds every key with its smallest access
 // index.  A matched access takes the id of block k of the nearest request on
 // its prior chain whose depth k is unmatched (k_ids_follow).  The ids do not
@@ -267,7 +273,7 @@ struct PriorHint {
   const uint64_t* blk_off;  // n_req + 1 access offsets of the requests
   const uint32_t* prior;    // n_req: an earlier request, or kNone
   uint32_t n_req;
-  uint32_t* lam;            // n_req: first unmatched depth, kNone if none (cleared to kNone)
+  uint32_t* lam;            // n_req: first unmatched depth (written by k_ids_lam)
   uint32_t* tile_req;       // request of the first access of every kReqTile accesses, and n_req - 1 last
 };
 constexpr uint32_t kReqTileLog2 = 11;  // 2048 accesses per entry of tile_req
@@ -297,66 +303,86 @@ __global__ void k_tile_req(PriorHint ph, uint32_t n_ub, const uint64_t* n_dev) {
   if (t == T) ph.tile_req[t] = ph.n_req - 1;
 }
 
-// kPriorK keys per thread, kInsThreads apart.  Each access finds its request
-// by binary search among the few requests its 2048-access tile spans
-// (tile_req).  A matched access writes kMatched and stops; an unmatched one
-// lowers its request's lam (one atomic per group of lanes in one request) and
-// settles its key in the table as k_ids_insert does.  The keys' loads, then
-// the previous requests' keys, then the slot loads of all unmatched keys go
-// out together, so a thread has kPriorK independent probes in flight.
+// lam[r], one thread per request: the number of leading depths at which r's
+// key equals that of prior[r] (the keys of both requests, as far as the
+// shorter one goes).  The keys are prefix keys: equal keys at depth k mean
+// equal prefixes through block k, hence equal keys at every depth below k,
+// so the equal depths are a leading run and a binary search over the depths
+// finds its end in about log2(n_r) pairs of key reads instead of one pair
+// per access.  A request with no hint, or none of whose blocks the hint
+// repeats, gets 0.  A hint that does not point to an earlier request, or
+// offsets that do not fit the keys, raise kErrInvalid.
+constexpr int kLamThreads = 256;
+__global__ void __launch_bounds__(kLamThreads) k_ids_lam(const ulonglong2* __restrict__ keys, uint32_t n_ub,
+                                                         const uint64_t* n_dev, InsCarry kc, PriorHint ph,
+                                                         DevStatus* st) {
+  grid_dep_sync();
+  const uint32_t r = blockIdx.x * kLamThreads + threadIdx.x;
+  if (r >= ph.n_req) return;
+  const uint32_t n = keys_used(n_ub, n_dev);
+  const uint32_t p = __ldg(&ph.prior[r]);
+  uint64_t lam = 0;
+  if (p != kNone && p >= r) {
+    raise_err(st, kErrInvalid);  // a hint must point to an earlier request
+  } else if (p != kNone) {
+    const uint64_t b = __ldg(&ph.blk_off[r]), e = __ldg(&ph.blk_off[r + 1]);
+    const uint64_t pb = __ldg(&ph.blk_off[p]), pe = __ldg(&ph.blk_off[p + 1]);
+    if (b > e || pb > pe || e > n || pe > n) {
+      raise_err(st, kErrInvalid);
+    } else {
+      uint64_t hi = e - b < pe - pb ? e - b : pe - pb;  // depths below lam are equal, depth hi is not (or the end)
+      while (lam < hi) {
+        const uint64_t mid = (lam + hi) >> 1;
+        const ulonglong2 x = carried_key(keys, (uint32_t)(b + mid), n, kc);
+        const ulonglong2 y = carried_key(keys, (uint32_t)(pb + mid), n, kc);
+        if (x.x == y.x && x.y == y.y && x.x < kP61 && x.y < kP61)  // a key that is not a field element is never equal
+          lam = mid + 1;
+        else
+          hi = mid;
+      }
+    }
+  }
+  ph.lam[r] = (uint32_t)lam;
+}
+
+// kPriorK accesses per thread, kInsThreads apart.  Each access finds its
+// request by binary search among the few requests its 2048-access tile
+// spans (tile_req); a depth below its request's lam repeats the hint and
+// writes kMatched without reading its key; any other access settles its key
+// in the table as k_ids_insert does.  The request searches, then the keys and
+// slot loads of the unmatched accesses go out together.
 constexpr int kPriorK = 1;
 template <int K>
 __global__ void __launch_bounds__(kInsThreads) k_ids_insert_prior(const ulonglong2* __restrict__ keys, uint32_t n_ub,
                                                                   const uint64_t* n_dev, ulonglong2* table,
                                                                   uint32_t log2m, uint64_t probe_cap,
-                                                                  uint32_t* __restrict__ slot_of, DevStatus* st,
-                                                                  InsCarry kc, PriorHint ph) {
+                                                                  uint32_t* __restrict__ slot_of, uint32_t* bits,
+                                                                  DevStatus* st, InsCarry kc, PriorHint ph) {
   grid_dep_sync();
+  report_keys_used(n_ub, n_dev, st);
   const uint32_t n = keys_used(n_ub, n_dev);
   const uint32_t base = blockIdx.x * (kInsThreads * K) + threadIdx.x;
   if (blockIdx.x * (kInsThreads * K) >= n) return;  // the whole CTA
-  ulonglong2 k[K], q[K];
-  uint32_t r[K];
-  uint64_t depth[K];
-  bool live[K], unm[K];
+  bool unm[K];
 #pragma unroll
   for (int j = 0; j < K; ++j) {
     const uint32_t i = base + j * kInsThreads;
-    live[j] = i < n;
-    k[j] = carried_key(keys, i, n, kc);
-  }
-#pragma unroll
-  for (int j = 0; j < K; ++j) {
-    const uint32_t i = base + j * kInsThreads;
-    r[j] = 0;
-    depth[j] = 0;
-    q[j] = make_ulonglong2(~0ULL, ~0ULL);
-    unm[j] = live[j];
-    if (!live[j]) continue;
-    if (k[j].x >= kP61 || k[j].y >= kP61) {
-      raise_err(st, kErrInvalid);
-      slot_of[i] = 0;
-      live[j] = unm[j] = false;
-      continue;
-    }
+    unm[j] = false;
+    if (i >= n) continue;
     const uint32_t t = i >> kReqTileLog2;
-    r[j] = req_at(ph.blk_off, __ldg(&ph.tile_req[t]), __ldg(&ph.tile_req[t + 1]), i);
-    depth[j] = i - __ldg(&ph.blk_off[r[j]]);
-    const uint32_t p = __ldg(&ph.prior[r[j]]);
-    if (p == kNone) continue;
-    if (p >= r[j]) {
-      raise_err(st, kErrInvalid);  // a hint must point to an earlier request
-      continue;
-    }
-    const uint64_t pb = __ldg(&ph.blk_off[p]), pn = __ldg(&ph.blk_off[p + 1]) - pb;
-    if (depth[j] < pn && pb + depth[j] < n) q[j] = carried_key(keys, (uint32_t)(pb + depth[j]), n, kc);
+    const uint32_t r = req_at(ph.blk_off, __ldg(&ph.tile_req[t]), __ldg(&ph.tile_req[t + 1]), i);
+    unm[j] = i - __ldg(&ph.blk_off[r]) >= __ldg(&ph.lam[r]);
+    if (!unm[j]) __stcs(&slot_of[i], kMatched);
   }
-  ulonglong2 cur[K];
+  ulonglong2 k[K], cur[K];
   uint64_t pos[K];
 #pragma unroll
   for (int j = 0; j < K; ++j) {
-    if (live[j] && q[j].x == k[j].x && q[j].y == k[j].y) {
-      __stcs(&slot_of[base + j * kInsThreads], kMatched);
+    const uint32_t i = base + j * kInsThreads;
+    k[j] = unm[j] ? carried_key(keys, i, n, kc) : make_ulonglong2(0, 0);
+    if (unm[j] && (k[j].x >= kP61 || k[j].y >= kP61)) {
+      raise_err(st, kErrInvalid);
+      slot_of[i] = 0;
       unm[j] = false;
     }
     pos[j] = home_slot(k[j].x, k[j].y, log2m);
@@ -364,13 +390,9 @@ __global__ void __launch_bounds__(kInsThreads) k_ids_insert_prior(const ulonglon
   }
 #pragma unroll
   for (int j = 0; j < K; ++j) {
-    const uint32_t am = __ballot_sync(kFull, unm[j]);
     if (!unm[j]) continue;
-    const unsigned grp = __match_any_sync(am, r[j]);
-    const uint32_t lo = __reduce_min_sync(grp, (uint32_t)depth[j]);
-    if ((threadIdx.x & 31) == (uint32_t)(__ffs(grp) - 1)) atomicMin(&ph.lam[r[j]], lo);
     settle(table, (1ULL << log2m) - 1, probe_cap, base + j * kInsThreads, k[j], pos[j], cur[j],
-           &slot_of[base + j * kInsThreads], st);
+           &slot_of[base + j * kInsThreads], bits, st);
   }
 }
 
@@ -396,7 +418,7 @@ __global__ void __launch_bounds__(kFoThreads) k_ids_follow(PriorHint ph, uint32_
       return;
     }
     const uint64_t tb = ph.blk_off[t];
-    const uint64_t lo = ph.lam[t];  // kNone (no unmatched depth) is above every hi
+    const uint64_t lo = ph.lam[t];  // depths [lo, n_t) of t are unmatched
     if (lo < hi) {
       if (!in_bounds(st, tb + hi - 1, b) || !in_bounds(st, b + hi - 1, ph.blk_off[ph.n_req])) return;
       for (uint64_t d = lo + lane; d < hi; d += 32) ids[b + d] = ids[tb + d];
@@ -561,29 +583,28 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
   const IdsLayout L = ids_layout(ws, n, hreq);
   const PriorHint ph = hint ? PriorHint{hint->blk_off, hint->prior, hint->n_req, L.lam, L.tile_req}
                             : PriorHint{nullptr, nullptr, 0, nullptr, nullptr};
-  // the status block, the table (all ones: empty), the first-occurrence
-  // bitmap and the hint's first unmatched depths are cleared by one launch
+  // the status block, the table (all ones: empty) and the first-occurrence
+  // bitmap are cleared by one launch
   auto start = [&](uint32_t log2m) -> bool {
-    const FillRange zf[4] = {{ws, L.zero_bytes, 0u},
+    const FillRange zf[3] = {{ws, L.zero_bytes, 0u},
                             {L.table, n > 0 ? sizeof(ulonglong2) << log2m : 0, ~0u},
-                            {L.bits, n > 0 ? sizeof(uint32_t) * L.nwords : 0, 0u},
-                            {L.lam, hint && n > 0 ? sizeof(uint32_t) * hreq : 0, ~0u}};
-    return fill_many_async(zf, 4, s) == PTC_OK && carry_errors(carry_err, n_carry, L.st, s) == PTC_OK;
+                            {L.bits, n > 0 ? sizeof(uint32_t) * L.nwords : 0, 0u}};
+    return fill_many_async(zf, 3, s) == PTC_OK && carry_errors(carry_err, n_carry, L.st, s) == PTC_OK;
   };
   auto run = [&](uint32_t log2m, uint64_t probe_cap) -> bool {
     const ulonglong2* k = reinterpret_cast<const ulonglong2*>(keys);
     const uint32_t n32 = (uint32_t)n;
     if (hint) {
       PTC_KERNEL("k_tile_req", s, k_tile_req, ceil_div_u32((n >> kReqTileLog2) + 2, 256), 256, 0, ph, n32, n_dev);
+      PTC_KERNEL("k_ids_lam", s, k_ids_lam, ceil_div_u32(hint->n_req, kLamThreads), kLamThreads, 0, k, n32, n_dev, ic,
+                 ph, L.st);
       PTC_KERNEL("k_ids_insert_prior", s, k_ids_insert_prior<kPriorK>, ceil_div_u32(n, kInsThreads * kPriorK),
-                 kInsThreads, 0, k, n32, n_dev, L.table, log2m, probe_cap, L.slot_of, L.st, ic, ph);
+                 kInsThreads, 0, k, n32, n_dev, L.table, log2m, probe_cap, L.slot_of, L.bits, L.st, ic, ph);
     } else {
       PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads * kInsK), kInsThreads, 0, k, n32, n_dev,
-                 L.table, log2m, probe_cap, L.slot_of, L.st, ic);
+                 L.table, log2m, probe_cap, L.slot_of, L.bits, L.st, ic);
     }
     const uint64_t m = 1ULL << log2m;
-    PTC_KERNEL("k_ids_mark", s, k_ids_mark, ceil_div_u32(m, kMkThreads * kMkPer), kMkThreads, 0, L.table, m, L.bits,
-               n32, n_dev, L.st);
     if (bitmap_ranks(L.bits, L.nwords, L.wpre, L.tcnt, L.tpre, &L.done[0], &L.st->value[0], s) != PTC_OK)
       return false;
     PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of,
