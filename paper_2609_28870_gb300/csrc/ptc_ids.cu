@@ -488,7 +488,6 @@ IdsLayout ids_layout(void* ws, uint64_t n, uint32_t n_req_hint = 0) {
   L.st = cv.take<DevStatus>(1);
   L.done = cv.take<uint32_t>(64);
   L.zero_bytes = cv.off;
-  L.table = cv.take<ulonglong2>(m);
   L.slot_of = cv.take<uint32_t>(nn);
   L.bits = cv.take<uint32_t>(L.nwords + 1);
   L.wpre = cv.take<uint32_t>(L.nwords + 1);
@@ -496,6 +495,10 @@ IdsLayout ids_layout(void* ws, uint64_t n, uint32_t n_req_hint = 0) {
   L.tpre = cv.take<uint32_t>(rank_tiles(L.nwords) + 1);
   L.lam = n_req_hint ? cv.take<uint32_t>(n_req_hint) : nullptr;
   L.tile_req = n_req_hint ? cv.take<uint32_t>((nn >> kReqTileLog2) + 2) : nullptr;
+  // the table last: it starts past every other array of the stage (and past
+  // stage a1's workspace, which the pipeline checks before it has stage a1
+  // fill the table)
+  L.table = cv.take<ulonglong2>(m);
   L.total = cv.bytes();
   return L;
 }
@@ -568,7 +571,8 @@ extern "C" size_t ptc_assign_ids_workspace_bytes(uint64_t n) { return ids_layout
 ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev, uint32_t* ids_out,
                         uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
                         cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc,
-                        uint64_t* nd_slot, uint32_t* err_slot, bool full_table, const IdsHint* hint) {
+                        uint64_t* nd_slot, uint32_t* err_slot, bool full_table, const IdsHint* hint,
+                        bool table_prefilled) {
   if (hint && (hint->n_req == 0 || !hint->blk_off || !hint->prior)) return PTC_ERR_INVALID_ARG;
   if (kc && (kc->tile_blocks == 0 || (kc->tile_blocks & (kc->tile_blocks - 1)) != 0)) return PTC_ERR_INVALID_ARG;
   const InsCarry ic = kc ? InsCarry{kc->carry, kc->lead, (uint32_t)__builtin_ctz(kc->tile_blocks)}
@@ -585,9 +589,13 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
                             : PriorHint{nullptr, nullptr, 0, nullptr, nullptr};
   // the status block, the table (all ones: empty) and the first-occurrence
   // bitmap are cleared by one launch
+  // the table of the first attempt may come already filled (ids_table_region)
+  bool prefilled = table_prefilled;
   auto start = [&](uint32_t log2m) -> bool {
+    const bool fill_table = n > 0 && !prefilled;
+    prefilled = false;
     const FillRange zf[3] = {{ws, L.zero_bytes, 0u},
-                            {L.table, n > 0 ? sizeof(ulonglong2) << log2m : 0, ~0u},
+                            {L.table, fill_table ? sizeof(ulonglong2) << log2m : 0, ~0u},
                             {L.bits, n > 0 ? sizeof(uint32_t) * L.nwords : 0, 0u}};
     return fill_many_async(zf, 3, s) == PTC_OK && carry_errors(carry_err, n_carry, L.st, s) == PTC_OK;
   };
@@ -647,6 +655,12 @@ extern "C" ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t*
                                      void* ws, size_t ws_bytes, void* stream) {
   return ptc::ids_impl(keys, n, nullptr, ids_out, nullptr, n_distinct_host_out, ws, ws_bytes, (cudaStream_t)stream,
                        nullptr, 0);
+}
+
+void ptc::ids_table_region(void* ws, uint64_t n, uint32_t n_req_hint, void** table, size_t* bytes) {
+  const IdsLayout L = ids_layout(ws, n, n_req_hint);
+  *table = L.table;
+  *bytes = n > 0 ? sizeof(ulonglong2) << small_table_log2(n) : 0;
 }
 
 bool ptc::ids_table_in_dram(uint64_t n) { return n / 3 + 64 > (1ULL << kL2TableLog2); }

@@ -5,6 +5,8 @@
 // the same stream.  Stage d has a region of its own: when stage c used the
 // matrix over runs, the curves come from those runs (still in stage c's
 // scratch) instead of a pass over every distance.
+#include <algorithm>
+
 #include "ptc_internal.h"
 
 namespace {
@@ -115,11 +117,21 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
   // carry as it reads them
   ptc::KeyCarry kc{L.carry, L.lead, 1};
   ptc::KeyCarry* kcp = keys_out ? nullptr : &kc;
+  // stage a1 is bound by integer issue, so it also fills stage a2's table
+  // (all ones: empty), which lies past stage a1's workspace and the session
+  // sort's in the shared scratch region
+  void* table = nullptr;
+  size_t table_bytes = 0;
+  ptc::ids_table_region(L.scratch, cap, hinted ? n_req : 0, &table, &table_bytes);
+  const size_t front = std::max(ptc_hash_blocks_workspace_bytes(n_req, n_tok, block_size),
+                                ptc::session_prior_bytes(n_req));
+  const bool fused_fill = table_bytes > 0 && static_cast<char*>(table) >= static_cast<char*>(L.scratch) + front;
   ptc_status rc = ptc::hash_impl(tokens, n_tok, req_tok_off, req_ts_us, n_req, block_size, seed, keys, cap, blk,
-                                 &unused, L.scratch, L.scratch_bytes, s, L.n_slot, &L.defer[0], kcp);
+                                 &unused, L.scratch, L.scratch_bytes, s, L.n_slot, &L.defer[0], kcp,
+                                 fused_fill ? table : nullptr, fused_fill ? table_bytes : 0);
   if (rc != PTC_OK) return rc;
   rc = ptc::ids_impl(keys, cap, L.n_slot, ids, &n, &d, L.scratch, L.scratch_bytes, s, &L.defer[0], 2, kcp,
-                     L.nd_slot, &L.defer[4], false, hp);
+                     L.nd_slot, &L.defer[4], false, hp, fused_fill);
   if (rc != PTC_OK) return rc;
   const ptc::ReuseDevIn din{L.nd_slot, &L.defer[4]};
   ptc::ReuseHostOut hout;
