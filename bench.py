@@ -150,14 +150,16 @@ def sort_passes(D):
     return (b + 7) // 8
 
 
-def kernel_model_bytes(name, T, N, L, D):
+def kernel_model_bytes(name, T, N, L, D, fill=0):
     """Algorithmic bytes one launch of `name` moves under the stage-byte model
-    (0: the kernel only touches scratch the model does not count)."""
+    (0: the kernel only touches scratch the model does not count).  `fill`:
+    the bytes of stage a2's id table that the pipeline has the hash grid set
+    (ptc_pipeline_table_fill_bytes), written by the hash kernel."""
     per_level = ((L - 1) * 8.125 + 4.125) / L * N  # the last level writes no partition
     return {
-        "k_hash_local": 4 * T + 16 * N,   # token stream in, block keys out
-        "k_hash16": 4 * T + 16 * N,       # the same, B = 16 path
-        "k_hash_tile": 4 * T + 16 * N,    # the same, other multiples of 16
+        "k_hash_local": 4 * T + 16 * N + fill,   # token stream in, block keys (and the table fill) out
+        "k_hash16": 4 * T + 16 * N + fill,       # the same, B = 16 path
+        "k_hash_tile": 4 * T + 16 * N + fill,    # the same, other multiples of 16
         "k_ids_insert": 16 * N,           # keys in
         "k_ids_insert_prior": 16 * N,     # keys in (the same stage, prior-request hint)
         "k_ids_gather": 4 * N,            # ids out
@@ -320,11 +322,11 @@ class Timer:
         return ms
 
 
-def kernel_table(ktimes, steps, T, N, D, Lbits):
+def kernel_table(ktimes, steps, T, N, D, Lbits, fill=0):
     kernels = []
     for name, launches_k, tot_ms in ktimes:
         per = tot_ms / max(launches_k, 1)
-        mb = kernel_model_bytes(name, T, N, Lbits, D)
+        mb = kernel_model_bytes(name, T, N, Lbits, D, fill)
         kernels.append({"name": name, "launches_per_step": launches_k / steps, "ms_per_step": tot_ms / steps,
                         "avg_launch_ms": per, "model_bytes_per_launch": mb,
                         "achieved_gbs": (mb / (per * 1e-3) / 1e9) if per > 0 else 0.0})
@@ -450,7 +452,7 @@ def run_ours(args, ws_world, rank, local):
     L.ptc_timer_enable(0)
     ktimes = read_timer(ptc)
     hbm, Lbits = hbm_fractions(T, N, ms_per_step, peak)
-    kernels = kernel_table(ktimes, args.steps, T, N, D, Lbits)
+    kernels = kernel_table(ktimes, args.steps, T, N, D, Lbits, L.ptc_pipeline_table_fill_bytes(R, T, BLOCK, 1))
     roof = roofline_of(kernels, peak, peak_kind, W)
     gold = golden_parity(W, N, D, plan.hits, plan.result()["saved"], caps) if not args.requests else None
     del plan, ws, tok, off, ts, ses, dev_t
@@ -562,7 +564,7 @@ def chat_extras(args, ptc, tracegen, dev, timer, slowest, peak, peak_kind, rank,
     timer.run(args.steps, plan.run, plan, ref)
     L.ptc_timer_enable(0)
     hbm, Lbits = hbm_fractions(T, N, ms, peak)
-    kernels = kernel_table(read_timer(ptc), args.steps, T, N, D, Lbits)
+    kernels = kernel_table(read_timer(ptc), args.steps, T, N, D, Lbits, L.ptc_pipeline_table_fill_bytes(R, T, BLOCK, 1))
     out = {"workload": WORKLOAD_NAMES[CHAT], "tokens": T, "requests": R, "accesses": N, "distinct_blocks": D,
            "capacities": G, "ms_per_step": round(ms, 4), "tokens_per_s": round(ws_world * T / (ms * 1e-3), 1),
            "accesses_per_s": round(ws_world * N / (ms * 1e-3), 1), "hbm_roofline": hbm,

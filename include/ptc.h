@@ -422,6 +422,15 @@ ptc_status ptc_session_lru_curves(const uint32_t* ids, uint64_t n, uint64_t n_di
  * wait for their own status; an error they raise is returned with stage d's.
  */
 size_t ptc_pipeline_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size, uint32_t n_cap);
+/*
+ * ptc_pipeline_table_fill_bytes — bytes of stage a2's id table that
+ * ptc_pipeline has the block-hash grid of stage a1 set to all ones while it
+ * hashes (the hash is bound by integer issue, so the fill uses DRAM time it
+ * leaves idle); 0 when stage a2 fills its own table.  with_sessions: whether
+ * the call passes req_session.  For reporting the hash kernel's bytes; it
+ * allocates and launches nothing.
+ */
+size_t ptc_pipeline_table_fill_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size, int with_sessions);
 ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off, const int64_t* req_ts_us,
                         const uint32_t* req_session, uint32_t n_session, uint32_t n_req, uint32_t block_size, uint64_t seed, const ptc_cost_model* cm,
                         const uint64_t* cap_host, uint32_t n_cap, ptc_u128* keys_out, uint64_t* req_blk_off_out,

@@ -46,6 +46,7 @@ constexpr int kWinTokens = 8192 + 256;
 constexpr int kWinWords = kWinTokens + kWinTokens / 16;
 
 constexpr int kEpochOffsets = 1;
+constexpr int kEpochWide = 2;  // st->tile_ctr slot counting the tiles of k_hash16_wide
 
 // ---------------------------------------------------------------- block scans
 // Exclusive sum over a CTA of kOffThreads threads; returns the CTA total in *total.
@@ -220,6 +221,7 @@ struct HashArgs {
   uint32_t* tile_lead;   // per tile: blocks before its first request start (keys left normalised)
   DevStatus* st;
   int aligned;
+  uint32_t* wide_list;  // k_hash16: tiles left to k_hash16_wide (their count in st->tile_ctr[kEpochWide])
   uint4* fill;          // a region the caller asked the hash grid to set to all ones, or null
   uint64_t fill_units;  // its 16-byte units
 };
@@ -513,14 +515,19 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_local(HashArgs a, const _
 // global offsets instead.
 constexpr int kH16Req = 256;
 
-__global__ void __launch_bounds__(kHashThreads, 8) k_hash16(HashArgs a, const __grid_constant__ HashConsts c) {
-  grid_dep_sync();
-  fill_share(a);
+// One tile of k_hash16.  WIDE = false: two-limb products, exact while every
+// token is below 2^27 (any vocabulary in use); a tile that holds a larger
+// token is left to k_hash16_wide (its index goes to wide_list) and returns
+// before it writes anything.  WIDE = true: three-limb products, exact for
+// every 32-bit token.  Keeping the three-limb code out of the common kernel
+// keeps that kernel's registers free of it (it spilled, and measured 1.0 ms
+// slower on the mixed 10B-token trace).
+template <bool WIDE>
+__device__ __forceinline__ void hash16_tile(const HashArgs& a, const HashConsts& c, uint32_t tile, uint64_t N) {
   __shared__ uint64_t s_boff[kH16Req + 1];
   __shared__ uint64_t s_toff[kH16Req + 1];
+  __shared__ uint32_t s_big;  // some block of the tile needs three limbs
   constexpr uint32_t TB = kHashThreads;
-  const uint32_t tile = blockIdx.x;
-  const uint64_t N = blocks_live(a.st, a.keys_cap);
   const uint64_t b0 = (uint64_t)tile * TB;
   if (b0 >= N) return;
   const uint64_t b_end = b0 + TB < N ? b0 + TB : N;
@@ -535,6 +542,7 @@ __global__ void __launch_bounds__(kHashThreads, 8) k_hash16(HashArgs a, const __
       s_toff[i] = a.tok_off[r_first + i];
     }
   }
+  if (threadIdx.x == 0) s_big = 0;
   __syncthreads();
   const uint32_t t = threadIdx.x;
   const uint64_t b = b0 + t;
@@ -611,10 +619,11 @@ __global__ void __launch_bounds__(kHashThreads, 8) k_hash16(HashArgs a, const __
     }
   }
   if (live) {
-    uint32_t any = 0;  // bits of the block's tokens above 2^27
+    if (!WIDE) {  // a token (or a word around the block: that only widens the test) reaching 2^27
+      uint32_t any = 0;
 #pragma unroll
-    for (int j = 0; j < 19; ++j) any |= wd[j];
-    if ((any >> 27) == 0) {  // every token fits two limbs (words outside the block only widen the test)
+      for (int j = 0; j < 19; ++j) any |= wd[j];
+      if (any >> 27) s_big = 1;
       uint64_t acc[4] = {0, 0, 0, 0};
       switch (m) {
         case 0: hash16_2<0>(wd, c, acc); break;
@@ -625,7 +634,7 @@ __global__ void __launch_bounds__(kHashThreads, 8) k_hash16(HashArgs a, const __
       // lazily reduced (below 2^62 + 3); p61_mul_lazy takes it as it is
       h0 = limbs2_lazy(acc[0], acc[1]) + c.csum[0][16];
       h1 = limbs2_lazy(acc[2], acc[3]) + c.csum[1][16];
-    } else {
+    } else {  // three limbs
       uint64_t acc[6] = {0, 0, 0, 0, 0, 0};
       switch (m) {
         case 0: hash16<0>(wd, c, acc); break;
@@ -669,6 +678,10 @@ __global__ void __launch_bounds__(kHashThreads, 8) k_hash16(HashArgs a, const __
     s_w1[w] = v1;
   }
   __syncthreads();
+  if (!WIDE && s_big) {  // the tile goes to k_hash16_wide, which writes all of it
+    if (t == 0) a.wide_list[atomicAdd(&a.st->tile_ctr[kEpochWide], 1u)] = tile;
+    return;
+  }
   if (w == 0) {  // exclusive prefix of the warp totals
     uint64_t z0 = lane < kHashThreads / 32 ? s_w0[lane] : 0, z1 = lane < kHashThreads / 32 ? s_w1[lane] : 0;
     const uint64_t x0 = z0, x1 = z1;
@@ -690,12 +703,18 @@ __global__ void __launch_bounds__(kHashThreads, 8) k_hash16(HashArgs a, const __
   __syncthreads();
   v0 = p61_fold(v0 + s_w0[w]);
   v1 = p61_fold(v1 + s_w1[w]);
-  s_p0[t] = v0;
-  s_p1[t] = v1;
-  __syncthreads();
+  // A request starting after b0 inside the tile subtracts the prefix before
+  // its start; when none does (a long request spans the tile), the prefixes
+  // are not exchanged.
+  const bool inner = !cached || (nreq >= 2 && s_boff[1] < b_end);
+  if (inner) {
+    s_p0[t] = v0;
+    s_p1[t] = v1;
+    __syncthreads();
+  }
   if (live) {
     const bool own_start = rstart >= b0;  // the request starts in this tile
-    if (own_start && rstart > b0) {
+    if (inner && own_start && rstart > b0) {
       const uint32_t sl = (uint32_t)(rstart - b0) - 1;
       v0 = p61_add(v0, kP61 - s_p0[sl]);
       v1 = p61_add(v1, kP61 - s_p1[sl]);
@@ -730,6 +749,25 @@ __global__ void __launch_bounds__(kHashThreads, 8) k_hash16(HashArgs a, const __
       }
     }
     a.tile_lead[tile] = lead;
+  }
+}
+
+__global__ void __launch_bounds__(kHashThreads, 8) k_hash16(HashArgs a, const __grid_constant__ HashConsts c) {
+  grid_dep_sync();
+  fill_share(a);
+  hash16_tile<false>(a, c, blockIdx.x, blocks_live(a.st, a.keys_cap));
+}
+
+// The tiles k_hash16 left (a token at or above 2^27), a persistent grid over
+// the list it wrote.
+__global__ void __launch_bounds__(kHashThreads) k_hash16_wide(HashArgs a, const __grid_constant__ HashConsts c) {
+  grid_dep_sync();
+  const uint64_t N = blocks_live(a.st, a.keys_cap);
+  const uint32_t n_wide = ld_relaxed_u32(&a.st->tile_ctr[kEpochWide]);
+  for (uint32_t j = blockIdx.x; j < n_wide; j += gridDim.x) {
+    const uint32_t tile = a.wide_list[j];
+    if (in_bounds(a.st, tile, (N + kHashThreads - 1) / kHashThreads)) hash16_tile<true>(a, c, tile, N);
+    __syncthreads();  // the next tile reuses the shared arrays
   }
 }
 
@@ -1103,8 +1141,11 @@ __global__ void __launch_bounds__(kChainWarps * 32) k_hash_carry(const HashCarry
 
 template <int G>
 void launch_hash(uint32_t grid, cudaStream_t s, const HashArgs& a, const HashConsts& c, bool full) {
-  if (G == 1 && full && a.aligned)
+  if (G == 1 && full && a.aligned) {
     PTC_KERNEL("k_hash16", s, k_hash16, grid, kHashThreads, 0, a, c);
+    const uint32_t wgrid = grid < (uint32_t)(2 * num_sms()) ? grid : (uint32_t)(2 * num_sms());
+    PTC_KERNEL("k_hash16_wide", s, k_hash16_wide, wgrid, kHashThreads, 0, a, c);
+  }
   else if (a.aligned && a.B % 16 == 0)
     PTC_KERNEL("k_hash_tile", s, k_hash_tile, grid, kHashThreads, 0, a, c);
   else if (full)
@@ -1135,6 +1176,7 @@ struct HashLayout {
   uint32_t* tile_lead;
   uint64_t* tables;
   uint32_t* tile_req;
+  uint32_t* wide_list;
   uint64_t hash_tiles;
   size_t zero_bytes;
   size_t total;
@@ -1154,6 +1196,7 @@ HashLayout hash_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   L.tile_lead = cv.take<uint32_t>(hash_tiles);
   L.tables = cv.take<uint64_t>(4 * 65536);
   L.tile_req = cv.take<uint32_t>(hash_tiles + 1);
+  L.wide_list = cv.take<uint32_t>(hash_tiles);
   L.hash_tiles = hash_tiles;
   L.total = cv.bytes();
   return L;
@@ -1243,6 +1286,7 @@ ptc_status ptc::hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t
   a.tile_req = L.tile_req;
   a.tile_agg = L.tile_agg;
   a.tile_lead = L.tile_lead;
+  a.wide_list = L.wide_list;
   a.st = L.st;
   a.aligned = aligned;
   const bool full = block_size == 16 * G;

@@ -63,7 +63,30 @@ PipeLayout pipe_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   return L;
 }
 
+// Stage a2's first table inside the scratch region, and whether it lies
+// past the scratch that stages a1 (and the session sort before it) use, so
+// that the hash grid may fill it while stage a1 runs.
+bool fused_table_fill(void* scratch, uint32_t n_req, uint64_t n_tok, uint32_t B, bool hinted, void** table,
+                      size_t* bytes) {
+  const uint64_t cap = n_tok / B ? n_tok / B : 1;
+  ptc::ids_table_region(scratch, cap, hinted ? n_req : 0, table, bytes);
+  const size_t front = std::max(ptc_hash_blocks_workspace_bytes(n_req, n_tok, B), ptc::session_prior_bytes(n_req));
+  return *bytes > 0 && static_cast<char*>(*table) >= static_cast<char*>(scratch) + front;
+}
+
 }  // namespace
+
+extern "C" size_t ptc_pipeline_table_fill_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size,
+                                                int with_sessions) {
+  if (block_size < 1 || block_size > PTC_MAX_BLOCK_SIZE || n_tok / block_size == 0) return 0;
+  const bool hinted = with_sessions && n_req > 0 && ptc::ids_table_in_dram(n_tok / block_size);
+  // the region's offset is what matters: lay it out from a scratch base of 256
+  void* table = nullptr;
+  size_t bytes = 0;
+  return fused_table_fill(reinterpret_cast<void*>(uintptr_t{256}), n_req, n_tok, block_size, hinted, &table, &bytes)
+             ? bytes
+             : 0;
+}
 
 extern "C" size_t ptc_pipeline_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size, uint32_t n_cap) {
   if (block_size == 0) block_size = 1;
@@ -122,10 +145,7 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
   // sort's in the shared scratch region
   void* table = nullptr;
   size_t table_bytes = 0;
-  ptc::ids_table_region(L.scratch, cap, hinted ? n_req : 0, &table, &table_bytes);
-  const size_t front = std::max(ptc_hash_blocks_workspace_bytes(n_req, n_tok, block_size),
-                                ptc::session_prior_bytes(n_req));
-  const bool fused_fill = table_bytes > 0 && static_cast<char*>(table) >= static_cast<char*>(L.scratch) + front;
+  const bool fused_fill = fused_table_fill(L.scratch, n_req, n_tok, block_size, hinted, &table, &table_bytes);
   ptc_status rc = ptc::hash_impl(tokens, n_tok, req_tok_off, req_ts_us, n_req, block_size, seed, keys, cap, blk,
                                  &unused, L.scratch, L.scratch_bytes, s, L.n_slot, &L.defer[0], kcp,
                                  fused_fill ? table : nullptr, fused_fill ? table_bytes : 0);

@@ -127,3 +127,24 @@ def test_trace_stats_host_checks_need_no_gpu(libptc):
     # workspace too small
     assert L.ptc_trace_stats(fake, fake, fake, None, 10, 5, fake, fake, fake, 2, 2, None, 0, None,
                              buf.ctypes.data, fake, 16, None) == 4
+
+
+def test_pipeline_table_fill_bytes(libptc):
+    """The id table that the pipeline's hash grid fills: a power of two of
+    16-byte slots, at least n / 3 of them (3 n / 4 once the table is larger
+    than the part of L2 it may use); nothing for an empty trace, or when the
+    table would overlap the hash stage's own scratch (small traces)."""
+    f = libptc.ptc_pipeline_table_fill_bytes
+    f.restype = ctypes.c_size_t
+    f.argtypes = [ctypes.c_uint32, ctypes.c_uint64, ctypes.c_uint32, ctypes.c_int]
+    assert f(10, 15, 16, 0) == 0
+    for n_req, n_tok, B, ses in ((100, 10**6, 16, 0), (582163, 9984375026, 16, 1), (2000, 2 * 10**9, 64, 1)):
+        b = f(n_req, n_tok, B, ses)
+        if b == 0:
+            assert n_tok < 10**8
+            continue
+        slots = b // 16
+        n = n_tok // B
+        assert b % 16 == 0 and slots & (slots - 1) == 0
+        assert slots >= (n // 4 * 3 if slots > (1 << 22) else n // 3)
+    assert f(582163, 9984375026, 16, 1) == 16 << 29
