@@ -17,6 +17,7 @@
 // without runs it is the sort of every (id, i).
 //
 //   k_ir_count     id-run starts per tile (ids < D checked); last CTA: prefixes
+//                  (k_ir_count4: 16-byte loads when the ids are 16-byte aligned)
 //   k_ir_mark      id-run records (start, first id) and the cuts, as a bitmap
 //                  over [0, D]
 //   k_bm_count / k_bm_words   ranks of the cuts (and the cut of each rank)
@@ -185,6 +186,78 @@ __global__ void __launch_bounds__(kIT) k_ir_mark(IrArgs a0) {
     }
     run += __popc(words[k]);
   }
+}
+
+// ---- the counting pass with 16-byte loads (ids 16-byte aligned): lane l of
+// warp w reads positions base + 128 k + 4 l .. + 3 (k < 4, base = the warp's
+// 512 positions), one load per four accesses.
+constexpr int kIR4 = kIR / 4;
+
+__device__ __forceinline__ uint4 ir_load4(const uint32_t* __restrict__ v, uint32_t p, uint32_t n) {
+  if (p + 4 <= n) return __ldcs(reinterpret_cast<const uint4*>(v + p));
+  return make_uint4(p < n ? v[p] : 0u, p + 1 < n ? v[p + 1] : 0u, p + 2 < n ? v[p + 2] : 0u, p + 3 < n ? v[p + 3] : 0u);
+}
+
+// Id-run starts among positions p .. p + 3 as bits 0..3 (the id left of p is
+// `il`), and whether an id is out of range.
+__device__ __forceinline__ uint32_t id_starts4(const uint4 v, uint32_t il, uint32_t p, uint32_t n, uint32_t D,
+                                               bool& bad) {
+  const uint32_t iv[4] = {v.x, v.y, v.z, v.w};
+  uint32_t x = 0, left = il;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const uint32_t j = p + e;
+    if (j < n) {
+      if (iv[e] >= D) bad = true;
+      x |= (j == 0 || iv[e] != left + 1u ? 1u : 0u) << e;
+    }
+    left = iv[e];
+  }
+  return x;
+}
+
+__device__ __forceinline__ uint32_t warp_id_starts4(const IrArgs& a, uint32_t base, uint32_t lane, uint4 (&v)[kIR4],
+                                                    uint32_t (&x)[kIR4], uint32_t (&il)[kIR4], bool& bad) {
+#pragma unroll
+  for (int k = 0; k < kIR4; ++k) v[k] = ir_load4(a.ids, base + 128 * k + 4 * lane, a.n);
+  uint32_t carry = (base > 0 && base - 1 < a.n) ? a.ids[base - 1] : 0u;
+  uint32_t cnt = 0;
+#pragma unroll
+  for (int k = 0; k < kIR4; ++k) {
+    const uint32_t up = __shfl_up_sync(kFull, v[k].w, 1);
+    il[k] = lane ? up : carry;
+    carry = __shfl_sync(kFull, v[k].w, 31);
+    x[k] = id_starts4(v[k], il[k], base + 128 * k + 4 * lane, a.n, a.D, bad);
+    cnt += __popc(x[k]);
+  }
+  return cnt;
+}
+
+__global__ void __launch_bounds__(kIT) k_ir_count4(IrArgs a0) {
+  grid_dep_sync();
+  __shared__ uint32_t s_wcnt[kIT / 32];
+  const IrArgs a = resolved(a0);
+  if (a0.nd && blockIdx.x == 0 && threadIdx.x == 0) {
+    a.st->value[4] = a0.nd[1];
+    a.st->value[5] = a0.nd[0];
+    a.st->value[6] = a0.ext_err ? *a0.ext_err : 0u;
+  }
+  const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  uint4 v[kIR4];
+  uint32_t x[kIR4], il[kIR4];
+  bool bad = false;
+  const uint32_t cnt = __reduce_add_sync(kFull, warp_id_starts4(a, tile * kITile + w * (32 * kIR), lane, v, x, il, bad));
+  if (lane == 0) s_wcnt[w] = cnt;
+  if (bad) raise_err(a.st, kErrInvalid);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t t = 0;
+    for (int ww = 0; ww < kIT / 32; ++ww) t += s_wcnt[ww];
+    a.tcnt[tile] = t;
+  }
+  if (!last_cta(a.done)) return;
+  const uint32_t R = cta_tiles_prefix(a.tcnt, a.tpre, a.ntiles);
+  if (threadIdx.x == 0) a.st->value[1] = R;
 }
 
 // Ranks of the cuts: per tile of kBmTile words the set bits, then (last CTA)
@@ -427,7 +500,13 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
   a.st = L.st;
   a.nd = din ? din->nd : nullptr;
   a.ext_err = din ? din->ids_err : nullptr;
-  PTC_KERNEL("k_ir_count", s, k_ir_count, L.ntiles, kIT, 0, a);
+  // the count with 16-byte loads when the ids allow them (measured faster);
+  // the marking pass stays one access per lane and round (the 16-byte form
+  // of it measured slower: 0.77 against 0.70 ms on the mixed 10B-token trace)
+  if ((reinterpret_cast<uintptr_t>(ids) & 15) == 0)
+    PTC_KERNEL("k_ir_count", s, k_ir_count4, L.ntiles, kIT, 0, a);
+  else
+    PTC_KERNEL("k_ir_count", s, k_ir_count, L.ntiles, kIT, 0, a);
   PTC_KERNEL("k_ir_mark", s, k_ir_mark, L.ntiles, kIT, 0, a);
   PTC_KERNEL("k_bm_count", s, k_bm_count, L.btiles, kIT, 0, L.cut, L.nwords, L.btiles, L.btcnt, L.btpre, &L.done[1], L.st);
   PTC_KERNEL("k_bm_words", s, k_bm_words, L.btiles, kIT, 0, L.cut, L.nwords, L.btpre, L.cwpre, L.cut_at);

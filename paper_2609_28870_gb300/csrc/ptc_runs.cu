@@ -34,6 +34,9 @@
 //   k_runs_count   run starts per tile; the last CTA scans the tile counts
 //   k_runs_mark    run starts again: bitmap, run index per 32-position word,
 //                  run (start, first value) records
+//                  (both with 16-byte loads, four accesses per lane and
+//                  round, when prev is 16-byte aligned: k_runs_count4,
+//                  k_runs_mark4)
 //   bitmap_ranks   the runs' keys (marked by k_runs_mark in a bitmap over
 //                  [0, n]) counted per word: the matrix holds each key's rank
 //                  among the distinct keys, so it has ceil(log2(R + 2))
@@ -188,6 +191,130 @@ __global__ void __launch_bounds__(kMT) k_runs_mark(MarkArgs a) {
       a.rec_a[r] = vval(pv[k]);
     }
     run += __popc(words[k]);
+  }
+  if (tile == a.ntiles - 1 && threadIdx.x == 0) a.rec_s[a.tpre[a.ntiles]] = a.n;
+}
+
+// ---- the same two passes with 16-byte loads (prev 16-byte aligned): lane l
+// of warp w reads positions base + 128 k + 4 l .. + 3 (k < 4, base = the
+// warp's 512 positions), one load per four accesses.
+constexpr int kMR4 = kMR / 4;
+
+// Four values from position p (a multiple of 4), kNone past n.
+__device__ __forceinline__ uint4 load4(const uint32_t* __restrict__ v, uint32_t p, uint32_t n) {
+  if (p + 4 <= n) return __ldcs(reinterpret_cast<const uint4*>(v + p));
+  return make_uint4(p < n ? v[p] : kNone, p + 1 < n ? v[p + 1] : kNone, p + 2 < n ? v[p + 2] : kNone,
+                    p + 3 < n ? v[p + 3] : kNone);
+}
+
+// Run starts among positions p .. p + 3 as bits 0..3, from their previous
+// uses v and the previous use `pl` at p - 1.  A run continues at j when
+// prev[j] = prev[j - 1] + 1 with prev[j - 1] a use, or both are first
+// accesses (as start_words, with prev values instead of v = prev + 1).
+__device__ __forceinline__ uint32_t starts4(const uint4 v, uint32_t pl, uint32_t p, uint32_t n, bool& bad) {
+  const uint32_t pv[4] = {v.x, v.y, v.z, v.w};
+  uint32_t x = 0, left = pl;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const uint32_t j = p + e, P = pv[e];
+    if (j < n) {
+      if (P != kNone && P >= j) bad = true;
+      const bool cont = j > 0 && ((P == left + 1u && left != kNone) || (P == kNone && left == kNone));
+      x |= (cont ? 0u : 1u) << e;
+    }
+    left = P;
+  }
+  return x;
+}
+
+// The warp's four loads and their run-start nibbles.
+__device__ __forceinline__ uint32_t warp_starts4(const MarkArgs& a, uint32_t base, uint32_t lane, uint4 (&v)[kMR4],
+                                                 uint32_t (&x)[kMR4], uint32_t (&pl)[kMR4], bool& bad) {
+#pragma unroll
+  for (int k = 0; k < kMR4; ++k) v[k] = load4(a.prev, base + 128 * k + 4 * lane, a.n);
+  uint32_t carry = (base > 0 && base - 1 < a.n) ? a.prev[base - 1] : kNone;  // lane 0 of the first round
+  uint32_t cnt = 0;
+#pragma unroll
+  for (int k = 0; k < kMR4; ++k) {
+    const uint32_t up = __shfl_up_sync(kFull, v[k].w, 1);
+    pl[k] = lane ? up : carry;
+    carry = __shfl_sync(kFull, v[k].w, 31);
+    x[k] = starts4(v[k], pl[k], base + 128 * k + 4 * lane, a.n, bad);
+    cnt += __popc(x[k]);
+  }
+  return cnt;
+}
+
+__global__ void __launch_bounds__(kMT) k_runs_count4(MarkArgs a) {
+  grid_dep_sync();
+  __shared__ uint32_t s_wcnt[kMT / 32];
+  const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  uint4 v[kMR4];
+  uint32_t x[kMR4], pl[kMR4];
+  bool bad = false;
+  const uint32_t cnt = __reduce_add_sync(kFull, warp_starts4(a, tile * kMTile + w * (32 * kMR), lane, v, x, pl, bad));
+  if (lane == 0) s_wcnt[w] = cnt;
+  if (bad) raise_err(a.st, kErrInvalid);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t t = 0;
+    for (int ww = 0; ww < kMT / 32; ++ww) t += s_wcnt[ww];
+    a.tcnt[tile] = t;
+  }
+  if (!last_cta(a.done)) return;
+  const uint32_t total = cta_tiles_prefix(a.tcnt, a.tpre, a.ntiles);
+  if (threadIdx.x == 0) a.st->value[1] = total;
+}
+
+__global__ void __launch_bounds__(kMT) k_runs_mark4(MarkArgs a) {
+  grid_dep_sync();
+  __shared__ uint32_t s_wcnt[kMT / 32];
+  const uint32_t tile = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const uint32_t base = tile * kMTile + w * (32 * kMR);
+  uint4 v[kMR4];
+  uint32_t x[kMR4], pl[kMR4];
+  bool bad = false;
+  const uint32_t cnt = __reduce_add_sync(kFull, warp_starts4(a, base, lane, v, x, pl, bad));
+  if (lane == 0) s_wcnt[w] = cnt;
+  if (tile == 0 && threadIdx.x == 0) atomicOr(&a.kbits[0], 1u);
+  __syncthreads();
+  uint32_t run = a.tpre[tile];
+  for (int ww = 0; ww < (int)w; ++ww) run += s_wcnt[ww];
+  const uint32_t g = lane >> 3, sh = 4 * (lane & 7);
+#pragma unroll
+  for (int k = 0; k < kMR4; ++k) {
+    const uint32_t p = base + 128 * k + 4 * lane;
+    // the 32-position word of lane group g (lanes 8g .. 8g + 7)
+    uint32_t word = x[k] << sh;
+    word |= __shfl_xor_sync(kFull, word, 1);
+    word |= __shfl_xor_sync(kFull, word, 2);
+    word |= __shfl_xor_sync(kFull, word, 4);
+    const uint32_t c0 = __popc(__shfl_sync(kFull, word, 0)), c1 = __popc(__shfl_sync(kFull, word, 8)),
+                   c2 = __popc(__shfl_sync(kFull, word, 16)), c3 = __popc(__shfl_sync(kFull, word, 24));
+    const uint32_t before = (g > 0 ? c0 : 0u) + (g > 1 ? c1 : 0u) + (g > 2 ? c2 : 0u);
+    if ((lane & 7) == 0 && base + 128 * k + 32 * g < a.n) {
+      a.bits[(base + 128 * k + 32 * g) >> 5] = word;
+      a.wpre[(base + 128 * k + 32 * g) >> 5] = run + before;
+    }
+    // The runs' keys for rank compression: a run's largest value is its last
+    // one, i.e. the value left of the next run's start, or the last access's.
+    // Nonzero keys are distinct; 0 is always entered, once.
+    uint32_t r = run + before + __popc(word & ((1u << sh) - 1u));
+    const uint32_t pv[4] = {v[k].x, v[k].y, v[k].z, v[k].w};
+    uint32_t left = pl[k];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const uint32_t j = p + e, vl = left + 1u, vj = pv[e] + 1u;  // v = prev + 1, none -> 0
+      if ((x[k] >> e) & 1u) {
+        a.rec_s[r] = j;
+        a.rec_a[r] = vj;
+        if (j > 0 && vl != 0) atomicOr(&a.kbits[vl >> 5], 1u << (vl & 31));
+        ++r;
+      }
+      if (j + 1 == a.n && vj != 0) atomicOr(&a.kbits[vj >> 5], 1u << (vj & 31));
+      left = pv[e];
+    }
+    run += c0 + c1 + c2 + c3;
   }
   if (tile == a.ntiles - 1 && threadIdx.x == 0) a.rec_s[a.tpre[a.ntiles]] = a.n;
 }
@@ -738,8 +865,13 @@ ptc_status stack_distance_runs(const uint32_t* prev, uint64_t n, uint32_t* dist_
   m.done = &M.done[63];
   m.kbits = M.kbits;
   m.st = M.st;
-  PTC_KERNEL("k_runs_count", s, k_runs_count, M.mtiles, kMT, 0, m);
-  PTC_KERNEL("k_runs_mark", s, k_runs_mark, M.mtiles, kMT, 0, m);
+  if ((reinterpret_cast<uintptr_t>(prev) & 15) == 0) {
+    PTC_KERNEL("k_runs_count", s, k_runs_count4, M.mtiles, kMT, 0, m);
+    PTC_KERNEL("k_runs_mark", s, k_runs_mark4, M.mtiles, kMT, 0, m);
+  } else {
+    PTC_KERNEL("k_runs_count", s, k_runs_count, M.mtiles, kMT, 0, m);
+    PTC_KERNEL("k_runs_mark", s, k_runs_mark, M.mtiles, kMT, 0, m);
+  }
   if (bitmap_ranks(M.kbits, M.kwords, M.kpre, M.ktcnt, M.ktpre, &M.done[62], nullptr, s) != PTC_OK) return PTC_ERR_CUDA;
   DevStatus h;
   ptc_status rc = end_call(M.st, s, &h);
