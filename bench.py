@@ -347,6 +347,71 @@ def roofline_of(kernels, peak, peak_kind, workload):
             "peak_source": f"{peak_kind} hbm_gbs"}
 
 
+def hint_matched(ptc, torch, ids, blk_off, ses):
+    """Accesses the prior-request hint matches (their block equals the block
+    at the same depth of the previous request of their session): the id
+    table's insert probes the others.  Counted from the step's ids."""
+    R = ses.numel()
+    order = torch.sort(ses.to(torch.int64), stable=True).indices
+    ss = ses.to(torch.int64)[order]
+    prior_sorted = torch.full((R,), -1, dtype=torch.int64, device=ids.device)
+    prior_sorted[1:] = torch.where(ss[1:] == ss[:-1], order[:-1], torch.full_like(order[:-1], -1))
+    prior = torch.empty_like(prior_sorted)
+    prior[order] = prior_sorted
+    n_r = blk_off[1:] - blk_off[:-1]
+    matched = 0
+    step = 1 << 16  # requests per slice: bounded temporaries
+    for r0 in range(0, R, step):
+        r1 = min(R, r0 + step)
+        cnt = n_r[r0:r1]
+        req = torch.repeat_interleave(torch.arange(r0, r1, device=ids.device), cnt)
+        k = torch.arange(int(cnt.sum()), device=ids.device) - torch.repeat_interleave(
+            torch.cumsum(cnt, 0) - cnt, cnt)
+        p = prior[req]
+        ok = (p >= 0) & (k < n_r[p.clamp(min=0)])
+        i = blk_off[req] + k
+        j = blk_off[p.clamp(min=0)] + k
+        eq = ok & (ids[i] == ids[j.clamp(max=ids.numel() - 1)])
+        matched += int(eq.sum())
+    return matched
+
+
+def id_table_roofline(ptc, torch, L, kernels, n_access, matched, table_bytes, dev):
+    """k_ids_insert_prior against the rate at which this GPU settles random
+    16-byte read-modify-write probes of a table of the same size, measured in
+    this run (ptc_probe_random_rmw): the insert's bound is that rate, not the
+    copy bandwidth."""
+    ins = next((k for k in kernels if k["name"] == "k_ids_insert_prior"), None)
+    if ins is None or table_bytes <= 0:
+        return None
+    probes = n_access - matched
+    slots = table_bytes // 16
+    table = torch.empty(slots * 2, dtype=torch.int64, device=dev)
+    sink = torch.zeros(1, dtype=torch.int64, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    best = None
+    for rep in range(3):
+        table.fill_(-1)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        rc = L.ptc_probe_random_rmw(table.data_ptr(), slots, probes, 0x5EED + rep, sink.data_ptr(), stream.cuda_stream)
+        e1.record(stream)
+        e1.synchronize()
+        if rc != 0:
+            raise RuntimeError(f"ptc_probe_random_rmw failed ({rc})")
+        ms = e0.elapsed_time(e1)
+        best = ms if best is None else min(best, ms)
+    del table, sink
+    achieved = probes / (ins["avg_launch_ms"] * 1e-3) / 1e9
+    peak = probes / (best * 1e-3) / 1e9
+    return {"kernel": "k_ids_insert_prior", "bound": "hbm random read-modify-write", "probes": probes,
+            "matched_by_hint": matched, "ms": round(ins["avg_launch_ms"], 4),
+            "achieved_gprobes_per_s": round(achieved, 2), "peak_gprobes_per_s": round(peak, 2),
+            "frac": round(achieved / peak, 4), "table_bytes": table_bytes,
+            "peak_how": "ptc_probe_random_rmw in this run: the same number of 16-byte slot loads at seeded random "
+                        "slots of an all-ones table of the same size, each claimed by a 128-bit CAS; best of 3"}
+
+
 def hbm_fractions(T, N, ms, peak):
     stages, Lbits = stage_model_bytes(T, N)
     model_total = sum(stages.values())
@@ -455,6 +520,19 @@ def run_ours(args, ws_world, rank, local):
     kernels = kernel_table(ktimes, args.steps, T, N, D, Lbits, L.ptc_pipeline_table_fill_bytes(R, T, BLOCK, 1))
     roof = roofline_of(kernels, peak, peak_kind, W)
     gold = golden_parity(W, N, D, plan.hits, plan.result()["saved"], caps) if not args.requests else None
+    # the id table's insert against the random read-modify-write rate (one
+    # more step with the ids kept, to count the accesses the hint matches)
+    id_table = None
+    if any(k["name"] == "k_ids_insert_prior" for k in kernels):
+        ids_t = torch.empty(N, dtype=torch.int32, device=dev)
+        boff_t = torch.empty(R + 1, dtype=torch.int64, device=dev)
+        ptc.PipelinePlan(tok, off, ts, BLOCK, caps, kind=ptc.PTC_COST_MEASURED, seed=0, ws=ws,
+                         outputs={"ids": ids_t, "req_blk_off": boff_t}, req_session=ses,
+                         n_session=tr.n_sessions).run()
+        matched = hint_matched(ptc, torch, ids_t, boff_t, ses)
+        del ids_t, boff_t
+        id_table = id_table_roofline(ptc, torch, L, kernels, N, matched,
+                                     L.ptc_pipeline_table_fill_bytes(R, T, BLOCK, 1), dev)
     del plan, ws, tok, off, ts, ses, dev_t
     torch.cuda.empty_cache()
 
@@ -496,6 +574,7 @@ def run_ours(args, ws_world, rank, local):
         "gpu_launches": launches,
         "clocks": clk,
         "parity_with_oracle_golden": gold,
+        "id_table_roofline": id_table,
     }
 
     # ---- the oracle on a bounded prefix of the same workload, and the GPU

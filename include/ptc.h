@@ -599,6 +599,22 @@ void ptc_timer_reset(void);
 uint32_t ptc_timer_read(ptc_kernel_time* out, uint32_t cap);
 uint64_t ptc_launch_count(void);
 
+/*
+ * ptc_probe_random_rmw — measurement hook (no counterpart in the paper:
+ * instrumentation for the roofline figures).  Launches on `stream`, without
+ * waiting, `probes` random read-modify-write probes of a table of `slots`
+ * 16-byte slots at `table` (device memory, 16-byte aligned, `slots` a power of
+ * two, every slot set to all ones by the caller beforehand): each probe reads
+ * the slot at a seeded pseudo-random index (SplitMix64) and, if it is still
+ * all ones, claims it with a 128-bit compare-and-swap, as the id table's
+ * insert does for a key it has not seen.  `sink` is 8 bytes of device memory
+ * the kernel may write.  The caller times the launch: probes over seconds is
+ * the random read-modify-write rate that bounds the insert.  Allocates
+ * nothing.  PTC_ERR_INVALID_ARG for a null, misaligned or non-power-of-two
+ * table.
+ */
+ptc_status ptc_probe_random_rmw(void* table, uint64_t slots, uint64_t probes, uint64_t seed, void* sink, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

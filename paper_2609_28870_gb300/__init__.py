@@ -133,6 +133,8 @@ def lib():
                                          ctypes.POINTER(U128), vp, sz, vp]
                 L.ptc_pipeline_workspace_bytes.restype = sz
                 L.ptc_pipeline_workspace_bytes.argtypes = [u32, u64, u32, u32]
+                L.ptc_probe_random_rmw.restype = st
+                L.ptc_probe_random_rmw.argtypes = [vp, u64, u64, u64, vp, vp]
                 L.ptc_pipeline_table_fill_bytes.restype = sz
                 L.ptc_pipeline_table_fill_bytes.argtypes = [u32, u64, u32, ctypes.c_int]
                 L.ptc_pipeline.restype = st
