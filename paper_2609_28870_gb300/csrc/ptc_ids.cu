@@ -272,6 +272,8 @@ constexpr uint32_t kMatched = kMatchedSlot;  // slot_of of a matched access
 struct PriorHint {
   const uint64_t* blk_off;  // n_req + 1 access offsets of the requests
   const uint32_t* prior;    // n_req: an earlier request, or kNone
+  const uint32_t* order;    // with sessions: the requests in session order (prior = the place before), or null
+  const uint32_t* pos;      //   and the place of every request in it
   uint32_t n_req;
   uint32_t* lam;            // n_req: first unmatched depth (written by k_ids_lam)
   uint32_t* tile_req;       // request of the first access of every kReqTile accesses, and n_req - 1 last
@@ -429,17 +431,101 @@ __global__ void __launch_bounds__(kFoThreads) k_ids_follow(PriorHint ph, uint32_
   }
 }
 
+// The same with the session order (the pipeline's hint: prior[r] is the
+// request just before r in its session): the warp of request r reads 32
+// ancestors at once, places pos[r] - 1, pos[r] - 2, ... of the order, down
+// to the session's first request (whose prior is none).  Ancestor i of the
+// window copies depths [lam, hi_i) when lam < hi_i, hi_i being the smallest
+// of hi and the lam of the ancestors before it (a prefix minimum over the
+// lanes), exactly as the walk one ancestor at a time would.  Two dependent
+// load rounds per 32 ancestors instead of one per ancestor.
+__global__ void __launch_bounds__(kFoThreads) k_ids_follow_win(PriorHint ph, uint32_t* __restrict__ ids,
+                                                               DevStatus* st) {
+  grid_dep_sync();
+  const uint32_t lane = threadIdx.x & 31;
+  const uint32_t r = blockIdx.x * (kFoThreads / 32) + (threadIdx.x >> 5);
+  if (r >= ph.n_req) return;
+  const uint64_t b = ph.blk_off[r], nr = ph.blk_off[r + 1] - b;
+  const uint32_t lr = ph.lam[r];
+  uint64_t hi = lr < nr ? lr : nr;
+  if (hi == 0) return;
+  const uint32_t j = ph.pos[r];
+  if (j >= ph.n_req || ph.order[j] != r || ph.prior[r] == kNone || j == 0 || ph.order[j - 1] != ph.prior[r]) {
+    if (lane == 0) raise_err(st, kErrInvalid);  // the order does not match the hint
+    return;
+  }
+  uint32_t carry_p = ph.prior[r];  // the prior of the nearest ancestor not yet read
+  for (uint32_t dist = 1;; dist += 32) {
+    const int64_t q = (int64_t)j - dist - lane;
+    const uint32_t a = q >= 0 ? __ldg(&ph.order[q]) : kNone;
+    uint32_t la = kNone, pa = kNone;
+    uint64_t ta = 0;
+    if (a != kNone) {
+      la = __ldg(&ph.lam[a]);
+      pa = __ldg(&ph.prior[a]);
+      ta = __ldg(&ph.blk_off[a]);
+    }
+    // the chain: the lane's ancestor is the prior of the lane before's, until
+    // a session's first request (prior none) ends it
+    uint32_t prev_p = __shfl_up_sync(kFull, pa, 1);
+    if (lane == 0) prev_p = carry_p;
+    const bool linked = prev_p == a && a != kNone;
+    const uint32_t ends = __ballot_sync(kFull, a != kNone && pa == kNone);
+    const uint32_t first_end = ends ? __ffs(ends) - 1 : 32u;
+    const bool valid = lane <= first_end && a != kNone;
+    if (__any_sync(kFull, lane <= first_end && !(valid && linked))) {
+      if (lane == 0) raise_err(st, kErrInvalid);  // a broken chain, or one that runs out with depths left
+      return;
+    }
+    // hi before this lane's ancestor: the prefix minimum of lam over the lanes before it
+    uint64_t m = valid ? (uint64_t)la : ~0ULL;
+    uint64_t incl = m;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint64_t y = __shfl_up_sync(kFull, incl, o);
+      if (lane >= (uint32_t)o) incl = y < incl ? y : incl;
+    }
+    uint64_t excl = __shfl_up_sync(kFull, incl, 1);
+    if (lane == 0) excl = ~0ULL;
+    const uint64_t hl = excl < hi ? excl : hi;
+    uint32_t todo = __ballot_sync(kFull, valid && (uint64_t)la < hl);
+    while (todo) {
+      const int src = __ffs(todo) - 1;
+      todo &= todo - 1;
+      const uint64_t lo = __shfl_sync(kFull, (uint64_t)la, src), top = __shfl_sync(kFull, hl, src);
+      const uint64_t tb = __shfl_sync(kFull, ta, src);
+      if (!in_bounds(st, tb + top - 1, b) || !in_bounds(st, b + top - 1, ph.blk_off[ph.n_req])) return;
+      for (uint64_t d = lo + lane; d < top; d += 32) ids[b + d] = ids[tb + d];
+    }
+    const uint64_t wmin = __shfl_sync(kFull, incl, 31);
+    hi = wmin < hi ? wmin : hi;
+    carry_p = __shfl_sync(kFull, pa, 31);
+    if (hi == 0) return;
+    if (first_end < 32) {  // the session's first request was reached with depths left
+      if (lane == 0) raise_err(st, kErrInvalid);
+      return;
+    }
+  }
+}
+
 // prior[r] = the previous request of r's session, from the requests sorted
 // stably by session label: neighbours in that order with the same label.
+// With `order` and `pos` (or null), also the session order itself: order[j]
+// = the request at place j, pos[r] = the place of request r.
 __global__ void k_session_prior(const uint32_t* __restrict__ ses_sorted, const uint32_t* __restrict__ req_sorted,
                                 const uint32_t* __restrict__ ses, uint32_t n_req, uint32_t n_session,
-                                uint32_t* __restrict__ prior, uint32_t* err) {
+                                uint32_t* __restrict__ prior, uint32_t* err, uint32_t* __restrict__ order,
+                                uint32_t* __restrict__ pos) {
   grid_dep_sync();
   const uint32_t j = blockIdx.x * blockDim.x + threadIdx.x;
   if (j >= n_req) return;
   if (ses[j] >= n_session) atomicOr(err, kErrInvalid);  // the sort sees only the label's low bits
-  const uint32_t sj = ses_sorted[j];
-  prior[req_sorted[j]] = (j > 0 && ses_sorted[j - 1] == sj) ? req_sorted[j - 1] : kNone;
+  const uint32_t sj = ses_sorted[j], rj = req_sorted[j];
+  prior[rj] = (j > 0 && ses_sorted[j - 1] == sj) ? req_sorted[j - 1] : kNone;
+  if (order) {
+    order[j] = rj;
+    pos[rj] = j;
+  }
 }
 
 // Slots for n keys at most: the full table holds 1.5 n.  The first attempt
@@ -585,8 +671,8 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
   const uint32_t hreq = hint ? hint->n_req : 0;
   if (!ws_ok(ws, ws_bytes, ids_layout(nullptr, n, hreq).total)) return PTC_ERR_WORKSPACE;
   const IdsLayout L = ids_layout(ws, n, hreq);
-  const PriorHint ph = hint ? PriorHint{hint->blk_off, hint->prior, hint->n_req, L.lam, L.tile_req}
-                            : PriorHint{nullptr, nullptr, 0, nullptr, nullptr};
+  const PriorHint ph = hint ? PriorHint{hint->blk_off, hint->prior, hint->order, hint->pos, hint->n_req, L.lam, L.tile_req}
+                            : PriorHint{nullptr, nullptr, nullptr, nullptr, 0, nullptr, nullptr};
   // the status block, the table (all ones: empty) and the first-occurrence
   // bitmap are cleared by one launch
   // the table of the first attempt may come already filled (ids_table_region)
@@ -618,8 +704,12 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
     PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of,
                  L.table, m, L.bits, L.wpre, n32, n_dev, ids_out, L.st);
     if (hint)
-      PTC_KERNEL("k_ids_follow", s, k_ids_follow, ceil_div_u32(hint->n_req, kFoThreads / 32), kFoThreads, 0, ph,
-                 ids_out, L.st);
+      if (ph.order)
+        PTC_KERNEL("k_ids_follow", s, k_ids_follow_win, ceil_div_u32(hint->n_req, kFoThreads / 32), kFoThreads, 0,
+                   ph, ids_out, L.st);
+      else
+        PTC_KERNEL("k_ids_follow", s, k_ids_follow, ceil_div_u32(hint->n_req, kFoThreads / 32), kFoThreads, 0, ph,
+                   ids_out, L.st);
     return true;
   };
   const uint32_t first_log2m = full_table ? L.log2m : small_table_log2(n);
@@ -678,7 +768,7 @@ extern "C" ptc_status ptc_assign_ids_prior(const ptc_u128* keys, uint64_t n, con
   if (n == 0 || n_req == 0)
     return ptc::ids_impl(keys, n, nullptr, ids_out, nullptr, n_distinct_host_out, ws, ws_bytes,
                          (cudaStream_t)stream, nullptr, 0);
-  const IdsHint h{req_blk_off, req_prior, n_req};
+  const IdsHint h{req_blk_off, req_prior, n_req, nullptr, nullptr};
   return ptc::ids_impl(keys, n, nullptr, ids_out, nullptr, n_distinct_host_out, ws, ws_bytes, (cudaStream_t)stream,
                        nullptr, 0, nullptr, nullptr, nullptr, false, &h);
 }
@@ -695,7 +785,7 @@ size_t ptc::session_prior_bytes(uint32_t n_req) {
 // pass over neighbours.  Queued on `s`; a label >= n_session raises
 // kErrInvalid into *err.
 void ptc::session_prior(const uint32_t* req_session, uint32_t n_req, uint32_t n_session, uint32_t* prior, void* ws,
-                        cudaStream_t s, uint32_t* err) {
+                        cudaStream_t s, uint32_t* err, uint32_t* order, uint32_t* pos) {
   Carver cv(ws);
   DevStatus* st = cv.take<DevStatus>(1);  // the sort has no bound to check and raises nothing
   void* sws = cv.take<unsigned char>(sort_pairs_bytes(n_req ? n_req : 1));
@@ -704,7 +794,7 @@ void ptc::session_prior(const uint32_t* req_session, uint32_t n_req, uint32_t n_
   const uint32_t *ks = nullptr, *vs = nullptr;
   sort_pairs(req_session, nullptr, n_req, bits, sws, s, st, &ks, &vs);
   PTC_KERNEL("k_session_prior", s, k_session_prior, ceil_div_u32(n_req, 256), 256, 0, ks, vs, req_session, n_req,
-             n_session, prior, err);
+             n_session, prior, err, order, pos);
 }
 
 extern "C" size_t ptc_session_prior_workspace_bytes(uint32_t n_req) {
@@ -724,7 +814,7 @@ extern "C" ptc_status ptc_session_prior(const uint32_t* req_session, uint32_t n_
   DevStatus* st = cv.take<DevStatus>(1);
   void* sws = cv.take<unsigned char>(session_prior_bytes(n_req));
   if (begin_call(ws, kStatusBytes, s) != PTC_OK) return PTC_ERR_CUDA;
-  session_prior(req_session, n_req, n_session, prior_out, sws, s, &st->err);
+  session_prior(req_session, n_req, n_session, prior_out, sws, s, &st->err, nullptr, nullptr);
   DevStatus h;
   return end_call(st, s, &h);
 }

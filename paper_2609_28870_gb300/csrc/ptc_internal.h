@@ -206,6 +206,8 @@ struct IdsHint {
   const uint64_t* blk_off;  // n_req + 1 (device)
   const uint32_t* prior;    // n_req (device)
   uint32_t n_req;
+  const uint32_t* order;    // optional (device): the requests in session order, prior[r] = the place before r
+  const uint32_t* pos;      //   and the place of every request in it
 };
 size_t ids_ws_bytes(uint64_t n, uint32_t n_req_hint);
 // Whether the id table for n keys is larger than the part of L2 it may take:
@@ -216,7 +218,8 @@ bool ids_table_in_dram(uint64_t n);
 // queued on `s` without waiting; scratch of session_prior_bytes(n_req).
 size_t session_prior_bytes(uint32_t n_req);
 void session_prior(const uint32_t* req_session, uint32_t n_req, uint32_t n_session, uint32_t* prior, void* ws,
-                   cudaStream_t s, uint32_t* err);
+                   cudaStream_t s, uint32_t* err, uint32_t* order = nullptr,
+                   uint32_t* pos = nullptr);
 ptc_status ids_impl(const ptc_u128* keys, uint64_t n_ub, const uint64_t* n_dev, uint32_t* ids_out,
                     uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
                     cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc = nullptr,

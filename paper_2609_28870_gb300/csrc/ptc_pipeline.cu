@@ -21,6 +21,8 @@ struct PipeLayout {
   size_t curves_bytes;
   uint32_t* defer;  // error words of stages a1, prior, b, c and a2, read with a later stage's
   uint32_t* prior;  // previous request of each request's session (sessions given)
+  uint32_t* order;  // the requests in session order, and the place of each in it (sessions given)
+  uint32_t* pos;
   uint64_t* n_slot;  // N as stage a1 left it, for stage a2
   uint64_t* nd_slot;  // D and N as stage a2 left them, for stage b
   ulonglong2* carry;  // per hash tile: the carry stage a2 adds to the keys (when they are not returned)
@@ -54,6 +56,8 @@ PipeLayout pipe_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   L.curves = cv.take<unsigned char>(L.curves_bytes);
   L.defer = cv.take<uint32_t>(5);
   L.prior = cv.take<uint32_t>(n_req ? n_req : 1);
+  L.order = cv.take<uint32_t>(n_req ? n_req : 1);
+  L.pos = cv.take<uint32_t>(n_req ? n_req : 1);
   L.n_slot = cv.take<uint64_t>(1);
   L.nd_slot = cv.take<uint64_t>(2);
   const uint64_t ct = keys ? 1 : ptc::hash_carry_tiles(n_tok, B);
@@ -133,8 +137,9 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
   // table gains from it
   // (the labels are checked whenever they are given)
   const bool hinted = req_session != nullptr && n_req > 0 && ptc::ids_table_in_dram(cap);
-  if (req_session && n_req > 0) ptc::session_prior(req_session, n_req, n_session, L.prior, L.scratch, s, &L.defer[1]);
-  const ptc::IdsHint hint{blk, L.prior, n_req};
+  if (req_session && n_req > 0)
+    ptc::session_prior(req_session, n_req, n_session, L.prior, L.scratch, s, &L.defer[1], L.order, L.pos);
+  const ptc::IdsHint hint{blk, L.prior, n_req, L.order, L.pos};
   const ptc::IdsHint* hp = hinted ? &hint : nullptr;
   // keys the caller does not take skip their carry pass: stage a2 adds the
   // carry as it reads them
