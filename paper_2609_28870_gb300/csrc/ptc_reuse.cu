@@ -24,7 +24,8 @@
 //   k_ir_inc1      elementary intervals per run; last CTA: prefixes and K
 //   k_ir_inc2      the K incidences (e, r)
 //   (sort_pairs)   stable radix sort of the incidences by e
-//   k_ir_fill      one warp per incidence writes prev / next of its accesses
+//   k_ir_links     the first access of each incidence's neighbours on its e
+//   k_ir_fill      prev / next of every access, written in position order
 //
 // When the incidences exceed a quarter of the accesses the stage falls back
 // to sorting every access (ptc_sort.cu).
@@ -317,8 +318,11 @@ struct IncArgs {
   uint32_t* tcnt;
   uint32_t* tpre;
   uint32_t* done;
+  const uint32_t* cut_at;   // id of every cut, by rank
   uint32_t* key;            // incidences: elementary interval
-  uint32_t* val;            //             run
+  uint32_t* val;            //             index in position order (the order written here)
+  uint32_t* ipos;           // per incidence, in position order: its first access
+  uint32_t* ilen;           //                                   and its accesses
   uint32_t max_tiles;       // tiles of tcnt / tpre
   DevStatus* st;            // value[3] <- K
 };
@@ -374,52 +378,79 @@ __global__ void __launch_bounds__(kIT) k_ir_inc2(IncArgs a, uint32_t R) {
   uint32_t total;
   uint32_t o = a.tpre[t] + cta_excl_u32(c, s_w, &total);
 #pragma unroll
-  for (int k = 0; k < kRunPer; ++k)
+  for (int k = 0; k < kRunPer; ++k) {
+    if (f[k] == e[k]) continue;
+    const uint32_t s0 = a.rec_s[r0 + k] - a.rec_x[r0 + k];  // the position of id y in the run is s0 + y
+    uint32_t lo = a.cut_at[f[k]];
     for (uint32_t iv = f[k]; iv < e[k]; ++iv) {
+      const uint32_t hi = a.cut_at[iv + 1];
       a.key[o] = iv;
-      a.val[o] = r0 + k;
+      a.val[o] = o;
+      a.ipos[o] = s0 + lo;
+      a.ilen[o] = hi - lo;
+      lo = hi;
       ++o;
     }
+  }
 }
 
 struct FillArgs {
-  const uint32_t* key;     // sorted incidences
-  const uint32_t* val;
+  const uint32_t* key;     // sorted incidences: elementary interval
+  const uint32_t* val;     //                    index in position order
   uint32_t K, n;
-  const uint32_t* rec_s;
-  const uint32_t* rec_x;
-  const uint32_t* cut_at;  // id of every cut, by rank
+  const uint32_t* ipos;    // per incidence in position order: first access, accesses
+  const uint32_t* ilen;
+  uint32_t* ip0;           // per incidence in position order: first access of the previous / next
+  uint32_t* in0;           // incidence on the same interval, or none
   uint32_t* prev;
   uint32_t* next;
   const DevStatus* st;     // for the checked build's bounds checks
 };
 
-// One warp per incidence (e, r): the accesses of run r with ids in e take
-// their previous / next use from the runs before / after r on e.
+// For every incidence (e, r), the incidences on e before and after it in
+// time are its neighbours in the order sorted by e (a stable sort of the
+// incidences, written in run order, i.e. time order).  Their first accesses
+// go to the incidence's place in position order.
+__global__ void __launch_bounds__(256) k_ir_links(FillArgs a) {
+  grid_dep_sync();
+  const uint32_t q = blockIdx.x * blockDim.x + threadIdx.x;
+  if (q >= a.K) return;
+  const uint32_t e = a.key[q], o = a.val[q];
+  const uint32_t p = q > 0 && a.key[q - 1] == e ? a.ipos[a.val[q - 1]] : kNone;
+  const uint32_t x = q + 1 < a.K && a.key[q + 1] == e ? a.ipos[a.val[q + 1]] : kNone;
+  if (in_bounds(a.st, o, a.K)) {
+    a.ip0[o] = p;
+    a.in0[o] = x;
+  }
+}
+
+// prev / next of every access, written in position order: the incidences in
+// position order tile the accesses, so a warp takes 32 consecutive
+// incidences (their records read with one coalesced load per array) and
+// writes their accesses one incidence after another: each store of the warp
+// covers consecutive accesses, and neighbouring incidences complete each
+// other's sectors back to back.  The access at offset t of an incidence
+// whose neighbours start at p0 / n0 has prev p0 + t and next n0 + t (ids and
+// positions run in step inside an id-run).
 __global__ void __launch_bounds__(256) k_ir_fill(FillArgs a) {
   grid_dep_sync();
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t warps = gridDim.x * (blockDim.x >> 5);
-  for (uint32_t q = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; q < a.K; q += warps) {
-    const uint32_t e = a.key[q], r = a.val[q];
-    const bool has_pred = q > 0 && a.key[q - 1] == e;
-    const bool has_succ = q + 1 < a.K && a.key[q + 1] == e;
-    const uint32_t lo = a.cut_at[e], hi = a.cut_at[e + 1];
-    const uint32_t s0 = a.rec_s[r] + (lo - a.rec_x[r]);
-    uint32_t p0 = kNone, n0 = kNone;
-    if (has_pred) {
-      const uint32_t rp = a.val[q - 1];
-      p0 = a.rec_s[rp] + (lo - a.rec_x[rp]);
-    }
-    if (has_succ) {
-      const uint32_t rn = a.val[q + 1];
-      n0 = a.rec_s[rn] + (lo - a.rec_x[rn]);
-    }
-    for (uint32_t t = lane; t < hi - lo; t += 32) {
-      const uint32_t j = s0 + t;
-      if (in_bounds(a.st, j, a.n)) {
-        a.prev[j] = has_pred ? p0 + t : kNone;
-        a.next[j] = has_succ ? n0 + t : kNone;
+  for (uint32_t o0 = ((blockIdx.x * blockDim.x + threadIdx.x) >> 5) * 32; o0 < a.K; o0 += warps * 32) {
+    const uint32_t o = o0 + lane;
+    const bool live = o < a.K;
+    const uint32_t S = live ? a.ipos[o] : 0u, Ln = live ? a.ilen[o] : 0u;
+    const uint32_t P = live ? a.ip0[o] : kNone, X = live ? a.in0[o] : kNone;
+    const uint32_t nq = a.K - o0 < 32u ? a.K - o0 : 32u;
+    for (uint32_t i = 0; i < nq; ++i) {
+      const uint32_t si = __shfl_sync(kFull, S, i), li = __shfl_sync(kFull, Ln, i);
+      const uint32_t pi = __shfl_sync(kFull, P, i), xi = __shfl_sync(kFull, X, i);
+      for (uint32_t t = lane; t < li; t += 32) {
+        const uint32_t j = si + t;
+        if (in_bounds(a.st, j, a.n)) {
+          a.prev[j] = pi != kNone ? pi + t : kNone;
+          a.next[j] = xi != kNone ? xi + t : kNone;
+        }
       }
     }
   }
@@ -433,6 +464,7 @@ struct ReuseLayout {
   uint32_t *cut, *cwpre, *cut_at, *btcnt, *btpre;
   uint32_t *rtcnt, *rtpre;
   uint32_t *key, *val;
+  uint32_t *ipos, *ilen, *ip0, *in0;  // per incidence in position order
   void* sort_ws;
   uint32_t ntiles, nwords, btiles, rtiles_max;
   uint64_t kcap;
@@ -468,6 +500,10 @@ ReuseLayout reuse_layout(void* ws, uint64_t n, uint64_t D, bool forced) {
   L.rtpre = cv.take<uint32_t>(L.rtiles_max + 1);
   L.key = cv.take<uint32_t>(L.kcap);
   L.val = cv.take<uint32_t>(L.kcap);
+  L.ipos = cv.take<uint32_t>(L.kcap);
+  L.ilen = cv.take<uint32_t>(L.kcap);
+  L.ip0 = cv.take<uint32_t>(L.kcap);
+  L.in0 = cv.take<uint32_t>(L.kcap);
   L.sort_ws = cv.take<unsigned char>(sort_pairs_bytes(L.kcap));
   L.total = cv.bytes();
   return L;
@@ -519,8 +555,11 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
   ia.tcnt = L.rtcnt;
   ia.tpre = L.rtpre;
   ia.done = &L.done[2];
+  ia.cut_at = L.cut_at;
   ia.key = L.key;
   ia.val = L.val;
+  ia.ipos = L.ipos;
+  ia.ilen = L.ilen;
   ia.max_tiles = L.rtiles_max;
   ia.st = L.st;
   const uint32_t g1 = L.rtiles_max < (uint32_t)(2 * num_sms()) ? L.rtiles_max : (uint32_t)(2 * num_sms());
@@ -551,14 +590,16 @@ ptc_status reuse_by_runs(const uint32_t* ids, uint64_t n, uint64_t D, uint32_t* 
   f.val = sval;
   f.K = (uint32_t)K;
   f.n = (uint32_t)n;
-  f.rec_s = L.rec_s;
-  f.rec_x = L.rec_x;
-  f.cut_at = L.cut_at;
+  f.ipos = L.ipos;
+  f.ilen = L.ilen;
+  f.ip0 = L.ip0;
+  f.in0 = L.in0;
   f.prev = prev_out;
   f.next = next_out;
   f.st = L.st;
-  const uint32_t fill_blocks = ceil_div_u32(K, 8) < (uint32_t)(16 * num_sms()) ? ceil_div_u32(K, 8)
-                                                                                : (uint32_t)(16 * num_sms());
+  PTC_KERNEL("k_ir_links", s, k_ir_links, ceil_div_u32(K, 256), 256, 0, f);
+  const uint32_t fill_blocks = ceil_div_u32(K, 256) < (uint32_t)(8 * num_sms()) ? ceil_div_u32(K, 256)
+                                                                                : (uint32_t)(8 * num_sms());
   PTC_KERNEL("k_ir_fill", s, k_ir_fill, fill_blocks, 256, 0, f);
   if (defer_err) return defer_status(L.st, defer_err, s);
   return end_call(L.st, s, &h);
