@@ -426,7 +426,8 @@ size_t ptc_pipeline_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t blo
  * ptc_pipeline_table_fill_bytes — bytes of stage a2's id table that
  * ptc_pipeline has the block-hash grid of stage a1 set to all ones while it
  * hashes (the hash is bound by integer issue, so the fill uses DRAM time it
- * leaves idle); 0 when stage a2 fills its own table.  with_sessions: whether
+ * leaves idle); 0 when stage a2 fills its own table (a table that fits in
+ * L2, or one that would overlap stage a1's scratch).  with_sessions: whether
  * the call passes req_session.  For reporting the hash kernel's bytes; it
  * allocates and launches nothing.
  */

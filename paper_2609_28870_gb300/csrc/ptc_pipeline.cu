@@ -67,13 +67,16 @@ PipeLayout pipe_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   return L;
 }
 
-// Stage a2's first table inside the scratch region, and whether it lies
-// past the scratch that stages a1 (and the session sort before it) use, so
-// that the hash grid may fill it while stage a1 runs.
+// Stage a2's first table inside the scratch region, and whether the hash
+// grid fills it while stage a1 runs: only a DRAM-sized table (a table that
+// fits in L2 is better filled by stage a2 just before its insert, which then
+// finds it in L2), and only when it lies past the scratch that stage a1
+// (and the session sort before it) use.
 bool fused_table_fill(void* scratch, uint32_t n_req, uint64_t n_tok, uint32_t B, bool hinted, void** table,
                       size_t* bytes) {
   const uint64_t cap = n_tok / B ? n_tok / B : 1;
   ptc::ids_table_region(scratch, cap, hinted ? n_req : 0, table, bytes);
+  if (!ptc::ids_table_in_dram(cap)) return false;
   const size_t front = std::max(ptc_hash_blocks_workspace_bytes(n_req, n_tok, B), ptc::session_prior_bytes(n_req));
   return *bytes > 0 && static_cast<char*>(*table) >= static_cast<char*>(scratch) + front;
 }
