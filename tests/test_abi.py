@@ -148,3 +148,16 @@ def test_pipeline_table_fill_bytes(libptc):
         assert b % 16 == 0 and slots & (slots - 1) == 0
         assert slots >= (n // 4 * 3 if slots > (1 << 22) else n // 3)
     assert f(582163, 9984375026, 16, 1) == 16 << 29
+
+
+def test_probe_random_rmw_rejects_bad_tables(libptc):
+    """Argument checks come before any CUDA call."""
+    f = libptc.ptc_probe_random_rmw
+    f.restype = ctypes.c_int
+    f.argtypes = [ctypes.c_void_p, ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint64, ctypes.c_void_p, ctypes.c_void_p]
+    invalid = 1
+    assert f(None, 1024, 10, 0, 256, None) == invalid            # no table
+    assert f(4096, 1000, 10, 0, 256, None) == invalid            # slots not a power of two
+    assert f(4104, 1024, 10, 0, 256, None) == invalid            # table not 16-byte aligned
+    assert f(4096, 1024, 10, 0, 260, None) == invalid            # sink not 8-byte aligned
+    assert f(4096, 1024, 0, 0, 256, None) == 0                   # no probes: nothing to do
