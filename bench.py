@@ -263,6 +263,34 @@ WORKLOAD_NAMES = {
 GOLDEN = os.path.join(ROOT, "tests", "golden", "big_configs.json")
 
 
+_HOST_BUFFERS = []  # registered host buffers: kept alive, unregistered at exit
+
+
+def registered_host_u32(n):
+    """n uint32 in page-locked host memory: an anonymous mapping asked for huge
+    pages, then registered with CUDA (cudaHostRegister).  Copies from it ran at
+    the host link's full 211 GB/s on a GB300 machine whether or not the box had
+    just run the whole test suite, where a buffer from torch's pinned-memory
+    allocator copied at 84-211 GB/s on its first passes."""
+    import atexit
+    import mmap
+
+    import numpy as np
+    import torch
+    nbytes = max(4 * int(n), 4096)
+    m = mmap.mmap(-1, nbytes, flags=mmap.MAP_PRIVATE | mmap.MAP_ANONYMOUS)
+    if hasattr(mmap, "MADV_HUGEPAGE"):
+        m.madvise(mmap.MADV_HUGEPAGE)
+    a = np.frombuffer(m, dtype=np.uint32, count=int(n))
+    rt = torch.cuda.cudart()
+    if int(rt.cudaHostRegister(a.ctypes.data, nbytes, 0)) != 0:
+        raise RuntimeError("cudaHostRegister failed for the token buffer")
+    _HOST_BUFFERS.append((m, a))
+    if len(_HOST_BUFFERS) == 1:
+        atexit.register(lambda: [rt.cudaHostUnregister(b.ctypes.data) for _, b in _HOST_BUFFERS])
+    return a
+
+
 def load_trace(workload, requests, dev):
     """The workload generated into page-locked host memory (the end-to-end leg
     copies from it) and copied once to the device."""
@@ -274,8 +302,9 @@ def load_trace(workload, requests, dev):
         tok_host = torch.from_numpy(tr.tokens.view(np.int32)).pin_memory()
     else:
         _, T, _ = tracegen.sizes(workload)
-        tok_host = torch.empty(T, dtype=torch.int32, pin_memory=True)
-        tr = tracegen.make(workload, token_buffer=tok_host.numpy().view(np.uint32))
+        buf = registered_host_u32(T)
+        tr = tracegen.make(workload, token_buffer=buf)
+        tok_host = torch.from_numpy(buf.view(np.int32))
     off_host = torch.from_numpy(tr.req_tok_off.view(np.int64)).pin_memory()
     ts_host = torch.from_numpy(tr.req_ts_us).pin_memory()
     ses_host = torch.from_numpy(np.ascontiguousarray(tr.req_session, dtype=np.uint32).view(np.int32)).pin_memory()
@@ -543,7 +572,8 @@ def run_ours(args, ws_world, rank, local):
     # runs the path and returns the curves to host memory
     hplan = ptc.HostPipelinePlan(*host_t[:3], BLOCK, caps, kind=ptc.PTC_COST_MEASURED, seed=0, device=dev,
                                  req_session=host_t[3], n_session=tr.n_sessions)
-    hplan.run()
+    for _ in range(max(args.warmup, 3)):  # the first copies out of a new page-locked buffer run slow
+        hplan.run()
     assert np.array_equal(hplan.hits, ref[0]) and np.array_equal(hplan.saved, ref[1])
     e2e_total = slowest(sum(timer.run(args.steps, hplan.run, hplan, ref)))
     h2d = 4 * T + 8 * (R + 1) + 8 * R + 4 * R
