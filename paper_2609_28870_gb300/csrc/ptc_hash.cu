@@ -520,8 +520,8 @@ constexpr int kH16Req = 256;
 // token is left to k_hash16_wide (its index goes to wide_list) and returns
 // before it writes anything.  WIDE = true: three-limb products, exact for
 // every 32-bit token.  Keeping the three-limb code out of the common kernel
-// keeps that kernel's registers free of it (it spilled, and measured 1.0 ms
-// slower on the mixed 10B-token trace).
+// keeps that kernel's registers free of it (with it the kernel spilled more
+// and took 0.7 ms longer on the mixed 10B-token trace).
 template <bool WIDE>
 __device__ __forceinline__ void hash16_tile(const HashArgs& a, const HashConsts& c, uint32_t tile, uint64_t N) {
   __shared__ uint64_t s_boff[kH16Req + 1];
