@@ -58,7 +58,7 @@ NOMINAL_HBM_GBS = 7900.0
 # "no counters", null) and how the capture was scaled to a full launch.
 NCU_TRAFFIC: dict[tuple[str, int], tuple[float, str, str]] = {
     ("k_hash16", 1): (645.6e6, "35e274868498a45b", "ncu --set full, first 6,000 requests, x 153.81 / 55.67"),
-    ("k_hash16", 3): (5.8443e+10, "8e5be046caac3151", "ncu --set full, first 60,000 requests: reads x tokens (9984.4M / 943.9M), "
+    ("k_hash16", 3): (5.8443e+10, "1cb4fded74c0cfbc", "ncu --set full, first 60,000 requests: reads x tokens (9984.4M / 943.9M), "
                       "key writes x blocks (623.75M / 58.97M), plus the full id-table fill (8.59 GB)"),
 }
 
