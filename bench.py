@@ -57,9 +57,9 @@ NOMINAL_HBM_GBS = 7900.0
 # sha256 prefix of the source file it was taken on (a changed source reads as
 # "no counters", null) and how the capture was scaled to a full launch.
 NCU_TRAFFIC: dict[tuple[str, int], tuple[float, str, str]] = {
-    ("k_hash16", 1): (645.6e6, "35e274868498a45b", "ncu --set full, first 6,000 requests, x 153.81 / 55.67"),
-    ("k_hash16", 3): (5.8443e+10, "1cb4fded74c0cfbc", "ncu --set full, first 60,000 requests: reads x tokens (9984.4M / 943.9M), "
-                      "key writes x blocks (623.75M / 58.97M), plus the full id-table fill (8.59 GB)"),
+    ("k_hash16", 1): (6.3766e+08, "d33ef0cf44921375", "ncu dram__bytes metrics, first 6,000 requests, x 153.81 / 55.67"),
+    ("k_hash16", 3): (4.9715e+10, "d33ef0cf44921375", "ncu dram__bytes metrics, first 60,000 requests: reads x tokens "
+                      "(9984.4M / 943.9M), key writes x blocks (623.75M / 58.97M)"),
 }
 
 
@@ -152,16 +152,24 @@ def sort_passes(D):
     return (b + 7) // 8
 
 
-def kernel_model_bytes(name, T, N, L, D, fill=0):
+def kernel_model_bytes(name, T, N, L, D, U=None):
     """Algorithmic bytes one launch of `name` moves under the stage-byte model
-    (0: the kernel only touches scratch the model does not count).  `fill`:
-    the bytes of stage a2's id table that the pipeline has the hash grid set
-    (ptc_pipeline_table_fill_bytes), written by the hash kernel."""
+    (0: the kernel only touches scratch the model does not count).  `U`: the
+    accesses the partitioned dedup settles (those the prior-request hint does
+    not match), for its kernels; None leaves them at 0."""
     per_level = ((L - 1) * 8.125 + 4.125) / L * N  # the last level writes no partition
+    pd = {} if U is None else {
+        "k_pd_flags": N / 4,               # the settled-access bitmap and its copy out
+        "k_pd_count": 16 * U + N / 8,      # settled keys (whole 32-byte sectors) and the bitmap in
+        "k_pd_scatter1": 32 * U + N / 8,   # settled keys in, bucket records out
+        "k_pd_count2": 16 * U,             # records in
+        "k_pd_scatter2": 32 * U,           # records in, partition records out
+        "k_pd_dedup": 16 * U,              # records in
+    }
     return {
-        "k_hash_local": 4 * T + 16 * N + fill,   # token stream in, block keys (and the table fill) out
-        "k_hash16": 4 * T + 16 * N + fill,       # the same, B = 16 path
-        "k_hash_tile": 4 * T + 16 * N + fill,    # the same, other multiples of 16
+        "k_hash_local": 4 * T + 16 * N,   # token stream in, block keys out
+        "k_hash16": 4 * T + 16 * N,       # the same, B = 16 path
+        "k_hash_tile": 4 * T + 16 * N,    # the same, other multiples of 16
         "k_ids_insert": 16 * N,           # keys in
         "k_ids_insert_prior": 16 * N,     # keys in (the same stage, prior-request hint)
         "k_ids_gather": 4 * N,            # ids out
@@ -173,6 +181,7 @@ def kernel_model_bytes(name, T, N, L, D, fill=0):
         "k_runs_mark": 4 * N,             # prev in (matrix over runs)
         "k_runs_expand": 4 * N,           # distances out (matrix over runs)
         "k_curves": 4 * N,                # distances in
+        **pd,
     }.get(name, 0.0)
 
 
@@ -191,7 +200,9 @@ KERNEL_SOURCE = {
     "k_curves": "ptc_curves.cu", "k_finalize": "ptc_curves.cu", "k_curves_fast": "ptc_curves.cu",
     "k_curves_runs": "ptc_curves.cu", "k_fill": "ptc_abi.cu", "k_copy_words": "ptc_abi.cu",
     "k_copy_err": "ptc_abi.cu", "k_carry_err": "ptc_abi.cu", "k_hash_carry": "ptc_hash.cu",
-    "k_rank_count": "ptc_abi.cu", "k_rank_words": "ptc_abi.cu",
+    "k_rank_count": "ptc_abi.cu", "k_rank_words": "ptc_abi.cu", "k_pd_flags": "ptc_ids.cu",
+    "k_pd_count": "ptc_ids.cu", "k_pd_rows1": "ptc_ids.cu", "k_pd_scatter1": "ptc_ids.cu",
+    "k_pd_count2": "ptc_ids.cu", "k_pd_rows2": "ptc_ids.cu", "k_pd_scatter2": "ptc_ids.cu", "k_pd_dedup": "ptc_ids.cu",
 }
 
 
@@ -353,11 +364,11 @@ class Timer:
         return ms
 
 
-def kernel_table(ktimes, steps, T, N, D, Lbits, fill=0):
+def kernel_table(ktimes, steps, T, N, D, Lbits, U=None):
     kernels = []
     for name, launches_k, tot_ms in ktimes:
         per = tot_ms / max(launches_k, 1)
-        mb = kernel_model_bytes(name, T, N, Lbits, D, fill)
+        mb = kernel_model_bytes(name, T, N, Lbits, D, U)
         kernels.append({"name": name, "launches_per_step": launches_k / steps, "ms_per_step": tot_ms / steps,
                         "avg_launch_ms": per, "model_bytes_per_launch": mb,
                         "achieved_gbs": (mb / (per * 1e-3) / 1e9) if per > 0 else 0.0})
@@ -407,16 +418,25 @@ def hint_matched(ptc, torch, ids, blk_off, ses):
     return matched
 
 
-def id_table_roofline(ptc, torch, L, kernels, n_access, matched, table_bytes, dev):
-    """k_ids_insert_prior against the rate at which this GPU settles random
-    16-byte read-modify-write probes of a table of the same size, measured in
-    this run (ptc_probe_random_rmw): the insert's bound is that rate, not the
-    copy bandwidth."""
-    ins = next((k for k in kernels if k["name"] == "k_ids_insert_prior"), None)
-    if ins is None or table_bytes <= 0:
+PD_KERNELS = ("k_pd_flags", "k_pd_count", "k_pd_rows1", "k_pd_scatter1", "k_pd_count2", "k_pd_rows2",
+              "k_pd_scatter2", "k_pd_dedup")
+
+
+def id_stage(ptc, torch, L, kernels, n_access, matched, peak, dev):
+    """The partitioned dedup's kernels against the measured copy bandwidth
+    (they stream their records), and, for comparison, the time a hash table
+    of DRAM size would need at best: the accesses it settles at the rate
+    this GPU completes random 16-byte read-modify-writes on such a table,
+    measured in this run (ptc_probe_random_rmw)."""
+    pd = [k for k in kernels if k["name"] in PD_KERNELS]
+    if not pd:
         return None
-    probes = n_access - matched
-    slots = table_bytes // 16
+    settled = n_access - matched
+    ms = sum(k["avg_launch_ms"] for k in pd)
+    mb = sum(k["model_bytes_per_launch"] for k in pd)
+    slots = 1
+    while slots < n_access // 4 * 3 + 64:  # the table method's first size for a DRAM-sized table
+        slots *= 2
     table = torch.empty(slots * 2, dtype=torch.int64, device=dev)
     sink = torch.zeros(1, dtype=torch.int64, device=dev)
     stream = torch.cuda.current_stream(dev)
@@ -425,22 +445,24 @@ def id_table_roofline(ptc, torch, L, kernels, n_access, matched, table_bytes, de
         table.fill_(-1)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        rc = L.ptc_probe_random_rmw(table.data_ptr(), slots, probes, 0x5EED + rep, sink.data_ptr(), stream.cuda_stream)
+        rc = L.ptc_probe_random_rmw(table.data_ptr(), slots, settled, 0x5EED + rep, sink.data_ptr(), stream.cuda_stream)
         e1.record(stream)
         e1.synchronize()
         if rc != 0:
             raise RuntimeError(f"ptc_probe_random_rmw failed ({rc})")
-        ms = e0.elapsed_time(e1)
-        best = ms if best is None else min(best, ms)
+        t = e0.elapsed_time(e1)
+        best = t if best is None else min(best, t)
     del table, sink
-    achieved = probes / (ins["avg_launch_ms"] * 1e-3) / 1e9
-    peak = probes / (best * 1e-3) / 1e9
-    return {"kernel": "k_ids_insert_prior", "bound": "hbm random read-modify-write", "probes": probes,
-            "matched_by_hint": matched, "ms": round(ins["avg_launch_ms"], 4),
-            "achieved_gprobes_per_s": round(achieved, 2), "peak_gprobes_per_s": round(peak, 2),
-            "frac": round(achieved / peak, 4), "table_bytes": table_bytes,
-            "peak_how": "ptc_probe_random_rmw in this run: the same number of 16-byte slot loads at seeded random "
-                        "slots of an all-ones table of the same size, each claimed by a 128-bit CAS; best of 3"}
+    achieved = mb / (ms * 1e-3) / 1e9
+    return {"method": "partitioned dedup (65,536 partitions by 16 key bits, shared-memory tables)",
+            "settled": settled, "matched_by_hint": matched, "ms": round(ms, 4),
+            "model_bytes": int(mb), "achieved_gbs": round(achieved, 1), "peak": peak,
+            "frac": round(achieved / peak, 4),
+            "kernels_ms": {k["name"]: round(k["avg_launch_ms"], 4) for k in pd},
+            "table_bound_ms": round(best, 4),
+            "table_bound_how": "ptc_probe_random_rmw in this run: one random 16-byte slot load plus a 128-bit CAS "
+                               f"claim per settled access, on an all-ones table of {slots * 16 / 1e9:.2f} GB; best "
+                               "of 3 (a lower bound for the hash-table method's insert)"}
 
 
 def hbm_fractions(T, N, ms, peak):
@@ -548,13 +570,10 @@ def run_ours(args, ws_world, rank, local):
     L.ptc_timer_enable(0)
     ktimes = read_timer(ptc)
     hbm, Lbits = hbm_fractions(T, N, ms_per_step, peak)
-    kernels = kernel_table(ktimes, args.steps, T, N, D, Lbits, L.ptc_pipeline_table_fill_bytes(R, T, BLOCK, 1))
-    roof = roofline_of(kernels, peak, peak_kind, W)
-    gold = golden_parity(W, N, D, plan.hits, plan.result()["saved"], caps) if not args.requests else None
-    # the id table's insert against the random read-modify-write rate (one
-    # more step with the ids kept, to count the accesses the hint matches)
-    id_table = None
-    if any(k["name"] == "k_ids_insert_prior" for k in kernels):
+    # the accesses the prior-request hint matches (one more step with the
+    # ids kept): the partitioned dedup settles the others
+    matched = None
+    if any(name in PD_KERNELS for name, _, _ in ktimes):
         ids_t = torch.empty(N, dtype=torch.int32, device=dev)
         boff_t = torch.empty(R + 1, dtype=torch.int64, device=dev)
         ptc.PipelinePlan(tok, off, ts, BLOCK, caps, kind=ptc.PTC_COST_MEASURED, seed=0, ws=ws,
@@ -562,8 +581,10 @@ def run_ours(args, ws_world, rank, local):
                          n_session=tr.n_sessions).run()
         matched = hint_matched(ptc, torch, ids_t, boff_t, ses)
         del ids_t, boff_t
-        id_table = id_table_roofline(ptc, torch, L, kernels, N, matched,
-                                     L.ptc_pipeline_table_fill_bytes(R, T, BLOCK, 1), dev)
+    kernels = kernel_table(ktimes, args.steps, T, N, D, Lbits, None if matched is None else N - matched)
+    roof = roofline_of(kernels, peak, peak_kind, W)
+    gold = golden_parity(W, N, D, plan.hits, plan.result()["saved"], caps) if not args.requests else None
+    ids_summary = id_stage(ptc, torch, L, kernels, N, matched, peak, dev) if matched is not None else None
     del plan, ws, tok, off, ts, ses, dev_t
     torch.cuda.empty_cache()
 
@@ -606,7 +627,7 @@ def run_ours(args, ws_world, rank, local):
         "gpu_launches": launches,
         "clocks": clk,
         "parity_with_oracle_golden": gold,
-        "id_table_roofline": id_table,
+        "id_stage": ids_summary,
     }
 
     # ---- the oracle on a bounded prefix of the same workload, and the GPU
@@ -675,7 +696,7 @@ def chat_extras(args, ptc, tracegen, dev, timer, slowest, peak, peak_kind, rank,
     timer.run(args.steps, plan.run, plan, ref)
     L.ptc_timer_enable(0)
     hbm, Lbits = hbm_fractions(T, N, ms, peak)
-    kernels = kernel_table(read_timer(ptc), args.steps, T, N, D, Lbits, L.ptc_pipeline_table_fill_bytes(R, T, BLOCK, 1))
+    kernels = kernel_table(read_timer(ptc), args.steps, T, N, D, Lbits)
     out = {"workload": WORKLOAD_NAMES[CHAT], "tokens": T, "requests": R, "accesses": N, "distinct_blocks": D,
            "capacities": G, "ms_per_step": round(ms, 4), "tokens_per_s": round(ws_world * T / (ms * 1e-3), 1),
            "accesses_per_s": round(ws_world * N / (ms * 1e-3), 1), "hbm_roofline": hbm,

@@ -176,6 +176,31 @@ ptc_status ptc_assign_ids_prior(const ptc_u128* keys, uint64_t n, const uint64_t
                                 size_t ws_bytes, void* stream);
 
 /*
+ * ptc_assign_ids_ex — ptc_assign_ids (n_req = 0) or ptc_assign_ids_prior
+ * (n_req > 0, same hint rules) with the way keys are deduplicated named.
+ * Every method gives the same ids and D:
+ *   PTC_IDS_TABLE        one open-addressing table of 16-byte slots: a first
+ *                        attempt with n / 3 slots (3 n / 4 once that is larger
+ *                        than 64 MB), the whole stage again with 1.5 n slots
+ *                        if a probe sequence outruns it
+ *   PTC_IDS_PARTITIONED  the keys to settle are moved, in streaming passes,
+ *                        into 65,536 partitions by 16 key bits, and each
+ *                        partition is deduplicated in a table in shared
+ *                        memory; a partition with more than 6,144 distinct
+ *                        keys sends the stage to the full table as above
+ *   PTC_IDS_AUTO         PTC_IDS_PARTITIONED when the first table would exceed
+ *                        64 MB (n above about 12.6M), else PTC_IDS_TABLE; what
+ *                        ptc_assign_ids and ptc_assign_ids_prior do
+ * Workspace: ptc_assign_ids_ex_workspace_bytes(n, n_req, method).  An
+ * unknown method is PTC_ERR_INVALID_ARG.
+ */
+enum { PTC_IDS_AUTO = 0, PTC_IDS_TABLE = 1, PTC_IDS_PARTITIONED = 2 };
+size_t ptc_assign_ids_ex_workspace_bytes(uint64_t n, uint32_t n_req, int method);
+ptc_status ptc_assign_ids_ex(const ptc_u128* keys, uint64_t n, const uint64_t* req_blk_off, const uint32_t* req_prior,
+                             uint32_t n_req, uint32_t* ids_out, uint64_t* n_distinct_host_out, int method, void* ws,
+                             size_t ws_bytes, void* stream);
+
+/*
  * ptc_session_prior — the hint above from session labels (Sec. 2.3,
  * sessions): prior_out[r] = the latest request before r with the same label,
  * or PTC_NONE for a session's first request.  req_session u32[n_req], labels
@@ -422,16 +447,6 @@ ptc_status ptc_session_lru_curves(const uint32_t* ids, uint64_t n, uint64_t n_di
  * wait for their own status; an error they raise is returned with stage d's.
  */
 size_t ptc_pipeline_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size, uint32_t n_cap);
-/*
- * ptc_pipeline_table_fill_bytes — bytes of stage a2's id table that
- * ptc_pipeline has the block-hash grid of stage a1 set to all ones while it
- * hashes (the hash is bound by integer issue, so the fill uses DRAM time it
- * leaves idle); 0 when stage a2 fills its own table (a table that fits in
- * L2, or one that would overlap stage a1's scratch).  with_sessions: whether
- * the call passes req_session.  For reporting the hash kernel's bytes; it
- * allocates and launches nothing.
- */
-size_t ptc_pipeline_table_fill_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size, int with_sessions);
 ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off, const int64_t* req_ts_us,
                         const uint32_t* req_session, uint32_t n_session, uint32_t n_req, uint32_t block_size, uint64_t seed, const ptc_cost_model* cm,
                         const uint64_t* cap_host, uint32_t n_cap, ptc_u128* keys_out, uint64_t* req_blk_off_out,

@@ -30,6 +30,7 @@ PTC_NONE = 0xFFFFFFFF
 PTC_COST_UNIFORM, PTC_COST_MEASURED, PTC_COST_LINEAR = 0, 1, 2
 PTC_SD_AUTO, PTC_SD_POINTS, PTC_SD_RUNS = 0, 1, 2
 PTC_REUSE_AUTO, PTC_REUSE_SORT, PTC_REUSE_RUNS = 0, 1, 2
+PTC_IDS_AUTO, PTC_IDS_TABLE, PTC_IDS_PARTITIONED = 0, 1, 2
 PTC_TOUCH_ROOT_FIRST, PTC_TOUCH_LEAF_FIRST = 0, 1
 PTC_RESIDENCY_BLOCK, PTC_RESIDENCY_REQUEST = 0, 1
 F_LIN = 6_600_000_000          # 2 x 3.3e9 active parameters, FLOPs per token
@@ -135,8 +136,6 @@ def lib():
                 L.ptc_pipeline_workspace_bytes.argtypes = [u32, u64, u32, u32]
                 L.ptc_probe_random_rmw.restype = st
                 L.ptc_probe_random_rmw.argtypes = [vp, u64, u64, u64, vp, vp]
-                L.ptc_pipeline_table_fill_bytes.restype = sz
-                L.ptc_pipeline_table_fill_bytes.argtypes = [u32, u64, u32, ctypes.c_int]
                 L.ptc_pipeline.restype = st
                 L.ptc_pipeline.argtypes = [vp, u64, vp, vp, vp, u32, u32, u32, u64, ctypes.POINTER(CostModel), vp, u32,
                                            vp, vp, vp, vp, vp, vp, ctypes.POINTER(u64), ctypes.POINTER(u64), vp, vp,
@@ -158,6 +157,10 @@ def lib():
                 L.ptc_belady_curves.restype = st
                 L.ptc_belady_curves.argtypes = [vp, u64, vp, u32, u32, ctypes.POINTER(CostModel), vp, u32, vp, vp, vp,
                                                 vp, sz, vp]
+                L.ptc_assign_ids_ex_workspace_bytes.restype = sz
+                L.ptc_assign_ids_ex_workspace_bytes.argtypes = [u64, u32, ctypes.c_int]
+                L.ptc_assign_ids_ex.restype = st
+                L.ptc_assign_ids_ex.argtypes = [vp, u64, vp, vp, u32, vp, ctypes.POINTER(u64), ctypes.c_int, vp, sz, vp]
                 L.ptc_assign_ids_prior_workspace_bytes.restype = sz
                 L.ptc_assign_ids_prior_workspace_bytes.argtypes = [u64, u32]
                 L.ptc_assign_ids_prior.restype = st
@@ -331,6 +334,23 @@ def ptc_assign_ids_prior(keys: torch.Tensor, req_blk_off: torch.Tensor, req_prio
     rc = lib().ptc_assign_ids_prior(_ptr(keys), n, _ptr(req_blk_off), _ptr(req_prior), R, _ptr(ids), ctypes.byref(d),
                                     _ptr(w), w.numel(), _stream(dev))
     _check("ptc_assign_ids_prior", rc)
+    return ids[:n], int(d.value)
+
+
+def ptc_assign_ids_ex(keys: torch.Tensor, method: int, req_blk_off: torch.Tensor | None = None,
+                      req_prior: torch.Tensor | None = None, ws: torch.Tensor | None = None):
+    """Dense ids by the named dedup method (PTC_IDS_AUTO / PTC_IDS_TABLE /
+    PTC_IDS_PARTITIONED), with the prior-request hint when req_blk_off and
+    req_prior are given.  Returns (ids int32[N], D)."""
+    dev = _dev(keys)
+    n = keys.shape[0]
+    R = req_prior.numel() if req_prior is not None else 0
+    ids = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
+    d = ctypes.c_uint64(0)
+    w = _workspace(lib().ptc_assign_ids_ex_workspace_bytes(n, R, method), dev, ws)
+    rc = lib().ptc_assign_ids_ex(_ptr(keys), n, _ptr(req_blk_off) if R else None, _ptr(req_prior) if R else None, R,
+                                 _ptr(ids), ctypes.byref(d), method, _ptr(w), w.numel(), _stream(dev))
+    _check("ptc_assign_ids_ex", rc)
     return ids[:n], int(d.value)
 
 

@@ -222,21 +222,7 @@ struct HashArgs {
   DevStatus* st;
   int aligned;
   uint32_t* wide_list;  // k_hash16: tiles left to k_hash16_wide (their count in st->tile_ctr[kEpochWide])
-  uint4* fill;          // a region the caller asked the hash grid to set to all ones, or null
-  uint64_t fill_units;  // its 16-byte units
 };
-
-// The hash kernels are bound by integer issue, not by DRAM, so a fill that
-// a later stage needs (the pipeline's id table) runs inside them: CTA x
-// writes all ones to units [x c, x c + c) of a.fill, c = ceil(units / grid),
-// before it looks at its own blocks.
-__device__ __forceinline__ void fill_share(const HashArgs& a) {
-  if (a.fill_units == 0) return;
-  const uint64_t c = (a.fill_units + gridDim.x - 1) / gridDim.x;
-  const uint64_t u0 = (uint64_t)blockIdx.x * c;
-  const uint64_t u1 = u0 + c < a.fill_units ? u0 + c : a.fill_units;
-  for (uint64_t u = u0 + threadIdx.x; u < u1; u += blockDim.x) __stcs(&a.fill[u], make_uint4(~0u, ~0u, ~0u, ~0u));
-}
 
 __device__ __forceinline__ uint32_t pad16(uint32_t i) { return i + (i >> 4); }
 
@@ -394,7 +380,6 @@ __device__ __forceinline__ void hash_finish(const HashArgs& a, uint32_t tile, ui
 template <int G, bool FULL>
 __global__ void __launch_bounds__(kHashThreads) k_hash_local(HashArgs a, const __grid_constant__ HashConsts c) {
   grid_dep_sync();
-  fill_share(a);
   __shared__ uint32_t s_tok[kWinWords];
   __shared__ uint64_t s_bnd[4];
   constexpr uint32_t TB = kHashThreads / G;
@@ -754,7 +739,6 @@ __device__ __forceinline__ void hash16_tile(const HashArgs& a, const HashConsts&
 
 __global__ void __launch_bounds__(kHashThreads, 8) k_hash16(HashArgs a, const __grid_constant__ HashConsts c) {
   grid_dep_sync();
-  fill_share(a);
   hash16_tile<false>(a, c, blockIdx.x, blocks_live(a.st, a.keys_cap));
 }
 
@@ -852,7 +836,6 @@ constexpr int kTileReq = 256;
 __global__ void __launch_bounds__(kHashThreads, 4) k_hash_tile(HashArgs a, const __grid_constant__ HashConsts c) {
   constexpr uint32_t TB = kHashThreads;
   grid_dep_sync();
-  fill_share(a);
   __shared__ uint64_t s_boff[kTileReq + 1];
   __shared__ uint64_t s_toff[kTileReq + 1];
   __shared__ uint64_t s_p0[TB], s_p1[TB];
@@ -1221,9 +1204,7 @@ ptc_status ptc::hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t
                          const int64_t* req_ts_us, uint32_t n_req, uint32_t block_size, uint64_t seed,
                          ptc_u128* keys_out, uint64_t keys_cap, uint64_t* req_blk_off_out,
                          uint64_t* n_access_host_out, void* ws, size_t ws_bytes, cudaStream_t s, uint64_t* n_slot,
-                         uint32_t* err_slot, KeyCarry* carry, void* fill_ones, size_t fill_bytes) {
-  if (fill_bytes && (fill_ones == nullptr || (fill_bytes & 15) != 0 || ((uintptr_t)fill_ones & 15) != 0))
-    return PTC_ERR_INVALID_ARG;
+                         uint32_t* err_slot, KeyCarry* carry) {
   if (block_size < 1 || block_size > PTC_MAX_BLOCK_SIZE) return PTC_ERR_INVALID_ARG;
   if (req_tok_off == nullptr || req_blk_off_out == nullptr || n_access_host_out == nullptr)
     return PTC_ERR_INVALID_ARG;
@@ -1238,7 +1219,6 @@ ptc_status ptc::hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t
   const uint32_t wait_test = test_wait_polls();
   if (wait_test && fill_async(&L.st->wait_test, wait_test, sizeof(uint32_t), s) != PTC_OK) return PTC_ERR_CUDA;
   if (n_req == 0) {
-    if (fill_bytes && fill_async(fill_ones, ~0u, fill_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
     if (fill_async(req_blk_off_out, 0u, sizeof(uint64_t), s) != PTC_OK) return PTC_ERR_CUDA;
     if (deferred) return defer_status(L.st, err_slot, s, n_slot, 0);
     DevStatus h;
@@ -1292,9 +1272,6 @@ ptc_status ptc::hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t
   const bool full = block_size == 16 * G;
   const uint64_t nb = n_tok / block_size < keys_cap ? n_tok / block_size : keys_cap;
   const uint32_t grid = ceil_div_u32(nb, tb);
-  a.fill = grid > 0 ? reinterpret_cast<uint4*>(fill_ones) : nullptr;
-  a.fill_units = grid > 0 ? fill_bytes / 16 : 0;
-  if (grid == 0 && fill_bytes && fill_async(fill_ones, ~0u, fill_bytes, s) != PTC_OK) return PTC_ERR_CUDA;
   if (grid > 0) {
     switch (G) {
       case 1: launch_hash<1>(grid, s, a, hc, full); break;

@@ -20,6 +20,8 @@
 //   k_verify_first first access of every id (atomicMin)
 //   k_verify       compares every access's B tokens and parent id with those
 //                  of the first access of its id.
+#include <algorithm>
+
 #include "ptc_internal.h"
 
 namespace ptc {
@@ -191,7 +193,8 @@ __global__ void __launch_bounds__(kInsThreads) k_ids_insert(const ulonglong2* __
 // occurrences, the bitmap's word prefixes giving ranks.  A first occurrence
 // finds its own bit set and is its own first occurrence, with no table read
 // (its bitmap word is shared with its neighbours, so the read is coalesced);
-// a later occurrence reads its slot's stored index.  kGaPer accesses per
+// a later occurrence reads its slot's stored index, or, after the
+// partitioned dedup (table null), finds the index in slot_of itself.  kGaPer accesses per
 // thread, kGaThreads apart, their dependent loads in flight together.
 constexpr int kGaThreads = 256;
 constexpr int kGaPer = 8;
@@ -219,8 +222,9 @@ __global__ void __launch_bounds__(kGaThreads) k_ids_gather(const uint32_t* __res
     if (f[k] == kMatchedSlot) continue;
     if ((own[k] >> (i & 31)) & 1u)
       f[k] = i;
-    else
+    else if (table)
       f[k] = in_bounds(st, f[k], m) ? __ldg(reinterpret_cast<const uint32_t*>(&table[f[k]]) + 3) : kNone;
+    // else (partitioned dedup): slot_of already holds the first occurrence
   }
   uint32_t wp[kGaPer], bw[kGaPer];
 #pragma unroll
@@ -528,6 +532,640 @@ __global__ void k_session_prior(const uint32_t* __restrict__ ses_sorted, const u
   }
 }
 
+// ---------------------------------------------------------------- partitioned dedup
+// With a table larger than L2 every settled key costs a random DRAM sector
+// (read, then the claimed sector written back), about 20 G keys/s.  The
+// partitioned method moves the keys to be settled (the unmatched accesses)
+// instead, in streaming passes, into 2^16 partitions by 16 bits of h0, and
+// settles every partition in a table of its own in shared memory:
+//   k_pd_flags     the bitmap of the accesses to settle: every access
+//                  without a hint; with one, the depths of each request from
+//                  its lam on (a warp per request)
+//   k_pd_count     level 1: per CTA of a persistent grid, the keys of its
+//                  range of accesses per bucket (h0 bits 53..60)
+//   k_pd_rows1     one CTA per bucket: the prefix of its counts over the
+//                  level-1 CTAs, and the bucket's total
+//   k_pd_scatter1  the same pass again: slot_of (matched or unmatched), and
+//                  a 16-byte record (96 key bits, access index) per
+//                  unmatched access, in bucket order
+//   k_pd_count2    level 2: per tile of kPdTile2 records of one bucket, the
+//                  records per partition (h0 bits 45..60); one atomic per
+//                  tile and partition claims the tile's place in it
+//   k_pd_rows2     one CTA per bucket: the bounds of its partitions
+//   k_pd_scatter2  every tile's records moved to their partitions
+//   k_pd_dedup     one partition at a time per CTA: every record settles its
+//                  key in a shared-memory table (key + smallest index); an
+//                  index that is never stored, or that a smaller one
+//                  replaces, is a repeat and goes to a list, whose entries
+//                  then take their key's smallest index into slot_of and
+//                  clear their bit.
+// The bitmap then holds exactly the first occurrences, and k_ids_gather reads
+// a repeat's first occurrence from slot_of itself.  A partition holding more
+// distinct keys than its shared table raises kErrTableFull, as an overfull
+// hash table does, and the call redoes the stage with the full table.
+// Both scatters sort a round's records by destination in shared memory
+// first, so that a warp's stores land in runs of consecutive records
+// rather than one 16-byte store per destination.
+constexpr int kPdThreads = 512;
+constexpr int kPdPer = 8;
+constexpr uint32_t kPdRound = kPdThreads * kPdPer;   // accesses per level-1 round (and staged records)
+constexpr uint32_t kPdBuckets = 256;                 // level 1: h0 bits 53..60
+constexpr uint32_t kPdParts = 65536;                 // level 2: h0 bits 45..60
+constexpr uint32_t kPdMaxG1 = 2048;                  // largest level-1 grid
+constexpr int kPd2Threads = 512;
+constexpr int kPd2Per = 8;
+constexpr uint32_t kPdTile2 = kPd2Threads * kPd2Per;  // 4096 records per level-2 tile
+constexpr int kPdDedupThreads = 512;
+constexpr int kPdDedupPer = 4;
+constexpr uint32_t kPdSlots = 6144;  // shared table: 96 KB
+constexpr uint32_t kPdList = 1536;   // repeats listed per partition: 12 KB
+constexpr size_t kPdDedupSmem = sizeof(ulonglong2) * kPdSlots + sizeof(uint2) * kPdList;
+
+constexpr size_t kPdStageSmem = sizeof(ulonglong2) * kPdRound;  // 64 KB
+static_assert(kPdTile2 == kPdRound, "both scatters stage one round of records");
+
+// The record of access i with key k: the same 96 key bits as a table slot.
+__device__ __forceinline__ ulonglong2 pd_record(ulonglong2 k, uint32_t i) {
+  return make_ulonglong2(k.x | ((k.y & 7ULL) << 61), (uint64_t)(uint32_t)(k.y >> 3) | ((uint64_t)i << 32));
+}
+__device__ __forceinline__ uint32_t pd_bucket(uint64_t w0) { return (uint32_t)(w0 >> 53) & (kPdBuckets - 1); }
+__device__ __forceinline__ uint32_t pd_part(uint64_t w0) { return (uint32_t)(w0 >> 45) & (kPdParts - 1); }
+
+// Exclusive prefix of v over threads 0..255 and the total, for a CTA of at
+// least 256 threads (the others pass 0); every thread calls it.
+__device__ __forceinline__ uint32_t scan256(uint32_t v, uint32_t* total) {
+  __shared__ uint32_t s_w[8];
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  uint32_t inc = v;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const uint32_t t = __shfl_up_sync(kFull, inc, d);
+    if (lane >= (uint32_t)d) inc += t;
+  }
+  if (w < 8 && lane == 31) s_w[w] = inc;
+  __syncthreads();
+  uint32_t before = 0, tot = 0;
+#pragma unroll
+  for (uint32_t k = 0; k < 8; ++k) {
+    const uint32_t x = s_w[k];
+    if (k < w) before += x;
+    tot += x;
+  }
+  __syncthreads();
+  *total = tot;
+  return before + inc - v;
+}
+
+// s_bst[0..256]: the bucket bounds in the level-1 records (prefix of tot1).
+__device__ __forceinline__ void pd_bucket_bounds(const uint32_t* tot1, uint32_t* s_bst) {
+  uint32_t total;
+  const uint32_t ex = scan256(threadIdx.x < kPdBuckets ? tot1[threadIdx.x] : 0u, &total);
+  if (threadIdx.x < kPdBuckets) s_bst[threadIdx.x] = ex;
+  if (threadIdx.x == 0) s_bst[kPdBuckets] = total;
+  __syncthreads();
+}
+
+// s_tp[0..256]: the first level-2 tile of every bucket, and the tile count.
+__device__ __forceinline__ void pd_tile_starts(const uint32_t* s_bst, uint32_t* s_tp) {
+  uint32_t total;
+  const uint32_t nt = threadIdx.x < kPdBuckets
+                          ? (uint32_t)(((uint64_t)s_bst[threadIdx.x + 1] - s_bst[threadIdx.x] + kPdTile2 - 1) / kPdTile2)
+                          : 0u;
+  const uint32_t ex = scan256(nt, &total);
+  if (threadIdx.x < kPdBuckets) s_tp[threadIdx.x] = ex;
+  if (threadIdx.x == 0) s_tp[kPdBuckets] = total;
+  __syncthreads();
+}
+
+struct PdArgs {
+  const ulonglong2* keys;
+  uint32_t n_ub;
+  const uint64_t* n_dev;
+  InsCarry kc;
+  PriorHint ph;        // ph.lam null: no hint
+  uint32_t per;        // accesses per level-1 CTA, a multiple of kPdRound
+  uint32_t* cnt1;      // [bucket * grid + cta]
+  uint32_t* off1;      // its prefix along each bucket's row
+  uint32_t* tot1;      // kPdBuckets totals
+  const uint32_t* ubits;  // the accesses to settle (k_pd_flags)
+  ulonglong2* rec1;    // n_ub records
+  DevStatus* st;
+};
+
+// The accesses to settle, as the bitmap `ubits`, and its copy `bits`, which
+// the dedup turns into the first occurrences (both zeroed before): without a
+// hint all of [0, n), one thread per word; with one, a warp per request sets
+// the bits of its depths from lam on (whole words by plain stores, the two
+// partial words at its ends by atomicOr, as neighbouring requests share
+// them).
+__global__ void __launch_bounds__(256) k_pd_flags(PriorHint ph, uint32_t n_ub, const uint64_t* n_dev,
+                                                  uint32_t* __restrict__ ubits, uint32_t* __restrict__ bits,
+                                                  uint32_t nwords) {
+  grid_dep_sync();
+  const uint32_t n = keys_used(n_ub, n_dev);
+  if (!ph.lam) {
+    const uint32_t w = blockIdx.x * 256 + threadIdx.x;
+    if (w < nwords) {
+      const uint64_t lo = 32ULL * w;
+      const uint32_t m = lo + 32 <= n ? ~0u : lo < n ? (1u << (n - lo)) - 1u : 0u;
+      ubits[w] = m;
+      bits[w] = m;
+    }
+    return;
+  }
+  const uint32_t r = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (r >= ph.n_req) return;
+  const uint64_t b = __ldg(&ph.blk_off[r]);
+  uint64_t e = __ldg(&ph.blk_off[r + 1]);
+  if (e > n) e = n;
+  if (e <= b) return;
+  const uint64_t l = __ldg(&ph.lam[r]);
+  const uint64_t u0 = l < e - b ? b + l : e;
+  if (u0 >= e) return;
+  const uint64_t w0 = u0 >> 5, w1 = (e - 1) >> 5;
+  for (uint64_t w = w0 + lane; w <= w1; w += 32) {
+    const uint32_t lo = w == w0 ? (uint32_t)(u0 & 31) : 0u;
+    const uint32_t hi = w == w1 ? (uint32_t)((e - 1) & 31) + 1 : 32u;
+    const uint32_t m = (hi == 32 ? ~0u : (1u << hi) - 1u) & ~((1u << lo) - 1u);
+    if (m == ~0u) {
+      ubits[w] = m;
+      bits[w] = m;
+    } else {
+      atomicOr(&ubits[w], m);
+      atomicOr(&bits[w], m);
+    }
+  }
+}
+
+// h0 of key i with the carry of its hash tile added (the first word of
+// carried_key, for a key whose second word is a field element).
+__device__ __forceinline__ uint64_t carried_h0(const ulonglong2* __restrict__ keys, uint32_t i, const InsCarry& kc) {
+  uint64_t x = __ldcs(reinterpret_cast<const unsigned long long*>(&keys[i]));
+  if (kc.carry) {
+    const uint32_t t = i >> kc.tile_shift;
+    if ((i & ((1u << kc.tile_shift) - 1u)) < __ldg(&kc.lead[t]) && x < kP61)
+      x = p61_add(x, __ldg(reinterpret_cast<const unsigned long long*>(&kc.carry[t])));
+  }
+  return x;
+}
+
+// Level 1, counting: the keys of CTA g's accesses [g per, (g + 1) per) per
+// bucket.  Only h0 is read (the bucket is in it).  The scatter below skips a
+// key whose h1 is not a field element as well, and raises kErrInvalid, so
+// the counts can only differ from it on input the call rejects.
+__global__ void __launch_bounds__(kPdThreads, 4) k_pd_count(PdArgs a) {
+  grid_dep_sync();
+  report_keys_used(a.n_ub, a.n_dev, a.st);
+  __shared__ uint32_t h[kPdBuckets];
+  for (uint32_t x = threadIdx.x; x < kPdBuckets; x += kPdThreads) h[x] = 0;
+  const uint32_t n = keys_used(a.n_ub, a.n_dev);
+  const uint64_t lo = (uint64_t)blockIdx.x * a.per;
+  const uint64_t hi = lo + a.per < n ? lo + a.per : n;
+  __syncthreads();
+  for (uint64_t base = lo; base < hi; base += kPdRound) {
+    bool u[kPdPer];
+    uint64_t x[kPdPer];
+#pragma unroll
+    for (int j = 0; j < kPdPer; ++j) {
+      const uint64_t i = base + j * kPdThreads + threadIdx.x;
+      u[j] = i < hi && ((__ldg(&a.ubits[i >> 5]) >> (i & 31)) & 1u);
+    }
+#pragma unroll
+    for (int j = 0; j < kPdPer; ++j)
+      x[j] = u[j] ? carried_h0(a.keys, (uint32_t)(base + j * kPdThreads + threadIdx.x), a.kc) : ~0ULL;
+#pragma unroll
+    for (int j = 0; j < kPdPer; ++j)
+      if (u[j] && x[j] < kP61) atomicAdd(&h[pd_bucket(x[j])], 1u);
+  }
+  __syncthreads();
+  for (uint32_t x = threadIdx.x; x < kPdBuckets; x += kPdThreads) a.cnt1[x * gridDim.x + blockIdx.x] = h[x];
+}
+
+// Level 1, scattering: the same accesses and keys as k_pd_count.  Each round
+// ranks its records per bucket, sorts them into shared memory by bucket, and
+// writes each bucket's run at the CTA's running place in the bucket.
+__global__ void __launch_bounds__(kPdThreads, 2) k_pd_scatter1(PdArgs a) {
+  grid_dep_sync();
+  extern __shared__ ulonglong2 stage[];  // kPdRound records
+  __shared__ uint32_t h[kPdBuckets];     // the next place in each bucket
+  __shared__ uint32_t c[kPdBuckets], so[kPdBuckets];  // the round's records per bucket, their offsets
+  __shared__ uint32_t s_bst[kPdBuckets + 1];
+  pd_bucket_bounds(a.tot1, s_bst);
+  for (uint32_t x = threadIdx.x; x < kPdBuckets; x += kPdThreads) {
+    h[x] = s_bst[x] + a.off1[x * gridDim.x + blockIdx.x];
+    c[x] = 0;
+  }
+  const uint32_t n = keys_used(a.n_ub, a.n_dev);
+  const uint64_t lo = (uint64_t)blockIdx.x * a.per;
+  const uint64_t hi = lo + a.per < n ? lo + a.per : n;
+  __syncthreads();
+  for (uint64_t base = lo; base < hi; base += kPdRound) {
+    bool u[kPdPer];
+    ulonglong2 k[kPdPer];
+    uint32_t rk[kPdPer];
+#pragma unroll
+    for (int j = 0; j < kPdPer; ++j) {
+      const uint64_t i = base + j * kPdThreads + threadIdx.x;
+      u[j] = i < hi && ((__ldg(&a.ubits[i >> 5]) >> (i & 31)) & 1u);
+    }
+#pragma unroll
+    for (int j = 0; j < kPdPer; ++j) {
+      const uint32_t i = (uint32_t)(base + j * kPdThreads + threadIdx.x);
+      k[j] = u[j] ? carried_key(a.keys, i, n, a.kc) : make_ulonglong2(0, 0);
+      if (u[j] && (k[j].x >= kP61 || k[j].y >= kP61)) {  // not a field element: never settled
+        raise_err(a.st, kErrInvalid);
+        u[j] = false;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < kPdPer; ++j) rk[j] = u[j] ? atomicAdd(&c[pd_bucket(k[j].x)], 1u) : 0u;
+    __syncthreads();
+    uint32_t nrec;
+    const uint32_t ex = scan256(threadIdx.x < kPdBuckets ? c[threadIdx.x] : 0u, &nrec);
+    if (threadIdx.x < kPdBuckets) so[threadIdx.x] = ex;
+    __syncthreads();
+#pragma unroll
+    for (int j = 0; j < kPdPer; ++j)
+      if (u[j])
+        stage[so[pd_bucket(k[j].x)] + rk[j]] = pd_record(k[j], (uint32_t)(base + j * kPdThreads + threadIdx.x));
+    __syncthreads();
+    for (uint32_t x = threadIdx.x; x < nrec; x += kPdThreads) {
+      const ulonglong2 r = stage[x];
+      const uint32_t d = pd_bucket(r.x);
+      const uint32_t at = h[d] + (x - so[d]);
+      if (at < a.n_ub)
+        __stcg(&a.rec1[at], r);
+      else
+        raise_err(a.st, kErrInvalid);
+    }
+    __syncthreads();
+    for (uint32_t x = threadIdx.x; x < kPdBuckets; x += kPdThreads) {
+      h[x] += c[x];
+      c[x] = 0;
+    }
+    __syncthreads();
+  }
+}
+
+// One CTA per bucket: the exclusive prefix of the bucket's counts along the
+// level-1 CTAs (its place in the bucket for each), and the bucket's total.
+__global__ void __launch_bounds__(256) k_pd_rows1(const uint32_t* __restrict__ cnt1, uint32_t g1,
+                                                  uint32_t* __restrict__ off1, uint32_t* __restrict__ tot1) {
+  grid_dep_sync();
+  const uint32_t* row = cnt1 + (size_t)blockIdx.x * g1;
+  uint32_t* out = off1 + (size_t)blockIdx.x * g1;
+  const uint32_t per = (g1 + 255) / 256;
+  const uint32_t a0 = threadIdx.x * per < g1 ? threadIdx.x * per : g1;
+  const uint32_t a1 = a0 + per < g1 ? a0 + per : g1;
+  uint32_t sum = 0;
+  for (uint32_t e = a0; e < a1; ++e) sum += row[e];
+  uint32_t total;
+  uint32_t run = scan256(sum, &total);
+  for (uint32_t e = a0; e < a1; ++e) {
+    const uint32_t v = row[e];
+    out[e] = run;
+    run += v;
+  }
+  if (threadIdx.x == 0) tot1[blockIdx.x] = total;
+}
+
+struct PdLevel2 {
+  const ulonglong2* rec1;
+  const uint32_t* tot1;
+  uint32_t* tot2;     // kPdParts totals (zeroed by the call)
+  uint32_t* rel2;     // [tile * 256 + partition of the bucket]: the tile's place in the partition
+  const uint32_t* base2;
+  ulonglong2* rec2;
+  uint32_t cap;       // records rec1 and rec2 hold
+  uint32_t max_tiles; // entries of rel2 / 256
+  DevStatus* st;
+};
+
+// Level 2 over tiles of kPdTile2 records of one bucket (a persistent grid
+// walks the tiles).  The count pass claims the tile's range of every
+// partition (the atomic's old value); the scatter pass writes the tile's
+// records there, ranked per partition inside the tile, so they fill the
+// claimed ranges exactly (both passes read the same records).
+template <bool SCATTER>
+__global__ void __launch_bounds__(kPd2Threads, 2) k_pd_level2(PdLevel2 a) {
+  grid_dep_sync();
+  extern __shared__ ulonglong2 stage[];  // scatter: kPdTile2 records
+  __shared__ uint32_t h[256], s_at[256], so[256];
+  __shared__ uint32_t s_bst[kPdBuckets + 1], s_tp[kPdBuckets + 1];
+  pd_bucket_bounds(a.tot1, s_bst);
+  pd_tile_starts(s_bst, s_tp);
+  const uint32_t T = s_tp[kPdBuckets];
+  if (T > a.max_tiles) {
+    if (threadIdx.x == 0 && blockIdx.x == 0) raise_err(a.st, kErrInvalid);
+    return;
+  }
+  for (uint32_t tile = blockIdx.x; tile < T; tile += gridDim.x) {
+    uint32_t lo = 0, hi = kPdBuckets - 1;  // the bucket: the last d with s_tp[d] <= tile
+    while (lo < hi) {
+      const uint32_t mid = (lo + hi + 1) >> 1;
+      if (s_tp[mid] <= tile)
+        lo = mid;
+      else
+        hi = mid - 1;
+    }
+    const uint64_t start = s_bst[lo] + (uint64_t)(tile - s_tp[lo]) * kPdTile2;
+    const uint64_t end = start + kPdTile2 < s_bst[lo + 1] ? start + kPdTile2 : s_bst[lo + 1];
+    const uint32_t pbase = lo << 8;
+    for (uint32_t x = threadIdx.x; x < 256; x += kPd2Threads) {
+      h[x] = 0;
+      if (SCATTER) s_at[x] = a.base2[pbase + x] + a.rel2[(size_t)tile * 256 + x];
+    }
+    __syncthreads();
+    ulonglong2 v[kPd2Per];
+    uint32_t rk[kPd2Per];
+#pragma unroll
+    for (int q = 0; q < kPd2Per; ++q) {
+      const uint64_t x = start + q * kPd2Threads + threadIdx.x;
+      v[q] = x < end && x < a.cap ? __ldcs(&a.rec1[x]) : make_ulonglong2(~0ULL, ~0ULL);
+    }
+#pragma unroll
+    for (int q = 0; q < kPd2Per; ++q)
+      rk[q] = v[q].x != ~0ULL ? atomicAdd(&h[pd_part(v[q].x) & 255], 1u) : 0u;
+    __syncthreads();
+    if (!SCATTER) {
+      for (uint32_t x = threadIdx.x; x < 256; x += kPd2Threads)
+        a.rel2[(size_t)tile * 256 + x] = h[x] ? atomicAdd(&a.tot2[pbase + x], h[x]) : 0u;
+    } else {  // sort the tile by partition in shared memory, then write the runs
+      uint32_t nrec;
+      const uint32_t ex = scan256(threadIdx.x < 256 ? h[threadIdx.x] : 0u, &nrec);
+      if (threadIdx.x < 256) so[threadIdx.x] = ex;
+      __syncthreads();
+#pragma unroll
+      for (int q = 0; q < kPd2Per; ++q)
+        if (v[q].x != ~0ULL) stage[so[pd_part(v[q].x) & 255] + rk[q]] = v[q];
+      __syncthreads();
+      for (uint32_t x = threadIdx.x; x < nrec; x += kPd2Threads) {
+        const ulonglong2 r = stage[x];
+        const uint32_t p2 = pd_part(r.x) & 255;
+        const uint32_t pos = s_at[p2] + (x - so[p2]);
+        if (pd_bucket(r.x) == lo && pos < a.cap)
+          __stcg(&a.rec2[pos], r);
+        else
+          raise_err(a.st, kErrInvalid);
+      }
+    }
+    __syncthreads();
+  }
+}
+
+// One CTA per bucket: the bounds of its 256 partitions (the bucket's bound
+// plus the prefix of their totals); base2[kPdParts] = the record count.
+__global__ void __launch_bounds__(256) k_pd_rows2(const uint32_t* __restrict__ tot1, const uint32_t* __restrict__ tot2,
+                                                  uint32_t* __restrict__ base2, DevStatus* st) {
+  grid_dep_sync();
+  __shared__ uint32_t s_bst[kPdBuckets + 1];
+  pd_bucket_bounds(tot1, s_bst);
+  const uint32_t d = blockIdx.x;
+  uint32_t total;
+  const uint32_t ex = scan256(tot2[d * 256 + threadIdx.x], &total);
+  base2[d * 256 + threadIdx.x] = s_bst[d] + ex;
+  if (threadIdx.x == 0 && total != s_bst[d + 1] - s_bst[d]) raise_err(st, kErrInvalid);
+  if (d == kPdBuckets - 1 && threadIdx.x == 0) base2[kPdParts] = s_bst[kPdBuckets];
+}
+
+__device__ __forceinline__ ulonglong2 ld_shared_v2(const ulonglong2* p) {
+  ulonglong2 v;
+  asm volatile("ld.volatile.shared.v2.u64 {%0, %1}, [%2];"
+               : "=l"(v.x), "=l"(v.y)
+               : "r"((uint32_t)__cvta_generic_to_shared(p))
+               : "memory");
+  return v;
+}
+
+__device__ __forceinline__ ulonglong2 cas128_shared(ulonglong2* addr, ulonglong2 cmp, ulonglong2 val) {
+  ulonglong2 old;
+  asm volatile(
+      "{\n\t.reg .b128 c, v, d;\n\t"
+      "mov.b128 c, {%2, %3};\n\t"
+      "mov.b128 v, {%4, %5};\n\t"
+      "atom.shared.cas.b128 d, [%6], c, v;\n\t"
+      "mov.b128 {%0, %1}, d;\n\t}"
+      : "=l"(old.x), "=l"(old.y)
+      : "l"(cmp.x), "l"(cmp.y), "l"(val.x), "l"(val.y), "r"((uint32_t)__cvta_generic_to_shared(addr))
+      : "memory");
+  return old;
+}
+
+// Home slot of a record in a partition's table of ts slots: h0's low 32 bits
+// (the partition fixes bits 45..60 only).
+__device__ __forceinline__ uint32_t pd_home(uint64_t w0, uint32_t ts) { return __umulhi((uint32_t)w0, ts); }
+
+// Settle record r in the shared table of ts slots: claim an empty slot with
+// one 128-bit CAS, or meet its key's slot, where the smaller of the two
+// indices stays.  The index that does not stay (r's own, or the one r's
+// atomicMin replaced) is a repeat: it comes back in *rep, with the slot in
+// *rs (*rep = kNone otherwise).  False when the table has no room (every
+// slot probed).
+__device__ __forceinline__ bool pd_insert(ulonglong2* tab, uint32_t ts, ulonglong2 r, uint32_t* rep, uint32_t* rs) {
+  const ulonglong2 empty = make_ulonglong2(~0ULL, ~0ULL);
+  const uint32_t idx = (uint32_t)(r.y >> 32);
+  *rep = kNone;
+  uint32_t s = pd_home(r.x, ts);
+  for (uint32_t probe = 0; probe < ts; ++probe) {
+    ulonglong2 cur = ld_shared_v2(&tab[s]);
+    if (cur.x == ~0ULL || cur.y == ~0ULL) {  // empty (or read while being claimed): the CAS settles it
+      cur = cas128_shared(&tab[s], empty, r);
+      if (cur.x == ~0ULL && cur.y == ~0ULL) return true;
+    }
+    if (cur.x == r.x && (uint32_t)cur.y == (uint32_t)r.y) {
+      uint32_t out = idx;
+      if ((uint32_t)(cur.y >> 32) > idx) {
+        const uint32_t old = atomicMin(reinterpret_cast<uint32_t*>(&tab[s]) + 3, idx);
+        out = old > idx ? old : idx;
+      }
+      *rep = out;
+      *rs = s;
+      return true;
+    }
+    s = s + 1 == ts ? 0 : s + 1;
+  }
+  return false;
+}
+
+// Appends (rep, rs) to the shared repeat list for the lanes that have one
+// (rep != kNone), one atomic per warp; past kPdList entries only the count
+// grows.  Every lane of the warp calls it.
+__device__ __forceinline__ void pd_list_push(uint32_t rep, uint32_t rs, uint2* list, uint32_t* nlist) {
+  const uint32_t m = __ballot_sync(kFull, rep != kNone);
+  if (!m) return;
+  const uint32_t lane = threadIdx.x & 31;
+  uint32_t base = 0;
+  if (lane == __ffs(m) - 1) base = atomicAdd(nlist, (uint32_t)__popc(m));
+  base = __shfl_sync(kFull, base, __ffs(m) - 1);
+  if (rep != kNone) {
+    const uint32_t k = base + __popc(m & ((1u << lane) - 1u));
+    if (k < kPdList) list[k] = make_uint2(rep, rs);
+  }
+}
+
+// The smallest index stored for r's key, or kNone if the key is not there.
+__device__ __forceinline__ uint32_t pd_find(const ulonglong2* tab, uint32_t ts, ulonglong2 r) {
+  uint32_t s = pd_home(r.x, ts);
+  for (uint32_t probe = 0; probe < ts; ++probe) {
+    const ulonglong2 cur = tab[s];
+    if (cur.x == r.x && (uint32_t)cur.y == (uint32_t)r.y) return (uint32_t)(cur.y >> 32);
+    if (cur.x == ~0ULL) return kNone;
+    s = s + 1 == ts ? 0 : s + 1;
+  }
+  return kNone;
+}
+
+__device__ __forceinline__ void pd_repeat(uint32_t* slot_of, uint32_t* bits, uint32_t i, uint32_t m) {
+  slot_of[i] = m;
+  atomicAnd(&bits[i >> 5], ~(1u << (i & 31)));
+}
+
+struct PdDedup {
+  const ulonglong2* rec2;
+  const uint32_t* base2;  // kPdParts + 1 partition bounds
+  uint32_t cap;
+  uint32_t* slot_of;
+  uint32_t* bits;
+  uint32_t n_ub;
+  DevStatus* st;
+};
+
+// A partition's table takes twice its records in slots (at most kPdSlots),
+// so small partitions clear little shared memory.  The loads of the next
+// chunk of records (or of the next partition's first chunk) are issued
+// before the current chunk is inserted, so they overlap its inserts.
+__global__ void __launch_bounds__(kPdDedupThreads, 2) k_pd_dedup(PdDedup a) {
+  grid_dep_sync();
+  extern __shared__ ulonglong2 tab[];  // kPdSlots, then the repeat list
+  uint2* list = reinterpret_cast<uint2*>(tab + kPdSlots);
+  __shared__ uint32_t s_nlist;
+  constexpr uint32_t kChunk = kPdDedupThreads * kPdDedupPer;
+  const ulonglong2 empty = make_ulonglong2(~0ULL, ~0ULL);
+  auto load = [&](ulonglong2(&dst)[kPdDedupPer], uint32_t c, uint32_t end) {
+#pragma unroll
+    for (int q = 0; q < kPdDedupPer; ++q) {
+      const uint32_t x = c + q * kPdDedupThreads + threadIdx.x;
+      dst[q] = x < end && x < a.cap ? __ldcs(&a.rec2[x]) : empty;
+    }
+  };
+  uint32_t p = blockIdx.x, b = 0, e = 0;
+  if (p < kPdParts) {
+    b = a.base2[p];
+    e = a.base2[p + 1];
+  }
+  ulonglong2 v[kPdDedupPer];
+  load(v, b, e);
+  while (p < kPdParts) {
+    const uint32_t pn = p + gridDim.x;
+    uint32_t bn = 0, en = 0;
+    if (pn < kPdParts) {
+      bn = a.base2[pn];
+      en = a.base2[pn + 1];
+    }
+    if (b >= e || e > a.cap) {  // nothing to settle (or bounds past the records: malformed)
+      if (b < e && threadIdx.x == 0) raise_err(a.st, kErrInvalid);
+      load(v, bn, en);
+    } else {
+      const uint32_t ts = e - b < kPdSlots / 2 ? ((2 * (e - b) + 31) & ~31u) : kPdSlots;
+      for (uint32_t x = threadIdx.x; x < ts; x += kPdDedupThreads) tab[x] = empty;
+      if (threadIdx.x == 0) s_nlist = 0;
+      __syncthreads();
+      bool full = false;
+      for (uint32_t c = b;; c += kChunk) {
+        const bool more = c + kChunk < e;
+        ulonglong2 w[kPdDedupPer];
+        if (more)
+          load(w, c + kChunk, e);
+        else
+          load(w, bn, en);
+#pragma unroll
+        for (int q = 0; q < kPdDedupPer; ++q) {
+          uint32_t rep = kNone, rs = 0;
+          if (v[q].x != ~0ULL && !pd_insert(tab, ts, v[q], &rep, &rs)) full = true;
+          pd_list_push(rep, rs, list, &s_nlist);
+        }
+#pragma unroll
+        for (int q = 0; q < kPdDedupPer; ++q) v[q] = w[q];
+        if (!more) break;
+      }
+      if (full) raise_err(a.st, kErrTableFull);
+      __syncthreads();
+      const uint32_t nl = s_nlist;
+      if (nl <= kPdList) {
+        for (uint32_t x = threadIdx.x; x < nl; x += kPdDedupThreads) {
+          const uint2 rp = list[x];
+          const uint32_t m = reinterpret_cast<const uint32_t*>(&tab[rp.y])[3];
+          if (m < rp.x && rp.x < a.n_ub) pd_repeat(a.slot_of, a.bits, rp.x, m);
+        }
+      } else {  // more repeats than the list holds: look every record up again
+        for (uint32_t c = b; c < e; c += kChunk) {
+          ulonglong2 r[kPdDedupPer];
+#pragma unroll
+          for (int q = 0; q < kPdDedupPer; ++q) {
+            const uint32_t x = c + q * kPdDedupThreads + threadIdx.x;
+            r[q] = x < e ? __ldcg(&a.rec2[x]) : empty;
+          }
+#pragma unroll
+          for (int q = 0; q < kPdDedupPer; ++q) {
+            if (r[q].x == ~0ULL) continue;
+            const uint32_t i = (uint32_t)(r[q].y >> 32), m = pd_find(tab, ts, r[q]);
+            if (m < i && i < a.n_ub) pd_repeat(a.slot_of, a.bits, i, m);
+          }
+        }
+      }
+      __syncthreads();
+    }
+    p = pn;
+    b = bn;
+    e = en;
+  }
+}
+
+// ids after the partitioned dedup: ubits marks the settled accesses, bits
+// their first occurrences; a settled access that is not a first occurrence
+// (a repeat) finds its first occurrence in slot_of.  Matched accesses are
+// left to k_ids_follow.
+__global__ void __launch_bounds__(kGaThreads) k_ids_gather_pd(const uint32_t* __restrict__ slot_of,
+                                                             const uint32_t* __restrict__ ubits,
+                                                             const uint32_t* __restrict__ bits,
+                                                             const uint32_t* __restrict__ wpre, uint32_t n_ub,
+                                                             const uint64_t* n_dev, uint32_t* __restrict__ ids) {
+  grid_dep_sync();
+  const uint32_t n = keys_used(n_ub, n_dev);
+  const uint32_t i0 = blockIdx.x * (kGaThreads * kGaPer) + threadIdx.x;
+  uint32_t f[kGaPer], own[kGaPer], uw[kGaPer];
+  // the three words of every access are read together (slot_of whether or
+  // not the access turns out to be a repeat: one coalesced stream)
+#pragma unroll
+  for (int k = 0; k < kGaPer; ++k) {
+    const uint32_t i = i0 + k * kGaThreads;
+    uw[k] = i < n ? __ldg(&ubits[i >> 5]) : 0u;
+    own[k] = i < n ? bits[i >> 5] : 0u;
+    f[k] = i < n ? __ldcs(&slot_of[i]) : 0u;
+  }
+#pragma unroll
+  for (int k = 0; k < kGaPer; ++k) {
+    const uint32_t i = i0 + k * kGaThreads;
+    if (!((uw[k] >> (i & 31)) & 1u))
+      f[k] = kMatchedSlot;
+    else if ((own[k] >> (i & 31)) & 1u)
+      f[k] = i;
+  }
+  uint32_t wp[kGaPer], bw[kGaPer];
+#pragma unroll
+  for (int k = 0; k < kGaPer; ++k) {
+    const uint32_t i = i0 + k * kGaThreads;
+    const bool ok = f[k] < n;
+    wp[k] = ok ? wpre[f[k] >> 5] : 0u;
+    bw[k] = f[k] == i ? own[k] : ok ? bits[f[k] >> 5] : 0u;
+  }
+#pragma unroll
+  for (int k = 0; k < kGaPer; ++k) {
+    const uint32_t i = i0 + k * kGaThreads;
+    if (i < n && f[k] != kMatchedSlot) ids[i] = f[k] < n ? wp[k] + __popc(bw[k] & ((1u << (f[k] & 31)) - 1u)) : kNone;
+  }
+}
+
 // Slots for n keys at most: the full table holds 1.5 n.  The first attempt
 // holds n / 3 while that is at most 2^22 slots (64 MB, half of L2): traces
 // that repeat most blocks fill it well below half, and it stays in L2.  A
@@ -554,17 +1192,23 @@ struct IdsLayout {
   DevStatus* st;
   uint32_t* done;
   ulonglong2* table;
-  uint32_t* slot_of;  // per access: its slot, or kMatched
+  uint32_t* slot_of;  // per access: its slot, or kMatched (partitioned: a repeat's first occurrence)
   uint32_t *bits, *wpre, *tcnt, *tpre;  // first-occurrence bitmap and its ranks
   uint32_t* lam;               // prior hint: first unmatched depth of each request
   uint32_t* tile_req;          // prior hint: request of every 2048th access
+  // partitioned dedup (null without it): level-1 counts and their prefix,
+  // bucket bounds and level-2 tiles, partition totals, bounds and cursors,
+  // and the records of both levels (in the table's region)
+  uint32_t *pd_ubits, *pd_cnt1, *pd_off1, *pd_tot1, *pd_tot2, *pd_rel2, *pd_base2;
+  ulonglong2 *pd_rec1, *pd_rec2;
+  uint32_t pd_max_tiles;
   uint32_t nwords;
   size_t zero_bytes;
   size_t total;
   uint32_t log2m;
 };
 
-IdsLayout ids_layout(void* ws, uint64_t n, uint32_t n_req_hint = 0) {
+IdsLayout ids_layout(void* ws, uint64_t n, uint32_t n_req_hint, bool pd) {
   IdsLayout L;
   Carver cv(ws);
   L.log2m = full_table_log2(n);
@@ -573,6 +1217,7 @@ IdsLayout ids_layout(void* ws, uint64_t n, uint32_t n_req_hint = 0) {
   L.nwords = ceil_div_u32(nn, 32);
   L.st = cv.take<DevStatus>(1);
   L.done = cv.take<uint32_t>(64);
+  L.pd_tot2 = pd ? cv.take<uint32_t>(kPdParts) : nullptr;  // zeroed with the status block
   L.zero_bytes = cv.off;
   L.slot_of = cv.take<uint32_t>(nn);
   L.bits = cv.take<uint32_t>(L.nwords + 1);
@@ -581,12 +1226,27 @@ IdsLayout ids_layout(void* ws, uint64_t n, uint32_t n_req_hint = 0) {
   L.tpre = cv.take<uint32_t>(rank_tiles(L.nwords) + 1);
   L.lam = n_req_hint ? cv.take<uint32_t>(n_req_hint) : nullptr;
   L.tile_req = n_req_hint ? cv.take<uint32_t>((nn >> kReqTileLog2) + 2) : nullptr;
+  L.pd_max_tiles = ceil_div_u32(nn, kPdTile2) + kPdBuckets;
+  L.pd_ubits = pd ? cv.take<uint32_t>(L.nwords + 1) : nullptr;
+  L.pd_cnt1 = pd ? cv.take<uint32_t>(kPdBuckets * kPdMaxG1) : nullptr;
+  L.pd_off1 = pd ? cv.take<uint32_t>(kPdBuckets * kPdMaxG1) : nullptr;
+  L.pd_tot1 = pd ? cv.take<uint32_t>(kPdBuckets) : nullptr;
+  L.pd_rel2 = pd ? cv.take<uint32_t>((size_t)L.pd_max_tiles * 256) : nullptr;
+  L.pd_base2 = pd ? cv.take<uint32_t>(kPdParts + 1) : nullptr;
   // the table last: it starts past every other array of the stage (and past
   // stage a1's workspace, which the pipeline checks before it has stage a1
-  // fill the table)
-  L.table = cv.take<ulonglong2>(m);
+  // fill the table); the partitioned dedup keeps its records there
+  L.table = cv.take<ulonglong2>(pd && 2 * nn > m ? 2 * nn : m);
+  L.pd_rec1 = pd ? L.table : nullptr;
+  L.pd_rec2 = pd && L.table ? L.table + nn : nullptr;
   L.total = cv.bytes();
   return L;
+}
+
+// Which dedup a first attempt takes: the partitioned one when asked, or (the
+// default) when the table would not fit in L2.
+bool ids_partitioned(uint64_t n, int method) {
+  return method == PTC_IDS_PARTITIONED || (method == PTC_IDS_AUTO && ids_table_in_dram(n));
 }
 
 // ---------------------------------------------------------------- verify
@@ -652,15 +1312,17 @@ __global__ void k_verify(const uint32_t* __restrict__ tokens, uint64_t n_tok, co
 
 using namespace ptc;
 
-extern "C" size_t ptc_assign_ids_workspace_bytes(uint64_t n) { return ids_layout(nullptr, n).total; }
+extern "C" size_t ptc_assign_ids_workspace_bytes(uint64_t n) {
+  return ids_layout(nullptr, n, 0, ids_partitioned(n, PTC_IDS_AUTO)).total;
+}
 
 ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev, uint32_t* ids_out,
                         uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
                         cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc,
-                        uint64_t* nd_slot, uint32_t* err_slot, bool full_table, const IdsHint* hint,
-                        bool table_prefilled) {
+                        uint64_t* nd_slot, uint32_t* err_slot, bool full_table, const IdsHint* hint, int method) {
   if (hint && (hint->n_req == 0 || !hint->blk_off || !hint->prior)) return PTC_ERR_INVALID_ARG;
   if (kc && (kc->tile_blocks == 0 || (kc->tile_blocks & (kc->tile_blocks - 1)) != 0)) return PTC_ERR_INVALID_ARG;
+  if (method != PTC_IDS_AUTO && method != PTC_IDS_TABLE && method != PTC_IDS_PARTITIONED) return PTC_ERR_INVALID_ARG;
   const InsCarry ic = kc ? InsCarry{kc->carry, kc->lead, (uint32_t)__builtin_ctz(kc->tile_blocks)}
                         : InsCarry{nullptr, nullptr, 0};
   if (n_distinct_host_out == nullptr) return PTC_ERR_INVALID_ARG;
@@ -669,40 +1331,40 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
   if (n >= (uint64_t)kNone) return PTC_ERR_OVERFLOW;
   if (n > 0 && (keys == nullptr || ids_out == nullptr)) return PTC_ERR_INVALID_ARG;
   const uint32_t hreq = hint ? hint->n_req : 0;
-  if (!ws_ok(ws, ws_bytes, ids_layout(nullptr, n, hreq).total)) return PTC_ERR_WORKSPACE;
-  const IdsLayout L = ids_layout(ws, n, hreq);
+  const bool pd_layout = ids_partitioned(n, method);
+  if (!ws_ok(ws, ws_bytes, ids_layout(nullptr, n, hreq, pd_layout).total)) return PTC_ERR_WORKSPACE;
+  const IdsLayout L = ids_layout(ws, n, hreq, pd_layout);
   const PriorHint ph = hint ? PriorHint{hint->blk_off, hint->prior, hint->order, hint->pos, hint->n_req, L.lam, L.tile_req}
                             : PriorHint{nullptr, nullptr, nullptr, nullptr, 0, nullptr, nullptr};
-  // the status block, the table (all ones: empty) and the first-occurrence
-  // bitmap are cleared by one launch
-  // the table of the first attempt may come already filled (ids_table_region)
-  bool prefilled = table_prefilled;
-  auto start = [&](uint32_t log2m) -> bool {
-    const bool fill_table = n > 0 && !prefilled;
-    prefilled = false;
-    const FillRange zf[3] = {{ws, L.zero_bytes, 0u},
+  const bool pd = pd_layout && !full_table;  // the first attempt deduplicates by partitions
+  // the status block, the table (all ones: empty; none for the partitioned
+  // dedup) and the bitmaps are cleared by one launch
+  auto start = [&](uint32_t log2m, bool table) -> bool {
+    const bool fill_table = n > 0 && table;
+    const FillRange zf[4] = {{ws, L.zero_bytes, 0u},
                             {L.table, fill_table ? sizeof(ulonglong2) << log2m : 0, ~0u},
-                            {L.bits, n > 0 ? sizeof(uint32_t) * L.nwords : 0, 0u}};
-    return fill_many_async(zf, 3, s) == PTC_OK && carry_errors(carry_err, n_carry, L.st, s) == PTC_OK;
+                            {L.bits, n > 0 ? sizeof(uint32_t) * L.nwords : 0, 0u},
+                            {L.pd_ubits, L.pd_ubits && n > 0 && !table ? sizeof(uint32_t) * L.nwords : 0, 0u}};
+    return fill_many_async(zf, 4, s) == PTC_OK && carry_errors(carry_err, n_carry, L.st, s) == PTC_OK;
   };
-  auto run = [&](uint32_t log2m, uint64_t probe_cap) -> bool {
-    const ulonglong2* k = reinterpret_cast<const ulonglong2*>(keys);
-    const uint32_t n32 = (uint32_t)n;
-    if (hint) {
-      PTC_KERNEL("k_tile_req", s, k_tile_req, ceil_div_u32((n >> kReqTileLog2) + 2, 256), 256, 0, ph, n32, n_dev);
-      PTC_KERNEL("k_ids_lam", s, k_ids_lam, ceil_div_u32(hint->n_req, kLamThreads), kLamThreads, 0, k, n32, n_dev, ic,
-                 ph, L.st);
-      PTC_KERNEL("k_ids_insert_prior", s, k_ids_insert_prior<kPriorK>, ceil_div_u32(n, kInsThreads * kPriorK),
-                 kInsThreads, 0, k, n32, n_dev, L.table, log2m, probe_cap, L.slot_of, L.bits, L.st, ic, ph);
-    } else {
-      PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads * kInsK), kInsThreads, 0, k, n32, n_dev,
-                 L.table, log2m, probe_cap, L.slot_of, L.bits, L.st, ic);
-    }
-    const uint64_t m = 1ULL << log2m;
+  const ulonglong2* k = reinterpret_cast<const ulonglong2*>(keys);
+  const uint32_t n32 = (uint32_t)n;
+  auto hint_prep = [&]() {
+    PTC_KERNEL("k_tile_req", s, k_tile_req, ceil_div_u32((n >> kReqTileLog2) + 2, 256), 256, 0, ph, n32, n_dev);
+    PTC_KERNEL("k_ids_lam", s, k_ids_lam, ceil_div_u32(hint->n_req, kLamThreads), kLamThreads, 0, k, n32, n_dev, ic,
+               ph, L.st);
+  };
+  // ranks of the first occurrences, the ids of the settled accesses, then
+  // those of the matched ones
+  auto finish = [&](const ulonglong2* table, uint64_t m) -> bool {
     if (bitmap_ranks(L.bits, L.nwords, L.wpre, L.tcnt, L.tpre, &L.done[0], &L.st->value[0], s) != PTC_OK)
       return false;
-    PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of,
-                 L.table, m, L.bits, L.wpre, n32, n_dev, ids_out, L.st);
+    if (table)
+      PTC_KERNEL("k_ids_gather", s, k_ids_gather, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of,
+                 table, m, L.bits, L.wpre, n32, n_dev, ids_out, L.st);
+    else
+      PTC_KERNEL("k_ids_gather", s, k_ids_gather_pd, ceil_div_u32(n, kGaThreads * kGaPer), kGaThreads, 0, L.slot_of,
+                 L.pd_ubits, L.bits, L.wpre, n32, n_dev, ids_out);
     if (hint)
       if (ph.order)
         PTC_KERNEL("k_ids_follow", s, k_ids_follow_win, ceil_div_u32(hint->n_req, kFoThreads / 32), kFoThreads, 0,
@@ -712,27 +1374,66 @@ ptc_status ptc::ids_impl(const ptc_u128* keys, uint64_t n, const uint64_t* n_dev
                    ids_out, L.st);
     return true;
   };
+  auto run = [&](uint32_t log2m, uint64_t probe_cap) -> bool {
+    if (hint) {
+      hint_prep();
+      PTC_KERNEL("k_ids_insert_prior", s, k_ids_insert_prior<kPriorK>, ceil_div_u32(n, kInsThreads * kPriorK),
+                 kInsThreads, 0, k, n32, n_dev, L.table, log2m, probe_cap, L.slot_of, L.bits, L.st, ic, ph);
+    } else {
+      PTC_KERNEL("k_ids_insert", s, k_ids_insert, ceil_div_u32(n, kInsThreads * kInsK), kInsThreads, 0, k, n32, n_dev,
+                 L.table, log2m, probe_cap, L.slot_of, L.bits, L.st, ic);
+    }
+    return finish(L.table, 1ULL << log2m);
+  };
+  auto run_pd = [&]() -> bool {
+    if (hint) hint_prep();
+    const uint32_t sms = (uint32_t)num_sms();
+    uint32_t g1 = std::min(ceil_div_u32(n, kPdRound), std::min(4 * sms, kPdMaxG1));
+    const uint32_t per = ceil_div_u32(ceil_div_u32(n, g1), kPdRound) * kPdRound;
+    g1 = ceil_div_u32(n, per);
+    if (cudaFuncSetAttribute(k_pd_scatter1, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPdStageSmem) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(k_pd_level2<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPdStageSmem) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(k_pd_dedup, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPdDedupSmem) !=
+            cudaSuccess)
+      return false;
+    PTC_KERNEL("k_pd_flags", s, k_pd_flags, hint ? ceil_div_u32(hint->n_req, 8) : ceil_div_u32(L.nwords, 256), 256,
+               0, ph, n32, n_dev, L.pd_ubits, L.bits, L.nwords);
+    const PdArgs pa{k, n32, n_dev, ic, ph, per, L.pd_cnt1, L.pd_off1, L.pd_tot1, L.pd_ubits, L.pd_rec1, L.st};
+    PTC_KERNEL("k_pd_count", s, k_pd_count, g1, kPdThreads, 0, pa);
+    PTC_KERNEL("k_pd_rows1", s, k_pd_rows1, kPdBuckets, 256, 0, L.pd_cnt1, g1, L.pd_off1, L.pd_tot1);
+    PTC_KERNEL("k_pd_scatter1", s, k_pd_scatter1, g1, kPdThreads, kPdStageSmem, pa);
+    const uint32_t g2 = std::min(L.pd_max_tiles, 4 * sms);
+    const PdLevel2 p2{L.pd_rec1, L.pd_tot1, L.pd_tot2, L.pd_rel2, L.pd_base2, L.pd_rec2, n32, L.pd_max_tiles, L.st};
+    PTC_KERNEL("k_pd_count2", s, k_pd_level2<false>, g2, kPd2Threads, 0, p2);
+    PTC_KERNEL("k_pd_rows2", s, k_pd_rows2, kPdBuckets, 256, 0, L.pd_tot1, L.pd_tot2, L.pd_base2, L.st);
+    PTC_KERNEL("k_pd_scatter2", s, k_pd_level2<true>, g2, kPd2Threads, kPdStageSmem, p2);
+    PTC_KERNEL("k_pd_dedup", s, k_pd_dedup, std::min(kPdParts, 2 * sms), kPdDedupThreads, kPdDedupSmem,
+               PdDedup{L.pd_rec2, L.pd_base2, n32, L.slot_of, L.bits, n32, L.st});
+    return finish(nullptr, 0);
+  };
   const uint32_t first_log2m = full_table ? L.log2m : small_table_log2(n);
-  if (!start(first_log2m)) return PTC_ERR_CUDA;
+  if (!start(first_log2m, !pd)) return PTC_ERR_CUDA;
   DevStatus h{};
   if (nd_slot && err_slot) {  // one attempt, nothing waits
     const uint32_t lg = first_log2m;
-    if (n > 0 && !run(lg, lg < L.log2m ? kSmallProbeCap : ~0ULL)) return PTC_ERR_CUDA;
+    if (n > 0 && !(pd ? run_pd() : run(lg, lg < L.log2m ? kSmallProbeCap : ~0ULL))) return PTC_ERR_CUDA;
     return defer_status(L.st, err_slot, s, nd_slot, 0, 2);
   }
   if (n > 0) {
     const uint32_t small = first_log2m;
-    if (!run(small, small < L.log2m ? kSmallProbeCap : ~0ULL)) return PTC_ERR_CUDA;
-    if (small < L.log2m) {
+    if (!(pd ? run_pd() : run(small, small < L.log2m ? kSmallProbeCap : ~0ULL))) return PTC_ERR_CUDA;
+    if (pd || small < L.log2m) {
       const ptc_status rc1 = end_call(L.st, s, &h);
-      // anything but a probe sequence outrunning the small table is final
+      // anything but a first attempt outrunning its table is final
       if (rc1 == PTC_OK || h.err != kErrTableFull) {
         *n_distinct_host_out = h.value[0];
         if (n_used_host_out) *n_used_host_out = h.value[1];
         return rc1;
       }
-      // the small table overflowed: redo with the full one
-      if (!start(L.log2m) || !run(L.log2m, ~0ULL)) return PTC_ERR_CUDA;
+      // the first attempt's table overflowed: redo with the full one
+      if (!start(L.log2m, true) || !run(L.log2m, ~0ULL)) return PTC_ERR_CUDA;
     }
   }
   const ptc_status rc = end_call(L.st, s, &h);
@@ -747,18 +1448,28 @@ extern "C" ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t*
                        nullptr, 0);
 }
 
-void ptc::ids_table_region(void* ws, uint64_t n, uint32_t n_req_hint, void** table, size_t* bytes) {
-  const IdsLayout L = ids_layout(ws, n, n_req_hint);
-  *table = L.table;
-  *bytes = n > 0 ? sizeof(ulonglong2) << small_table_log2(n) : 0;
-}
-
 bool ptc::ids_table_in_dram(uint64_t n) { return n / 3 + 64 > (1ULL << kL2TableLog2); }
 
-size_t ptc::ids_ws_bytes(uint64_t n, uint32_t n_req_hint) { return ids_layout(nullptr, n, n_req_hint).total; }
+size_t ptc::ids_ws_bytes(uint64_t n, uint32_t n_req_hint) {
+  return ids_layout(nullptr, n, n_req_hint, ids_partitioned(n, PTC_IDS_AUTO)).total;
+}
 
 extern "C" size_t ptc_assign_ids_prior_workspace_bytes(uint64_t n, uint32_t n_req) {
-  return ids_layout(nullptr, n, n_req ? n_req : 1).total;
+  return ids_layout(nullptr, n, n_req ? n_req : 1, ids_partitioned(n, PTC_IDS_AUTO)).total;
+}
+
+extern "C" size_t ptc_assign_ids_ex_workspace_bytes(uint64_t n, uint32_t n_req, int method) {
+  return ids_layout(nullptr, n, n_req, ids_partitioned(n, method)).total;
+}
+
+extern "C" ptc_status ptc_assign_ids_ex(const ptc_u128* keys, uint64_t n, const uint64_t* req_blk_off,
+                                        const uint32_t* req_prior, uint32_t n_req, uint32_t* ids_out,
+                                        uint64_t* n_distinct_host_out, int method, void* ws, size_t ws_bytes,
+                                        void* stream) {
+  if (n > 0 && n_req > 0 && (!req_blk_off || !req_prior)) return PTC_ERR_INVALID_ARG;
+  const IdsHint h{req_blk_off, req_prior, n_req, nullptr, nullptr};
+  return ptc::ids_impl(keys, n, nullptr, ids_out, nullptr, n_distinct_host_out, ws, ws_bytes, (cudaStream_t)stream,
+                       nullptr, 0, nullptr, nullptr, nullptr, false, n > 0 && n_req > 0 ? &h : nullptr, method);
 }
 
 extern "C" ptc_status ptc_assign_ids_prior(const ptc_u128* keys, uint64_t n, const uint64_t* req_blk_off,

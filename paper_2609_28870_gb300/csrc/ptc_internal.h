@@ -189,17 +189,16 @@ uint64_t hash_carry_tiles(uint64_t n_tok, uint32_t block_size);
 ptc_status hash_impl(const uint32_t* tokens, uint64_t n_tok, const uint64_t* req_tok_off, const int64_t* req_ts_us,
                      uint32_t n_req, uint32_t block_size, uint64_t seed, ptc_u128* keys_out, uint64_t keys_cap,
                      uint64_t* req_blk_off_out, uint64_t* n_access_host_out, void* ws, size_t ws_bytes,
-                     cudaStream_t s, uint64_t* n_slot, uint32_t* err_slot, KeyCarry* carry = nullptr,
-                     void* fill_ones = nullptr, size_t fill_bytes = 0);
+                     cudaStream_t s, uint64_t* n_slot, uint32_t* err_slot, KeyCarry* carry = nullptr);
 // Stage a2 (ptc_ids.cu) over n_ub keys, of which the first min(*n_dev, n_ub)
 // are used when `n_dev` (device memory) is given.  Error words at
 // `carry_err` join the call's own.  Reports the number used and D.  With
 // `kc` each key gets its tile's carry as it is read.
 // With `nd_slot` and `err_slot` (device memory) the call does not wait: it
-// makes one attempt with the small table and leaves D in nd_slot[0], the
-// number of keys used in nd_slot[1] and its error word in *err_slot (a
-// probe sequence that outran the small table shows as exactly
-// kErrTableFull; redo the stage then with `full_table`).
+// makes one attempt (the partitioned dedup, or the table's small first
+// size) and leaves D in nd_slot[0], the number of keys used in nd_slot[1]
+// and its error word in *err_slot (an attempt that outran its table shows as
+// exactly kErrTableFull; redo the stage then with `full_table`).
 // The prior-request hint of stage a2 (ptc_assign_ids_prior): prior[r] is an
 // earlier request whose blocks request r is likely to repeat, or PTC_NONE.
 struct IdsHint {
@@ -212,7 +211,8 @@ struct IdsHint {
 size_t ids_ws_bytes(uint64_t n, uint32_t n_req_hint);
 // Whether the id table for n keys is larger than the part of L2 it may take:
 // only then do the table probes the prior-request hint saves cost DRAM
-// traffic; an L2-resident table probes faster than the hint's extra reads.
+// traffic (an L2-resident table probes faster than the hint's extra reads),
+// and only then does stage a2 deduplicate by partitions instead.
 bool ids_table_in_dram(uint64_t n);
 // The previous request of each request's session (ptc_session_prior),
 // queued on `s` without waiting; scratch of session_prior_bytes(n_req).
@@ -224,11 +224,7 @@ ptc_status ids_impl(const ptc_u128* keys, uint64_t n_ub, const uint64_t* n_dev, 
                     uint64_t* n_used_host_out, uint64_t* n_distinct_host_out, void* ws, size_t ws_bytes,
                     cudaStream_t s, const uint32_t* carry_err, uint32_t n_carry, const KeyCarry* kc = nullptr,
                     uint64_t* nd_slot = nullptr, uint32_t* err_slot = nullptr, bool full_table = false,
-                    const IdsHint* hint = nullptr, bool table_prefilled = false);
-// Where ids_impl's first attempt (full_table false) keeps its table in the
-// workspace `ws`, and its bytes; ids_impl with table_prefilled = true takes
-// that region as already set to all ones (empty).
-void ids_table_region(void* ws, uint64_t n, uint32_t n_req_hint, void** table, size_t* bytes);
+                    const IdsHint* hint = nullptr, int method = PTC_IDS_AUTO);
 ptc_status stack_distance_view(const uint32_t* prev, uint64_t n, uint32_t* dist_out, int method, void* ws,
                                size_t ws_bytes, cudaStream_t s, RunsView* view, uint32_t* defer_err);
 // Stage b as ptc_reuse_indices does it (ptc_reuse.cu); with `defer_err` the

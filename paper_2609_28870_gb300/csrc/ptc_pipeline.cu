@@ -67,33 +67,7 @@ PipeLayout pipe_layout(void* ws, uint32_t n_req, uint64_t n_tok, uint32_t B, uin
   return L;
 }
 
-// Stage a2's first table inside the scratch region, and whether the hash
-// grid fills it while stage a1 runs: only a DRAM-sized table (a table that
-// fits in L2 is better filled by stage a2 just before its insert, which then
-// finds it in L2), and only when it lies past the scratch that stage a1
-// (and the session sort before it) use.
-bool fused_table_fill(void* scratch, uint32_t n_req, uint64_t n_tok, uint32_t B, bool hinted, void** table,
-                      size_t* bytes) {
-  const uint64_t cap = n_tok / B ? n_tok / B : 1;
-  ptc::ids_table_region(scratch, cap, hinted ? n_req : 0, table, bytes);
-  if (!ptc::ids_table_in_dram(cap)) return false;
-  const size_t front = std::max(ptc_hash_blocks_workspace_bytes(n_req, n_tok, B), ptc::session_prior_bytes(n_req));
-  return *bytes > 0 && static_cast<char*>(*table) >= static_cast<char*>(scratch) + front;
-}
-
 }  // namespace
-
-extern "C" size_t ptc_pipeline_table_fill_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size,
-                                                int with_sessions) {
-  if (block_size < 1 || block_size > PTC_MAX_BLOCK_SIZE || n_tok / block_size == 0) return 0;
-  const bool hinted = with_sessions && n_req > 0 && ptc::ids_table_in_dram(n_tok / block_size);
-  // the region's offset is what matters: lay it out from a scratch base of 256
-  void* table = nullptr;
-  size_t bytes = 0;
-  return fused_table_fill(reinterpret_cast<void*>(uintptr_t{256}), n_req, n_tok, block_size, hinted, &table, &bytes)
-             ? bytes
-             : 0;
-}
 
 extern "C" size_t ptc_pipeline_workspace_bytes(uint32_t n_req, uint64_t n_tok, uint32_t block_size, uint32_t n_cap) {
   if (block_size == 0) block_size = 1;
@@ -148,18 +122,11 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
   // carry as it reads them
   ptc::KeyCarry kc{L.carry, L.lead, 1};
   ptc::KeyCarry* kcp = keys_out ? nullptr : &kc;
-  // stage a1 is bound by integer issue, so it also fills stage a2's table
-  // (all ones: empty), which lies past stage a1's workspace and the session
-  // sort's in the shared scratch region
-  void* table = nullptr;
-  size_t table_bytes = 0;
-  const bool fused_fill = fused_table_fill(L.scratch, n_req, n_tok, block_size, hinted, &table, &table_bytes);
   ptc_status rc = ptc::hash_impl(tokens, n_tok, req_tok_off, req_ts_us, n_req, block_size, seed, keys, cap, blk,
-                                 &unused, L.scratch, L.scratch_bytes, s, L.n_slot, &L.defer[0], kcp,
-                                 fused_fill ? table : nullptr, fused_fill ? table_bytes : 0);
+                                 &unused, L.scratch, L.scratch_bytes, s, L.n_slot, &L.defer[0], kcp);
   if (rc != PTC_OK) return rc;
   rc = ptc::ids_impl(keys, cap, L.n_slot, ids, &n, &d, L.scratch, L.scratch_bytes, s, &L.defer[0], 2, kcp,
-                     L.nd_slot, &L.defer[4], false, hp, fused_fill);
+                     L.nd_slot, &L.defer[4], false, hp);
   if (rc != PTC_OK) return rc;
   const ptc::ReuseDevIn din{L.nd_slot, &L.defer[4]};
   ptc::ReuseHostOut hout;
@@ -168,8 +135,9 @@ extern "C" ptc_status ptc_pipeline(const uint32_t* tokens, uint64_t n_tok, const
   *n_distinct_host_out = d = hout.D;
   if (rc != PTC_OK) return rc;
   if (hout.ids_err) {
-    // stage a2's small table overflowed (or a1 / a2 failed): redo a2 with the
-    // full table, waiting for it, then stage b with the host's N and D
+    // stage a2's first attempt outran its table (or a1 / a2 failed): redo a2
+    // with the full table, waiting for it, then stage b with the host's N
+    // and D
     if (hout.ids_err != ptc::kErrTableFull) return ptc::status_of(hout.ids_err);
     rc = ptc::ids_impl(keys, cap, L.n_slot, ids, &n, &d, L.scratch, L.scratch_bytes, s, &L.defer[0], 2, kcp, nullptr,
                        nullptr, true, hp);

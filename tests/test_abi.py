@@ -129,25 +129,21 @@ def test_trace_stats_host_checks_need_no_gpu(libptc):
                              buf.ctypes.data, fake, 16, None) == 4
 
 
-def test_pipeline_table_fill_bytes(libptc):
-    """The id table that the pipeline's hash grid fills: a power of two of
-    16-byte slots, at least n / 3 of them (3 n / 4 once the table is larger
-    than the part of L2 it may use); nothing for an empty trace, or when the
-    table would overlap the hash stage's own scratch (small traces)."""
-    f = libptc.ptc_pipeline_table_fill_bytes
-    f.restype = ctypes.c_size_t
-    f.argtypes = [ctypes.c_uint32, ctypes.c_uint64, ctypes.c_uint32, ctypes.c_int]
-    assert f(10, 15, 16, 0) == 0
-    for n_req, n_tok, B, ses in ((100, 10**6, 16, 0), (582163, 9984375026, 16, 1), (2000, 2 * 10**9, 64, 1)):
-        b = f(n_req, n_tok, B, ses)
-        if b == 0:
-            assert n_tok < 10**8
-            continue
-        slots = b // 16
-        n = n_tok // B
-        assert b % 16 == 0 and slots & (slots - 1) == 0
-        assert slots >= (n // 4 * 3 if slots > (1 << 22) else n // 3)
-    assert f(582163, 9984375026, 16, 1) == 16 << 29
+def test_assign_ids_ex_checks_and_workspace(libptc):
+    """An unknown dedup method is rejected before any CUDA call; the
+    partitioned method's workspace holds its records and counters."""
+    import paper_2609_28870_gb300 as ptc
+    L = ptc.lib()
+    d = ctypes.c_uint64(0)
+    assert L.ptc_assign_ids_ex(None, 0, None, None, 0, None, ctypes.byref(d), 7, None, 0, None) == 1
+    w = L.ptc_assign_ids_ex_workspace_bytes
+    n = 100_000
+    assert w(n, 0, ptc.PTC_IDS_PARTITIONED) > w(n, 0, ptc.PTC_IDS_TABLE)
+    assert w(n, 0, ptc.PTC_IDS_PARTITIONED) >= 32 * n                       # records of both levels
+    assert w(n, 0, ptc.PTC_IDS_AUTO) == w(n, 0, ptc.PTC_IDS_TABLE)        # small: the table
+    big = 50_000_000
+    assert w(big, 0, ptc.PTC_IDS_AUTO) == w(big, 0, ptc.PTC_IDS_PARTITIONED)  # beyond L2: partitions
+    assert w(big, 0, ptc.PTC_IDS_AUTO) == L.ptc_assign_ids_workspace_bytes(big)
 
 
 def test_probe_random_rmw_rejects_bad_tables(libptc):
