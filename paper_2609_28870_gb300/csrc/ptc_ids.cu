@@ -697,6 +697,38 @@ __global__ void __launch_bounds__(256) k_pd_flags(PriorHint ph, uint32_t n_ub, c
   }
 }
 
+// The carries of the hash tiles that a round of kPdRound accesses from
+// `base` spans (base a multiple of kPdRound, hence of every tile size; a
+// hash tile holds 8 to 256 blocks), read once per round into shared memory:
+// entry t is tile (base >> tile_shift) + t, up to hi.
+constexpr uint32_t kPdRoundTiles = kPdRound / 8;
+__device__ __forceinline__ void pd_round_carry(const InsCarry& kc, uint64_t base, uint64_t hi, uint32_t* s_lead,
+                                               ulonglong2* s_cy) {
+  if (!kc.carry) return;
+  const uint32_t nt = kPdRound >> kc.tile_shift;
+  const uint64_t t0 = base >> kc.tile_shift;
+  for (uint32_t t = threadIdx.x; t < nt; t += blockDim.x)
+    if (((t0 + t) << kc.tile_shift) < hi) {
+      s_lead[t] = __ldg(&kc.lead[t0 + t]);
+      s_cy[t] = __ldg(&kc.carry[t0 + t]);
+    }
+}
+
+// Key i of the round from `base`, with its tile's carry added (as
+// carried_key does) from the round's shared copy.
+__device__ __forceinline__ ulonglong2 pd_key(const ulonglong2* __restrict__ keys, uint32_t i, uint64_t base,
+                                             const InsCarry& kc, const uint32_t* s_lead, const ulonglong2* s_cy) {
+  ulonglong2 k = __ldcs(&keys[i]);
+  if (kc.carry) {
+    const uint32_t t = (uint32_t)(i - base) >> kc.tile_shift;
+    if ((i & ((1u << kc.tile_shift) - 1u)) < s_lead[t] && k.x < kP61 && k.y < kP61) {
+      const ulonglong2 c = s_cy[t];
+      k = make_ulonglong2(p61_add(k.x, c.x), p61_add(k.y, c.y));
+    }
+  }
+  return k;
+}
+
 // h0 of key i with the carry of its hash tile added (the first word of
 // carried_key, for a key whose second word is a field element).
 __device__ __forceinline__ uint64_t carried_h0(const ulonglong2* __restrict__ keys, uint32_t i, const InsCarry& kc) {
@@ -750,6 +782,8 @@ __global__ void __launch_bounds__(kPdThreads, 2) k_pd_scatter1(PdArgs a) {
   __shared__ uint32_t h[kPdBuckets];     // the next place in each bucket
   __shared__ uint32_t c[kPdBuckets], so[kPdBuckets];  // the round's records per bucket, their offsets
   __shared__ uint32_t s_bst[kPdBuckets + 1];
+  __shared__ uint32_t s_lead[kPdRoundTiles];
+  __shared__ ulonglong2 s_cy[kPdRoundTiles];
   pd_bucket_bounds(a.tot1, s_bst);
   for (uint32_t x = threadIdx.x; x < kPdBuckets; x += kPdThreads) {
     h[x] = s_bst[x] + a.off1[x * gridDim.x + blockIdx.x];
@@ -758,6 +792,7 @@ __global__ void __launch_bounds__(kPdThreads, 2) k_pd_scatter1(PdArgs a) {
   const uint32_t n = keys_used(a.n_ub, a.n_dev);
   const uint64_t lo = (uint64_t)blockIdx.x * a.per;
   const uint64_t hi = lo + a.per < n ? lo + a.per : n;
+  pd_round_carry(a.kc, lo, hi, s_lead, s_cy);
   __syncthreads();
   for (uint64_t base = lo; base < hi; base += kPdRound) {
     bool u[kPdPer];
@@ -771,7 +806,7 @@ __global__ void __launch_bounds__(kPdThreads, 2) k_pd_scatter1(PdArgs a) {
 #pragma unroll
     for (int j = 0; j < kPdPer; ++j) {
       const uint32_t i = (uint32_t)(base + j * kPdThreads + threadIdx.x);
-      k[j] = u[j] ? carried_key(a.keys, i, n, a.kc) : make_ulonglong2(0, 0);
+      k[j] = u[j] ? pd_key(a.keys, i, base, a.kc, s_lead, s_cy) : make_ulonglong2(0, 0);
       if (u[j] && (k[j].x >= kP61 || k[j].y >= kP61)) {  // not a field element: never settled
         raise_err(a.st, kErrInvalid);
         u[j] = false;
@@ -803,6 +838,7 @@ __global__ void __launch_bounds__(kPdThreads, 2) k_pd_scatter1(PdArgs a) {
       h[x] += c[x];
       c[x] = 0;
     }
+    pd_round_carry(a.kc, base + kPdRound, hi, s_lead, s_cy);  // the next round's (its reads of these are done)
     __syncthreads();
   }
 }
@@ -955,34 +991,30 @@ __device__ __forceinline__ ulonglong2 cas128_shared(ulonglong2* addr, ulonglong2
 // (the partition fixes bits 45..60 only).
 __device__ __forceinline__ uint32_t pd_home(uint64_t w0, uint32_t ts) { return __umulhi((uint32_t)w0, ts); }
 
-// Settle record r in the shared table of ts slots: claim an empty slot with
-// one 128-bit CAS, or meet its key's slot, where the smaller of the two
-// indices stays.  The index that does not stay (r's own, or the one r's
-// atomicMin replaced) is a repeat: it comes back in *rep, with the slot in
-// *rs (*rep = kNone otherwise).  False when the table has no room (every
-// slot probed).
-__device__ __forceinline__ bool pd_insert(ulonglong2* tab, uint32_t ts, ulonglong2 r, uint32_t* rep, uint32_t* rs) {
+// One probe for record r at slot sl of the shared table (linear probing from
+// pd_home): claim the slot if it is empty, with one 128-bit CAS, or meet r's
+// key there, where the smaller of the two indices stays.  The index that
+// does not stay (r's own, or the one r's atomicMin replaced) is a repeat: it
+// comes back in *rep with the slot in *rs.  True when r is settled here;
+// false when the slot holds another key (probe the next one).
+__device__ __forceinline__ bool pd_probe(ulonglong2* tab, uint32_t ts, ulonglong2 r, uint32_t sl, uint32_t* rep,
+                                         uint32_t* rs) {
   const ulonglong2 empty = make_ulonglong2(~0ULL, ~0ULL);
   const uint32_t idx = (uint32_t)(r.y >> 32);
-  *rep = kNone;
-  uint32_t s = pd_home(r.x, ts);
-  for (uint32_t probe = 0; probe < ts; ++probe) {
-    ulonglong2 cur = ld_shared_v2(&tab[s]);
-    if (cur.x == ~0ULL || cur.y == ~0ULL) {  // empty (or read while being claimed): the CAS settles it
-      cur = cas128_shared(&tab[s], empty, r);
-      if (cur.x == ~0ULL && cur.y == ~0ULL) return true;
+  ulonglong2 cur = ld_shared_v2(&tab[sl]);
+  if (cur.x == ~0ULL || cur.y == ~0ULL) {  // empty (or read while being claimed): the CAS settles it
+    cur = cas128_shared(&tab[sl], empty, r);
+    if (cur.x == ~0ULL && cur.y == ~0ULL) return true;
+  }
+  if (cur.x == r.x && (uint32_t)cur.y == (uint32_t)r.y) {
+    uint32_t out = idx;
+    if ((uint32_t)(cur.y >> 32) > idx) {
+      const uint32_t old = atomicMin(reinterpret_cast<uint32_t*>(&tab[sl]) + 3, idx);
+      out = old > idx ? old : idx;
     }
-    if (cur.x == r.x && (uint32_t)cur.y == (uint32_t)r.y) {
-      uint32_t out = idx;
-      if ((uint32_t)(cur.y >> 32) > idx) {
-        const uint32_t old = atomicMin(reinterpret_cast<uint32_t*>(&tab[s]) + 3, idx);
-        out = old > idx ? old : idx;
-      }
-      *rep = out;
-      *rs = s;
-      return true;
-    }
-    s = s + 1 == ts ? 0 : s + 1;
+    *rep = out;
+    *rs = sl;
+    return true;
   }
   return false;
 }
@@ -1078,10 +1110,31 @@ __global__ void __launch_bounds__(kPdDedupThreads, 2) k_pd_dedup(PdDedup a) {
           load(w, c + kChunk, e);
         else
           load(w, bn, en);
+        // one probe per lane per round: a lane that settles its record takes
+        // its next one at once, so a long probe run holds back only its own
+        // lane's queue rather than the whole warp at every record
+        uint32_t nv = 0;
 #pragma unroll
-        for (int q = 0; q < kPdDedupPer; ++q) {
+        for (int q = 0; q < kPdDedupPer; ++q) nv += v[q].x != ~0ULL;
+        uint32_t sl = pd_home(v[0].x, ts), probes = 0;
+        while (__any_sync(kFull, nv > 0)) {
           uint32_t rep = kNone, rs = 0;
-          if (v[q].x != ~0ULL && !pd_insert(tab, ts, v[q], &rep, &rs)) full = true;
+          if (nv > 0) {
+            bool done = pd_probe(tab, ts, v[0], sl, &rep, &rs);
+            if (!done && ++probes >= ts) {  // every slot probed: no room
+              full = true;
+              done = true;
+            }
+            if (done) {
+              --nv;
+#pragma unroll
+              for (int q = 0; q + 1 < kPdDedupPer; ++q) v[q] = v[q + 1];
+              sl = pd_home(v[0].x, ts);
+              probes = 0;
+            } else {
+              sl = sl + 1 == ts ? 0 : sl + 1;
+            }
+          }
           pd_list_push(rep, rs, list, &s_nlist);
         }
 #pragma unroll
