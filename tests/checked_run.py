@@ -4,7 +4,8 @@ Run by tests/test_gpu_checked.py in a process of its own (a process loads one
 build): the checked build checks every index that comes from data another
 stage or the caller wrote before using it, and reports a miss as
 PTC_ERR_BOUNDS instead of touching memory.  Every call here must succeed and
-match the oracle."""
+match the oracle (the partitioned dedup of the id stage included, with and
+without a prior-request hint)."""
 import os
 import sys
 
@@ -21,6 +22,9 @@ assert b"checked" in ptc.lib().ptc_version(), ptc.lib().ptc_version()
 import oracle  # noqa: E402
 import tracegen  # noqa: E402
 from tests.gpu_util import assert_same, oracle_run, to_gpu  # noqa: E402
+
+
+NONE = 0xFFFFFFFF
 
 
 def u32(a):
@@ -58,6 +62,11 @@ def main():
             assert_same(g, o)
         off = outs["req_blk_off"]
         N = ids.size
+        keys = outs["keys"].view(-1, 2)[:N]
+        prior = u32(np.asarray([NONE] + list(range(tr.n_req - 1)), np.uint32)[: tr.n_req])
+        for hint in ((None, None), (off, prior)):
+            pid, pd = ptc.ptc_assign_ids_ex(keys, ptc.PTC_IDS_PARTITIONED, *hint)
+            assert pd == D and np.array_equal(ptc.u32(pid), ids)
         bel = ptc.ptc_belady_curves(outs["prev"][:N], off, B, caps)
         h, s, raw = oracle.belady_curves(ids, oracle.block_offsets(tr.req_tok_off, B), B, caps)
         assert bel["hits"] == h and bel["saved"] == s and bel["raw_hits"] == raw
