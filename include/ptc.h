@@ -151,20 +151,21 @@ ptc_status ptc_assign_ids(const ptc_u128* keys, uint64_t n, uint32_t* ids_out, u
 
 /*
  * ptc_assign_ids_prior — the ids of ptc_assign_ids, with a prior-request hint
- * that saves table probes.  Sec. 2.3: a turn of a multi-turn session sends
+ * that saves work: fewer keys to settle in the table or the partitions.  Sec. 2.3: a turn of a multi-turn session sends
  * the whole context again, so request r usually repeats every block of an
  * earlier request of its session and appends to it.  req_prior[r] names such
  * an earlier request (or PTC_NONE).  The leading depths of r whose keys
  * equal those of the same depths of req_prior[r] are repeats: they are not
- * inserted into the table and take their ids from the prior request's chain;
- * only the other accesses are inserted.  The keys must be prefix keys as
+ * settled (inserted into the table, or moved into the partitions of the
+ * partitioned dedup) and take their ids from the prior request's chain;
+ * only the other accesses are settled.  The keys must be prefix keys as
  * ptc_hash_blocks writes them (equal keys at depth k imply equal keys at
  * every depth below k), so the end of that leading run is found by a binary
  * search over the depths, reading about 2 log2(n_r) keys per request rather
  * than the prior request's key of every access.  The ids are then exactly
  * those of ptc_assign_ids for ANY hint with req_prior[r] < r or PTC_NONE (a
- * poor hint only costs probes); req_prior[r] >= r is PTC_ERR_INVALID_ARG.
- * A key that is not a field element is reported when it is inserted; the
+ * poor hint only costs time); req_prior[r] >= r is PTC_ERR_INVALID_ARG.
+ * A key that is not a field element is reported when it is settled; the
  * keys of repeated depths are only compared.
  *   keys         ptc_u128[n] as for ptc_assign_ids, prefix keys
  *   req_blk_off  u64[n_req + 1] from ptc_hash_blocks (req_blk_off[n_req] == n)
@@ -440,8 +441,10 @@ ptc_status ptc_session_lru_curves(const uint32_t* ids, uint64_t n, uint64_t n_di
  *       them, stage a2 takes the previous request of each request's session
  *       as its prior-request hint (ptc_session_prior, ptc_assign_ids_prior):
  *       a turn of a session re-sends that request's context (Sec. 2.3), so
- *       most of its blocks need no table probe.  The results do not depend
- *       on the sessions; only the time does.
+ *       most of its blocks need not be settled.  The hint is taken only
+ *       when the id table would exceed L2 (then stage a2 deduplicates by
+ *       partitions, ptc_assign_ids_ex).  The results do not depend on the
+ *       sessions; only the time does.
  * The workspace holds the intermediate arrays not supplied plus the largest
  * scratch of any stage (ptc_pipeline_workspace_bytes).  Stages b and c do not
  * wait for their own status; an error they raise is returned with stage d's.
@@ -625,7 +628,8 @@ uint64_t ptc_launch_count(void);
  * all ones, claims it with a 128-bit compare-and-swap, as the id table's
  * insert does for a key it has not seen.  `sink` is 8 bytes of device memory
  * the kernel may write.  The caller times the launch: probes over seconds is
- * the random read-modify-write rate that bounds the insert.  Allocates
+ * the random read-modify-write rate that bounds the table method's insert
+ * on a table of that size (the bench sets it beside the partitioned dedup).  Allocates
  * nothing.  PTC_ERR_INVALID_ARG for a null, misaligned or non-power-of-two
  * table.
  */
