@@ -538,16 +538,16 @@ __global__ void k_session_prior(const uint32_t* __restrict__ ses_sorted, const u
 // partitioned method moves the keys to be settled (the unmatched accesses)
 // instead, in streaming passes, into 2^16 partitions by 16 bits of h0, and
 // settles every partition in a table of its own in shared memory:
-//   k_pd_flags     the bitmap of the accesses to settle: every access
-//                  without a hint; with one, the depths of each request from
-//                  its lam on (a warp per request)
+//   k_pd_flags     the bitmap of the accesses to settle (ubits), and its
+//                  copy that becomes the first-occurrence bitmap (bits):
+//                  every access without a hint; with one, the depths of each
+//                  request from its lam on (a warp per request)
 //   k_pd_count     level 1: per CTA of a persistent grid, the keys of its
 //                  range of accesses per bucket (h0 bits 53..60)
 //   k_pd_rows1     one CTA per bucket: the prefix of its counts over the
 //                  level-1 CTAs, and the bucket's total
-//   k_pd_scatter1  the same pass again: slot_of (matched or unmatched), and
-//                  a 16-byte record (96 key bits, access index) per
-//                  unmatched access, in bucket order
+//   k_pd_scatter1  the same pass again: a 16-byte record (96 key bits,
+//                  access index) per access to settle, in bucket order
 //   k_pd_count2    level 2: per tile of kPdTile2 records of one bucket, the
 //                  records per partition (h0 bits 45..60); one atomic per
 //                  tile and partition claims the tile's place in it
@@ -559,8 +559,9 @@ __global__ void k_session_prior(const uint32_t* __restrict__ ses_sorted, const u
 //                  replaces, is a repeat and goes to a list, whose entries
 //                  then take their key's smallest index into slot_of and
 //                  clear their bit.
-// The bitmap then holds exactly the first occurrences, and k_ids_gather reads
-// a repeat's first occurrence from slot_of itself.  A partition holding more
+// bits then holds exactly the first occurrences, and k_ids_gather_pd reads a
+// repeat's first occurrence from slot_of itself (slot_of is written for the
+// repeats only; ubits tells the settled accesses from the matched ones).  A partition holding more
 // distinct keys than its shared table raises kErrTableFull, as an overfull
 // hash table does, and the call redoes the stage with the full table.
 // Both scatters sort a round's records by destination in shared memory
