@@ -275,13 +275,52 @@ GOLDEN = os.path.join(ROOT, "tests", "golden", "big_configs.json")
 
 
 _HOST_BUFFERS = []  # registered host buffers: kept alive, unregistered at exit
+HOST_PLACEMENT = {}  # where the token buffer's pages were asked to live (reported with e2e)
 
 
-def registered_host_u32(n):
+def gpu_numa_node(dev):
+    """The host NUMA node of the GPU's PCI device (sysfs numa_node), or None
+    where the system does not say."""
+    try:
+        import torch
+        p = torch.cuda.get_device_properties(dev)
+        path = f"/sys/bus/pci/devices/{p.pci_domain_id:04x}:{p.pci_bus_id:02x}:{p.pci_device_id:02x}.0/numa_node"
+        with open(path) as fh:
+            node = int(fh.read().strip())
+        return node if node >= 0 else None
+    except Exception:
+        return None
+
+
+def prefer_node(addr, nbytes, node):
+    """Asks the kernel to place the pages of [addr, addr + nbytes), not yet
+    touched, on NUMA node `node` (mbind with MPOL_PREFERRED: other nodes
+    still serve it when that one is full).  True if the call succeeded."""
+    import ctypes
+    import platform
+    nr = {"aarch64": 235, "x86_64": 237}.get(platform.machine())
+    if nr is None or node is None or node >= 1024:
+        return False
+    try:
+        libc = ctypes.CDLL(None, use_errno=True)
+        libc.syscall.restype = ctypes.c_long
+        mask = (ctypes.c_ulong * 16)()
+        mask[node // 64] |= 1 << (node % 64)
+        mpol_preferred = 1
+        rc = libc.syscall(ctypes.c_long(nr), ctypes.c_void_p(addr), ctypes.c_ulong(nbytes),
+                          ctypes.c_int(mpol_preferred), mask, ctypes.c_ulong(16 * 64 + 1), ctypes.c_uint(0))
+        return rc == 0
+    except Exception:
+        return False
+
+
+def registered_host_u32(n, dev=None):
     """n uint32 in page-locked host memory: an anonymous mapping asked for huge
-    pages, then registered with CUDA (cudaHostRegister).  Copies from it ran at
-    the host link's full 211 GB/s on a GB300 machine whether or not the box had
-    just run the whole test suite, where a buffer from torch's pinned-memory
+    pages (and, where the system names the GPU's NUMA node, for pages on that
+    node: the copy engine reads a far node's memory through the link between
+    the CPUs), then registered with CUDA (cudaHostRegister).  End-to-end steps
+    over this buffer measured 226-250 ms on some boxes and 305-569 ms on
+    others before the node was asked for; a buffer from torch's pinned-memory
     allocator copied at 84-211 GB/s on its first passes."""
     import atexit
     import mmap
@@ -290,9 +329,11 @@ def registered_host_u32(n):
     import torch
     nbytes = max(4 * int(n), 4096)
     m = mmap.mmap(-1, nbytes, flags=mmap.MAP_PRIVATE | mmap.MAP_ANONYMOUS)
+    a = np.frombuffer(m, dtype=np.uint32, count=int(n))
+    node = gpu_numa_node(dev) if dev is not None else None
+    HOST_PLACEMENT.update({"gpu_numa_node": node, "placed": prefer_node(a.ctypes.data, nbytes, node)})
     if hasattr(mmap, "MADV_HUGEPAGE"):
         m.madvise(mmap.MADV_HUGEPAGE)
-    a = np.frombuffer(m, dtype=np.uint32, count=int(n))
     rt = torch.cuda.cudart()
     if int(rt.cudaHostRegister(a.ctypes.data, nbytes, 0)) != 0:
         raise RuntimeError("cudaHostRegister failed for the token buffer")
@@ -313,7 +354,7 @@ def load_trace(workload, requests, dev):
         tok_host = torch.from_numpy(tr.tokens.view(np.int32)).pin_memory()
     else:
         _, T, _ = tracegen.sizes(workload)
-        buf = registered_host_u32(T)
+        buf = registered_host_u32(T, dev)
         tr = tracegen.make(workload, token_buffer=buf)
         tok_host = torch.from_numpy(buf.view(np.int32))
     off_host = torch.from_numpy(tr.req_tok_off.view(np.int64)).pin_memory()
@@ -623,7 +664,8 @@ def run_ours(args, ws_world, rank, local):
         "e2e": {"value": round(e2e_value, 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_total / args.steps, 4),
                 "call": "ptc_pipeline_host: trace in page-locked host memory, copied inside the call; curves "
-                        "returned to host memory"},
+                        "returned to host memory",
+                "host_pages": dict(HOST_PLACEMENT) or None},
         "gpu_launches": launches,
         "clocks": clk,
         "parity_with_oracle_golden": gold,
